@@ -1,0 +1,140 @@
+"""Workload definitions: shapes, constants, seeds (no arithmetic of the method).
+
+Every workload is synthetic and seeded (``synth``); the image datasets of the
+paper's experiments are replaced by inputs of the same shape and value range.
+A layer is a plain dict understood by both the CUDA driver (``net.py``) and
+the float64 oracle:
+
+  kind            "dense" | "conv"
+  W               float64 weights, dense [N_out, N_in], conv [C_out, C_in, k, k]
+  tau_v, tau_I    membrane / synaptic time constants (math.inf allowed)
+  v_th            threshold
+  t_first, t_end  DSTD window; M steps; grid T_m = t_first + m dt - t_offset
+  t_offset        in (-dt/2, dt/2]
+  t_head_l, t_tail_l, gamma_head, gamma_tail, gamma_q  synfire penalty terms
+  conv only       stride, pad, in_shape (C, H, W)
+
+Synfire constants follow App. C.1 with mid-range values of Tab. search_space:
+tau_width = 1, tau_shift = 0.1, tau_margin = 0.1, t_head = t_tail = 0.2,
+gamma_head = 0.05, gamma_tail = 0.01, gamma_Q = 1e-3, tau_soft = 0.02, tau_in = 1.
+Layer l's window is [l tau_shift - tau_margin, l tau_shift + tau_width + tau_margin]
+and its penalty edges t_head^(l) = l tau_shift + t_head,
+t_tail^(l) = l tau_shift + tau_width - t_tail.
+
+Weight means mu_l (dense configs 2 and 3) make about 80% of each layer's
+neurons fire at initialisation on the seed-0 batch with M = 32 and
+t_offset = 0; they were found once by bisection with the oracle
+(``oracle/calibrate_configs.py``) and are frozen here.
+"""
+
+import math
+
+import numpy as np
+
+from . import synth
+
+INF = math.inf
+
+SYNFIRE = dict(tau_in=1.0, tau_width=1.0, tau_shift=0.1, tau_margin=0.1, t_head=0.2, t_tail=0.2,
+               gamma_head=0.05, gamma_tail=0.01, gamma_q=1e-3, tau_soft=0.02)
+
+# seeds: inputs 0, layer-l weights 1000 + l, labels 7, t_offset draws 11
+SEED_INPUT, SEED_W, SEED_LABELS, SEED_OFFSET = 0, 1000, 7, 11
+
+# frozen calibration (80% firing at init), see module docstring
+CFG2_MU = (0.03523, 0.01520, 0.01951)
+CFG3_MU_TIMES_N = 17.4
+
+
+def synfire_layer(l, syn=SYNFIRE):
+    """Window and penalty edges of layer l >= 1 (App. C.1)."""
+    return dict(
+        t_first=l * syn["tau_shift"] - syn["tau_margin"],
+        t_end=l * syn["tau_shift"] + syn["tau_width"] + syn["tau_margin"],
+        t_head_l=l * syn["tau_shift"] + syn["t_head"],
+        t_tail_l=l * syn["tau_shift"] + syn["tau_width"] - syn["t_tail"],
+        gamma_head=syn["gamma_head"], gamma_tail=syn["gamma_tail"], gamma_q=syn["gamma_q"])
+
+
+def _dense(W, tau_v, tau_I, M, t_first, t_end, v_th=1.0, **kw):
+    d = dict(kind="dense", W=W, tau_v=tau_v, tau_I=tau_I, v_th=v_th, M=M, t_first=t_first,
+             t_end=t_end, t_offset=0.0, t_head_l=0.0, t_tail_l=0.0, gamma_head=0.0,
+             gamma_tail=0.0, gamma_q=0.0)
+    d.update(kw)
+    return d
+
+
+def config1(scale=1.0, batch=8):
+    """Single dense layer 64 -> 32, B = 8, M = 16 over [0, 1], (tau_m, tau_s) = (0.5, 0.25).
+
+    Inputs U[0, 0.8) with 20% silent; W ~ N(0, 1/64) * 4 * scale (scale 12 is
+    the "1b" variant, where about a third of the outputs fire); loss = sum of
+    the output spike times that fire.
+    """
+    W = synth.normal_weights(SEED_W + 1, (32, 64), 0.0, 1.0 / 8.0) * 4.0 * scale
+    return dict(
+        name="cfg1" if scale == 1.0 else "cfg1b",
+        workload=f"dense LIF layer 64->32, B={batch}, M=16, tau=(0.5,0.25)" + ("" if scale == 1.0 else " x12 weights"),
+        batch=batch, in_shape=(64,), loss="sum_t", tau_soft=None,
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.uniform_spikes(seed, (B, 64), 0.0, 0.8, 0.2),
+        layers=[_dense(W, 0.5, 0.25, 16, 0.0, 1.0)])
+
+
+def config2(batch=256, M=32):
+    """3-layer dense MLP 784-800-800-10, B = 256, M = 32, (tau_m, tau_s) = (0.5, 0.25).
+
+    Inputs: 28x28 intensities x ~ U[0,1) with 60% zeros, t = 1 - x (x = 0
+    silent); synfire windows per layer; loss = CE over softmax(-t/tau_soft)
+    with 10 random labels + T + gamma_Q Q.
+    """
+    sizes = [784, 800, 800, 10]
+    layers = []
+    for l in range(1, 4):
+        W = synth.normal_weights(SEED_W + l, (sizes[l], sizes[l - 1]), CFG2_MU[l - 1],
+                                 1.0 / math.sqrt(sizes[l - 1]))
+        layers.append(_dense(W, 0.5, 0.25, M, **synfire_layer(l)))
+    return dict(
+        name="cfg2", workload=f"dense LIF TTFS MLP 784-800-800-10, B={batch}, M={M}, tau=(0.5,0.25), synfire CE+T+Q",
+        batch=batch, in_shape=(784,), loss="ce", tau_soft=SYNFIRE["tau_soft"], n_classes=10,
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.intensity_spikes(seed, (B, 784), 0.6, SYNFIRE["tau_in"]),
+        labels=lambda seed=SEED_LABELS, B=batch: synth.labels(seed, B, 10),
+        layers=layers)
+
+
+def config3(N, M, batch=128, tau=(0.4, 0.2)):
+    """One dense layer N -> N, B = 128, M steps over [0, 1], (tau_m, tau_s) = (0.4, 0.2).
+
+    Inputs U[0, 1) with 10% silent; W = mu + N(0, 1/N) with mu N = 17.4;
+    loss = sum of the output spike times that fire (one fwd+bwd pass).
+    """
+    W = synth.normal_weights(SEED_W + 1, (N, N), CFG3_MU_TIMES_N / N, 1.0 / math.sqrt(N))
+    return dict(
+        name=f"cfg3_N{N}_M{M}", workload=f"dense LIF layer {N}->{N}, B={batch}, M={M}, tau={tau}",
+        batch=batch, in_shape=(N,), loss="sum_t", tau_soft=None,
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.uniform_spikes(seed, (B, N), 0.0, 1.0, 0.1),
+        layers=[_dense(W, tau[0], tau[1], M, 0.0, 1.0)])
+
+
+def draw_offsets(layers, seed=SEED_OFFSET):
+    """Per-layer t_offset draws (Alg. 2), returned as a list."""
+    dts = [(L["t_end"] - L["t_first"]) / L["M"] for L in layers]
+    return synth.t_offsets(seed, dts)
+
+
+def with_offsets(cfg, offsets):
+    """Copy of cfg whose layers carry the given t_offsets."""
+    out = dict(cfg)
+    out["layers"] = [dict(L, t_offset=float(o)) for L, o in zip(cfg["layers"], offsets)]
+    return out
+
+
+def t_max(layer):
+    """Length of a layer's DSTD window (the time scale of its tolerances)."""
+    return layer["t_end"] - layer["t_first"]
+
+
+def as_float32_layer(layer):
+    """The layer with weights rounded to float32, as the CUDA path sees them."""
+    out = dict(layer)
+    out["W"] = np.asarray(layer["W"], np.float32).astype(np.float64)
+    return out
