@@ -1,0 +1,398 @@
+#!/usr/bin/env python
+"""Benchmark: DSTD LIF forward+backward samples/s on one GB300.
+
+Workload (default): the 3-layer dense TTFS MLP 784-800-800-10, batch 256,
+M = 32 DSTD steps, (tau_m, tau_s) = (0.5, 0.25), synfire windows, CE + T +
+gamma_Q Q; one step = forward of all layers, loss, backward of all layers
+(the whole hot path: binning, contraction, scan/solve/select, dw^, both
+backward contractions). Synthetic seeded inputs of the shape of 28x28
+images (60% zero pixels, t = 1 - x); random-init weights of that
+architecture. L2 (129 MB) is flushed before every timed step.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One JSON line on stdout (rank 0). ``--impl reference`` times the float64
+CPU oracle on the host cores instead.
+"""
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "DSTD LIF fwd+bwd samples/s at 1 GB300; % of tensor/HBM roofline; peak mem"
+UNIT = "samples/s"
+WORKLOAD = "dense LIF TTFS MLP 784-800-800-10, B=256, M=32, tau=(0.5,0.25), synfire CE+T+Q, fwd+bwd"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--math", default="bf16x3", choices=["bf16x3", "bf16", "f32"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (reported baseline; spawn pool, one single-threaded worker per core)
+# ---------------------------------------------------------------------------
+_WORKER_CFG = None
+
+
+def _oracle_worker(args):
+    """Oracle fwd+bwd of samples [lo, hi) of the bench batch; returns (n, seconds)."""
+    global _WORKER_CFG
+    lo, hi = args
+    import numpy as np
+    from paper_2607_14672_gb300 import configs
+    from oracle import network
+    if _WORKER_CFG is None:
+        cfg = configs.config2()
+        _WORKER_CFG = (cfg, np.asarray(cfg["inputs"](), np.float32).astype(np.float64), cfg["labels"]())
+    cfg, t0, lab = _WORKER_CFG
+    t = time.perf_counter()
+    network.train_objective(t0[lo:hi], cfg["layers"], lab[lo:hi], cfg["tau_soft"])
+    return hi - lo, time.perf_counter() - t
+
+
+class OraclePool:
+    """Spawned single-threaded workers, one per host core (up to max_workers)."""
+
+    def __init__(self, max_workers=16):
+        import multiprocessing as mp
+        for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+            os.environ[v] = "1"
+        try:
+            ncpu = len(os.sched_getaffinity(0))
+        except Exception:
+            ncpu = os.cpu_count() or 1
+        self.workers = max(1, min(ncpu, max_workers))
+        self.pool = mp.get_context("spawn").Pool(self.workers)
+        self.pool.map(_oracle_worker, [(0, 1)] * self.workers)   # import + build the workload once
+
+    def run(self, samples_per_worker):
+        w, k = self.workers, samples_per_worker
+        chunks = [((i * k) % 256, (i * k) % 256 + k) for i in range(w)]
+        res = self.pool.map(_oracle_worker, chunks)
+        n = sum(r[0] for r in res)
+        wall = max(r[1] for r in res)
+        return n, wall
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+
+
+def oracle_throughput(samples_per_worker=8, max_workers=16):
+    """Oracle fwd+bwd of the bench workload on a bounded sample of the batch."""
+    pool = OraclePool(max_workers)
+    try:
+        n, wall = pool.run(samples_per_worker)
+    finally:
+        pool.close()
+    return {"value": n / wall, "unit": UNIT, "cores": pool.workers, "kind": "oracle",
+            "sample": f"{n} of the 256 samples ({samples_per_worker} per worker), float64 NumPy fwd+bwd of all 3 "
+                      f"layers + CE/T/Q, {pool.workers} spawned single-threaded workers, samples / slowest worker"}
+
+
+def run_reference(args, rank):
+    if rank != 0:
+        return 0
+    t_all = time.perf_counter()
+    pool = OraclePool()
+    per = 2
+    tot_n, tot_t = 0, 0.0
+    try:
+        for k in range(args.warmup + args.steps):
+            n, wall = pool.run(per)
+            if k >= args.warmup:
+                tot_n += n
+                tot_t += wall
+    finally:
+        pool.close()
+    v = tot_n / tot_t
+    ms = 256 / v * 1000.0
+    base = {"value": v, "unit": UNIT, "cores": pool.workers, "kind": "oracle",
+            "sample": f"each step {per * pool.workers} of the 256 samples ({per} per worker), float64 NumPy fwd+bwd"
+                      f" of all 3 layers + CE/T/Q on {pool.workers} spawned single-threaded workers"}
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD + " (oracle on host cores)", "global_batch": 256},
+            "impl": "reference", "cpu_baseline": base,
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "wall_s": time.perf_counter() - t_all}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            t0 = time.time()
+            while not self.lines and time.time() - t0 < 5.0:   # wait for the first sample
+                time.sleep(0.02)
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for nm, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        sm.sort()
+        med = sm[len(sm) // 2] if sm else None
+        return {"sm_mhz": med, "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def run_ours(args, rank, world, local):
+    import numpy as np
+    import torch
+
+    from paper_2607_14672_gb300 import build as _b
+    _b.build()
+    from paper_2607_14672_gb300 import configs, dstd, net
+
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    cfg = configs.config2()
+    cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
+    B = cfg["batch"]
+    n = net.DenseNet(cfg, args.math, device=dev)
+    t0 = np.asarray(cfg["inputs"](seed=configs.SEED_INPUT + rank), np.float32)
+    lab = cfg["labels"](seed=configs.SEED_LABELS + rank).astype(np.int32)
+    n.set_inputs(t0, lab)
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > L2
+
+    # warm-up (eager), then capture one step in a CUDA graph
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup)):
+            n.step()
+        stream.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            n.step()
+        for _ in range(args.warmup):
+            graph.replay()
+        stream.synchronize()
+    assert dstd.device_status(clear=True) == 0
+
+    # timed region: K graph replays, L2 flushed before each, events on the stream
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    # ~0.5 s of untimed replays right before the timed region, so the clock
+    # record (nvidia-smi, 20 ms period) covers the GPU under this load
+    with torch.cuda.stream(stream):
+        t_load = time.time()
+        while time.time() - t_load < 0.5:
+            flush.zero_()
+            for _ in range(8):
+                graph.replay()
+            stream.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for k in range(args.steps):
+            flush.zero_()
+            ev[k][0].record(stream)
+            graph.replay()
+            ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    ms_steps = [a.elapsed_time(b) for a, b in ev]
+    ms = sum(ms_steps) / len(ms_steps)
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+    value = world * B / (ms / 1000.0)
+    status = dstd.device_status(clear=True)
+
+    # per-kernel device times (eager pass with event timing; host runs ahead)
+    n_kt = min(args.steps, 50)
+    dstd.timing_enable(True)
+    with torch.cuda.stream(stream):
+        for k in range(n_kt):
+            flush.zero_()
+            torch.cuda._sleep(20_000_000)   # let the host enqueue the whole step first
+            n.step()
+    kt = dstd.timing_read()
+    dstd.timing_enable(False)
+    launches_per_step = n.launches_per_step()
+    counted = sum(c for _, c in kt.values())
+
+    # end to end through the public API: pinned H2D of the inputs, step, D2H of the loss
+    pin_t = torch.from_numpy(t0).pin_memory()
+    pin_l = torch.from_numpy(lab).pin_memory()
+    loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
+    with torch.cuda.stream(stream):
+        torch.cuda.synchronize()
+        t_e = time.perf_counter()
+        n_e2e = min(args.steps, 200)
+        for k in range(n_e2e):
+            n.t_in.copy_(pin_t, non_blocking=True)
+            n.labels.copy_(pin_l, non_blocking=True)
+            graph.replay()
+            loss_h.copy_(n.loss, non_blocking=True)
+            stream.synchronize()
+            _ = float(loss_h[0])
+        e2e_ms = (time.perf_counter() - t_e) * 1000.0 / n_e2e
+    e2e = {"value": world * B / (e2e_ms / 1000.0), "unit": UNIT,
+           "h2d_bytes_per_step": int(pin_t.numel() * 4 + pin_l.numel() * 4), "d2h_bytes_per_step": 4,
+           "ms_per_step": e2e_ms, "path": "DenseNet.step captured in a CUDA graph, replayed per step"}
+
+    # roofline of the dominant kernel
+    pk, pk_src = peaks()
+    Mp = max(8, 1 << (cfg["layers"][0]["M"] - 1).bit_length())
+    npass = {"bf16x3": 3, "bf16": 1, "f32": 1}[args.math]
+    per_kind = {k: (v[0] / v[1], v[1] // n_kt) for k, v in kt.items() if v[1] > 0}
+    dom = max(kt, key=lambda k: kt[k][0])
+    sizes = n.sizes
+    roof = None
+    if dom in ("gemm_fwd_scan", "gemm_dW", "gemm_dS_gradt") and args.math != "f32":
+        # per-launch flops of this kind summed over layers / launches of the kind
+        algo, dense = 0.0, 0.0
+        for l in range(len(sizes) - 1):
+            n_in, n_out = sizes[l], sizes[l + 1]
+            if dom == "gemm_dS_gradt" and l == 0:
+                continue
+            algo += 2 * 2 * B * n_in * n_out
+            r_out = (n_out + 127) // 128 * 128
+            r_in = (n_in + 127) // 128 * 128
+            k_in = (n_in + 63) // 64 * 64
+            k_out = (n_out + 63) // 64 * 64
+            cols = B * Mp
+            dense += 2 * npass * {"gemm_fwd_scan": r_out * cols * k_in, "gemm_dW": r_out * r_in * cols,
+                                  "gemm_dS_gradt": r_in * cols * k_out}[dom]
+        nl = per_kind[dom][1]
+        t_avg = per_kind[dom][0] / 1000.0
+        peak = pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+        achieved = algo / nl / t_avg / 1e12
+        roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None,
+                "dense_achieved": dense / nl / t_avg / 1e12, "dense_frac": dense / nl / t_avg / 1e12 / peak,
+                "peak_source": f"{pk_src} bf16 (burst)",
+                "note": "achieved = method flops (2 grid weights per input spike); dense_* = tensor-core flops "
+                        "issued by the dense formulation (Mp/2 x the method's, x3 for bf16x3)"}
+    else:
+        roof = {"kernel": dom, "bound": "hbm", "achieved": None, "peak": pk.get("hbm_gbs"), "unit": "GB/s",
+                "frac": None, "traffic": None, "peak_source": pk_src}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": {"bf16x3": "bf16x3", "bf16": "bf16", "f32": "f32"}[args.math],
+            "data": "synthetic (seeded 28x28 intensity maps, 60% zero pixels; random-init weights)",
+            "config": {"workload": WORKLOAD, "global_batch": B * world, "per_gpu_batch": B, "M": 32,
+                       "layers": [784, 800, 800, 10], "math": args.math, "l2": "flushed (512 MB write) before each "
+                       "timed step", "parallelism": "replicas" if world > 1 else "single"},
+            "roofline": roof, "clocks": clk, "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps,
+            "gpu_launches_counted_eager": {"steps": n_kt, "launches": counted},
+            "kernel_ms": {k: round(v[0], 5) for k, v in per_kind.items()},
+            "memory": {"peak_allocated_bytes": int(torch.cuda.max_memory_allocated(dev)) - flush.numel(),
+                       "workspace_bytes": int(n.workspace.numel()),
+                       "saved_state_bytes": int(sum(x.numel() for x in n.saved) + sum(x.numel() * 4 for x in n.t)),
+                       "exact_candidate_bytes": int(sum(B * sizes[l] * sizes[l + 1] * 16
+                                                        for l in range(len(sizes) - 1))),
+                       "note": "peak excludes the L2-flush buffer; exact = the exact method's retained "
+                               "candidates (16 B per sample x neuron x input, Tab. computational_complexity)"},
+            "device_status": status}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        try:
+            line["cpu_baseline"] = oracle_throughput()
+        except Exception as e:  # the baseline is reported, never fatal
+            line["cpu_baseline"] = {"value": None, "error": repr(e)}
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    args = parse()
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, rank)
+    return run_ours(args, rank, world, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

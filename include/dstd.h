@@ -1,0 +1,191 @@
+/*
+ * dstd.h -- C-ABI of libdstd: differentiable spike-time discretization (DSTD)
+ * for time-to-first-spike LIF layers on one GB300 (sm_103a).
+ *
+ * Method (arxiv 2607.14672): a LIF neuron (Eq. LIF_model_TTFS)
+ *     dv/dt = -v/tau_m + I,   dI/dt = -I/tau_s + sum_j w_ij delta(t - t_j)
+ * fires once, when v first reaches v_th. DSTD (App. B, Alg. 2) replaces each
+ * input spike t_j by weights s_jm on two neighbouring points of a fixed grid
+ *     T_m = t_first + m dt - t_offset,  m = 0..M,  dt = (t_end - t_first)/M,
+ * with s_jm = K_DSTD(t_j - T_m) (Eq. DSTD_kernel, Tab. DSTD_kernels), forms
+ * w^_im = sum_j w_ij s_jm (Eq. DSTD), and takes as spike time the first root
+ * of the discretised potential over the M intervals [T_q, T_{q+1})
+ * (Tab. timing_DSTD, Eq. timing_DSTD). The backward pass is the analytic
+ * gradient of that spike time (implicit function theorem).
+ *
+ * Conventions shared by every entry point
+ *  - All array pointers are DEVICE memory owned by the caller, row-major,
+ *    float32 unless stated, and must be 16-byte aligned. The library never
+ *    allocates device memory; scratch comes from a caller workspace whose
+ *    size the *_workspace_bytes queries return.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ *    default stream). No call synchronises the device except
+ *    dstd_device_status().
+ *  - Silent neurons carry IEEE +INFINITY, in inputs and outputs.
+ *  - Return 0 on success or a negative DSTD_E_* code; arguments are checked
+ *    before anything is launched, so an error return launched nothing
+ *    (DSTD_E_CUDA excepted: a launch was attempted and failed).
+ *  - Device-side waits (TMA / tensor-core pipelines) are bounded; a wait
+ *    that expires sets a device status word that dstd_device_status()
+ *    returns as DSTD_E_TIMEOUT. No kernel traps.
+ *  - Readings where the paper is silent (stated once here, used everywhere):
+ *    candidates exist for q = 0..M-1 only and a neuron without a crossing by
+ *    T_M is silent; a spike before T_{-1} = T_0 - dt gets no grid weight;
+ *    a spike exactly on T_m uses the t >= 0 column of Tab. DSTD_kernels.
+ */
+#ifndef DSTD_H
+#define DSTD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *dstd_stream_t; /* same type as cudaStream_t */
+
+enum {
+    DSTD_OK = 0,
+    DSTD_E_INVALID = -1,     /* null pointer, non-positive size, bad constant */
+    DSTD_E_UNSUPPORTED = -2, /* valid request outside what this build supports */
+    DSTD_E_WORKSPACE = -3,   /* workspace smaller than the query returned */
+    DSTD_E_CUDA = -4,        /* a CUDA runtime call or launch failed */
+    DSTD_E_TIMEOUT = -5,     /* a bounded device-side wait expired */
+    DSTD_E_NO_DEVICE = -6    /* no usable sm_103 device */
+};
+
+/* Arithmetic of the contraction w^ = W s (the only dense contraction).
+ *  F32    CUDA-core fp32 FMA GEMM (reference precision).
+ *  BF16X3 tcgen05 tensor cores, each fp32 operand split into bf16 hi + lo,
+ *         three products (hi*hi + hi*lo + lo*hi) accumulated in fp32 TMEM:
+ *         ~2^-17 relative operand error, for fp32 workloads.
+ *  BF16   tcgen05 tensor cores, bf16 operands, fp32 accumulation.
+ * Scan, solve, binning and every epilogue run in fp32 in all modes. */
+typedef enum { DSTD_MATH_F32 = 0, DSTD_MATH_BF16X3 = 1, DSTD_MATH_BF16 = 2 } dstd_math;
+
+/* One layer's constants (App. B.1 grid, App. C.1 synfire penalty).
+ *  tau_m, tau_s    tau_v and tau_I of Eq. LIF_model_TTFS; > 0 or INFINITY.
+ *  v_th            threshold, > 0.
+ *  t_first, t_end  DSTD window (App. C.1), t_end > t_first; M >= 1 steps.
+ *  t_offset        grid shift, in (-dt/2, dt/2] (Alg. 2 draws it per layer).
+ *  t_head, t_tail  penalty edges t_head^(l), t_tail^(l) (Eq. temporal_penalty).
+ *  gamma_head, gamma_tail, gamma_q   penalty weights (0 disables a term).
+ *  penalty_norm    factor applied to T and gamma_Q Q and to their gradients:
+ *                  1/B for dense layers (mini-batch mean, Eq. cost_function),
+ *                  1/(B H W) for conv layers (App. C.1). */
+typedef struct {
+    float tau_m, tau_s;
+    float v_th;
+    float t_first, t_end;
+    int32_t M;
+    float t_offset;
+    float t_head, t_tail;
+    float gamma_head, gamma_tail, gamma_q;
+    float penalty_norm;
+} dstd_params;
+
+/* Per-neuron state that dstd_dense_fwd saves for dstd_dense_bwd:
+ * q (int32, interval index of the spike, M if silent), s (spike time minus
+ * T_q), vdot (dv^/dt at the spike, floored at 1e-6 v_th/dt), each [B, N_out].
+ * Opaque to the caller apart from its size. */
+size_t dstd_dense_saved_bytes(int B, int N_out);
+
+/* Workspace bytes needed by dstd_dense_fwd and dstd_dense_bwd (the max of the
+ * two) for these sizes and math mode; 0 on invalid arguments. */
+size_t dstd_dense_workspace_bytes(int B, int N_in, int N_out, const dstd_params *p, dstd_math math);
+
+/* Binning alone (Eq. DSTD_kernel, Tab. DSTD_kernels): spike times -> grid
+ * weights.
+ *  t_in  [B, N]      input spike times (+inf = silent).
+ *  s     [B, M, N]   out: s_jm for m = 0..M-1 (zero outside the support).
+ *  ds    [B, M, N]   out (may be NULL): d s_jm / d t_j (one-sided at knots). */
+int dstd_binning(const float *t_in, int B, int N, const dstd_params *p, float *s, float *ds,
+                 dstd_stream_t stream);
+
+/* Binning + contraction alone: w^_im = sum_j w_ij s_jm (Eq. DSTD).
+ *  t_in [B, N_in], W [N_out, N_in]  ->  what [B, N_out, M]. */
+int dstd_dense_what(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                    dstd_math math, float *what, void *workspace, size_t ws_bytes, dstd_stream_t stream);
+
+/* Scan + threshold solve + first-spike select alone, from given w^
+ * (Tab. timing_DSTD, Eq. timing_DSTD), plus the penalty terms.
+ *  what    [B, N_out, M]  discretised inputs w^_im.
+ *  t_out   [B, N_out]     out: spike times (+inf = silent).
+ *  saved   dstd_dense_saved_bytes(B, N_out) bytes, out (may be NULL).
+ *  penalty float[4] out (may be NULL): {norm * T, gamma_q * norm * Q,
+ *          number of silent neurons, number of firing neurons}. Q needs
+ *          the weight row sums: w_rowsum [N_out] (may be NULL = Q term 0). */
+int dstd_scan_solve(const float *what, int B, int N_out, const dstd_params *p, const float *w_rowsum,
+                    float *t_out, void *saved, float *penalty, dstd_stream_t stream);
+
+/* Forward of one dense DSTD layer (Alg. 2 body): binning, contraction,
+ * scan/solve/select, silent mask and penalty terms.
+ *  t_in [B, N_in], W [N_out, N_in] (fp32; converted per call for tensor cores).
+ *  t_out [B, N_out], saved, penalty[4] as in dstd_scan_solve. */
+int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                   dstd_math math, float *t_out, void *saved, float *penalty, void *workspace,
+                   size_t ws_bytes, dstd_stream_t stream);
+
+/* Backward of one dense DSTD layer.
+ *  g_t_out [B, N_out] dC/dt_out from above (the loss or the next layer); the
+ *          layer adds its own temporal-penalty gradient (params) itself.
+ *  g_t_in  [B, N_in]  out (may be NULL): dC/dt_in; 0 for silent inputs.
+ *  g_W     [N_out, N_in] out (overwritten): dC/dW including the dead-neuron
+ *          term -gamma_q * norm * (number of samples where neuron i is silent).
+ * dt_i/dw^_im = -K(t_i - T_m)/v^'(t_i) for m <= q_i (IFT on v^(t_i) = v_th). */
+int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const void *saved,
+                   const float *g_t_out, int B, int N_in, int N_out, const dstd_params *p, dstd_math math,
+                   float *g_t_in, float *g_W, void *workspace, size_t ws_bytes, dstd_stream_t stream);
+
+/* Cross-entropy over softmax(-t/tau_soft) (Eqs. cost_function, L, S_i),
+ * mini-batch mean; a silent output enters with the constant time t_silent
+ * and passes no gradient.
+ *  t_L [B, C], labels [B] int32 in [0, C); loss float[1] out; g_t_L [B, C] out. */
+int dstd_ce_loss(const float *t_L, const int32_t *labels, int B, int C, float tau_soft, float t_silent,
+                 float *loss, float *g_t_L, dstd_stream_t stream);
+
+/* Loss = sum of the output spike times that fire; g = 1 where fired, else 0.
+ *  t [n]; loss float[1] out; g [n] out. */
+int dstd_sum_t_loss(const float *t, int64_t n, float *loss, float *g, dstd_stream_t stream);
+
+/* AdamW step (App. C.1; decoupled weight decay), in place on w, m, v [n];
+ * step is the 1-based update count. */
+int dstd_adamw(float *w, const float *g, float *m, float *v, int64_t n, float lr, float beta1,
+               float beta2, float eps, float weight_decay, int step, dstd_stream_t stream);
+
+/* Kernel timing (tracing). While enabled, the library brackets every kernel
+ * it launches with a CUDA event pair on the launching stream and files the
+ * pair under the kernel's kind (dstd_kernel_kind_name); launches made while
+ * the stream is being captured into a CUDA graph are not timed.
+ * dstd_timing_enable(on) turns timing on/off and clears the counters.
+ * dstd_timing_read(kind, total_ms, launches) synchronises the device and
+ * returns the accumulated device time and launch count of one kind. */
+int dstd_timing_enable(int on);
+int dstd_timing_read(int kind, float *total_ms, int64_t *launches);
+int dstd_kernel_kind_count(void);
+const char *dstd_kernel_kind_name(int kind);
+
+/* Self-test of the bounded device waits (failure detection without a fault):
+ * launches one block whose thread waits on an mbarrier that nothing ever
+ * completes, giving up after timeout_us microseconds (at most 10 s) and
+ * setting the device status word, which dstd_device_status() then reports as
+ * DSTD_E_TIMEOUT. The context stays usable. */
+int dstd_selftest_wait_timeout(uint32_t timeout_us, dstd_stream_t stream);
+
+/* Synchronises the current device and returns DSTD_OK, DSTD_E_TIMEOUT if a
+ * bounded device wait expired since the last clear, or DSTD_E_CUDA.
+ * clear != 0 resets the status word. */
+int dstd_device_status(int clear);
+
+/* Message for a DSTD_E_* code (static string). */
+const char *dstd_error_string(int code);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int dstd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DSTD_H */

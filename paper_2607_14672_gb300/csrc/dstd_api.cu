@@ -1,0 +1,585 @@
+// C-ABI entry points of libdstd (include/dstd.h): argument checks, workspace
+// layout and the order of kernel launches for one dense DSTD layer.
+#include "dstd_internal.cuh"
+
+#include <math.h>
+#include <string.h>
+
+#include <mutex>
+#include <utility>
+#include <vector>
+
+namespace dstd {
+int tc_gemm_splits_valid(int K, int splits);
+}
+
+using namespace dstd;
+
+namespace {
+
+constexpr int kVersion = 100;  // 0.1.0
+
+// 256-byte bump allocator over a caller workspace (nullptr base = size query)
+struct Bump {
+    char *base;
+    size_t off = 0;
+    explicit Bump(void *b) : base(static_cast<char *>(b)) {}
+    template <class T>
+    T *take(size_t count) {
+        off = (off + 255) & ~(size_t)255;
+        T *p = base ? reinterpret_cast<T *>(base + off) : nullptr;
+        off += count * sizeof(T);
+        return p;
+    }
+};
+
+bool finite_pos_or_inf(float x) { return (x > 0.0f && isfinite(x)) || (isinf(x) && x > 0.0f); }
+
+int check_params(const dstd_params *p) {
+    if (!p) return DSTD_E_INVALID;
+    if (!finite_pos_or_inf(p->tau_m) || !finite_pos_or_inf(p->tau_s)) return DSTD_E_INVALID;
+    if (!(p->v_th > 0.0f) || !isfinite(p->v_th)) return DSTD_E_INVALID;
+    if (!isfinite(p->t_first) || !isfinite(p->t_end) || !(p->t_end > p->t_first)) return DSTD_E_INVALID;
+    if (p->M < 1) return DSTD_E_INVALID;
+    if (p->M > 256) return DSTD_E_UNSUPPORTED;
+    const double dt = ((double)p->t_end - (double)p->t_first) / p->M;
+    if (!isfinite(p->t_offset) || !(p->t_offset > -dt / 2) || !(p->t_offset <= dt / 2 * (1 + 1e-6)))
+        return DSTD_E_INVALID;
+    if (!isfinite(p->gamma_head) || !isfinite(p->gamma_tail) || !isfinite(p->gamma_q) ||
+        !isfinite(p->penalty_norm) || isnan(p->t_head) || isnan(p->t_tail))
+        return DSTD_E_INVALID;
+    return DSTD_OK;
+}
+
+int check_math(dstd_math m, int Mp) {
+    if (m != DSTD_MATH_F32 && m != DSTD_MATH_BF16X3 && m != DSTD_MATH_BF16) return DSTD_E_INVALID;
+    if (m != DSTD_MATH_F32 && Mp > 128) return DSTD_E_UNSUPPORTED;  // one sample per tensor-core tile
+    return DSTD_OK;
+}
+
+OpKind op_of(dstd_math m) {
+    return m == DSTD_MATH_F32 ? OpKind::F32 : (m == DSTD_MATH_BF16X3 ? OpKind::BF16X3 : OpKind::BF16);
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int device_ok() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DSTD_E_NO_DEVICE;
+    static int cached_dev = -1, cached_ok = 0;
+    if (dev == cached_dev) return cached_ok ? DSTD_OK : DSTD_E_NO_DEVICE;
+    int maj = 0, min = 0;
+    if (cudaDeviceGetAttribute(&maj, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&min, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+        return DSTD_E_NO_DEVICE;
+    cached_dev = dev;
+    cached_ok = (maj == 10 && min == 3);
+    return cached_ok ? DSTD_OK : DSTD_E_NO_DEVICE;
+}
+
+inline int cu(cudaError_t e) { return e == cudaSuccess ? DSTD_OK : DSTD_E_CUDA; }
+
+// ---------------------------------------------------------------------------
+// Kernel timing: an event pair per launch, filed by kernel kind.
+// ---------------------------------------------------------------------------
+enum Kind {
+    KK_PREP = 0, KK_BIN, KK_BIN_T, KK_GEMM_FWD, KK_SCAN, KK_DWHAT, KK_GEMM_DS, KK_GT, KK_GEMM_DW, KK_REDUCE,
+    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_COUNT
+};
+const char *const kKindNames[KK_COUNT] = {
+    "prep_weights", "binning", "binning_T", "gemm_fwd_scan", "scan_solve", "dwhat", "gemm_dS_gradt",
+    "gradt_gather", "gemm_dW", "dw_reduce", "loss", "adamw", "binning_public", "what_public", "selftest"};
+
+struct Timing {
+    std::mutex mu;
+    bool on = false;
+    std::vector<cudaEvent_t> pool;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending[KK_COUNT];
+    double ms[KK_COUNT] = {};
+    long long n[KK_COUNT] = {};
+};
+Timing g_timing;
+
+cudaEvent_t take_event() {
+    cudaEvent_t e = nullptr;
+    if (!g_timing.pool.empty()) {
+        e = g_timing.pool.back();
+        g_timing.pool.pop_back();
+    } else if (cudaEventCreate(&e) != cudaSuccess) {
+        e = nullptr;
+    }
+    return e;
+}
+
+// drain pending pairs into the totals (caller holds the lock, device synced)
+void drain_pending() {
+    for (int k = 0; k < KK_COUNT; ++k) {
+        for (auto &pr : g_timing.pending[k]) {
+            float ms = 0.f;
+            if (cudaEventElapsedTime(&ms, pr.first, pr.second) == cudaSuccess) {
+                g_timing.ms[k] += ms;
+                g_timing.n[k] += 1;
+            }
+            g_timing.pool.push_back(pr.first);
+            g_timing.pool.push_back(pr.second);
+        }
+        g_timing.pending[k].clear();
+    }
+}
+
+struct Timed {
+    int kind;
+    cudaStream_t st;
+    cudaEvent_t a = nullptr;
+    Timed(int k, cudaStream_t s) : kind(k), st(s) {
+        if (!g_timing.on) return;
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return;
+        std::lock_guard<std::mutex> lk(g_timing.mu);
+        a = take_event();
+        if (a && cudaEventRecord(a, s) != cudaSuccess) a = nullptr;
+    }
+    ~Timed() {
+        if (!a) return;
+        std::lock_guard<std::mutex> lk(g_timing.mu);
+        cudaEvent_t b = take_event();
+        if (b && cudaEventRecord(b, st) == cudaSuccess) g_timing.pending[kind].push_back({a, b});
+        else g_timing.pool.push_back(a);
+    }
+};
+#define TRY(x)                       \
+    do {                             \
+        int _r = (x);                \
+        if (_r != DSTD_OK) return _r; \
+    } while (0)
+
+// ---------------------------------------------------------------------------
+// Workspace layouts (one for the forward, one for the backward; both start at
+// the workspace base).
+// ---------------------------------------------------------------------------
+struct FwdWs {
+    __nv_bfloat16 *w_hi = nullptr, *w_lo = nullptr, *s_hi = nullptr, *s_lo = nullptr;
+    float *s32 = nullptr, *D = nullptr, *rowsum = nullptr;
+    size_t bytes = 0;
+    int kpad = 0;
+};
+
+FwdWs fwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool need_D) {
+    FwdWs w;
+    Bump b(base);
+    w.kpad = pad8(N_in);
+    const long long cols = (long long)B * Mp;
+    w.rowsum = b.take<float>(N_out);
+    if (op == OpKind::F32) {
+        w.s32 = b.take<float>((size_t)cols * w.kpad);
+        w.D = b.take<float>((size_t)N_out * cols);
+    } else {
+        w.w_hi = b.take<__nv_bfloat16>((size_t)N_out * w.kpad);
+        if (op == OpKind::BF16X3) w.w_lo = b.take<__nv_bfloat16>((size_t)N_out * w.kpad);
+        w.s_hi = b.take<__nv_bfloat16>((size_t)cols * w.kpad);
+        if (op == OpKind::BF16X3) w.s_lo = b.take<__nv_bfloat16>((size_t)cols * w.kpad);
+        if (need_D) w.D = b.take<float>((size_t)N_out * cols);
+    }
+    w.bytes = b.off;
+    return w;
+}
+
+struct BwdWs {
+    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *dB_hi = nullptr,
+                  *dB_lo = nullptr, *sT_hi = nullptr, *sT_lo = nullptr;
+    float *wt32 = nullptr, *dA32 = nullptr, *dB32 = nullptr, *sT32 = nullptr, *DS = nullptr, *part = nullptr,
+          *count = nullptr;
+    int ldt = 0, ldn = 0, ldbm = 0, ldp = 0, splits = 1;
+    size_t bytes = 0;
+};
+
+int dw_splits(int N_in, int N_out, int K, OpKind op) {
+    const int tm = op == OpKind::F32 ? 64 : 128, tn = op == OpKind::F32 ? 64 : 128;
+    const long long tiles = (long long)((N_out + tm - 1) / tm) * ((N_in + tn - 1) / tn);
+    const int kunit = op == OpKind::F32 ? 16 : 64;
+    const int ktiles = (K + kunit - 1) / kunit;
+    long long want = (2 * 152 + tiles - 1) / tiles;
+    int s = (int)(want < 1 ? 1 : (want > ktiles ? ktiles : want));
+    if (s > 64) s = 64;
+    if (op != OpKind::F32)
+        while (s > 1 && !tc_gemm_splits_valid(K, s)) --s;
+    return s < 1 ? 1 : s;
+}
+
+BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool need_gt) {
+    BwdWs w;
+    Bump b(base);
+    const long long cols = (long long)B * Mp;
+    w.ldt = pad8(N_out);
+    w.ldn = pad8(N_out);
+    w.ldbm = pad8((int)cols);
+    w.ldp = (N_in + 3) & ~3;
+    w.splits = dw_splits(N_in, N_out, (int)cols, op);
+    w.count = b.take<float>(N_out);
+    w.part = b.take<float>((size_t)w.splits * N_out * w.ldp);
+    if (op == OpKind::F32) {
+        w.dA32 = b.take<float>((size_t)N_out * w.ldbm);
+        w.dB32 = b.take<float>((size_t)cols * w.ldn);
+        w.sT32 = b.take<float>((size_t)N_in * w.ldbm);
+        if (need_gt) {
+            w.wt32 = b.take<float>((size_t)N_in * w.ldt);
+            w.DS = b.take<float>((size_t)N_in * cols);
+        }
+    } else {
+        const bool three = op == OpKind::BF16X3;
+        w.dA_hi = b.take<__nv_bfloat16>((size_t)N_out * w.ldbm);
+        if (three) w.dA_lo = b.take<__nv_bfloat16>((size_t)N_out * w.ldbm);
+        w.dB_hi = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
+        if (three) w.dB_lo = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
+        w.sT_hi = b.take<__nv_bfloat16>((size_t)N_in * w.ldbm);
+        if (three) w.sT_lo = b.take<__nv_bfloat16>((size_t)N_in * w.ldbm);
+        if (need_gt) {
+            w.wt_hi = b.take<__nv_bfloat16>((size_t)N_in * w.ldt);
+            if (three) w.wt_lo = b.take<__nv_bfloat16>((size_t)N_in * w.ldt);
+        }
+    }
+    w.bytes = b.off;
+    return w;
+}
+
+struct Saved {
+    int *q;
+    float *s, *vdot;
+};
+Saved saved_view(void *saved, int B, int N_out) {
+    Bump b(saved);
+    Saved v;
+    v.q = b.take<int>((size_t)B * N_out);
+    v.s = b.take<float>((size_t)B * N_out);
+    v.vdot = b.take<float>((size_t)B * N_out);
+    return v;
+}
+
+int check_sizes(int B, int N_in, int N_out) {
+    if (B < 1 || N_in < 1 || N_out < 1) return DSTD_E_INVALID;
+    // grid limits: B is a grid y extent (<= 65535); row tiles of 32 for N
+    if (B > 65535 || N_in > (1 << 20) || N_out > (1 << 20)) return DSTD_E_UNSUPPORTED;
+    return DSTD_OK;
+}
+
+// forward up to w^: binning + contraction; Scan epilogue fused (TC) unless
+// `store_D` (then the fp32 w^ lands in ws.D, layout [N_out, B*Mp]).
+int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N_out, const LifConst &c, OpKind op,
+                       const FwdWs &ws, bool store_D, const Saved *sv, float *t_out, float *penalty,
+                       cudaStream_t st) {
+    const long long cols = (long long)B * c.Mp;
+    if (op == OpKind::F32) {
+        {
+            Timed tm(KK_PREP, st);
+            TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, nullptr, nullptr, 0, nullptr, 0,
+                                       ws.rowsum, st)));
+        }
+        {
+            Timed tm(KK_BIN, st);
+            TRY(cu(launch_binning(t_in, B, N_in, c, op, false, ws.s32, nullptr, ws.kpad, st)));
+        }
+        {
+            Timed tm(KK_GEMM_FWD, st);
+            TRY(cu(launch_sgemm_tn(W, N_in, ws.s32, ws.kpad, ws.D, (int)cols, N_out, (int)cols, N_in, 1, 0, st)));
+        }
+        if (!store_D) {
+            Timed tm(KK_SCAN, st);
+            TRY(cu(launch_scan_solve(ws.D, c.Mp, cols, B, N_out, c, ws.rowsum, t_out, sv->q, sv->s, sv->vdot,
+                                     penalty, st)));
+        }
+        return DSTD_OK;
+    }
+    {
+        Timed tm(KK_PREP, st);
+        TRY(cu(launch_prep_weights(W, N_out, N_in, op, ws.w_hi, ws.w_lo, ws.kpad, nullptr, nullptr, 0, nullptr, 0,
+                                   ws.rowsum, st)));
+    }
+    {
+        Timed tm(KK_BIN, st);
+        TRY(cu(launch_binning(t_in, B, N_in, c, op, false, ws.s_hi, ws.s_lo, ws.kpad, st)));
+    }
+    TcEpiArgs a{};
+    a.c = c;
+    a.B = B;
+    a.N = N_out;
+    Timed tm(KK_GEMM_FWD, st);
+    if (store_D) {
+        a.D = ws.D;
+        a.ldd = cols;
+        a.zstride = 0;
+        return cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
+                                 Epi::Store, a, st));
+    }
+    a.rowsum = ws.rowsum;
+    a.t_out = t_out;
+    a.q = sv->q;
+    a.s = sv->s;
+    a.vdot = sv->vdot;
+    a.penalty = penalty;
+    return cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
+                             Epi::Scan, a, st));
+}
+
+}  // namespace
+
+extern "C" {
+
+int dstd_version(void) { return kVersion; }
+
+const char *dstd_error_string(int code) {
+    switch (code) {
+        case DSTD_OK: return "ok";
+        case DSTD_E_INVALID: return "invalid argument";
+        case DSTD_E_UNSUPPORTED: return "unsupported size or mode";
+        case DSTD_E_WORKSPACE: return "workspace too small";
+        case DSTD_E_CUDA: return "CUDA call or kernel launch failed";
+        case DSTD_E_TIMEOUT: return "a bounded device-side wait expired";
+        case DSTD_E_NO_DEVICE: return "no usable sm_103 device";
+        default: return "unknown error code";
+    }
+}
+
+size_t dstd_dense_saved_bytes(int B, int N_out) {
+    if (B < 1 || N_out < 1) return 0;
+    Bump b(nullptr);
+    b.take<int>((size_t)B * N_out);
+    b.take<float>((size_t)B * N_out);
+    b.take<float>((size_t)B * N_out);
+    return b.off;
+}
+
+size_t dstd_dense_workspace_bytes(int B, int N_in, int N_out, const dstd_params *p, dstd_math math) {
+    if (check_sizes(B, N_in, N_out) != DSTD_OK || check_params(p) != DSTD_OK) return 0;
+    const int Mp = padded_M(p->M);
+    if (check_math(math, Mp) != DSTD_OK) return 0;
+    const OpKind op = op_of(math);
+    size_t f = fwd_layout(nullptr, B, N_in, N_out, Mp, op, true).bytes;
+    size_t g = bwd_layout(nullptr, B, N_in, N_out, Mp, op, true).bytes;
+    return f > g ? f : g;
+}
+
+int dstd_binning(const float *t_in, int B, int N, const dstd_params *p, float *s, float *ds,
+                 dstd_stream_t stream) {
+    if (!t_in || !s || B < 1 || N < 1) return DSTD_E_INVALID;
+    TRY(check_params(p));
+    TRY(device_ok());
+    LifConst c = make_const(*p, padded_M(p->M));
+    Timed tm(KK_BIN_PUB, (cudaStream_t)stream);
+    return cu(launch_binning_public(t_in, B, N, c, s, ds, (cudaStream_t)stream));
+}
+
+int dstd_dense_what(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                    dstd_math math, float *what, void *workspace, size_t ws_bytes, dstd_stream_t stream) {
+    if (!t_in || !W || !what || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace)) return DSTD_E_INVALID;
+    const OpKind op = op_of(math);
+    if (ws_bytes < fwd_layout(nullptr, B, N_in, N_out, Mp, op, true).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    FwdWs ws = fwd_layout(workspace, B, N_in, N_out, Mp, op, true);
+    TRY(dense_forward_core(t_in, W, B, N_in, N_out, c, op, ws, true, nullptr, nullptr, nullptr, st));
+    Timed tm(KK_WHAT_PUB, st);
+    return cu(launch_what_to_public(ws.D, (long long)B * Mp, B, N_out, p->M, Mp, what, st));
+}
+
+int dstd_scan_solve(const float *what, int B, int N_out, const dstd_params *p, const float *w_rowsum, float *t_out,
+                    void *saved, float *penalty, dstd_stream_t stream) {
+    if (!what || !t_out || B < 1 || N_out < 1) return DSTD_E_INVALID;
+    TRY(check_params(p));
+    TRY(device_ok());
+    cudaStream_t st = (cudaStream_t)stream;
+    LifConst c = make_const(*p, padded_M(p->M));
+    Saved sv{nullptr, nullptr, nullptr};
+    if (saved) sv = saved_view(saved, B, N_out);
+    if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
+    Timed tm(KK_SCAN, st);
+    return cu(launch_scan_solve(what, (long long)N_out * p->M, p->M, B, N_out, c, w_rowsum, t_out, sv.q, sv.s,
+                                sv.vdot, penalty, st));
+}
+
+int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                   dstd_math math, float *t_out, void *saved, float *penalty, void *workspace, size_t ws_bytes,
+                   dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    const OpKind op = op_of(math);
+    if (ws_bytes < fwd_layout(nullptr, B, N_in, N_out, Mp, op, false).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    FwdWs ws = fwd_layout(workspace, B, N_in, N_out, Mp, op, false);
+    Saved sv = saved_view(saved, B, N_out);
+    if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
+    return dense_forward_core(t_in, W, B, N_in, N_out, c, op, ws, false, &sv, t_out, penalty, st);
+}
+
+int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const void *saved, const float *g_t_out,
+                   int B, int N_in, int N_out, const dstd_params *p, dstd_math math, float *g_t_in, float *g_W,
+                   void *workspace, size_t ws_bytes, dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved || !g_W || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    const OpKind op = op_of(math);
+    const bool need_gt = g_t_in != nullptr;
+    if (ws_bytes < bwd_layout(nullptr, B, N_in, N_out, Mp, op, need_gt).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    BwdWs ws = bwd_layout(workspace, B, N_in, N_out, Mp, op, need_gt);
+    Saved sv = saved_view(const_cast<void *>(saved), B, N_out);
+    const long long cols = (long long)B * Mp;
+    const float qcoef = -p->gamma_q * p->penalty_norm;
+    if (op == OpKind::F32) {
+        {
+            Timed tm(KK_DWHAT, st);
+            TRY(cu(launch_dwhat(t_out, sv.q, sv.s, sv.vdot, g_t_out, B, N_out, c, op, ws.dA32, nullptr, ws.ldbm,
+                                ws.dB32, nullptr, ws.ldn, ws.count, st)));
+        }
+        if (need_gt) {
+            {
+                Timed tm(KK_PREP, st);
+                TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, nullptr, nullptr, 0, ws.wt32,
+                                           ws.ldt, nullptr, st)));
+            }
+            {
+                Timed tm(KK_GEMM_DS, st);
+                TRY(cu(launch_sgemm_tn(ws.wt32, ws.ldt, ws.dB32, ws.ldn, ws.DS, (int)cols, N_in, (int)cols, N_out, 1,
+                                       0, st)));
+            }
+            {
+                Timed tm(KK_GT, st);
+                TRY(cu(launch_gt_from_ds(ws.DS, cols, t_in, B, N_in, c, g_t_in, st)));
+            }
+        }
+        {
+            Timed tm(KK_BIN_T, st);
+            TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT32, nullptr, ws.ldbm, st)));
+        }
+        const long long zs = (long long)N_out * ws.ldp;
+        {
+            Timed tm(KK_GEMM_DW, st);
+            TRY(cu(launch_sgemm_tn(ws.dA32, ws.ldbm, ws.sT32, ws.ldbm, ws.part, ws.ldp, N_out, N_in, (int)cols,
+                                   ws.splits, zs, st)));
+        }
+        Timed tm(KK_REDUCE, st);
+        return cu(launch_dw_reduce(ws.part, ws.splits, zs, ws.ldp, N_out, N_in, ws.count, qcoef, g_W, st));
+    }
+    {
+        Timed tm(KK_DWHAT, st);
+        TRY(cu(launch_dwhat(t_out, sv.q, sv.s, sv.vdot, g_t_out, B, N_out, c, op, ws.dA_hi, ws.dA_lo, ws.ldbm,
+                            ws.dB_hi, ws.dB_lo, ws.ldn, ws.count, st)));
+    }
+    if (need_gt) {
+        {
+            Timed tm(KK_PREP, st);
+            TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, ws.wt_hi, ws.wt_lo, ws.ldt, nullptr,
+                                       0, nullptr, st)));
+        }
+        TcEpiArgs a{};
+        a.c = c;
+        a.B = B;
+        a.N = N_in;
+        a.t_in = t_in;
+        a.g_t_in = g_t_in;
+        Timed tm(KK_GEMM_DS, st);
+        TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dB_hi, ws.dB_lo, ws.ldn, N_in, (int)cols, N_out, 1, op,
+                              Epi::GradT, a, st)));
+    }
+    {
+        Timed tm(KK_BIN_T, st);
+        TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st)));
+    }
+    TcEpiArgs a{};
+    a.D = ws.part;
+    a.ldd = ws.ldp;
+    a.zstride = (long long)N_out * ws.ldp;
+    {
+        Timed tm(KK_GEMM_DW, st);
+        TRY(cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, N_out, N_in, (int)cols,
+                              ws.splits, op, Epi::Store, a, st)));
+    }
+    Timed tm(KK_REDUCE, st);
+    return cu(launch_dw_reduce(ws.part, ws.splits, a.zstride, ws.ldp, N_out, N_in, ws.count, qcoef, g_W, st));
+}
+
+int dstd_ce_loss(const float *t_L, const int32_t *labels, int B, int C, float tau_soft, float t_silent, float *loss,
+                 float *g_t_L, dstd_stream_t stream) {
+    if (!t_L || !labels || !loss || !g_t_L || B < 1 || C < 1) return DSTD_E_INVALID;
+    if (!(tau_soft > 0.0f) || !isfinite(tau_soft) || !isfinite(t_silent)) return DSTD_E_INVALID;
+    TRY(device_ok());
+    Timed tm(KK_LOSS, (cudaStream_t)stream);
+    return cu(launch_ce_loss(t_L, labels, B, C, tau_soft, t_silent, loss, g_t_L, (cudaStream_t)stream));
+}
+
+int dstd_sum_t_loss(const float *t, int64_t n, float *loss, float *g, dstd_stream_t stream) {
+    if (!t || !loss || !g || n < 1) return DSTD_E_INVALID;
+    TRY(device_ok());
+    Timed tm(KK_LOSS, (cudaStream_t)stream);
+    return cu(launch_sum_t(t, n, loss, g, (cudaStream_t)stream));
+}
+
+int dstd_adamw(float *w, const float *g, float *m, float *v, int64_t n, float lr, float beta1, float beta2, float eps,
+               float weight_decay, int step, dstd_stream_t stream) {
+    if (!w || !g || !m || !v || n < 1 || step < 1) return DSTD_E_INVALID;
+    if (!(lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) || !(beta2 >= 0.0f && beta2 < 1.0f) || !(eps > 0.0f))
+        return DSTD_E_INVALID;
+    TRY(device_ok());
+    Timed tm(KK_ADAMW, (cudaStream_t)stream);
+    return cu(launch_adamw(w, g, m, v, n, lr, beta1, beta2, eps, weight_decay, step, (cudaStream_t)stream));
+}
+
+int dstd_timing_enable(int on) {
+    if (cudaDeviceSynchronize() != cudaSuccess) return DSTD_E_CUDA;
+    std::lock_guard<std::mutex> lk(g_timing.mu);
+    drain_pending();
+    for (int k = 0; k < KK_COUNT; ++k) {
+        g_timing.ms[k] = 0.0;
+        g_timing.n[k] = 0;
+    }
+    g_timing.on = on != 0;
+    return DSTD_OK;
+}
+
+int dstd_timing_read(int kind, float *total_ms, int64_t *launches) {
+    if (kind < 0 || kind >= KK_COUNT || !total_ms || !launches) return DSTD_E_INVALID;
+    if (cudaDeviceSynchronize() != cudaSuccess) return DSTD_E_CUDA;
+    std::lock_guard<std::mutex> lk(g_timing.mu);
+    drain_pending();
+    *total_ms = (float)g_timing.ms[kind];
+    *launches = g_timing.n[kind];
+    return DSTD_OK;
+}
+
+int dstd_kernel_kind_count(void) { return KK_COUNT; }
+
+const char *dstd_kernel_kind_name(int kind) {
+    return (kind >= 0 && kind < KK_COUNT) ? kKindNames[kind] : "unknown";
+}
+
+int dstd_selftest_wait_timeout(uint32_t timeout_us, dstd_stream_t stream) {
+    if (timeout_us == 0 || timeout_us > 10000000u) return DSTD_E_INVALID;
+    TRY(device_ok());
+    Timed tm(KK_SELFTEST, (cudaStream_t)stream);
+    return cu(launch_wait_selftest(1000ull * timeout_us, (cudaStream_t)stream));
+}
+
+int dstd_device_status(int clear) {
+    if (cudaDeviceSynchronize() != cudaSuccess) return DSTD_E_CUDA;
+    unsigned int s = 0;
+    if (status_read(&s, clear) != cudaSuccess) return DSTD_E_CUDA;
+    return (s & STATUS_TIMEOUT) ? DSTD_E_TIMEOUT : DSTD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,511 @@
+// Tensor-core contraction of the DSTD layer on sm_103a (tcgen05 + TMA).
+//
+// D[r, c] = sum_k A[r, k] B[c, k] with A and B bf16, K-major, staged by TMA
+// (128-byte swizzle, no multicast) through a STAGES-deep mbarrier ring; one
+// thread issues tcgen05.mma (cta_group::1, M = 128, N = BN, K = 16 per
+// instruction) into an fp32 accumulator in TMEM; four warps read it back
+// with tcgen05.ld (lane = row) and run the fused epilogue:
+//   Store  plain fp32 tile (split-K partials of the weight gradient),
+//   Scan   rows = neurons, columns = (sample, grid step): the scan / threshold
+//          solve / first-spike select of Tab. timing_DSTD, so w^ never
+//          reaches HBM,
+//   GradT  rows = inputs, columns = (sample, grid step): the input-time
+//          gradient sum_m dS ds/dt, so dS never reaches HBM.
+// BF16X3 splits each fp32 operand into bf16 hi + lo and accumulates
+// hi*hi + hi*lo + lo*hi (three MMAs per K step) for ~fp32 operand accuracy.
+//
+// Every mbarrier wait is bounded (about 2 s of %globaltimer); an expired wait
+// sets the device status word, skips the epilogue and frees TMEM.
+#include "dstd_internal.cuh"
+
+#include <cuda.h>
+#include <mutex>
+
+namespace dstd {
+
+// device status word: bit STATUS_TIMEOUT is set by an expired bounded wait
+__device__ unsigned int g_status = 0;
+
+__device__ __forceinline__ void set_status(unsigned int code) { atomicOr(&g_status, code); }
+
+cudaError_t status_read(unsigned int *out, int clear) {
+    cudaError_t e = cudaMemcpyFromSymbol(out, g_status, sizeof(unsigned int));
+    if (e != cudaSuccess || !clear) return e;
+    unsigned int z = 0;
+    return cudaMemcpyToSymbol(g_status, &z, sizeof(z));
+}
+
+namespace tc {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // bf16 elements per 128-byte swizzled row
+constexpr unsigned long long WAIT_NS = 2000000000ull;
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ uint64_t globaltimer() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// bounded wait: false if the phase did not complete within limit_ns
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          unsigned long long limit_ns = WAIT_NS) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    for (;;) {
+        for (int i = 0; i < 64; ++i)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (globaltimer() - t0 > limit_ns) return false;
+    }
+}
+
+// One thread waits on a barrier phase that never completes; the bounded wait
+// expires and records a timeout in the status word.
+__global__ void k_wait_selftest(unsigned long long limit_ns) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        if (!mbar_wait(&bar, 0, limit_ns)) set_status(STATUS_TIMEOUT);
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint64_t *bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+            "r"(dst),
+        "l"((uint64_t)map), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
+        "}\n" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_u32(bar))
+                 : "memory");
+}
+
+// 32 lanes x 32 consecutive fp32 columns; the wait is in the same asm block
+// so the registers are valid when the statement completes.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        "tcgen05.wait::ld.sync.aligned;\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]),
+          "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]),
+          "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor (tcgen05 format): K-major operand tile with
+// 128-byte rows in 128-byte-swizzle layout; 8-row core-matrix groups are
+// 1024 bytes apart (SBO); LBO is not used by swizzled K-major layouts.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address >> 4
+    d |= (uint64_t)1 << 16;                     // LBO (encoded, ignored)
+    d |= (uint64_t)(1024u >> 4) << 32;          // SBO
+    d |= (uint64_t)1 << 46;                     // descriptor version
+    d |= (uint64_t)2 << 61;                     // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+template <int NPASS, int BN>
+struct Cfg {
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int NOP = (NPASS == 3) ? 2 : 1;
+    static constexpr int STAGE = NOP * (A_BYTES + B_BYTES);
+    static constexpr int STAGES = (200 * 1024) / STAGE > 8 ? 8 : (200 * 1024) / STAGE;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+};
+
+// ---------------------------------------------------------------------------
+// Epilogues. Each thread owns one accumulator row (its TMEM lane).
+// ---------------------------------------------------------------------------
+template <int BN>
+__device__ __forceinline__ void epi_store(uint32_t tbase, int row, int col0, int R, int Cn, const TcEpiArgs &a) {
+    float *D = a.D + (long long)blockIdx.z * a.zstride;
+#pragma unroll 1
+    for (int cc = 0; cc < BN; cc += 32) {
+        float v[32];
+        tmem_ld32(tbase + cc, v);
+        if (row < R) {
+            float *dst = D + (long long)row * a.ldd + col0 + cc;
+            if (col0 + cc + 32 <= Cn && (a.ldd % 4) == 0) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4)
+                    *reinterpret_cast<float4 *>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (col0 + cc + j < Cn) dst[j] = v[j];
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ float warp_sum_tc(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+template <int BN>
+__device__ __forceinline__ void epi_scan(uint32_t tbase, int row, int col0, const TcEpiArgs &a) {
+    const LifConst &c = a.c;
+    const int Mp = c.Mp;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    ScanState st;
+    scan_reset(st, c.M);
+#pragma unroll 1
+    for (int cc = 0; cc < BN; cc += 32) {
+        float v[32];
+        tmem_ld32(tbase + cc, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const int col = col0 + cc + j;
+            const int m = col & (Mp - 1);
+            if (m == 0) scan_reset(st, c.M);
+            if (m < c.M) scan_step(c, st, v[j], m);
+            if (m == Mp - 1) {
+                const int b = col / Mp;
+                if (row < a.N && b < a.B) {
+                    long long o = (long long)b * a.N + row;
+                    bool fired = st.q < c.M;
+                    float t = fired ? c.T0 + (float)st.q * c.dt + st.s : INFINITY;
+                    a.t_out[o] = t;
+                    a.q[o] = st.q;
+                    a.s[o] = st.s;
+                    a.vdot[o] = st.vdot;
+                    if (fired) {
+                        float pv, pg;
+                        penalty_T(c, t, pv, pg);
+                        acc[0] += pv;
+                        acc[3] += 1.f;
+                    } else {
+                        if (a.rowsum) acc[1] += -c.g_q * c.norm * a.rowsum[row];
+                        acc[2] += 1.f;
+                    }
+                }
+            }
+        }
+    }
+    if (a.penalty) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float s = warp_sum_tc(acc[k]);
+            if ((threadIdx.x & 31) == 0 && s != 0.f) atomicAdd(&a.penalty[k], s);
+        }
+    }
+}
+
+template <int BN>
+__device__ __forceinline__ void epi_gradt(uint32_t tbase, int row, int col0, const TcEpiArgs &a) {
+    const LifConst &c = a.c;
+    const int Mp = c.Mp;
+    BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+    float g = 0.f;
+#pragma unroll 1
+    for (int cc = 0; cc < BN; cc += 32) {
+        float v[32];
+        tmem_ld32(tbase + cc, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const int col = col0 + cc + j;
+            const int m = col & (Mp - 1);
+            const int b = col / Mp;
+            if (m == 0) {
+                g = 0.f;
+                w.k = -100;
+                if (row < a.N && b < a.B) {
+                    float x = a.t_in[(long long)b * a.N + row];
+                    if (isfinite(x)) w = bin_weights(c, x, true);
+                }
+            }
+            if (m < c.M) {
+                if (m == w.k) g += v[j] * w.dR;
+                if (m == w.k + 1) g += v[j] * w.dL;
+            }
+            if (m == Mp - 1 && row < a.N && b < a.B) a.g_t_in[(long long)b * a.N + row] = g;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// The kernel.
+// ---------------------------------------------------------------------------
+template <int NPASS, int BN, int EPI>
+__global__ void __launch_bounds__(128, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap mA_hi, const __grid_constant__ CUtensorMap mA_lo,
+              const __grid_constant__ CUtensorMap mB_hi, const __grid_constant__ CUtensorMap mB_lo, int R, int Cn,
+              int ktiles, int kt_per_split, TcEpiArgs args) {
+    using C = Cfg<NPASS, BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + C::STAGES * C::STAGE);
+    uint64_t *empty = full + C::STAGES;
+    uint64_t *accf = empty + C::STAGES;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(accf + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int col0 = blockIdx.x * BN, row0 = blockIdx.y * BM;
+    const int kt0 = blockIdx.z * kt_per_split;
+    int nkt = ktiles - kt0;
+    if (nkt > kt_per_split) nkt = kt_per_split;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(accf, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 0) tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0 && nkt > 0) {
+            // TMA producer
+            for (int i = 0; i < nkt; ++i) {
+                const int s = i % C::STAGES;
+                const uint32_t ph = (uint32_t)(i / C::STAGES) & 1u;
+                if (!mbar_wait(&empty[s], ph ^ 1u)) {
+                    set_status(STATUS_TIMEOUT);
+                    break;
+                }
+                mbar_expect_tx(&full[s], (uint32_t)C::STAGE);
+                const int kx = (kt0 + i) * BK;
+                const uint32_t st = smem_u32(smem + s * C::STAGE);
+                tma_load_2d(st, &mA_hi, &full[s], kx, row0);
+                if (NPASS == 3) tma_load_2d(st + C::A_BYTES, &mA_lo, &full[s], kx, row0);
+                tma_load_2d(st + C::NOP * C::A_BYTES, &mB_hi, &full[s], kx, col0);
+                if (NPASS == 3) tma_load_2d(st + C::NOP * C::A_BYTES + C::B_BYTES, &mB_lo, &full[s], kx, col0);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0 && nkt > 0) {
+            // MMA issuer
+            constexpr uint32_t idesc = idesc_bf16(BM, BN);
+            bool ok = true;
+            for (int i = 0; i < nkt; ++i) {
+                const int s = i % C::STAGES;
+                const uint32_t ph = (uint32_t)(i / C::STAGES) & 1u;
+                if (!mbar_wait(&full[s], ph)) {
+                    set_status(STATUS_TIMEOUT);
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
+                const uint32_t a_lo = a_hi + C::A_BYTES;
+                const uint32_t b_hi = a_hi + C::NOP * C::A_BYTES;
+                const uint32_t b_lo = b_hi + C::B_BYTES;
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk) {
+                    const uint64_t da = sdesc_sw128(a_hi + kk * 32);
+                    const uint64_t db = sdesc_sw128(b_hi + kk * 32);
+                    mma_bf16(tmem, da, db, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                    if (NPASS == 3) {
+                        mma_bf16(tmem, da, sdesc_sw128(b_lo + kk * 32), idesc, 1u);
+                        mma_bf16(tmem, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
+                    }
+                }
+                mma_commit(&empty[s]);
+            }
+            if (ok) mma_commit(accf);
+        }
+        __syncwarp();
+    }
+
+    // epilogue: all four warps, warp w owns TMEM lanes 32w .. 32w+31
+    const bool acc_ok = (nkt > 0) && mbar_wait(accf, 0);
+    tc_fence_after();
+    if (acc_ok) {
+        const uint32_t tbase = tmem + ((uint32_t)(warp * 32) << 16);
+        const int row = row0 + warp * 32 + lane;
+        if (EPI == (int)Epi::Store) epi_store<BN>(tbase, row, col0, R, Cn, args);
+        else if (EPI == (int)Epi::Scan) epi_scan<BN>(tbase, row, col0, args);
+        else epi_gradt<BN>(tbase, row, col0, args);
+    } else if (nkt > 0) {
+        set_status(STATUS_TIMEOUT);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, C::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------
+// Host side: tensor maps and launch.
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn get_encode() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// rows x cols bf16 matrix with row stride ld elements; box = box_rows x 64
+static bool make_map(CUtensorMap *m, const void *ptr, int rows, int cols, int ld, int box_rows) {
+    EncodeTiledFn enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t gstride[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int NPASS, int BN, int EPI>
+static cudaError_t launch_one(const CUtensorMap &a_hi, const CUtensorMap &a_lo, const CUtensorMap &b_hi,
+                              const CUtensorMap &b_lo, int R, int Cn, int K, int splits, const TcEpiArgs &args,
+                              cudaStream_t st) {
+    using C = Cfg<NPASS, BN>;
+    static bool attr_set = false;  // per instantiation
+    if (!attr_set) {
+        cudaError_t e =
+            cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int ktiles = (K + BK - 1) / BK;
+    const int per = (ktiles + splits - 1) / splits;
+    dim3 grid((Cn + BN - 1) / BN, (R + BM - 1) / BM, splits);
+    k_tc_gemm<NPASS, BN, EPI><<<grid, 128, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per, args);
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+
+cudaError_t launch_wait_selftest(unsigned long long limit_ns, cudaStream_t st) {
+    tc::k_wait_selftest<<<1, 32, 0, st>>>(limit_ns);
+    return cudaGetLastError();
+}
+
+int tc_gemm_splits_valid(int K, int splits) {
+    const int ktiles = (K + tc::BK - 1) / tc::BK;
+    const int per = (ktiles + splits - 1) / splits;
+    return per * (splits - 1) < ktiles;
+}
+
+cudaError_t launch_tc_gemm(const __nv_bfloat16 *A_hi, const __nv_bfloat16 *A_lo, int lda, const __nv_bfloat16 *B_hi,
+                           const __nv_bfloat16 *B_lo, int ldb, int R, int Cn, int K, int splits, OpKind op, Epi epi,
+                           const TcEpiArgs &args, cudaStream_t st) {
+    constexpr int BN = 128;
+    CUtensorMap a_hi, a_lo, b_hi, b_lo;
+    const bool three = (op == OpKind::BF16X3);
+    if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM) || !tc::make_map(&b_hi, B_hi, Cn, K, ldb, BN))
+        return cudaErrorInvalidValue;
+    if (three) {
+        if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM) || !tc::make_map(&b_lo, B_lo, Cn, K, ldb, BN))
+            return cudaErrorInvalidValue;
+    } else {
+        a_lo = a_hi;
+        b_lo = b_hi;
+    }
+    if (splits < 1) splits = 1;
+    if (three) {
+        switch (epi) {
+            case Epi::Store: return tc::launch_one<3, BN, 0>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+            case Epi::Scan: return tc::launch_one<3, BN, 1>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+            default: return tc::launch_one<3, BN, 2>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+        }
+    }
+    switch (epi) {
+        case Epi::Store: return tc::launch_one<1, BN, 0>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+        case Epi::Scan: return tc::launch_one<1, BN, 1>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+        default: return tc::launch_one<1, BN, 2>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+    }
+}
+
+}  // namespace dstd

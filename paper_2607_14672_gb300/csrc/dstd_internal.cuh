@@ -1,0 +1,246 @@
+// Internal declarations of libdstd: per-layer constants, LIF device math,
+// launch helpers. Not part of the public ABI (include/dstd.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/dstd.h"
+
+namespace dstd {
+
+// ---------------------------------------------------------------------------
+// Per-layer constants, computed on the host in double and rounded once.
+//
+// With rates av = 1/tau_m, aI = 1/tau_s (0 for an infinite constant) and
+// lam = aI - av, the spike kernel of Tab. kernel is, for every row,
+//     K(s) = e^{-av s} phi(s),  phi(s) = (1 - e^{-lam s}) / lam  (= s if lam = 0),
+// the response of v to a unit impulse in I. The DSTD kernel of
+// Tab. DSTD_kernels becomes, with r = t - T_k in [0, dt) for a spike in bin k,
+//     weight at T_k     : e^{av r} phi(dt - r) / phi(dt)        (t >= 0 column)
+//     weight at T_{k+1} : e^{aI (r - dt)} phi(r) / phi(dt)       (t < 0 column)
+// which is the table's expression rewritten with expm1 so that no difference
+// of nearly equal exponentials is formed.
+// ---------------------------------------------------------------------------
+struct LifConst {
+    float av, aI, lam;     // rates; lam = aI - av
+    int lam_zero;          // lam == 0 exactly (tau_m == tau_s, incl. both inf)
+    float T0, dt, inv_dt;  // T_0 = t_first - t_offset, step
+    float rv, rI, KD;      // e^{-av dt}, e^{-aI dt}, K(dt)
+    float inv_phi_dt;      // 1 / phi(dt)
+    float vth;
+    int M, Mp;             // steps, padded bin axis of the internal layouts
+    float vdot_floor;      // lower bound on dv^/dt at a spike (1e-6 v_th / dt)
+    float t_head, t_tail, g_head, g_tail, g_q, norm;
+};
+
+LifConst make_const(const dstd_params &p, int Mp);
+int padded_M(int M);       // next power of two >= max(M, 8)
+
+__device__ __forceinline__ float phi_f(const LifConst &c, float x) {
+    return c.lam_zero ? x : -expm1f(-c.lam * x) / c.lam;
+}
+// inverse of phi: the s with phi(s) = y (needs 1 - lam y > 0)
+__device__ __forceinline__ float phi_inv_f(const LifConst &c, float y) {
+    return c.lam_zero ? y : -log1pf(-c.lam * y) / c.lam;
+}
+// K(s) = e^{-av s} phi(s), s >= 0
+__device__ __forceinline__ float kernel_K(const LifConst &c, float s) {
+    return __expf(-c.av * s) * phi_f(c, s);
+}
+
+// DSTD grid weights of one finite spike t: bin k (= floor((t - T0)/dt)), the
+// weights wR at T_k and wL at T_{k+1}, and optionally their t-derivatives.
+struct BinW {
+    int k;
+    float wR, wL, dR, dL;
+};
+__device__ __forceinline__ BinW bin_weights(const LifConst &c, float t, bool deriv) {
+    BinW b;
+    float u = (t - c.T0) * c.inv_dt;
+    float kf = floorf(u);
+    b.k = (int)fmaxf(fminf(kf, 1e9f), -1e9f);
+    float r = t - (c.T0 + kf * c.dt);
+    r = fminf(fmaxf(r, 0.0f), c.dt);
+    float pR = phi_f(c, c.dt - r), pL = phi_f(c, r);
+    float eR = expf(c.av * r), eL = expf(c.aI * (r - c.dt));
+    b.wR = eR * pR * c.inv_phi_dt;
+    b.wL = eL * pL * c.inv_phi_dt;
+    if (deriv) {
+        // d/dr of the two columns: phi'(x) = e^{-lam x}
+        float dpR = c.lam_zero ? 1.0f : expf(-c.lam * (c.dt - r));
+        float dpL = c.lam_zero ? 1.0f : expf(-c.lam * r);
+        b.dR = eR * (c.av * pR - dpR) * c.inv_phi_dt;
+        b.dL = eL * (c.aI * pL + dpL) * c.inv_phi_dt;
+    } else {
+        b.dR = b.dL = 0.0f;
+    }
+    return b;
+}
+
+// ---------------------------------------------------------------------------
+// Scan over the M intervals of one neuron (Tab. timing_DSTD via state).
+//
+// The prefix sums a_iq, b_iq of Tab. timing_DSTD are carried as the exact
+// state (v, I) at T_q: at each grid point I jumps by w^_q, and over one step
+// (v, I) <- (rv v + KD I, rI I). On interval q the potential is
+//     v^(s) = e^{-av s} (v_q + phi(s) I_q),  s = t - T_q in [0, dt),
+// with at most one interior extremum. The first interval whose maximum
+// reaches v_th holds the spike; its root is found by safeguarded Newton.
+// ---------------------------------------------------------------------------
+struct ScanState {
+    float v, I;
+    int q;       // M while silent
+    float s, vdot;
+};
+
+__device__ __forceinline__ void scan_reset(ScanState &st, int M) {
+    st.v = 0.f; st.I = 0.f; st.q = M; st.s = 0.f; st.vdot = 0.f;
+}
+
+__device__ __forceinline__ float vhat_at(const LifConst &c, float v0, float I0, float s) {
+    return __expf(-c.av * s) * (v0 + phi_f(c, s) * I0);
+}
+
+// first root of v^(s) = v_th on [0, hi] given v^(0) < v_th <= v^(hi)
+__device__ __forceinline__ float interval_root(const LifConst &c, float v0, float I0, float hi) {
+    if (c.av == 0.0f) {
+        // v^ = v0 + phi(s) I0 is monotone here: invert phi in closed form
+        float s = phi_inv_f(c, (c.vth - v0) / I0);
+        return fminf(fmaxf(s, 0.0f), hi);
+    }
+    float lo = 0.0f;
+    float s = 0.5f * hi;
+    for (int it = 0; it < 48; ++it) {
+        float e = __expf(-c.av * s);
+        float f = e * (v0 + phi_f(c, s) * I0) - c.vth;
+        if (f >= 0.0f) hi = s; else lo = s;
+        float df = -c.av * (f + c.vth) + I0 * __expf(-c.aI * s);
+        float sn = s - f / df;
+        if (!(df > 0.0f) || !(sn > lo) || !(sn < hi)) sn = 0.5f * (lo + hi);
+        if (fabsf(sn - s) <= 1e-7f * c.dt || hi - lo <= 1e-7f * c.dt) { s = sn; break; }
+        s = sn;
+    }
+    return fminf(fmaxf(s, 0.0f), hi);
+}
+
+// Consume w^_m for interval m (m = 0..M-1, in order).
+__device__ __forceinline__ void scan_step(const LifConst &c, ScanState &st, float w, int m) {
+    if (st.q < c.M) return;
+    float v0 = st.v;
+    float I0 = st.I + w;
+    float ve = c.rv * v0 + c.KD * I0;
+    float s = -1.0f;
+    if (v0 >= c.vth) {
+        s = 0.0f;
+    } else if (ve >= c.vth) {
+        s = interval_root(c, v0, I0, c.dt);
+    } else if (c.av > 0.0f && c.aI > 0.0f && I0 > 0.0f) {
+        // interior maximum: dv^/ds > 0 at s = 0 and < 0 at s = dt
+        float d0 = -c.av * v0 + I0;
+        float dE = -c.av * ve + c.rI * I0;
+        if (d0 > 0.0f && dE < 0.0f) {
+            // e^{-lam s*} = 1 + lam y with y = (av v0 - I0)/(I0 aI)
+            float y = (c.av * v0 - I0) / (I0 * c.aI);
+            float sp = c.lam_zero ? -y : -log1pf(c.lam * y) / c.lam;
+            sp = fminf(fmaxf(sp, 0.0f), c.dt);
+            if (vhat_at(c, v0, I0, sp) >= c.vth) s = interval_root(c, v0, I0, sp);
+        }
+    }
+    if (s >= 0.0f) {
+        st.q = m;
+        st.s = s;
+        float Ic = I0 * __expf(-c.aI * s);
+        st.vdot = fmaxf(-c.av * c.vth + Ic, c.vdot_floor);
+    }
+    st.v = ve;
+    st.I = c.rI * I0;
+}
+
+// Temporal penalty of one firing neuron (Eq. temporal_penalty) and dT/dt,
+// both times norm.
+__device__ __forceinline__ void penalty_T(const LifConst &c, float t, float &val, float &grad) {
+    val = 0.f; grad = 0.f;
+    if (t < c.t_head) { float d = t - c.t_head; val += c.g_head * d * d; grad += 2.f * c.g_head * d; }
+    if (t > c.t_tail) { float d = t - c.t_tail; val += c.g_tail * d * d; grad += 2.f * c.g_tail * d; }
+    val *= c.norm; grad *= c.norm;
+}
+
+// ---------------------------------------------------------------------------
+// Device status word (bounded waits that expire set it); it lives in the
+// tensor-core translation unit, the only device code that waits.
+// ---------------------------------------------------------------------------
+constexpr unsigned int STATUS_TIMEOUT = 1u;
+cudaError_t status_read(unsigned int *out, int clear);
+cudaError_t launch_wait_selftest(unsigned long long limit_ns, cudaStream_t st);
+
+// ---------------------------------------------------------------------------
+// Kernel launch entry points (host functions that launch on a stream).
+// Layouts: "internal" bin axis padded to Mp (power of two), rows of 16-bit
+// operands padded to a multiple of 8 elements (TMA needs 16-byte strides).
+// ---------------------------------------------------------------------------
+enum class OpKind { F32 = 0, BF16X3 = 1, BF16 = 2 };
+
+inline int pad8(int x) { return (x + 7) & ~7; }
+
+// W fp32 [R, C] -> hi/lo bf16 [R, ldo] (and optional transpose [C, ldt]),
+// fp32 copy (F32 path), row sums [R].
+cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bfloat16 *hi, __nv_bfloat16 *lo,
+                                int ldo, __nv_bfloat16 *hiT, __nv_bfloat16 *loT, int ldt, float *f32T,
+                                int ldf, float *rowsum, cudaStream_t st);
+// t [B, N] -> grid weights in the layout chosen by `transposed`:
+//  !transposed: [B*Mp, ldk] (row (b,m), column j)    (contraction operand)
+//   transposed: [N, ldk'] with ldk' >= B*Mp (row j, column (b,m))
+// as bf16 hi/lo (BF16X3), bf16 hi (BF16) or fp32 (F32). Pad entries are 0.
+cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKind op, bool transposed,
+                           void *hi, void *lo, int ld, cudaStream_t st);
+// public-layout binning: s, ds [B, M, N] fp32
+cudaError_t launch_binning_public(const float *t, int B, int N, const LifConst &c, float *s, float *ds,
+                                  cudaStream_t st);
+// scan/solve from w^ with element (b, i, m) at what[b*sb + i*si + m]
+cudaError_t launch_scan_solve(const float *what, long long sb, long long si, int B, int N, const LifConst &c,
+                              const float *rowsum, float *t_out, int *q, float *s, float *vdot, float *penalty,
+                              cudaStream_t st);
+// dw^ from saved state; writes [B*Mp, ldn] (row (b,m), col i) and [N, ldbm]
+// (row i, col (b,m)) in the operand format; silent counts per neuron.
+cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
+                         int B, int N, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda,
+                         void *b_hi, void *b_lo, int ldb, float *silent_count, cudaStream_t st);
+// g_t_in from dS stored as D[j, (b,m)] (row stride ldd)
+cudaError_t launch_gt_from_ds(const float *D, long long ldd, const float *t_in, int B, int N, const LifConst &c,
+                              float *g_t_in, cudaStream_t st);
+// g_W[i, j] = sum_z part[z][i, j] - g_q*norm*count[i]
+cudaError_t launch_dw_reduce(const float *part, int splits, long long zstride, int ldp, int R, int C,
+                             const float *count, float qcoef, float *g_W, cudaStream_t st);
+// copy internal w^ D[i, (b, m)] (ld) -> public [B, N, M]
+cudaError_t launch_what_to_public(const float *D, long long ld, int B, int N, int M, int Mp, float *out,
+                                  cudaStream_t st);
+
+// D = A B^T, fp32 CUDA cores. A [R, K] (lda), B [Cn, K] (ldb), D [R, Cn] (ldd);
+// split-K over `splits` writes D + z*zstride.
+cudaError_t launch_sgemm_tn(const float *A, int lda, const float *Bm, int ldb, float *D, int ldd, int R, int Cn,
+                            int K, int splits, long long zstride, cudaStream_t st);
+
+// tcgen05 GEMM D = A B^T on bf16 operands (hi/lo for BF16X3), fp32 TMEM
+// accumulation, with a fused epilogue.
+enum class Epi { Store = 0, Scan = 1, GradT = 2 };
+struct TcEpiArgs {
+    // Store
+    float *D; long long ldd; long long zstride;
+    // Scan (rows = neurons i, columns = (b, m))
+    LifConst c; int B; int N; const float *rowsum; float *t_out; int *q; float *s; float *vdot; float *penalty;
+    // GradT (rows = inputs j, columns = (b, m))
+    const float *t_in; float *g_t_in;
+};
+cudaError_t launch_tc_gemm(const __nv_bfloat16 *A_hi, const __nv_bfloat16 *A_lo, int lda,
+                           const __nv_bfloat16 *B_hi, const __nv_bfloat16 *B_lo, int ldb, int R, int Cn, int K,
+                           int splits, OpKind op, Epi epi, const TcEpiArgs &args, cudaStream_t st);
+
+cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
+                           float *loss, float *g, cudaStream_t st);
+cudaError_t launch_sum_t(const float *t, long long n, float *loss, float *g, cudaStream_t st);
+cudaError_t launch_adamw(float *w, const float *g, float *m, float *v, long long n, float lr, float b1, float b2,
+                         float eps, float wd, int step, cudaStream_t st);
+
+}  // namespace dstd

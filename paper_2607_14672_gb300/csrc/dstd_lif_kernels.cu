@@ -1,0 +1,513 @@
+// Memory-bound kernels of the DSTD layer: weight preparation, binning (the
+// prologue of Eq. DSTD), the scan/solve/select of Tab. timing_DSTD on a
+// materialised w^, the backward's dw^ generation and input-time gradient,
+// split-K reduction, losses and AdamW.
+#include "dstd_internal.cuh"
+
+#include <math.h>
+
+namespace dstd {
+
+int padded_M(int M) {
+    int p = 8;
+    while (p < M) p <<= 1;
+    return p;
+}
+
+LifConst make_const(const dstd_params &p, int Mp) {
+    LifConst c{};
+    const double tv = p.tau_m, ti = p.tau_s;
+    const double av = isinf(tv) ? 0.0 : 1.0 / tv;
+    const double aI = isinf(ti) ? 0.0 : 1.0 / ti;
+    const double lam = aI - av;
+    const double dt = ((double)p.t_end - (double)p.t_first) / p.M;
+    const double phi_dt = lam == 0.0 ? dt : -expm1(-lam * dt) / lam;
+    c.av = (float)av;
+    c.aI = (float)aI;
+    c.lam = (float)lam;
+    c.lam_zero = (lam == 0.0);
+    c.T0 = (float)((double)p.t_first - (double)p.t_offset);
+    c.dt = (float)dt;
+    c.inv_dt = (float)(1.0 / dt);
+    c.rv = (float)exp(-av * dt);
+    c.rI = (float)exp(-aI * dt);
+    c.KD = (float)(exp(-av * dt) * phi_dt);
+    c.inv_phi_dt = (float)(1.0 / phi_dt);
+    c.vth = p.v_th;
+    c.M = p.M;
+    c.Mp = Mp;
+    c.vdot_floor = (float)(1e-6 * p.v_th / dt);
+    c.t_head = p.t_head;
+    c.t_tail = p.t_tail;
+    c.g_head = p.gamma_head;
+    c.g_tail = p.gamma_tail;
+    c.g_q = p.gamma_q;
+    c.norm = p.penalty_norm;
+    return c;
+}
+
+static inline unsigned blocks_for(long long n, int threads) {
+    return (unsigned)((n + threads - 1) / threads);
+}
+
+__device__ __forceinline__ void split_bf16(float x, __nv_bfloat16 &hi, __nv_bfloat16 &lo) {
+    hi = __float2bfloat16_rn(x);
+    lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+
+// ---------------------------------------------------------------------------
+// Weights: fp32 [R, C] -> bf16 hi/lo [R, ldo] (zero pad), transposed copies
+// [C, ldt] (bf16 hi/lo) or [C, ldf] (fp32), row sums.
+// ---------------------------------------------------------------------------
+__global__ void k_prep_weights(const float *__restrict__ W, int R, int C, int op, __nv_bfloat16 *hi,
+                               __nv_bfloat16 *lo, int ldo, __nv_bfloat16 *hiT, __nv_bfloat16 *loT, int ldt,
+                               float *f32T, int ldf, float *rowsum) {
+    __shared__ float tile[32][33];
+    const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
+    const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+    for (int yy = ty; yy < 32; yy += 8) {
+        int r = by + yy, cc = bx + tx;
+        float x = (r < R && cc < C) ? W[(long long)r * C + cc] : 0.0f;
+        tile[yy][tx] = x;
+        if (hi && r < R && cc < ldo) {
+            __nv_bfloat16 h, l;
+            split_bf16(x, h, l);
+            hi[(long long)r * ldo + cc] = h;
+            if (lo) lo[(long long)r * ldo + cc] = l;
+        }
+    }
+    __syncthreads();
+    // transposed writes: row = column index of W
+    for (int yy = ty; yy < 32; yy += 8) {
+        int cc = bx + yy, r = by + tx;
+        float x = tile[tx][yy];
+        if (hiT && cc < C && r < ldt) {
+            __nv_bfloat16 h, l;
+            split_bf16(x, h, l);
+            hiT[(long long)cc * ldt + r] = h;
+            if (loT) loT[(long long)cc * ldt + r] = l;
+        }
+        if (f32T && cc < C && r < ldf) f32T[(long long)cc * ldf + r] = x;
+    }
+    if (rowsum && ty == 0) {
+        // one warp per 32 rows of this tile column block: accumulate partial sums
+        int r = by + tx;
+        if (r < R) {
+            float sum = 0.0f;
+            for (int k = 0; k < 32; ++k) sum += tile[tx][k];
+            atomicAdd(&rowsum[r], sum);
+        }
+    }
+    (void)op;
+}
+
+cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bfloat16 *hi, __nv_bfloat16 *lo,
+                                int ldo, __nv_bfloat16 *hiT, __nv_bfloat16 *loT, int ldt, float *f32T, int ldf,
+                                float *rowsum, cudaStream_t st) {
+    if (rowsum) {
+        cudaError_t e = cudaMemsetAsync(rowsum, 0, sizeof(float) * R, st);
+        if (e != cudaSuccess) return e;
+    }
+    int cmax = C > ldo ? C : ldo;
+    int rmax = R > ldt ? R : ldt;
+    if (ldf > rmax) rmax = ldf;
+    dim3 grid((cmax + 31) / 32, (rmax + 31) / 32);
+    k_prep_weights<<<grid, dim3(32, 8), 0, st>>>(W, R, C, (int)op, hi, lo, ldo, hiT, loT, ldt, f32T, ldf, rowsum);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Binning (Eq. DSTD_kernel): one thread per (sample, pair of inputs) writes
+// the Mp rows of its two columns; rows m >= M and padding columns are zero.
+// ---------------------------------------------------------------------------
+template <int OP>
+__global__ void k_binning_rows(const float *__restrict__ t, int B, int N, LifConst c, void *hi, void *lo,
+                               int ld) {
+    const int b = blockIdx.y;
+    const int j0 = 2 * (blockIdx.x * blockDim.x + threadIdx.x);
+    if (j0 >= ld) return;
+    BinW w0{-100, 0.f, 0.f, 0.f, 0.f}, w1{-100, 0.f, 0.f, 0.f, 0.f};
+    if (j0 < N) {
+        float x = t[(long long)b * N + j0];
+        if (isfinite(x)) w0 = bin_weights(c, x, false);
+    }
+    if (j0 + 1 < N) {
+        float x = t[(long long)b * N + j0 + 1];
+        if (isfinite(x)) w1 = bin_weights(c, x, false);
+    }
+    for (int m = 0; m < c.Mp; ++m) {
+        float v0 = 0.f, v1 = 0.f;
+        if (m < c.M) {
+            v0 = (m == w0.k) ? w0.wR : ((m == w0.k + 1) ? w0.wL : 0.f);
+            v1 = (m == w1.k) ? w1.wR : ((m == w1.k + 1) ? w1.wL : 0.f);
+        }
+        long long off = ((long long)b * c.Mp + m) * ld + j0;
+        if (OP == 0) {
+            *reinterpret_cast<float2 *>((float *)hi + off) = make_float2(v0, v1);
+        } else {
+            __nv_bfloat16 h0, l0, h1, l1;
+            split_bf16(v0, h0, l0);
+            split_bf16(v1, h1, l1);
+            *reinterpret_cast<__nv_bfloat162 *>((__nv_bfloat16 *)hi + off) = __halves2bfloat162(h0, h1);
+            if (OP == 1) *reinterpret_cast<__nv_bfloat162 *>((__nv_bfloat16 *)lo + off) = __halves2bfloat162(l0, l1);
+        }
+    }
+}
+
+// transposed: row j, columns (b, m); one thread per (j, b) writes Mp
+// contiguous values with 16-byte stores.
+template <int OP>
+__global__ void k_binning_cols(const float *__restrict__ t, int B, int N, LifConst c, void *hi, void *lo,
+                               int ld) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= B) return;
+    for (int j = blockIdx.y; j < N; j += gridDim.y) {
+        BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+        float x = t[(long long)b * N + j];
+        if (isfinite(x)) w = bin_weights(c, x, false);
+        const long long base = (long long)j * ld + (long long)b * c.Mp;
+        for (int m0 = 0; m0 < c.Mp; m0 += 8) {
+            float v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                int m = m0 + u;
+                v[u] = (m < c.M) ? ((m == w.k) ? w.wR : ((m == w.k + 1) ? w.wL : 0.f)) : 0.f;
+            }
+            if (OP == 0) {
+                float4 *p = reinterpret_cast<float4 *>((float *)hi + base + m0);
+                p[0] = make_float4(v[0], v[1], v[2], v[3]);
+                p[1] = make_float4(v[4], v[5], v[6], v[7]);
+            } else {
+                __align__(16) __nv_bfloat16 h[8], l[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) split_bf16(v[u], h[u], l[u]);
+                *reinterpret_cast<uint4 *>((__nv_bfloat16 *)hi + base + m0) = *reinterpret_cast<uint4 *>(h);
+                if (OP == 1)
+                    *reinterpret_cast<uint4 *>((__nv_bfloat16 *)lo + base + m0) = *reinterpret_cast<uint4 *>(l);
+            }
+        }
+    }
+}
+
+cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKind op, bool transposed, void *hi,
+                           void *lo, int ld, cudaStream_t st) {
+    if (!transposed) {
+        int pairs = (ld + 1) / 2;
+        dim3 grid(blocks_for(pairs, 128), B);
+        if (op == OpKind::F32) k_binning_rows<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+        else if (op == OpKind::BF16X3) k_binning_rows<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+        else k_binning_rows<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+    } else {
+        dim3 grid(blocks_for(B, 128), N < 65535 ? N : 65535);
+        if (op == OpKind::F32) k_binning_cols<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+        else if (op == OpKind::BF16X3) k_binning_cols<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+        else k_binning_cols<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+    }
+    return cudaGetLastError();
+}
+
+__global__ void k_binning_public(const float *__restrict__ t, int B, int N, LifConst c, float *s, float *ds) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)B * N) return;
+    int b = (int)(idx / N), j = (int)(idx % N);
+    BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+    float x = t[idx];
+    if (isfinite(x)) w = bin_weights(c, x, ds != nullptr);
+    for (int m = 0; m < c.M; ++m) {
+        long long o = ((long long)b * c.M + m) * N + j;
+        s[o] = (m == w.k) ? w.wR : ((m == w.k + 1) ? w.wL : 0.f);
+        if (ds) ds[o] = (m == w.k) ? w.dR : ((m == w.k + 1) ? w.dL : 0.f);
+    }
+}
+
+cudaError_t launch_binning_public(const float *t, int B, int N, const LifConst &c, float *s, float *ds,
+                                  cudaStream_t st) {
+    long long n = (long long)B * N;
+    k_binning_public<<<blocks_for(n, 256), 256, 0, st>>>(t, B, N, c, s, ds);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Scan/solve/select from a materialised w^ (one thread per neuron), with the
+// temporal penalty and dead-neuron sums (warp-reduced, one atomic per warp).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__device__ __forceinline__ void finish_neuron(const LifConst &c, const ScanState &st, int b, int i, int N,
+                                              const float *rowsum, float *t_out, int *q, float *s, float *vdot,
+                                              float acc[4]) {
+    long long o = (long long)b * N + i;
+    bool fired = st.q < c.M;
+    float t = fired ? c.T0 + (float)st.q * c.dt + st.s : INFINITY;
+    t_out[o] = t;
+    if (q) q[o] = st.q;
+    if (s) s[o] = st.s;
+    if (vdot) vdot[o] = st.vdot;
+    if (fired) {
+        float pv, pg;
+        penalty_T(c, t, pv, pg);
+        acc[0] += pv;
+        acc[3] += 1.0f;
+    } else {
+        if (rowsum) acc[1] += -c.g_q * c.norm * rowsum[i];
+        acc[2] += 1.0f;
+    }
+}
+
+__device__ __forceinline__ void flush_penalty(float acc[4], float *penalty) {
+    if (!penalty) return;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        float v = warp_sum(acc[k]);
+        if ((threadIdx.x & 31) == 0 && v != 0.0f) atomicAdd(&penalty[k], v);
+    }
+}
+
+__global__ void k_scan_solve(const float *__restrict__ what, long long sb, long long si, int B, int N, LifConst c,
+                             const float *__restrict__ rowsum, float *t_out, int *q, float *s, float *vdot,
+                             float *penalty) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (idx < (long long)B * N) {
+        int b = (int)(idx / N), i = (int)(idx % N);
+        const float *w = what + b * sb + i * si;
+        ScanState st;
+        scan_reset(st, c.M);
+        for (int m = 0; m < c.M; ++m) {
+            scan_step(c, st, w[m], m);
+            if (st.q < c.M) break;
+        }
+        finish_neuron(c, st, b, i, N, rowsum, t_out, q, s, vdot, acc);
+    }
+    flush_penalty(acc, penalty);
+}
+
+cudaError_t launch_scan_solve(const float *what, long long sb, long long si, int B, int N, const LifConst &c,
+                              const float *rowsum, float *t_out, int *q, float *s, float *vdot, float *penalty,
+                              cudaStream_t st) {
+    long long n = (long long)B * N;
+    k_scan_solve<<<blocks_for(n, 256), 256, 0, st>>>(what, sb, si, B, N, c, rowsum, t_out, q, s, vdot, penalty);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Backward, step 1: dC/dw^_im = -g_i K(t_i - T_m) / v^'(t_i) for m <= q_i
+// (implicit function theorem on v^(t_i) = v_th), g_i = upstream + dT/dt_i.
+// Writes it as the K-major operand of both backward contractions:
+//   A layout [N, lda]:    row i, columns (b, m)     (dW = dw^T . s)
+//   B layout [B*Mp, ldb]: row (b, m), column i      (dS = dw^ . W)
+// ---------------------------------------------------------------------------
+template <int OP>
+__global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__ qv, const float *__restrict__ sv,
+                        const float *__restrict__ vd, const float *__restrict__ g_up, int B, int N, LifConst c,
+                        void *a_hi, void *a_lo, int lda, void *b_hi, void *b_lo, int ldb, float *count) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)B * N) return;
+    const int b = (int)(idx / N), i = (int)(idx % N);
+    const int q = qv[idx];
+    float coef = 0.f, s0 = 0.f;
+    if (q < c.M) {
+        float pv, pg;
+        penalty_T(c, t_out[idx], pv, pg);
+        float g = (g_up ? g_up[idx] : 0.f) + pg;
+        coef = -g / vd[idx];
+        s0 = sv[idx];
+    } else if (count) {
+        atomicAdd(&count[i], 1.0f);
+    }
+    const long long abase = (long long)i * lda + (long long)b * c.Mp;
+    for (int m0 = 0; m0 < c.Mp; m0 += 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            int m = m0 + u;
+            v[u] = (q < c.M && m <= q) ? coef * kernel_K(c, s0 + (float)(q - m) * c.dt) : 0.f;
+        }
+        if (OP == 0) {
+            float4 *p = reinterpret_cast<float4 *>((float *)a_hi + abase + m0);
+            p[0] = make_float4(v[0], v[1], v[2], v[3]);
+            p[1] = make_float4(v[4], v[5], v[6], v[7]);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) ((float *)b_hi)[((long long)b * c.Mp + m0 + u) * ldb + i] = v[u];
+        } else {
+            __align__(16) __nv_bfloat16 h[8], l[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) split_bf16(v[u], h[u], l[u]);
+            *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + abase + m0) = *reinterpret_cast<uint4 *>(h);
+            if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + abase + m0) = *reinterpret_cast<uint4 *>(l);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                long long o = ((long long)b * c.Mp + m0 + u) * ldb + i;
+                ((__nv_bfloat16 *)b_hi)[o] = h[u];
+                if (OP == 1) ((__nv_bfloat16 *)b_lo)[o] = l[u];
+            }
+        }
+    }
+}
+
+cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
+                         int B, int N, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda, void *b_hi,
+                         void *b_lo, int ldb, float *silent_count, cudaStream_t st) {
+    if (silent_count) {
+        cudaError_t e = cudaMemsetAsync(silent_count, 0, sizeof(float) * N, st);
+        if (e != cudaSuccess) return e;
+    }
+    long long n = (long long)B * N;
+    unsigned g = blocks_for(n, 256);
+    if (op == OpKind::F32)
+        k_dwhat<0><<<g, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, b_hi, b_lo, ldb, silent_count);
+    else if (op == OpKind::BF16X3)
+        k_dwhat<1><<<g, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, b_hi, b_lo, ldb, silent_count);
+    else
+        k_dwhat<2><<<g, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, b_hi, b_lo, ldb, silent_count);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Backward, input times: g_t_j = sum_{m in {k, k+1}} dS[j, (b, m)] ds_jm/dt_j.
+// ---------------------------------------------------------------------------
+__global__ void k_gt_from_ds(const float *__restrict__ D, long long ldd, const float *__restrict__ t_in, int B,
+                             int N, LifConst c, float *g_t_in) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)B * N) return;
+    const int b = (int)(idx / N), j = (int)(idx % N);
+    float x = t_in[idx];
+    float g = 0.f;
+    if (isfinite(x)) {
+        BinW w = bin_weights(c, x, true);
+        const float *row = D + (long long)j * ldd + (long long)b * c.Mp;
+        if (w.k >= 0 && w.k < c.M) g += row[w.k] * w.dR;
+        if (w.k + 1 >= 0 && w.k + 1 < c.M) g += row[w.k + 1] * w.dL;
+    }
+    g_t_in[idx] = g;
+}
+
+cudaError_t launch_gt_from_ds(const float *D, long long ldd, const float *t_in, int B, int N, const LifConst &c,
+                              float *g_t_in, cudaStream_t st) {
+    long long n = (long long)B * N;
+    k_gt_from_ds<<<blocks_for(n, 256), 256, 0, st>>>(D, ldd, t_in, B, N, c, g_t_in);
+    return cudaGetLastError();
+}
+
+__global__ void k_dw_reduce(const float *__restrict__ part, int splits, long long zstride, int ldp, int R, int C,
+                            const float *__restrict__ count, float qcoef, float *g_W) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)R * C) return;
+    int i = (int)(idx / C), j = (int)(idx % C);
+    float s = 0.f;
+    for (int z = 0; z < splits; ++z) s += part[z * zstride + (long long)i * ldp + j];
+    if (count) s += qcoef * count[i];
+    g_W[idx] = s;
+}
+
+cudaError_t launch_dw_reduce(const float *part, int splits, long long zstride, int ldp, int R, int C,
+                             const float *count, float qcoef, float *g_W, cudaStream_t st) {
+    long long n = (long long)R * C;
+    k_dw_reduce<<<blocks_for(n, 256), 256, 0, st>>>(part, splits, zstride, ldp, R, C, count, qcoef, g_W);
+    return cudaGetLastError();
+}
+
+__global__ void k_what_to_public(const float *__restrict__ D, long long ld, int B, int N, int M, int Mp,
+                                 float *out) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)B * N * M) return;
+    int m = (int)(idx % M);
+    long long r = idx / M;
+    int i = (int)(r % N), b = (int)(r / N);
+    out[idx] = D[(long long)i * ld + (long long)b * Mp + m];
+}
+
+cudaError_t launch_what_to_public(const float *D, long long ld, int B, int N, int M, int Mp, float *out,
+                                  cudaStream_t st) {
+    long long n = (long long)B * N * M;
+    k_what_to_public<<<blocks_for(n, 256), 256, 0, st>>>(D, ld, B, N, M, Mp, out);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Losses and optimizer.
+// ---------------------------------------------------------------------------
+__global__ void k_ce_loss(const float *__restrict__ t, const int32_t *__restrict__ lab, int B, int C, float tau_soft,
+                          float t_silent, float *loss, float *g) {
+    int b = blockIdx.x * blockDim.x + threadIdx.x;
+    float contrib = 0.f;
+    if (b < B) {
+        const float *tb = t + (long long)b * C;
+        float zmax = -INFINITY;
+        for (int k = 0; k < C; ++k) {
+            float x = isfinite(tb[k]) ? tb[k] : t_silent;
+            zmax = fmaxf(zmax, -x / tau_soft);
+        }
+        float den = 0.f;
+        for (int k = 0; k < C; ++k) {
+            float x = isfinite(tb[k]) ? tb[k] : t_silent;
+            den += expf(-x / tau_soft - zmax);
+        }
+        int y = lab[b];
+        for (int k = 0; k < C; ++k) {
+            bool fin = isfinite(tb[k]);
+            float x = fin ? tb[k] : t_silent;
+            float p = expf(-x / tau_soft - zmax) / den;
+            if (k == y) contrib = -(-x / tau_soft - zmax - logf(den));
+            float gg = -(p - (k == y ? 1.f : 0.f)) / tau_soft / (float)B;
+            g[(long long)b * C + k] = fin ? gg : 0.f;
+        }
+    }
+    float v = warp_sum(contrib / (float)B);
+    if ((threadIdx.x & 31) == 0 && v != 0.f) atomicAdd(loss, v);
+}
+
+cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
+                           float *loss, float *g, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(loss, 0, sizeof(float), st);
+    if (e != cudaSuccess) return e;
+    k_ce_loss<<<blocks_for(B, 128), 128, 0, st>>>(t, lab, B, C, tau_soft, t_silent, loss, g);
+    return cudaGetLastError();
+}
+
+__global__ void k_sum_t(const float *__restrict__ t, long long n, float *loss, float *g) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    float c = 0.f;
+    if (idx < n) {
+        float x = t[idx];
+        bool f = isfinite(x);
+        g[idx] = f ? 1.f : 0.f;
+        c = f ? x : 0.f;
+    }
+    float v = warp_sum(c);
+    if ((threadIdx.x & 31) == 0 && v != 0.f) atomicAdd(loss, v);
+}
+
+cudaError_t launch_sum_t(const float *t, long long n, float *loss, float *g, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(loss, 0, sizeof(float), st);
+    if (e != cudaSuccess) return e;
+    k_sum_t<<<blocks_for(n, 256), 256, 0, st>>>(t, n, loss, g);
+    return cudaGetLastError();
+}
+
+__global__ void k_adamw(float *w, const float *__restrict__ g, float *m, float *v, long long n, float lr, float b1,
+                        float b2, float eps, float wd, float bc1, float bc2) {
+    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= n) return;
+    float gi = g[idx];
+    float wi = w[idx] * (1.f - lr * wd);
+    float mi = b1 * m[idx] + (1.f - b1) * gi;
+    float vi = b2 * v[idx] + (1.f - b2) * gi * gi;
+    m[idx] = mi;
+    v[idx] = vi;
+    w[idx] = wi - lr * (mi / bc1) / (sqrtf(vi / bc2) + eps);
+}
+
+cudaError_t launch_adamw(float *w, const float *g, float *m, float *v, long long n, float lr, float b1, float b2,
+                         float eps, float wd, int step, cudaStream_t st) {
+    float bc1 = (float)(1.0 - pow((double)b1, step));
+    float bc2 = (float)(1.0 - pow((double)b2, step));
+    k_adamw<<<blocks_for(n, 256), 256, 0, st>>>(w, g, m, v, n, lr, b1, b2, eps, wd, bc1, bc2);
+    return cudaGetLastError();
+}
+
+}  // namespace dstd

@@ -1,0 +1,237 @@
+"""Thin Python binding of libdstd (include/dstd.h): argument marshalling only.
+
+Every function takes CUDA float32 torch tensors (int32 for labels, any dtype
+for opaque byte buffers), checks shapes and dtypes, and calls the C entry
+point of the same name on the given stream (default: torch's current
+stream). All arithmetic happens in the library's kernels; there is no
+fallback of any kind. A missing library raises at load time.
+"""
+
+import ctypes
+import os
+
+from .build import LIB_PATH
+
+MATH = {"f32": 0, "bf16x3": 1, "bf16": 2}
+
+ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "workspace too small",
+          -4: "CUDA call or kernel launch failed", -5: "a bounded device-side wait expired",
+          -6: "no usable sm_103 device"}
+
+EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning", "dstd_dense_what",
+           "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
+           "dstd_adamw", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
+           "dstd_timing_read", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout")
+
+
+class DstdError(RuntimeError):
+    def __init__(self, code, where):
+        super().__init__(f"{where}: {ERRORS.get(code, 'unknown error')} (code {code})")
+        self.code = code
+
+
+class Params(ctypes.Structure):
+    """dstd_params of include/dstd.h."""
+    _fields_ = [("tau_m", ctypes.c_float), ("tau_s", ctypes.c_float), ("v_th", ctypes.c_float),
+                ("t_first", ctypes.c_float), ("t_end", ctypes.c_float), ("M", ctypes.c_int32),
+                ("t_offset", ctypes.c_float), ("t_head", ctypes.c_float), ("t_tail", ctypes.c_float),
+                ("gamma_head", ctypes.c_float), ("gamma_tail", ctypes.c_float), ("gamma_q", ctypes.c_float),
+                ("penalty_norm", ctypes.c_float)]
+
+
+def params(layer, penalty_norm=0.0):
+    """dstd_params from a layer dict (see configs.py)."""
+    return Params(float(layer["tau_v"]), float(layer["tau_I"]), float(layer["v_th"]), float(layer["t_first"]),
+                  float(layer["t_end"]), int(layer["M"]), float(layer.get("t_offset", 0.0)),
+                  float(layer.get("t_head_l", 0.0)), float(layer.get("t_tail_l", 0.0)),
+                  float(layer.get("gamma_head", 0.0)), float(layer.get("gamma_tail", 0.0)),
+                  float(layer.get("gamma_q", 0.0)), float(penalty_norm))
+
+
+_LIB = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+_SZ = ctypes.c_size_t
+_I64 = ctypes.c_int64
+_PP = ctypes.POINTER(Params)
+
+
+def load(path=None):
+    """Load libdstd.so (built by ``build.build()``); raises if it is missing."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libdstd.so not found at {p}: build it first (python -m paper_2607_14672_gb300.build)")
+    lib = ctypes.CDLL(p)
+    sig = {
+        "dstd_dense_saved_bytes": (_SZ, [_I, _I]),
+        "dstd_dense_workspace_bytes": (_SZ, [_I, _I, _I, _PP, _I]),
+        "dstd_binning": (_I, [_P, _I, _I, _PP, _P, _P, _P]),
+        "dstd_dense_what": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _SZ, _P]),
+        "dstd_scan_solve": (_I, [_P, _I, _I, _PP, _P, _P, _P, _P, _P]),
+        "dstd_dense_fwd": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _P, _SZ, _P]),
+        "dstd_dense_bwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
+        "dstd_ce_loss": (_I, [_P, _P, _I, _I, _F, _F, _P, _P, _P]),
+        "dstd_sum_t_loss": (_I, [_P, _I64, _P, _P, _P]),
+        "dstd_adamw": (_I, [_P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I, _P]),
+        "dstd_device_status": (_I, [_I]),
+        "dstd_error_string": (ctypes.c_char_p, [_I]),
+        "dstd_version": (_I, []),
+        "dstd_timing_enable": (_I, [_I]),
+        "dstd_timing_read": (_I, [_I, ctypes.POINTER(_F), ctypes.POINTER(_I64)]),
+        "dstd_kernel_kind_count": (_I, []),
+        "dstd_kernel_kind_name": (ctypes.c_char_p, [_I]),
+        "dstd_selftest_wait_timeout": (_I, [ctypes.c_uint32, _P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _LIB = lib
+    return lib
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(stream):
+    if stream is not None:
+        return stream if isinstance(stream, int) else stream.cuda_stream
+    import torch
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _check(code, where):
+    if code != 0:
+        raise DstdError(code, where)
+
+
+def _f32(x, name, shape=None):
+    import torch
+    if x.dtype != torch.float32 or not x.is_cuda or not x.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA float32 tensor")
+    if shape is not None and tuple(x.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(x.shape)}, expected {tuple(shape)}")
+
+
+def version():
+    return load().dstd_version()
+
+
+def error_string(code):
+    return load().dstd_error_string(code).decode()
+
+
+def dense_saved_bytes(B, N_out):
+    return load().dstd_dense_saved_bytes(B, N_out)
+
+
+def dense_workspace_bytes(B, N_in, N_out, p, math_mode):
+    return load().dstd_dense_workspace_bytes(B, N_in, N_out, ctypes.byref(p), MATH[math_mode])
+
+
+def binning(t_in, p, s, ds=None, stream=None):
+    B, N = t_in.shape
+    _f32(t_in, "t_in")
+    _f32(s, "s", (B, p.M, N))
+    if ds is not None:
+        _f32(ds, "ds", (B, p.M, N))
+    _check(load().dstd_binning(_ptr(t_in), B, N, ctypes.byref(p), _ptr(s), _ptr(ds), _stream(stream)),
+           "dstd_binning")
+
+
+def dense_what(t_in, W, p, math_mode, what, workspace, stream=None):
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(what, "what", (B, N_out, p.M))
+    _check(load().dstd_dense_what(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), MATH[math_mode],
+                                  _ptr(what), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                  _stream(stream)), "dstd_dense_what")
+
+
+def scan_solve(what, p, w_rowsum, t_out, saved=None, penalty=None, stream=None):
+    B, N_out, M = what.shape
+    _f32(what, "what")
+    _f32(t_out, "t_out", (B, N_out))
+    _check(load().dstd_scan_solve(_ptr(what), B, N_out, ctypes.byref(p), _ptr(w_rowsum), _ptr(t_out), _ptr(saved),
+                                  _ptr(penalty), _stream(stream)), "dstd_scan_solve")
+
+
+def dense_fwd(t_in, W, p, math_mode, t_out, saved, penalty, workspace, stream=None):
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(t_out, "t_out", (B, N_out))
+    _check(load().dstd_dense_fwd(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), MATH[math_mode], _ptr(t_out),
+                                 _ptr(saved), _ptr(penalty), _ptr(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_dense_fwd")
+
+
+def dense_bwd(t_in, W, t_out, saved, g_t_out, p, math_mode, g_t_in, g_W, workspace, stream=None):
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(g_W, "g_W", (N_out, N_in))
+    if g_t_in is not None:
+        _f32(g_t_in, "g_t_in", (B, N_in))
+    _check(load().dstd_dense_bwd(_ptr(t_in), _ptr(W), _ptr(t_out), _ptr(saved), _ptr(g_t_out), B, N_in, N_out,
+                                 ctypes.byref(p), MATH[math_mode], _ptr(g_t_in), _ptr(g_W), _ptr(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_dense_bwd")
+
+
+def ce_loss(t_L, labels, tau_soft, t_silent, loss, g_t_L, stream=None):
+    B, C = t_L.shape
+    _f32(t_L, "t_L")
+    _check(load().dstd_ce_loss(_ptr(t_L), _ptr(labels), B, C, float(tau_soft), float(t_silent), _ptr(loss),
+                               _ptr(g_t_L), _stream(stream)), "dstd_ce_loss")
+
+
+def sum_t_loss(t, loss, g, stream=None):
+    _f32(t, "t")
+    _check(load().dstd_sum_t_loss(_ptr(t), t.numel(), _ptr(loss), _ptr(g), _stream(stream)), "dstd_sum_t_loss")
+
+
+def adamw(w, g, m, v, lr, beta1, beta2, eps, weight_decay, step, stream=None):
+    _f32(w, "w")
+    _check(load().dstd_adamw(_ptr(w), _ptr(g), _ptr(m), _ptr(v), w.numel(), float(lr), float(beta1), float(beta2),
+                             float(eps), float(weight_decay), int(step), _stream(stream)), "dstd_adamw")
+
+
+def device_status(clear=True):
+    """DSTD_OK (0) or DSTD_E_TIMEOUT after synchronising the device."""
+    return load().dstd_device_status(1 if clear else 0)
+
+
+
+def timing_enable(on=True):
+    """Turn per-kernel event timing on/off (clears the counters)."""
+    _check(load().dstd_timing_enable(1 if on else 0), "dstd_timing_enable")
+
+
+def timing_read():
+    """{kernel kind: (total ms, launches)} accumulated since timing_enable."""
+    lib = load()
+    out = {}
+    for k in range(lib.dstd_kernel_kind_count()):
+        ms = _F()
+        n = _I64()
+        _check(lib.dstd_timing_read(k, ctypes.byref(ms), ctypes.byref(n)), "dstd_timing_read")
+        out[lib.dstd_kernel_kind_name(k).decode()] = (ms.value, n.value)
+    return out
+
+
+def selftest_wait_timeout(timeout_us, stream=None):
+    """Launch the bounded-wait self-test (see include/dstd.h)."""
+    _check(load().dstd_selftest_wait_timeout(int(timeout_us), _stream(stream)), "dstd_selftest_wait_timeout")

@@ -1,0 +1,110 @@
+"""Multi-layer driver over the C-ABI: the Alg. 2 layer loop, the loss of
+Eq. cost_function and the reverse pass, with persistent device buffers.
+
+Every step of the hot path runs in libdstd's kernels; this module only owns
+the torch buffers, orders the C calls, and can capture a whole training step
+in a CUDA graph (buffers never move, so a captured step replays on new data
+copied into ``t_in``).
+"""
+
+import torch
+
+from . import dstd
+
+
+class DenseNet:
+    """A stack of dense DSTD layers (configs.py layer dicts) on one GPU."""
+
+    def __init__(self, cfg, math_mode="bf16x3", batch=None, device="cuda", with_adamw=False):
+        self.cfg = cfg
+        self.math = math_mode
+        self.B = int(batch or cfg["batch"])
+        self.layers = [dict(L) for L in cfg["layers"]]
+        self.loss_kind = cfg.get("loss", "sum_t")
+        dev = torch.device(device)
+        self.device = dev
+        B = self.B
+        self.W = [torch.tensor(L["W"], dtype=torch.float32, device=dev).contiguous() for L in self.layers]
+        self.sizes = [self.W[0].shape[1]] + [w.shape[0] for w in self.W]
+        self.p = [dstd.params(L, penalty_norm=1.0 / B) for L in self.layers]
+        self.t_in = torch.full((B, self.sizes[0]), float("inf"), dtype=torch.float32, device=dev)
+        self.t = [torch.empty((B, n), dtype=torch.float32, device=dev) for n in self.sizes[1:]]
+        self.g = [torch.zeros((B, n), dtype=torch.float32, device=dev) for n in self.sizes[1:]]
+        self.saved = [torch.empty(dstd.dense_saved_bytes(B, n), dtype=torch.uint8, device=dev)
+                      for n in self.sizes[1:]]
+        self.penalty = torch.zeros((len(self.W), 4), dtype=torch.float32, device=dev)
+        self.gW = [torch.empty_like(w) for w in self.W]
+        ws = max(dstd.dense_workspace_bytes(B, self.sizes[l], self.sizes[l + 1], self.p[l], math_mode)
+                 for l in range(len(self.W)))
+        if ws == 0:
+            raise ValueError("unsupported layer sizes or constants for the library")
+        self.workspace = torch.empty(ws, dtype=torch.uint8, device=dev)
+        self.loss = torch.zeros(1, dtype=torch.float32, device=dev)
+        self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.with_adamw = with_adamw
+        if with_adamw:
+            self.m = [torch.zeros_like(w) for w in self.W]
+            self.v = [torch.zeros_like(w) for w in self.W]
+            self.adam_step = 0
+
+    # -- inputs -----------------------------------------------------------
+    def set_offsets(self, offsets):
+        for p, L, o in zip(self.p, self.layers, offsets):
+            p.t_offset = float(o)
+            L["t_offset"] = float(o)
+
+    def set_inputs(self, t0, labels=None):
+        self.t_in.copy_(torch.as_tensor(t0, dtype=torch.float32), non_blocking=True)
+        if labels is not None:
+            self.labels.copy_(torch.as_tensor(labels, dtype=torch.int32), non_blocking=True)
+
+    # -- passes -------------------------------------------------------------
+    def layer_input(self, l):
+        return self.t_in if l == 0 else self.t[l - 1]
+
+    def forward(self, stream=None):
+        for l in range(len(self.W)):
+            dstd.dense_fwd(self.layer_input(l), self.W[l], self.p[l], self.math, self.t[l], self.saved[l],
+                           self.penalty[l], self.workspace, stream)
+
+    def loss_grad(self, stream=None):
+        if self.loss_kind == "ce":
+            dstd.ce_loss(self.t[-1], self.labels, self.cfg["tau_soft"], self.layers[-1]["t_end"], self.loss,
+                         self.g[-1], stream)
+        else:
+            dstd.sum_t_loss(self.t[-1], self.loss, self.g[-1], stream)
+
+    def backward(self, stream=None):
+        for l in range(len(self.W) - 1, -1, -1):
+            g_in = self.g[l - 1] if l > 0 else None
+            dstd.dense_bwd(self.layer_input(l), self.W[l], self.t[l], self.saved[l], self.g[l], self.p[l],
+                           self.math, g_in, self.gW[l], self.workspace, stream)
+
+    def optimizer(self, lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=1e-2, stream=None):
+        self.adam_step += 1
+        for w, g, m, v in zip(self.W, self.gW, self.m, self.v):
+            dstd.adamw(w, g, m, v, lr, betas[0], betas[1], eps, weight_decay, self.adam_step, stream)
+
+    def step(self, stream=None):
+        """One training step: forward, loss, backward (and AdamW if enabled)."""
+        self.forward(stream)
+        self.loss_grad(stream)
+        self.backward(stream)
+        if self.with_adamw:
+            self.optimizer(stream=stream)
+
+    def objective(self):
+        """Eq. cost_function on the last batch: loss + T + gamma_Q Q (device scalar)."""
+        return self.loss[0] + self.penalty[:, 0].sum() + self.penalty[:, 1].sum()
+
+    def launches_per_step(self):
+        """Kernels the library launches per ``step`` (memsets not counted)."""
+        tc = self.math != "f32"
+        L = len(self.W)
+        n = L * (3 if tc else 4)                  # fwd: prep + binning + gemm(+fused scan) [+ scan]
+        n += 1                                    # loss
+        n += L * 4                                # bwd: dw^ + binning^T + dW gemm + reduce
+        n += (L - 1) * (2 if tc else 3)           # bwd input times: prep W^T + dS gemm [+ gather]
+        if self.with_adamw:
+            n += L
+        return n

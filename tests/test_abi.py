@@ -1,0 +1,106 @@
+"""CPU checks of the C-ABI: the library builds for sm_103a, loads, exports every
+function include/dstd.h declares, and rejects bad arguments on the host
+before anything is launched (no GPU needed)."""
+
+import ctypes
+import math
+import os
+import re
+import shutil
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"),
+                                reason="nvcc not available")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_14672_gb300 import build, dstd
+    build.build()
+    return dstd.load()
+
+
+def declared_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(dstd_\w+)\s*\(", src))
+    return names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 13
+    for n in names:
+        assert hasattr(lib, n), n
+    from paper_2607_14672_gb300 import dstd
+    assert set(dstd.EXPORTS) == names
+
+
+def test_version_and_errors(lib):
+    from paper_2607_14672_gb300 import dstd
+    assert dstd.version() == 100
+    for code, msg in dstd.ERRORS.items():
+        assert dstd.error_string(code) == msg
+    assert dstd.error_string(-99) == "unknown error code"
+
+
+def _layer(M=32, **kw):
+    from paper_2607_14672_gb300 import dstd
+    L = dict(tau_v=0.5, tau_I=0.25, v_th=1.0, t_first=0.0, t_end=1.2, M=M, t_offset=0.0)
+    L.update(kw)
+    return dstd.params(L, 1.0 / 8)
+
+
+def test_size_queries(lib):
+    from paper_2607_14672_gb300 import dstd
+    p = _layer()
+    # q, s, vdot: 320 bytes each at 256-byte aligned offsets 0, 512, 1024
+    assert dstd.dense_saved_bytes(8, 10) == 2 * 512 + 8 * 10 * 4
+    for m in ("f32", "bf16x3", "bf16"):
+        assert dstd.dense_workspace_bytes(256, 784, 800, p, m) > 0
+    # bf16x3 carries two copies of each operand
+    assert dstd.dense_workspace_bytes(256, 784, 800, p, "bf16x3") > dstd.dense_workspace_bytes(256, 784, 800, p, "bf16")
+    # invalid constants -> 0
+    for bad in (dict(tau_v=-1.0), dict(tau_I=0.0), dict(v_th=0.0), dict(t_end=-1.0), dict(M=0),
+                dict(t_offset=0.5), dict(t_offset=-0.02), dict(tau_v=math.nan)):
+        assert dstd.dense_workspace_bytes(8, 16, 16, _layer(**bad), "f32") == 0, bad
+    # infinite time constants are valid
+    assert dstd.dense_workspace_bytes(8, 16, 16, _layer(tau_v=math.inf, tau_I=math.inf), "f32") > 0
+    # tensor-core modes take M <= 128; the fp32 mode up to 256; beyond that nothing
+    assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=200), "bf16x3") == 0
+    assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=200), "f32") > 0
+    assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=300), "f32") == 0
+    assert dstd.dense_workspace_bytes(0, 16, 16, p, "f32") == 0
+    assert dstd.dense_workspace_bytes(8, 0, 16, p, "f32") == 0
+
+
+def test_null_and_bad_arguments_rejected_on_host(lib):
+    from paper_2607_14672_gb300 import dstd
+    p = ctypes.byref(_layer())
+    one = ctypes.c_void_p(256)
+    assert lib.dstd_dense_fwd(None, one, 8, 16, 16, p, 0, one, one, None, one, 1 << 20, None) == -1
+    assert lib.dstd_dense_fwd(one, one, 0, 16, 16, p, 0, one, one, None, one, 1 << 20, None) == -1
+    assert lib.dstd_dense_fwd(one, one, 8, 16, 16, None, 0, one, one, None, one, 1 << 20, None) == -1
+    assert lib.dstd_dense_fwd(one, one, 8, 16, 16, p, 7, one, one, None, one, 1 << 20, None) == -1
+    # misaligned pointer
+    odd = ctypes.c_void_p(258)
+    assert lib.dstd_dense_fwd(odd, one, 8, 16, 16, p, 0, one, one, None, one, 1 << 20, None) == -1
+    # workspace too small
+    assert lib.dstd_dense_fwd(one, one, 8, 16, 16, p, 1, one, one, None, one, 16, None) == -3
+    assert lib.dstd_dense_bwd(one, one, one, one, one, 8, 16, 16, p, 1, None, None, one, 1 << 20, None) == -1
+    assert lib.dstd_dense_bwd(one, one, one, one, one, 8, 16, 16, p, 1, None, one, one, 16, None) == -3
+    assert lib.dstd_binning(None, 8, 16, p, one, None, None) == -1
+    assert lib.dstd_scan_solve(one, 8, 16, p, None, None, None, None, None) == -1
+    assert lib.dstd_dense_what(one, one, 8, 16, 16, p, 0, None, one, 1 << 20, None) == -1
+    assert lib.dstd_ce_loss(one, one, 8, 10, ctypes.c_float(0.0), ctypes.c_float(1.0), one, one, None) == -1
+    assert lib.dstd_sum_t_loss(one, 0, one, one, None) == -1
+    assert lib.dstd_adamw(one, one, one, one, 10, ctypes.c_float(1e-3), ctypes.c_float(1.5), ctypes.c_float(0.9),
+                          ctypes.c_float(1e-8), ctypes.c_float(0.0), 1, None) == -1
+    assert lib.dstd_adamw(one, one, one, one, 10, ctypes.c_float(1e-3), ctypes.c_float(0.9), ctypes.c_float(0.9),
+                          ctypes.c_float(1e-8), ctypes.c_float(0.0), 0, None) == -1

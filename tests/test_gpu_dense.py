@@ -1,0 +1,345 @@
+"""GPU parity of the dense DSTD layer against the float64 oracle.
+
+Tolerances:
+  spike times   |dt| <= 1e-4 * T_max (T_max = the layer's window length);
+  firing masks  identical except where the oracle's peak v^ lies within 1e-5
+                of v_th (those neurons are also left out of time parity);
+  gradients     relative L2 error <= 1e-3;
+  binning       weights to 2e-6 absolute (values are O(1) fp32 numbers).
+The CUDA path sees float32 inputs, so the oracle runs on the float32-rounded
+values of the same seeded inputs. The bf16 math mode is compared with the
+oracle run on bf16-rounded contraction operands (reading R9).
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from helpers import bf16, decode_saved, dense_layer, f32, oracle_forward, rel_l2, well_conditioned
+from oracle import dstd as odstd, losses as olosses
+
+pytestmark = pytest.mark.gpu
+
+INF = math.inf
+TAUS = [(0.5, 0.25), (INF, INF), (INF, 0.3), (0.3, INF), (0.4, 0.4), (1.0, 0.25), (0.25, 0.5)]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    from paper_2607_14672_gb300 import build, dstd
+    build.build()
+    dstd.load()
+    assert dstd.device_status(clear=True) == 0
+    yield
+    assert dstd.device_status(clear=True) == 0
+
+
+def dev(x, dtype=torch.float32):
+    return torch.tensor(np.asarray(x), dtype=dtype, device="cuda").contiguous()
+
+
+def host(x):
+    return x.detach().cpu().numpy().astype(np.float64)
+
+
+def run_fwd(t_in, layer, math_mode, penalty_norm=None):
+    from paper_2607_14672_gb300 import dstd
+    B, N_in = t_in.shape
+    N_out = layer["W"].shape[0]
+    p = dstd.params(layer, penalty_norm if penalty_norm is not None else 1.0 / B)
+    ws = torch.empty(dstd.dense_workspace_bytes(B, N_in, N_out, p, math_mode), dtype=torch.uint8, device="cuda")
+    t = dev(t_in)
+    W = dev(layer["W"])
+    t_out = torch.empty(B, N_out, device="cuda")
+    saved = torch.empty(dstd.dense_saved_bytes(B, N_out), dtype=torch.uint8, device="cuda")
+    pen = torch.empty(4, device="cuda")
+    dstd.dense_fwd(t, W, p, math_mode, t_out, saved, pen, ws)
+    torch.cuda.synchronize()
+    return dict(t=host(t_out), saved=saved, pen=host(pen), p=p, ws=ws, t_dev=t, W_dev=W, t_out_dev=t_out)
+
+
+def check_times(t_gpu, ctx, layer, tol_scale=1.0, margin=1e-5):
+    """Masks and spike times against the oracle; returns the number compared."""
+    Tmax = layer["t_end"] - layer["t_first"]
+    ok = well_conditioned(ctx, layer["v_th"], margin)
+    fired_o = np.isfinite(ctx["t"])
+    fired_g = np.isfinite(t_gpu)
+    bad = ok & (fired_o != fired_g)
+    assert not bad.any(), f"{bad.sum()} firing-mask mismatches outside the near-threshold band"
+    both = ok & fired_o & fired_g
+    err = np.abs(t_gpu[both] - ctx["t"][both])
+    assert err.size == 0 or err.max() <= 1e-4 * Tmax * tol_scale, f"max |dt| = {err.max():.3e}"
+    return int(both.sum())
+
+
+# ---------------------------------------------------------------------------
+# step a1: binning
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("tau_v,tau_I", TAUS)
+def test_binning_matches_oracle(tau_v, tau_I):
+    from paper_2607_14672_gb300 import dstd
+    layer = dict(tau_v=tau_v, tau_I=tau_I, v_th=1.0, t_first=0.1, t_end=1.3, M=20, t_offset=0.017)
+    T, dt = odstd.grid(0.1, 1.3, 20, 0.017)
+    g = np.random.default_rng(3)
+    t = g.uniform(-0.2, 1.5, (5, 300))                     # before, inside and after the window
+    t[:, :20] = T[g.integers(0, 21, 20)]                   # exactly on grid points
+    t[g.random(t.shape) < 0.1] = INF
+    t = f32(t)
+    s = torch.empty(5, 20, 300, device="cuda")
+    ds = torch.empty(5, 20, 300, device="cuda")
+    dstd.binning(dev(t), dstd.params(layer), s, ds)
+    torch.cuda.synchronize()
+    ref = odstd.binning(t, T, dt, tau_v, tau_I)
+    np.testing.assert_allclose(host(s), ref, rtol=0, atol=2e-6)
+    dref = odstd.binning(t, T, dt, tau_v, tau_I, derivative=True)
+    # derivatives are one-sided at knots; compare away from them
+    u = (t - T[0]) / dt
+    away = np.abs(u - np.round(u)) > 1e-3
+    away3 = np.broadcast_to(away[:, None, :], dref.shape)
+    scale = np.abs(dref).max()
+    np.testing.assert_allclose(host(ds)[away3], dref[away3], rtol=0, atol=2e-5 * scale)
+
+
+# ---------------------------------------------------------------------------
+# step a2: contraction w^ = W s
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("math_mode,rel", [("f32", 1e-5), ("bf16x3", 3e-5), ("bf16", None)])
+@pytest.mark.parametrize("shape", [(3, 37, 130, 20), (8, 200, 300, 32), (16, 784, 100, 8)])
+def test_contraction_matches_oracle(math_mode, rel, shape):
+    from paper_2607_14672_gb300 import dstd
+    B, N_in, N_out, M = shape
+    t_in, layer = dense_layer(B, N_in, N_out, M, 0.5, 0.25, seed=N_in, t_offset=0.01)
+    t_in, W = f32(t_in), f32(layer["W"])
+    layer["W"] = W
+    p = dstd.params(layer, 1.0 / B)
+    ws = torch.empty(dstd.dense_workspace_bytes(B, N_in, N_out, p, math_mode), dtype=torch.uint8, device="cuda")
+    what = torch.empty(B, N_out, M, device="cuda")
+    dstd.dense_what(dev(t_in), dev(W), p, math_mode, what, ws)
+    torch.cuda.synchronize()
+    T, dt = odstd.grid(layer["t_first"], layer["t_end"], M, layer["t_offset"])
+    s = odstd.binning(t_in, T, dt, 0.5, 0.25)
+    if math_mode == "bf16":
+        ref = np.einsum("bmj,ij->bim", bf16(s), bf16(W))
+        bound = 2.0 ** -16 * np.einsum("bmj,ij->bim", np.abs(s), np.abs(W)) + 1e-6
+    else:
+        ref = np.einsum("bmj,ij->bim", s, W)
+        bound = rel * np.einsum("bmj,ij->bim", np.abs(s), np.abs(W)) + 1e-7
+    err = np.abs(host(what) - ref)
+    assert (err <= bound).all(), f"max err/bound {np.max(err / bound):.3f}"
+
+
+# ---------------------------------------------------------------------------
+# steps a3/a4: scan, threshold solve, first-spike select (from given w^)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("tau_v,tau_I", TAUS)
+@pytest.mark.parametrize("M", [16, 20, 64])
+def test_scan_solve_matches_oracle(tau_v, tau_I, M):
+    from paper_2607_14672_gb300 import dstd
+    t_in, layer = dense_layer(16, 96, 200, M, tau_v, tau_I, seed=M + 7, t_offset=-0.004)
+    T, dt = odstd.grid(layer["t_first"], layer["t_end"], M, layer["t_offset"])
+    s = odstd.binning(f32(t_in), T, dt, tau_v, tau_I)
+    what = f32(np.einsum("bmj,ij->bim", s, f32(layer["W"])))
+    ctx = odstd.solve(what, T, dt, tau_v, tau_I, 1.0)
+    p = dstd.params(layer, 1.0 / 16)
+    t_out = torch.empty(16, 200, device="cuda")
+    saved = torch.empty(dstd.dense_saved_bytes(16, 200), dtype=torch.uint8, device="cuda")
+    dstd.scan_solve(dev(what), p, None, t_out, saved, None)
+    torch.cuda.synchronize()
+    tg = host(t_out)
+    n = check_times(tg, ctx, layer)
+    assert n > 500
+    q, sv, vd = decode_saved(saved.cpu().numpy(), 16, 200)
+    ok = well_conditioned(ctx, 1.0, 1e-4) & np.isfinite(ctx["t"])
+    # the spike's interval (a crossing on a grid point may land on either side)
+    assert np.mean(q[ok] == ctx["q"][ok]) > 0.999
+    assert np.all(np.abs(q[ok] - ctx["q"][ok]) <= 1)
+    np.testing.assert_allclose(vd[ok], np.maximum(ctx["vdot"][ok], odstd.vdot_floor(1.0, dt)), rtol=2e-3)
+    assert np.all(q[~np.isfinite(tg)] == M)
+
+
+# ---------------------------------------------------------------------------
+# whole layer forward
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("math_mode", ["f32", "bf16x3"])
+@pytest.mark.parametrize("tau_v,tau_I", TAUS)
+def test_forward_matches_oracle(math_mode, tau_v, tau_I):
+    t_in, layer = dense_layer(12, 150, 260, 32, tau_v, tau_I, seed=5, t_offset=0.013)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    r = run_fwd(t_in, layer, math_mode)
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    assert check_times(r["t"], ctx, layer) > 1000
+
+
+def test_forward_bf16_matches_rounded_oracle():
+    t_in, layer = dense_layer(16, 256, 256, 32, 0.5, 0.25, seed=9)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    r = run_fwd(t_in, layer, "bf16")
+    ctx = oracle_forward(t_in, layer["W"], layer, operand_round=bf16)
+    # bf16 operands: s is rounded from fp32 on the GPU and from fp64 in the
+    # oracle, which can differ by one bf16 step; tolerance and margin widen.
+    assert check_times(r["t"], ctx, layer, tol_scale=5.0, margin=1e-3) > 1500
+
+
+@pytest.mark.parametrize("math_mode", ["f32", "bf16x3"])
+@pytest.mark.parametrize("shape", [(1, 1, 1, 1), (1, 8, 129, 8), (2, 13, 7, 3), (5, 64, 32, 128), (3, 300, 257, 100)])
+def test_forward_ragged_shapes(math_mode, shape):
+    B, N_in, N_out, M = shape
+    t_in, layer = dense_layer(B, N_in, N_out, M, 0.5, 0.25, seed=B + N_in + M, fire=0.5)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    r = run_fwd(t_in, layer, math_mode)
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    check_times(r["t"], ctx, layer)
+
+
+def test_forward_f32_long_grid():
+    # M = 256 runs on the CUDA-core path only
+    t_in, layer = dense_layer(4, 64, 48, 256, 0.5, 0.25, seed=2)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    r = run_fwd(t_in, layer, "f32")
+    check_times(r["t"], oracle_forward(t_in, layer["W"], layer), layer)
+
+
+@pytest.mark.parametrize("math_mode", ["f32", "bf16x3", "bf16"])
+def test_all_silent_and_early_inputs(math_mode):
+    _, layer = dense_layer(4, 32, 40, 16, 0.5, 0.25, seed=1)
+    layer["W"] = f32(layer["W"])
+    r = run_fwd(np.full((4, 32), INF), layer, math_mode)
+    assert np.isinf(r["t"]).all()
+    assert r["pen"][2] == 4 * 40 and r["pen"][3] == 0
+    # inputs before T_{-1} carry no weight (reading R2): all silent as well
+    r2 = run_fwd(np.full((4, 32), -5.0), layer, math_mode)
+    assert np.isinf(r2["t"]).all()
+
+
+def test_penalty_terms_match_oracle():
+    t_in, layer = dense_layer(16, 120, 90, 32, 0.5, 0.25, seed=4, gammas=(0.05, 0.01, 1e-3), edges=(0.35, 0.7),
+                              fire=0.6)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    r = run_fwd(t_in, layer, "bf16x3")
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    Tv, _ = olosses.temporal_penalty(ctx["t"], 0.35, 0.7, 0.05, 0.01, 1.0 / 16)
+    Qv, cnt = olosses.dead_neuron_penalty(ctx["t"], layer["W"].sum(1), 1e-3, 1.0 / 16)
+    assert abs(r["pen"][0] - Tv) <= 1e-4 * abs(Tv) + 1e-7
+    assert abs(r["pen"][1] - Qv) <= 1e-4 * abs(Qv) + 1e-7
+    assert r["pen"][2] == (~np.isfinite(ctx["t"])).sum()
+    assert r["pen"][3] == np.isfinite(ctx["t"]).sum()
+
+
+# ---------------------------------------------------------------------------
+# whole layer backward
+# ---------------------------------------------------------------------------
+def _drop_ill_conditioned(t_in, layer, margin=1e-4):
+    """Keep the samples none of whose neurons grazes the threshold."""
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    keep = well_conditioned(ctx, layer["v_th"], margin).all(1)
+    return t_in[keep]
+
+
+@pytest.mark.parametrize("math_mode", ["f32", "bf16x3"])
+@pytest.mark.parametrize("tau_v,tau_I", TAUS)
+def test_backward_matches_oracle(math_mode, tau_v, tau_I):
+    from paper_2607_14672_gb300 import dstd
+    t_in, layer = dense_layer(24, 140, 150, 32, tau_v, tau_I, seed=17, t_offset=0.007,
+                              gammas=(0.05, 0.01, 1e-3), edges=(0.35, 0.8), fire=0.6)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    t_in = _drop_ill_conditioned(t_in, layer)
+    B = t_in.shape[0]
+    assert B >= 6
+    r = run_fwd(t_in, layer, math_mode)
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    check_times(r["t"], ctx, layer)
+    g = np.random.default_rng(2).normal(1.0, 0.5, r["t"].shape)
+    gup = np.where(np.isfinite(ctx["t"]), g, 0.0)
+    g_t_in = torch.empty(B, 140, device="cuda")
+    g_W = torch.empty(150, 140, device="cuda")
+    dstd.dense_bwd(r["t_dev"], r["W_dev"], r["t_out_dev"], r["saved"], dev(gup), r["p"], math_mode, g_t_in, g_W,
+                   r["ws"])
+    torch.cuda.synchronize()
+    # oracle: upstream + temporal-penalty gradient, then IFT backward, plus Q
+    _, gT = olosses.temporal_penalty(ctx["t"], 0.35, 0.8, 0.05, 0.01, 1.0 / B)
+    T, dt = ctx["T"], ctx["dt"]
+    gW_ref, gt_ref, _ = odstd.backward_dense(ctx, t_in, layer["W"], gup + gT, T, dt, tau_v, tau_I, 1.0)
+    _, cnt = olosses.dead_neuron_penalty(ctx["t"], layer["W"].sum(1), 1e-3, 1.0 / B)
+    gW_ref = gW_ref - 1e-3 / B * cnt[:, None]
+    assert rel_l2(host(g_W), gW_ref) <= 1e-3
+    assert rel_l2(host(g_t_in), gt_ref) <= 1e-3
+    assert np.all(host(g_t_in)[~np.isfinite(t_in)] == 0)
+
+
+def test_backward_without_input_gradient():
+    from paper_2607_14672_gb300 import dstd
+    t_in, layer = dense_layer(8, 64, 96, 16, 0.5, 0.25, seed=23)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    t_in = _drop_ill_conditioned(t_in, layer)
+    r = run_fwd(t_in, layer, "bf16x3")
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    gup = np.where(np.isfinite(ctx["t"]), 1.0, 0.0)
+    g_W = torch.empty(96, 64, device="cuda")
+    dstd.dense_bwd(r["t_dev"], r["W_dev"], r["t_out_dev"], r["saved"], dev(gup), r["p"], "bf16x3", None, g_W, r["ws"])
+    torch.cuda.synchronize()
+    gW_ref, _, _ = odstd.backward_dense(ctx, t_in, layer["W"], gup, ctx["T"], ctx["dt"], 0.5, 0.25, 1.0)
+    assert rel_l2(host(g_W), gW_ref) <= 1e-3
+
+
+# ---------------------------------------------------------------------------
+# losses and optimizer
+# ---------------------------------------------------------------------------
+def test_ce_loss_matches_oracle():
+    from paper_2607_14672_gb300 import dstd
+    g = np.random.default_rng(5)
+    t = f32(g.uniform(0.9, 1.4, (300, 10)))
+    t[g.random(t.shape) < 0.1] = INF
+    t[0, :] = INF
+    lab = g.integers(0, 10, 300)
+    loss = torch.empty(1, device="cuda")
+    gt = torch.empty(300, 10, device="cuda")
+    dstd.ce_loss(dev(t), dev(lab, torch.int32), 0.02, 1.4, loss, gt)
+    torch.cuda.synchronize()
+    L, G = olosses.ce_loss(t, lab, 0.02, 1.4)
+    assert abs(host(loss)[0] - L) <= 1e-5 * abs(L)
+    np.testing.assert_allclose(host(gt), G, rtol=1e-4, atol=1e-6)
+
+
+def test_sum_t_loss():
+    from paper_2607_14672_gb300 import dstd
+    t = np.array([0.5, INF, 1.25, 2.0, INF], np.float32)
+    loss = torch.empty(1, device="cuda")
+    gt = torch.empty(5, device="cuda")
+    dstd.sum_t_loss(dev(t), loss, gt)
+    torch.cuda.synchronize()
+    assert host(loss)[0] == pytest.approx(3.75)
+    np.testing.assert_array_equal(host(gt), [1, 0, 1, 1, 0])
+
+
+def test_adamw_matches_oracle():
+    from paper_2607_14672_gb300 import dstd
+    g = np.random.default_rng(6)
+    w0 = f32(g.normal(size=1000))
+    w, m, v = dev(w0), torch.zeros(1000, device="cuda"), torch.zeros(1000, device="cuda")
+    wr, mr, vr = w0.copy(), np.zeros(1000), np.zeros(1000)
+    for step in range(1, 4):
+        gr = f32(g.normal(size=1000))
+        dstd.adamw(w, dev(gr), m, v, 1e-3, 0.9, 0.999, 1e-8, 1e-2, step)
+        wr, mr, vr = olosses.adamw_step(wr, gr, mr, vr, step, 1e-3, 0.9, 0.999, 1e-8, 1e-2)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(host(w), wr, rtol=1e-5, atol=1e-7)
+
+
+# ---------------------------------------------------------------------------
+# host-side errors on a GPU machine and the device status word
+# ---------------------------------------------------------------------------
+def test_errors_leave_device_usable():
+    from paper_2607_14672_gb300 import dstd
+    _, layer = dense_layer(4, 16, 16, 200, 0.5, 0.25, seed=1, fire=0.0)
+    p = dstd.params(layer, 0.25)
+    assert dstd.dense_workspace_bytes(4, 16, 16, p, "bf16x3") == 0
+    ws = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
+    t_out = torch.empty(4, 16, device="cuda")
+    saved = torch.empty(dstd.dense_saved_bytes(4, 16), dtype=torch.uint8, device="cuda")
+    with pytest.raises(dstd.DstdError) as e:
+        dstd.dense_fwd(torch.zeros(4, 16, device="cuda"), torch.zeros(16, 16, device="cuda"), p, "bf16x3",
+                       t_out, saved, None, ws)
+    assert e.value.code == -2
+    assert dstd.device_status() == 0
