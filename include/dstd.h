@@ -55,14 +55,16 @@ enum {
     DSTD_E_NO_DEVICE = -6    /* no usable sm_103 device */
 };
 
-/* Arithmetic of the contraction w^ = W s (the only dense contraction).
- *  F32    CUDA-core fp32 FMA GEMM (reference precision).
- *  BF16X3 tcgen05 tensor cores, each fp32 operand split into bf16 hi + lo,
- *         three products (hi*hi + hi*lo + lo*hi) accumulated in fp32 TMEM:
- *         ~2^-17 relative operand error, for fp32 workloads.
- *  BF16   tcgen05 tensor cores, bf16 operands, fp32 accumulation.
+/* Arithmetic of the contractions (w^ = W s and its two transposes).
+ *  F32   CUDA-core fp32 FMA GEMMs (reference precision).
+ *  X3    tcgen05 tensor cores, each fp32 operand split into a 16-bit hi + lo
+ *        pair and three products (hi*hi + hi*lo + lo*hi) accumulated in fp32
+ *        TMEM, for fp32 workloads. Forward: fp16 pairs, W scaled per row by a
+ *        power of two into fp16 range (~2^-21 relative operand error; spike
+ *        times need it). Backward: bf16 pairs (~2^-17; gradients need 1e-3).
+ *  BF16  tcgen05 tensor cores, bf16 operands, fp32 accumulation.
  * Scan, solve, binning and every epilogue run in fp32 in all modes. */
-typedef enum { DSTD_MATH_F32 = 0, DSTD_MATH_BF16X3 = 1, DSTD_MATH_BF16 = 2 } dstd_math;
+typedef enum { DSTD_MATH_F32 = 0, DSTD_MATH_X3 = 1, DSTD_MATH_BF16 = 2 } dstd_math;
 
 /* One layer's constants (App. B.1 grid, App. C.1 synfire penalty).
  *  tau_m, tau_s    tau_v and tau_I of Eq. LIF_model_TTFS; > 0 or INFINITY.

@@ -52,14 +52,19 @@ int check_params(const dstd_params *p) {
 }
 
 int check_math(dstd_math m, int Mp) {
-    if (m != DSTD_MATH_F32 && m != DSTD_MATH_BF16X3 && m != DSTD_MATH_BF16) return DSTD_E_INVALID;
+    if (m != DSTD_MATH_F32 && m != DSTD_MATH_X3 && m != DSTD_MATH_BF16) return DSTD_E_INVALID;
     if (m != DSTD_MATH_F32 && Mp > 128) return DSTD_E_UNSUPPORTED;  // one sample per tensor-core tile
     return DSTD_OK;
 }
 
+// operand format of the forward contraction and of the two backward ones
 OpKind op_of(dstd_math m) {
-    return m == DSTD_MATH_F32 ? OpKind::F32 : (m == DSTD_MATH_BF16X3 ? OpKind::BF16X3 : OpKind::BF16);
+    return m == DSTD_MATH_F32 ? OpKind::F32 : (m == DSTD_MATH_X3 ? OpKind::F16X3 : OpKind::BF16);
 }
+OpKind bwd_op_of(dstd_math m) {
+    return m == DSTD_MATH_F32 ? OpKind::F32 : (m == DSTD_MATH_X3 ? OpKind::BF16X3 : OpKind::BF16);
+}
+bool two_part(OpKind op) { return op == OpKind::BF16X3 || op == OpKind::F16X3; }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -158,8 +163,8 @@ struct Timed {
 // the workspace base).
 // ---------------------------------------------------------------------------
 struct FwdWs {
-    __nv_bfloat16 *w_hi = nullptr, *w_lo = nullptr, *s_hi = nullptr, *s_lo = nullptr;
-    float *s32 = nullptr, *D = nullptr, *rowsum = nullptr;
+    uint16_t *w_hi = nullptr, *w_lo = nullptr, *s_hi = nullptr, *s_lo = nullptr;  // 16-bit operands
+    float *s32 = nullptr, *D = nullptr, *rowsum = nullptr, *row_scale = nullptr;
     size_t bytes = 0;
     int kpad = 0;
 };
@@ -174,10 +179,11 @@ FwdWs fwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
         w.s32 = b.take<float>((size_t)cols * w.kpad);
         w.D = b.take<float>((size_t)N_out * cols);
     } else {
-        w.w_hi = b.take<__nv_bfloat16>((size_t)N_out * w.kpad);
-        if (op == OpKind::BF16X3) w.w_lo = b.take<__nv_bfloat16>((size_t)N_out * w.kpad);
-        w.s_hi = b.take<__nv_bfloat16>((size_t)cols * w.kpad);
-        if (op == OpKind::BF16X3) w.s_lo = b.take<__nv_bfloat16>((size_t)cols * w.kpad);
+        w.w_hi = b.take<uint16_t>((size_t)N_out * w.kpad);
+        if (two_part(op)) w.w_lo = b.take<uint16_t>((size_t)N_out * w.kpad);
+        w.s_hi = b.take<uint16_t>((size_t)cols * w.kpad);
+        if (two_part(op)) w.s_lo = b.take<uint16_t>((size_t)cols * w.kpad);
+        if (op == OpKind::F16X3) w.row_scale = b.take<float>(N_out);
         if (need_D) w.D = b.take<float>((size_t)N_out * cols);
     }
     w.bytes = b.off;
@@ -291,8 +297,12 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
     }
     {
         Timed tm(KK_PREP, st);
-        TRY(cu(launch_prep_weights(W, N_out, N_in, op, ws.w_hi, ws.w_lo, ws.kpad, nullptr, nullptr, 0, nullptr, 0,
-                                   ws.rowsum, st)));
+        if (op == OpKind::F16X3)
+            TRY(cu(launch_prep_weights_f16(W, N_out, N_in, (__half *)ws.w_hi, (__half *)ws.w_lo, ws.kpad,
+                                           ws.row_scale, ws.rowsum, st)));
+        else
+            TRY(cu(launch_prep_weights(W, N_out, N_in, op, (__nv_bfloat16 *)ws.w_hi, (__nv_bfloat16 *)ws.w_lo,
+                                       ws.kpad, nullptr, nullptr, 0, nullptr, 0, ws.rowsum, st)));
     }
     {
         Timed tm(KK_BIN, st);
@@ -302,6 +312,7 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
     a.c = c;
     a.B = B;
     a.N = N_out;
+    a.row_scale = ws.row_scale;
     Timed tm(KK_GEMM_FWD, st);
     if (store_D) {
         a.D = ws.D;
@@ -354,7 +365,7 @@ size_t dstd_dense_workspace_bytes(int B, int N_in, int N_out, const dstd_params 
     if (check_math(math, Mp) != DSTD_OK) return 0;
     const OpKind op = op_of(math);
     size_t f = fwd_layout(nullptr, B, N_in, N_out, Mp, op, true).bytes;
-    size_t g = bwd_layout(nullptr, B, N_in, N_out, Mp, op, true).bytes;
+    size_t g = bwd_layout(nullptr, B, N_in, N_out, Mp, bwd_op_of(math), true).bytes;
     return f > g ? f : g;
 }
 
@@ -431,13 +442,14 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
     const int Mp = padded_M(p->M);
     TRY(check_math(math, Mp));
     if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
-    const OpKind op = op_of(math);
+    const OpKind bop = bwd_op_of(math);
+    const OpKind op = bop;
     const bool need_gt = g_t_in != nullptr;
-    if (ws_bytes < bwd_layout(nullptr, B, N_in, N_out, Mp, op, need_gt).bytes) return DSTD_E_WORKSPACE;
+    if (ws_bytes < bwd_layout(nullptr, B, N_in, N_out, Mp, bop, need_gt).bytes) return DSTD_E_WORKSPACE;
     TRY(device_ok());
     LifConst c = make_const(*p, Mp);
     cudaStream_t st = (cudaStream_t)stream;
-    BwdWs ws = bwd_layout(workspace, B, N_in, N_out, Mp, op, need_gt);
+    BwdWs ws = bwd_layout(workspace, B, N_in, N_out, Mp, bop, need_gt);
     Saved sv = saved_view(const_cast<void *>(saved), B, N_out);
     const long long cols = (long long)B * Mp;
     const float qcoef = -p->gamma_q * p->penalty_norm;

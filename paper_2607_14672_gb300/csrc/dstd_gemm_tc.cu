@@ -11,8 +11,12 @@
 //          reaches HBM,
 //   GradT  rows = inputs, columns = (sample, grid step): the input-time
 //          gradient sum_m dS ds/dt, so dS never reaches HBM.
-// BF16X3 splits each fp32 operand into bf16 hi + lo and accumulates
-// hi*hi + hi*lo + lo*hi (three MMAs per K step) for ~fp32 operand accuracy.
+// The three-product split (fp32 operand = 16-bit hi + lo) accumulates
+// hi*hi + hi*lo + lo*hi (three MMAs per K step). The tensor core's fp32
+// accumulation error grows with the number of MMAs summed into one
+// accumulator, so the main hi*hi products of successive k-tiles go round-robin
+// into P_MAIN separate TMEM accumulators and the small corrections into one
+// more; the epilogue adds them in fp32 registers.
 //
 // Every mbarrier wait is bounded (about 2 s of %globaltimer); an expired wait
 // sets the device status word, skips the epilogue and frees TMEM.
@@ -161,6 +165,25 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The tile's value at columns [cc, cc+32) of this lane: the sum of the n_main
+// main accumulators (columns p*BN + cc) and, with corr, the correction one.
+template <int BN>
+__device__ __forceinline__ void tmem_ld_acc(uint32_t tbase, int cc, int n_main, bool corr, float (&v)[32]) {
+    tmem_ld32(tbase + cc, v);
+    for (int p = 1; p < n_main; ++p) {
+        float u[32];
+        tmem_ld32(tbase + p * BN + cc, u);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] += u[j];
+    }
+    if (corr) {
+        float u[32];
+        tmem_ld32(tbase + 3 * BN + cc, u);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] += u[j];
+    }
+}
+
 // Shared-memory matrix descriptor (tcgen05 format): K-major operand tile with
 // 128-byte rows in 128-byte-swizzle layout; 8-row core-matrix groups are
 // 1024 bytes apart (SBO); LBO is not used by swizzled K-major layouts.
@@ -174,9 +197,11 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
     return d;
 }
 
-// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+// Instruction descriptor, kind::f16: D fp32, A and B both bf16 (format 1)
+// or both fp16 (format 0), both K-major.
+__host__ __device__ constexpr uint32_t idesc_16bit(int M, int N, bool f16) {
+    return (1u << 4) | ((f16 ? 0u : 1u) << 7) | ((f16 ? 0u : 1u) << 10) | ((uint32_t)(N >> 3) << 17) |
+           ((uint32_t)(M >> 4) << 24);
 }
 
 template <int NPASS, int BN>
@@ -187,19 +212,29 @@ struct Cfg {
     static constexpr int STAGE = NOP * (A_BYTES + B_BYTES);
     static constexpr int STAGES = (200 * 1024) / STAGE > 8 ? 8 : (200 * 1024) / STAGE;
     static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
-    static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+    // accumulators: P_MAIN round-robin copies of the tile for the main
+    // products (plus one for the hi*lo + lo*hi corrections when NPASS = 3)
+    static constexpr int P_MAIN = (NPASS == 3) ? 3 : 4;
+    static constexpr uint32_t TMEM_COLS = 4 * BN;  // 512 for BN = 128
+    static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
 };
 
 // ---------------------------------------------------------------------------
 // Epilogues. Each thread owns one accumulator row (its TMEM lane).
 // ---------------------------------------------------------------------------
+// Each warp of the epilogue owns one TMEM lane quarter (warp % 4) and a
+// range of 32-column chunks [c_lo, c_hi) of the tile.
 template <int BN>
-__device__ __forceinline__ void epi_store(uint32_t tbase, int row, int col0, int R, int Cn, const TcEpiArgs &a) {
+__device__ __forceinline__ void epi_store(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                          int c_hi, int R, int Cn, const TcEpiArgs &a) {
     float *D = a.D + (long long)blockIdx.z * a.zstride;
+    const float rs = (a.row_scale && row < R) ? a.row_scale[row] : 1.0f;
 #pragma unroll 1
-    for (int cc = 0; cc < BN; cc += 32) {
+    for (int cc = c_lo; cc < c_hi; cc += 32) {
         float v[32];
-        tmem_ld32(tbase + cc, v);
+        tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] *= rs;
         if (row < R) {
             float *dst = D + (long long)row * a.ldd + col0 + cc;
             if (col0 + cc + 32 <= Cn && (a.ldd % 4) == 0) {
@@ -222,23 +257,26 @@ __device__ __forceinline__ float warp_sum_tc(float x) {
 }
 
 template <int BN>
-__device__ __forceinline__ void epi_scan(uint32_t tbase, int row, int col0, const TcEpiArgs &a) {
+__device__ __forceinline__ void epi_scan(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                         int c_hi, const TcEpiArgs &a) {
     const LifConst &c = a.c;
     const int Mp = c.Mp;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    const float rs = (a.row_scale && row < a.N) ? a.row_scale[row] : 1.0f;
     ScanState st;
     scan_reset(st, c.M);
 #pragma unroll 1
-    for (int cc = 0; cc < BN; cc += 32) {
+    for (int cc = c_lo; cc < c_hi; cc += 32) {
         float v[32];
-        tmem_ld32(tbase + cc, v);
+        tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
             const int col = col0 + cc + j;
             const int m = col & (Mp - 1);
             if (m == 0) scan_reset(st, c.M);
-            if (m < c.M) scan_step(c, st, v[j], m);
+            if (m < c.M) scan_step(c, st, v[j] * rs, m);
             if (m == Mp - 1) {
+                scan_finish(c, st);
                 const int b = col / Mp;
                 if (row < a.N && b < a.B) {
                     long long o = (long long)b * a.N + row;
@@ -271,15 +309,16 @@ __device__ __forceinline__ void epi_scan(uint32_t tbase, int row, int col0, cons
 }
 
 template <int BN>
-__device__ __forceinline__ void epi_gradt(uint32_t tbase, int row, int col0, const TcEpiArgs &a) {
+__device__ __forceinline__ void epi_gradt(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                          int c_hi, const TcEpiArgs &a) {
     const LifConst &c = a.c;
     const int Mp = c.Mp;
     BinW w{-100, 0.f, 0.f, 0.f, 0.f};
     float g = 0.f;
 #pragma unroll 1
-    for (int cc = 0; cc < BN; cc += 32) {
+    for (int cc = c_lo; cc < c_hi; cc += 32) {
         float v[32];
-        tmem_ld32(tbase + cc, v);
+        tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
             const int col = col0 + cc + j;
@@ -305,8 +344,11 @@ __device__ __forceinline__ void epi_gradt(uint32_t tbase, int row, int col0, con
 // ---------------------------------------------------------------------------
 // The kernel.
 // ---------------------------------------------------------------------------
-template <int NPASS, int BN, int EPI>
-__global__ void __launch_bounds__(128, 1)
+constexpr int NWARPS = 16;  // 4 TMEM lane quarters x 4 column groups
+constexpr int NTHREADS = NWARPS * 32;
+
+template <int NPASS, int BN, int EPI, bool F16>
+__global__ void __launch_bounds__(NTHREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA_hi, const __grid_constant__ CUtensorMap mA_lo,
               const __grid_constant__ CUtensorMap mB_hi, const __grid_constant__ CUtensorMap mB_lo, int R, int Cn,
               int ktiles, int kt_per_split, TcEpiArgs args) {
@@ -362,7 +404,7 @@ __global__ void __launch_bounds__(128, 1)
     } else if (warp == 1) {
         if (lane == 0 && nkt > 0) {
             // MMA issuer
-            constexpr uint32_t idesc = idesc_bf16(BM, BN);
+            constexpr uint32_t idesc = idesc_16bit(BM, BN, F16);
             bool ok = true;
             for (int i = 0; i < nkt; ++i) {
                 const int s = i % C::STAGES;
@@ -377,14 +419,16 @@ __global__ void __launch_bounds__(128, 1)
                 const uint32_t a_lo = a_hi + C::A_BYTES;
                 const uint32_t b_hi = a_hi + C::NOP * C::A_BYTES;
                 const uint32_t b_lo = b_hi + C::B_BYTES;
+                const uint32_t acc_main = tmem + (uint32_t)((i % C::P_MAIN) * BN);
+                const uint32_t acc_corr = tmem + (uint32_t)(3 * BN);
 #pragma unroll
                 for (int kk = 0; kk < BK / 16; ++kk) {
                     const uint64_t da = sdesc_sw128(a_hi + kk * 32);
                     const uint64_t db = sdesc_sw128(b_hi + kk * 32);
-                    mma_bf16(tmem, da, db, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                    mma_bf16(acc_main, da, db, idesc, (i >= C::P_MAIN || kk > 0) ? 1u : 0u);
                     if (NPASS == 3) {
-                        mma_bf16(tmem, da, sdesc_sw128(b_lo + kk * 32), idesc, 1u);
-                        mma_bf16(tmem, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
+                        mma_bf16(acc_corr, da, sdesc_sw128(b_lo + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                        mma_bf16(acc_corr, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
                     }
                 }
                 mma_commit(&empty[s]);
@@ -394,15 +438,28 @@ __global__ void __launch_bounds__(128, 1)
         __syncwarp();
     }
 
-    // epilogue: all four warps, warp w owns TMEM lanes 32w .. 32w+31
+    // epilogue: all 16 warps; warp w reads TMEM lane quarter w % 4 (rows
+    // 32(w%4) .. +31) and column group w / 4. Scan and GradT keep a sample's
+    // columns in one thread, so a group takes whole samples (a sample spans
+    // max(1, Mp/32) chunks of 32 columns).
     const bool acc_ok = (nkt > 0) && mbar_wait(accf, 0);
     tc_fence_after();
     if (acc_ok) {
-        const uint32_t tbase = tmem + ((uint32_t)(warp * 32) << 16);
-        const int row = row0 + warp * 32 + lane;
-        if (EPI == (int)Epi::Store) epi_store<BN>(tbase, row, col0, R, Cn, args);
-        else if (EPI == (int)Epi::Scan) epi_scan<BN>(tbase, row, col0, args);
-        else epi_gradt<BN>(tbase, row, col0, args);
+        const int quarter = warp & 3, group = warp >> 2;
+        const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16);
+        const int row = row0 + quarter * 32 + lane;
+        int c_lo = group * 32, c_hi = c_lo + 32;
+        if (EPI != (int)Epi::Store) {
+            const int cps = args.c.Mp > 32 ? args.c.Mp / 32 : 1;  // chunks per sample
+            c_lo = group * cps * 32;
+            c_hi = c_lo + cps * 32;
+            if (c_lo >= BN) c_lo = c_hi = BN;
+        }
+        const int n_main = nkt < C::P_MAIN ? nkt : C::P_MAIN;
+        const bool corr = (NPASS == 3);
+        if (EPI == (int)Epi::Store) epi_store<BN>(tbase, n_main, corr, row, col0, c_lo, c_hi, R, Cn, args);
+        else if (EPI == (int)Epi::Scan) epi_scan<BN>(tbase, n_main, corr, row, col0, c_lo, c_hi, args);
+        else epi_gradt<BN>(tbase, n_main, corr, row, col0, c_lo, c_hi, args);
     } else if (nkt > 0) {
         set_status(STATUS_TIMEOUT);
     }
@@ -432,21 +489,22 @@ static EncodeTiledFn get_encode() {
     return fn;
 }
 
-// rows x cols bf16 matrix with row stride ld elements; box = box_rows x 64
-static bool make_map(CUtensorMap *m, const void *ptr, int rows, int cols, int ld, int box_rows) {
+// rows x cols 16-bit matrix with row stride ld elements; box = box_rows x 64
+static bool make_map(CUtensorMap *m, const void *ptr, int rows, int cols, int ld, int box_rows, bool f16) {
     EncodeTiledFn enc = get_encode();
     if (!enc) return false;
     cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     cuuint64_t gstride[1] = {(cuuint64_t)ld * 2};
     cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), gdim, gstride, box, estr,
+    CUresult r = enc(m, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                     const_cast<void *>(ptr), gdim, gstride, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
 
-template <int NPASS, int BN, int EPI>
+template <int NPASS, int BN, int EPI, bool F16>
 static cudaError_t launch_one(const CUtensorMap &a_hi, const CUtensorMap &a_lo, const CUtensorMap &b_hi,
                               const CUtensorMap &b_lo, int R, int Cn, int K, int splits, const TcEpiArgs &args,
                               cudaStream_t st) {
@@ -454,14 +512,14 @@ static cudaError_t launch_one(const CUtensorMap &a_hi, const CUtensorMap &a_lo, 
     static bool attr_set = false;  // per instantiation
     if (!attr_set) {
         cudaError_t e =
-            cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+            cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI, F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     const int ktiles = (K + BK - 1) / BK;
     const int per = (ktiles + splits - 1) / splits;
     dim3 grid((Cn + BN - 1) / BN, (R + BM - 1) / BM, splits);
-    k_tc_gemm<NPASS, BN, EPI><<<grid, 128, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per, args);
+    k_tc_gemm<NPASS, BN, EPI, F16><<<grid, NTHREADS, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per, args);
     return cudaGetLastError();
 }
 
@@ -478,34 +536,38 @@ int tc_gemm_splits_valid(int K, int splits) {
     return per * (splits - 1) < ktiles;
 }
 
-cudaError_t launch_tc_gemm(const __nv_bfloat16 *A_hi, const __nv_bfloat16 *A_lo, int lda, const __nv_bfloat16 *B_hi,
-                           const __nv_bfloat16 *B_lo, int ldb, int R, int Cn, int K, int splits, OpKind op, Epi epi,
-                           const TcEpiArgs &args, cudaStream_t st) {
+cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo, int ldb,
+                           int R, int Cn, int K, int splits, OpKind op, Epi epi, const TcEpiArgs &args,
+                           cudaStream_t st) {
     constexpr int BN = 128;
     CUtensorMap a_hi, a_lo, b_hi, b_lo;
-    const bool three = (op == OpKind::BF16X3);
-    if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM) || !tc::make_map(&b_hi, B_hi, Cn, K, ldb, BN))
+    const bool three = (op == OpKind::BF16X3 || op == OpKind::F16X3);
+    const bool f16 = (op == OpKind::F16X3);
+    if (op == OpKind::F32) return cudaErrorInvalidValue;
+    if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM, f16) || !tc::make_map(&b_hi, B_hi, Cn, K, ldb, BN, f16))
         return cudaErrorInvalidValue;
     if (three) {
-        if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM) || !tc::make_map(&b_lo, B_lo, Cn, K, ldb, BN))
+        if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM, f16) || !tc::make_map(&b_lo, B_lo, Cn, K, ldb, BN, f16))
             return cudaErrorInvalidValue;
     } else {
         a_lo = a_hi;
         b_lo = b_hi;
     }
     if (splits < 1) splits = 1;
-    if (three) {
-        switch (epi) {
-            case Epi::Store: return tc::launch_one<3, BN, 0>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
-            case Epi::Scan: return tc::launch_one<3, BN, 1>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
-            default: return tc::launch_one<3, BN, 2>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
-        }
+#define DSTD_TC_LAUNCH(NP, F)                                                                              \
+    switch (epi) {                                                                                         \
+        case Epi::Store: return tc::launch_one<NP, BN, 0, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st); \
+        case Epi::Scan: return tc::launch_one<NP, BN, 1, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);  \
+        default: return tc::launch_one<NP, BN, 2, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);         \
     }
-    switch (epi) {
-        case Epi::Store: return tc::launch_one<1, BN, 0>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
-        case Epi::Scan: return tc::launch_one<1, BN, 1>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
-        default: return tc::launch_one<1, BN, 2>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);
+    if (f16) {
+        DSTD_TC_LAUNCH(3, true)
+    } else if (three) {
+        DSTD_TC_LAUNCH(3, false)
+    } else {
+        DSTD_TC_LAUNCH(1, false)
     }
+#undef DSTD_TC_LAUNCH
 }
 
 }  // namespace dstd

@@ -4,6 +4,7 @@
 
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <stdint.h>
 
 #include "../../include/dstd.h"
@@ -32,6 +33,7 @@ struct LifConst {
     float vth;
     int M, Mp;             // steps, padded bin axis of the internal layouts
     float vdot_floor;      // lower bound on dv^/dt at a spike (1e-6 v_th / dt)
+    float Kmax;            // max of K(s) over s in [0, dt] (with a 1e-6 relative margin)
     float t_head, t_tail, g_head, g_tail, g_q, norm;
 };
 
@@ -87,16 +89,20 @@ __device__ __forceinline__ BinW bin_weights(const LifConst &c, float t, bool der
 // (v, I) <- (rv v + KD I, rI I). On interval q the potential is
 //     v^(s) = e^{-av s} (v_q + phi(s) I_q),  s = t - T_q in [0, dt),
 // with at most one interior extremum. The first interval whose maximum
-// reaches v_th holds the spike; its root is found by safeguarded Newton.
+// reaches v_th holds the spike. The scan only finds that interval (a cheap
+// bound, max(v_q, 0) + max(I_q, 0) Kmax >= v_th, gates the exact checks);
+// its root is solved once afterwards (scan_finish), by safeguarded Newton,
+// so the lanes of a warp solve together instead of once per interval.
 // ---------------------------------------------------------------------------
 struct ScanState {
     float v, I;
     int q;       // M while silent
+    float v0, I0, hi;  // state at T_q and bracket end of the firing interval
     float s, vdot;
 };
 
 __device__ __forceinline__ void scan_reset(ScanState &st, int M) {
-    st.v = 0.f; st.I = 0.f; st.q = M; st.s = 0.f; st.vdot = 0.f;
+    st.v = 0.f; st.I = 0.f; st.q = M; st.v0 = 0.f; st.I0 = 0.f; st.hi = 0.f; st.s = 0.f; st.vdot = 0.f;
 }
 
 __device__ __forceinline__ float vhat_at(const LifConst &c, float v0, float I0, float s) {
@@ -128,34 +134,44 @@ __device__ __forceinline__ float interval_root(const LifConst &c, float v0, floa
 // Consume w^_m for interval m (m = 0..M-1, in order).
 __device__ __forceinline__ void scan_step(const LifConst &c, ScanState &st, float w, int m) {
     if (st.q < c.M) return;
-    float v0 = st.v;
-    float I0 = st.I + w;
-    float ve = c.rv * v0 + c.KD * I0;
-    float s = -1.0f;
-    if (v0 >= c.vth) {
-        s = 0.0f;
-    } else if (ve >= c.vth) {
-        s = interval_root(c, v0, I0, c.dt);
-    } else if (c.av > 0.0f && c.aI > 0.0f && I0 > 0.0f) {
-        // interior maximum: dv^/ds > 0 at s = 0 and < 0 at s = dt
-        float d0 = -c.av * v0 + I0;
-        float dE = -c.av * ve + c.rI * I0;
-        if (d0 > 0.0f && dE < 0.0f) {
-            // e^{-lam s*} = 1 + lam y with y = (av v0 - I0)/(I0 aI)
-            float y = (c.av * v0 - I0) / (I0 * c.aI);
-            float sp = c.lam_zero ? -y : -log1pf(c.lam * y) / c.lam;
-            sp = fminf(fmaxf(sp, 0.0f), c.dt);
-            if (vhat_at(c, v0, I0, sp) >= c.vth) s = interval_root(c, v0, I0, sp);
-        }
-    }
-    if (s >= 0.0f) {
-        st.q = m;
-        st.s = s;
-        float Ic = I0 * __expf(-c.aI * s);
-        st.vdot = fmaxf(-c.av * c.vth + Ic, c.vdot_floor);
-    }
+    const float v0 = st.v;
+    const float I0 = st.I + w;
+    const float ve = c.rv * v0 + c.KD * I0;
     st.v = ve;
     st.I = c.rI * I0;
+    if (fmaxf(v0, 0.0f) + fmaxf(I0, 0.0f) * c.Kmax < c.vth) return;  // v^ < v_th on this interval
+    float hi = -1.0f;
+    if (v0 >= c.vth) {
+        hi = 0.0f;
+    } else if (ve >= c.vth) {
+        hi = c.dt;
+    } else if (c.av > 0.0f && c.aI > 0.0f && I0 > 0.0f) {
+        // interior maximum: dv^/ds > 0 at s = 0 and < 0 at s = dt
+        const float d0 = -c.av * v0 + I0;
+        const float dE = -c.av * ve + c.rI * I0;
+        if (d0 > 0.0f && dE < 0.0f) {
+            // e^{-lam s*} = 1 + lam y with y = (av v0 - I0)/(I0 aI)
+            const float y = (c.av * v0 - I0) / (I0 * c.aI);
+            float sp = c.lam_zero ? -y : -log1pf(c.lam * y) / c.lam;
+            sp = fminf(fmaxf(sp, 0.0f), c.dt);
+            if (vhat_at(c, v0, I0, sp) >= c.vth) hi = sp;
+        }
+    }
+    if (hi >= 0.0f) {
+        st.q = m;
+        st.v0 = v0;
+        st.I0 = I0;
+        st.hi = hi;
+    }
+}
+
+// Root of the firing interval and dv^/dt there (once per neuron).
+__device__ __forceinline__ void scan_finish(const LifConst &c, ScanState &st) {
+    if (st.q >= c.M) return;
+    const float s = st.hi > 0.0f ? interval_root(c, st.v0, st.I0, st.hi) : 0.0f;
+    st.s = s;
+    const float Ic = st.I0 * __expf(-c.aI * s);
+    st.vdot = fmaxf(-c.av * c.vth + Ic, c.vdot_floor);
 }
 
 // Temporal penalty of one firing neuron (Eq. temporal_penalty) and dT/dt,
@@ -180,10 +196,17 @@ cudaError_t launch_wait_selftest(unsigned long long limit_ns, cudaStream_t st);
 // Layouts: "internal" bin axis padded to Mp (power of two), rows of 16-bit
 // operands padded to a multiple of 8 elements (TMA needs 16-byte strides).
 // ---------------------------------------------------------------------------
-enum class OpKind { F32 = 0, BF16X3 = 1, BF16 = 2 };
+// Operand formats of a contraction: fp32 (CUDA cores), bf16 hi+lo, bf16,
+// fp16 hi+lo (values pre-scaled into fp16 range by the producer).
+enum class OpKind { F32 = 0, BF16X3 = 1, BF16 = 2, F16X3 = 3 };
 
 inline int pad8(int x) { return (x + 7) & ~7; }
 
+// W fp32 [R, C] -> fp16 hi/lo [R, ldo] of W * 2^k_i with one power of two
+// per row (largest |w| of the row near 2^14), inv_scale [R] = 2^-k_i, and
+// row sums [R]. One warp per row.
+cudaError_t launch_prep_weights_f16(const float *W, int R, int C, __half *hi, __half *lo, int ldo, float *inv_scale,
+                                    float *rowsum, cudaStream_t st);
 // W fp32 [R, C] -> hi/lo bf16 [R, ldo] (and optional transpose [C, ldt]),
 // fp32 copy (F32 path), row sums [R].
 cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bfloat16 *hi, __nv_bfloat16 *lo,
@@ -226,6 +249,7 @@ cudaError_t launch_sgemm_tn(const float *A, int lda, const float *Bm, int ldb, f
 // accumulation, with a fused epilogue.
 enum class Epi { Store = 0, Scan = 1, GradT = 2 };
 struct TcEpiArgs {
+    const float *row_scale;  // per-row factor applied to the accumulator (Store, Scan), may be null
     // Store
     float *D; long long ldd; long long zstride;
     // Scan (rows = neurons i, columns = (b, m))
@@ -233,9 +257,10 @@ struct TcEpiArgs {
     // GradT (rows = inputs j, columns = (b, m))
     const float *t_in; float *g_t_in;
 };
-cudaError_t launch_tc_gemm(const __nv_bfloat16 *A_hi, const __nv_bfloat16 *A_lo, int lda,
-                           const __nv_bfloat16 *B_hi, const __nv_bfloat16 *B_lo, int ldb, int R, int Cn, int K,
-                           int splits, OpKind op, Epi epi, const TcEpiArgs &args, cudaStream_t st);
+// A, B: 16-bit operands (bf16 for BF16X3 / BF16, fp16 for F16X3)
+cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo, int ldb,
+                           int R, int Cn, int K, int splits, OpKind op, Epi epi, const TcEpiArgs &args,
+                           cudaStream_t st);
 
 cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
                            float *loss, float *g, cudaStream_t st);

@@ -37,6 +37,15 @@ LifConst make_const(const dstd_params &p, int Mp) {
     c.M = p.M;
     c.Mp = Mp;
     c.vdot_floor = (float)(1e-6 * p.v_th / dt);
+    {
+        // K(s) = e^{-av s} phi(s) rises to a single maximum (or keeps rising
+        // when av = 0 or aI = 0); take it at min(dt, peak time)
+        double tp = dt;
+        if (av > 0.0 && aI > 0.0) tp = (lam == 0.0) ? 1.0 / av : log(aI / av) / lam;
+        const double s_ = tp < dt ? tp : dt;
+        const double phis = lam == 0.0 ? s_ : -expm1(-lam * s_) / lam;
+        c.Kmax = (float)(exp(-av * s_) * phis * (1.0 + 1e-6));
+    }
     c.t_head = p.t_head;
     c.t_tail = p.t_tail;
     c.g_head = p.gamma_head;
@@ -101,6 +110,56 @@ __global__ void k_prep_weights(const float *__restrict__ W, int R, int C, int op
     (void)op;
 }
 
+__device__ __forceinline__ void split_f16(float x, __half &hi, __half &lo) {
+    hi = __float2half_rn(x);
+    lo = __float2half_rn(x - __half2float(hi));
+}
+
+__global__ void k_prep_weights_f16(const float *__restrict__ W, int R, int C, __half *hi, __half *lo, int ldo,
+                                   float *inv_scale, float *rowsum) {
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= R) return;
+    const float *w = W + (long long)warp * C;
+    float amax = 0.f, sum = 0.f;
+    for (int j = lane; j < C; j += 32) {
+        float x = w[j];
+        amax = fmaxf(amax, fabsf(x));
+        sum += x;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+        sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    }
+    // power of two bringing the row's largest |w| into [2^13, 2^14]
+    int k = 0;
+    if (amax > 0.f && isfinite(amax)) {
+        int e;
+        frexpf(amax, &e);  // amax = f 2^e, f in [0.5, 1)
+        k = 14 - e;
+        k = k > 100 ? 100 : (k < -100 ? -100 : k);
+    }
+    const float sc = ldexpf(1.0f, k);
+    for (int j = lane; j < ldo; j += 32) {
+        __half h, l;
+        split_f16(j < C ? w[j] * sc : 0.f, h, l);
+        hi[(long long)warp * ldo + j] = h;
+        lo[(long long)warp * ldo + j] = l;
+    }
+    if (lane == 0) {
+        inv_scale[warp] = ldexpf(1.0f, -k);
+        if (rowsum) rowsum[warp] = sum;
+    }
+}
+
+cudaError_t launch_prep_weights_f16(const float *W, int R, int C, __half *hi, __half *lo, int ldo, float *inv_scale,
+                                    float *rowsum, cudaStream_t st) {
+    const long long threads = (long long)R * 32;
+    k_prep_weights_f16<<<blocks_for(threads, 256), 256, 0, st>>>(W, R, C, hi, lo, ldo, inv_scale, rowsum);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bfloat16 *hi, __nv_bfloat16 *lo,
                                 int ldo, __nv_bfloat16 *hiT, __nv_bfloat16 *loT, int ldt, float *f32T, int ldf,
                                 float *rowsum, cudaStream_t st) {
@@ -144,6 +203,12 @@ __global__ void k_binning_rows(const float *__restrict__ t, int B, int N, LifCon
         long long off = ((long long)b * c.Mp + m) * ld + j0;
         if (OP == 0) {
             *reinterpret_cast<float2 *>((float *)hi + off) = make_float2(v0, v1);
+        } else if (OP == 3) {
+            __half h0, l0, h1, l1;
+            split_f16(v0, h0, l0);
+            split_f16(v1, h1, l1);
+            *reinterpret_cast<__half2 *>((__half *)hi + off) = __halves2half2(h0, h1);
+            *reinterpret_cast<__half2 *>((__half *)lo + off) = __halves2half2(l0, l1);
         } else {
             __nv_bfloat16 h0, l0, h1, l1;
             split_bf16(v0, h0, l0);
@@ -196,6 +261,7 @@ cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKi
         dim3 grid(blocks_for(pairs, 128), B);
         if (op == OpKind::F32) k_binning_rows<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
         else if (op == OpKind::BF16X3) k_binning_rows<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+        else if (op == OpKind::F16X3) k_binning_rows<3><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
         else k_binning_rows<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
     } else {
         dim3 grid(blocks_for(B, 128), N < 65535 ? N : 65535);
@@ -281,6 +347,7 @@ __global__ void k_scan_solve(const float *__restrict__ what, long long sb, long 
             scan_step(c, st, w[m], m);
             if (st.q < c.M) break;
         }
+        scan_finish(c, st);
         finish_neuron(c, st, b, i, N, rowsum, t_out, q, s, vdot, acc);
     }
     flush_penalty(acc, penalty);

@@ -12,7 +12,7 @@ import os
 
 from .build import LIB_PATH
 
-MATH = {"f32": 0, "bf16x3": 1, "bf16": 2}
+MATH = {"f32": 0, "x3": 1, "bf16": 2}
 
 ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "workspace too small",
           -4: "CUDA call or kernel launch failed", -5: "a bounded device-side wait expired",

@@ -15,7 +15,7 @@ from . import dstd
 class DenseNet:
     """A stack of dense DSTD layers (configs.py layer dicts) on one GPU."""
 
-    def __init__(self, cfg, math_mode="bf16x3", batch=None, device="cuda", with_adamw=False):
+    def __init__(self, cfg, math_mode="x3", batch=None, device="cuda", with_adamw=False):
         self.cfg = cfg
         self.math = math_mode
         self.B = int(batch or cfg["batch"])

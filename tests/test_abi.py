@@ -62,10 +62,10 @@ def test_size_queries(lib):
     p = _layer()
     # q, s, vdot: 320 bytes each at 256-byte aligned offsets 0, 512, 1024
     assert dstd.dense_saved_bytes(8, 10) == 2 * 512 + 8 * 10 * 4
-    for m in ("f32", "bf16x3", "bf16"):
+    for m in ("f32", "x3", "bf16"):
         assert dstd.dense_workspace_bytes(256, 784, 800, p, m) > 0
-    # bf16x3 carries two copies of each operand
-    assert dstd.dense_workspace_bytes(256, 784, 800, p, "bf16x3") > dstd.dense_workspace_bytes(256, 784, 800, p, "bf16")
+    # the three-product split carries two copies of each operand
+    assert dstd.dense_workspace_bytes(256, 784, 800, p, "x3") > dstd.dense_workspace_bytes(256, 784, 800, p, "bf16")
     # invalid constants -> 0
     for bad in (dict(tau_v=-1.0), dict(tau_I=0.0), dict(v_th=0.0), dict(t_end=-1.0), dict(M=0),
                 dict(t_offset=0.5), dict(t_offset=-0.02), dict(tau_v=math.nan)):
@@ -73,7 +73,7 @@ def test_size_queries(lib):
     # infinite time constants are valid
     assert dstd.dense_workspace_bytes(8, 16, 16, _layer(tau_v=math.inf, tau_I=math.inf), "f32") > 0
     # tensor-core modes take M <= 128; the fp32 mode up to 256; beyond that nothing
-    assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=200), "bf16x3") == 0
+    assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=200), "x3") == 0
     assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=200), "f32") > 0
     assert dstd.dense_workspace_bytes(8, 16, 16, _layer(M=300), "f32") == 0
     assert dstd.dense_workspace_bytes(0, 16, 16, p, "f32") == 0

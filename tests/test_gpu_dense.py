@@ -105,7 +105,7 @@ def test_binning_matches_oracle(tau_v, tau_I):
 # ---------------------------------------------------------------------------
 # step a2: contraction w^ = W s
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("math_mode,rel", [("f32", 1e-5), ("bf16x3", 3e-5), ("bf16", None)])
+@pytest.mark.parametrize("math_mode,rel", [("f32", 1e-5), ("x3", 3e-5), ("bf16", None)])
 @pytest.mark.parametrize("shape", [(3, 37, 130, 20), (8, 200, 300, 32), (16, 784, 100, 8)])
 def test_contraction_matches_oracle(math_mode, rel, shape):
     from paper_2607_14672_gb300 import dstd
@@ -120,12 +120,20 @@ def test_contraction_matches_oracle(math_mode, rel, shape):
     torch.cuda.synchronize()
     T, dt = odstd.grid(layer["t_first"], layer["t_end"], M, layer["t_offset"])
     s = odstd.binning(t_in, T, dt, 0.5, 0.25)
+    ds = odstd.binning(t_in, T, dt, 0.5, 0.25, derivative=True)
+    aW = np.abs(W)
+    # an fp32 spike time is known to ~1e-7 absolute, so any fp32 binning sees
+    # t perturbed by that much: allow 3e-7 |ds/dt| per term
+    bound = 3e-7 * np.einsum("bmj,ij->bim", np.abs(ds), aW) + 1e-7
     if math_mode == "bf16":
         ref = np.einsum("bmj,ij->bim", bf16(s), bf16(W))
-        bound = 2.0 ** -16 * np.einsum("bmj,ij->bim", np.abs(s), np.abs(W)) + 1e-6
+        # bf16(s) from fp32 vs fp64 can differ by one bf16 step in single terms
+        ws_abs = np.abs(s)[:, None, :, :] * aW[None, :, None, :]          # [B, N_out, M, N_in]
+        # plus the tensor-core fp32 accumulation over K/16 products
+        bound = bound + 2.0 ** -14 * ws_abs.sum(-1) + 2.0 ** -8 * ws_abs.max(-1)
     else:
         ref = np.einsum("bmj,ij->bim", s, W)
-        bound = rel * np.einsum("bmj,ij->bim", np.abs(s), np.abs(W)) + 1e-7
+        bound = bound + rel * np.einsum("bmj,ij->bim", np.abs(s), aW)
     err = np.abs(host(what) - ref)
     assert (err <= bound).all(), f"max err/bound {np.max(err / bound):.3f}"
 
@@ -162,7 +170,7 @@ def test_scan_solve_matches_oracle(tau_v, tau_I, M):
 # ---------------------------------------------------------------------------
 # whole layer forward
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("math_mode", ["f32", "bf16x3"])
+@pytest.mark.parametrize("math_mode", ["f32", "x3"])
 @pytest.mark.parametrize("tau_v,tau_I", TAUS)
 def test_forward_matches_oracle(math_mode, tau_v, tau_I):
     t_in, layer = dense_layer(12, 150, 260, 32, tau_v, tau_I, seed=5, t_offset=0.013)
@@ -182,7 +190,7 @@ def test_forward_bf16_matches_rounded_oracle():
     assert check_times(r["t"], ctx, layer, tol_scale=5.0, margin=1e-3) > 1500
 
 
-@pytest.mark.parametrize("math_mode", ["f32", "bf16x3"])
+@pytest.mark.parametrize("math_mode", ["f32", "x3"])
 @pytest.mark.parametrize("shape", [(1, 1, 1, 1), (1, 8, 129, 8), (2, 13, 7, 3), (5, 64, 32, 128), (3, 300, 257, 100)])
 def test_forward_ragged_shapes(math_mode, shape):
     B, N_in, N_out, M = shape
@@ -201,7 +209,7 @@ def test_forward_f32_long_grid():
     check_times(r["t"], oracle_forward(t_in, layer["W"], layer), layer)
 
 
-@pytest.mark.parametrize("math_mode", ["f32", "bf16x3", "bf16"])
+@pytest.mark.parametrize("math_mode", ["f32", "x3", "bf16"])
 def test_all_silent_and_early_inputs(math_mode):
     _, layer = dense_layer(4, 32, 40, 16, 0.5, 0.25, seed=1)
     layer["W"] = f32(layer["W"])
@@ -217,14 +225,19 @@ def test_penalty_terms_match_oracle():
     t_in, layer = dense_layer(16, 120, 90, 32, 0.5, 0.25, seed=4, gammas=(0.05, 0.01, 1e-3), edges=(0.35, 0.7),
                               fire=0.6)
     t_in, layer["W"] = f32(t_in), f32(layer["W"])
-    r = run_fwd(t_in, layer, "bf16x3")
+    r = run_fwd(t_in, layer, "x3")
     ctx = oracle_forward(t_in, layer["W"], layer)
-    Tv, _ = olosses.temporal_penalty(ctx["t"], 0.35, 0.7, 0.05, 0.01, 1.0 / 16)
-    Qv, cnt = olosses.dead_neuron_penalty(ctx["t"], layer["W"].sum(1), 1e-3, 1.0 / 16)
+    check_times(r["t"], ctx, layer)
+    # the penalty arithmetic, on the spike times the GPU produced (a neuron
+    # grazing the threshold or the window end may fire on one side only)
+    Tv, _ = olosses.temporal_penalty(r["t"], 0.35, 0.7, 0.05, 0.01, 1.0 / 16)
+    Qv, cnt = olosses.dead_neuron_penalty(r["t"], layer["W"].sum(1), 1e-3, 1.0 / 16)
     assert abs(r["pen"][0] - Tv) <= 1e-4 * abs(Tv) + 1e-7
     assert abs(r["pen"][1] - Qv) <= 1e-4 * abs(Qv) + 1e-7
-    assert r["pen"][2] == (~np.isfinite(ctx["t"])).sum()
-    assert r["pen"][3] == np.isfinite(ctx["t"]).sum()
+    assert r["pen"][2] == (~np.isfinite(r["t"])).sum()
+    assert r["pen"][3] == np.isfinite(r["t"]).sum()
+    ok = well_conditioned(ctx, 1.0)
+    assert abs(r["pen"][3] - np.isfinite(ctx["t"]).sum()) <= (~ok).sum()
 
 
 # ---------------------------------------------------------------------------
@@ -237,7 +250,7 @@ def _drop_ill_conditioned(t_in, layer, margin=1e-4):
     return t_in[keep]
 
 
-@pytest.mark.parametrize("math_mode", ["f32", "bf16x3"])
+@pytest.mark.parametrize("math_mode", ["f32", "x3"])
 @pytest.mark.parametrize("tau_v,tau_I", TAUS)
 def test_backward_matches_oracle(math_mode, tau_v, tau_I):
     from paper_2607_14672_gb300 import dstd
@@ -273,11 +286,11 @@ def test_backward_without_input_gradient():
     t_in, layer = dense_layer(8, 64, 96, 16, 0.5, 0.25, seed=23)
     t_in, layer["W"] = f32(t_in), f32(layer["W"])
     t_in = _drop_ill_conditioned(t_in, layer)
-    r = run_fwd(t_in, layer, "bf16x3")
+    r = run_fwd(t_in, layer, "x3")
     ctx = oracle_forward(t_in, layer["W"], layer)
     gup = np.where(np.isfinite(ctx["t"]), 1.0, 0.0)
     g_W = torch.empty(96, 64, device="cuda")
-    dstd.dense_bwd(r["t_dev"], r["W_dev"], r["t_out_dev"], r["saved"], dev(gup), r["p"], "bf16x3", None, g_W, r["ws"])
+    dstd.dense_bwd(r["t_dev"], r["W_dev"], r["t_out_dev"], r["saved"], dev(gup), r["p"], "x3", None, g_W, r["ws"])
     torch.cuda.synchronize()
     gW_ref, _, _ = odstd.backward_dense(ctx, t_in, layer["W"], gup, ctx["T"], ctx["dt"], 0.5, 0.25, 1.0)
     assert rel_l2(host(g_W), gW_ref) <= 1e-3
@@ -334,12 +347,12 @@ def test_errors_leave_device_usable():
     from paper_2607_14672_gb300 import dstd
     _, layer = dense_layer(4, 16, 16, 200, 0.5, 0.25, seed=1, fire=0.0)
     p = dstd.params(layer, 0.25)
-    assert dstd.dense_workspace_bytes(4, 16, 16, p, "bf16x3") == 0
+    assert dstd.dense_workspace_bytes(4, 16, 16, p, "x3") == 0
     ws = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
     t_out = torch.empty(4, 16, device="cuda")
     saved = torch.empty(dstd.dense_saved_bytes(4, 16), dtype=torch.uint8, device="cuda")
     with pytest.raises(dstd.DstdError) as e:
-        dstd.dense_fwd(torch.zeros(4, 16, device="cuda"), torch.zeros(16, 16, device="cuda"), p, "bf16x3",
+        dstd.dense_fwd(torch.zeros(4, 16, device="cuda"), torch.zeros(16, 16, device="cuda"), p, "x3",
                        t_out, saved, None, ws)
     assert e.value.code == -2
     assert dstd.device_status() == 0

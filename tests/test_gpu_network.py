@@ -2,7 +2,7 @@
 the runtime pieces: CUDA-graph replay, kernel timing, bounded waits.
 
 The 784-800-800-10 workload is checked at its full batch of 256, in the
-bench's launch configuration (bf16x3 tensor cores, M = 32), layer by layer
+bench's launch configuration (x3 tensor-core split, M = 32), layer by layer
 with teacher forcing: each oracle layer is fed the GPU's previous-layer
 spike times, so a near-threshold flip upstream cannot propagate.
 """
@@ -33,7 +33,7 @@ def host(x):
     return x.detach().cpu().numpy().astype(np.float64)
 
 
-def _cfg2_net(math_mode="bf16x3", batch=256, keep=None, offsets=None):
+def _cfg2_net(math_mode="x3", batch=256, keep=None, offsets=None):
     from paper_2607_14672_gb300 import configs, net
     cfg = configs.config2(batch=batch)
     if offsets is not None:
@@ -58,55 +58,63 @@ def _teacher_forced_forward(n, t0):
     return ctxs
 
 
-@pytest.mark.parametrize("math_mode", ["bf16x3", "f32"])
+@pytest.mark.parametrize("math_mode", ["x3", "f32"])
 def test_cfg2_full_batch_teacher_forced(math_mode):
-    from paper_2607_14672_gb300 import configs
+    from paper_2607_14672_gb300 import configs, dstd
     offsets = configs.draw_offsets(configs.config2()["layers"])
     cfg, n, t0, lab = _cfg2_net(math_mode, offsets=offsets)
-    n.forward()
+    n.step()
     torch.cuda.synchronize()
+    B = t0.shape[0]
     ctxs = _teacher_forced_forward(n, t0)
-    clean = np.ones(t0.shape[0], bool)
+    ill = []
     for l, (ctx, L) in enumerate(zip(ctxs, n.layers)):
         tg = host(n.t[l])
         ok = well_conditioned(ctx, L["v_th"])
+        ill.append(~ok)
         fo, fg = np.isfinite(ctx["t"]), np.isfinite(tg)
         assert not (ok & (fo != fg)).any(), f"layer {l + 1}: mask mismatch"
         both = ok & fo & fg
         err = np.abs(tg[both] - ctx["t"][both]).max()
         assert err <= 1e-4 * configs.t_max(L), f"layer {l + 1}: max |dt| {err:.2e}"
         assert both.sum() > 0.5 * tg.size
-        clean &= well_conditioned(ctx, L["v_th"], 1e-4).all(1)
-    assert clean.sum() >= 200
-    # backward on the samples no neuron of which grazes the threshold
-    keep = np.nonzero(clean)[0]
-    cfg, n, t0, lab = _cfg2_net(math_mode, keep=keep, offsets=offsets)
-    n.step()
-    torch.cuda.synchronize()
-    B = t0.shape[0]
-    ctxs = _teacher_forced_forward(n, t0)
+    # CE gradient of the output layer
     tL = host(n.t[-1])
     _, gL = olosses.ce_loss(tL, lab, cfg["tau_soft"], n.layers[-1]["t_end"])
     assert rel_l2(host(n.g[-1]), gL) <= 1e-5
+    # backward, layer by layer with teacher forcing: both sides get the same
+    # upstream gradient; neurons whose peak grazes the threshold get a total
+    # gradient of zero on both sides (GPU: upstream = -dT/dt cancels the
+    # layer's own penalty term; oracle: zero)
+    g_up = host(n.g[-1])
+    gW_buf = [torch.empty_like(w) for w in n.W]
     for l in range(len(n.layers) - 1, -1, -1):
         L, ctx = n.layers[l], ctxs[l]
         Wl = f32(L["W"])
+        tg = host(n.t[l])
+        _, pg = olosses.temporal_penalty(tg, L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], 1.0 / B)
         _, gT = olosses.temporal_penalty(ctx["t"], L["t_head_l"], L["t_tail_l"], L["gamma_head"],
                                          L["gamma_tail"], 1.0 / B)
-        g_up = host(n.g[l])
+        g_gpu = np.where(ill[l], -pg, g_up)
+        g_ora = np.where(ill[l], 0.0, g_up + gT)
+        x_dev = n.layer_input(l)
         x = t0 if l == 0 else host(n.t[l - 1])
-        gW, gin, _ = odstd.backward_dense(ctx, x, Wl, g_up + gT, ctx["T"], ctx["dt"], L["tau_v"], L["tau_I"],
-                                          L["v_th"])
-        _, cnt = olosses.dead_neuron_penalty(ctx["t"], Wl.sum(1), L["gamma_q"], 1.0 / B)
+        g_in = torch.empty_like(x_dev) if l > 0 else None
+        dstd.dense_bwd(x_dev, n.W[l], n.t[l], n.saved[l], torch.tensor(g_gpu, dtype=torch.float32, device="cuda"),
+                       n.p[l], math_mode, g_in, gW_buf[l], n.workspace)
+        torch.cuda.synchronize()
+        gW, gin, _ = odstd.backward_dense(ctx, x, Wl, g_ora, ctx["T"], ctx["dt"], L["tau_v"], L["tau_I"], L["v_th"])
+        _, cnt = olosses.dead_neuron_penalty(tg, Wl.sum(1), L["gamma_q"], 1.0 / B)
         gW = gW - L["gamma_q"] / B * cnt[:, None]
-        assert rel_l2(host(n.gW[l]), gW) <= 1e-3, f"layer {l + 1} dW"
+        assert rel_l2(host(gW_buf[l]), gW) <= 1e-3, f"layer {l + 1} dW"
         if l > 0:
-            assert rel_l2(host(n.g[l - 1]), gin) <= 1e-3, f"layer {l + 1} dt_in"
+            assert rel_l2(host(g_in), gin) <= 1e-3, f"layer {l + 1} dt_in"
+            g_up = host(g_in)
 
 
 def test_cfg2_objective_matches_free_running_oracle():
     from paper_2607_14672_gb300 import configs
-    cfg, n, t0, lab = _cfg2_net("bf16x3", keep=np.arange(64))
+    cfg, n, t0, lab = _cfg2_net("x3", keep=np.arange(64))
     n.step()
     torch.cuda.synchronize()
     layers = [dict(L, W=f32(L["W"])) for L in n.layers]
@@ -118,7 +126,7 @@ def test_cfg2_objective_matches_free_running_oracle():
 
 
 def test_graph_replay_equals_eager():
-    cfg, n, t0, lab = _cfg2_net("bf16x3", batch=256)
+    cfg, n, t0, lab = _cfg2_net("x3", batch=256)
     n.step()
     torch.cuda.synchronize()
     t_e = [host(x) for x in n.t]
@@ -143,7 +151,7 @@ def test_graph_replay_equals_eager():
 
 def test_kernel_timing_counts_launches():
     from paper_2607_14672_gb300 import dstd
-    cfg, n, t0, lab = _cfg2_net("bf16x3", batch=64, keep=np.arange(64))
+    cfg, n, t0, lab = _cfg2_net("x3", batch=64, keep=np.arange(64))
     n.step()
     dstd.timing_enable(True)
     for _ in range(3):
@@ -161,7 +169,7 @@ def test_bounded_wait_reports_timeout():
     dstd.selftest_wait_timeout(20000)          # 20 ms wait on a barrier nothing completes
     assert dstd.device_status(clear=True) == -5
     # the context is still usable afterwards
-    cfg, n, t0, lab = _cfg2_net("bf16x3", batch=16, keep=np.arange(16))
+    cfg, n, t0, lab = _cfg2_net("x3", batch=16, keep=np.arange(16))
     n.step()
     assert dstd.device_status(clear=True) == 0
     assert np.isfinite(float(n.objective()))
@@ -171,7 +179,7 @@ def test_bounded_wait_reports_timeout():
 def test_cfg3_single_layer(N, M):
     from paper_2607_14672_gb300 import configs, net
     cfg = configs.config3(N, M, batch=16)
-    n = net.DenseNet(cfg, "bf16x3", batch=16)
+    n = net.DenseNet(cfg, "x3", batch=16)
     t0 = f32(cfg["inputs"](B=16))
     n.set_inputs(t0)
     n.forward()
@@ -192,7 +200,7 @@ def test_cfg3_full_size_sampled():
     # sampled outputs the oracle computes one by one
     from paper_2607_14672_gb300 import configs, net
     cfg = configs.config3(16384, 128)
-    n = net.DenseNet(cfg, "bf16x3")
+    n = net.DenseNet(cfg, "x3")
     t0 = f32(cfg["inputs"]())
     n.set_inputs(t0)
     n.forward()
