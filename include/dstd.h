@@ -129,6 +129,28 @@ int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
                    dstd_math math, float *t_out, void *saved, float *penalty, void *workspace,
                    size_t ws_bytes, dstd_stream_t stream);
 
+/* The layer forward of dstd_dense_fwd for callers that cannot allocate
+ * device memory: code that runs where cudaMalloc is unavailable or
+ * forbidden (inside a host callback, a real-time loop that may not touch the
+ * allocator, a plugin whose host application owns every allocation) and has
+ * no workspace to pass. It computes exactly what dstd_dense_fwd computes,
+ * with the same arguments minus the workspace; the caller still provides
+ * t_in, W, t_out, saved and penalty. (The paper has no counterpart: this is
+ * a deployment convenience of this library.)
+ * Scratch: a fixed 32 MiB array in device memory, part of the library's
+ * image, present on every GPU that loads the library until the process
+ * exits. A call whose scratch need (dstd_dense_workspace_bytes' forward part)
+ * exceeds 32 MiB returns DSTD_E_WORKSPACE and launches nothing; the 784-800
+ * and 800-800 layers at B = 256, M = 32 fit. No call allocates or frees.
+ * Every call uses the same array, which keeps whatever the previous call
+ * left there (each call overwrites all the scratch it reads), so two calls
+ * that can overlap on the GPU (different streams, or different host threads)
+ * race; serialise them. The first call on each device looks up the array's
+ * device address (cudaGetSymbolAddress) with that device current; make that
+ * first call before starting any stream capture. */
+int dstd_dense_fwd_noalloc(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                           dstd_math math, float *t_out, void *saved, float *penalty, dstd_stream_t stream);
+
 /* Backward of one dense DSTD layer.
  *  g_t_out [B, N_out] dC/dt_out from above (the loss or the next layer); the
  *          layer adds its own temporal-penalty gradient (params) itself.

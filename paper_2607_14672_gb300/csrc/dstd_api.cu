@@ -587,6 +587,63 @@ int dstd_selftest_wait_timeout(uint32_t timeout_us, dstd_stream_t stream) {
     return cu(launch_wait_selftest(1000ull * timeout_us, (cudaStream_t)stream));
 }
 
+// ---------------------------------------------------------------------------
+// Layer forward that allocates nothing (scratch in a static device array).
+// ---------------------------------------------------------------------------
+}  // extern "C"
+
+namespace {
+
+// Fixed scratch for dstd_dense_fwd_noalloc: 32 MiB, resident on every GPU
+// that loads this library, for as long as the process runs.
+constexpr size_t kNoAllocScratchBytes = 32ull << 20;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[128] = {};
+
+// Device address of the scratch array on the current device. The array's
+// name is only a host-side stand-in, so its address is looked up (once per
+// device, with that device current) and cached.
+int noalloc_scratch(void **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DSTD_E_NO_DEVICE;
+    if (dev < 0 || dev >= 128) return DSTD_E_UNSUPPORTED;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return DSTD_E_CUDA;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return DSTD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dstd_dense_fwd_noalloc(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                           dstd_math math, float *t_out, void *saved, float *penalty, dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(saved)) return DSTD_E_INVALID;
+    const OpKind op = op_of(math);
+    if (fwd_layout(nullptr, B, N_in, N_out, Mp, op, false).bytes > kNoAllocScratchBytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    void *scratch = nullptr;
+    TRY(noalloc_scratch(&scratch));
+    LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    FwdWs ws = fwd_layout(scratch, B, N_in, N_out, Mp, op, false);
+    Saved sv = saved_view(saved, B, N_out);
+    if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
+    return dense_forward_core(t_in, W, B, N_in, N_out, c, op, ws, false, &sv, t_out, penalty, st);
+}
+
 int dstd_device_status(int clear) {
     if (cudaDeviceSynchronize() != cudaSuccess) return DSTD_E_CUDA;
     unsigned int s = 0;

@@ -21,7 +21,8 @@ ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "
 EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning", "dstd_dense_what",
            "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
            "dstd_adamw", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
-           "dstd_timing_read", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout")
+           "dstd_timing_read", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
+           "dstd_dense_fwd_noalloc")
 
 
 class DstdError(RuntimeError):
@@ -85,6 +86,7 @@ def load(path=None):
         "dstd_kernel_kind_count": (_I, []),
         "dstd_kernel_kind_name": (ctypes.c_char_p, [_I]),
         "dstd_selftest_wait_timeout": (_I, [ctypes.c_uint32, _P]),
+        "dstd_dense_fwd_noalloc": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -176,6 +178,20 @@ def dense_fwd(t_in, W, p, math_mode, t_out, saved, penalty, workspace, stream=No
     _check(load().dstd_dense_fwd(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), MATH[math_mode], _ptr(t_out),
                                  _ptr(saved), _ptr(penalty), _ptr(workspace),
                                  workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_dense_fwd")
+
+
+def dense_fwd_noalloc(t_in, W, p, math_mode, t_out, saved, penalty=None, stream=None):
+    """dstd_dense_fwd without a workspace: for callers that cannot allocate
+    device memory; scratch is the library's fixed 32 MiB device array, shared
+    by every call (do not overlap calls on the GPU)."""
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(t_out, "t_out", (B, N_out))
+    _check(load().dstd_dense_fwd_noalloc(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), MATH[math_mode],
+                                         _ptr(t_out), _ptr(saved), _ptr(penalty), _stream(stream)),
+           "dstd_dense_fwd_noalloc")
 
 
 def dense_bwd(t_in, W, t_out, saved, g_t_out, p, math_mode, g_t_in, g_W, workspace, stream=None):
