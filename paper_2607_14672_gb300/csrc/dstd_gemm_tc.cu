@@ -90,6 +90,18 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
     }
 }
 
+// bounded wait with a sleep between polls, for warps that have nothing else
+// to do (the epilogue warps during the main loop)
+__device__ __forceinline__ bool mbar_wait_sleep(uint64_t *bar, uint32_t parity,
+                                                unsigned long long limit_ns = WAIT_NS) {
+    const uint64_t t0 = globaltimer();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (globaltimer() - t0 > limit_ns) return false;
+        __nanosleep(256);
+    }
+}
+
 // One thread waits on a barrier phase that never completes; the bounded wait
 // expires and records a timeout in the status word.
 __global__ void k_wait_selftest(unsigned long long limit_ns) {
@@ -256,12 +268,36 @@ __device__ __forceinline__ float warp_sum_tc(float x) {
     return x;
 }
 
-template <int BN>
-__device__ __forceinline__ void epi_scan(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                         int c_hi, const TcEpiArgs &a) {
+// Output of one neuron of one sample (spike time, saved state, penalty sums).
+__device__ __forceinline__ void scan_emit(const LifConst &c, const ScanState &st, int b, int row,
+                                          const TcEpiArgs &a, float (&acc)[4]) {
+    if (row >= a.N || b >= a.B) return;
+    const long long o = (long long)b * a.N + row;
+    const bool fired = st.q < c.M;
+    const float t = fired ? c.T0 + (float)st.q * c.dt + st.s : INFINITY;
+    a.t_out[o] = t;
+    a.q[o] = st.q;
+    a.s[o] = st.s;
+    a.vdot[o] = st.vdot;
+    if (fired) {
+        float pv, pg;
+        penalty_T(c, t, pv, pg);
+        acc[0] += pv;
+        acc[3] += 1.f;
+    } else {
+        if (a.rowsum) acc[1] += -c.g_q * c.norm * a.rowsum[row];
+        acc[2] += 1.f;
+    }
+}
+
+// Scan epilogue over chunks of 32 columns; SUB = min(Mp, 32) columns of one
+// sample are scanned per unrolled block, so the sample-end work appears once
+// per block instead of once per column.
+template <int BN, int SUB>
+__device__ __forceinline__ void epi_scan_sub(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                             int c_hi, const TcEpiArgs &a, float (&acc)[4]) {
     const LifConst &c = a.c;
     const int Mp = c.Mp;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
     const float rs = (a.row_scale && row < a.N) ? a.row_scale[row] : 1.0f;
     ScanState st;
     scan_reset(st, c.M);
@@ -270,35 +306,28 @@ __device__ __forceinline__ void epi_scan(uint32_t tbase, int n_main, bool corr, 
         float v[32];
         tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int col = col0 + cc + j;
-            const int m = col & (Mp - 1);
-            if (m == 0) scan_reset(st, c.M);
-            if (m < c.M) scan_step(c, st, v[j] * rs, m);
-            if (m == Mp - 1) {
+        for (int sb = 0; sb < 32; sb += SUB) {
+            const int col = col0 + cc + sb;          // first column of this block
+            const int m0 = col & (Mp - 1);
+            if (m0 == 0) scan_reset(st, c.M);
+#pragma unroll
+            for (int j = 0; j < SUB; ++j)
+                if (m0 + j < c.M) scan_step(c, st, v[sb + j] * rs, m0 + j);
+            if (m0 + SUB == Mp) {
                 scan_finish(c, st);
-                const int b = col / Mp;
-                if (row < a.N && b < a.B) {
-                    long long o = (long long)b * a.N + row;
-                    bool fired = st.q < c.M;
-                    float t = fired ? c.T0 + (float)st.q * c.dt + st.s : INFINITY;
-                    a.t_out[o] = t;
-                    a.q[o] = st.q;
-                    a.s[o] = st.s;
-                    a.vdot[o] = st.vdot;
-                    if (fired) {
-                        float pv, pg;
-                        penalty_T(c, t, pv, pg);
-                        acc[0] += pv;
-                        acc[3] += 1.f;
-                    } else {
-                        if (a.rowsum) acc[1] += -c.g_q * c.norm * a.rowsum[row];
-                        acc[2] += 1.f;
-                    }
-                }
+                scan_emit(c, st, col / Mp, row, a, acc);
             }
         }
     }
+}
+
+template <int BN>
+__device__ __forceinline__ void epi_scan(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                         int c_hi, const TcEpiArgs &a) {
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (a.c.Mp == 8) epi_scan_sub<BN, 8>(tbase, n_main, corr, row, col0, c_lo, c_hi, a, acc);
+    else if (a.c.Mp == 16) epi_scan_sub<BN, 16>(tbase, n_main, corr, row, col0, c_lo, c_hi, a, acc);
+    else epi_scan_sub<BN, 32>(tbase, n_main, corr, row, col0, c_lo, c_hi, a, acc);
     if (a.penalty) {
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -308,9 +337,9 @@ __device__ __forceinline__ void epi_scan(uint32_t tbase, int n_main, bool corr, 
     }
 }
 
-template <int BN>
-__device__ __forceinline__ void epi_gradt(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                          int c_hi, const TcEpiArgs &a) {
+template <int BN, int SUB>
+__device__ __forceinline__ void epi_gradt_sub(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                              int c_hi, const TcEpiArgs &a) {
     const LifConst &c = a.c;
     const int Mp = c.Mp;
     BinW w{-100, 0.f, 0.f, 0.f, 0.f};
@@ -320,25 +349,36 @@ __device__ __forceinline__ void epi_gradt(uint32_t tbase, int n_main, bool corr,
         float v[32];
         tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int col = col0 + cc + j;
-            const int m = col & (Mp - 1);
+        for (int sb = 0; sb < 32; sb += SUB) {
+            const int col = col0 + cc + sb;
+            const int m0 = col & (Mp - 1);
             const int b = col / Mp;
-            if (m == 0) {
+            if (m0 == 0) {
                 g = 0.f;
                 w.k = -100;
                 if (row < a.N && b < a.B) {
-                    float x = a.t_in[(long long)b * a.N + row];
+                    const float x = a.t_in[(long long)b * a.N + row];
                     if (isfinite(x)) w = bin_weights(c, x, true);
                 }
             }
-            if (m < c.M) {
-                if (m == w.k) g += v[j] * w.dR;
-                if (m == w.k + 1) g += v[j] * w.dL;
+            // the two grid points of the spike (m = k, k + 1), if in this block
+#pragma unroll
+            for (int j = 0; j < SUB; ++j) {
+                const int m = m0 + j;
+                g += (m == w.k && m < c.M) ? v[sb + j] * w.dR : 0.f;
+                g += (m == w.k + 1 && m < c.M) ? v[sb + j] * w.dL : 0.f;
             }
-            if (m == Mp - 1 && row < a.N && b < a.B) a.g_t_in[(long long)b * a.N + row] = g;
+            if (m0 + SUB == Mp && row < a.N && b < a.B) a.g_t_in[(long long)b * a.N + row] = g;
         }
     }
+}
+
+template <int BN>
+__device__ __forceinline__ void epi_gradt(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
+                                          int c_hi, const TcEpiArgs &a) {
+    if (a.c.Mp == 8) epi_gradt_sub<BN, 8>(tbase, n_main, corr, row, col0, c_lo, c_hi, a);
+    else if (a.c.Mp == 16) epi_gradt_sub<BN, 16>(tbase, n_main, corr, row, col0, c_lo, c_hi, a);
+    else epi_gradt_sub<BN, 32>(tbase, n_main, corr, row, col0, c_lo, c_hi, a);
 }
 
 // ---------------------------------------------------------------------------
@@ -442,7 +482,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // 32(w%4) .. +31) and column group w / 4. Scan and GradT keep a sample's
     // columns in one thread, so a group takes whole samples (a sample spans
     // max(1, Mp/32) chunks of 32 columns).
-    const bool acc_ok = (nkt > 0) && mbar_wait(accf, 0);
+    const bool acc_ok = (nkt > 0) && mbar_wait_sleep(accf, 0);
     tc_fence_after();
     if (acc_ok) {
         const int quarter = warp & 3, group = warp >> 2;

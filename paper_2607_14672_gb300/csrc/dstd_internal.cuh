@@ -131,6 +131,28 @@ __device__ __forceinline__ float interval_root(const LifConst &c, float v0, floa
     return fminf(fmaxf(s, 0.0f), hi);
 }
 
+// Exact firing test of one interval whose cheap bound reached v_th: the
+// bracket end for the root (0 if v^ is already at v_th at T_q, dt if v^(dt)
+// >= v_th, the interior maximum if only that reaches v_th), or -1. Kept out
+// of line so the per-interval fast path of the scan stays small.
+static __device__ __noinline__ float scan_interval_test(const LifConst &c, float v0, float I0, float ve) {
+    if (v0 >= c.vth) return 0.0f;
+    if (ve >= c.vth) return c.dt;
+    if (c.av > 0.0f && c.aI > 0.0f && I0 > 0.0f) {
+        // interior maximum: dv^/ds > 0 at s = 0 and < 0 at s = dt
+        const float d0 = -c.av * v0 + I0;
+        const float dE = -c.av * ve + c.rI * I0;
+        if (d0 > 0.0f && dE < 0.0f) {
+            // e^{-lam s*} = 1 + lam y with y = (av v0 - I0)/(I0 aI)
+            const float y = (c.av * v0 - I0) / (I0 * c.aI);
+            float sp = c.lam_zero ? -y : -log1pf(c.lam * y) / c.lam;
+            sp = fminf(fmaxf(sp, 0.0f), c.dt);
+            if (vhat_at(c, v0, I0, sp) >= c.vth) return sp;
+        }
+    }
+    return -1.0f;
+}
+
 // Consume w^_m for interval m (m = 0..M-1, in order).
 __device__ __forceinline__ void scan_step(const LifConst &c, ScanState &st, float w, int m) {
     if (st.q < c.M) return;
@@ -140,23 +162,7 @@ __device__ __forceinline__ void scan_step(const LifConst &c, ScanState &st, floa
     st.v = ve;
     st.I = c.rI * I0;
     if (fmaxf(v0, 0.0f) + fmaxf(I0, 0.0f) * c.Kmax < c.vth) return;  // v^ < v_th on this interval
-    float hi = -1.0f;
-    if (v0 >= c.vth) {
-        hi = 0.0f;
-    } else if (ve >= c.vth) {
-        hi = c.dt;
-    } else if (c.av > 0.0f && c.aI > 0.0f && I0 > 0.0f) {
-        // interior maximum: dv^/ds > 0 at s = 0 and < 0 at s = dt
-        const float d0 = -c.av * v0 + I0;
-        const float dE = -c.av * ve + c.rI * I0;
-        if (d0 > 0.0f && dE < 0.0f) {
-            // e^{-lam s*} = 1 + lam y with y = (av v0 - I0)/(I0 aI)
-            const float y = (c.av * v0 - I0) / (I0 * c.aI);
-            float sp = c.lam_zero ? -y : -log1pf(c.lam * y) / c.lam;
-            sp = fminf(fmaxf(sp, 0.0f), c.dt);
-            if (vhat_at(c, v0, I0, sp) >= c.vth) hi = sp;
-        }
-    }
+    const float hi = scan_interval_test(c, v0, I0, ve);
     if (hi >= 0.0f) {
         st.q = m;
         st.v0 = v0;
