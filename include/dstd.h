@@ -162,6 +162,31 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
                    const float *g_t_out, int B, int N_in, int N_out, const dstd_params *p, dstd_math math,
                    float *g_t_in, float *g_W, void *workspace, size_t ws_bytes, dstd_stream_t stream);
 
+/* Convolutional DSTD layer (3x3 / k x k filters, stride, zero-spike padding),
+ * the implicit-GEMM form of the same contraction: output position
+ * (b, y, x) plays the role of a sample and filter tap (kh, kw, c) of an input.
+ *  t_in   [B, H, W, C_in]     input spike times, NHWC (+inf = silent).
+ *  W      [C_out, k, k, C_in] weights (tap-major rows).
+ *  t_out  [B, Ho, Wo, C_out]  NHWC, Ho = (H + 2 pad - k)/stride + 1 (same Wo).
+ *  saved  dstd_dense_saved_bytes(B*Ho*Wo, C_out) bytes.
+ *  penalty as in dstd_dense_fwd; set p->penalty_norm = 1/(B*Ho*Wo) (App. C.1:
+ *          T and Q of conv layers are divided by the spatial size).
+ * Tensor-core math modes only (DSTD_MATH_F32 returns DSTD_E_UNSUPPORTED).
+ * Padding taps read silent inputs. Images are processed in chunks so the
+ * gathered operand stays near 1 GiB; the workspace query accounts for it. */
+size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k, int stride, int pad,
+                                 const dstd_params *p, dstd_math math);
+int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C_in, int C_out, int k, int stride,
+                  int pad, const dstd_params *p, dstd_math math, float *t_out, void *saved, float *penalty,
+                  void *workspace, size_t ws_bytes, dstd_stream_t stream);
+/* Backward of the conv layer: g_t_out [B, Ho, Wo, C_out]; g_t_in [B, H, W, C_in]
+ * (may be NULL; overwritten); g_W [C_out, k, k, C_in] (overwritten, with the
+ * dead-neuron term -gamma_q * norm * silent count of the output channel). */
+int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const void *saved, const float *g_t_out,
+                  int B, int H, int Wd, int C_in, int C_out, int k, int stride, int pad, const dstd_params *p,
+                  dstd_math math, float *g_t_in, float *g_W, void *workspace, size_t ws_bytes,
+                  dstd_stream_t stream);
+
 /* Cross-entropy over softmax(-t/tau_soft) (Eqs. cost_function, L, S_i),
  * mini-batch mean; a silent output enters with the constant time t_silent
  * and passes no gradient.

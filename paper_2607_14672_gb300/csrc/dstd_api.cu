@@ -331,6 +331,93 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
                              Epi::Scan, a, st));
 }
 
+// ---------------------------------------------------------------------------
+// Convolution layers: output positions act as samples, filter taps as the
+// contraction axis; the binned inputs are gathered per filter tap (im2col)
+// for a chunk of whole images at a time, so the scratch stays bounded.
+// ---------------------------------------------------------------------------
+constexpr size_t kConvChunkBudget = 1ull << 30;  // bytes of im2col operands per chunk
+
+struct ConvPlan {
+    ConvGeom g;
+    int K, kpad, npos, chunk, nchunks;
+};
+
+int conv_plan(int B, int H, int W, int C, int k, int stride, int pad, int Mp, bool two, ConvPlan *pl) {
+    if (B < 1 || H < 1 || W < 1 || C < 1 || k < 1 || stride < 1 || pad < 0 || pad >= k) return DSTD_E_INVALID;
+    const int Ho = (H + 2 * pad - k) / stride + 1, Wo = (W + 2 * pad - k) / stride + 1;
+    if (Ho < 1 || Wo < 1) return DSTD_E_INVALID;
+    const long long K = (long long)k * k * C;
+    const long long npos = (long long)B * Ho * Wo;
+    if (K > 65535 || npos * Mp > (1ll << 31) - 1 || B > 65535) return DSTD_E_UNSUPPORTED;
+    pl->g = ConvGeom{B, H, W, C, Ho, Wo, k, stride, pad};
+    pl->K = (int)K;
+    pl->kpad = pad8((int)K);
+    pl->npos = (int)npos;
+    const long long img = (long long)Ho * Wo;
+    const long long per_img = img * Mp * (long long)pl->kpad * 2 * (two ? 2 : 1);
+    long long imgs = (long long)(kConvChunkBudget / (size_t)(per_img > 0 ? per_img : 1));
+    if (imgs < 1) imgs = 1;
+    if (imgs > B) imgs = B;
+    pl->chunk = (int)(imgs * img);
+    pl->nchunks = (int)((npos + pl->chunk - 1) / pl->chunk);
+    return DSTD_OK;
+}
+
+struct ConvFwdWs {
+    uint16_t *w_hi = nullptr, *w_lo = nullptr, *s_hi = nullptr, *s_lo = nullptr;
+    float *rowsum = nullptr, *row_scale = nullptr;
+    size_t bytes = 0;
+};
+
+ConvFwdWs conv_fwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKind op) {
+    ConvFwdWs w;
+    Bump b(base);
+    const bool two = two_part(op);
+    w.rowsum = b.take<float>(Cout);
+    w.row_scale = b.take<float>(Cout);
+    w.w_hi = b.take<uint16_t>((size_t)Cout * pl.kpad);
+    if (two) w.w_lo = b.take<uint16_t>((size_t)Cout * pl.kpad);
+    w.s_hi = b.take<uint16_t>((size_t)pl.chunk * Mp * pl.kpad);
+    if (two) w.s_lo = b.take<uint16_t>((size_t)pl.chunk * Mp * pl.kpad);
+    w.bytes = b.off;
+    return w;
+}
+
+struct ConvBwdWs {
+    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *dB_hi = nullptr,
+                  *dB_lo = nullptr, *sT_hi = nullptr, *sT_lo = nullptr;
+    float *part = nullptr, *count = nullptr;
+    int ldt = 0, ldn = 0, ldbm = 0, ldp = 0, splits = 1;
+    size_t bytes = 0;
+};
+
+ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKind op, bool need_gt) {
+    ConvBwdWs w;
+    Bump b(base);
+    const bool two = two_part(op);
+    const long long cols = (long long)pl.chunk * Mp;
+    w.ldt = pad8(Cout);
+    w.ldn = pad8(Cout);
+    w.ldbm = pad8((int)cols);
+    w.ldp = (pl.K + 3) & ~3;
+    w.splits = dw_splits(pl.K, Cout, (int)cols, op);
+    w.count = b.take<float>(Cout);
+    w.part = b.take<float>((size_t)w.splits * Cout * w.ldp);
+    w.dA_hi = b.take<__nv_bfloat16>((size_t)Cout * w.ldbm);
+    if (two) w.dA_lo = b.take<__nv_bfloat16>((size_t)Cout * w.ldbm);
+    w.dB_hi = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
+    if (two) w.dB_lo = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
+    w.sT_hi = b.take<__nv_bfloat16>((size_t)pl.K * w.ldbm);
+    if (two) w.sT_lo = b.take<__nv_bfloat16>((size_t)pl.K * w.ldbm);
+    if (need_gt) {
+        w.wt_hi = b.take<__nv_bfloat16>((size_t)pl.K * w.ldt);
+        if (two) w.wt_lo = b.take<__nv_bfloat16>((size_t)pl.K * w.ldt);
+    }
+    w.bytes = b.off;
+    return w;
+}
+
 }  // namespace
 
 extern "C" {
@@ -550,6 +637,147 @@ int dstd_adamw(float *w, const float *g, float *m, float *v, int64_t n, float lr
     TRY(device_ok());
     Timed tm(KK_ADAMW, (cudaStream_t)stream);
     return cu(launch_adamw(w, g, m, v, n, lr, beta1, beta2, eps, weight_decay, step, (cudaStream_t)stream));
+}
+
+size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k, int stride, int pad,
+                                 const dstd_params *p, dstd_math math) {
+    if (check_params(p) != DSTD_OK || C_out < 1) return 0;
+    const int Mp = padded_M(p->M);
+    if (math == DSTD_MATH_F32 || check_math(math, Mp) != DSTD_OK) return 0;
+    ConvPlan pl;
+    if (conv_plan(B, H, W, C_in, k, stride, pad, Mp, true, &pl) != DSTD_OK) return 0;
+    size_t f = conv_fwd_layout(nullptr, pl, C_out, Mp, op_of(math)).bytes;
+    size_t g = conv_bwd_layout(nullptr, pl, C_out, Mp, bwd_op_of(math), true).bytes;
+    return f > g ? f : g;
+}
+
+int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C_in, int C_out, int k, int stride,
+                  int pad, const dstd_params *p, dstd_math math, float *t_out, void *saved, float *penalty,
+                  void *workspace, size_t ws_bytes, dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved || !workspace || C_out < 1) return DSTD_E_INVALID;
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    if (math == DSTD_MATH_F32) return DSTD_E_UNSUPPORTED;
+    TRY(check_math(math, Mp));
+    if (C_out > (1 << 20)) return DSTD_E_UNSUPPORTED;
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    ConvPlan pl;
+    TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, &pl));
+    const OpKind op = op_of(math);
+    if (ws_bytes < conv_fwd_layout(nullptr, pl, C_out, Mp, op).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    ConvFwdWs ws = conv_fwd_layout(workspace, pl, C_out, Mp, op);
+    Saved sv = saved_view(saved, pl.npos, C_out);
+    if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
+    {
+        Timed tm(KK_PREP, st);
+        if (op == OpKind::F16X3)
+            TRY(cu(launch_prep_weights_f16(W, C_out, pl.K, (__half *)ws.w_hi, (__half *)ws.w_lo, pl.kpad,
+                                           ws.row_scale, ws.rowsum, st)));
+        else
+            TRY(cu(launch_prep_weights(W, C_out, pl.K, op, (__nv_bfloat16 *)ws.w_hi, (__nv_bfloat16 *)ws.w_lo,
+                                       pl.kpad, nullptr, nullptr, 0, nullptr, 0, ws.rowsum, st)));
+    }
+    for (int ch = 0; ch < pl.nchunks; ++ch) {
+        const int pos0 = ch * pl.chunk;
+        const int npos = (pl.npos - pos0) < pl.chunk ? (pl.npos - pos0) : pl.chunk;
+        {
+            Timed tm(KK_BIN, st);
+            TRY(cu(launch_binning_im2col(t_in, pl.g, pos0, npos, c, op, false, ws.s_hi, ws.s_lo, pl.kpad, st)));
+        }
+        TcEpiArgs a{};
+        a.c = c;
+        a.B = npos;
+        a.N = C_out;
+        a.row_scale = op == OpKind::F16X3 ? ws.row_scale : nullptr;
+        a.rowsum = ws.rowsum;
+        const long long off = (long long)pos0 * C_out;
+        a.t_out = t_out + off;
+        a.q = sv.q + off;
+        a.s = sv.s + off;
+        a.vdot = sv.vdot + off;
+        a.penalty = penalty;
+        Timed tm(KK_GEMM_FWD, st);
+        TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, pl.kpad, ws.s_hi, ws.s_lo, pl.kpad, C_out, npos * Mp, pl.K, 1, op,
+                              Epi::Scan, a, st)));
+    }
+    return DSTD_OK;
+}
+
+int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const void *saved, const float *g_t_out,
+                  int B, int H, int Wd, int C_in, int C_out, int k, int stride, int pad, const dstd_params *p,
+                  dstd_math math, float *g_t_in, float *g_W, void *workspace, size_t ws_bytes,
+                  dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved || !g_W || !workspace || C_out < 1) return DSTD_E_INVALID;
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    if (math == DSTD_MATH_F32) return DSTD_E_UNSUPPORTED;
+    TRY(check_math(math, Mp));
+    if (C_out > (1 << 20)) return DSTD_E_UNSUPPORTED;
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    ConvPlan pl;
+    TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, &pl));
+    const OpKind bop = bwd_op_of(math);
+    const bool need_gt = g_t_in != nullptr;
+    if (ws_bytes < conv_bwd_layout(nullptr, pl, C_out, Mp, bop, need_gt).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    ConvBwdWs ws = conv_bwd_layout(workspace, pl, C_out, Mp, bop, need_gt);
+    Saved sv = saved_view(const_cast<void *>(saved), pl.npos, C_out);
+    const float qcoef = -p->gamma_q * p->penalty_norm;
+    if (need_gt) {
+        TRY(cu(cudaMemsetAsync(g_t_in, 0, sizeof(float) * (size_t)B * H * Wd * C_in, st)));
+        Timed tm(KK_PREP, st);
+        TRY(cu(launch_prep_weights(W, C_out, pl.K, bop, nullptr, nullptr, 0, ws.wt_hi, ws.wt_lo, ws.ldt, nullptr, 0,
+                                   nullptr, st)));
+    }
+    for (int ch = 0; ch < pl.nchunks; ++ch) {
+        const int pos0 = ch * pl.chunk;
+        const int npos = (pl.npos - pos0) < pl.chunk ? (pl.npos - pos0) : pl.chunk;
+        const long long off = (long long)pos0 * C_out;
+        const long long cols = (long long)npos * Mp;
+        const bool last = (ch == pl.nchunks - 1);
+        {
+            Timed tm(KK_DWHAT, st);
+            TRY(cu(launch_dwhat(t_out + off, sv.q + off, sv.s + off, sv.vdot + off, g_t_out ? g_t_out + off : nullptr,
+                                npos, C_out, c, bop, ws.dA_hi, ws.dA_lo, ws.ldbm, ws.dB_hi, ws.dB_lo, ws.ldn,
+                                ws.count, st, ch > 0)));
+        }
+        if (need_gt) {
+            TcEpiArgs a{};
+            a.c = c;
+            a.B = npos;
+            a.N = pl.K;
+            a.t_in = t_in;
+            a.g_t_in = g_t_in;
+            a.conv = 1;
+            a.pos0 = pos0;
+            a.g = pl.g;
+            Timed tm(KK_GEMM_DS, st);
+            TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dB_hi, ws.dB_lo, ws.ldn, pl.K, (int)cols, C_out, 1,
+                                  bop, Epi::GradT, a, st)));
+        }
+        {
+            Timed tm(KK_BIN_T, st);
+            TRY(cu(launch_binning_im2col(t_in, pl.g, pos0, npos, c, bop, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st)));
+        }
+        TcEpiArgs a{};
+        a.D = ws.part;
+        a.ldd = ws.ldp;
+        a.zstride = (long long)C_out * ws.ldp;
+        {
+            Timed tm(KK_GEMM_DW, st);
+            TRY(cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, C_out, pl.K, (int)cols,
+                                  ws.splits, bop, Epi::Store, a, st)));
+        }
+        Timed tm(KK_REDUCE, st);
+        TRY(cu(launch_dw_reduce(ws.part, ws.splits, a.zstride, ws.ldp, C_out, pl.K, last ? ws.count : nullptr, qcoef,
+                                g_W, st, ch > 0)));
+    }
+    return DSTD_OK;
 }
 
 int dstd_timing_enable(int on) {

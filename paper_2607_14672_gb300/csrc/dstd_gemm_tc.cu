@@ -353,11 +353,25 @@ __device__ __forceinline__ void epi_gradt_sub(uint32_t tbase, int n_main, bool c
             const int col = col0 + cc + sb;
             const int m0 = col & (Mp - 1);
             const int b = col / Mp;
+            long long e = -1;  // input element this (row, sample) reads; -1 = none
+            if (row < a.N && b < a.B) {
+                if (!a.conv) {
+                    e = (long long)b * a.N + row;
+                } else {
+                    const ConvGeom &geo = a.g;
+                    const int pos = a.pos0 + b;
+                    const int cch = row % geo.C, kw = (row / geo.C) % geo.k, kh = row / (geo.C * geo.k);
+                    const int x = pos % geo.Wo, y = (pos / geo.Wo) % geo.Ho, bb = pos / (geo.Wo * geo.Ho);
+                    const int iy = y * geo.s + kh - geo.p, ix = x * geo.s + kw - geo.p;
+                    if (iy >= 0 && iy < geo.H && ix >= 0 && ix < geo.W)
+                        e = (((long long)bb * geo.H + iy) * geo.W + ix) * geo.C + cch;
+                }
+            }
             if (m0 == 0) {
                 g = 0.f;
                 w.k = -100;
-                if (row < a.N && b < a.B) {
-                    const float x = a.t_in[(long long)b * a.N + row];
+                if (e >= 0) {
+                    const float x = a.t_in[e];
                     if (isfinite(x)) w = bin_weights(c, x, true);
                 }
             }
@@ -368,7 +382,10 @@ __device__ __forceinline__ void epi_gradt_sub(uint32_t tbase, int n_main, bool c
                 g += (m == w.k && m < c.M) ? v[sb + j] * w.dR : 0.f;
                 g += (m == w.k + 1 && m < c.M) ? v[sb + j] * w.dL : 0.f;
             }
-            if (m0 + SUB == Mp && row < a.N && b < a.B) a.g_t_in[(long long)b * a.N + row] = g;
+            if (m0 + SUB == Mp && e >= 0) {
+                if (a.conv) atomicAdd(&a.g_t_in[e], g);
+                else a.g_t_in[e] = g;
+            }
         }
     }
 }

@@ -224,6 +224,18 @@ cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bf
 // as bf16 hi/lo (BF16X3), bf16 hi (BF16) or fp32 (F32). Pad entries are 0.
 cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKind op, bool transposed,
                            void *hi, void *lo, int ld, cudaStream_t st);
+// Convolution geometry: input [B, H, W, C] (NHWC), filter k x k, stride s,
+// zero-spike padding p, output [B, Ho, Wo, Cout]. An output position
+// pos = (b*Ho + y)*Wo + x plays the role of a sample; the contraction axis is
+// kidx = (kh*k + kw)*C + c (filter layout [Cout, k, k, C]).
+struct ConvGeom {
+    int B, H, W, C, Ho, Wo, k, s, p;
+};
+// im2col binning of positions [pos0, pos0 + npos): the grid weights of the
+// input spike under each filter tap. !transposed: [npos*Mp, ld] (row (pos, m),
+// column kidx); transposed: [K, ld] (row kidx, column (pos, m)).
+cudaError_t launch_binning_im2col(const float *t, const ConvGeom &g, int pos0, int npos, const LifConst &c,
+                                  OpKind op, bool transposed, void *hi, void *lo, int ld, cudaStream_t st);
 // public-layout binning: s, ds [B, M, N] fp32
 cudaError_t launch_binning_public(const float *t, int B, int N, const LifConst &c, float *s, float *ds,
                                   cudaStream_t st);
@@ -233,15 +245,17 @@ cudaError_t launch_scan_solve(const float *what, long long sb, long long si, int
                               cudaStream_t st);
 // dw^ from saved state; writes [B*Mp, ldn] (row (b,m), col i) and [N, ldbm]
 // (row i, col (b,m)) in the operand format; silent counts per neuron.
+// (silent_count is zeroed first unless accumulate_count)
 cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                          int B, int N, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda,
-                         void *b_hi, void *b_lo, int ldb, float *silent_count, cudaStream_t st);
+                         void *b_hi, void *b_lo, int ldb, float *silent_count, cudaStream_t st,
+                         bool accumulate_count = false);
 // g_t_in from dS stored as D[j, (b,m)] (row stride ldd)
 cudaError_t launch_gt_from_ds(const float *D, long long ldd, const float *t_in, int B, int N, const LifConst &c,
                               float *g_t_in, cudaStream_t st);
-// g_W[i, j] = sum_z part[z][i, j] - g_q*norm*count[i]
+// g_W[i, j] (+)= sum_z part[z][i, j] + qcoef*count[i] (count may be null)
 cudaError_t launch_dw_reduce(const float *part, int splits, long long zstride, int ldp, int R, int C,
-                             const float *count, float qcoef, float *g_W, cudaStream_t st);
+                             const float *count, float qcoef, float *g_W, cudaStream_t st, bool accumulate = false);
 // copy internal w^ D[i, (b, m)] (ld) -> public [B, N, M]
 cudaError_t launch_what_to_public(const float *D, long long ld, int B, int N, int M, int Mp, float *out,
                                   cudaStream_t st);
@@ -260,8 +274,11 @@ struct TcEpiArgs {
     float *D; long long ldd; long long zstride;
     // Scan (rows = neurons i, columns = (b, m))
     LifConst c; int B; int N; const float *rowsum; float *t_out; int *q; float *s; float *vdot; float *penalty;
-    // GradT (rows = inputs j, columns = (b, m))
+    // GradT (rows = inputs j, columns = (b, m)); with conv != 0 the rows are
+    // filter taps kidx, the columns (output position, m), and each result is
+    // added atomically into the input element the tap reads (col2im)
     const float *t_in; float *g_t_in;
+    int conv; int pos0; ConvGeom g;
 };
 // A, B: 16-bit operands (bf16 for BF16X3 / BF16, fp16 for F16X3)
 cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo, int ldb,

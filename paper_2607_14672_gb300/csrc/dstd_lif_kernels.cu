@@ -272,6 +272,107 @@ cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKi
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// im2col binning for convolutions: the grid weights of the input spike that
+// filter tap kidx = (kh*k + kw)*C + c reads at output position pos
+// (out-of-image taps read a silent input, i.e. zero weights).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float im2col_time(const float *__restrict__ t, const ConvGeom &g, int pos, int kidx) {
+    const int c = kidx % g.C;
+    const int kw = (kidx / g.C) % g.k;
+    const int kh = kidx / (g.C * g.k);
+    const int x = pos % g.Wo;
+    const int y = (pos / g.Wo) % g.Ho;
+    const int b = pos / (g.Wo * g.Ho);
+    const int iy = y * g.s + kh - g.p, ix = x * g.s + kw - g.p;
+    if (iy < 0 || iy >= g.H || ix < 0 || ix >= g.W) return INFINITY;
+    return t[(((long long)b * g.H + iy) * g.W + ix) * g.C + c];
+}
+
+template <int OP>
+__global__ void k_binning_im2col_rows(const float *__restrict__ t, ConvGeom g, int pos0, int npos, LifConst c,
+                                      void *hi, void *lo, int ld) {
+    const int K = g.k * g.k * g.C;
+    const int j0 = 2 * (blockIdx.x * blockDim.x + threadIdx.x);
+    if (j0 >= ld) return;
+    for (int pl = blockIdx.y; pl < npos; pl += gridDim.y) {
+        BinW w0{-100, 0.f, 0.f, 0.f, 0.f}, w1{-100, 0.f, 0.f, 0.f, 0.f};
+        if (j0 < K) {
+            float x = im2col_time(t, g, pos0 + pl, j0);
+            if (isfinite(x)) w0 = bin_weights(c, x, false);
+        }
+        if (j0 + 1 < K) {
+            float x = im2col_time(t, g, pos0 + pl, j0 + 1);
+            if (isfinite(x)) w1 = bin_weights(c, x, false);
+        }
+        for (int m = 0; m < c.Mp; ++m) {
+            float v0 = 0.f, v1 = 0.f;
+            if (m < c.M) {
+                v0 = (m == w0.k) ? w0.wR : ((m == w0.k + 1) ? w0.wL : 0.f);
+                v1 = (m == w1.k) ? w1.wR : ((m == w1.k + 1) ? w1.wL : 0.f);
+            }
+            long long off = ((long long)pl * c.Mp + m) * ld + j0;
+            if (OP == 3) {
+                __half h0, l0, h1, l1;
+                split_f16(v0, h0, l0);
+                split_f16(v1, h1, l1);
+                *reinterpret_cast<__half2 *>((__half *)hi + off) = __halves2half2(h0, h1);
+                *reinterpret_cast<__half2 *>((__half *)lo + off) = __halves2half2(l0, l1);
+            } else {
+                __nv_bfloat16 h0, l0, h1, l1;
+                split_bf16(v0, h0, l0);
+                split_bf16(v1, h1, l1);
+                *reinterpret_cast<__nv_bfloat162 *>((__nv_bfloat16 *)hi + off) = __halves2bfloat162(h0, h1);
+                if (OP == 1)
+                    *reinterpret_cast<__nv_bfloat162 *>((__nv_bfloat16 *)lo + off) = __halves2bfloat162(l0, l1);
+            }
+        }
+    }
+}
+
+template <int OP>
+__global__ void k_binning_im2col_cols(const float *__restrict__ t, ConvGeom g, int pos0, int npos, LifConst c,
+                                      void *hi, void *lo, int ld) {
+    const int K = g.k * g.k * g.C;
+    const int pl = blockIdx.x * blockDim.x + threadIdx.x;
+    if (pl >= npos) return;
+    for (int kidx = blockIdx.y; kidx < K; kidx += gridDim.y) {
+        BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+        float x = im2col_time(t, g, pos0 + pl, kidx);
+        if (isfinite(x)) w = bin_weights(c, x, false);
+        const long long base = (long long)kidx * ld + (long long)pl * c.Mp;
+        for (int m0 = 0; m0 < c.Mp; m0 += 8) {
+            __align__(16) __nv_bfloat16 h[8], l[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                int m = m0 + u;
+                float v = (m < c.M) ? ((m == w.k) ? w.wR : ((m == w.k + 1) ? w.wL : 0.f)) : 0.f;
+                split_bf16(v, h[u], l[u]);
+            }
+            *reinterpret_cast<uint4 *>((__nv_bfloat16 *)hi + base + m0) = *reinterpret_cast<uint4 *>(h);
+            if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)lo + base + m0) = *reinterpret_cast<uint4 *>(l);
+        }
+    }
+}
+
+cudaError_t launch_binning_im2col(const float *t, const ConvGeom &g, int pos0, int npos, const LifConst &c,
+                                  OpKind op, bool transposed, void *hi, void *lo, int ld, cudaStream_t st) {
+    const int K = g.k * g.k * g.C;
+    if (!transposed) {
+        dim3 grid(blocks_for((ld + 1) / 2, 128), npos < 65535 ? npos : 65535);
+        if (op == OpKind::F16X3) k_binning_im2col_rows<3><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, hi, lo, ld);
+        else if (op == OpKind::BF16X3) k_binning_im2col_rows<1><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, hi, lo, ld);
+        else if (op == OpKind::BF16) k_binning_im2col_rows<2><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, hi, lo, ld);
+        else return cudaErrorInvalidValue;
+    } else {
+        dim3 grid(blocks_for(npos, 128), K < 65535 ? K : 65535);
+        if (op == OpKind::BF16X3) k_binning_im2col_cols<1><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, hi, lo, ld);
+        else if (op == OpKind::BF16) k_binning_im2col_cols<2><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, hi, lo, ld);
+        else return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
 __global__ void k_binning_public(const float *__restrict__ t, int B, int N, LifConst c, float *s, float *ds) {
     long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)B * N) return;
@@ -418,8 +519,8 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
 
 cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                          int B, int N, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda, void *b_hi,
-                         void *b_lo, int ldb, float *silent_count, cudaStream_t st) {
-    if (silent_count) {
+                         void *b_lo, int ldb, float *silent_count, cudaStream_t st, bool accumulate_count) {
+    if (silent_count && !accumulate_count) {
         cudaError_t e = cudaMemsetAsync(silent_count, 0, sizeof(float) * N, st);
         if (e != cudaSuccess) return e;
     }
@@ -461,20 +562,21 @@ cudaError_t launch_gt_from_ds(const float *D, long long ldd, const float *t_in, 
 }
 
 __global__ void k_dw_reduce(const float *__restrict__ part, int splits, long long zstride, int ldp, int R, int C,
-                            const float *__restrict__ count, float qcoef, float *g_W) {
+                            const float *__restrict__ count, float qcoef, float *g_W, int accumulate) {
     long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)R * C) return;
     int i = (int)(idx / C), j = (int)(idx % C);
     float s = 0.f;
     for (int z = 0; z < splits; ++z) s += part[z * zstride + (long long)i * ldp + j];
     if (count) s += qcoef * count[i];
-    g_W[idx] = s;
+    g_W[idx] = accumulate ? g_W[idx] + s : s;
 }
 
 cudaError_t launch_dw_reduce(const float *part, int splits, long long zstride, int ldp, int R, int C,
-                             const float *count, float qcoef, float *g_W, cudaStream_t st) {
+                             const float *count, float qcoef, float *g_W, cudaStream_t st, bool accumulate) {
     long long n = (long long)R * C;
-    k_dw_reduce<<<blocks_for(n, 256), 256, 0, st>>>(part, splits, zstride, ldp, R, C, count, qcoef, g_W);
+    k_dw_reduce<<<blocks_for(n, 256), 256, 0, st>>>(part, splits, zstride, ldp, R, C, count, qcoef, g_W,
+                                                    accumulate ? 1 : 0);
     return cudaGetLastError();
 }
 

@@ -22,7 +22,7 @@ EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning
            "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
            "dstd_adamw", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
-           "dstd_dense_fwd_noalloc")
+           "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd")
 
 
 class DstdError(RuntimeError):
@@ -87,6 +87,9 @@ def load(path=None):
         "dstd_kernel_kind_name": (ctypes.c_char_p, [_I]),
         "dstd_selftest_wait_timeout": (_I, [ctypes.c_uint32, _P]),
         "dstd_dense_fwd_noalloc": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _P]),
+        "dstd_conv_workspace_bytes": (_SZ, [_I, _I, _I, _I, _I, _I, _I, _I, _PP, _I]),
+        "dstd_conv_fwd": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _P, _SZ, _P]),
+        "dstd_conv_bwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -205,6 +208,41 @@ def dense_bwd(t_in, W, t_out, saved, g_t_out, p, math_mode, g_t_in, g_W, workspa
     _check(load().dstd_dense_bwd(_ptr(t_in), _ptr(W), _ptr(t_out), _ptr(saved), _ptr(g_t_out), B, N_in, N_out,
                                  ctypes.byref(p), MATH[math_mode], _ptr(g_t_in), _ptr(g_W), _ptr(workspace),
                                  workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_dense_bwd")
+
+
+def conv_out_hw(H, W, k, stride, pad):
+    return (H + 2 * pad - k) // stride + 1, (W + 2 * pad - k) // stride + 1
+
+
+def conv_workspace_bytes(B, H, W, C_in, C_out, k, stride, pad, p, math_mode):
+    return load().dstd_conv_workspace_bytes(B, H, W, C_in, C_out, k, stride, pad, ctypes.byref(p), MATH[math_mode])
+
+
+def conv_fwd(t_in, W, stride, pad, p, math_mode, t_out, saved, penalty, workspace, stream=None):
+    """t_in [B, H, W, C_in] NHWC, W [C_out, k, k, C_in] -> t_out [B, Ho, Wo, C_out]."""
+    B, H, Wd, C = t_in.shape
+    C_out, k = W.shape[0], W.shape[1]
+    Ho, Wo = conv_out_hw(H, Wd, k, stride, pad)
+    _f32(t_in, "t_in")
+    _f32(W, "W", (C_out, k, k, C))
+    _f32(t_out, "t_out", (B, Ho, Wo, C_out))
+    _check(load().dstd_conv_fwd(_ptr(t_in), _ptr(W), B, H, Wd, C, C_out, k, stride, pad, ctypes.byref(p),
+                                MATH[math_mode], _ptr(t_out), _ptr(saved), _ptr(penalty), _ptr(workspace),
+                                workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_conv_fwd")
+
+
+def conv_bwd(t_in, W, t_out, saved, g_t_out, stride, pad, p, math_mode, g_t_in, g_W, workspace, stream=None):
+    B, H, Wd, C = t_in.shape
+    C_out, k = W.shape[0], W.shape[1]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (C_out, k, k, C))
+    _f32(g_W, "g_W", (C_out, k, k, C))
+    if g_t_in is not None:
+        _f32(g_t_in, "g_t_in", (B, H, Wd, C))
+    _check(load().dstd_conv_bwd(_ptr(t_in), _ptr(W), _ptr(t_out), _ptr(saved), _ptr(g_t_out), B, H, Wd, C, C_out, k,
+                                stride, pad, ctypes.byref(p), MATH[math_mode], _ptr(g_t_in), _ptr(g_W),
+                                _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
+           "dstd_conv_bwd")
 
 
 def ce_loss(t_L, labels, tau_soft, t_silent, loss, g_t_L, stream=None):

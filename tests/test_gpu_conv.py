@@ -1,0 +1,140 @@
+"""GPU parity of the convolutional DSTD layer against the float64 oracle.
+
+The oracle's conv layer works channel-major (t [B, C, H, W], W [O, C, k, k]);
+the library works NHWC (t [B, H, W, C], W [O, k, k, C]); the tests transpose.
+Tolerances as for dense layers: |dt| <= 1e-4 T_max with masks identical
+outside the 1e-5 near-threshold band, gradients to 1e-3 relative L2.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from helpers import f32, rel_l2
+from oracle import dstd as odstd, losses as olosses, network as onet
+
+pytestmark = pytest.mark.gpu
+
+INF = math.inf
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    from paper_2607_14672_gb300 import build, dstd
+    build.build()
+    dstd.load()
+    assert dstd.device_status(clear=True) == 0
+    yield
+    assert dstd.device_status(clear=True) == 0
+
+
+def dev(x):
+    return torch.tensor(np.ascontiguousarray(x), dtype=torch.float32, device="cuda")
+
+
+def host(x):
+    return x.detach().cpu().numpy().astype(np.float64)
+
+
+def conv_case(B, C, H, O, k, stride, pad, M, tau, seed, wmean, gammas=(0.0, 0.0, 0.0), silent=0.3):
+    g = np.random.default_rng(seed)
+    t = f32(np.where(g.random((B, C, H, H)) < silent, INF, g.uniform(0, 1, (B, C, H, H))))
+    W = f32(g.normal(wmean, 1.0 / math.sqrt(C * k * k), (O, C, k, k)))
+    L = dict(kind="conv", W=W, tau_v=tau[0], tau_I=tau[1], v_th=1.0, t_first=0.0, t_end=1.2, M=M, t_offset=0.011,
+             stride=stride, pad=pad, t_head_l=0.35, t_tail_l=0.8, gamma_head=gammas[0], gamma_tail=gammas[1],
+             gamma_q=gammas[2])
+    return t, L
+
+
+def run_conv_fwd(t, L, math_mode="x3"):
+    from paper_2607_14672_gb300 import dstd
+    B, C, H, Wd = t.shape
+    O, _, k, _ = L["W"].shape
+    Ho, Wo = dstd.conv_out_hw(H, Wd, k, L["stride"], L["pad"])
+    p = dstd.params(L, 1.0 / (B * Ho * Wo))
+    ws = torch.empty(dstd.conv_workspace_bytes(B, H, Wd, C, O, k, L["stride"], L["pad"], p, math_mode),
+                     dtype=torch.uint8, device="cuda")
+    t_in = dev(t.transpose(0, 2, 3, 1))
+    Wg = dev(L["W"].transpose(0, 2, 3, 1))
+    t_out = torch.empty(B, Ho, Wo, O, device="cuda")
+    saved = torch.empty(dstd.dense_saved_bytes(B * Ho * Wo, O), dtype=torch.uint8, device="cuda")
+    pen = torch.empty(4, device="cuda")
+    dstd.conv_fwd(t_in, Wg, L["stride"], L["pad"], p, math_mode, t_out, saved, pen, ws)
+    torch.cuda.synchronize()
+    return dict(t=host(t_out).transpose(0, 3, 1, 2), t_in=t_in, W=Wg, t_out=t_out, saved=saved, pen=host(pen), p=p,
+                ws=ws)
+
+
+def check(t_gpu, ctx, L):
+    ok = np.abs(ctx["vpeak"] - L["v_th"]) > 1e-5
+    fo, fg = np.isfinite(ctx["t"]), np.isfinite(t_gpu)
+    assert not (ok & (fo != fg)).any()
+    both = ok & fo & fg
+    assert both.sum() > 0.2 * t_gpu.size
+    assert np.abs(t_gpu[both] - ctx["t"][both]).max() <= 1e-4 * (L["t_end"] - L["t_first"])
+    return ok
+
+
+# weight means giving about 60% firing with 64 input channels (scaled by 64/C)
+WMEAN64 = {(0.5, 0.25): 0.035, (INF, INF): 0.0052, (1.0, 0.25): 0.024}
+
+
+@pytest.mark.parametrize("tau", [(0.5, 0.25), (INF, INF), (1.0, 0.25)])
+@pytest.mark.parametrize("C,H,O,stride", [(64, 8, 48, 1), (64, 9, 64, 2), (3, 12, 64, 1), (128, 6, 130, 1)])
+def test_conv_forward_matches_oracle(tau, C, H, O, stride):
+    t, L = conv_case(2, C, H, O, 3, stride, 1, 32, tau, seed=C + H, wmean=WMEAN64[tau] * 64 / C)
+    r = run_conv_fwd(t, L)
+    ctx = onet.forward_layer(t, L)
+    check(r["t"], ctx, L)
+
+
+def test_conv_backward_matches_oracle():
+    from paper_2607_14672_gb300 import dstd
+    t, L = conv_case(2, 64, 8, 48, 3, 1, 1, 32, (0.5, 0.25), seed=3, wmean=0.035, gammas=(0.05, 0.01, 1e-3))
+    r = run_conv_fwd(t, L)
+    ctx = onet.forward_layer(t, L)
+    ok = check(r["t"], ctx, L)
+    B, O, Ho, Wo = ctx["t"].shape
+    nrm = 1.0 / (B * Ho * Wo)
+    g = np.random.default_rng(4).normal(0.0, 1.0, ctx["t"].shape)
+    ill = ~ok
+    tg = r["t"]
+    _, pg = olosses.temporal_penalty(tg, 0.35, 0.8, 0.05, 0.01, nrm)
+    _, gT = olosses.temporal_penalty(ctx["t"], 0.35, 0.8, 0.05, 0.01, nrm)
+    g_gpu = np.where(ill, -pg, g)
+    g_ora = np.where(ill, 0.0, g + gT)
+    g_t_in = torch.empty_like(r["t_in"])
+    g_W = torch.empty_like(r["W"])
+    dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g_gpu.transpose(0, 2, 3, 1)), 1, 1, r["p"], "x3",
+                  g_t_in, g_W, r["ws"])
+    torch.cuda.synchronize()
+    gW, gin = onet.backward_layer(ctx, L, g_ora)
+    cnt = (~np.isfinite(tg)).sum((0, 2, 3))
+    gW = gW - 1e-3 * nrm * cnt[:, None, None, None]
+    assert rel_l2(host(g_W).transpose(0, 3, 1, 2), gW) <= 1e-3
+    assert rel_l2(host(g_t_in).transpose(0, 3, 1, 2), gin) <= 1e-3
+
+
+def test_conv_chunked_matches_unchunked():
+    # 32 images of 32x32x64 at M = 32 exceed one ~1 GiB im2col chunk; the
+    # result must not depend on where the chunks fall.
+    from paper_2607_14672_gb300 import dstd
+    t, L = conv_case(32, 64, 32, 64, 3, 1, 1, 32, (INF, INF), seed=9, wmean=0.0052)
+    full = run_conv_fwd(t, L)
+    parts = [run_conv_fwd(t[i:i + 8], L) for i in range(0, 32, 8)]
+    tp = np.concatenate([q["t"] for q in parts], 0)
+    np.testing.assert_array_equal(np.isfinite(full["t"]), np.isfinite(tp))
+    fin = np.isfinite(tp)
+    assert np.abs(full["t"][fin] - tp[fin]).max() <= 1e-6
+    # weight gradient is a sum over images (no penalty terms here)
+    g = np.where(np.isfinite(full["t"]), 1.0, 0.0)
+    gWs = []
+    for r, sl in [(full, slice(0, 32))] + [(q, slice(i, i + 8)) for q, i in zip(parts, range(0, 32, 8))]:
+        g_W = torch.empty_like(r["W"])
+        dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g[sl].transpose(0, 2, 3, 1)), 1, 1, r["p"],
+                      "x3", None, g_W, r["ws"])
+        torch.cuda.synchronize()
+        gWs.append(host(g_W))
+    assert rel_l2(gWs[0], sum(gWs[1:])) <= 1e-5
