@@ -137,10 +137,10 @@ int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
  * with the same arguments minus the workspace; the caller still provides
  * t_in, W, t_out, saved and penalty. (The paper has no counterpart: this is
  * a deployment convenience of this library.)
- * Scratch: a fixed 32 MiB array in device memory, part of the library's
+ * Scratch: a fixed 64 MiB array in device memory, part of the library's
  * image, present on every GPU that loads the library until the process
  * exits. A call whose scratch need (dstd_dense_workspace_bytes' forward part)
- * exceeds 32 MiB returns DSTD_E_WORKSPACE and launches nothing; the 784-800
+ * exceeds 64 MiB returns DSTD_E_WORKSPACE and launches nothing; the 784-800
  * and 800-800 layers at B = 256, M = 32 fit. No call allocates or frees.
  * Every call uses the same array, which keeps whatever the previous call
  * left there (each call overwrites all the scratch it reads), so two calls

@@ -166,7 +166,7 @@ struct FwdWs {
     uint16_t *w_hi = nullptr, *w_lo = nullptr, *s_hi = nullptr, *s_lo = nullptr;  // 16-bit operands
     float *s32 = nullptr, *D = nullptr, *rowsum = nullptr, *row_scale = nullptr;
     size_t bytes = 0;
-    int kpad = 0;
+    int kpad = 0, ldD = 0;
 };
 
 FwdWs fwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool need_D) {
@@ -184,7 +184,11 @@ FwdWs fwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
         w.s_hi = b.take<uint16_t>((size_t)cols * w.kpad);
         if (two_part(op)) w.s_lo = b.take<uint16_t>((size_t)cols * w.kpad);
         if (op == OpKind::F16X3) w.row_scale = b.take<float>(N_out);
-        if (need_D) w.D = b.take<float>((size_t)N_out * cols);
+        // w^ in fp32: [N_out, B*Mp] for the public copy (need_D), else the
+        // scan's layout [B*Mp, ldD] (row (b, m), column i)
+        w.ldD = (N_out + 3) & ~3;
+        w.D = b.take<float>((size_t)cols * w.ldD);  // >= N_out * cols
+        (void)need_D;
     }
     w.bytes = b.off;
     return w;
@@ -290,8 +294,8 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
         }
         if (!store_D) {
             Timed tm(KK_SCAN, st);
-            TRY(cu(launch_scan_solve(ws.D, c.Mp, cols, B, N_out, c, ws.rowsum, t_out, sv->q, sv->s, sv->vdot,
-                                     penalty, st)));
+            TRY(cu(launch_scan_solve(ws.D, c.Mp, cols, 1, B, N_out, c, nullptr, ws.rowsum, t_out, sv->q, sv->s,
+                                     sv->vdot, penalty, st)));
         }
         return DSTD_OK;
     }
@@ -312,23 +316,28 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
     a.c = c;
     a.B = B;
     a.N = N_out;
-    a.row_scale = ws.row_scale;
-    Timed tm(KK_GEMM_FWD, st);
     if (store_D) {
+        Timed tm(KK_GEMM_FWD, st);
+        a.row_scale = ws.row_scale;
         a.D = ws.D;
         a.ldd = cols;
         a.zstride = 0;
         return cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
                                  Epi::Store, a, st));
     }
-    a.rowsum = ws.rowsum;
-    a.t_out = t_out;
-    a.q = sv->q;
-    a.s = sv->s;
-    a.vdot = sv->vdot;
-    a.penalty = penalty;
-    return cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
-                             Epi::Scan, a, st));
+    // w^ with rows (b, m) and columns i, so that the scan reads the M values
+    // of 32 neurons of a sample as 32-wide coalesced rows
+    {
+        Timed tm(KK_GEMM_FWD, st);
+        a.D = ws.D;
+        a.ldd = ws.ldD;
+        a.zstride = 0;
+        TRY(cu(launch_tc_gemm(ws.s_hi, ws.s_lo, ws.kpad, ws.w_hi, ws.w_lo, ws.kpad, (int)cols, N_out, N_in, 1, op,
+                              Epi::Store, a, st)));
+    }
+    Timed tm(KK_SCAN, st);
+    return cu(launch_scan_solve(ws.D, (long long)c.Mp * ws.ldD, 1, ws.ldD, B, N_out, c, ws.row_scale, ws.rowsum,
+                                t_out, sv->q, sv->s, sv->vdot, penalty, st));
 }
 
 // ---------------------------------------------------------------------------
@@ -343,7 +352,7 @@ struct ConvPlan {
     int K, kpad, npos, chunk, nchunks;
 };
 
-int conv_plan(int B, int H, int W, int C, int k, int stride, int pad, int Mp, bool two, ConvPlan *pl) {
+int conv_plan(int B, int H, int W, int C, int k, int stride, int pad, int Mp, bool two, int Cout, ConvPlan *pl) {
     if (B < 1 || H < 1 || W < 1 || C < 1 || k < 1 || stride < 1 || pad < 0 || pad >= k) return DSTD_E_INVALID;
     const int Ho = (H + 2 * pad - k) / stride + 1, Wo = (W + 2 * pad - k) / stride + 1;
     if (Ho < 1 || Wo < 1) return DSTD_E_INVALID;
@@ -355,7 +364,8 @@ int conv_plan(int B, int H, int W, int C, int k, int stride, int pad, int Mp, bo
     pl->kpad = pad8((int)K);
     pl->npos = (int)npos;
     const long long img = (long long)Ho * Wo;
-    const long long per_img = img * Mp * (long long)pl->kpad * 2 * (two ? 2 : 1);
+    // per image: the im2col operands and the fp32 w^ of its positions
+    const long long per_img = img * Mp * ((long long)pl->kpad * 2 * (two ? 2 : 1) + (long long)((Cout + 3) & ~3) * 4);
     long long imgs = (long long)(kConvChunkBudget / (size_t)(per_img > 0 ? per_img : 1));
     if (imgs < 1) imgs = 1;
     if (imgs > B) imgs = B;
@@ -366,7 +376,8 @@ int conv_plan(int B, int H, int W, int C, int k, int stride, int pad, int Mp, bo
 
 struct ConvFwdWs {
     uint16_t *w_hi = nullptr, *w_lo = nullptr, *s_hi = nullptr, *s_lo = nullptr;
-    float *rowsum = nullptr, *row_scale = nullptr;
+    float *rowsum = nullptr, *row_scale = nullptr, *D = nullptr;
+    int ldD = 0;
     size_t bytes = 0;
 };
 
@@ -380,6 +391,8 @@ ConvFwdWs conv_fwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
     if (two) w.w_lo = b.take<uint16_t>((size_t)Cout * pl.kpad);
     w.s_hi = b.take<uint16_t>((size_t)pl.chunk * Mp * pl.kpad);
     if (two) w.s_lo = b.take<uint16_t>((size_t)pl.chunk * Mp * pl.kpad);
+    w.ldD = (Cout + 3) & ~3;
+    w.D = b.take<float>((size_t)pl.chunk * Mp * w.ldD);  // w^ of a chunk: row (pos, m), column o
     w.bytes = b.off;
     return w;
 }
@@ -496,8 +509,8 @@ int dstd_scan_solve(const float *what, int B, int N_out, const dstd_params *p, c
     if (saved) sv = saved_view(saved, B, N_out);
     if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
     Timed tm(KK_SCAN, st);
-    return cu(launch_scan_solve(what, (long long)N_out * p->M, p->M, B, N_out, c, w_rowsum, t_out, sv.q, sv.s,
-                                sv.vdot, penalty, st));
+    return cu(launch_scan_solve(what, (long long)N_out * p->M, p->M, 1, B, N_out, c, nullptr, w_rowsum, t_out, sv.q,
+                                sv.s, sv.vdot, penalty, st));
 }
 
 int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
@@ -645,7 +658,7 @@ size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k
     const int Mp = padded_M(p->M);
     if (math == DSTD_MATH_F32 || check_math(math, Mp) != DSTD_OK) return 0;
     ConvPlan pl;
-    if (conv_plan(B, H, W, C_in, k, stride, pad, Mp, true, &pl) != DSTD_OK) return 0;
+    if (conv_plan(B, H, W, C_in, k, stride, pad, Mp, true, C_out, &pl) != DSTD_OK) return 0;
     size_t f = conv_fwd_layout(nullptr, pl, C_out, Mp, op_of(math)).bytes;
     size_t g = conv_bwd_layout(nullptr, pl, C_out, Mp, bwd_op_of(math), true).bytes;
     return f > g ? f : g;
@@ -662,7 +675,7 @@ int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C
     if (C_out > (1 << 20)) return DSTD_E_UNSUPPORTED;
     if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
     ConvPlan pl;
-    TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, &pl));
+    TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, C_out, &pl));
     const OpKind op = op_of(math);
     if (ws_bytes < conv_fwd_layout(nullptr, pl, C_out, Mp, op).bytes) return DSTD_E_WORKSPACE;
     TRY(device_ok());
@@ -688,20 +701,19 @@ int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C
             TRY(cu(launch_binning_im2col(t_in, pl.g, pos0, npos, c, op, false, ws.s_hi, ws.s_lo, pl.kpad, st)));
         }
         TcEpiArgs a{};
-        a.c = c;
-        a.B = npos;
-        a.N = C_out;
-        a.row_scale = op == OpKind::F16X3 ? ws.row_scale : nullptr;
-        a.rowsum = ws.rowsum;
+        a.D = ws.D;
+        a.ldd = ws.ldD;
+        a.zstride = 0;
+        {
+            Timed tm(KK_GEMM_FWD, st);
+            TRY(cu(launch_tc_gemm(ws.s_hi, ws.s_lo, pl.kpad, ws.w_hi, ws.w_lo, pl.kpad, npos * Mp, C_out, pl.K, 1, op,
+                                  Epi::Store, a, st)));
+        }
         const long long off = (long long)pos0 * C_out;
-        a.t_out = t_out + off;
-        a.q = sv.q + off;
-        a.s = sv.s + off;
-        a.vdot = sv.vdot + off;
-        a.penalty = penalty;
-        Timed tm(KK_GEMM_FWD, st);
-        TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, pl.kpad, ws.s_hi, ws.s_lo, pl.kpad, C_out, npos * Mp, pl.K, 1, op,
-                              Epi::Scan, a, st)));
+        Timed tr(KK_SCAN, st);
+        TRY(cu(launch_scan_solve(ws.D, (long long)Mp * ws.ldD, 1, ws.ldD, npos, C_out, c,
+                                 op == OpKind::F16X3 ? ws.row_scale : nullptr, ws.rowsum, t_out + off, sv.q + off,
+                                 sv.s + off, sv.vdot + off, penalty, st)));
     }
     return DSTD_OK;
 }
@@ -718,7 +730,7 @@ int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const v
     if (C_out > (1 << 20)) return DSTD_E_UNSUPPORTED;
     if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
     ConvPlan pl;
-    TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, &pl));
+    TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, C_out, &pl));
     const OpKind bop = bwd_op_of(math);
     const bool need_gt = g_t_in != nullptr;
     if (ws_bytes < conv_bwd_layout(nullptr, pl, C_out, Mp, bop, need_gt).bytes) return DSTD_E_WORKSPACE;
@@ -822,9 +834,9 @@ int dstd_selftest_wait_timeout(uint32_t timeout_us, dstd_stream_t stream) {
 
 namespace {
 
-// Fixed scratch for dstd_dense_fwd_noalloc: 32 MiB, resident on every GPU
+// Fixed scratch for dstd_dense_fwd_noalloc: 64 MiB, resident on every GPU
 // that loads this library, for as long as the process runs.
-constexpr size_t kNoAllocScratchBytes = 32ull << 20;
+constexpr size_t kNoAllocScratchBytes = 64ull << 20;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 std::mutex g_noalloc_mu;

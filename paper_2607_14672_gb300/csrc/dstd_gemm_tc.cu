@@ -1,14 +1,12 @@
 // Tensor-core contraction of the DSTD layer on sm_103a (tcgen05 + TMA).
 //
-// D[r, c] = sum_k A[r, k] B[c, k] with A and B bf16, K-major, staged by TMA
+// D[r, c] = sum_k A[r, k] B[c, k] with A and B 16-bit, K-major, staged by TMA
 // (128-byte swizzle, no multicast) through a STAGES-deep mbarrier ring; one
 // thread issues tcgen05.mma (cta_group::1, M = 128, N = BN, K = 16 per
-// instruction) into an fp32 accumulator in TMEM; four warps read it back
-// with tcgen05.ld (lane = row) and run the fused epilogue:
-//   Store  plain fp32 tile (split-K partials of the weight gradient),
-//   Scan   rows = neurons, columns = (sample, grid step): the scan / threshold
-//          solve / first-spike select of Tab. timing_DSTD, so w^ never
-//          reaches HBM,
+// instruction) into fp32 accumulators in TMEM; eight warps read them back
+// with tcgen05.ld (lane = row) and run the epilogue:
+//   Store  plain fp32 tile (w^ of the forward, rows = (sample, grid step),
+//          columns = neurons; split-K partials of the weight gradient),
 //   GradT  rows = inputs, columns = (sample, grid step): the input-time
 //          gradient sum_m dS ds/dt, so dS never reaches HBM.
 // The three-product split (fp32 operand = 16-bit hi + lo) accumulates
@@ -64,16 +62,22 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
                  : "memory");
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// try_wait with a suspend-time hint: the thread parks in hardware until the
+// phase completes or about 1 ms passes, instead of spinning on issue slots
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{\n"
         ".reg .pred p;\n"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
         "selp.u32 %0, 1, 0, p;\n"
         "}\n"
         : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)
         : "memory");
     return ok != 0;
 }
@@ -234,295 +238,279 @@ struct Cfg {
 // ---------------------------------------------------------------------------
 // Epilogues. Each thread owns one accumulator row (its TMEM lane).
 // ---------------------------------------------------------------------------
-// Each warp of the epilogue owns one TMEM lane quarter (warp % 4) and a
-// range of 32-column chunks [c_lo, c_hi) of the tile.
-template <int BN>
-__device__ __forceinline__ void epi_store(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                          int c_hi, int R, int Cn, const TcEpiArgs &a) {
-    float *D = a.D + (long long)blockIdx.z * a.zstride;
-    const float rs = (a.row_scale && row < R) ? a.row_scale[row] : 1.0f;
-#pragma unroll 1
-    for (int cc = c_lo; cc < c_hi; cc += 32) {
-        float v[32];
-        tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
+// ---------------------------------------------------------------------------
+// Epilogues. Each epilogue warp owns one TMEM lane quarter (rows 32q..32q+31)
+// and one column group; a thread owns one accumulator row. The work on a
+// chunk of 32 columns is written against registers, so a tile whose group
+// chunk is a single one can be drained from TMEM first (and TMEM handed back
+// to the MMA warp) before the chunk is processed.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void store_chunk(const float (&v)[32], int row, int col0, int cc, int R, int Cn,
+                                            const TcEpiArgs &a, int split) {
+    if (row >= R) return;
+    float *D = a.D + (long long)split * a.zstride;
+    const float rs = a.row_scale ? a.row_scale[row] : 1.0f;
+    float *dst = D + (long long)row * a.ldd + col0 + cc;
+    if (col0 + cc + 32 <= Cn && (a.ldd % 4) == 0) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] *= rs;
-        if (row < R) {
-            float *dst = D + (long long)row * a.ldd + col0 + cc;
-            if (col0 + cc + 32 <= Cn && (a.ldd % 4) == 0) {
-#pragma unroll
-                for (int j = 0; j < 32; j += 4)
-                    *reinterpret_cast<float4 *>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-            } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (col0 + cc + j < Cn) dst[j] = v[j];
-            }
-        }
-    }
-}
-
-__device__ __forceinline__ float warp_sum_tc(float x) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    return x;
-}
-
-// Output of one neuron of one sample (spike time, saved state, penalty sums).
-__device__ __forceinline__ void scan_emit(const LifConst &c, const ScanState &st, int b, int row,
-                                          const TcEpiArgs &a, float (&acc)[4]) {
-    if (row >= a.N || b >= a.B) return;
-    const long long o = (long long)b * a.N + row;
-    const bool fired = st.q < c.M;
-    const float t = fired ? c.T0 + (float)st.q * c.dt + st.s : INFINITY;
-    a.t_out[o] = t;
-    a.q[o] = st.q;
-    a.s[o] = st.s;
-    a.vdot[o] = st.vdot;
-    if (fired) {
-        float pv, pg;
-        penalty_T(c, t, pv, pg);
-        acc[0] += pv;
-        acc[3] += 1.f;
+        for (int j = 0; j < 32; j += 4)
+            *reinterpret_cast<float4 *>(dst + j) =
+                make_float4(v[j] * rs, v[j + 1] * rs, v[j + 2] * rs, v[j + 3] * rs);
     } else {
-        if (a.rowsum) acc[1] += -c.g_q * c.norm * a.rowsum[row];
-        acc[2] += 1.f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (col0 + cc + j < Cn) dst[j] = v[j] * rs;
     }
 }
 
-// Scan epilogue over chunks of 32 columns; SUB = min(Mp, 32) columns of one
-// sample are scanned per unrolled block, so the sample-end work appears once
-// per block instead of once per column.
-template <int BN, int SUB>
-__device__ __forceinline__ void epi_scan_sub(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                             int c_hi, const TcEpiArgs &a, float (&acc)[4]) {
+// Input-time gradient over one chunk (dense: row = input j; conv: row = tap).
+template <int SUB>
+__device__ __forceinline__ void gradt_chunk(const float (&v)[32], int row, int colbase, BinW &w, float &g,
+                                            const TcEpiArgs &a) {
     const LifConst &c = a.c;
     const int Mp = c.Mp;
-    const float rs = (a.row_scale && row < a.N) ? a.row_scale[row] : 1.0f;
-    ScanState st;
-    scan_reset(st, c.M);
-#pragma unroll 1
-    for (int cc = c_lo; cc < c_hi; cc += 32) {
-        float v[32];
-        tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
 #pragma unroll
-        for (int sb = 0; sb < 32; sb += SUB) {
-            const int col = col0 + cc + sb;          // first column of this block
-            const int m0 = col & (Mp - 1);
-            if (m0 == 0) scan_reset(st, c.M);
-#pragma unroll
-            for (int j = 0; j < SUB; ++j)
-                if (m0 + j < c.M) scan_step(c, st, v[sb + j] * rs, m0 + j);
-            if (m0 + SUB == Mp) {
-                scan_finish(c, st);
-                scan_emit(c, st, col / Mp, row, a, acc);
+    for (int sb = 0; sb < 32; sb += SUB) {
+        const int col = colbase + sb;
+        const int m0 = col & (Mp - 1);
+        const int b = col / Mp;
+        long long e = -1;  // input element this (row, sample) reads; -1 = none
+        if (row < a.N && b < a.B) {
+            if (!a.conv) {
+                e = (long long)b * a.N + row;
+            } else {
+                const ConvGeom &geo = a.g;
+                const int pos = a.pos0 + b;
+                const int cch = row % geo.C, kw = (row / geo.C) % geo.k, kh = row / (geo.C * geo.k);
+                const int x = pos % geo.Wo, y = (pos / geo.Wo) % geo.Ho, bb = pos / (geo.Wo * geo.Ho);
+                const int iy = y * geo.s + kh - geo.p, ix = x * geo.s + kw - geo.p;
+                if (iy >= 0 && iy < geo.H && ix >= 0 && ix < geo.W)
+                    e = (((long long)bb * geo.H + iy) * geo.W + ix) * geo.C + cch;
             }
         }
-    }
-}
-
-template <int BN>
-__device__ __forceinline__ void epi_scan(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                         int c_hi, const TcEpiArgs &a) {
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    if (a.c.Mp == 8) epi_scan_sub<BN, 8>(tbase, n_main, corr, row, col0, c_lo, c_hi, a, acc);
-    else if (a.c.Mp == 16) epi_scan_sub<BN, 16>(tbase, n_main, corr, row, col0, c_lo, c_hi, a, acc);
-    else epi_scan_sub<BN, 32>(tbase, n_main, corr, row, col0, c_lo, c_hi, a, acc);
-    if (a.penalty) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            float s = warp_sum_tc(acc[k]);
-            if ((threadIdx.x & 31) == 0 && s != 0.f) atomicAdd(&a.penalty[k], s);
-        }
-    }
-}
-
-template <int BN, int SUB>
-__device__ __forceinline__ void epi_gradt_sub(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                              int c_hi, const TcEpiArgs &a) {
-    const LifConst &c = a.c;
-    const int Mp = c.Mp;
-    BinW w{-100, 0.f, 0.f, 0.f, 0.f};
-    float g = 0.f;
-#pragma unroll 1
-    for (int cc = c_lo; cc < c_hi; cc += 32) {
-        float v[32];
-        tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
-#pragma unroll
-        for (int sb = 0; sb < 32; sb += SUB) {
-            const int col = col0 + cc + sb;
-            const int m0 = col & (Mp - 1);
-            const int b = col / Mp;
-            long long e = -1;  // input element this (row, sample) reads; -1 = none
-            if (row < a.N && b < a.B) {
-                if (!a.conv) {
-                    e = (long long)b * a.N + row;
-                } else {
-                    const ConvGeom &geo = a.g;
-                    const int pos = a.pos0 + b;
-                    const int cch = row % geo.C, kw = (row / geo.C) % geo.k, kh = row / (geo.C * geo.k);
-                    const int x = pos % geo.Wo, y = (pos / geo.Wo) % geo.Ho, bb = pos / (geo.Wo * geo.Ho);
-                    const int iy = y * geo.s + kh - geo.p, ix = x * geo.s + kw - geo.p;
-                    if (iy >= 0 && iy < geo.H && ix >= 0 && ix < geo.W)
-                        e = (((long long)bb * geo.H + iy) * geo.W + ix) * geo.C + cch;
-                }
-            }
-            if (m0 == 0) {
-                g = 0.f;
-                w.k = -100;
-                if (e >= 0) {
-                    const float x = a.t_in[e];
-                    if (isfinite(x)) w = bin_weights(c, x, true);
-                }
-            }
-            // the two grid points of the spike (m = k, k + 1), if in this block
-#pragma unroll
-            for (int j = 0; j < SUB; ++j) {
-                const int m = m0 + j;
-                g += (m == w.k && m < c.M) ? v[sb + j] * w.dR : 0.f;
-                g += (m == w.k + 1 && m < c.M) ? v[sb + j] * w.dL : 0.f;
-            }
-            if (m0 + SUB == Mp && e >= 0) {
-                if (a.conv) atomicAdd(&a.g_t_in[e], g);
-                else a.g_t_in[e] = g;
+        if (m0 == 0) {
+            g = 0.f;
+            w.k = -100;
+            if (e >= 0) {
+                const float x = a.t_in[e];
+                if (isfinite(x)) w = bin_weights(c, x, true);
             }
         }
+        // the two grid points of the spike (m = k, k + 1), if in this block
+#pragma unroll
+        for (int j = 0; j < SUB; ++j) {
+            const int m = m0 + j;
+            g += (m == w.k && m < c.M) ? v[sb + j] * w.dR : 0.f;
+            g += (m == w.k + 1 && m < c.M) ? v[sb + j] * w.dL : 0.f;
+        }
+        if (m0 + SUB == Mp && e >= 0) {
+            if (a.conv) atomicAdd(&a.g_t_in[e], g);
+            else a.g_t_in[e] = g;
+        }
     }
-}
-
-template <int BN>
-__device__ __forceinline__ void epi_gradt(uint32_t tbase, int n_main, bool corr, int row, int col0, int c_lo,
-                                          int c_hi, const TcEpiArgs &a) {
-    if (a.c.Mp == 8) epi_gradt_sub<BN, 8>(tbase, n_main, corr, row, col0, c_lo, c_hi, a);
-    else if (a.c.Mp == 16) epi_gradt_sub<BN, 16>(tbase, n_main, corr, row, col0, c_lo, c_hi, a);
-    else epi_gradt_sub<BN, 32>(tbase, n_main, corr, row, col0, c_lo, c_hi, a);
 }
 
 // ---------------------------------------------------------------------------
-// The kernel.
+// The kernel: persistent, one CTA per SM looping over output tiles.
+//   warp 0      TMA producer (one lane)
+//   warp 1      TMEM allocation, MMA issuer (one lane)
+//   warps 2-9   epilogue (warp w: lane quarter w % 4, column group (w-2)/4 of
+//               64 columns; a thread owns one accumulator row of its group)
+// Barriers: full/empty per smem stage; acc_full (MMA -> epilogue, per tile);
+// acc_empty (epilogue -> MMA: the accumulator may be overwritten), 8 warps.
 // ---------------------------------------------------------------------------
-constexpr int NWARPS = 16;  // 4 TMEM lane quarters x 4 column groups
-constexpr int NTHREADS = NWARPS * 32;
+constexpr int NEPI = 8;
+constexpr int NTHREADS = (2 + NEPI) * 32;
+constexpr int GCOLS = 64;  // accumulator columns per epilogue warp group (BN / (NEPI / 4))
+
+struct TileInfo {
+    int row0, col0, kt0, nkt, split;
+};
+
+__device__ __forceinline__ TileInfo tile_info(int t, int n_row, int n_col, int ktiles, int kt_per_split, int BNv) {
+    TileInfo ti;
+    const int per_split = n_row * n_col;
+    ti.split = t / per_split;
+    const int rem = t % per_split;
+    ti.row0 = (rem % n_row) * BM;
+    ti.col0 = (rem / n_row) * BNv;
+    ti.kt0 = ti.split * kt_per_split;
+    ti.nkt = ktiles - ti.kt0;
+    if (ti.nkt > kt_per_split) ti.nkt = kt_per_split;
+    return ti;
+}
 
 template <int NPASS, int BN, int EPI, bool F16>
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA_hi, const __grid_constant__ CUtensorMap mA_lo,
               const __grid_constant__ CUtensorMap mB_hi, const __grid_constant__ CUtensorMap mB_lo, int R, int Cn,
-              int ktiles, int kt_per_split, TcEpiArgs args) {
+              int ktiles, int kt_per_split, int n_row, int n_col, int n_split, TcEpiArgs args) {
     using C = Cfg<NPASS, BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + C::STAGES * C::STAGE);
     uint64_t *empty = full + C::STAGES;
-    uint64_t *accf = empty + C::STAGES;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(accf + 1);
+    uint64_t *acc_full = empty + C::STAGES;
+    uint64_t *acc_empty = acc_full + 1;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int col0 = blockIdx.x * BN, row0 = blockIdx.y * BM;
-    const int kt0 = blockIdx.z * kt_per_split;
-    int nkt = ktiles - kt0;
-    if (nkt > kt_per_split) nkt = kt_per_split;
+    const int ntiles = n_row * n_col * n_split;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(accf, 1);
+        mbar_init(acc_full, 1);
+        mbar_init(acc_empty, NEPI);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
-    if (warp == 0) tmem_alloc(tmem_slot, C::TMEM_COLS);
+    if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0) {
-        if (lane == 0 && nkt > 0) {
-            // TMA producer
-            for (int i = 0; i < nkt; ++i) {
-                const int s = i % C::STAGES;
-                const uint32_t ph = (uint32_t)(i / C::STAGES) & 1u;
-                if (!mbar_wait(&empty[s], ph ^ 1u)) {
-                    set_status(STATUS_TIMEOUT);
-                    break;
+        if (lane == 0) {
+            // TMA producer: stage ring shared by all tiles of this CTA
+            uint32_t it = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                const TileInfo ti = tile_info(t, n_row, n_col, ktiles, kt_per_split, BN);
+                for (int i = 0; i < ti.nkt; ++i, ++it) {
+                    const int s = it % C::STAGES;
+                    const uint32_t ph = (it / C::STAGES) & 1u;
+                    if (!mbar_wait(&empty[s], ph ^ 1u)) {
+                        set_status(STATUS_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(&full[s], (uint32_t)C::STAGE);
+                    const int kx = (ti.kt0 + i) * BK;
+                    const uint32_t st = smem_u32(smem + s * C::STAGE);
+                    tma_load_2d(st, &mA_hi, &full[s], kx, ti.row0);
+                    if (NPASS == 3) tma_load_2d(st + C::A_BYTES, &mA_lo, &full[s], kx, ti.row0);
+                    tma_load_2d(st + C::NOP * C::A_BYTES, &mB_hi, &full[s], kx, ti.col0);
+                    if (NPASS == 3) tma_load_2d(st + C::NOP * C::A_BYTES + C::B_BYTES, &mB_lo, &full[s], kx, ti.col0);
                 }
-                mbar_expect_tx(&full[s], (uint32_t)C::STAGE);
-                const int kx = (kt0 + i) * BK;
-                const uint32_t st = smem_u32(smem + s * C::STAGE);
-                tma_load_2d(st, &mA_hi, &full[s], kx, row0);
-                if (NPASS == 3) tma_load_2d(st + C::A_BYTES, &mA_lo, &full[s], kx, row0);
-                tma_load_2d(st + C::NOP * C::A_BYTES, &mB_hi, &full[s], kx, col0);
-                if (NPASS == 3) tma_load_2d(st + C::NOP * C::A_BYTES + C::B_BYTES, &mB_lo, &full[s], kx, col0);
             }
         }
         __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0 && nkt > 0) {
+        if (lane == 0) {
             // MMA issuer
             constexpr uint32_t idesc = idesc_16bit(BM, BN, F16);
+            uint32_t it = 0, j = 0;
             bool ok = true;
-            for (int i = 0; i < nkt; ++i) {
-                const int s = i % C::STAGES;
-                const uint32_t ph = (uint32_t)(i / C::STAGES) & 1u;
-                if (!mbar_wait(&full[s], ph)) {
-                    set_status(STATUS_TIMEOUT);
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
-                const uint32_t a_lo = a_hi + C::A_BYTES;
-                const uint32_t b_hi = a_hi + C::NOP * C::A_BYTES;
-                const uint32_t b_lo = b_hi + C::B_BYTES;
-                const uint32_t acc_main = tmem + (uint32_t)((i % C::P_MAIN) * BN);
-                const uint32_t acc_corr = tmem + (uint32_t)(3 * BN);
-#pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk) {
-                    const uint64_t da = sdesc_sw128(a_hi + kk * 32);
-                    const uint64_t db = sdesc_sw128(b_hi + kk * 32);
-                    mma_bf16(acc_main, da, db, idesc, (i >= C::P_MAIN || kk > 0) ? 1u : 0u);
-                    if (NPASS == 3) {
-                        mma_bf16(acc_corr, da, sdesc_sw128(b_lo + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
-                        mma_bf16(acc_corr, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
+                const TileInfo ti = tile_info(t, n_row, n_col, ktiles, kt_per_split, BN);
+                if (j > 0) {
+                    // the epilogue of the previous tile has taken the accumulator
+                    if (!mbar_wait(acc_empty, (j - 1) & 1u)) {
+                        set_status(STATUS_TIMEOUT);
+                        break;
                     }
+                    tc_fence_after();
                 }
-                mma_commit(&empty[s]);
+                for (int i = 0; i < ti.nkt; ++i, ++it) {
+                    const int s = it % C::STAGES;
+                    const uint32_t ph = (it / C::STAGES) & 1u;
+                    if (!mbar_wait(&full[s], ph)) {
+                        set_status(STATUS_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
+                    const uint32_t a_lo = a_hi + C::A_BYTES;
+                    const uint32_t b_hi = a_hi + C::NOP * C::A_BYTES;
+                    const uint32_t b_lo = b_hi + C::B_BYTES;
+                    const uint32_t acc_main = tmem + (uint32_t)((i % C::P_MAIN) * BN);
+                    const uint32_t acc_corr = tmem + (uint32_t)(3 * BN);
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint64_t da = sdesc_sw128(a_hi + kk * 32);
+                        const uint64_t db = sdesc_sw128(b_hi + kk * 32);
+                        mma_bf16(acc_main, da, db, idesc, (i >= C::P_MAIN || kk > 0) ? 1u : 0u);
+                        if (NPASS == 3) {
+                            mma_bf16(acc_corr, da, sdesc_sw128(b_lo + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                            mma_bf16(acc_corr, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
+                        }
+                    }
+                    mma_commit(&empty[s]);
+                }
+                if (ok) mma_commit(acc_full);
             }
-            if (ok) mma_commit(accf);
         }
         __syncwarp();
-    }
-
-    // epilogue: all 16 warps; warp w reads TMEM lane quarter w % 4 (rows
-    // 32(w%4) .. +31) and column group w / 4. Scan and GradT keep a sample's
-    // columns in one thread, so a group takes whole samples (a sample spans
-    // max(1, Mp/32) chunks of 32 columns).
-    const bool acc_ok = (nkt > 0) && mbar_wait_sleep(accf, 0);
-    tc_fence_after();
-    if (acc_ok) {
-        const int quarter = warp & 3, group = warp >> 2;
+    } else {
+        // epilogue warps
+        const int ew = warp - 2;
+        const int quarter = warp & 3, group = ew >> 2;
         const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16);
-        const int row = row0 + quarter * 32 + lane;
-        int c_lo = group * 32, c_hi = c_lo + 32;
-        if (EPI != (int)Epi::Store) {
-            const int cps = args.c.Mp > 32 ? args.c.Mp / 32 : 1;  // chunks per sample
-            c_lo = group * cps * 32;
-            c_hi = c_lo + cps * 32;
-            if (c_lo >= BN) c_lo = c_hi = BN;
+        // columns of a group: GCOLS, or a whole sample when one spans more
+        const int span = (EPI != (int)Epi::Store && args.c.Mp > GCOLS) ? args.c.Mp : GCOLS;
+        int c_lo = group * span, c_hi = c_lo + span;
+        if (c_lo >= BN) c_lo = c_hi = BN;
+        if (c_hi > BN) c_hi = BN;
+        uint32_t j = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
+            const TileInfo ti = tile_info(t, n_row, n_col, ktiles, kt_per_split, BN);
+            if (!mbar_wait_sleep(acc_full, j & 1u)) {
+                set_status(STATUS_TIMEOUT);
+                break;
+            }
+            tc_fence_after();
+            const int row = ti.row0 + quarter * 32 + lane;
+            const int n_main = ti.nkt < C::P_MAIN ? ti.nkt : C::P_MAIN;
+            const bool corr = (NPASS == 3);
+            if (c_hi - c_lo == GCOLS) {
+                // drain the group's chunks, hand the accumulator back, then work
+                float v[GCOLS / 32][32];
+#pragma unroll
+                for (int h = 0; h < GCOLS / 32; ++h) tmem_ld_acc<BN>(tbase, c_lo + 32 * h, n_main, corr, v[h]);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acc_empty);
+                if (EPI == (int)Epi::Store) {
+#pragma unroll
+                    for (int h = 0; h < GCOLS / 32; ++h) store_chunk(v[h], row, ti.col0, c_lo + 32 * h, R, Cn, args, ti.split);
+                } else {
+                    BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+                    float g = 0.f;
+                    if (args.c.Mp == 8) {
+#pragma unroll
+                        for (int h = 0; h < GCOLS / 32; ++h) gradt_chunk<8>(v[h], row, ti.col0 + c_lo + 32 * h, w, g, args);
+                    } else if (args.c.Mp == 16) {
+#pragma unroll
+                        for (int h = 0; h < GCOLS / 32; ++h) gradt_chunk<16>(v[h], row, ti.col0 + c_lo + 32 * h, w, g, args);
+                    } else {
+#pragma unroll
+                        for (int h = 0; h < GCOLS / 32; ++h) gradt_chunk<32>(v[h], row, ti.col0 + c_lo + 32 * h, w, g, args);
+                    }
+                }
+            } else {
+                // a sample spans more than GCOLS columns (Mp > GCOLS) or the
+                // group is idle: work chunk by chunk out of TMEM, then hand it back
+                BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+                float g = 0.f;
+                for (int cc = c_lo; cc < c_hi; cc += 32) {
+                    float v[32];
+                    tmem_ld_acc<BN>(tbase, cc, n_main, corr, v);
+                    if (EPI == (int)Epi::GradT) gradt_chunk<32>(v, row, ti.col0 + cc, w, g, args);
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acc_empty);
+            }
         }
-        const int n_main = nkt < C::P_MAIN ? nkt : C::P_MAIN;
-        const bool corr = (NPASS == 3);
-        if (EPI == (int)Epi::Store) epi_store<BN>(tbase, n_main, corr, row, col0, c_lo, c_hi, R, Cn, args);
-        else if (EPI == (int)Epi::Scan) epi_scan<BN>(tbase, n_main, corr, row, col0, c_lo, c_hi, args);
-        else epi_gradt<BN>(tbase, n_main, corr, row, col0, c_lo, c_hi, args);
-    } else if (nkt > 0) {
-        set_status(STATUS_TIMEOUT);
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, C::TMEM_COLS);
+    if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
 }
 
 // ---------------------------------------------------------------------------
@@ -561,22 +549,32 @@ static bool make_map(CUtensorMap *m, const void *ptr, int rows, int cols, int ld
     return r == CUDA_SUCCESS;
 }
 
+static int num_sms() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+    }
+    return n;
+}
+
 template <int NPASS, int BN, int EPI, bool F16>
 static cudaError_t launch_one(const CUtensorMap &a_hi, const CUtensorMap &a_lo, const CUtensorMap &b_hi,
                               const CUtensorMap &b_lo, int R, int Cn, int K, int splits, const TcEpiArgs &args,
                               cudaStream_t st) {
     using C = Cfg<NPASS, BN>;
-    static bool attr_set = false;  // per instantiation
-    if (!attr_set) {
-        cudaError_t e =
-            cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI, F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    cudaError_t e =
+        cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI, F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
     const int ktiles = (K + BK - 1) / BK;
     const int per = (ktiles + splits - 1) / splits;
-    dim3 grid((Cn + BN - 1) / BN, (R + BM - 1) / BM, splits);
-    k_tc_gemm<NPASS, BN, EPI, F16><<<grid, NTHREADS, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per, args);
+    const int n_row = (R + BM - 1) / BM, n_col = (Cn + BN - 1) / BN;
+    const long long ntiles = (long long)n_row * n_col * splits;
+    const int grid = (int)(ntiles < num_sms() ? ntiles : num_sms());
+    k_tc_gemm<NPASS, BN, EPI, F16><<<grid, NTHREADS, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per,
+                                                                       n_row, n_col, splits, args);
     return cudaGetLastError();
 }
 
@@ -614,8 +612,7 @@ cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const vo
 #define DSTD_TC_LAUNCH(NP, F)                                                                              \
     switch (epi) {                                                                                         \
         case Epi::Store: return tc::launch_one<NP, BN, 0, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st); \
-        case Epi::Scan: return tc::launch_one<NP, BN, 1, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);  \
-        default: return tc::launch_one<NP, BN, 2, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);         \
+        default: return tc::launch_one<NP, BN, 1, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);         \
     }
     if (f16) {
         DSTD_TC_LAUNCH(3, true)

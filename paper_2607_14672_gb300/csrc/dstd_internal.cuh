@@ -109,65 +109,118 @@ __device__ __forceinline__ float vhat_at(const LifConst &c, float v0, float I0, 
     return __expf(-c.av * s) * (v0 + phi_f(c, s) * I0);
 }
 
-// first root of v^(s) = v_th on [0, hi] given v^(0) < v_th <= v^(hi)
+// first root of v^(s) = v_th on [0, hi] given v^(0) < v_th <= v^(hi):
+// Newton from the secant guess inside the shrinking bracket (bisection when a
+// step leaves it). v^ - v_th is formed with one rounding (fma, accurate
+// exponentials), so its fp32 noise is about 1e-7 v_th. The iteration ends
+// with the Newton step taken from a point where |v^ - v_th| <= 4e-7 v_th
+// (which lands within the noise of the root), or when the step or the
+// bracket is below 1e-6 dt: two or three steps from the secant guess; a
+// nearly tangential crossing can fall back to bisection, hence up to 24.
 __device__ __forceinline__ float interval_root(const LifConst &c, float v0, float I0, float hi) {
     if (c.av == 0.0f) {
         // v^ = v0 + phi(s) I0 is monotone here: invert phi in closed form
         float s = phi_inv_f(c, (c.vth - v0) / I0);
         return fminf(fmaxf(s, 0.0f), hi);
     }
+    const float tol = 1e-6f * c.dt;
+    const float ftol = 4e-7f * fabsf(c.vth);
     float lo = 0.0f;
-    float s = 0.5f * hi;
-    for (int it = 0; it < 48; ++it) {
-        float e = __expf(-c.av * s);
-        float f = e * (v0 + phi_f(c, s) * I0) - c.vth;
-        if (f >= 0.0f) hi = s; else lo = s;
-        float df = -c.av * (f + c.vth) + I0 * __expf(-c.aI * s);
+    const float vhi = vhat_at(c, v0, I0, hi);
+    float s = (vhi > v0) ? hi * (c.vth - v0) / (vhi - v0) : 0.5f * hi;
+    s = fminf(fmaxf(s, 0.0f), hi);
+    for (int it = 0; it < 24; ++it) {
+        const float em = expf(-c.av * s);
+        const float ph = phi_f(c, s);
+        const float f = fmaf(em, fmaf(ph, I0, v0), -c.vth);
+        if (f > 0.0f) hi = s; else lo = s;
+        // dv^/ds = -av v^ + I0 e^{-aI s}, with e^{-aI s} = e^{-av s} (1 - lam phi(s))
+        const float df = fmaf(I0 * em, 1.0f - c.lam * ph, -c.av * (f + c.vth));
         float sn = s - f / df;
-        if (!(df > 0.0f) || !(sn > lo) || !(sn < hi)) sn = 0.5f * (lo + hi);
-        if (fabsf(sn - s) <= 1e-7f * c.dt || hi - lo <= 1e-7f * c.dt) { s = sn; break; }
+        if (!(df > 0.0f) || !(sn >= lo) || !(sn <= hi)) sn = 0.5f * (lo + hi);
+        const bool done = fabsf(f) <= ftol || fabsf(sn - s) <= tol || hi - lo <= tol;
         s = sn;
+        if (done) break;
     }
     return fminf(fmaxf(s, 0.0f), hi);
 }
 
 // Exact firing test of one interval whose cheap bound reached v_th: the
 // bracket end for the root (0 if v^ is already at v_th at T_q, dt if v^(dt)
-// >= v_th, the interior maximum if only that reaches v_th), or -1. Kept out
-// of line so the per-interval fast path of the scan stays small.
-static __device__ __noinline__ float scan_interval_test(const LifConst &c, float v0, float I0, float ve) {
-    if (v0 >= c.vth) return 0.0f;
-    if (ve >= c.vth) return c.dt;
-    if (c.av > 0.0f && c.aI > 0.0f && I0 > 0.0f) {
+// >= v_th, the interior maximum if only that reaches v_th), or -1. Out of
+// line where it runs once per interval (scan_step), inline where it runs
+// once per block of intervals (scan_block).
+__device__ __forceinline__ float interval_test(float av, float aI, float lam, int lam_zero, float rI, float dt,
+                                               float vth, float v0, float I0, float ve) {
+    if (v0 >= vth) return 0.0f;
+    if (ve >= vth) return dt;
+    if (av > 0.0f && aI > 0.0f && I0 > 0.0f) {
         // interior maximum: dv^/ds > 0 at s = 0 and < 0 at s = dt
-        const float d0 = -c.av * v0 + I0;
-        const float dE = -c.av * ve + c.rI * I0;
+        const float d0 = -av * v0 + I0;
+        const float dE = -av * ve + rI * I0;
         if (d0 > 0.0f && dE < 0.0f) {
             // e^{-lam s*} = 1 + lam y with y = (av v0 - I0)/(I0 aI)
-            const float y = (c.av * v0 - I0) / (I0 * c.aI);
-            float sp = c.lam_zero ? -y : -log1pf(c.lam * y) / c.lam;
-            sp = fminf(fmaxf(sp, 0.0f), c.dt);
-            if (vhat_at(c, v0, I0, sp) >= c.vth) return sp;
+            const float y = (av * v0 - I0) / (I0 * aI);
+            float sp = lam_zero ? -y : -log1pf(lam * y) / lam;
+            sp = fminf(fmaxf(sp, 0.0f), dt);
+            const float ph = lam_zero ? sp : -expm1f(-lam * sp) / lam;
+            if (__expf(-av * sp) * (v0 + ph * I0) >= vth) return sp;
         }
     }
     return -1.0f;
 }
-
-// Consume w^_m for interval m (m = 0..M-1, in order).
-__device__ __forceinline__ void scan_step(const LifConst &c, ScanState &st, float w, int m) {
+// Consume w^_m for the SUB intervals m0 .. m0+SUB-1 of one neuron at once,
+// with the grid weights in registers (w[off + j] * rs for interval m0 + j).
+// Same result as SUB calls of scan_step, in two phases so that the lanes of
+// a warp stay together: a branch-free pass runs the recurrence and picks the
+// first interval where v^ reaches v_th at an end point, or has an interior
+// maximum that the cheap bound does not exclude; the exact test then runs
+// once, for all lanes at their own candidate. Only an interior maximum that
+// stays below v_th fails it; the pass then restarts after that interval.
+template <int SUB>
+__device__ __forceinline__ void scan_block(const LifConst &c, ScanState &st, const float (&w)[32], int off, float rs,
+                                           int m0) {
     if (st.q < c.M) return;
-    const float v0 = st.v;
-    const float I0 = st.I + w;
-    const float ve = c.rv * v0 + c.KD * I0;
-    st.v = ve;
-    st.I = c.rI * I0;
-    if (fmaxf(v0, 0.0f) + fmaxf(I0, 0.0f) * c.Kmax < c.vth) return;  // v^ < v_th on this interval
-    const float hi = scan_interval_test(c, v0, I0, ve);
-    if (hi >= 0.0f) {
-        st.q = m;
-        st.v0 = v0;
-        st.I0 = I0;
-        st.hi = hi;
+    const int nvalid = c.M - m0;  // intervals of the block below M
+    if (nvalid <= 0) return;
+    const float v_in = st.v, I_in = st.I;
+    int j0 = 0;
+    for (int pass = 0; pass < SUB; ++pass) {
+        float v = v_in, I = I_in;
+        int cand = SUB;
+        float cv0 = 0.f, cI0 = 0.f, cve = 0.f;
+#pragma unroll
+        for (int j = 0; j < SUB; ++j) {
+            const float I0 = I + w[off + j] * rs;
+            const float ve = c.rv * v + c.KD * I0;
+            // v^ reaches v_th at an end of the interval, or may at an
+            // interior maximum (rising at s = 0, falling at s = dt, bound met)
+            const float d0 = -c.av * v + I0;
+            const float dE = -c.av * ve + c.rI * I0;
+            const bool endp = (v >= c.vth) | (ve >= c.vth);
+            const bool peak = (d0 > 0.0f) & (dE < 0.0f) & (fmaxf(v, 0.0f) + fmaxf(I0, 0.0f) * c.Kmax >= c.vth);
+            const bool take = (cand == SUB) & (j >= j0) & (j < nvalid) & (endp | peak);
+            cand = take ? j : cand;
+            cv0 = take ? v : cv0;
+            cI0 = take ? I0 : cI0;
+            cve = take ? ve : cve;
+            v = ve;
+            I = c.rI * I0;
+        }
+        if (pass == 0) {
+            st.v = v;
+            st.I = I;
+        }
+        if (cand == SUB) return;
+        const float hi = interval_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, cv0, cI0, cve);
+        if (hi >= 0.0f) {
+            st.q = m0 + cand;
+            st.v0 = cv0;
+            st.I0 = cI0;
+            st.hi = hi;
+            return;
+        }
+        j0 = cand + 1;
     }
 }
 
@@ -176,8 +229,9 @@ __device__ __forceinline__ void scan_finish(const LifConst &c, ScanState &st) {
     if (st.q >= c.M) return;
     const float s = st.hi > 0.0f ? interval_root(c, st.v0, st.I0, st.hi) : 0.0f;
     st.s = s;
-    const float Ic = st.I0 * __expf(-c.aI * s);
-    st.vdot = fmaxf(-c.av * c.vth + Ic, c.vdot_floor);
+    // dv^/dt at the spike, -av v_th + I(t), formed with one rounding: when
+    // it is small the two terms nearly cancel
+    st.vdot = fmaxf(fmaf(st.I0, expf(-c.aI * s), -c.av * c.vth), c.vdot_floor);
 }
 
 // Temporal penalty of one firing neuron (Eq. temporal_penalty) and dT/dt,
@@ -239,10 +293,11 @@ cudaError_t launch_binning_im2col(const float *t, const ConvGeom &g, int pos0, i
 // public-layout binning: s, ds [B, M, N] fp32
 cudaError_t launch_binning_public(const float *t, int B, int N, const LifConst &c, float *s, float *ds,
                                   cudaStream_t st);
-// scan/solve from w^ with element (b, i, m) at what[b*sb + i*si + m]
-cudaError_t launch_scan_solve(const float *what, long long sb, long long si, int B, int N, const LifConst &c,
-                              const float *rowsum, float *t_out, int *q, float *s, float *vdot, float *penalty,
-                              cudaStream_t st);
+// scan/solve from w^ with element (b, i, m) at what[b*sb + i*si + m*sm],
+// scaled by scale[i] when scale is not null
+cudaError_t launch_scan_solve(const float *what, long long sb, long long si, long long sm, int B, int N,
+                              const LifConst &c, const float *scale, const float *rowsum, float *t_out, int *q,
+                              float *s, float *vdot, float *penalty, cudaStream_t st);
 // dw^ from saved state; writes [B*Mp, ldn] (row (b,m), col i) and [N, ldbm]
 // (row i, col (b,m)) in the operand format; silent counts per neuron.
 // (silent_count is zeroed first unless accumulate_count)
@@ -267,13 +322,13 @@ cudaError_t launch_sgemm_tn(const float *A, int lda, const float *Bm, int ldb, f
 
 // tcgen05 GEMM D = A B^T on bf16 operands (hi/lo for BF16X3), fp32 TMEM
 // accumulation, with a fused epilogue.
-enum class Epi { Store = 0, Scan = 1, GradT = 2 };
+enum class Epi { Store = 0, GradT = 1 };
 struct TcEpiArgs {
     const float *row_scale;  // per-row factor applied to the accumulator (Store, Scan), may be null
     // Store
     float *D; long long ldd; long long zstride;
-    // Scan (rows = neurons i, columns = (b, m))
-    LifConst c; int B; int N; const float *rowsum; float *t_out; int *q; float *s; float *vdot; float *penalty;
+    // GradT: layer constants and sizes (rows N, samples B)
+    LifConst c; int B; int N;
     // GradT (rows = inputs j, columns = (b, m)); with conv != 0 the rows are
     // filter taps kidx, the columns (output position, m), and each result is
     // added atomically into the input element the tap reads (col2im)

@@ -59,6 +59,20 @@ static inline unsigned blocks_for(long long n, int threads) {
     return (unsigned)((n + threads - 1) / threads);
 }
 
+// blocks_for capped at 8 blocks per SM, for grid-stride kernels that end in
+// one atomic per block
+static unsigned grid_cap(long long n, int threads) {
+    static int sms = 0;
+    if (sms == 0) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+            sms <= 0)
+            sms = 148;
+    }
+    const unsigned b = blocks_for(n, threads), cap = 8u * (unsigned)sms;
+    return b < 1 ? 1 : (b < cap ? b : cap);
+}
+
 __device__ __forceinline__ void split_bf16(float x, __nv_bfloat16 &hi, __nv_bfloat16 &lo) {
     hi = __float2bfloat16_rn(x);
     lo = __float2bfloat16_rn(x - __bfloat162float(hi));
@@ -425,27 +439,50 @@ __device__ __forceinline__ void finish_neuron(const LifConst &c, const ScanState
     }
 }
 
+// Block-wide sums of the four penalty terms, one atomic per term per block
+// (blockDim.x a multiple of 32, at most 1024; every thread of the block calls).
 __device__ __forceinline__ void flush_penalty(float acc[4], float *penalty) {
+    __shared__ float part[32][4];
     if (!penalty) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        float v = warp_sum(acc[k]);
-        if ((threadIdx.x & 31) == 0 && v != 0.0f) atomicAdd(&penalty[k], v);
+        const float v = warp_sum(acc[k]);
+        if (lane == 0) part[warp][k] = v;
+    }
+    __syncthreads();
+    if (warp == 0) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float v = lane < nw ? part[lane][k] : 0.0f;
+            v = warp_sum(v);
+            if (lane == 0 && v != 0.0f) atomicAdd(&penalty[k], v);
+        }
     }
 }
 
-__global__ void k_scan_solve(const float *__restrict__ what, long long sb, long long si, int B, int N, LifConst c,
-                             const float *__restrict__ rowsum, float *t_out, int *q, float *s, float *vdot,
-                             float *penalty) {
-    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+// One thread per neuron (b, i), neurons i of a sample on consecutive
+// threads; element (b, i, m) of w^ at what[b*sb + i*si + m*sm], times
+// scale[i] when given. The bins are read SUB at a time into registers (all
+// loads of a block in flight together) and scanned by scan_block; a neuron
+// stops reading once it fires.
+template <int SUB>
+__global__ void __launch_bounds__(256, 3) k_scan_solve(const float *__restrict__ what, long long sb, long long si, long long sm, int B, int N,
+                             LifConst c, const float *__restrict__ scale, const float *__restrict__ rowsum,
+                             float *t_out, int *q, float *s, float *vdot, float *penalty) {
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    if (idx < (long long)B * N) {
-        int b = (int)(idx / N), i = (int)(idx % N);
+    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < (long long)B * N;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int b = (int)(idx / N), i = (int)(idx % N);
         const float *w = what + b * sb + i * si;
+        const float sc = scale ? scale[i] : 1.0f;
         ScanState st;
         scan_reset(st, c.M);
-        for (int m = 0; m < c.M; ++m) {
-            scan_step(c, st, w[m], m);
+        for (int m0 = 0; m0 < c.M; m0 += SUB) {
+            float x[32];
+#pragma unroll
+            for (int j = 0; j < SUB; ++j) x[j] = (m0 + j < c.M) ? __ldg(w + (long long)(m0 + j) * sm) : 0.0f;
+            scan_block<SUB>(c, st, x, 0, sc, m0);
             if (st.q < c.M) break;
         }
         scan_finish(c, st);
@@ -454,11 +491,17 @@ __global__ void k_scan_solve(const float *__restrict__ what, long long sb, long 
     flush_penalty(acc, penalty);
 }
 
-cudaError_t launch_scan_solve(const float *what, long long sb, long long si, int B, int N, const LifConst &c,
-                              const float *rowsum, float *t_out, int *q, float *s, float *vdot, float *penalty,
-                              cudaStream_t st) {
+cudaError_t launch_scan_solve(const float *what, long long sb, long long si, long long sm, int B, int N,
+                              const LifConst &c, const float *scale, const float *rowsum, float *t_out, int *q,
+                              float *s, float *vdot, float *penalty, cudaStream_t st) {
     long long n = (long long)B * N;
-    k_scan_solve<<<blocks_for(n, 256), 256, 0, st>>>(what, sb, si, B, N, c, rowsum, t_out, q, s, vdot, penalty);
+    const unsigned g = grid_cap(n, 256);
+    if (c.M <= 8)
+        k_scan_solve<8><<<g, 256, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty);
+    else if (c.M <= 16)
+        k_scan_solve<16><<<g, 256, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty);
+    else
+        k_scan_solve<32><<<g, 256, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty);
     return cudaGetLastError();
 }
 

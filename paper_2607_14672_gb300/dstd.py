@@ -185,7 +185,7 @@ def dense_fwd(t_in, W, p, math_mode, t_out, saved, penalty, workspace, stream=No
 
 def dense_fwd_noalloc(t_in, W, p, math_mode, t_out, saved, penalty=None, stream=None):
     """dstd_dense_fwd without a workspace: for callers that cannot allocate
-    device memory; scratch is the library's fixed 32 MiB device array, shared
+    device memory; scratch is the library's fixed 64 MiB device array, shared
     by every call (do not overlap calls on the GPU)."""
     B, N_in = t_in.shape
     N_out = W.shape[0]

@@ -101,7 +101,7 @@ class DenseNet:
         """Kernels the library launches per ``step`` (memsets not counted)."""
         tc = self.math != "f32"
         L = len(self.W)
-        n = L * (3 if tc else 4)                  # fwd: prep + binning + gemm(+fused scan) [+ scan]
+        n = L * 4                                 # fwd: prep + binning + gemm (+ fused scan) + root solve / scan
         n += 1                                    # loss
         n += L * 4                                # bwd: dw^ + binning^T + dW gemm + reduce
         n += (L - 1) * (2 if tc else 3)           # bwd input times: prep W^T + dS gemm [+ gather]

@@ -2,7 +2,7 @@
 workspace one (dstd_dense_fwd), through the C-ABI.
 
 dstd_dense_fwd_noalloc serves callers that cannot allocate device memory;
-its scratch is the library's fixed 32 MiB device array, shared by all calls.
+its scratch is the library's fixed 64 MiB device array, shared by all calls.
 Two calls in a row (different layers, different sizes) must each give what
 dstd_dense_fwd gives on the same inputs: spike times within 1e-4 T_max (the
 parity tolerance of the other tests; in fact bitwise), identical firing
