@@ -316,28 +316,28 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
     a.c = c;
     a.B = B;
     a.N = N_out;
+    a.row_scale = ws.row_scale;
     if (store_D) {
         Timed tm(KK_GEMM_FWD, st);
-        a.row_scale = ws.row_scale;
         a.D = ws.D;
         a.ldd = cols;
         a.zstride = 0;
         return cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
                                  Epi::Store, a, st));
     }
-    // w^ with rows (b, m) and columns i, so that the scan reads the M values
-    // of 32 neurons of a sample as 32-wide coalesced rows
+    // w^ with rows i and columns (b, m): the Mp bins of a neuron are 128
+    // contiguous bytes (Mp = 32) that the scan reads with 16-byte loads
     {
         Timed tm(KK_GEMM_FWD, st);
         a.D = ws.D;
-        a.ldd = ws.ldD;
+        a.ldd = cols;
         a.zstride = 0;
-        TRY(cu(launch_tc_gemm(ws.s_hi, ws.s_lo, ws.kpad, ws.w_hi, ws.w_lo, ws.kpad, (int)cols, N_out, N_in, 1, op,
+        TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
                               Epi::Store, a, st)));
     }
     Timed tm(KK_SCAN, st);
-    return cu(launch_scan_solve(ws.D, (long long)c.Mp * ws.ldD, 1, ws.ldD, B, N_out, c, ws.row_scale, ws.rowsum,
-                                t_out, sv->q, sv->s, sv->vdot, penalty, st));
+    return cu(launch_scan_solve(ws.D, c.Mp, cols, 1, B, N_out, c, nullptr, ws.rowsum, t_out, sv->q, sv->s,
+                                sv->vdot, penalty, st));
 }
 
 // ---------------------------------------------------------------------------
@@ -700,19 +700,20 @@ int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C
             Timed tm(KK_BIN, st);
             TRY(cu(launch_binning_im2col(t_in, pl.g, pos0, npos, c, op, false, ws.s_hi, ws.s_lo, pl.kpad, st)));
         }
+        const long long cols = (long long)npos * Mp;
         TcEpiArgs a{};
         a.D = ws.D;
-        a.ldd = ws.ldD;
+        a.ldd = cols;
         a.zstride = 0;
+        a.row_scale = op == OpKind::F16X3 ? ws.row_scale : nullptr;
         {
             Timed tm(KK_GEMM_FWD, st);
-            TRY(cu(launch_tc_gemm(ws.s_hi, ws.s_lo, pl.kpad, ws.w_hi, ws.w_lo, pl.kpad, npos * Mp, C_out, pl.K, 1, op,
+            TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, pl.kpad, ws.s_hi, ws.s_lo, pl.kpad, C_out, (int)cols, pl.K, 1, op,
                                   Epi::Store, a, st)));
         }
         const long long off = (long long)pos0 * C_out;
         Timed tr(KK_SCAN, st);
-        TRY(cu(launch_scan_solve(ws.D, (long long)Mp * ws.ldD, 1, ws.ldD, npos, C_out, c,
-                                 op == OpKind::F16X3 ? ws.row_scale : nullptr, ws.rowsum, t_out + off, sv.q + off,
+        TRY(cu(launch_scan_solve(ws.D, Mp, cols, 1, npos, C_out, c, nullptr, ws.rowsum, t_out + off, sv.q + off,
                                  sv.s + off, sv.vdot + off, penalty, st)));
     }
     return DSTD_OK;

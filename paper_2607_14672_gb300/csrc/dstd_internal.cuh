@@ -27,6 +27,7 @@ namespace dstd {
 struct LifConst {
     float av, aI, lam;     // rates; lam = aI - av
     int lam_zero;          // lam == 0 exactly (tau_m == tau_s, incl. both inf)
+    float inv_lam;         // 1 / lam (0 when lam_zero)
     float T0, dt, inv_dt;  // T_0 = t_first - t_offset, step
     float rv, rI, KD;      // e^{-av dt}, e^{-aI dt}, K(dt)
     float inv_phi_dt;      // 1 / phi(dt)
@@ -127,16 +128,17 @@ __device__ __forceinline__ float interval_root(const LifConst &c, float v0, floa
     const float ftol = 4e-7f * fabsf(c.vth);
     float lo = 0.0f;
     const float vhi = vhat_at(c, v0, I0, hi);
-    float s = (vhi > v0) ? hi * (c.vth - v0) / (vhi - v0) : 0.5f * hi;
+    float s = (vhi > v0) ? hi * __fdividef(c.vth - v0, vhi - v0) : 0.5f * hi;
     s = fminf(fmaxf(s, 0.0f), hi);
     for (int it = 0; it < 24; ++it) {
         const float em = expf(-c.av * s);
-        const float ph = phi_f(c, s);
+        const float ph = c.lam_zero ? s : -expm1f(-c.lam * s) * c.inv_lam;
         const float f = fmaf(em, fmaf(ph, I0, v0), -c.vth);
         if (f > 0.0f) hi = s; else lo = s;
         // dv^/ds = -av v^ + I0 e^{-aI s}, with e^{-aI s} = e^{-av s} (1 - lam phi(s))
         const float df = fmaf(I0 * em, 1.0f - c.lam * ph, -c.av * (f + c.vth));
-        float sn = s - f / df;
+        // (the step is self-correcting: a fast quotient is enough)
+        float sn = s - __fdividef(f, df);
         if (!(df > 0.0f) || !(sn >= lo) || !(sn <= hi)) sn = 0.5f * (lo + hi);
         const bool done = fabsf(f) <= ftol || fabsf(sn - s) <= tol || hi - lo <= tol;
         s = sn;

@@ -26,6 +26,7 @@ LifConst make_const(const dstd_params &p, int Mp) {
     c.aI = (float)aI;
     c.lam = (float)lam;
     c.lam_zero = (lam == 0.0);
+    c.inv_lam = lam == 0.0 ? 0.0f : (float)(1.0 / lam);
     c.T0 = (float)((double)p.t_first - (double)p.t_offset);
     c.dt = (float)dt;
     c.inv_dt = (float)(1.0 / dt);
@@ -461,29 +462,142 @@ __device__ __forceinline__ void flush_penalty(float acc[4], float *penalty) {
     }
 }
 
-// One thread per neuron (b, i), neurons i of a sample on consecutive
-// threads; element (b, i, m) of w^ at what[b*sb + i*si + m*sm], times
-// scale[i] when given. The bins are read SUB at a time into registers (all
-// loads of a block in flight together) and scanned by scan_block; a neuron
-// stops reading once it fires.
-template <int SUB>
-__global__ void __launch_bounds__(256, 3) k_scan_solve(const float *__restrict__ what, long long sb, long long si, long long sm, int B, int N,
-                             LifConst c, const float *__restrict__ scale, const float *__restrict__ rowsum,
-                             float *t_out, int *q, float *s, float *vdot, float *penalty) {
+// Exact test of an interval whose v^ has an interior maximum (dv^/ds > 0 at
+// s = 0, < 0 at s = dt) and whose cheap bound reached v_th: the bracket end
+// for the root, or -1. Before the exact maximum (a log and two exponentials)
+// it tries a tighter bound: on [0, s*] v^ >= v0 and e^{-aI s} <= 1 give
+//   v^(s*) <= v0 + max_s [ -av v0 s + I0 (1 - e^{-aI s}) / aI ],
+// whose maximiser has e^{-aI s} = av v0 / I0. Out of line: it runs rarely.
+static __device__ __noinline__ float interior_test(float av, float aI, float lam, int lam_zero, float rI, float dt,
+                                                   float vth, float v0, float I0, float ve) {
+    if (!(av > 0.0f && aI > 0.0f && I0 > 0.0f)) return -1.0f;
+    float g;
+    const float inv_aI = 1.0f / aI;
+    if (v0 > 0.0f) {
+        const float sm = logf(I0 / (av * v0)) * inv_aI;
+        g = sm < dt ? -av * v0 * sm + (I0 - av * v0) * inv_aI : -av * v0 * dt + I0 * (1.0f - rI) * inv_aI;
+    } else {
+        g = -av * v0 * dt + I0 * (1.0f - rI) * inv_aI;
+    }
+    // margin: rounding of the bound's own terms
+    if (v0 + g + 1e-6f * (fabsf(v0) + fabsf(g)) < vth) return -1.0f;
+    return interval_test(av, aI, lam, lam_zero, rI, dt, vth, v0, I0, ve);
+}
+
+// One thread per neuron (b, i); element (b, i, m) of w^ at
+// what[b*sb + i*si + m*sm], times scale[i] when given. SUB bins at a time
+// are loaded together (16-byte loads when sm = 1 and rows are 16-byte
+// aligned) into the thread's own row of shared memory (stride SUB + 4
+// floats: 16-byte accesses of 8 consecutive lanes hit distinct banks). The
+// scan walks the bins four at a time: one 16-byte read, the recurrence, and
+// a branch-free flag per bin for "v^ may reach v_th here" (end point at
+// v_th, or an interior maximum that the cheap bound does not exclude). Only
+// a group with a flag leaves the loop: the group is walked again bin by bin
+// with the exact tests (interior_test out of line), and the scan resumes
+// after the tested bin if it does not fire.
+constexpr int SCAN_THREADS = 256;
+
+// One interval of the walk, with explicit fma so that the fast walk and the
+// exact re-walk round alike: the end state and the two flags.
+struct BinStep {
+    float ve, In;
+    bool endp, peak;
+};
+__device__ __forceinline__ BinStep bin_step(const LifConst &c, float v, float I0) {
+    BinStep r;
+    r.ve = fmaf(c.KD, I0, c.rv * v);
+    r.In = c.rI * I0;
+    r.endp = r.ve >= c.vth;
+    r.peak = (fmaf(-c.av, v, I0) > 0.0f) & (fmaf(-c.av, r.ve, r.In) < 0.0f) &
+             (fmaf(fmaxf(I0, 0.0f), c.Kmax, fmaxf(v, 0.0f)) >= c.vth);
+    return r;
+}
+
+template <int SUB, bool VEC, bool WIDE>
+__global__ void __launch_bounds__(SCAN_THREADS, 4) k_scan_solve(const float *__restrict__ what, long long sb,
+                                                                long long si, long long sm, int B, int N, LifConst c,
+                                                                const float *__restrict__ scale,
+                                                                const float *__restrict__ rowsum, float *t_out,
+                                                                int *q, float *s, float *vdot, float *penalty) {
+    constexpr int LD = SUB + 4;
+    __shared__ __align__(16) float sw[SCAN_THREADS * LD];
+    float *row = sw + threadIdx.x * LD;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < (long long)B * N;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const int b = (int)(idx / N), i = (int)(idx % N);
+    const long long n = (long long)B * N;
+    for (long long idx = (long long)blockIdx.x * SCAN_THREADS + threadIdx.x; idx < n;
+         idx += (long long)gridDim.x * SCAN_THREADS) {
+        int b, i;
+        if (WIDE) {
+            b = (int)(idx / N);
+            i = (int)(idx % N);
+        } else {
+            b = (int)((unsigned)idx / (unsigned)N);
+            i = (int)((unsigned)idx - (unsigned)b * (unsigned)N);
+        }
         const float *w = what + b * sb + i * si;
         const float sc = scale ? scale[i] : 1.0f;
         ScanState st;
         scan_reset(st, c.M);
-        for (int m0 = 0; m0 < c.M; m0 += SUB) {
-            float x[32];
+        float v = 0.f, I = 0.f;
+        for (int m0 = 0; m0 < c.M && st.q == c.M; m0 += SUB) {
+            const int mend = (c.M - m0) < SUB ? (c.M - m0) : SUB;
+            if (VEC && mend == SUB) {
 #pragma unroll
-            for (int j = 0; j < SUB; ++j) x[j] = (m0 + j < c.M) ? __ldg(w + (long long)(m0 + j) * sm) : 0.0f;
-            scan_block<SUB>(c, st, x, 0, sc, m0);
-            if (st.q < c.M) break;
+                for (int j = 0; j < SUB; j += 4) {
+                    const float4 u = __ldg(reinterpret_cast<const float4 *>(w + m0 + j));
+                    *reinterpret_cast<float4 *>(row + j) = make_float4(u.x * sc, u.y * sc, u.z * sc, u.w * sc);
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < SUB; ++j) row[j] = (j < mend) ? __ldg(w + (m0 + j) * sm) * sc : 0.0f;
+            }
+            int j = 0;
+            while (j < mend) {
+                // fast walk: groups of 4 bins, no branch inside a group
+                float vg = v, Ig = I;
+                int g = j & ~3;
+                bool flag = false;
+                for (; g < mend; g += 4) {
+                    const float4 x = *reinterpret_cast<const float4 *>(row + g);
+                    const float xs[4] = {x.x, x.y, x.z, x.w};
+                    vg = v;
+                    Ig = I;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const BinStep r = bin_step(c, v, I + xs[u]);
+                        flag |= (g + u >= j) & (g + u < mend) & (r.endp | r.peak);
+                        v = r.ve;
+                        I = r.In;
+                    }
+                    if (flag) break;
+                }
+                if (!flag) break;
+                // exact walk of the flagged group from its first bin
+                v = vg;
+                I = Ig;
+                int k = g;
+                float hi = -1.0f, I0 = 0.f;
+                for (; k < g + 4 && k < mend; ++k) {
+                    I0 = I + row[k];
+                    const BinStep r = bin_step(c, v, I0);
+                    if (k >= j) {
+                        if (r.endp) hi = c.dt;
+                        else if (r.peak)
+                            hi = interior_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, v, I0, r.ve);
+                        if (hi >= 0.0f) break;
+                    }
+                    v = r.ve;
+                    I = r.In;
+                }
+                if (hi >= 0.0f) {
+                    st.q = m0 + k;
+                    st.v0 = v;
+                    st.I0 = I0;
+                    st.hi = hi;
+                    break;
+                }
+                j = k;  // the flagged bins of the group did not fire; go on after them
+            }
         }
         scan_finish(c, st);
         finish_neuron(c, st, b, i, N, rowsum, t_out, q, s, vdot, acc);
@@ -495,13 +609,24 @@ cudaError_t launch_scan_solve(const float *what, long long sb, long long si, lon
                               const LifConst &c, const float *scale, const float *rowsum, float *t_out, int *q,
                               float *s, float *vdot, float *penalty, cudaStream_t st) {
     long long n = (long long)B * N;
-    const unsigned g = grid_cap(n, 256);
-    if (c.M <= 8)
-        k_scan_solve<8><<<g, 256, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty);
-    else if (c.M <= 16)
-        k_scan_solve<16><<<g, 256, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty);
-    else
-        k_scan_solve<32><<<g, 256, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty);
+    const unsigned g = grid_cap(n, SCAN_THREADS);
+    const bool vec = sm == 1 && (si % 4) == 0 && (sb % 4) == 0 && (reinterpret_cast<uintptr_t>(what) % 16) == 0;
+    const bool wide = n >= (1ll << 31);
+#define DSTD_SCAN_L(SUB, V, W) \
+    k_scan_solve<SUB, V, W><<<g, SCAN_THREADS, 0, st>>>(what, sb, si, sm, B, N, c, scale, rowsum, t_out, q, s, vdot, penalty)
+#define DSTD_SCAN(SUB)                          \
+    if (wide) DSTD_SCAN_L(SUB, false, true);    \
+    else if (vec) DSTD_SCAN_L(SUB, true, false); \
+    else DSTD_SCAN_L(SUB, false, false);
+    if (c.M <= 8) {
+        DSTD_SCAN(8)
+    } else if (c.M <= 16) {
+        DSTD_SCAN(16)
+    } else {
+        DSTD_SCAN(32)
+    }
+#undef DSTD_SCAN
+#undef DSTD_SCAN_L
     return cudaGetLastError();
 }
 
