@@ -214,6 +214,78 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------
+# roofline arithmetic (per launch, averaged over the layers of a kind)
+# ---------------------------------------------------------------------------
+# DRAM bytes read + written per launch, averaged over the kind's launches in
+# one step, from `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum`
+# on `python bench.py --steps 5 --warmup 3 --profile` (the per-launch table
+# in profiles/launches_cfg2_step.md); to be set to None when the kernel
+# changes after that capture.
+TRAFFIC_PER_LAUNCH = {
+    ("gemm_dW", "x3"): 44.1e6,
+    ("gemm_fwd_scan", "x3"): 27.8e6,
+    ("scan_solve", "x3"): 17.6e6,
+}
+
+
+def kind_rooflines(per_kind, sizes, B, Mp, npass, math_mode, pk, pk_src):
+    """Achieved vs peak for each kernel kind of the step.
+
+    Contractions are tensor-bound: achieved = the method's flops (2 grid
+    weights per input spike: 4 B N_in N_out per contraction) per launch /
+    time; dense_* = the tensor-core flops the dense formulation issues (Mp/2
+    times that, times npass for the three-product split). Binning, scan/solve,
+    dw^, the split-K reduction and weight prep are HBM-bound: achieved = the
+    bytes the kernel must move (inputs read once, outputs written once) /
+    time.
+    """
+    L = len(sizes) - 1
+    hbm = pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    tc_peak = pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    e = 4 if math_mode in ("x3", "f32") else 2            # bytes per operand element (hi+lo, or fp32)
+    pad8 = lambda x: (x + 7) // 8 * 8
+    algo_b, algo_f, dense_f = {}, {}, {}
+
+    def add(d, k, v):
+        d[k] = d.get(k, 0.0) + v
+
+    for l in range(L):
+        ni, no = sizes[l], sizes[l + 1]
+        cols = B * Mp
+        add(algo_b, "prep_weights", no * ni * 4 + no * pad8(ni) * e)
+        add(algo_b, "binning", B * ni * 4 + cols * pad8(ni) * e)
+        add(algo_b, "scan_solve", B * no * Mp * 4 + B * no * 16)
+        add(algo_b, "dwhat", B * no * 20 + 2 * B * no * Mp * e)
+        add(algo_b, "binning_T", B * ni * 4 + ni * cols * e)
+        add(algo_b, "dw_reduce", 3 * no * ni * 4 + no * ni * 4)
+        r_out, r_in = (no + 127) // 128 * 128, (ni + 127) // 128 * 128
+        k_in, k_out = (ni + 63) // 64 * 64, (no + 63) // 64 * 64
+        add(algo_f, "gemm_fwd_scan", 4 * B * ni * no)
+        add(dense_f, "gemm_fwd_scan", 2 * npass * r_out * cols * k_in)
+        add(algo_f, "gemm_dW", 4 * B * ni * no)
+        add(dense_f, "gemm_dW", 2 * npass * r_out * r_in * cols)
+        if l > 0:
+            add(algo_f, "gemm_dS_gradt", 4 * B * ni * no)
+            add(dense_f, "gemm_dS_gradt", 2 * npass * r_in * cols * k_out)
+    out = {}
+    for k, (t_ms, nl) in per_kind.items():
+        t = t_ms / 1000.0
+        if k in algo_f and math_mode != "f32":
+            a = algo_f[k] / nl / t
+            dn = dense_f[k] / nl / t
+            out[k] = {"bound": "tensor", "achieved": a / 1e12, "peak": tc_peak, "unit": "TFLOP/s",
+                      "frac": a / 1e12 / tc_peak, "dense_achieved": dn / 1e12, "dense_frac": dn / 1e12 / tc_peak,
+                      "per_launch_flops": algo_f[k] / nl, "per_launch_dense_flops": dense_f[k] / nl,
+                      "peak_source": f"{pk_src} bf16 (burst)", "launch_us": t_ms * 1000.0}
+        elif k in algo_b:
+            a = algo_b[k] / nl / t
+            out[k] = {"bound": "hbm", "achieved": a / 1e9, "peak": hbm, "unit": "GB/s", "frac": a / 1e9 / hbm,
+                      "per_launch_bytes": algo_b[k] / nl, "peak_source": f"{pk_src} copy",
+                      "launch_us": t_ms * 1000.0}
+    return out
+
+
+# ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
 def run_ours(args, rank, world, local):
@@ -327,42 +399,17 @@ def run_ours(args, rank, world, local):
            "h2d_bytes_per_step": int(pin_t.numel() * 4 + pin_l.numel() * 4), "d2h_bytes_per_step": 4,
            "ms_per_step": e2e_ms, "path": "DenseNet.step captured in a CUDA graph, replayed per step"}
 
-    # roofline of the dominant kernel
+    # roofline of the dominant kernel, and of every kernel kind of the step
     pk, pk_src = peaks()
     Mp = max(8, 1 << (cfg["layers"][0]["M"] - 1).bit_length())
     npass = {"x3": 3, "bf16": 1, "f32": 1}[args.math]
     per_kind = {k: (v[0] / v[1], v[1] // n_kt) for k, v in kt.items() if v[1] > 0}
     dom = max(kt, key=lambda k: kt[k][0])
     sizes = n.sizes
-    roof = None
-    if dom in ("gemm_fwd_scan", "gemm_dW", "gemm_dS_gradt") and args.math != "f32":
-        # per-launch flops of this kind summed over layers / launches of the kind
-        algo, dense = 0.0, 0.0
-        for l in range(len(sizes) - 1):
-            n_in, n_out = sizes[l], sizes[l + 1]
-            if dom == "gemm_dS_gradt" and l == 0:
-                continue
-            algo += 2 * 2 * B * n_in * n_out
-            r_out = (n_out + 127) // 128 * 128
-            r_in = (n_in + 127) // 128 * 128
-            k_in = (n_in + 63) // 64 * 64
-            k_out = (n_out + 63) // 64 * 64
-            cols = B * Mp
-            dense += 2 * npass * {"gemm_fwd_scan": r_out * cols * k_in, "gemm_dW": r_out * r_in * cols,
-                                  "gemm_dS_gradt": r_in * cols * k_out}[dom]
-        nl = per_kind[dom][1]
-        t_avg = per_kind[dom][0] / 1000.0
-        peak = pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
-        achieved = algo / nl / t_avg / 1e12
-        roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": None,
-                "dense_achieved": dense / nl / t_avg / 1e12, "dense_frac": dense / nl / t_avg / 1e12 / peak,
-                "peak_source": f"{pk_src} bf16 (burst)",
-                "note": "achieved = method flops (2 grid weights per input spike); dense_* = tensor-core flops "
-                        "issued by the dense formulation (Mp/2 x the method's, x3 for the three-product split)"}
-    else:
-        roof = {"kernel": dom, "bound": "hbm", "achieved": None, "peak": pk.get("hbm_gbs"), "unit": "GB/s",
-                "frac": None, "traffic": None, "peak_source": pk_src}
+    rooflines = kind_rooflines(per_kind, sizes, B, Mp, npass, args.math, pk, pk_src)
+    roof = dict(rooflines.get(dom, {"bound": None, "achieved": None, "peak": None, "unit": None, "frac": None}))
+    roof["kernel"] = dom
+    roof["traffic"] = TRAFFIC_PER_LAUNCH.get((dom, args.math))
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -371,7 +418,7 @@ def run_ours(args, rank, world, local):
             "config": {"workload": WORKLOAD, "global_batch": B * world, "per_gpu_batch": B, "M": 32,
                        "layers": [784, 800, 800, 10], "math": args.math, "l2": "flushed (512 MB write) before each "
                        "timed step", "parallelism": "replicas" if world > 1 else "single"},
-            "roofline": roof, "clocks": clk, "e2e": e2e,
+            "roofline": roof, "rooflines": rooflines, "clocks": clk, "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps,
             "gpu_launches_counted_eager": {"steps": n_kt, "launches": counted},
             "kernel_ms": {k: round(v[0], 5) for k, v in per_kind.items()},
