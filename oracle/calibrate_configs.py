@@ -2,18 +2,18 @@
 
 Finds, by bisection with the float64 oracle, the weight mean mu_l for which
 80% of layer l's neurons fire at initialisation on the seed-0 input batch
-(M = 32, t_offset = 0); layer l sees the previous layer's calibrated output.
-Prints the values that the workload definitions freeze (CFG2_MU and
-CFG3_MU_TIMES_N). Calls only the oracle and the seeded generators.
+(t_offset = 0); layer l sees the previous layer's calibrated output. Prints
+the values that the workload definitions freeze (CFG2_MU, CFG3_MU_TIMES_N,
+CFG4_MU, CFG5_MU). Calls only the oracle and the seeded generators.
 
-    python -m oracle.calibrate_configs
+    python -m oracle.calibrate_configs [2] [3] [4] [5]
 """
 
 import math
 
 import numpy as np
 
-from oracle import dstd, losses
+from oracle import dstd, lif, losses, network
 from paper_2607_14672_gb300 import synth
 
 
@@ -50,6 +50,75 @@ def calibrate_cfg3():
     return out
 
 
+def _fired_fraction(what, T, dt, tau_v, tau_I, v_th=1.0):
+    """Share of neurons whose v^ reaches v_th on some interval (the interval
+    maxima of Tab. timing_DSTD's potential, without solving for the time)."""
+    M = T.size - 1
+    lo, hi = T[:M], T[1:M + 1]
+    c = lif.interval_coeffs(lif.lif_case(tau_v, tau_I), tau_v, tau_I, np.broadcast_to(lo, what.shape), what, T[0])
+    return float(np.mean(np.any(lif.interval_peak(c, lo, hi) >= v_th, axis=-1)))
+
+
+def _bisect(frac, target=0.8, lo=-0.5, hi=0.5, iters=26):
+    """mu with frac(mu) ~ target; frac increases with mu. The bracket is
+    widened first until it holds the target."""
+    for _ in range(12):
+        if frac(hi) >= target:
+            break
+        lo, hi = hi, 2.0 * hi
+    for _ in range(12):
+        if frac(lo) < target:
+            break
+        lo, hi = 2.0 * lo, lo
+    for _ in range(iters):
+        mu = 0.5 * (lo + hi)
+        lo, hi = (mu, hi) if frac(mu) < target else (lo, mu)
+    return 0.5 * (lo + hi)
+
+
+def calibrate_conv(cfg, batch, verbose=True):
+    """mu_l for a conv stack (configs 4, 5): w^(mu) = w^(Z) + mu w^(ones) by
+    linearity of the contraction, so each bisection step only re-evaluates
+    the interval maxima; the chosen mu's spike times feed the next layer."""
+    t = cfg["inputs"](B=batch)
+    mus = []
+    for l, L in enumerate(cfg["layers"], start=1):
+        T, dt = dstd.grid(L["t_first"], L["t_end"], L["M"], 0.0)
+        tv, ti = L["tau_v"], L["tau_I"]
+        B = t.shape[0]
+        if L["kind"] == "conv":
+            C, H, Wd = t.shape[1:]
+            Z = synth.normal_weights(1000 + l, L["W"].shape, 0.0, 1.0 / math.sqrt(C * 9))
+            s = dstd.binning(t.reshape(B, -1), T, dt, tv, ti).reshape(B, L["M"], C, H, Wd)
+            A = network.conv_what(s, Z, L["stride"], L["pad"])
+            U = network.conv_what(s, np.ones((1,) + Z.shape[1:]), L["stride"], L["pad"])
+            shape = A.shape
+            A, U = A.reshape(B, -1, L["M"]), U.reshape(B, -1, L["M"])
+            Ur = np.broadcast_to(U.reshape(B, 1, -1, L["M"]), (B, shape[1], shape[2] * shape[3], L["M"])).reshape(A.shape)
+        else:
+            x = t.reshape(B, -1)
+            Z = synth.normal_weights(1000 + l, L["W"].shape, 0.0, 1.0 / math.sqrt(x.shape[1]))
+            s = dstd.binning(x, T, dt, tv, ti)
+            A = np.einsum("bmj,ij->bim", s, Z)
+            Ur = np.broadcast_to(np.einsum("bmj->bm", s)[:, None, :], A.shape)
+        mu = _bisect(lambda m: _fired_fraction(A + m * Ur, T, dt, tv, ti))
+        mus.append(mu)
+        ctx = dstd.solve(A + mu * Ur, T, dt, tv, ti, 1.0)
+        t = ctx["t"].reshape((B,) + tuple(shape[1:4])) if L["kind"] == "conv" else ctx["t"]
+        if verbose:
+            print(f"layer {l}: mu {mu:.5f}, fired {np.isfinite(ctx['t']).mean():.3f}", flush=True)
+    return mus
+
+
 if __name__ == "__main__":
-    print("CFG2_MU", [round(m, 5) for m in calibrate_cfg2()])
-    print("CFG3 mu*N", [round(m, 2) for m in calibrate_cfg3()])
+    import sys
+    from paper_2607_14672_gb300 import configs
+    which = sys.argv[1:] or ["2", "3", "4", "5"]
+    if "2" in which:
+        print("CFG2_MU", [round(m, 5) for m in calibrate_cfg2()])
+    if "3" in which:
+        print("CFG3 mu*N", [round(m, 2) for m in calibrate_cfg3()])
+    if "4" in which:
+        print("CFG4_MU", tuple(round(m, 5) for m in calibrate_conv(configs.config4(), batch=2)))
+    if "5" in which:
+        print("CFG5_MU", tuple(round(m, 5) for m in calibrate_conv(configs.config5(), batch=1)))

@@ -21,10 +21,10 @@ Layer l's window is [l tau_shift - tau_margin, l tau_shift + tau_width + tau_mar
 and its penalty edges t_head^(l) = l tau_shift + t_head,
 t_tail^(l) = l tau_shift + tau_width - t_tail.
 
-Weight means mu_l (dense configs 2 and 3) make about 80% of each layer's
-neurons fire at initialisation on the seed-0 batch with M = 32 and
-t_offset = 0; they were found once by bisection with the oracle
-(``oracle/calibrate_configs.py``) and are frozen here.
+Weight means mu_l (configs 2-5) make about 80% of each layer's neurons fire
+at initialisation on the seed-0 batch with t_offset = 0; they were found once
+by bisection with the oracle (``oracle/calibrate_configs.py``) and are frozen
+here.
 """
 
 import math
@@ -44,6 +44,9 @@ SEED_INPUT, SEED_W, SEED_LABELS, SEED_OFFSET = 0, 1000, 7, 11
 # frozen calibration (80% firing at init), see module docstring
 CFG2_MU = (0.03523, 0.01520, 0.01951)
 CFG3_MU_TIMES_N = 17.4
+CFG4_MU = (0.09306, 0.00761, 0.01274, 0.01387, 0.00942, 0.00637, 0.00514, 0.00285, 0.00093)
+CFG5_MU = (0.96918, 0.01896, 0.02438, 0.0258, 0.02676, 0.02719, 0.02923, 0.01346, 0.01353, 0.01343,
+           0.01367, 0.01382, 0.01358, 0.01714, 0.00673, 0.00686, 0.00689, 0.00699, 0.00697, 0.00077)
 
 
 def synfire_layer(l, syn=SYNFIRE):
@@ -113,6 +116,75 @@ def config3(N, M, batch=128, tau=(0.4, 0.2)):
         batch=batch, in_shape=(N,), loss="sum_t", tau_soft=None,
         inputs=lambda seed=SEED_INPUT, B=batch: synth.uniform_spikes(seed, (B, N), 0.0, 1.0, 0.1),
         layers=[_dense(W, tau[0], tau[1], M, 0.0, 1.0)])
+
+
+def _conv(W, tau_v, tau_I, M, stride, in_shape, **kw):
+    d = _dense(W, tau_v, tau_I, M, **kw)
+    d.update(kind="conv", stride=stride, pad=1, in_shape=tuple(in_shape))
+    return d
+
+
+def conv_stack(in_shape, channels, strides, n_classes, tau, M, mus, seed_w=SEED_W):
+    """3x3 conv layers (pad 1, i.e. silent padding) then a dense readout.
+
+    Layer l (1-based) has W = mu_l + N(0, 1/fan_in), fan_in = C_in * 9 for a
+    conv layer and the flattened (C, H, W) size for the readout, and the
+    synfire window of layer l. Returns the layer dicts and the output shape
+    of every layer.
+    """
+    C, H, Wd = in_shape
+    layers, shapes = [], []
+    for l, (co, st) in enumerate(zip(channels, strides), start=1):
+        W = synth.normal_weights(seed_w + l, (co, C, 3, 3), mus[l - 1], 1.0 / math.sqrt(C * 9))
+        layers.append(_conv(W, tau[0], tau[1], M, st, (C, H, Wd), **synfire_layer(l)))
+        H, Wd = (H + 2 - 3) // st + 1, (Wd + 2 - 3) // st + 1
+        C = co
+        shapes.append((C, H, Wd))
+    l = len(channels) + 1
+    n_in = C * H * Wd
+    W = synth.normal_weights(seed_w + l, (n_classes, n_in), mus[l - 1], 1.0 / math.sqrt(n_in))
+    layers.append(_dense(W, tau[0], tau[1], M, **synfire_layer(l)))
+    shapes.append((n_classes,))
+    return layers, shapes
+
+
+def config4(batch=128, M=32):
+    """9-layer conv TTFS SNN on 32x32x3 inputs (Syn-SNN-9 shapes), B = 128, M = 32.
+
+    3x3 convs with channels 64-64-128-128-256-256-512-512, stride 2 at layers
+    2, 4 and 6 (32 -> 16 -> 8 -> 4), then a dense 8192 -> 10 readout;
+    (tau_m, tau_s) = (inf, inf); pixels x ~ U[0,1), t = 1 - x; bf16 operands
+    with fp32 accumulation and state; CE + T + Q with AdamW.
+    """
+    chans = [64, 64, 128, 128, 256, 256, 512, 512]
+    strides = [1, 2, 1, 2, 1, 2, 1, 1]
+    layers, shapes = conv_stack((3, 32, 32), chans, strides, 10, (INF, INF), M, CFG4_MU)
+    return dict(
+        name="cfg4", workload=f"conv LIF TTFS SNN 9 layers on 32x32x3, B={batch}, M={M}, tau=(inf,inf), bf16",
+        batch=batch, in_shape=(3, 32, 32), loss="ce", tau_soft=SYNFIRE["tau_soft"], n_classes=10, math="bf16",
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.intensity_spikes(seed, (B, 3, 32, 32), 0.0, SYNFIRE["tau_in"]),
+        labels=lambda seed=SEED_LABELS, B=batch: synth.labels(seed, B, 10),
+        layers=layers, shapes=shapes)
+
+
+def config5(batch=256, M=64):
+    """20-layer conv TTFS SNN on 28x28x1 inputs (Syn-SNN-20 shapes), B = 256, M = 64.
+
+    19 3x3 convs with 64 channels (layers 1-6), 128 (7-13) and 256 (14-19),
+    stride 2 at layers 7 and 14 (28 -> 14 -> 7), then a dense 12544 -> 10
+    readout; (tau_m, tau_s) = (1.0, 0.25) = (4 tau_s, tau_s); staggered
+    synfire windows (tau_shift = 0.1); pixels x ~ U[0,1), t = 1 - x; bf16
+    operands; CE + T + Q with AdamW.
+    """
+    chans = [64] * 6 + [128] * 7 + [256] * 6
+    strides = [1] * 6 + [2] + [1] * 6 + [2] + [1] * 5
+    layers, shapes = conv_stack((1, 28, 28), chans, strides, 10, (1.0, 0.25), M, CFG5_MU)
+    return dict(
+        name="cfg5", workload=f"conv LIF TTFS SNN 20 layers on 28x28x1, B={batch}, M={M}, tau=(1.0,0.25), bf16",
+        batch=batch, in_shape=(1, 28, 28), loss="ce", tau_soft=SYNFIRE["tau_soft"], n_classes=10, math="bf16",
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.intensity_spikes(seed, (B, 1, 28, 28), 0.0, SYNFIRE["tau_in"]),
+        labels=lambda seed=SEED_LABELS, B=batch: synth.labels(seed, B, 10),
+        layers=layers, shapes=shapes)
 
 
 def draw_offsets(layers, seed=SEED_OFFSET):

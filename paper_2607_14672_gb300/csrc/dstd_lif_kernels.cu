@@ -656,12 +656,22 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
         atomicAdd(&count[i], 1.0f);
     }
     const long long abase = (long long)i * lda + (long long)b * c.Mp;
+    // K(x) at x = s0 + (q - m) dt. Away from the spike K = (e^{-av x} -
+    // e^{-aI x}) / lam (x e^{-av x} when lam = 0) with fast exponentials; the
+    // spike's own bin and the one before it (x < 2 dt, where that difference
+    // cancels) take the expm1 form.
+    const float Kq = (q < c.M) ? kernel_K(c, s0) : 0.f;
+    const float Kq1 = (q < c.M) ? kernel_K(c, s0 + c.dt) : 0.f;
     for (int m0 = 0; m0 < c.Mp; m0 += 8) {
         float v[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            int m = m0 + u;
-            v[u] = (q < c.M && m <= q) ? coef * kernel_K(c, s0 + (float)(q - m) * c.dt) : 0.f;
+            const int m = m0 + u;
+            const float x = s0 + (float)(q - m) * c.dt;
+            const float ev = __expf(-c.av * x);
+            const float Kf = c.lam_zero ? x * ev : (ev - __expf(-c.aI * x)) * c.inv_lam;
+            const float K = (m == q) ? Kq : ((m == q - 1) ? Kq1 : Kf);
+            v[u] = (q < c.M && m <= q) ? coef * K : 0.f;
         }
         if (OP == 0) {
             float4 *p = reinterpret_cast<float4 *>((float *)a_hi + abase + m0);

@@ -108,3 +108,132 @@ class DenseNet:
         if self.with_adamw:
             n += L
         return n
+
+
+class ConvNet:
+    """A stack of conv DSTD layers and a dense readout (configs 4 and 5) on one GPU.
+
+    Spike tensors are NHWC ([B, H, W, C]); filters are kept as [C_out, k, k,
+    C_in]. The layer dicts hold oracle-layout weights ([C_out, C_in, k, k]
+    filters; the readout's columns in (C, H, W) order), which the constructor
+    permutes once, so both sides compute the same network. T and Q of a conv
+    layer are normalised by B Ho Wo (App. C.1).
+    """
+
+    def __init__(self, cfg, math_mode=None, batch=None, device="cuda", with_adamw=True):
+        self.cfg = cfg
+        self.math = math_mode or cfg.get("math", "bf16")
+        self.B = B = int(batch or cfg["batch"])
+        self.layers = [dict(L) for L in cfg["layers"]]
+        dev = torch.device(device)
+        self.device = dev
+        C, H, Wd = cfg["in_shape"]
+        self.in_shape = (H, Wd, C)
+        self.W, self.p, self.t, self.g, self.saved, self.geom = [], [], [], [], [], []
+        ws = 0
+        shape = (H, Wd, C)
+        for L in self.layers:
+            Wl = torch.tensor(L["W"], dtype=torch.float32)
+            if L["kind"] == "conv":
+                Hh, Ww, Cc = shape
+                k, st, pad = Wl.shape[2], L["stride"], L["pad"]
+                Ho, Wo = dstd.conv_out_hw(Hh, Ww, k, st, pad)
+                Co = Wl.shape[0]
+                self.W.append(Wl.permute(0, 2, 3, 1).contiguous().to(dev))
+                p = dstd.params(L, penalty_norm=1.0 / (B * Ho * Wo))
+                need = dstd.conv_workspace_bytes(B, Hh, Ww, Cc, Co, k, st, pad, p, self.math)
+                self.geom.append((Hh, Ww, Cc, k, st, pad))
+                shape = (Ho, Wo, Co)
+                self.saved.append(torch.empty(dstd.dense_saved_bytes(B * Ho * Wo, Co), dtype=torch.uint8, device=dev))
+            else:
+                Hh, Ww, Cc = shape
+                n_out = Wl.shape[0]
+                # readout columns: oracle order (c, y, x) -> NHWC order (y, x, c)
+                Wl = Wl.reshape(n_out, Cc, Hh, Ww).permute(0, 2, 3, 1).reshape(n_out, -1) if Hh * Ww > 1 else Wl
+                self.W.append(Wl.contiguous().to(dev))
+                p = dstd.params(L, penalty_norm=1.0 / B)
+                need = dstd.dense_workspace_bytes(B, Hh * Ww * Cc, n_out, p, self.math)
+                self.geom.append(None)
+                shape = (n_out,)
+                self.saved.append(torch.empty(dstd.dense_saved_bytes(B, n_out), dtype=torch.uint8, device=dev))
+            if need == 0:
+                raise ValueError("unsupported layer sizes or constants for the library")
+            ws = max(ws, need)
+            self.p.append(p)
+            self.t.append(torch.empty((B,) + shape, dtype=torch.float32, device=dev))
+            self.g.append(torch.zeros((B,) + shape, dtype=torch.float32, device=dev))
+        self.t_in = torch.full((B, H, Wd, C), float("inf"), dtype=torch.float32, device=dev)
+        self.penalty = torch.zeros((len(self.W), 4), dtype=torch.float32, device=dev)
+        self.gW = [torch.empty_like(w) for w in self.W]
+        self.workspace = torch.empty(ws, dtype=torch.uint8, device=dev)
+        self.loss = torch.zeros(1, dtype=torch.float32, device=dev)
+        self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.with_adamw = with_adamw
+        if with_adamw:
+            self.m = [torch.zeros_like(w) for w in self.W]
+            self.v = [torch.zeros_like(w) for w in self.W]
+            self.adam_step = 0
+
+    def set_offsets(self, offsets):
+        for p, L, o in zip(self.p, self.layers, offsets):
+            p.t_offset = float(o)
+            L["t_offset"] = float(o)
+
+    def set_inputs(self, t0, labels=None):
+        """t0 in the oracle's [B, C, H, W] layout (or already NHWC via ``set_inputs_nhwc``)."""
+        x = torch.as_tensor(t0, dtype=torch.float32)
+        self.t_in.copy_(x.permute(0, 2, 3, 1), non_blocking=True)
+        if labels is not None:
+            self.labels.copy_(torch.as_tensor(labels, dtype=torch.int32), non_blocking=True)
+
+    def layer_input(self, l):
+        return self.t_in if l == 0 else self.t[l - 1]
+
+    def forward(self, stream=None):
+        for l, L in enumerate(self.layers):
+            x = self.layer_input(l)
+            if self.geom[l] is not None:
+                _, _, _, k, st, pad = self.geom[l]
+                dstd.conv_fwd(x, self.W[l], st, pad, self.p[l], self.math, self.t[l], self.saved[l],
+                              self.penalty[l], self.workspace, stream)
+            else:
+                dstd.dense_fwd(x.reshape(self.B, -1), self.W[l], self.p[l], self.math, self.t[l], self.saved[l],
+                               self.penalty[l], self.workspace, stream)
+
+    def loss_grad(self, stream=None):
+        dstd.ce_loss(self.t[-1], self.labels, self.cfg["tau_soft"], self.layers[-1]["t_end"], self.loss,
+                     self.g[-1], stream)
+
+    def backward(self, stream=None):
+        for l in range(len(self.layers) - 1, -1, -1):
+            x = self.layer_input(l)
+            g_in = self.g[l - 1] if l > 0 else None
+            if self.geom[l] is not None:
+                _, _, _, k, st, pad = self.geom[l]
+                dstd.conv_bwd(x, self.W[l], self.t[l], self.saved[l], self.g[l], st, pad, self.p[l], self.math,
+                              g_in, self.gW[l], self.workspace, stream)
+            else:
+                dstd.dense_bwd(x.reshape(self.B, -1), self.W[l], self.t[l], self.saved[l], self.g[l], self.p[l],
+                               self.math, None if g_in is None else g_in.reshape(self.B, -1), self.gW[l],
+                               self.workspace, stream)
+
+    def optimizer(self, lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=1e-2, stream=None):
+        self.adam_step += 1
+        for w, g, m, v in zip(self.W, self.gW, self.m, self.v):
+            dstd.adamw(w, g, m, v, lr, betas[0], betas[1], eps, weight_decay, self.adam_step, stream)
+
+    def step(self, stream=None):
+        """One training step: forward, loss, backward, AdamW."""
+        self.forward(stream)
+        self.loss_grad(stream)
+        self.backward(stream)
+        if self.with_adamw:
+            self.optimizer(stream=stream)
+
+    def objective(self):
+        return self.loss[0] + self.penalty[:, 0].sum() + self.penalty[:, 1].sum()
+
+    def dead_fraction(self):
+        """Share of silent neurons per layer on the last batch (from the Q counters)."""
+        pen = self.penalty.detach().cpu()
+        return (pen[:, 2] / (pen[:, 2] + pen[:, 3]).clamp(min=1.0)).tolist()
