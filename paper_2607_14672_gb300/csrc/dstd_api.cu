@@ -199,6 +199,7 @@ struct BwdWs {
                   *dB_lo = nullptr, *sT_hi = nullptr, *sT_lo = nullptr;
     float *wt32 = nullptr, *dA32 = nullptr, *dB32 = nullptr, *sT32 = nullptr, *DS = nullptr, *part = nullptr,
           *count = nullptr;
+    float4 *bw = nullptr;  // per-input bin index and kernel derivatives (input-time gradient)
     int ldt = 0, ldn = 0, ldbm = 0, ldp = 0, splits = 1;
     size_t bytes = 0;
 };
@@ -226,8 +227,8 @@ BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
     w.ldp = (N_in + 3) & ~3;
     w.splits = dw_splits(N_in, N_out, (int)cols, op);
     w.count = b.take<float>(N_out);
-    w.part = b.take<float>((size_t)w.splits * N_out * w.ldp);
     if (op == OpKind::F32) {
+        w.part = b.take<float>((size_t)w.splits * N_out * w.ldp);  // split-K partials (the tensor-core path adds atomically)
         w.dA32 = b.take<float>((size_t)N_out * w.ldbm);
         w.dB32 = b.take<float>((size_t)cols * w.ldn);
         w.sT32 = b.take<float>((size_t)N_in * w.ldbm);
@@ -246,6 +247,7 @@ BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
         if (need_gt) {
             w.wt_hi = b.take<__nv_bfloat16>((size_t)N_in * w.ldt);
             if (three) w.wt_lo = b.take<__nv_bfloat16>((size_t)N_in * w.ldt);
+            w.bw = b.take<float4>((size_t)B * N_in);
         }
     }
     w.bytes = b.off;
@@ -416,7 +418,7 @@ ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
     w.ldp = (pl.K + 3) & ~3;
     w.splits = dw_splits(pl.K, Cout, (int)cols, op);
     w.count = b.take<float>(Cout);
-    w.part = b.take<float>((size_t)w.splits * Cout * w.ldp);
+    // (dW adds into g_W atomically: no split-K partials)
     w.dA_hi = b.take<__nv_bfloat16>((size_t)Cout * w.ldbm);
     if (two) w.dA_lo = b.take<__nv_bfloat16>((size_t)Cout * w.ldbm);
     w.dB_hi = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
@@ -593,6 +595,11 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
         TRY(cu(launch_dwhat(t_out, sv.q, sv.s, sv.vdot, g_t_out, B, N_out, c, op, ws.dA_hi, ws.dA_lo, ws.ldbm,
                             ws.dB_hi, ws.dB_lo, ws.ldn, ws.count, st)));
     }
+    {
+        // s^T for dW, and the per-input kernel derivatives the dS epilogue needs
+        Timed tm(KK_BIN_T, st);
+        TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st, ws.bw)));
+    }
     if (need_gt) {
         {
             Timed tm(KK_PREP, st);
@@ -605,25 +612,23 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
         a.N = N_in;
         a.t_in = t_in;
         a.g_t_in = g_t_in;
+        a.bw = ws.bw;
         Timed tm(KK_GEMM_DS, st);
         TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dB_hi, ws.dB_lo, ws.ldn, N_in, (int)cols, N_out, 1, op,
                               Epi::GradT, a, st)));
     }
-    {
-        Timed tm(KK_BIN_T, st);
-        TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st)));
-    }
+    // dW = dw^T s: the split-K slices add into g_W (zeroed here); split 0
+    // also adds the dead-neuron term qcoef * count_i
+    TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)N_out * N_in, st)));
     TcEpiArgs a{};
-    a.D = ws.part;
-    a.ldd = ws.ldp;
-    a.zstride = (long long)N_out * ws.ldp;
-    {
-        Timed tm(KK_GEMM_DW, st);
-        TRY(cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, N_out, N_in, (int)cols,
-                              ws.splits, op, Epi::Store, a, st)));
-    }
-    Timed tm(KK_REDUCE, st);
-    return cu(launch_dw_reduce(ws.part, ws.splits, a.zstride, ws.ldp, N_out, N_in, ws.count, qcoef, g_W, st));
+    a.D = g_W;
+    a.ldd = N_in;
+    a.atomic = 1;
+    a.qcount = ws.count;
+    a.qcoef = qcoef;
+    Timed tm(KK_GEMM_DW, st);
+    return cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, N_out, N_in, (int)cols,
+                             ws.splits, op, Epi::Store, a, st));
 }
 
 int dstd_ce_loss(const float *t_L, const int32_t *labels, int B, int C, float tau_soft, float t_silent, float *loss,
@@ -777,18 +782,18 @@ int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const v
             Timed tm(KK_BIN_T, st);
             TRY(cu(launch_binning_im2col(t_in, pl.g, pos0, npos, c, bop, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st)));
         }
+        // dW over all chunks and split-K slices adds into g_W (zeroed before
+        // the first chunk); the last chunk's split 0 adds the dead-neuron term
+        if (ch == 0) TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)C_out * pl.K, st)));
         TcEpiArgs a{};
-        a.D = ws.part;
-        a.ldd = ws.ldp;
-        a.zstride = (long long)C_out * ws.ldp;
-        {
-            Timed tm(KK_GEMM_DW, st);
-            TRY(cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, C_out, pl.K, (int)cols,
-                                  ws.splits, bop, Epi::Store, a, st)));
-        }
-        Timed tm(KK_REDUCE, st);
-        TRY(cu(launch_dw_reduce(ws.part, ws.splits, a.zstride, ws.ldp, C_out, pl.K, last ? ws.count : nullptr, qcoef,
-                                g_W, st, ch > 0)));
+        a.D = g_W;
+        a.ldd = pl.K;
+        a.atomic = 1;
+        a.qcount = last ? ws.count : nullptr;
+        a.qcoef = qcoef;
+        Timed tm(KK_GEMM_DW, st);
+        TRY(cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, C_out, pl.K, (int)cols,
+                              ws.splits, bop, Epi::Store, a, st)));
     }
     return DSTD_OK;
 }

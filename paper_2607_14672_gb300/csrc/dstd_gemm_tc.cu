@@ -248,8 +248,24 @@ struct Cfg {
 __device__ __forceinline__ void store_chunk(const float (&v)[32], int row, int col0, int cc, int R, int Cn,
                                             const TcEpiArgs &a, int split) {
     if (row >= R) return;
-    float *D = a.D + (long long)split * a.zstride;
     const float rs = a.row_scale ? a.row_scale[row] : 1.0f;
+    if (a.atomic) {
+        const float add = (a.qcount && split == 0) ? a.qcoef * a.qcount[row] : 0.0f;
+        float *dst = a.D + (long long)row * a.ldd + col0 + cc;
+        if (col0 + cc + 32 <= Cn && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4)
+                atomicAdd(reinterpret_cast<float4 *>(dst + j), make_float4(fmaf(v[j], rs, add), fmaf(v[j + 1], rs, add),
+                                                                           fmaf(v[j + 2], rs, add),
+                                                                           fmaf(v[j + 3], rs, add)));
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (col0 + cc + j < Cn) atomicAdd(dst + j, fmaf(v[j], rs, add));
+        }
+        return;
+    }
+    float *D = a.D + (long long)split * a.zstride;
     float *dst = D + (long long)row * a.ldd + col0 + cc;
     if (col0 + cc + 32 <= Cn && (a.ldd % 4) == 0) {
 #pragma unroll
@@ -292,8 +308,15 @@ __device__ __forceinline__ void gradt_chunk(const float (&v)[32], int row, int c
             g = 0.f;
             w.k = -100;
             if (e >= 0) {
-                const float x = a.t_in[e];
-                if (isfinite(x)) w = bin_weights(c, x, true);
+                if (a.bw) {
+                    const float4 q = a.bw[e];
+                    w.k = __float_as_int(q.x);
+                    w.dR = q.y;
+                    w.dL = q.z;
+                } else {
+                    const float x = a.t_in[e];
+                    if (isfinite(x)) w = bin_weights(c, x, true);
+                }
             }
         }
         // the two grid points of the spike (m = k, k + 1), if in this block

@@ -278,8 +278,10 @@ cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bf
 //  !transposed: [B*Mp, ldk] (row (b,m), column j)    (contraction operand)
 //   transposed: [N, ldk'] with ldk' >= B*Mp (row j, column (b,m))
 // as bf16 hi/lo (BF16X3), bf16 hi (BF16) or fp32 (F32). Pad entries are 0.
+// With transposed and bw != null, also bw[b*N + j] = (k as int bits, ds/dt at
+// T_k, ds/dt at T_{k+1}, 0) per input (k = -100 when silent).
 cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKind op, bool transposed,
-                           void *hi, void *lo, int ld, cudaStream_t st);
+                           void *hi, void *lo, int ld, cudaStream_t st, float4 *bw = nullptr);
 // Convolution geometry: input [B, H, W, C] (NHWC), filter k x k, stride s,
 // zero-spike padding p, output [B, Ho, Wo, Cout]. An output position
 // pos = (b*Ho + y)*Wo + x plays the role of a sample; the contraction axis is
@@ -327,14 +329,18 @@ cudaError_t launch_sgemm_tn(const float *A, int lda, const float *Bm, int ldb, f
 enum class Epi { Store = 0, GradT = 1 };
 struct TcEpiArgs {
     const float *row_scale;  // per-row factor applied to the accumulator (Store, Scan), may be null
-    // Store
+    // Store: split z writes D + z*zstride, or with atomic != 0 every split
+    // adds into D (zeroed by the caller) and split 0 also adds
+    // qcoef * qcount[row] when qcount is given (the Q term of dW)
     float *D; long long ldd; long long zstride;
+    int atomic; const float *qcount; float qcoef;
     // GradT: layer constants and sizes (rows N, samples B)
     LifConst c; int B; int N;
     // GradT (rows = inputs j, columns = (b, m)); with conv != 0 the rows are
     // filter taps kidx, the columns (output position, m), and each result is
     // added atomically into the input element the tap reads (col2im)
     const float *t_in; float *g_t_in;
+    const float4 *bw;  // dense GradT: per-input (k, ds/dt at T_k, at T_{k+1}) from the binning, or null
     int conv; int pos0; ConvGeom g;
 };
 // A, B: 16-bit operands (bf16 for BF16X3 / BF16, fp16 for F16X3)

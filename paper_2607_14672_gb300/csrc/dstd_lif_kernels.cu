@@ -130,48 +130,85 @@ __device__ __forceinline__ void split_f16(float x, __half &hi, __half &lo) {
     lo = __float2half_rn(x - __half2float(hi));
 }
 
-__global__ void k_prep_weights_f16(const float *__restrict__ W, int R, int C, __half *hi, __half *lo, int ldo,
-                                   float *inv_scale, float *rowsum) {
-    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (warp >= R) return;
-    const float *w = W + (long long)warp * C;
+// One block per row: every load of the row is in flight at once (the row
+// is read once into registers, up to PREP_PER_THREAD values per thread, and
+// re-read from memory only for longer rows).
+constexpr int PREP_THREADS = 256, PREP_PER_THREAD = 8;
+
+__global__ void __launch_bounds__(PREP_THREADS) k_prep_weights_f16(const float *__restrict__ W, int R, int C,
+                                                                 __half *hi, __half *lo, int ldo, float *inv_scale,
+                                                                 float *rowsum) {
+    __shared__ float red_max[PREP_THREADS / 32], red_sum[PREP_THREADS / 32];
+    __shared__ float sc_sh;
+    const int r = blockIdx.x;
+    if (r >= R) return;
+    const float *w = W + (long long)r * C;
+    float x[PREP_PER_THREAD];
     float amax = 0.f, sum = 0.f;
-    for (int j = lane; j < C; j += 32) {
-        float x = w[j];
-        amax = fmaxf(amax, fabsf(x));
-        sum += x;
+#pragma unroll
+    for (int u = 0; u < PREP_PER_THREAD; ++u) {
+        const int j = threadIdx.x + u * PREP_THREADS;
+        x[u] = j < C ? w[j] : 0.f;
+        amax = fmaxf(amax, fabsf(x[u]));
+        sum += x[u];
+    }
+    for (int j = threadIdx.x + PREP_PER_THREAD * PREP_THREADS; j < C; j += PREP_THREADS) {
+        const float y = w[j];
+        amax = fmaxf(amax, fabsf(y));
+        sum += y;
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
         sum += __shfl_xor_sync(0xffffffffu, sum, o);
     }
-    // power of two bringing the row's largest |w| into [2^13, 2^14]
-    int k = 0;
-    if (amax > 0.f && isfinite(amax)) {
-        int e;
-        frexpf(amax, &e);  // amax = f 2^e, f in [0.5, 1)
-        k = 14 - e;
-        k = k > 100 ? 100 : (k < -100 ? -100 : k);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        red_max[warp] = amax;
+        red_sum[warp] = sum;
     }
-    const float sc = ldexpf(1.0f, k);
-    for (int j = lane; j < ldo; j += 32) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float m = 0.f, t = 0.f;
+        for (int k = 0; k < PREP_THREADS / 32; ++k) {
+            m = fmaxf(m, red_max[k]);
+            t += red_sum[k];
+        }
+        // power of two bringing the row's largest |w| into [2^13, 2^14]
+        int k = 0;
+        if (m > 0.f && isfinite(m)) {
+            int e;
+            frexpf(m, &e);  // m = f 2^e, f in [0.5, 1)
+            k = 14 - e;
+            k = k > 100 ? 100 : (k < -100 ? -100 : k);
+        }
+        sc_sh = ldexpf(1.0f, k);
+        inv_scale[r] = ldexpf(1.0f, -k);
+        if (rowsum) rowsum[r] = t;
+    }
+    __syncthreads();
+    const float sc = sc_sh;
+#pragma unroll
+    for (int u = 0; u < PREP_PER_THREAD; ++u) {
+        const int j = threadIdx.x + u * PREP_THREADS;
+        if (j < ldo) {
+            __half h, l;
+            split_f16(x[u] * sc, h, l);
+            hi[(long long)r * ldo + j] = h;
+            lo[(long long)r * ldo + j] = l;
+        }
+    }
+    for (int j = threadIdx.x + PREP_PER_THREAD * PREP_THREADS; j < ldo; j += PREP_THREADS) {
         __half h, l;
         split_f16(j < C ? w[j] * sc : 0.f, h, l);
-        hi[(long long)warp * ldo + j] = h;
-        lo[(long long)warp * ldo + j] = l;
-    }
-    if (lane == 0) {
-        inv_scale[warp] = ldexpf(1.0f, -k);
-        if (rowsum) rowsum[warp] = sum;
+        hi[(long long)r * ldo + j] = h;
+        lo[(long long)r * ldo + j] = l;
     }
 }
 
 cudaError_t launch_prep_weights_f16(const float *W, int R, int C, __half *hi, __half *lo, int ldo, float *inv_scale,
                                     float *rowsum, cudaStream_t st) {
-    const long long threads = (long long)R * 32;
-    k_prep_weights_f16<<<blocks_for(threads, 256), 256, 0, st>>>(W, R, C, hi, lo, ldo, inv_scale, rowsum);
+    k_prep_weights_f16<<<R, PREP_THREADS, 0, st>>>(W, R, C, hi, lo, ldo, inv_scale, rowsum);
     return cudaGetLastError();
 }
 
@@ -234,43 +271,61 @@ __global__ void k_binning_rows(const float *__restrict__ t, int B, int N, LifCon
     }
 }
 
-// transposed: row j, columns (b, m); one thread per (j, b) writes Mp
-// contiguous values with 16-byte stores.
+// transposed: row j, columns (b, m). A warp takes 32 consecutive samples of
+// one input j: each lane evaluates the grid weights of its own sample, then
+// the warp writes the 32 samples' Mp bins as consecutive 16-byte chunks
+// (lane l writes chunk l of each round, taking the weights of the chunk's
+// sample by shuffle), so every store instruction fills whole sectors. With
+// bw != null each lane also writes (k, ds/dt at T_k, ds/dt at T_{k+1}) of
+// its sample to bw[b*N + j] (k = -100 for a silent input) for the input-time
+// gradient.
 template <int OP>
-__global__ void k_binning_cols(const float *__restrict__ t, int B, int N, LifConst c, void *hi, void *lo,
-                               int ld) {
-    const int b = blockIdx.x * blockDim.x + threadIdx.x;
-    if (b >= B) return;
+__global__ void k_binning_cols(const float *__restrict__ t, int B, int N, LifConst c, void *hi, void *lo, int ld,
+                               float4 *bw) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int b0 = (blockIdx.x * (blockDim.x >> 5) + warp) * 32;
+    if (b0 >= B) return;
+    const int cps = c.Mp / 8;  // 8-bin chunks per sample
     for (int j = blockIdx.y; j < N; j += gridDim.y) {
+        const int b = b0 + lane;
         BinW w{-100, 0.f, 0.f, 0.f, 0.f};
-        float x = t[(long long)b * N + j];
-        if (isfinite(x)) w = bin_weights(c, x, false);
-        const long long base = (long long)j * ld + (long long)b * c.Mp;
-        for (int m0 = 0; m0 < c.Mp; m0 += 8) {
+        if (b < B) {
+            const float x = t[(long long)b * N + j];
+            if (isfinite(x)) w = bin_weights(c, x, bw != nullptr);
+            if (bw) bw[(long long)b * N + j] = make_float4(__int_as_float(w.k), w.dR, w.dL, 0.f);
+        }
+        const long long rowbase = (long long)j * ld + (long long)b0 * c.Mp;
+        for (int r = 0; r < cps; ++r) {
+            const int gc = r * 32 + lane;  // chunk of the warp's 32 samples
+            const int sl = gc / cps, ch = gc - sl * cps;
+            const int kk = __shfl_sync(0xffffffffu, w.k, sl);
+            const float wR = __shfl_sync(0xffffffffu, w.wR, sl);
+            const float wL = __shfl_sync(0xffffffffu, w.wL, sl);
+            if (b0 + sl >= B) continue;
             float v[8];
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-                int m = m0 + u;
-                v[u] = (m < c.M) ? ((m == w.k) ? w.wR : ((m == w.k + 1) ? w.wL : 0.f)) : 0.f;
+                const int m = ch * 8 + u;
+                v[u] = (m < c.M) ? ((m == kk) ? wR : ((m == kk + 1) ? wL : 0.f)) : 0.f;
             }
+            const long long off = rowbase + (long long)gc * 8;
             if (OP == 0) {
-                float4 *p = reinterpret_cast<float4 *>((float *)hi + base + m0);
+                float4 *p = reinterpret_cast<float4 *>((float *)hi + off);
                 p[0] = make_float4(v[0], v[1], v[2], v[3]);
                 p[1] = make_float4(v[4], v[5], v[6], v[7]);
             } else {
                 __align__(16) __nv_bfloat16 h[8], l[8];
 #pragma unroll
                 for (int u = 0; u < 8; ++u) split_bf16(v[u], h[u], l[u]);
-                *reinterpret_cast<uint4 *>((__nv_bfloat16 *)hi + base + m0) = *reinterpret_cast<uint4 *>(h);
-                if (OP == 1)
-                    *reinterpret_cast<uint4 *>((__nv_bfloat16 *)lo + base + m0) = *reinterpret_cast<uint4 *>(l);
+                *reinterpret_cast<uint4 *>((__nv_bfloat16 *)hi + off) = *reinterpret_cast<uint4 *>(h);
+                if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)lo + off) = *reinterpret_cast<uint4 *>(l);
             }
         }
     }
 }
 
 cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKind op, bool transposed, void *hi,
-                           void *lo, int ld, cudaStream_t st) {
+                           void *lo, int ld, cudaStream_t st, float4 *bw) {
     if (!transposed) {
         int pairs = (ld + 1) / 2;
         dim3 grid(blocks_for(pairs, 128), B);
@@ -280,9 +335,9 @@ cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKi
         else k_binning_rows<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
     } else {
         dim3 grid(blocks_for(B, 128), N < 65535 ? N : 65535);
-        if (op == OpKind::F32) k_binning_cols<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
-        else if (op == OpKind::BF16X3) k_binning_cols<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
-        else k_binning_cols<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
+        if (op == OpKind::F32) k_binning_cols<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
+        else if (op == OpKind::BF16X3) k_binning_cols<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
+        else k_binning_cols<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
     }
     return cudaGetLastError();
 }

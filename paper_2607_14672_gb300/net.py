@@ -103,7 +103,7 @@ class DenseNet:
         L = len(self.W)
         n = L * 4                                 # fwd: prep + binning + gemm (+ fused scan) + root solve / scan
         n += 1                                    # loss
-        n += L * 4                                # bwd: dw^ + binning^T + dW gemm + reduce
+        n += L * (3 if tc else 4)                 # bwd: dw^ + binning^T + dW gemm [+ split-K reduce]
         n += (L - 1) * (2 if tc else 3)           # bwd input times: prep W^T + dS gemm [+ gather]
         if self.with_adamw:
             n += L

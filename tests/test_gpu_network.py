@@ -145,8 +145,10 @@ def test_graph_replay_equals_eager():
     torch.cuda.synchronize()
     for a, b in zip(t_e, n.t):
         np.testing.assert_array_equal(a, host(b))
+    # dW adds its split-K slices with fp32 atomics, in whatever order they
+    # finish: equal to fp32 rounding, not bitwise
     for a, b in zip(gW_e, n.gW):
-        np.testing.assert_array_equal(a, host(b))
+        assert np.abs(a - host(b)).max() <= 1e-5 * np.abs(a).max()
 
 
 def test_kernel_timing_counts_launches():
