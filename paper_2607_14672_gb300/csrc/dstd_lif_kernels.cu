@@ -692,11 +692,20 @@ cudaError_t launch_scan_solve(const float *what, long long sb, long long si, lon
 //   A layout [N, lda]:    row i, columns (b, m)     (dW = dw^T . s)
 //   B layout [B*Mp, ldb]: row (b, m), column i      (dS = dw^ . W)
 // ---------------------------------------------------------------------------
+// Two adjacent lanes share one neuron (b, i): lane h = 0, 1 takes the
+// 16-byte chunks h, h+2, h+4, ... of its Mp bins, so that every 16-byte
+// store of the (i, (b, m)) layout is half of a sector the other lane fills in
+// the same instruction; the ((b, m), i) layout is written element-wise, 16
+// consecutive neurons per row and instruction.
 template <int OP>
 __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__ qv, const float *__restrict__ sv,
                         const float *__restrict__ vd, const float *__restrict__ g_up, int B, int N, LifConst c,
                         void *a_hi, void *a_lo, int lda, void *b_hi, void *b_lo, int ldb, float *count) {
-    long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    constexpr int EB = OP == 0 ? 4 : 2;  // bytes per element
+    constexpr int BPC = 16 / EB;         // bins per 16-byte chunk
+    const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const long long idx = tid >> 1;
+    const int h = (int)(tid & 1);
     if (idx >= (long long)B * N) return;
     const int b = (int)(idx / N), i = (int)(idx % N);
     const int q = qv[idx];
@@ -704,10 +713,10 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
     if (q < c.M) {
         float pv, pg;
         penalty_T(c, t_out[idx], pv, pg);
-        float g = (g_up ? g_up[idx] : 0.f) + pg;
+        const float g = (g_up ? g_up[idx] : 0.f) + pg;
         coef = -g / vd[idx];
         s0 = sv[idx];
-    } else if (count) {
+    } else if (count && h == 0) {
         atomicAdd(&count[i], 1.0f);
     }
     const long long abase = (long long)i * lda + (long long)b * c.Mp;
@@ -717,10 +726,12 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
     // cancels) take the expm1 form.
     const float Kq = (q < c.M) ? kernel_K(c, s0) : 0.f;
     const float Kq1 = (q < c.M) ? kernel_K(c, s0 + c.dt) : 0.f;
-    for (int m0 = 0; m0 < c.Mp; m0 += 8) {
-        float v[8];
+    const int nch = c.Mp / BPC;
+    for (int ch = h; ch < nch; ch += 2) {
+        const int m0 = ch * BPC;
+        float v[BPC];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < BPC; ++u) {
             const int m = m0 + u;
             const float x = s0 + (float)(q - m) * c.dt;
             const float ev = __expf(-c.av * x);
@@ -729,22 +740,20 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
             v[u] = (q < c.M && m <= q) ? coef * K : 0.f;
         }
         if (OP == 0) {
-            float4 *p = reinterpret_cast<float4 *>((float *)a_hi + abase + m0);
-            p[0] = make_float4(v[0], v[1], v[2], v[3]);
-            p[1] = make_float4(v[4], v[5], v[6], v[7]);
+            *reinterpret_cast<float4 *>((float *)a_hi + abase + m0) = make_float4(v[0], v[1], v[2], v[3]);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) ((float *)b_hi)[((long long)b * c.Mp + m0 + u) * ldb + i] = v[u];
+            for (int u = 0; u < BPC; ++u) ((float *)b_hi)[((long long)b * c.Mp + m0 + u) * ldb + i] = v[u];
         } else {
-            __align__(16) __nv_bfloat16 h[8], l[8];
+            __align__(16) __nv_bfloat16 hh[BPC], ll[BPC];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) split_bf16(v[u], h[u], l[u]);
-            *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + abase + m0) = *reinterpret_cast<uint4 *>(h);
-            if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + abase + m0) = *reinterpret_cast<uint4 *>(l);
+            for (int u = 0; u < BPC; ++u) split_bf16(v[u], hh[u], ll[u]);
+            *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + abase + m0) = *reinterpret_cast<uint4 *>(hh);
+            if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + abase + m0) = *reinterpret_cast<uint4 *>(ll);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                long long o = ((long long)b * c.Mp + m0 + u) * ldb + i;
-                ((__nv_bfloat16 *)b_hi)[o] = h[u];
-                if (OP == 1) ((__nv_bfloat16 *)b_lo)[o] = l[u];
+            for (int u = 0; u < BPC; ++u) {
+                const long long o = ((long long)b * c.Mp + m0 + u) * ldb + i;
+                ((__nv_bfloat16 *)b_hi)[o] = hh[u];
+                if (OP == 1) ((__nv_bfloat16 *)b_lo)[o] = ll[u];
             }
         }
     }
@@ -757,7 +766,7 @@ cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const
         cudaError_t e = cudaMemsetAsync(silent_count, 0, sizeof(float) * N, st);
         if (e != cudaSuccess) return e;
     }
-    long long n = (long long)B * N;
+    long long n = 2ll * B * N;  // two lanes per neuron
     unsigned g = blocks_for(n, 256);
     if (op == OpKind::F32)
         k_dwhat<0><<<g, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, b_hi, b_lo, ldb, silent_count);
@@ -863,8 +872,68 @@ __global__ void k_ce_loss(const float *__restrict__ t, const int32_t *__restrict
     if ((threadIdx.x & 31) == 0 && v != 0.f) atomicAdd(loss, v);
 }
 
+// Batches of up to 1024 samples and up to 32 classes: one block, one thread
+// per sample with its row in registers, a block reduction, the loss written
+// directly (no zeroing launch, no atomics).
+constexpr int CE_MAX_C = 32;
+__global__ void __launch_bounds__(1024) k_ce_loss_block(const float *__restrict__ t, const int32_t *__restrict__ lab,
+                                                        int B, int C, float tau_soft, float t_silent, float *loss,
+                                                        float *g) {
+    __shared__ float part[32];
+    const int b = threadIdx.x;
+    const float inv_tau = 1.0f / tau_soft;
+    float contrib = 0.f;
+    if (b < B) {
+        const float *tb = t + (long long)b * C;
+        float z[CE_MAX_C];
+        bool fin[CE_MAX_C];
+        const int y = lab[b];
+        float zmax = -INFINITY, zy = 0.f;
+#pragma unroll
+        for (int k = 0; k < CE_MAX_C; ++k) {
+            if (k < C) {
+                const float x = tb[k];
+                fin[k] = isfinite(x);
+                z[k] = -(fin[k] ? x : t_silent) * inv_tau;
+                zmax = fmaxf(zmax, z[k]);
+                if (k == y) zy = z[k];
+            }
+        }
+        float den = 0.f;
+#pragma unroll
+        for (int k = 0; k < CE_MAX_C; ++k) {
+            if (k < C) {
+                z[k] = expf(z[k] - zmax);  // e_k = exp(z_k - zmax)
+                den += z[k];
+            }
+        }
+        const float inv_den = 1.0f / den;
+        const float scale = -inv_tau / (float)B;
+#pragma unroll
+        for (int k = 0; k < CE_MAX_C; ++k) {
+            if (k < C) {
+                const float p = z[k] * inv_den;
+                g[(long long)b * C + k] = fin[k] ? scale * (p - (k == y ? 1.f : 0.f)) : 0.f;
+            }
+        }
+        contrib = -(zy - zmax - logf(den)) / (float)B;
+    }
+    const float v = warp_sum(contrib);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = v;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        float u = threadIdx.x < (int)((blockDim.x + 31) >> 5) ? part[threadIdx.x] : 0.f;
+        u = warp_sum(u);
+        if (threadIdx.x == 0) loss[0] = u;
+    }
+}
+
 cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
                            float *loss, float *g, cudaStream_t st) {
+    if (B <= 1024 && C <= CE_MAX_C) {
+        k_ce_loss_block<<<1, (B + 31) / 32 * 32, 0, st>>>(t, lab, B, C, tau_soft, t_silent, loss, g);
+        return cudaGetLastError();
+    }
     cudaError_t e = cudaMemsetAsync(loss, 0, sizeof(float), st);
     if (e != cudaSuccess) return e;
     k_ce_loss<<<blocks_for(B, 128), 128, 0, st>>>(t, lab, B, C, tau_soft, t_silent, loss, g);
