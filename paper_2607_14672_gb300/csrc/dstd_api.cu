@@ -204,6 +204,19 @@ struct BwdWs {
     size_t bytes = 0;
 };
 
+// split-K factor of the forward contraction: enough splits to give every SM
+// a tile when the output has fewer tiles than SMs, each split at least two
+// 64-deep K slices
+int fwd_splits(int N_out, long long cols, int N_in) {
+    const long long tiles = (long long)((N_out + 127) / 128) * ((cols + 127) / 128);
+    const int ktiles = (N_in + 63) / 64;
+    long long s = tiles >= 152 ? 1 : 152 / tiles;
+    if (s > ktiles / 2) s = ktiles / 2;
+    if (s < 1) s = 1;
+    while (s > 1 && !tc_gemm_splits_valid(N_in, (int)s)) --s;
+    return (int)s;
+}
+
 int dw_splits(int N_in, int N_out, int K, OpKind op) {
     const int tm = op == OpKind::F32 ? 64 : 128, tn = op == OpKind::F32 ? 64 : 128;
     const long long tiles = (long long)((N_out + tm - 1) / tm) * ((N_in + tn - 1) / tn);
@@ -328,14 +341,19 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
                                  Epi::Store, a, st));
     }
     // w^ with rows i and columns (b, m): the Mp bins of a neuron are 128
-    // contiguous bytes (Mp = 32) that the scan reads with 16-byte loads
+    // contiguous bytes (Mp = 32) that the scan reads with 16-byte loads. With
+    // fewer output tiles than SMs (a narrow layer) K is split across CTAs
+    // whose partial sums add into w^ (zeroed first).
     {
+        const int splits = fwd_splits(N_out, cols, N_in);
+        if (splits > 1) TRY(cu(cudaMemsetAsync(ws.D, 0, sizeof(float) * (size_t)N_out * cols, st)));
         Timed tm(KK_GEMM_FWD, st);
         a.D = ws.D;
         a.ldd = cols;
         a.zstride = 0;
-        TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, 1, op,
-                              Epi::Store, a, st)));
+        a.atomic = splits > 1;
+        TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, splits,
+                              op, Epi::Store, a, st)));
     }
     Timed tm(KK_SCAN, st);
     return cu(launch_scan_solve(ws.D, c.Mp, cols, 1, B, N_out, c, nullptr, ws.rowsum, t_out, sv->q, sv->s,
@@ -600,7 +618,11 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
         Timed tm(KK_BIN_T, st);
         TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st, ws.bw)));
     }
-    if (need_gt) {
+    if (need_gt && N_out <= kGradtSmallMaxOut) {
+        // few outputs: the input-time gradient by its definition, no contraction
+        Timed tm(KK_GT, st);
+        TRY(cu(launch_gradt_small(W, N_out, N_in, B, c, ws.bw, ws.dA_hi, ws.dA_lo, ws.ldbm, g_t_in, st)));
+    } else if (need_gt) {
         {
             Timed tm(KK_PREP, st);
             TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, ws.wt_hi, ws.wt_lo, ws.ldt, nullptr,

@@ -309,6 +309,13 @@ cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const
                          int B, int N, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda,
                          void *b_hi, void *b_lo, int ldb, float *silent_count, cudaStream_t st,
                          bool accumulate_count = false);
+// g_t_in of a layer with few outputs (N_out <= kGradtSmallMaxOut) directly
+// from W, dw^ (operand layout [N_out, ld] over (b, m), hi/lo or hi only) and
+// the per-input bin index / kernel derivatives bw.
+constexpr int kGradtSmallMaxOut = 32;
+cudaError_t launch_gradt_small(const float *W, int N_out, int N_in, int B, const LifConst &c, const float4 *bw,
+                               const __nv_bfloat16 *d_hi, const __nv_bfloat16 *d_lo, int ld, float *g_t_in,
+                               cudaStream_t st);
 // g_t_in from dS stored as D[j, (b,m)] (row stride ldd)
 cudaError_t launch_gt_from_ds(const float *D, long long ldd, const float *t_in, int B, int N, const LifConst &c,
                               float *g_t_in, cudaStream_t st);

@@ -803,6 +803,42 @@ cudaError_t launch_gt_from_ds(const float *D, long long ldd, const float *t_in, 
     return cudaGetLastError();
 }
 
+// Input-time gradient of a layer with few outputs, straight from its
+// definition: g_t[b, j] = sum_n W[n, j] (dw^[b, n, k] ds_k/dt + dw^[b, n, k+1]
+// ds_{k+1}/dt) over the two grid points k, k+1 of input j (the derivative of
+// Tab. DSTD_kernels), with k and the derivatives from the transposed binning
+// (bw) and dw^ from its (n, (b, m)) operand layout, fp32 = hi + lo. One
+// thread per (b, j); 2 N_out multiply-adds each.
+__global__ void k_gradt_small(const float *__restrict__ W, int N_out, int N_in, int B, LifConst c,
+                              const float4 *__restrict__ bw, const __nv_bfloat16 *__restrict__ d_hi,
+                              const __nv_bfloat16 *__restrict__ d_lo, int ld, float *g_t_in) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)B * N_in) return;
+    const int b = (int)(idx / N_in), j = (int)(idx % N_in);
+    const float4 q = bw[idx];
+    const int k = __float_as_int(q.x);
+    const bool in0 = k >= 0 && k < c.M, in1 = k + 1 >= 0 && k + 1 < c.M;
+    float g = 0.f;
+    if (in0 || in1) {
+        for (int n = 0; n < N_out; ++n) {
+            const long long base = (long long)n * ld + (long long)b * c.Mp + k;
+            float d0 = 0.f, d1 = 0.f;
+            if (in0) d0 = __bfloat162float(d_hi[base]) + (d_lo ? __bfloat162float(d_lo[base]) : 0.f);
+            if (in1) d1 = __bfloat162float(d_hi[base + 1]) + (d_lo ? __bfloat162float(d_lo[base + 1]) : 0.f);
+            g = fmaf(W[(long long)n * N_in + j], fmaf(d0, q.y, d1 * q.z), g);
+        }
+    }
+    g_t_in[idx] = g;
+}
+
+cudaError_t launch_gradt_small(const float *W, int N_out, int N_in, int B, const LifConst &c, const float4 *bw,
+                               const __nv_bfloat16 *d_hi, const __nv_bfloat16 *d_lo, int ld, float *g_t_in,
+                               cudaStream_t st) {
+    long long n = (long long)B * N_in;
+    k_gradt_small<<<blocks_for(n, 256), 256, 0, st>>>(W, N_out, N_in, B, c, bw, d_hi, d_lo, ld, g_t_in);
+    return cudaGetLastError();
+}
+
 __global__ void k_dw_reduce(const float *__restrict__ part, int splits, long long zstride, int ldp, int R, int C,
                             const float *__restrict__ count, float qcoef, float *g_W, int accumulate) {
     long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;

@@ -104,7 +104,9 @@ class DenseNet:
         n = L * 4                                 # fwd: prep + binning + gemm (+ fused scan) + root solve / scan
         n += 1                                    # loss
         n += L * (3 if tc else 4)                 # bwd: dw^ + binning^T + dW gemm [+ split-K reduce]
-        n += (L - 1) * (2 if tc else 3)           # bwd input times: prep W^T + dS gemm [+ gather]
+        for l in range(1, L):                     # bwd input times: prep W^T + dS gemm [+ gather],
+            small = tc and self.sizes[l + 1] <= 32  # or one direct kernel for a layer with few outputs
+            n += 1 if small else (2 if tc else 3)
         if self.with_adamw:
             n += L
         return n
