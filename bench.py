@@ -222,9 +222,16 @@ class ClockSampler:
 # in profiles/launches_cfg2_step.md); to be set to None when the kernel
 # changes after that capture.
 TRAFFIC_PER_LAUNCH = {
-    ("gemm_dW", "x3"): 44.1e6,
-    ("gemm_fwd_scan", "x3"): 27.8e6,
+    ("gemm_dW", "x3"): 45.4e6,
+    ("gemm_fwd_scan", "x3"): 28.0e6,
+    ("gemm_dS_gradt", "x3"): 32.2e6,
     ("scan_solve", "x3"): 17.6e6,
+    ("dwhat", "x3"): 2.9e6,
+    ("binning", "x3"): 0.83e6,
+    ("binning_T", "x3"): 0.83e6,
+    ("gradt_gather", "x3"): 3.6e6,
+    ("prep_weights", "x3"): 1.9e6,
+    ("loss", "x3"): 0.04e6,
 }
 
 
@@ -410,6 +417,8 @@ def run_ours(args, rank, world, local):
     roof = dict(rooflines.get(dom, {"bound": None, "achieved": None, "peak": None, "unit": None, "frac": None}))
     roof["kernel"] = dom
     roof["traffic"] = TRAFFIC_PER_LAUNCH.get((dom, args.math))
+    for k, r in rooflines.items():
+        r["traffic"] = TRAFFIC_PER_LAUNCH.get((k, args.math))
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
