@@ -29,7 +29,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "DSTD LIF fwd+bwd samples/s at 1 GB300; % of tensor/HBM roofline; peak mem"
 UNIT = "samples/s"
-WORKLOAD = "dense LIF TTFS MLP 784-800-800-10, B=256, M=32, tau=(0.5,0.25), synfire CE+T+Q, fwd+bwd"
+WORKLOAD = "dense LIF TTFS MLP 784-800-800-10, B=256, M=32, tau=(0.5,0.25), synfire CE+T+Q, fwd+bwd+AdamW"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -242,7 +242,7 @@ def kind_rooflines(per_kind, sizes, B, Mp, npass, math_mode, pk, pk_src):
     weights per input spike: 4 B N_in N_out per contraction) per launch /
     time; dense_* = the tensor-core flops the dense formulation issues (Mp/2
     times that, times npass for the three-product split). Binning, scan/solve,
-    dw^, the split-K reduction and weight prep are HBM-bound: achieved = the
+    dw^, the split-K reduction, weight prep and AdamW are HBM-bound: achieved = the
     bytes the kernel must move (inputs read once, outputs written once) /
     time.
     """
@@ -265,6 +265,7 @@ def kind_rooflines(per_kind, sizes, B, Mp, npass, math_mode, pk, pk_src):
         add(algo_b, "dwhat", B * no * 20 + 2 * B * no * Mp * e)
         add(algo_b, "binning_T", B * ni * 4 + ni * cols * e)
         add(algo_b, "dw_reduce", 3 * no * ni * 4 + no * ni * 4)
+        add(algo_b, "adamw", 7 * no * ni * 4)              # read w, g, m, v; write w, m, v
         r_out, r_in = (no + 127) // 128 * 128, (ni + 127) // 128 * 128
         k_in, k_out = (ni + 63) // 64 * 64, (no + 63) // 64 * 64
         add(algo_f, "gemm_fwd_scan", 4 * B * ni * no)
@@ -312,7 +313,7 @@ def run_ours(args, rank, world, local):
     cfg = configs.config2()
     cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
     B = cfg["batch"]
-    n = net.DenseNet(cfg, args.math, device=dev)
+    n = net.DenseNet(cfg, args.math, device=dev, with_adamw=True)
     t0 = np.asarray(cfg["inputs"](seed=configs.SEED_INPUT + rank), np.float32)
     lab = cfg["labels"](seed=configs.SEED_LABELS + rank).astype(np.int32)
     n.set_inputs(t0, lab)

@@ -203,6 +203,25 @@ int dstd_sum_t_loss(const float *t, int64_t n, float *loss, float *g, dstd_strea
 int dstd_adamw(float *w, const float *g, float *m, float *v, int64_t n, float lr, float beta1,
                float beta2, float eps, float weight_decay, int step, dstd_stream_t stream);
 
+/* AdamW step (App. C.1) on up to 32 parameter tensors in one launch, with the
+ * update count kept in device memory, so that a CUDA graph that captures the
+ * call advances it on every replay.
+ *  w[i], g[i], m[i], v[i]: host arrays of count device pointers, tensor i
+ *      holding n[i] floats (w, m, v updated in place, g read);
+ *  step: device int32[2], caller-owned, 8-byte aligned; step[0] = updates done
+ *      so far (0 before the first), which the call uses plus one for the bias
+ *      corrections and then stores; step[1] is the kernel's scratch and must
+ *      be 0 before the first call (the call leaves it 0);
+ *  lr_dev: optional device float read at run time in place of lr (a warm-up
+ *      schedule under graph replay), or NULL.
+ * Calls that share one step buffer must not overlap on the GPU. Returns
+ * DSTD_E_INVALID for count outside [1, 32], a null pointer, n[i] < 1 or
+ * invalid hyperparameters; nothing is launched then. */
+int dstd_adamw_multi(int count, float *const *w, const float *const *g, float *const *m,
+                     float *const *v, const int64_t *n, float lr, float beta1, float beta2,
+                     float eps, float weight_decay, int32_t *step, const float *lr_dev,
+                     dstd_stream_t stream);
+
 /* Kernel timing (tracing). While enabled, the library brackets every kernel
  * it launches with a CUDA event pair on the launching stream and files the
  * pair under the kernel's kind (dstd_kernel_kind_name); launches made while

@@ -159,6 +159,62 @@ struct Timed {
     } while (0)
 
 // ---------------------------------------------------------------------------
+// Side streams. Launches of one call that do not depend on each other (in
+// the backward: dw^ beside the transposed binning and the weight transpose)
+// run on two library-owned streams: Fork makes both wait for
+// the work already enqueued on the caller's stream, and join() (or the
+// destructor) makes the caller's stream wait for both again. Under stream
+// capture this becomes a fork and a join in the graph. The side streams are
+// per device and shared; a Fork holds a lock from fork to join, so calls from
+// several host threads enqueue one after the other. If a stream or event
+// cannot be had, every launch stays on the caller's stream.
+// ---------------------------------------------------------------------------
+struct SideSet {
+    cudaStream_t s[2] = {nullptr, nullptr};
+    cudaEvent_t fork = nullptr, join[2] = {nullptr, nullptr};
+    int state = 0;  // 0 not made, 1 ready, -1 unavailable
+};
+constexpr int kMaxDevices = 64;
+SideSet g_side[kMaxDevices];
+std::mutex g_side_mu;
+
+struct Fork {
+    cudaStream_t main, side[2];
+    SideSet *ss = nullptr;
+    std::unique_lock<std::mutex> lk;
+    explicit Fork(cudaStream_t st) : main(st), side{st, st}, lk(g_side_mu) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return;
+        SideSet &q = g_side[dev];
+        if (q.state == 0) {
+            bool good = cudaEventCreateWithFlags(&q.fork, cudaEventDisableTiming) == cudaSuccess;
+            for (int i = 0; i < 2 && good; ++i)
+                good = cudaStreamCreateWithFlags(&q.s[i], cudaStreamNonBlocking) == cudaSuccess &&
+                       cudaEventCreateWithFlags(&q.join[i], cudaEventDisableTiming) == cudaSuccess;
+            q.state = good ? 1 : -1;
+        }
+        if (q.state != 1 || cudaEventRecord(q.fork, st) != cudaSuccess) return;
+        for (int i = 0; i < 2; ++i)
+            if (cudaStreamWaitEvent(q.s[i], q.fork, 0) == cudaSuccess) side[i] = q.s[i];
+        ss = &q;
+    }
+    int join() {
+        if (!ss) return DSTD_OK;
+        int r = DSTD_OK;
+        for (int i = 0; i < 2; ++i) {
+            if (side[i] == main) continue;
+            if (cudaEventRecord(ss->join[i], side[i]) != cudaSuccess ||
+                cudaStreamWaitEvent(main, ss->join[i], 0) != cudaSuccess)
+                r = DSTD_E_CUDA;
+            side[i] = main;
+        }
+        ss = nullptr;
+        return r;
+    }
+    ~Fork() { join(); }
+};
+
+// ---------------------------------------------------------------------------
 // Workspace layouts (one for the forward, one for the backward; both start at
 // the workspace base).
 // ---------------------------------------------------------------------------
@@ -195,8 +251,8 @@ FwdWs fwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
 }
 
 struct BwdWs {
-    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *dB_hi = nullptr,
-                  *dB_lo = nullptr, *sT_hi = nullptr, *sT_lo = nullptr;
+    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *sT_hi = nullptr,
+                  *sT_lo = nullptr;
     float *wt32 = nullptr, *dA32 = nullptr, *dB32 = nullptr, *sT32 = nullptr, *DS = nullptr, *part = nullptr,
           *count = nullptr;
     float4 *bw = nullptr;  // per-input bin index and kernel derivatives (input-time gradient)
@@ -251,10 +307,10 @@ BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
         }
     } else {
         const bool three = op == OpKind::BF16X3;
+        // dw^ once, [N_out, B*Mp]: the A operand of dW and, read transposed,
+        // the B operand of dS
         w.dA_hi = b.take<__nv_bfloat16>((size_t)N_out * w.ldbm);
         if (three) w.dA_lo = b.take<__nv_bfloat16>((size_t)N_out * w.ldbm);
-        w.dB_hi = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
-        if (three) w.dB_lo = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
         w.sT_hi = b.take<__nv_bfloat16>((size_t)N_in * w.ldbm);
         if (three) w.sT_lo = b.take<__nv_bfloat16>((size_t)N_in * w.ldbm);
         if (need_gt) {
@@ -314,6 +370,8 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
         }
         return DSTD_OK;
     }
+    // (the weight split and the binning are independent, but a fork/join
+    // around two kernels this short costs more than their overlap gains)
     {
         Timed tm(KK_PREP, st);
         if (op == OpKind::F16X3)
@@ -418,8 +476,8 @@ ConvFwdWs conv_fwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
 }
 
 struct ConvBwdWs {
-    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *dB_hi = nullptr,
-                  *dB_lo = nullptr, *sT_hi = nullptr, *sT_lo = nullptr;
+    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *sT_hi = nullptr,
+                  *sT_lo = nullptr;
     float *part = nullptr, *count = nullptr;
     int ldt = 0, ldn = 0, ldbm = 0, ldp = 0, splits = 1;
     size_t bytes = 0;
@@ -437,10 +495,10 @@ ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
     w.splits = dw_splits(pl.K, Cout, (int)cols, op);
     w.count = b.take<float>(Cout);
     // (dW adds into g_W atomically: no split-K partials)
+    // dw^ of a chunk once, [Cout, positions*Mp]: dW's A operand and, read
+    // transposed, the B operand of dS
     w.dA_hi = b.take<__nv_bfloat16>((size_t)Cout * w.ldbm);
     if (two) w.dA_lo = b.take<__nv_bfloat16>((size_t)Cout * w.ldbm);
-    w.dB_hi = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
-    if (two) w.dB_lo = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
     w.sT_hi = b.take<__nv_bfloat16>((size_t)pl.K * w.ldbm);
     if (two) w.sT_lo = b.take<__nv_bfloat16>((size_t)pl.K * w.ldbm);
     if (need_gt) {
@@ -608,26 +666,34 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
         Timed tm(KK_REDUCE, st);
         return cu(launch_dw_reduce(ws.part, ws.splits, zs, ws.ldp, N_out, N_in, ws.count, qcoef, g_W, st));
     }
+    const bool small_gt = need_gt && N_out <= kGradtSmallMaxOut;
     {
-        Timed tm(KK_DWHAT, st);
-        TRY(cu(launch_dwhat(t_out, sv.q, sv.s, sv.vdot, g_t_out, B, N_out, c, op, ws.dA_hi, ws.dA_lo, ws.ldbm,
-                            ws.dB_hi, ws.dB_lo, ws.ldn, ws.count, st)));
+        // three independent producers: dw^ (caller's stream), s^T with the
+        // per-input kernel derivatives (side 0), and W^T for dS plus the
+        // zeroing of dW (side 1)
+        Fork f(st);
+        {
+            Timed tm(KK_BIN_T, f.side[0]);
+            TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, f.side[0], ws.bw)));
+        }
+        if (need_gt && !small_gt) {
+            Timed tm(KK_PREP, f.side[1]);
+            TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, ws.wt_hi, ws.wt_lo, ws.ldt, nullptr,
+                                       0, nullptr, f.side[1])));
+        }
+        TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)N_out * N_in, f.side[1])));
+        {
+            Timed tm(KK_DWHAT, st);
+            TRY(cu(launch_dwhat(t_out, sv.q, sv.s, sv.vdot, g_t_out, B, N_out, c, op, ws.dA_hi, ws.dA_lo, ws.ldbm,
+                                nullptr, nullptr, 0, ws.count, st)));
+        }
+        TRY(f.join());
     }
-    {
-        // s^T for dW, and the per-input kernel derivatives the dS epilogue needs
-        Timed tm(KK_BIN_T, st);
-        TRY(cu(launch_binning(t_in, B, N_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st, ws.bw)));
-    }
-    if (need_gt && N_out <= kGradtSmallMaxOut) {
+    if (small_gt) {
         // few outputs: the input-time gradient by its definition, no contraction
         Timed tm(KK_GT, st);
         TRY(cu(launch_gradt_small(W, N_out, N_in, B, c, ws.bw, ws.dA_hi, ws.dA_lo, ws.ldbm, g_t_in, st)));
     } else if (need_gt) {
-        {
-            Timed tm(KK_PREP, st);
-            TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, ws.wt_hi, ws.wt_lo, ws.ldt, nullptr,
-                                       0, nullptr, st)));
-        }
         TcEpiArgs a{};
         a.c = c;
         a.B = B;
@@ -636,12 +702,12 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
         a.g_t_in = g_t_in;
         a.bw = ws.bw;
         Timed tm(KK_GEMM_DS, st);
-        TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dB_hi, ws.dB_lo, ws.ldn, N_in, (int)cols, N_out, 1, op,
-                              Epi::GradT, a, st)));
+        // dw^ read transposed from its dW layout [N_out, B*Mp]
+        TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dA_hi, ws.dA_lo, ws.ldbm, N_in, (int)cols, N_out, 1, op,
+                              Epi::GradT, a, st, true)));
     }
-    // dW = dw^T s: the split-K slices add into g_W (zeroed here); split 0
+    // dW = dw^T s: the split-K slices add into g_W (zeroed above); split 0
     // also adds the dead-neuron term qcoef * count_i
-    TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)N_out * N_in, st)));
     TcEpiArgs a{};
     a.D = g_W;
     a.ldd = N_in;
@@ -677,6 +743,31 @@ int dstd_adamw(float *w, const float *g, float *m, float *v, int64_t n, float lr
     TRY(device_ok());
     Timed tm(KK_ADAMW, (cudaStream_t)stream);
     return cu(launch_adamw(w, g, m, v, n, lr, beta1, beta2, eps, weight_decay, step, (cudaStream_t)stream));
+}
+
+int dstd_adamw_multi(int count, float *const *w, const float *const *g, float *const *m, float *const *v,
+                     const int64_t *n, float lr, float beta1, float beta2, float eps, float weight_decay,
+                     int32_t *step, const float *lr_dev, dstd_stream_t stream) {
+    if (count < 1 || count > kAdamMaxTensors || !w || !g || !m || !v || !n || !step) return DSTD_E_INVALID;
+    if ((reinterpret_cast<uintptr_t>(step) & 7) != 0) return DSTD_E_INVALID;
+    if (!(lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) || !(beta2 >= 0.0f && beta2 < 1.0f) || !(eps > 0.0f))
+        return DSTD_E_INVALID;
+    AdamMultiArgs a{};
+    for (int i = 0; i < count; ++i) {
+        if (!w[i] || !g[i] || !m[i] || !v[i] || n[i] < 1) return DSTD_E_INVALID;
+        a.seg[i] = AdamSeg{w[i], g[i], m[i], v[i], (long long)n[i], 0};
+    }
+    a.count = count;
+    a.lr = lr;
+    a.b1 = beta1;
+    a.b2 = beta2;
+    a.eps = eps;
+    a.wd = weight_decay;
+    a.step = step;
+    a.lr_dev = lr_dev;
+    TRY(device_ok());
+    Timed tm(KK_ADAMW, (cudaStream_t)stream);
+    return cu(launch_adamw_multi(a, (cudaStream_t)stream));
 }
 
 size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k, int stride, int pad,
@@ -783,8 +874,8 @@ int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const v
         {
             Timed tm(KK_DWHAT, st);
             TRY(cu(launch_dwhat(t_out + off, sv.q + off, sv.s + off, sv.vdot + off, g_t_out ? g_t_out + off : nullptr,
-                                npos, C_out, c, bop, ws.dA_hi, ws.dA_lo, ws.ldbm, ws.dB_hi, ws.dB_lo, ws.ldn,
-                                ws.count, st, ch > 0)));
+                                npos, C_out, c, bop, ws.dA_hi, ws.dA_lo, ws.ldbm, nullptr, nullptr, 0, ws.count, st,
+                                ch > 0)));
         }
         if (need_gt) {
             TcEpiArgs a{};
@@ -797,8 +888,8 @@ int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const v
             a.pos0 = pos0;
             a.g = pl.g;
             Timed tm(KK_GEMM_DS, st);
-            TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dB_hi, ws.dB_lo, ws.ldn, pl.K, (int)cols, C_out, 1,
-                                  bop, Epi::GradT, a, st)));
+            TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dA_hi, ws.dA_lo, ws.ldbm, pl.K, (int)cols, C_out, 1,
+                                  bop, Epi::GradT, a, st, true)));
         }
         {
             Timed tm(KK_BIN_T, st);

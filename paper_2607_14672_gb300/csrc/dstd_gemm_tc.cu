@@ -1,7 +1,10 @@
 // Tensor-core contraction of the DSTD layer on sm_103a (tcgen05 + TMA).
 //
-// D[r, c] = sum_k A[r, k] B[c, k] with A and B 16-bit, K-major, staged by TMA
-// (128-byte swizzle, no multicast) through a STAGES-deep mbarrier ring; one
+// D[r, c] = sum_k A[r, k] B[c, k] with A and B 16-bit, staged by TMA
+// (128-byte swizzle, no multicast) through a STAGES-deep mbarrier ring. A is
+// K-major; B is K-major ([C, K] rows) or, with BMN, MN-major ([K, C] rows:
+// the tensor core reads it transposed, so an operand written for one
+// contraction serves the transposed one without a second copy). One
 // thread issues tcgen05.mma (cta_group::1, M = 128, N = BN, K = 16 per
 // instruction) into fp32 accumulators in TMEM; eight warps read them back
 // with tcgen05.ld (lane = row) and run the epilogue:
@@ -213,11 +216,25 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
     return d;
 }
 
+// MN-major operand in 128-byte-swizzle layout: 64 consecutive MN elements
+// fill a 128-byte row, one row per k; 8 rows form a 1024-byte atom. SBO =
+// 1024 bytes between the 8-row groups along K, LBO = the distance between
+// the 64-wide atom columns along MN.
+__device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t saddr, uint32_t lbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address >> 4
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;  // LBO: next 64 MN elements
+    d |= (uint64_t)(1024u >> 4) << 32;          // SBO: next 8 k
+    d |= (uint64_t)1 << 46;                     // descriptor version
+    d |= (uint64_t)2 << 61;                     // 128-byte swizzle
+    return d;
+}
+
 // Instruction descriptor, kind::f16: D fp32, A and B both bf16 (format 1)
-// or both fp16 (format 0), both K-major.
-__host__ __device__ constexpr uint32_t idesc_16bit(int M, int N, bool f16) {
-    return (1u << 4) | ((f16 ? 0u : 1u) << 7) | ((f16 ? 0u : 1u) << 10) | ((uint32_t)(N >> 3) << 17) |
-           ((uint32_t)(M >> 4) << 24);
+// or both fp16 (format 0); A K-major, B K-major or (b_mn) MN-major.
+__host__ __device__ constexpr uint32_t idesc_16bit(int M, int N, bool f16, bool b_mn = false) {
+    return (1u << 4) | ((f16 ? 0u : 1u) << 7) | ((f16 ? 0u : 1u) << 10) | ((b_mn ? 1u : 0u) << 16) |
+           ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 template <int NPASS, int BN>
@@ -363,7 +380,7 @@ __device__ __forceinline__ TileInfo tile_info(int t, int n_row, int n_col, int k
     return ti;
 }
 
-template <int NPASS, int BN, int EPI, bool F16>
+template <int NPASS, int BN, int EPI, bool F16, bool BMN>
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA_hi, const __grid_constant__ CUtensorMap mA_lo,
               const __grid_constant__ CUtensorMap mB_hi, const __grid_constant__ CUtensorMap mB_lo, int R, int Cn,
@@ -416,8 +433,19 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                     const uint32_t st = smem_u32(smem + s * C::STAGE);
                     tma_load_2d(st, &mA_hi, &full[s], kx, ti.row0);
                     if (NPASS == 3) tma_load_2d(st + C::A_BYTES, &mA_lo, &full[s], kx, ti.row0);
-                    tma_load_2d(st + C::NOP * C::A_BYTES, &mB_hi, &full[s], kx, ti.col0);
-                    if (NPASS == 3) tma_load_2d(st + C::NOP * C::A_BYTES + C::B_BYTES, &mB_lo, &full[s], kx, ti.col0);
+                    const uint32_t sb = st + C::NOP * C::A_BYTES;
+                    if (!BMN) {
+                        tma_load_2d(sb, &mB_hi, &full[s], kx, ti.col0);
+                        if (NPASS == 3) tma_load_2d(sb + C::B_BYTES, &mB_lo, &full[s], kx, ti.col0);
+                    } else {
+                        // BK rows of k, each 64 columns wide per box
+#pragma unroll
+                        for (int h = 0; h < BN / 64; ++h) {
+                            tma_load_2d(sb + h * (BK * 128), &mB_hi, &full[s], ti.col0 + 64 * h, kx);
+                            if (NPASS == 3)
+                                tma_load_2d(sb + C::B_BYTES + h * (BK * 128), &mB_lo, &full[s], ti.col0 + 64 * h, kx);
+                        }
+                    }
                 }
             }
         }
@@ -425,7 +453,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // MMA issuer
-            constexpr uint32_t idesc = idesc_16bit(BM, BN, F16);
+            constexpr uint32_t idesc = idesc_16bit(BM, BN, F16, BMN);
             uint32_t it = 0, j = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
@@ -456,10 +484,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const uint64_t da = sdesc_sw128(a_hi + kk * 32);
-                        const uint64_t db = sdesc_sw128(b_hi + kk * 32);
+                        // K step of 16: 32 bytes along a K-major row, or 16
+                        // rows (two 1024-byte atoms) of an MN-major tile
+                        const uint64_t db = BMN ? sdesc_sw128_mn(b_hi + kk * 2048, BK * 128) : sdesc_sw128(b_hi + kk * 32);
                         mma_bf16(acc_main, da, db, idesc, (i >= C::P_MAIN || kk > 0) ? 1u : 0u);
                         if (NPASS == 3) {
-                            mma_bf16(acc_corr, da, sdesc_sw128(b_lo + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                            const uint64_t dbl =
+                                BMN ? sdesc_sw128_mn(b_lo + kk * 2048, BK * 128) : sdesc_sw128(b_lo + kk * 32);
+                            mma_bf16(acc_corr, da, dbl, idesc, (i > 0 || kk > 0) ? 1u : 0u);
                             mma_bf16(acc_corr, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
                         }
                     }
@@ -583,21 +615,21 @@ static int num_sms() {
     return n;
 }
 
-template <int NPASS, int BN, int EPI, bool F16>
+template <int NPASS, int BN, int EPI, bool F16, bool BMN>
 static cudaError_t launch_one(const CUtensorMap &a_hi, const CUtensorMap &a_lo, const CUtensorMap &b_hi,
                               const CUtensorMap &b_lo, int R, int Cn, int K, int splits, const TcEpiArgs &args,
                               cudaStream_t st) {
     using C = Cfg<NPASS, BN>;
-    cudaError_t e =
-        cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI, F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<NPASS, BN, EPI, F16, BMN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     const int ktiles = (K + BK - 1) / BK;
     const int per = (ktiles + splits - 1) / splits;
     const int n_row = (R + BM - 1) / BM, n_col = (Cn + BN - 1) / BN;
     const long long ntiles = (long long)n_row * n_col * splits;
     const int grid = (int)(ntiles < num_sms() ? ntiles : num_sms());
-    k_tc_gemm<NPASS, BN, EPI, F16><<<grid, NTHREADS, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per,
-                                                                       n_row, n_col, splits, args);
+    k_tc_gemm<NPASS, BN, EPI, F16, BMN><<<grid, NTHREADS, C::SMEM, st>>>(a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, per,
+                                                                            n_row, n_col, splits, args);
     return cudaGetLastError();
 }
 
@@ -616,26 +648,31 @@ int tc_gemm_splits_valid(int K, int splits) {
 
 cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo, int ldb,
                            int R, int Cn, int K, int splits, OpKind op, Epi epi, const TcEpiArgs &args,
-                           cudaStream_t st) {
+                           cudaStream_t st, bool b_mn) {
     constexpr int BN = 128;
     CUtensorMap a_hi, a_lo, b_hi, b_lo;
     const bool three = (op == OpKind::BF16X3 || op == OpKind::F16X3);
     const bool f16 = (op == OpKind::F16X3);
     if (op == OpKind::F32) return cudaErrorInvalidValue;
-    if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM, f16) || !tc::make_map(&b_hi, B_hi, Cn, K, ldb, BN, f16))
-        return cudaErrorInvalidValue;
+    // the Store epilogue runs with a K-major B, the GradT one with an MN-major B
+    if (b_mn != (epi == Epi::GradT)) return cudaErrorInvalidValue;
+    // K-major B: [Cn, K] rows, boxes of BN rows x 64 k; MN-major B: [K, Cn]
+    // rows, boxes of 64 k-rows x 64 columns
+    auto map_b = [&](CUtensorMap *m, const void *p) {
+        return b_mn ? tc::make_map(m, p, K, Cn, ldb, tc::BK, f16) : tc::make_map(m, p, Cn, K, ldb, BN, f16);
+    };
+    if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM, f16) || !map_b(&b_hi, B_hi)) return cudaErrorInvalidValue;
     if (three) {
-        if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM, f16) || !tc::make_map(&b_lo, B_lo, Cn, K, ldb, BN, f16))
-            return cudaErrorInvalidValue;
+        if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM, f16) || !map_b(&b_lo, B_lo)) return cudaErrorInvalidValue;
     } else {
         a_lo = a_hi;
         b_lo = b_hi;
     }
     if (splits < 1) splits = 1;
-#define DSTD_TC_LAUNCH(NP, F)                                                                              \
-    switch (epi) {                                                                                         \
-        case Epi::Store: return tc::launch_one<NP, BN, 0, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st); \
-        default: return tc::launch_one<NP, BN, 1, F>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);         \
+#define DSTD_TC_LAUNCH(NP, F)                                                                                      \
+    switch (epi) {                                                                                                 \
+        case Epi::Store: return tc::launch_one<NP, BN, 0, F, false>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st); \
+        default: return tc::launch_one<NP, BN, 1, F, true>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, splits, args, st);          \
     }
     if (f16) {
         DSTD_TC_LAUNCH(3, true)

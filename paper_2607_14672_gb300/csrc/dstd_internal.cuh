@@ -350,15 +350,36 @@ struct TcEpiArgs {
     const float4 *bw;  // dense GradT: per-input (k, ds/dt at T_k, at T_{k+1}) from the binning, or null
     int conv; int pos0; ConvGeom g;
 };
-// A, B: 16-bit operands (bf16 for BF16X3 / BF16, fp16 for F16X3)
+// A, B: 16-bit operands (bf16 for BF16X3 / BF16, fp16 for F16X3). A is
+// [R, K] rows (stride lda). B is [Cn, K] rows (stride ldb) for Epi::Store and
+// [K, Cn] rows (b_mn: read transposed by the tensor core) for Epi::GradT.
 cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo, int ldb,
                            int R, int Cn, int K, int splits, OpKind op, Epi epi, const TcEpiArgs &args,
-                           cudaStream_t st);
+                           cudaStream_t st, bool b_mn = false);
 
 cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
                            float *loss, float *g, cudaStream_t st);
 cudaError_t launch_sum_t(const float *t, long long n, float *loss, float *g, cudaStream_t st);
 cudaError_t launch_adamw(float *w, const float *g, float *m, float *v, long long n, float lr, float b1, float b2,
                          float eps, float wd, int step, cudaStream_t st);
+
+// one parameter tensor of a multi-tensor AdamW launch (off: set by the launcher)
+struct AdamSeg {
+    float *w;
+    const float *g;
+    float *m;
+    float *v;
+    long long n, off;
+};
+constexpr int kAdamMaxTensors = 32;
+struct AdamMultiArgs {
+    AdamSeg seg[kAdamMaxTensors];
+    int count;
+    long long total;
+    float lr, b1, b2, eps, wd;
+    int32_t *step;        // device: [0] updates done so far, [1] block ticket (0 between calls)
+    const float *lr_dev;  // device learning rate, or null for lr
+};
+cudaError_t launch_adamw_multi(const AdamMultiArgs &args, cudaStream_t st);
 
 }  // namespace dstd

@@ -688,9 +688,12 @@ cudaError_t launch_scan_solve(const float *what, long long sb, long long si, lon
 // ---------------------------------------------------------------------------
 // Backward, step 1: dC/dw^_im = -g_i K(t_i - T_m) / v^'(t_i) for m <= q_i
 // (implicit function theorem on v^(t_i) = v_th), g_i = upstream + dT/dt_i.
-// Writes it as the K-major operand of both backward contractions:
-//   A layout [N, lda]:    row i, columns (b, m)     (dW = dw^T . s)
-//   B layout [B*Mp, ldb]: row (b, m), column i      (dS = dw^ . W)
+// Writes it in the layout
+//   A [N, lda]: row i, columns (b, m)
+// which dW = dw^T . s reads as its K-major A operand and the tensor-core dS =
+// dw^ . W reads transposed (MN-major B). The fp32 mode's CUDA-core dS wants
+// the transposed copy too, when b is given:
+//   B [B*Mp, ldb]: row (b, m), column i
 // ---------------------------------------------------------------------------
 // Two adjacent lanes share one neuron (b, i): lane h = 0, 1 takes the
 // 16-byte chunks h, h+2, h+4, ... of its Mp bins, so that every 16-byte
@@ -741,19 +744,23 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
         }
         if (OP == 0) {
             *reinterpret_cast<float4 *>((float *)a_hi + abase + m0) = make_float4(v[0], v[1], v[2], v[3]);
+            if (b_hi) {
 #pragma unroll
-            for (int u = 0; u < BPC; ++u) ((float *)b_hi)[((long long)b * c.Mp + m0 + u) * ldb + i] = v[u];
+                for (int u = 0; u < BPC; ++u) ((float *)b_hi)[((long long)b * c.Mp + m0 + u) * ldb + i] = v[u];
+            }
         } else {
             __align__(16) __nv_bfloat16 hh[BPC], ll[BPC];
 #pragma unroll
             for (int u = 0; u < BPC; ++u) split_bf16(v[u], hh[u], ll[u]);
             *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + abase + m0) = *reinterpret_cast<uint4 *>(hh);
             if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + abase + m0) = *reinterpret_cast<uint4 *>(ll);
+            if (b_hi) {
 #pragma unroll
-            for (int u = 0; u < BPC; ++u) {
-                const long long o = ((long long)b * c.Mp + m0 + u) * ldb + i;
-                ((__nv_bfloat16 *)b_hi)[o] = hh[u];
-                if (OP == 1) ((__nv_bfloat16 *)b_lo)[o] = ll[u];
+                for (int u = 0; u < BPC; ++u) {
+                    const long long o = ((long long)b * c.Mp + m0 + u) * ldb + i;
+                    ((__nv_bfloat16 *)b_hi)[o] = hh[u];
+                    if (OP == 1) ((__nv_bfloat16 *)b_lo)[o] = ll[u];
+                }
             }
         }
     }
@@ -1014,6 +1021,94 @@ cudaError_t launch_adamw(float *w, const float *g, float *m, float *v, long long
     float bc1 = (float)(1.0 - pow((double)b1, step));
     float bc2 = (float)(1.0 - pow((double)b2, step));
     k_adamw<<<blocks_for(n, 256), 256, 0, st>>>(w, g, m, v, n, lr, b1, b2, eps, wd, bc1, bc2);
+    return cudaGetLastError();
+}
+
+// All parameter tensors of a network in one launch, with the update count in
+// device memory (so a captured CUDA graph advances it on every replay): each
+// block reads step[0], uses step[0] + 1 for the bias corrections, and the
+// last block to finish (ticket in step[1]) stores the new count and resets the
+// ticket. Element e of the concatenation belongs to the segment whose offset
+// range holds it; with VEC the offsets and sizes are in units of 4 floats.
+template <int VEC>
+__global__ void __launch_bounds__(256) k_adamw_multi(const AdamMultiArgs a) {
+    __shared__ float s_bc[2];
+    __shared__ float s_lr;
+    __shared__ int s_step;
+    if (threadIdx.x == 0) {
+        const int step = *reinterpret_cast<volatile int32_t *>(a.step) + 1;
+        s_step = step;
+        // fp32 (FP64 is slow on this part): 1 - beta^t to within a few ulp
+        s_bc[0] = 1.f - powf(a.b1, (float)step);
+        s_bc[1] = 1.f - powf(a.b2, (float)step);
+        s_lr = a.lr_dev ? *a.lr_dev : a.lr;
+    }
+    __syncthreads();
+    const float bc1 = s_bc[0], bc2 = s_bc[1], lr = s_lr;
+    const float decay = 1.f - lr * a.wd;
+    const long long units = a.total;
+    int k = 0;
+    for (long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x; u < units;
+         u += (long long)gridDim.x * blockDim.x) {
+        while (k + 1 < a.count && u >= a.seg[k + 1].off) ++k;  // u only grows
+        const AdamSeg &sg = a.seg[k];
+        const long long e = u - sg.off;
+        if (VEC) {
+            const float4 gi = reinterpret_cast<const float4 *>(sg.g)[e];
+            float4 wi = reinterpret_cast<float4 *>(sg.w)[e];
+            float4 mi = reinterpret_cast<float4 *>(sg.m)[e];
+            float4 vi = reinterpret_cast<float4 *>(sg.v)[e];
+            float *wp = &wi.x, *mp = &mi.x, *vp = &vi.x;
+            const float *gp = &gi.x;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                mp[j] = a.b1 * mp[j] + (1.f - a.b1) * gp[j];
+                vp[j] = a.b2 * vp[j] + (1.f - a.b2) * gp[j] * gp[j];
+                wp[j] = wp[j] * decay - lr * (mp[j] / bc1) / (sqrtf(vp[j] / bc2) + a.eps);
+            }
+            reinterpret_cast<float4 *>(sg.m)[e] = mi;
+            reinterpret_cast<float4 *>(sg.v)[e] = vi;
+            reinterpret_cast<float4 *>(sg.w)[e] = wi;
+        } else {
+            const float gi = sg.g[e];
+            const float mi = a.b1 * sg.m[e] + (1.f - a.b1) * gi;
+            const float vi = a.b2 * sg.v[e] + (1.f - a.b2) * gi * gi;
+            sg.m[e] = mi;
+            sg.v[e] = vi;
+            sg.w[e] = sg.w[e] * decay - lr * (mi / bc1) / (sqrtf(vi / bc2) + a.eps);
+        }
+    }
+    // every block has read step[0] before it takes a ticket
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const unsigned int ticket = atomicAdd(reinterpret_cast<unsigned int *>(a.step + 1), 1u);
+        if (ticket == gridDim.x - 1) {
+            a.step[0] = s_step;
+            a.step[1] = 0;
+            __threadfence();
+        }
+    }
+}
+
+cudaError_t launch_adamw_multi(const AdamMultiArgs &args, cudaStream_t st) {
+    AdamMultiArgs a = args;
+    bool vec = true;
+    for (int i = 0; i < a.count; ++i) {
+        const AdamSeg &sg = a.seg[i];
+        vec = vec && (sg.n % 4) == 0 && ((reinterpret_cast<uintptr_t>(sg.w) | reinterpret_cast<uintptr_t>(sg.g) |
+                                          reinterpret_cast<uintptr_t>(sg.m) | reinterpret_cast<uintptr_t>(sg.v)) &
+                                         15) == 0;
+    }
+    long long off = 0;
+    for (int i = 0; i < a.count; ++i) {
+        a.seg[i].off = off;
+        off += vec ? a.seg[i].n / 4 : a.seg[i].n;
+    }
+    a.total = off;
+    const unsigned g = grid_cap(off > 0 ? off : 1, 256);
+    if (vec) k_adamw_multi<1><<<g, 256, 0, st>>>(a);
+    else k_adamw_multi<0><<<g, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

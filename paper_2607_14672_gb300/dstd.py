@@ -20,7 +20,7 @@ ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "
 
 EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning", "dstd_dense_what",
            "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
-           "dstd_adamw", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
+           "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd")
 
@@ -78,6 +78,7 @@ def load(path=None):
         "dstd_ce_loss": (_I, [_P, _P, _I, _I, _F, _F, _P, _P, _P]),
         "dstd_sum_t_loss": (_I, [_P, _I64, _P, _P, _P]),
         "dstd_adamw": (_I, [_P, _P, _P, _P, _I64, _F, _F, _F, _F, _F, _I, _P]),
+        "dstd_adamw_multi": (_I, [_I, _P, _P, _P, _P, _P, _F, _F, _F, _F, _F, _P, _P, _P]),
         "dstd_device_status": (_I, [_I]),
         "dstd_error_string": (ctypes.c_char_p, [_I]),
         "dstd_version": (_I, []),
@@ -261,6 +262,24 @@ def adamw(w, g, m, v, lr, beta1, beta2, eps, weight_decay, step, stream=None):
     _f32(w, "w")
     _check(load().dstd_adamw(_ptr(w), _ptr(g), _ptr(m), _ptr(v), w.numel(), float(lr), float(beta1), float(beta2),
                              float(eps), float(weight_decay), int(step), _stream(stream)), "dstd_adamw")
+
+
+def adamw_multi(ws, gs, ms, vs, lr, beta1, beta2, eps, weight_decay, step, lr_dev=None, stream=None):
+    """One AdamW launch over the tensors ws (in place, with gs, ms, vs alike);
+    step is a device int32[2] tensor holding (updates done, 0)."""
+    k = len(ws)
+    if not (len(gs) == len(ms) == len(vs) == k):
+        raise ValueError("adamw_multi: tensor lists differ in length")
+    for w in ws:
+        _f32(w, "w")
+    import torch
+    if step.dtype != torch.int32 or step.numel() != 2 or not step.is_cuda:
+        raise ValueError("adamw_multi: step must be a device int32 tensor of 2 elements")
+    arr = lambda xs: (ctypes.c_void_p * k)(*[x.data_ptr() for x in xs])
+    n = (ctypes.c_int64 * k)(*[w.numel() for w in ws])
+    _check(load().dstd_adamw_multi(k, arr(ws), arr(gs), arr(ms), arr(vs), n, float(lr), float(beta1), float(beta2),
+                                   float(eps), float(weight_decay), _ptr(step), _ptr(lr_dev), _stream(stream)),
+           "dstd_adamw_multi")
 
 
 def device_status(clear=True):

@@ -45,7 +45,8 @@ class DenseNet:
         if with_adamw:
             self.m = [torch.zeros_like(w) for w in self.W]
             self.v = [torch.zeros_like(w) for w in self.W]
-            self.adam_step = 0
+            # (updates done, kernel scratch): advanced on the device by each AdamW launch
+            self.adam_state = torch.zeros(2, dtype=torch.int32, device=dev)
 
     # -- inputs -----------------------------------------------------------
     def set_offsets(self, offsets):
@@ -81,9 +82,8 @@ class DenseNet:
                            self.math, g_in, self.gW[l], self.workspace, stream)
 
     def optimizer(self, lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=1e-2, stream=None):
-        self.adam_step += 1
-        for w, g, m, v in zip(self.W, self.gW, self.m, self.v):
-            dstd.adamw(w, g, m, v, lr, betas[0], betas[1], eps, weight_decay, self.adam_step, stream)
+        dstd.adamw_multi(self.W, self.gW, self.m, self.v, lr, betas[0], betas[1], eps, weight_decay,
+                         self.adam_state, None, stream)
 
     def step(self, stream=None):
         """One training step: forward, loss, backward (and AdamW if enabled)."""
@@ -108,7 +108,7 @@ class DenseNet:
             small = tc and self.sizes[l + 1] <= 32  # or one direct kernel for a layer with few outputs
             n += 1 if small else (2 if tc else 3)
         if self.with_adamw:
-            n += L
+            n += 1                                # one AdamW launch for all layers
         return n
 
 
@@ -174,7 +174,8 @@ class ConvNet:
         if with_adamw:
             self.m = [torch.zeros_like(w) for w in self.W]
             self.v = [torch.zeros_like(w) for w in self.W]
-            self.adam_step = 0
+            # (updates done, kernel scratch): advanced on the device by each AdamW launch
+            self.adam_state = torch.zeros(2, dtype=torch.int32, device=dev)
 
     def set_offsets(self, offsets):
         for p, L, o in zip(self.p, self.layers, offsets):
@@ -220,9 +221,8 @@ class ConvNet:
                                self.workspace, stream)
 
     def optimizer(self, lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=1e-2, stream=None):
-        self.adam_step += 1
-        for w, g, m, v in zip(self.W, self.gW, self.m, self.v):
-            dstd.adamw(w, g, m, v, lr, betas[0], betas[1], eps, weight_decay, self.adam_step, stream)
+        dstd.adamw_multi(self.W, self.gW, self.m, self.v, lr, betas[0], betas[1], eps, weight_decay,
+                         self.adam_state, None, stream)
 
     def step(self, stream=None):
         """One training step: forward, loss, backward, AdamW."""

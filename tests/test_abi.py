@@ -104,3 +104,17 @@ def test_null_and_bad_arguments_rejected_on_host(lib):
                           ctypes.c_float(1e-8), ctypes.c_float(0.0), 1, None) == -1
     assert lib.dstd_adamw(one, one, one, one, 10, ctypes.c_float(1e-3), ctypes.c_float(0.9), ctypes.c_float(0.9),
                           ctypes.c_float(1e-8), ctypes.c_float(0.0), 0, None) == -1
+    # multi-tensor AdamW: tensor count, null step buffer, misaligned step buffer, empty tensor, bad beta
+    ptrs = (ctypes.c_void_p * 33)(*([256] * 33))
+    ns = (ctypes.c_int64 * 33)(*([10] * 33))
+    hyper = (ctypes.c_float(1e-3), ctypes.c_float(0.9), ctypes.c_float(0.999), ctypes.c_float(1e-8),
+             ctypes.c_float(0.0))
+    assert lib.dstd_adamw_multi(0, ptrs, ptrs, ptrs, ptrs, ns, *hyper, one, None, None) == -1
+    assert lib.dstd_adamw_multi(33, ptrs, ptrs, ptrs, ptrs, ns, *hyper, one, None, None) == -1
+    assert lib.dstd_adamw_multi(2, ptrs, ptrs, ptrs, ptrs, ns, *hyper, None, None, None) == -1
+    assert lib.dstd_adamw_multi(2, ptrs, ptrs, ptrs, ptrs, ns, *hyper, ctypes.c_void_p(260), None, None) == -1
+    n0 = (ctypes.c_int64 * 2)(10, 0)
+    assert lib.dstd_adamw_multi(2, ptrs, ptrs, ptrs, ptrs, n0, *hyper, one, None, None) == -1
+    assert lib.dstd_adamw_multi(2, ptrs, ptrs, ptrs, ptrs, ns, ctypes.c_float(1e-3), ctypes.c_float(1.0),
+                                ctypes.c_float(0.999), ctypes.c_float(1e-8), ctypes.c_float(0.0), one, None,
+                                None) == -1

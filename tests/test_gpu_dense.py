@@ -354,6 +354,48 @@ def test_adamw_matches_oracle():
     np.testing.assert_allclose(host(w), wr, rtol=1e-5, atol=1e-7)
 
 
+def test_adamw_multi_matches_oracle_under_graph_replay():
+    """Three tensors (one of them not a multiple of 4 floats, so the scalar
+    path runs) updated by one launch per step; the launch is captured once in
+    a CUDA graph and replayed, and the device step counter must advance the
+    bias corrections on every replay (App. C.1)."""
+    from paper_2607_14672_gb300 import dstd
+    g = np.random.default_rng(16)
+    for sizes in ((1000, 64, 4096), (1000, 63, 7)):
+        w0 = [f32(g.normal(size=n)) for n in sizes]
+        grads = [[f32(g.normal(size=n)) for n in sizes] for _ in range(4)]
+        ws = [dev(x) for x in w0]
+        ms = [torch.zeros(n, device="cuda") for n in sizes]
+        vs = [torch.zeros(n, device="cuda") for n in sizes]
+        gs = [torch.empty(n, device="cuda") for n in sizes]
+        step = torch.zeros(2, dtype=torch.int32, device="cuda")
+        lr = torch.full((1,), 2e-3, device="cuda")
+        ref = [(x.astype(np.float64), np.zeros(n), np.zeros(n)) for x, n in zip(w0, sizes)]
+        # first update eagerly, the next three by graph replay
+        for gd, x in zip(gs, grads[0]):
+            gd.copy_(dev(x))
+        dstd.adamw_multi(ws, gs, ms, vs, 1e-3, 0.9, 0.999, 1e-8, 1e-2, step, lr)
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=s):
+            dstd.adamw_multi(ws, gs, ms, vs, 1e-3, 0.9, 0.999, 1e-8, 1e-2, step, lr, stream=s)
+        torch.cuda.synchronize()
+        # capture launched nothing: still one update done
+        assert host(step).tolist() == [1, 0]
+        for k in range(1, 4):
+            for gd, x in zip(gs, grads[k]):
+                gd.copy_(dev(x))
+            graph.replay()
+        torch.cuda.synchronize()
+        assert host(step).tolist() == [4, 0]
+        for k in range(4):
+            ref = [olosses.adamw_step(wr, gr, mr, vr, k + 1, 2e-3, 0.9, 0.999, 1e-8, 1e-2)
+                   for (wr, mr, vr), gr in zip(ref, grads[k])]
+        for x, (wr, _, _) in zip(ws, ref):
+            np.testing.assert_allclose(host(x), wr, rtol=1e-5, atol=1e-7)
+
+
 # ---------------------------------------------------------------------------
 # host-side errors on a GPU box and the device status word
 # ---------------------------------------------------------------------------
