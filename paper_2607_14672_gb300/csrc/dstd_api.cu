@@ -278,12 +278,26 @@ int dw_splits(int N_in, int N_out, int K, OpKind op) {
     const long long tiles = (long long)((N_out + tm - 1) / tm) * ((N_in + tn - 1) / tn);
     const int kunit = op == OpKind::F32 ? 16 : 64;
     const int ktiles = (K + kunit - 1) / kunit;
-    long long want = (2 * 152 + tiles - 1) / tiles;
-    int s = (int)(want < 1 ? 1 : (want > ktiles ? ktiles : want));
-    if (s > 64) s = 64;
-    if (op != OpKind::F32)
-        while (s > 1 && !tc_gemm_splits_valid(K, s)) --s;
-    return s < 1 ? 1 : s;
+    if (op == OpKind::F32) {
+        long long want = (2 * 152 + tiles - 1) / tiles;
+        int s = (int)(want < 1 ? 1 : (want > ktiles ? ktiles : want));
+        return s < 1 ? 1 : (s > 64 ? 64 : s);
+    }
+    // persistent tensor-core contraction on 152 SMs: the busiest CTA runs
+    // ceil(items / 152) work items of ceil(ktiles / s) K slices each, plus
+    // about two slices of pipeline fill and epilogue per item
+    int best = 1;
+    long long best_cost = -1;
+    for (int s = 1; s <= 64 && s <= ktiles; ++s) {
+        if (!tc_gemm_splits_valid(K, s)) continue;
+        const long long rounds = (tiles * s + 151) / 152;
+        const long long cost = rounds * ((ktiles + s - 1) / s + 2);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = s;
+        }
+    }
+    return best;
 }
 
 BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool need_gt) {

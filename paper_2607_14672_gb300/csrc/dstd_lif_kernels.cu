@@ -60,9 +60,7 @@ static inline unsigned blocks_for(long long n, int threads) {
     return (unsigned)((n + threads - 1) / threads);
 }
 
-// blocks_for capped at 8 blocks per SM, for grid-stride kernels that end in
-// one atomic per block
-static unsigned grid_cap(long long n, int threads) {
+static int num_sms_cached() {
     static int sms = 0;
     if (sms == 0) {
         int dev = 0;
@@ -70,6 +68,13 @@ static unsigned grid_cap(long long n, int threads) {
             sms <= 0)
             sms = 148;
     }
+    return sms;
+}
+
+// blocks_for capped at 8 blocks per SM, for grid-stride kernels that end in
+// one atomic per block
+static unsigned grid_cap(long long n, int threads) {
+    const int sms = num_sms_cached();
     const unsigned b = blocks_for(n, threads), cap = 8u * (unsigned)sms;
     return b < 1 ? 1 : (b < cap ? b : cap);
 }
@@ -324,9 +329,125 @@ __global__ void k_binning_cols(const float *__restrict__ t, int B, int N, LifCon
     }
 }
 
+// 16-bit operands, written sparse: of the Mp bins of an input only two are
+// nonzero, so the operand is first zero-filled with 16-byte stores and the
+// two weights (hi and lo parts) are then stored element-wise by the same
+// thread (program order makes the later store win). OP 1: bf16 hi + lo,
+// 2: bf16, 3: fp16 hi + lo.
+template <int OP>
+__device__ __forceinline__ void split16(float x, uint16_t &h, uint16_t &l) {
+    if (OP == 3) {
+        __half hh, ll;
+        split_f16(x, hh, ll);
+        h = __half_as_ushort(hh);
+        l = __half_as_ushort(ll);
+    } else {
+        __nv_bfloat16 hh, ll;
+        split_bf16(x, hh, ll);
+        h = __bfloat16_as_ushort(hh);
+        l = __bfloat16_as_ushort(ll);
+    }
+}
+
+// rows (b, m), columns j: a block of ROWS8_THREADS takes one sample and as
+// many consecutive columns; it zero-fills that Mp x columns patch with
+// 16-byte stores, synchronises (which orders the block's global stores), and
+// then each thread stores the two weights of its own column (rows m >= M and
+// columns >= N stay zero).
+constexpr int ROWS8_THREADS = 128;
+template <int OP>
+__global__ void __launch_bounds__(ROWS8_THREADS) k_binning_rows8(const float *__restrict__ t, int B, int N,
+                                                                 LifConst c, uint16_t *hi, uint16_t *lo, int ld) {
+    const int b = blockIdx.y;
+    const int col0 = blockIdx.x * ROWS8_THREADS;
+    const int nch = ((ld - col0) < ROWS8_THREADS ? (ld - col0) : ROWS8_THREADS) / 8;  // 16-byte chunks per row
+    const long long base = (long long)b * c.Mp * ld + col0;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    for (int idx = threadIdx.x; idx < c.Mp * nch; idx += ROWS8_THREADS) {
+        const int m = idx / nch, cc = idx - m * nch;
+        const long long o = base + (long long)m * ld + 8 * cc;
+        *reinterpret_cast<uint4 *>(hi + o) = z;
+        if (OP != 2) *reinterpret_cast<uint4 *>(lo + o) = z;
+    }
+    __syncthreads();
+    const int j = col0 + threadIdx.x;
+    if (j >= N) return;
+    const float x = t[(long long)b * N + j];
+    if (!isfinite(x)) return;
+    const BinW w = bin_weights(c, x, false);
+    uint16_t h, l;
+    if (w.k >= 0 && w.k < c.M) {
+        split16<OP>(w.wR, h, l);
+        const long long o = base + (long long)w.k * ld + threadIdx.x;
+        hi[o] = h;
+        if (OP != 2) lo[o] = l;
+    }
+    if (w.k + 1 >= 0 && w.k + 1 < c.M) {
+        split16<OP>(w.wL, h, l);
+        const long long o = base + (long long)(w.k + 1) * ld + threadIdx.x;
+        hi[o] = h;
+        if (OP != 2) lo[o] = l;
+    }
+}
+
+// row j, columns (b, m): a warp takes 32 consecutive samples of one input j,
+// zero-fills their 32 x Mp bins (consecutive 16-byte chunks, one per lane per
+// round), then each lane stores the two weights of its own sample; with bw
+// != null it also writes (k, ds/dt at T_k, ds/dt at T_{k+1}) of its sample
+// to bw[b*N + j] (k = -100 for a silent input) for the input-time gradient.
+template <int OP>
+__global__ void k_binning_cols8(const float *__restrict__ t, int B, int N, LifConst c, uint16_t *hi, uint16_t *lo,
+                                int ld, float4 *bw) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int b0 = (blockIdx.x * (blockDim.x >> 5) + warp) * 32;
+    if (b0 >= B) return;
+    const int ns = (B - b0) < 32 ? (B - b0) : 32;
+    const int nch = ns * c.Mp / 8;  // 16-byte chunks of the warp's samples
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    const int b = b0 + lane;
+    for (int j = blockIdx.y; j < N; j += gridDim.y) {
+        const long long rowbase = (long long)j * ld + (long long)b0 * c.Mp;
+        for (int g = lane; g < nch; g += 32) {
+            *reinterpret_cast<uint4 *>(hi + rowbase + 8 * g) = z;
+            if (OP != 2) *reinterpret_cast<uint4 *>(lo + rowbase + 8 * g) = z;
+        }
+        // the zeros of a lane's sample were stored by other lanes: order them
+        // before its weights
+        __syncwarp();
+        if (b >= B) continue;
+        BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+        const float x = t[(long long)b * N + j];
+        if (isfinite(x)) w = bin_weights(c, x, bw != nullptr);
+        if (bw) bw[(long long)b * N + j] = make_float4(__int_as_float(w.k), w.dR, w.dL, 0.f);
+        const long long o = rowbase + (long long)lane * c.Mp;
+        uint16_t h, l;
+        if (w.k >= 0 && w.k < c.M) {
+            split16<OP>(w.wR, h, l);
+            hi[o + w.k] = h;
+            if (OP != 2) lo[o + w.k] = l;
+        }
+        if (w.k + 1 >= 0 && w.k + 1 < c.M) {
+            split16<OP>(w.wL, h, l);
+            hi[o + w.k + 1] = h;
+            if (OP != 2) lo[o + w.k + 1] = l;
+        }
+    }
+}
+
 cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKind op, bool transposed, void *hi,
                            void *lo, int ld, cudaStream_t st, float4 *bw) {
+    uint16_t *h16 = static_cast<uint16_t *>(hi), *l16 = static_cast<uint16_t *>(lo);
+    // the sparse writers need 16-byte aligned rows of 8-element multiples
+    const bool sparse = op != OpKind::F32 && (ld % 8) == 0 && ((reinterpret_cast<uintptr_t>(hi) |
+                                                                 reinterpret_cast<uintptr_t>(lo)) & 15) == 0;
     if (!transposed) {
+        if (sparse) {
+            dim3 grid(blocks_for(ld, ROWS8_THREADS), B);
+            if (op == OpKind::BF16X3) k_binning_rows8<1><<<grid, ROWS8_THREADS, 0, st>>>(t, B, N, c, h16, l16, ld);
+            else if (op == OpKind::F16X3) k_binning_rows8<3><<<grid, ROWS8_THREADS, 0, st>>>(t, B, N, c, h16, l16, ld);
+            else k_binning_rows8<2><<<grid, ROWS8_THREADS, 0, st>>>(t, B, N, c, h16, l16, ld);
+            return cudaGetLastError();
+        }
         int pairs = (ld + 1) / 2;
         dim3 grid(blocks_for(pairs, 128), B);
         if (op == OpKind::F32) k_binning_rows<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
@@ -335,6 +456,11 @@ cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKi
         else k_binning_rows<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
     } else {
         dim3 grid(blocks_for(B, 128), N < 65535 ? N : 65535);
+        if (sparse && op != OpKind::F16X3) {
+            if (op == OpKind::BF16X3) k_binning_cols8<1><<<grid, 128, 0, st>>>(t, B, N, c, h16, l16, ld, bw);
+            else k_binning_cols8<2><<<grid, 128, 0, st>>>(t, B, N, c, h16, l16, ld, bw);
+            return cudaGetLastError();
+        }
         if (op == OpKind::F32) k_binning_cols<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
         else if (op == OpKind::BF16X3) k_binning_cols<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
         else k_binning_cols<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
@@ -543,17 +669,21 @@ static __device__ __noinline__ float interior_test(float av, float aI, float lam
 // what[b*sb + i*si + m*sm], times scale[i] when given. SUB bins at a time
 // are loaded together (16-byte loads when sm = 1 and rows are 16-byte
 // aligned) into the thread's own row of shared memory (stride SUB + 4
-// floats: 16-byte accesses of 8 consecutive lanes hit distinct banks). The
-// scan walks the bins four at a time: one 16-byte read, the recurrence, and
-// a branch-free flag per bin for "v^ may reach v_th here" (end point at
-// v_th, or an interior maximum that the cheap bound does not exclude). Only
-// a group with a flag leaves the loop: the group is walked again bin by bin
-// with the exact tests (interior_test out of line), and the scan resumes
-// after the tested bin if it does not fire.
+// floats: 16-byte accesses of 8 consecutive lanes hit distinct banks).
+// Each block of SUB bins takes two passes:
+//   fast  all SUB bins, four per 16-byte read, branch-free: the recurrence,
+//         and bit u of a mask for "v^ may reach v_th in bin u" (end point at
+//         v_th, or an interior maximum that the cheap bound does not
+//         exclude); the state at every eighth bin is kept in registers;
+//   exact the flagged bins in order: from the nearest kept state, walk to
+//         the bin and test it exactly (interior_test out of line). The first
+//         bin that passes holds the spike.
+// A lane whose candidate fails goes straight to its next flagged bin, so no
+// lane walks a block twice.
 constexpr int SCAN_THREADS = 256;
 
-// One interval of the walk, with explicit fma so that the fast walk and the
-// exact re-walk round alike: the end state and the two flags.
+// One interval of the walk, with explicit fma so that the fast pass and the
+// exact pass round alike: the end state and the two flags.
 struct BinStep {
     float ve, In;
     bool endp, peak;
@@ -574,7 +704,9 @@ __global__ void __launch_bounds__(SCAN_THREADS, 4) k_scan_solve(const float *__r
                                                                 const float *__restrict__ scale,
                                                                 const float *__restrict__ rowsum, float *t_out,
                                                                 int *q, float *s, float *vdot, float *penalty) {
+    static_assert(SUB % 8 == 0 && SUB <= 32, "blocks of 8, 16 or 32 bins");
     constexpr int LD = SUB + 4;
+    constexpr int NCK = SUB / 8;  // kept states per block
     __shared__ __align__(16) float sw[SCAN_THREADS * LD];
     float *row = sw + threadIdx.x * LD;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -606,52 +738,54 @@ __global__ void __launch_bounds__(SCAN_THREADS, 4) k_scan_solve(const float *__r
 #pragma unroll
                 for (int j = 0; j < SUB; ++j) row[j] = (j < mend) ? __ldg(w + (m0 + j) * sm) * sc : 0.0f;
             }
-            int j = 0;
-            while (j < mend) {
-                // fast walk: groups of 4 bins, no branch inside a group
-                float vg = v, Ig = I;
-                int g = j & ~3;
-                bool flag = false;
-                for (; g < mend; g += 4) {
-                    const float4 x = *reinterpret_cast<const float4 *>(row + g);
-                    const float xs[4] = {x.x, x.y, x.z, x.w};
-                    vg = v;
-                    Ig = I;
+            // fast pass
+            float kv[NCK], kI[NCK];
+            uint32_t mask = 0u;
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const BinStep r = bin_step(c, v, I + xs[u]);
-                        flag |= (g + u >= j) & (g + u < mend) & (r.endp | r.peak);
-                        v = r.ve;
-                        I = r.In;
-                    }
-                    if (flag) break;
+            for (int g = 0; g < SUB; g += 4) {
+                if ((g & 7) == 0) {
+                    kv[g >> 3] = v;
+                    kI[g >> 3] = I;
                 }
-                if (!flag) break;
-                // exact walk of the flagged group from its first bin
-                v = vg;
-                I = Ig;
-                int k = g;
-                float hi = -1.0f, I0 = 0.f;
-                for (; k < g + 4 && k < mend; ++k) {
-                    I0 = I + row[k];
-                    const BinStep r = bin_step(c, v, I0);
-                    if (k >= j) {
-                        if (r.endp) hi = c.dt;
-                        else if (r.peak)
-                            hi = interior_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, v, I0, r.ve);
-                        if (hi >= 0.0f) break;
-                    }
+                const float4 x = *reinterpret_cast<const float4 *>(row + g);
+                const float xs[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const BinStep r = bin_step(c, v, I + xs[u]);
+                    if (r.endp | r.peak) mask |= 1u << (g + u);
                     v = r.ve;
                     I = r.In;
                 }
+            }
+            if (mend < 32) mask &= (1u << mend) - 1u;
+            // exact pass
+            while (mask) {
+                const int m = __ffs(mask) - 1;
+                mask &= mask - 1u;
+                const int gk = m >> 3;
+                float vw = kv[0], Iw = kI[0];
+#pragma unroll
+                for (int k = 1; k < NCK; ++k) {
+                    vw = (gk == k) ? kv[k] : vw;
+                    Iw = (gk == k) ? kI[k] : Iw;
+                }
+                for (int k = gk * 8; k < m; ++k) {
+                    const BinStep r = bin_step(c, vw, Iw + row[k]);
+                    vw = r.ve;
+                    Iw = r.In;
+                }
+                const float I0 = Iw + row[m];
+                const BinStep r = bin_step(c, vw, I0);
+                float hi = -1.0f;
+                if (r.endp) hi = c.dt;
+                else if (r.peak) hi = interior_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, vw, I0, r.ve);
                 if (hi >= 0.0f) {
-                    st.q = m0 + k;
-                    st.v0 = v;
+                    st.q = m0 + m;
+                    st.v0 = vw;
                     st.I0 = I0;
                     st.hi = hi;
                     break;
                 }
-                j = k;  // the flagged bins of the group did not fire; go on after them
             }
         }
         scan_finish(c, st);
@@ -724,23 +858,36 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
     }
     const long long abase = (long long)i * lda + (long long)b * c.Mp;
     // K(x) at x = s0 + (q - m) dt. Away from the spike K = (e^{-av x} -
-    // e^{-aI x}) / lam (x e^{-av x} when lam = 0) with fast exponentials; the
-    // spike's own bin and the one before it (x < 2 dt, where that difference
-    // cancels) take the expm1 form.
-    const float Kq = (q < c.M) ? kernel_K(c, s0) : 0.f;
-    const float Kq1 = (q < c.M) ? kernel_K(c, s0 + c.dt) : 0.f;
+    // e^{-aI x}) / lam (x e^{-av x} when lam = 0): both exponentials are taken
+    // at the first bin of a chunk and advance by the factors e^{av dt},
+    // e^{aI dt} per bin (x falls by dt); the spike's own bin and the one
+    // before it (x < 2 dt, where that difference cancels) take the expm1
+    // form. Chunks after the spike's bin, and every chunk of a silent
+    // neuron, are zero.
+    const bool fired = q < c.M;
+    const float Kq = fired ? kernel_K(c, s0) : 0.f;
+    const float Kq1 = fired ? kernel_K(c, s0 + c.dt) : 0.f;
+    const float fv = __expf(c.av * c.dt), fI = __expf(c.aI * c.dt);
     const int nch = c.Mp / BPC;
     for (int ch = h; ch < nch; ch += 2) {
         const int m0 = ch * BPC;
         float v[BPC];
+        if (!fired || m0 > q) {
 #pragma unroll
-        for (int u = 0; u < BPC; ++u) {
-            const int m = m0 + u;
-            const float x = s0 + (float)(q - m) * c.dt;
-            const float ev = __expf(-c.av * x);
-            const float Kf = c.lam_zero ? x * ev : (ev - __expf(-c.aI * x)) * c.inv_lam;
-            const float K = (m == q) ? Kq : ((m == q - 1) ? Kq1 : Kf);
-            v[u] = (q < c.M && m <= q) ? coef * K : 0.f;
+            for (int u = 0; u < BPC; ++u) v[u] = 0.f;
+        } else {
+            float x = s0 + (float)(q - m0) * c.dt;
+            float ev = __expf(-c.av * x), eI = __expf(-c.aI * x);
+#pragma unroll
+            for (int u = 0; u < BPC; ++u) {
+                const int m = m0 + u;
+                const float Kf = c.lam_zero ? x * ev : (ev - eI) * c.inv_lam;
+                const float K = (m == q) ? Kq : ((m == q - 1) ? Kq1 : Kf);
+                v[u] = (m <= q) ? coef * K : 0.f;
+                ev *= fv;
+                eI *= fI;
+                x -= c.dt;
+            }
         }
         if (OP == 0) {
             *reinterpret_cast<float4 *>((float *)a_hi + abase + m0) = make_float4(v[0], v[1], v[2], v[3]);
@@ -1025,69 +1172,66 @@ cudaError_t launch_adamw(float *w, const float *g, float *m, float *v, long long
 }
 
 // All parameter tensors of a network in one launch, with the update count in
-// device memory (so a captured CUDA graph advances it on every replay): each
-// block reads step[0], uses step[0] + 1 for the bias corrections, and the
-// last block to finish (ticket in step[1]) stores the new count and resets the
-// ticket. Element e of the concatenation belongs to the segment whose offset
-// range holds it; with VEC the offsets and sizes are in units of 4 floats.
+// device memory (so a captured CUDA graph advances it on every replay).
+// step[0] holds the count and step[1] a ticket; read together as one 64-bit
+// word, each block adds one to the ticket at its start and so learns the
+// count, and the block that draws the last ticket (every other block has then
+// drawn its own) stores count + 1 with the ticket reset. Element e of the
+// concatenation belongs to the segment whose offset range holds it; with VEC
+// the offsets and sizes are in units of 4 floats. One unit per thread: its
+// loads are issued before the count arrives.
 template <int VEC>
 __global__ void __launch_bounds__(256) k_adamw_multi(const AdamMultiArgs a) {
-    __shared__ float s_bc[2];
-    __shared__ float s_lr;
-    __shared__ int s_step;
-    if (threadIdx.x == 0) {
-        const int step = *reinterpret_cast<volatile int32_t *>(a.step) + 1;
-        s_step = step;
-        // fp32 (FP64 is slow on this part): 1 - beta^t to within a few ulp
-        s_bc[0] = 1.f - powf(a.b1, (float)step);
-        s_bc[1] = 1.f - powf(a.b2, (float)step);
-        s_lr = a.lr_dev ? *a.lr_dev : a.lr;
-    }
-    __syncthreads();
-    const float bc1 = s_bc[0], bc2 = s_bc[1], lr = s_lr;
-    const float decay = 1.f - lr * a.wd;
-    const long long units = a.total;
+    __shared__ unsigned long long s_old;
+    unsigned long long *word = reinterpret_cast<unsigned long long *>(a.step);
+    if (threadIdx.x == 0) s_old = atomicAdd(word, 1ull << 32);
+    const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const bool live = u < a.total;
     int k = 0;
-    for (long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x; u < units;
-         u += (long long)gridDim.x * blockDim.x) {
-        while (k + 1 < a.count && u >= a.seg[k + 1].off) ++k;  // u only grows
-        const AdamSeg &sg = a.seg[k];
-        const long long e = u - sg.off;
+    while (k + 1 < a.count && u >= a.seg[k + 1].off) ++k;
+    const AdamSeg &sg = a.seg[k];
+    const long long e = live ? u - sg.off : 0;
+    float4 gi = make_float4(0.f, 0.f, 0.f, 0.f), wi = gi, mi = gi, vi = gi;
+    if (live) {
         if (VEC) {
-            const float4 gi = reinterpret_cast<const float4 *>(sg.g)[e];
-            float4 wi = reinterpret_cast<float4 *>(sg.w)[e];
-            float4 mi = reinterpret_cast<float4 *>(sg.m)[e];
-            float4 vi = reinterpret_cast<float4 *>(sg.v)[e];
-            float *wp = &wi.x, *mp = &mi.x, *vp = &vi.x;
-            const float *gp = &gi.x;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                mp[j] = a.b1 * mp[j] + (1.f - a.b1) * gp[j];
-                vp[j] = a.b2 * vp[j] + (1.f - a.b2) * gp[j] * gp[j];
-                wp[j] = wp[j] * decay - lr * (mp[j] / bc1) / (sqrtf(vp[j] / bc2) + a.eps);
-            }
-            reinterpret_cast<float4 *>(sg.m)[e] = mi;
-            reinterpret_cast<float4 *>(sg.v)[e] = vi;
-            reinterpret_cast<float4 *>(sg.w)[e] = wi;
+            gi = reinterpret_cast<const float4 *>(sg.g)[e];
+            wi = reinterpret_cast<const float4 *>(sg.w)[e];
+            mi = reinterpret_cast<const float4 *>(sg.m)[e];
+            vi = reinterpret_cast<const float4 *>(sg.v)[e];
         } else {
-            const float gi = sg.g[e];
-            const float mi = a.b1 * sg.m[e] + (1.f - a.b1) * gi;
-            const float vi = a.b2 * sg.v[e] + (1.f - a.b2) * gi * gi;
-            sg.m[e] = mi;
-            sg.v[e] = vi;
-            sg.w[e] = sg.w[e] * decay - lr * (mi / bc1) / (sqrtf(vi / bc2) + a.eps);
+            gi.x = sg.g[e];
+            wi.x = sg.w[e];
+            mi.x = sg.m[e];
+            vi.x = sg.v[e];
         }
     }
-    // every block has read step[0] before it takes a ticket
     __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const unsigned int ticket = atomicAdd(reinterpret_cast<unsigned int *>(a.step + 1), 1u);
-        if (ticket == gridDim.x - 1) {
-            a.step[0] = s_step;
-            a.step[1] = 0;
-            __threadfence();
-        }
+    const unsigned long long old = s_old;
+    const int step = (int)(unsigned)(old & 0xffffffffull) + 1;
+    if (threadIdx.x == 0 && (old >> 32) == (unsigned long long)(gridDim.x - 1))
+        *word = (unsigned long long)(unsigned)step;  // count + 1, ticket 0
+    if (!live) return;
+    // fp32 (FP64 is slow on this part): 1 - beta^t to within a few ulp
+    const float bc1 = 1.f - powf(a.b1, (float)step);
+    const float bc2 = 1.f - powf(a.b2, (float)step);
+    const float lr = a.lr_dev ? *a.lr_dev : a.lr;
+    const float decay = 1.f - lr * a.wd;
+    float *wp = &wi.x, *mp = &mi.x, *vp = &vi.x;
+    const float *gp = &gi.x;
+#pragma unroll
+    for (int j = 0; j < (VEC ? 4 : 1); ++j) {
+        mp[j] = a.b1 * mp[j] + (1.f - a.b1) * gp[j];
+        vp[j] = a.b2 * vp[j] + (1.f - a.b2) * gp[j] * gp[j];
+        wp[j] = wp[j] * decay - lr * (mp[j] / bc1) / (sqrtf(vp[j] / bc2) + a.eps);
+    }
+    if (VEC) {
+        reinterpret_cast<float4 *>(sg.m)[e] = mi;
+        reinterpret_cast<float4 *>(sg.v)[e] = vi;
+        reinterpret_cast<float4 *>(sg.w)[e] = wi;
+    } else {
+        sg.m[e] = mi.x;
+        sg.v[e] = vi.x;
+        sg.w[e] = wi.x;
     }
 }
 
@@ -1106,7 +1250,7 @@ cudaError_t launch_adamw_multi(const AdamMultiArgs &args, cudaStream_t st) {
         off += vec ? a.seg[i].n / 4 : a.seg[i].n;
     }
     a.total = off;
-    const unsigned g = grid_cap(off > 0 ? off : 1, 256);
+    const unsigned g = blocks_for(off > 0 ? off : 1, 256);
     if (vec) k_adamw_multi<1><<<g, 256, 0, st>>>(a);
     else k_adamw_multi<0><<<g, 256, 0, st>>>(a);
     return cudaGetLastError();
