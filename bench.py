@@ -235,14 +235,15 @@ TRAFFIC_PER_LAUNCH = {
 }
 
 
-def kind_rooflines(per_kind, sizes, B, Mp, npass, math_mode, pk, pk_src):
+def kind_rooflines(per_kind, sizes, B, M, Mp, npass, math_mode, pk, pk_src):
     """Achieved vs peak for each kernel kind of the step.
 
     Contractions are tensor-bound: achieved = the method's flops (2 grid
     weights per input spike: 4 B N_in N_out per contraction) per launch /
     time; dense_* = the tensor-core flops the dense formulation issues (Mp/2
     times that, times npass for the three-product split). Binning, scan/solve,
-    dw^, the split-K reduction, weight prep and AdamW are HBM-bound: achieved = the
+    dw^, the split-K reduction, weight prep, AdamW and the few-output (narrow)
+    layer kernels are HBM-bound: achieved = the
     bytes the kernel must move (inputs read once, outputs written once) /
     time.
     """
@@ -259,6 +260,14 @@ def kind_rooflines(per_kind, sizes, B, Mp, npass, math_mode, pk, pk_src):
     for l in range(L):
         ni, no = sizes[l], sizes[l + 1]
         cols = B * Mp
+        from paper_2607_14672_gb300.net import narrow_layer
+        if narrow_layer(ni, no, M, math_mode):
+            # few outputs: one CUDA-core kernel each way; bytes = spike times and
+            # weights in, per-neuron state out (and the reverse for the backward)
+            add(algo_b, "narrow_fwd", B * ni * 4 + no * ni * 4 + 16 * B * no)
+            add(algo_b, "narrow_bwd", B * ni * 4 + no * ni * 4 + 20 * B * no + B * ni * 4 + no * ni * 4)
+            add(algo_b, "adamw", 7 * no * ni * 4)
+            continue
         add(algo_b, "prep_weights", no * ni * 4 + no * pad8(ni) * e)
         add(algo_b, "binning", B * ni * 4 + cols * pad8(ni) * e)
         add(algo_b, "scan_solve", B * no * Mp * 4 + B * no * 16)
@@ -414,7 +423,7 @@ def run_ours(args, rank, world, local):
     per_kind = {k: (v[0] / v[1], v[1] // n_kt) for k, v in kt.items() if v[1] > 0}
     dom = max(kt, key=lambda k: kt[k][0])
     sizes = n.sizes
-    rooflines = kind_rooflines(per_kind, sizes, B, Mp, npass, args.math, pk, pk_src)
+    rooflines = kind_rooflines(per_kind, sizes, B, cfg["layers"][0]["M"], Mp, npass, args.math, pk, pk_src)
     roof = dict(rooflines.get(dom, {"bound": None, "achieved": None, "peak": None, "unit": None, "frac": None}))
     roof["kernel"] = dom
     roof["traffic"] = TRAFFIC_PER_LAUNCH.get((dom, args.math))

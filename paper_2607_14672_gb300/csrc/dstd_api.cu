@@ -89,11 +89,12 @@ inline int cu(cudaError_t e) { return e == cudaSuccess ? DSTD_OK : DSTD_E_CUDA; 
 // ---------------------------------------------------------------------------
 enum Kind {
     KK_PREP = 0, KK_BIN, KK_BIN_T, KK_GEMM_FWD, KK_SCAN, KK_DWHAT, KK_GEMM_DS, KK_GT, KK_GEMM_DW, KK_REDUCE,
-    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_COUNT
+    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_NARROW_FWD, KK_NARROW_BWD, KK_COUNT
 };
 const char *const kKindNames[KK_COUNT] = {
     "prep_weights", "binning", "binning_T", "gemm_fwd_scan", "scan_solve", "dwhat", "gemm_dS_gradt",
-    "gradt_gather", "gemm_dW", "dw_reduce", "loss", "adamw", "binning_public", "what_public", "selftest"};
+    "gradt_gather", "gemm_dW", "dw_reduce", "loss", "adamw", "binning_public", "what_public", "selftest", "narrow_fwd",
+    "narrow_bwd"};
 
 struct Timing {
     std::mutex mu;
@@ -359,10 +360,22 @@ int check_sizes(int B, int N_in, int N_out) {
 
 // forward up to w^: binning + contraction; Scan epilogue fused (TC) unless
 // `store_D` (then the fp32 w^ lands in ws.D, layout [N_out, B*Mp]).
+// A layer with few outputs runs on CUDA cores in fp32 (fp32 and three-product
+// modes; the bf16 mode keeps its bf16 operands on the tensor cores).
+bool narrow_layer(int N_in, int N_out, int M, OpKind op) {
+    return N_out <= kNarrowMaxOut && N_in <= kNarrowMaxIn && M <= 94 &&
+           narrow_fwd_smem(N_in, N_out, M, padded_M(M)) <= kNarrowMaxSmem &&
+           (op == OpKind::F32 || op == OpKind::F16X3 || op == OpKind::BF16X3);
+}
+
 int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N_out, const LifConst &c, OpKind op,
                        const FwdWs &ws, bool store_D, const Saved *sv, float *t_out, float *penalty,
                        cudaStream_t st) {
     const long long cols = (long long)B * c.Mp;
+    if (!store_D && narrow_layer(N_in, N_out, c.M, op)) {
+        Timed tm(KK_NARROW_FWD, st);
+        return cu(launch_narrow_fwd(t_in, W, B, N_in, N_out, c, t_out, sv->q, sv->s, sv->vdot, penalty, st));
+    }
     if (op == OpKind::F32) {
         {
             Timed tm(KK_PREP, st);
@@ -645,6 +658,11 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
     Saved sv = saved_view(const_cast<void *>(saved), B, N_out);
     const long long cols = (long long)B * Mp;
     const float qcoef = -p->gamma_q * p->penalty_norm;
+    if (narrow_layer(N_in, N_out, c.M, op)) {
+        Timed tm(KK_NARROW_BWD, st);
+        return cu(launch_narrow_bwd(t_in, W, t_out, sv.q, sv.s, sv.vdot, g_t_out, B, N_in, N_out, c, qcoef, g_t_in,
+                                    g_W, st));
+    }
     if (op == OpKind::F32) {
         {
             Timed tm(KK_DWHAT, st);

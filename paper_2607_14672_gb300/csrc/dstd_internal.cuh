@@ -59,11 +59,15 @@ struct BinW {
     int k;
     float wR, wL, dR, dL;
 };
+// the grid step k of a finite spike t (clamped far outside the grid)
+__device__ __forceinline__ float bin_floor(const LifConst &c, float t) { return floorf((t - c.T0) * c.inv_dt); }
+__device__ __forceinline__ int bin_index(const LifConst &c, float t) {
+    return (int)fmaxf(fminf(bin_floor(c, t), 1e9f), -1e9f);
+}
 __device__ __forceinline__ BinW bin_weights(const LifConst &c, float t, bool deriv) {
     BinW b;
-    float u = (t - c.T0) * c.inv_dt;
-    float kf = floorf(u);
-    b.k = (int)fmaxf(fminf(kf, 1e9f), -1e9f);
+    const float kf = bin_floor(c, t);
+    b.k = bin_index(c, t);
     float r = t - (c.T0 + kf * c.dt);
     r = fminf(fmaxf(r, 0.0f), c.dt);
     float pR = phi_f(c, c.dt - r), pL = phi_f(c, r);
@@ -313,6 +317,18 @@ cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const
 // from W, dw^ (operand layout [N_out, ld] over (b, m), hi/lo or hi only) and
 // the per-input bin index / kernel derivatives bw.
 constexpr int kGradtSmallMaxOut = 32;
+// Layers with at most kNarrowMaxOut outputs run forward and backward on CUDA
+// cores in fp32 (sparse over the two grid points of each input spike).
+constexpr int kNarrowMaxOut = 32;
+constexpr int kNarrowMaxIn = 4096;       // the forward sorts a sample's inputs in shared memory
+constexpr size_t kNarrowMaxSmem = 200 * 1024;  // and holds W there: its shared memory, at most this
+size_t narrow_fwd_smem(int N_in, int N_out, int M, int Mp);
+cudaError_t launch_narrow_fwd(const float *t, const float *W, int B, int N_in, int N_out, const LifConst &c,
+                              float *t_out, int *q, float *s, float *vdot, float *penalty, cudaStream_t st);
+// zeroes g_W, then adds every block's share
+cudaError_t launch_narrow_bwd(const float *t_in, const float *W, const float *t_out, const int *q, const float *s,
+                              const float *vdot, const float *g_up, int B, int N_in, int N_out, const LifConst &c,
+                              float qcoef, float *g_t_in, float *g_W, cudaStream_t st);
 cudaError_t launch_gradt_small(const float *W, int N_out, int N_in, int B, const LifConst &c, const float4 *bw,
                                const __nv_bfloat16 *d_hi, const __nv_bfloat16 *d_lo, int ld, float *g_t_in,
                                cudaStream_t st);

@@ -698,15 +698,73 @@ __device__ __forceinline__ BinStep bin_step(const LifConst &c, float v, float I0
     return r;
 }
 
+// The two passes over SUB bins m0 .. m0+SUB-1 of one neuron, whose w^
+// values sit in row[0 .. SUB) (shared memory, 16-byte aligned, zero past
+// mend), starting from the state (v, I) at T_m0. On a spike, fills st (bin,
+// state at its start, bracket end) and returns true; otherwise leaves (v, I)
+// at the end of the block.
+template <int SUB>
+__device__ __forceinline__ bool scan_walk(const LifConst &c, const float *row, int m0, int mend, float &v, float &I,
+                                          ScanState &st) {
+    static_assert(SUB % 8 == 0 && SUB <= 32, "blocks of 8, 16 or 32 bins");
+    constexpr int NCK = SUB / 8;  // kept states per block
+    float kv[NCK], kI[NCK];
+    uint32_t mask = 0u;
+#pragma unroll
+    for (int g = 0; g < SUB; g += 4) {
+        if ((g & 7) == 0) {
+            kv[g >> 3] = v;
+            kI[g >> 3] = I;
+        }
+        const float4 x = *reinterpret_cast<const float4 *>(row + g);
+        const float xs[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const BinStep r = bin_step(c, v, I + xs[u]);
+            if (r.endp | r.peak) mask |= 1u << (g + u);
+            v = r.ve;
+            I = r.In;
+        }
+    }
+    if (mend < 32) mask &= (1u << mend) - 1u;
+    while (mask) {
+        const int m = __ffs(mask) - 1;
+        mask &= mask - 1u;
+        const int gk = m >> 3;
+        float vw = kv[0], Iw = kI[0];
+#pragma unroll
+        for (int k = 1; k < NCK; ++k) {
+            vw = (gk == k) ? kv[k] : vw;
+            Iw = (gk == k) ? kI[k] : Iw;
+        }
+        for (int k = gk * 8; k < m; ++k) {
+            const BinStep r = bin_step(c, vw, Iw + row[k]);
+            vw = r.ve;
+            Iw = r.In;
+        }
+        const float I0 = Iw + row[m];
+        const BinStep r = bin_step(c, vw, I0);
+        float hi = -1.0f;
+        if (r.endp) hi = c.dt;
+        else if (r.peak) hi = interior_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, vw, I0, r.ve);
+        if (hi >= 0.0f) {
+            st.q = m0 + m;
+            st.v0 = vw;
+            st.I0 = I0;
+            st.hi = hi;
+            return true;
+        }
+    }
+    return false;
+}
+
 template <int SUB, bool VEC, bool WIDE>
 __global__ void __launch_bounds__(SCAN_THREADS, 4) k_scan_solve(const float *__restrict__ what, long long sb,
                                                                 long long si, long long sm, int B, int N, LifConst c,
                                                                 const float *__restrict__ scale,
                                                                 const float *__restrict__ rowsum, float *t_out,
                                                                 int *q, float *s, float *vdot, float *penalty) {
-    static_assert(SUB % 8 == 0 && SUB <= 32, "blocks of 8, 16 or 32 bins");
     constexpr int LD = SUB + 4;
-    constexpr int NCK = SUB / 8;  // kept states per block
     __shared__ __align__(16) float sw[SCAN_THREADS * LD];
     float *row = sw + threadIdx.x * LD;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -738,55 +796,7 @@ __global__ void __launch_bounds__(SCAN_THREADS, 4) k_scan_solve(const float *__r
 #pragma unroll
                 for (int j = 0; j < SUB; ++j) row[j] = (j < mend) ? __ldg(w + (m0 + j) * sm) * sc : 0.0f;
             }
-            // fast pass
-            float kv[NCK], kI[NCK];
-            uint32_t mask = 0u;
-#pragma unroll
-            for (int g = 0; g < SUB; g += 4) {
-                if ((g & 7) == 0) {
-                    kv[g >> 3] = v;
-                    kI[g >> 3] = I;
-                }
-                const float4 x = *reinterpret_cast<const float4 *>(row + g);
-                const float xs[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const BinStep r = bin_step(c, v, I + xs[u]);
-                    if (r.endp | r.peak) mask |= 1u << (g + u);
-                    v = r.ve;
-                    I = r.In;
-                }
-            }
-            if (mend < 32) mask &= (1u << mend) - 1u;
-            // exact pass
-            while (mask) {
-                const int m = __ffs(mask) - 1;
-                mask &= mask - 1u;
-                const int gk = m >> 3;
-                float vw = kv[0], Iw = kI[0];
-#pragma unroll
-                for (int k = 1; k < NCK; ++k) {
-                    vw = (gk == k) ? kv[k] : vw;
-                    Iw = (gk == k) ? kI[k] : Iw;
-                }
-                for (int k = gk * 8; k < m; ++k) {
-                    const BinStep r = bin_step(c, vw, Iw + row[k]);
-                    vw = r.ve;
-                    Iw = r.In;
-                }
-                const float I0 = Iw + row[m];
-                const BinStep r = bin_step(c, vw, I0);
-                float hi = -1.0f;
-                if (r.endp) hi = c.dt;
-                else if (r.peak) hi = interior_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, vw, I0, r.ve);
-                if (hi >= 0.0f) {
-                    st.q = m0 + m;
-                    st.v0 = vw;
-                    st.I0 = I0;
-                    st.hi = hi;
-                    break;
-                }
-            }
+            if (scan_walk<SUB>(c, row, m0, mend, v, I, st)) break;
         }
         scan_finish(c, st);
         finish_neuron(c, st, b, i, N, rowsum, t_out, q, s, vdot, acc);
@@ -816,6 +826,338 @@ cudaError_t launch_scan_solve(const float *what, long long sb, long long si, lon
     }
 #undef DSTD_SCAN
 #undef DSTD_SCAN_L
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Layers with few outputs (N_out <= kNarrowMaxOut) on CUDA cores, in fp32.
+// A 128-row tensor-core tile would be mostly padding here, and each input
+// spike touches only two grid points, so the contraction is done sparse.
+// ---------------------------------------------------------------------------
+constexpr int NARROW_FWD_THREADS = 512, NARROW_BWD_THREADS = 1024;
+
+// Forward, one block per sample b: w^_im = sum_j W_ij s_jm (Eq. DSTD) from
+// the two grid weights of each input spike (wR at T_k, wL at T_{k+1}), then
+// the scan/solve/select of the sample's N_out neurons (one thread each) and
+// the penalty sums. The inputs are first put in a stable order by grid step
+// (a counting sort whose within-step order is the input order, so the sums
+// below have a fixed order and the forward is bitwise reproducible): warp w
+// ranks its own contiguous slice of inputs by key k + 1 in [0, M] (M + 1 = no
+// grid weight) with __match_any_sync, the per-warp counts give every (warp,
+// key) its offset, and a second pass places (j, wR, wL). Then one warp per
+// grid point m sums, for every output at once (registers), the inputs of
+// step m - 1 (their wL) and of step m (their wR): the lanes stride over
+// those inputs, reading W_.j as one row of the transposed copy of W in
+// shared memory, and a fixed butterfly of shuffles adds the lanes.
+template <int SUB, int NOUT>
+__global__ void __launch_bounds__(NARROW_FWD_THREADS) k_narrow_fwd(const float *__restrict__ t,
+                                                                 const float *__restrict__ W, int N_in, int N_out,
+                                                                 LifConst c, float *t_out, int *q, float *s,
+                                                                 float *vdot, float *penalty) {
+    constexpr int NW = NARROW_FWD_THREADS / 32;
+    extern __shared__ __align__(16) unsigned char nsm[];
+    const int NK = c.M + 2;  // keys 0 .. M, and M + 1 for "no weight"
+    // w^ first: its rows (Mp floats, Mp a power of two >= 8) stay 32-byte
+    // aligned for the scan's 16-byte reads, and so does W^T after it
+    float *acc = reinterpret_cast<float *>(nsm);        // [N_out][Mp]
+    float *ws = acc + N_out * c.Mp;                      // [N_out][N_in]: W
+    float *rsum = ws + (size_t)N_in * N_out;             // [N_out]
+    int *hist = reinterpret_cast<int *>(rsum + N_out);   // [NW][NK]: counts, then offsets
+    int *start = hist + NW * NK;                         // [NK + 1]
+    int *upos = start + NK + 1;                          // [N_in]: rank within (warp, key)
+    int *sj = upos + N_in;                               // [N_in]: inputs sorted by key
+    float2 *sw = reinterpret_cast<float2 *>((reinterpret_cast<uintptr_t>(sj + N_in) + 7) & ~uintptr_t(7));  // (wR, wL)
+    const int b = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float *tb = t + (long long)b * N_in;
+    auto key_of = [&](float x) {
+        if (!isfinite(x)) return c.M + 1;
+        const int k = bin_index(c, x);
+        return (k >= -1 && k < c.M) ? k + 1 : c.M + 1;
+    };
+    // warp w owns inputs [j_lo, j_hi), whole rounds of 32 (at most NR rounds);
+    // the spike times are loaded once, first, and kept for both passes
+    constexpr int NR = (kNarrowMaxIn + NW * 32 - 1) / (NW * 32);
+    const int C = (((N_in + NW - 1) / NW) + 31) & ~31;
+    const int j_lo = warp * C, j_hi = (j_lo + C) < N_in ? (j_lo + C) : N_in;
+    float xr[NR];
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+        const int j = j_lo + 32 * r + lane;
+        xr[r] = (32 * r < C && j < j_hi) ? tb[j] : INFINITY;
+    }
+    for (int e = threadIdx.x; e < N_out * c.Mp; e += NARROW_FWD_THREADS) acc[e] = 0.f;
+    for (int e = threadIdx.x; e < NW * NK; e += NARROW_FWD_THREADS) hist[e] = 0;
+    // W as it is: 16-byte copies when the sizes allow (consecutive threads,
+    // consecutive addresses: no bank conflicts)
+    if (((N_in * N_out) & 3) == 0 && (reinterpret_cast<uintptr_t>(W) & 15) == 0 &&
+        (reinterpret_cast<uintptr_t>(ws) & 15) == 0) {
+        const int nq = (N_in * N_out) >> 2;
+        for (int e0 = threadIdx.x; e0 < nq; e0 += 4 * NARROW_FWD_THREADS) {
+            float4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int e = e0 + u * NARROW_FWD_THREADS;
+                if (e < nq) v[u] = reinterpret_cast<const float4 *>(W)[e];
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int e = e0 + u * NARROW_FWD_THREADS;
+                if (e < nq) reinterpret_cast<float4 *>(ws)[e] = v[u];
+            }
+        }
+    } else {
+        for (int e = threadIdx.x; e < N_in * N_out; e += NARROW_FWD_THREADS) ws[e] = W[e];
+    }
+    __syncthreads();
+    // pass 1: ranks within (warp, key)
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+        if (32 * r >= C) break;
+        const int j = j_lo + 32 * r + lane;
+        const int key = (j < j_hi) ? key_of(xr[r]) : c.M + 1;
+        const unsigned match = __match_any_sync(0xffffffffu, key);
+        const unsigned lt = match & ((1u << lane) - 1u);
+        const int base = hist[warp * NK + key];
+        if (j < j_hi) upos[j] = base + __popc(lt);
+        __syncwarp();
+        if (lt == 0) hist[warp * NK + key] = base + __popc(match);
+        __syncwarp();
+    }
+    // row sums of W (dead-neuron term), warp w taking rows w, w + NW, ...
+    for (int i = warp; i < N_out; i += NW) {
+        float r = 0.f;
+        for (int j = lane; j < N_in; j += 32) r += ws[i * N_in + j];
+        r = warp_sum(r);
+        if (lane == 0) rsum[i] = r;
+    }
+    __syncthreads();
+    // offsets: the start of each key (an exclusive scan over keys by warp 0,
+    // up to 96 keys), then of each (warp, key) in warp order
+    if (warp == 0) {
+        int tot[3], run = 0;
+#pragma unroll
+        for (int r = 0; r < 3; ++r) {
+            const int k = lane * 3 + r;
+            int n = 0;
+            if (k < NK)
+                for (int w = 0; w < NW; ++w) n += hist[w * NK + k];
+            tot[r] = n;
+            run += n;
+        }
+        int incl = run;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        int ex = incl - run;
+#pragma unroll
+        for (int r = 0; r < 3; ++r) {
+            const int k = lane * 3 + r;
+            if (k < NK) start[k] = ex;
+            ex += tot[r];
+        }
+        if (lane == 31) start[NK] = incl;
+    }
+    __syncthreads();
+    if (threadIdx.x < NK) {
+        const int k = threadIdx.x;
+        int run = start[k];
+        for (int w = 0; w < NW; ++w) {
+            const int n = hist[w * NK + k];
+            hist[w * NK + k] = run;
+            run += n;
+        }
+    }
+    __syncthreads();
+    // pass 2: place (j, wR, wL) of every input with a weight
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+        if (32 * r >= C) break;
+        const int j = j_lo + 32 * r + lane;
+        if (j >= j_hi) continue;
+        const float x = xr[r];
+        const int key = key_of(x);
+        if (key > c.M) continue;
+        const BinW w = bin_weights(c, x, false);
+        const int pos = hist[warp * NK + key] + upos[j];
+        sj[pos] = j;
+        sw[pos] = make_float2(w.wR, w.wL);
+    }
+    __syncthreads();
+    // w^_.m: warp per grid point m; step m - 1 (key m) gives wL, step m
+    // (key m + 1) gives wR
+    for (int m = warp; m < c.M; m += NW) {
+        float a[NOUT];
+#pragma unroll
+        for (int i = 0; i < NOUT; ++i) a[i] = 0.f;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int p0 = start[m + h], p1 = start[m + h + 1];
+            for (int p = p0 + lane; p < p1; p += 32) {
+                const float2 ww = sw[p];
+                const float wv = h ? ww.x : ww.y;
+                const float *col = ws + sj[p];
+#pragma unroll
+                for (int i = 0; i < NOUT; ++i)
+                    if (i < N_out) a[i] = fmaf(col[i * N_in], wv, a[i]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < NOUT; ++i) {
+            if (i >= N_out) break;
+            const float r = warp_sum(a[i]);
+            if (lane == 0) acc[i * c.Mp + m] = r;
+        }
+    }
+    __syncthreads();
+    float pacc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (threadIdx.x < N_out) {
+        const int i = threadIdx.x;
+        ScanState st;
+        scan_reset(st, c.M);
+        float v = 0.f, I = 0.f;
+        for (int m0 = 0; m0 < c.M; m0 += SUB) {
+            const int mend = (c.M - m0) < SUB ? (c.M - m0) : SUB;
+            if (scan_walk<SUB>(c, acc + i * c.Mp + m0, m0, mend, v, I, st)) break;
+        }
+        scan_finish(c, st);
+        finish_neuron(c, st, b, i, N_out, rsum, t_out, q, s, vdot, pacc);
+    }
+    flush_penalty(pacc, penalty);
+}
+
+size_t narrow_fwd_smem(int N_in, int N_out, int M, int Mp) {
+    const int NW = NARROW_FWD_THREADS / 32, NK = M + 2;
+    return sizeof(float) * ((size_t)N_in * N_out + (size_t)N_out * Mp + N_out) +
+           sizeof(int) * ((size_t)NW * NK + NK + 1 + 2 * N_in + 1) + sizeof(float2) * (size_t)N_in + 16;
+}
+
+cudaError_t launch_narrow_fwd(const float *t, const float *W, int B, int N_in, int N_out, const LifConst &c,
+                              float *t_out, int *q, float *s, float *vdot, float *penalty, cudaStream_t st) {
+    if (N_out < 1 || N_out > kNarrowMaxOut || N_in > kNarrowMaxIn || c.M + 2 > 96) return cudaErrorInvalidValue;
+    const size_t smem = narrow_fwd_smem(N_in, N_out, c.M, c.Mp);
+    if (smem > kNarrowMaxSmem) return cudaErrorInvalidValue;
+    cudaError_t e = cudaSuccess;
+#define DSTD_NARROW_FWD(S, NO)                                                                                    \
+    e = cudaFuncSetAttribute(k_narrow_fwd<S, NO>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);        \
+    if (e != cudaSuccess) return e;                                                                                \
+    k_narrow_fwd<S, NO><<<B, NARROW_FWD_THREADS, smem, st>>>(t, W, N_in, N_out, c, t_out, q, s, vdot, penalty);
+#define DSTD_NARROW_FWD_NO(S) \
+    if (N_out <= 8) {         \
+        DSTD_NARROW_FWD(S, 8) \
+    } else if (N_out <= 16) { \
+        DSTD_NARROW_FWD(S, 16) \
+    } else {                  \
+        DSTD_NARROW_FWD(S, 32) \
+    }
+    if (c.Mp <= 8) {
+        DSTD_NARROW_FWD_NO(8)
+    } else if (c.Mp <= 16) {
+        DSTD_NARROW_FWD_NO(16)
+    } else {
+        DSTD_NARROW_FWD_NO(32)
+    }
+#undef DSTD_NARROW_FWD_NO
+#undef DSTD_NARROW_FWD
+    return cudaGetLastError();
+}
+
+// Backward, one block per NARROW_SAMPLES samples:
+//   dw^_im = -g_i K(t_i - T_m) / v^'(t_i) for m <= q_i (as k_dwhat, in fp32,
+//            in shared memory), and the count of silent neurons per output;
+//   per input j and sample: its grid point k and the weights and their
+//            t-derivatives (Tab. DSTD_kernels), the input-time gradient
+//            g_t_j = sum_i W_ij (dw^_ik ds_k/dt + dw^_i,k+1 ds_k+1/dt), and
+//            dW_ij += dw^_ik wR + dw^_i,k+1 wL;
+// the block adds its dW (and the dead-neuron term qcoef * silent count) into
+// g_W, which the caller zeroes.
+constexpr int NARROW_SAMPLES = 2;
+template <int NOUT>  // a bound on N_out: 8, 16 or 32
+__global__ void __launch_bounds__(NARROW_BWD_THREADS) k_narrow_bwd(const float *__restrict__ t_in,
+                                                             const float *__restrict__ W,
+                                                             const float *__restrict__ t_out,
+                                                             const int *__restrict__ qv, const float *__restrict__ sv,
+                                                             const float *__restrict__ vd,
+                                                             const float *__restrict__ g_up, int B, int N_in,
+                                                             int N_out, LifConst c, float qcoef, float *g_t_in,
+                                                             float *g_W) {
+    extern __shared__ __align__(16) float nsh[];
+    const int b0 = blockIdx.x * NARROW_SAMPLES;
+    const int nb = (B - b0) < NARROW_SAMPLES ? (B - b0) : NARROW_SAMPLES;
+    float *dw = nsh;                                     // [nb][N_out][Mp]
+    float *cnt = nsh + NARROW_SAMPLES * N_out * c.Mp;    // [N_out]
+    for (int e = threadIdx.x; e < N_out; e += NARROW_BWD_THREADS) cnt[e] = 0.f;
+    __syncthreads();
+    for (int e = threadIdx.x; e < nb * N_out * c.Mp; e += NARROW_BWD_THREADS) {
+        const int m = e % c.Mp, r = e / c.Mp;
+        const int i = r % N_out, sb = r / N_out;
+        const long long idx = (long long)(b0 + sb) * N_out + i;
+        const int q = qv[idx];
+        float val = 0.f;
+        if (q < c.M) {
+            if (m <= q) {
+                float pv, pg;
+                penalty_T(c, t_out[idx], pv, pg);
+                const float g = (g_up ? g_up[idx] : 0.f) + pg;
+                val = -g / vd[idx] * kernel_K(c, sv[idx] + (float)(q - m) * c.dt);
+            }
+        } else if (m == 0) {
+            atomicAdd(&cnt[i], 1.0f);
+        }
+        dw[e] = val;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < N_in; j += NARROW_BWD_THREADS) {
+        float wcol[NOUT], dacc[NOUT];
+#pragma unroll
+        for (int i = 0; i < NOUT; ++i) {
+            wcol[i] = (i < N_out) ? W[(long long)i * N_in + j] : 0.f;
+            dacc[i] = 0.f;
+        }
+        for (int sb = 0; sb < nb; ++sb) {
+            const float x = t_in[(long long)(b0 + sb) * N_in + j];
+            BinW w{-100, 0.f, 0.f, 0.f, 0.f};
+            if (isfinite(x)) w = bin_weights(c, x, g_t_in != nullptr);
+            const bool in0 = w.k >= 0 && w.k < c.M, in1 = w.k + 1 >= 0 && w.k + 1 < c.M;
+            const float *d = dw + sb * N_out * c.Mp;
+            float gt = 0.f;
+#pragma unroll
+            for (int i = 0; i < NOUT; ++i) {
+                if (i < N_out) {
+                    const float d0 = in0 ? d[i * c.Mp + w.k] : 0.f;
+                    const float d1 = in1 ? d[i * c.Mp + w.k + 1] : 0.f;
+                    gt = fmaf(wcol[i], fmaf(d0, w.dR, d1 * w.dL), gt);
+                    dacc[i] = fmaf(d0, w.wR, fmaf(d1, w.wL, dacc[i]));
+                }
+            }
+            if (g_t_in) g_t_in[(long long)(b0 + sb) * N_in + j] = gt;
+        }
+#pragma unroll
+        for (int i = 0; i < NOUT; ++i)
+            if (i < N_out) atomicAdd(&g_W[(long long)i * N_in + j], fmaf(qcoef, cnt[i], dacc[i]));
+    }
+}
+
+cudaError_t launch_narrow_bwd(const float *t_in, const float *W, const float *t_out, const int *q, const float *s,
+                              const float *vdot, const float *g_up, int B, int N_in, int N_out, const LifConst &c,
+                              float qcoef, float *g_t_in, float *g_W, cudaStream_t st) {
+    if (N_out < 1 || N_out > kNarrowMaxOut) return cudaErrorInvalidValue;
+    cudaError_t e = cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)N_out * N_in, st);
+    if (e != cudaSuccess) return e;
+    const size_t smem = sizeof(float) * ((size_t)NARROW_SAMPLES * N_out * c.Mp + N_out);
+    const unsigned g = (unsigned)((B + NARROW_SAMPLES - 1) / NARROW_SAMPLES);
+#define DSTD_NARROW_BWD(NO)                                                                                    \
+    k_narrow_bwd<NO><<<g, NARROW_BWD_THREADS, smem, st>>>(t_in, W, t_out, q, s, vdot, g_up, B, N_in, N_out, c, qcoef, \
+                                                     g_t_in, g_W);
+    if (N_out <= 8) {
+        DSTD_NARROW_BWD(8)
+    } else if (N_out <= 16) {
+        DSTD_NARROW_BWD(16)
+    } else {
+        DSTD_NARROW_BWD(32)
+    }
+#undef DSTD_NARROW_BWD
     return cudaGetLastError();
 }
 

@@ -12,6 +12,18 @@ import torch
 from . import dstd
 
 
+def narrow_layer(n_in, n_out, M, math_mode):
+    """True when the library runs this dense layer on its few-output CUDA-core
+    path (one kernel each way): the same test as the library's, including the
+    shared memory its forward needs (W transposed, the sorted inputs)."""
+    if n_out > 32 or n_in > 4096 or M > 94 or math_mode not in ("x3", "f32"):
+        return False
+    Mp = max(8, 1 << (M - 1).bit_length())
+    nk = M + 2
+    smem = 4 * (n_in * n_out + n_out * Mp + n_out) + 4 * (16 * nk + nk + 1 + 2 * n_in + 1) + 8 * n_in + 16
+    return smem <= 200 * 1024
+
+
 class DenseNet:
     """A stack of dense DSTD layers (configs.py layer dicts) on one GPU."""
 
@@ -101,12 +113,16 @@ class DenseNet:
         """Kernels the library launches per ``step`` (memsets not counted)."""
         tc = self.math != "f32"
         L = len(self.W)
-        n = L * 4                                 # fwd: prep + binning + gemm (+ fused scan) + root solve / scan
-        n += 1                                    # loss
-        n += L * (3 if tc else 4)                 # bwd: dw^ + binning^T + dW gemm [+ split-K reduce]
-        for l in range(1, L):                     # bwd input times: prep W^T + dS gemm [+ gather],
-            small = tc and self.sizes[l + 1] <= 32  # or one direct kernel for a layer with few outputs
-            n += 1 if small else (2 if tc else 3)
+        n = 1                                     # loss
+        for l in range(L):
+            n_in, n_out = self.sizes[l], self.sizes[l + 1]
+            if narrow_layer(n_in, n_out, self.layers[l]["M"], self.math):
+                n += 2                            # few outputs: one fused kernel each way (CUDA cores)
+                continue
+            n += 4                                # fwd: prep + binning + gemm + scan/solve
+            n += 3 if tc else 4                   # bwd: dw^ + binning^T + dW gemm [+ split-K reduce]
+            if l > 0:                             # bwd input times: prep W^T + dS gemm [+ gather]
+                n += 2 if tc else 3
         if self.with_adamw:
             n += 1                                # one AdamW launch for all layers
         return n
