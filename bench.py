@@ -222,16 +222,18 @@ class ClockSampler:
 # in profiles/launches_cfg2_step.md); to be set to None when the kernel
 # changes after that capture.
 TRAFFIC_PER_LAUNCH = {
-    ("gemm_dW", "x3"): 45.4e6,
-    ("gemm_fwd_scan", "x3"): 28.0e6,
+    ("gemm_dW", "x3"): 54.8e6,
+    ("gemm_fwd_scan", "x3"): 28.6e6,
     ("gemm_dS_gradt", "x3"): 32.2e6,
-    ("scan_solve", "x3"): 17.6e6,
-    ("dwhat", "x3"): 2.9e6,
-    ("binning", "x3"): 0.83e6,
-    ("binning_T", "x3"): 0.83e6,
-    ("gradt_gather", "x3"): 3.6e6,
-    ("prep_weights", "x3"): 1.9e6,
+    ("scan_solve", "x3"): 26.3e6,
+    ("dwhat", "x3"): 3.9e6,
+    ("binning", "x3"): 0.82e6,
+    ("binning_T", "x3"): 0.82e6,
+    ("prep_weights", "x3"): 2.55e6,
     ("loss", "x3"): 0.04e6,
+    ("adamw", "x3"): 20.4e6,
+    ("narrow_fwd", "x3"): 0.92e6,
+    ("narrow_bwd", "x3"): 0.97e6,
 }
 
 
