@@ -224,13 +224,19 @@ int dstd_adamw_multi(int count, float *const *w, const float *const *g, float *c
 
 /* Kernel timing (tracing). While enabled, the library brackets every kernel
  * it launches with a CUDA event pair on the launching stream and files the
- * pair under the kernel's kind (dstd_kernel_kind_name); launches made while
- * the stream is being captured into a CUDA graph are not timed.
+ * pair under the kernel's kind (dstd_kernel_kind_name).
  * dstd_timing_enable(on) turns timing on/off and clears the counters.
  * dstd_timing_read(kind, total_ms, launches) synchronises the device and
  * returns the accumulated device time and launch count of one kind. */
 int dstd_timing_enable(int on);
 int dstd_timing_read(int kind, float *total_ms, int64_t *launches);
+/* While timing is enabled, launches made on a stream that is being captured
+ * into a CUDA graph are bracketed by event-record nodes of the graph instead
+ * (the events stay with the graph: dstd_timing_enable drops them from the
+ * library's lists without reusing them). After each replay of such a graph,
+ * dstd_timing_collect() synchronises the device and adds that replay's
+ * device time between every pair to its kind's totals. */
+int dstd_timing_collect(void);
 int dstd_kernel_kind_count(void);
 const char *dstd_kernel_kind_name(int kind);
 

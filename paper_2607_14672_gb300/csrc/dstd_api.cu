@@ -101,6 +101,9 @@ struct Timing {
     bool on = false;
     std::vector<cudaEvent_t> pool;
     std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending[KK_COUNT];
+    // pairs captured into a CUDA graph as event-record nodes: every replay
+    // records them again; dstd_timing_collect adds one replay's worth
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> graph[KK_COUNT];
     double ms[KK_COUNT] = {};
     long long n[KK_COUNT] = {};
 };
@@ -133,24 +136,39 @@ void drain_pending() {
     }
 }
 
+// Brackets the launches of one scope with an event pair: recorded directly
+// in eager mode, or, on a stream being captured, as external event-record
+// nodes of the graph (read back per replay by dstd_timing_collect).
 struct Timed {
     int kind;
     cudaStream_t st;
     cudaEvent_t a = nullptr;
+    bool captured = false;
     Timed(int k, cudaStream_t s) : kind(k), st(s) {
         if (!g_timing.on) return;
         cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-        if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return;
+        if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) return;
+        captured = cs == cudaStreamCaptureStatusActive;
+        if (cs != cudaStreamCaptureStatusNone && !captured) return;
         std::lock_guard<std::mutex> lk(g_timing.mu);
         a = take_event();
-        if (a && cudaEventRecord(a, s) != cudaSuccess) a = nullptr;
+        const cudaError_t e = captured ? cudaEventRecordWithFlags(a, s, cudaEventRecordExternal) : cudaEventRecord(a, s);
+        if (a && e != cudaSuccess) {
+            g_timing.pool.push_back(a);
+            a = nullptr;
+        }
     }
     ~Timed() {
         if (!a) return;
         std::lock_guard<std::mutex> lk(g_timing.mu);
         cudaEvent_t b = take_event();
-        if (b && cudaEventRecord(b, st) == cudaSuccess) g_timing.pending[kind].push_back({a, b});
-        else g_timing.pool.push_back(a);
+        const cudaError_t e =
+            !b ? cudaErrorUnknown : (captured ? cudaEventRecordWithFlags(b, st, cudaEventRecordExternal) : cudaEventRecord(b, st));
+        if (e == cudaSuccess) (captured ? g_timing.graph : g_timing.pending)[kind].push_back({a, b});
+        else {
+            g_timing.pool.push_back(a);
+            if (b) g_timing.pool.push_back(b);
+        }
     }
 };
 #define TRY(x)                       \
@@ -397,20 +415,27 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
         }
         return DSTD_OK;
     }
-    // (the weight split and the binning are independent, but a fork/join
-    // around two kernels this short costs more than their overlap gains)
-    {
-        Timed tm(KK_PREP, st);
-        if (op == OpKind::F16X3)
-            TRY(cu(launch_prep_weights_f16(W, N_out, N_in, (__half *)ws.w_hi, (__half *)ws.w_lo, ws.kpad,
-                                           ws.row_scale, ws.rowsum, st)));
-        else
-            TRY(cu(launch_prep_weights(W, N_out, N_in, op, (__nv_bfloat16 *)ws.w_hi, (__nv_bfloat16 *)ws.w_lo,
-                                       ws.kpad, nullptr, nullptr, 0, nullptr, 0, ws.rowsum, st)));
-    }
-    {
+    // the weight split and the binning are independent: one launch does both
+    // for the x3 forward (a fork/join around two kernels this short costs
+    // more than their overlap gains)
+    if (op == OpKind::F16X3 && (ws.kpad % 8) == 0) {
         Timed tm(KK_BIN, st);
-        TRY(cu(launch_binning(t_in, B, N_in, c, op, false, ws.s_hi, ws.s_lo, ws.kpad, st)));
+        TRY(cu(launch_fwd_operands_f16(t_in, B, N_in, c, ws.s_hi, ws.s_lo, ws.kpad, W, N_out, (__half *)ws.w_hi,
+                                       (__half *)ws.w_lo, ws.row_scale, ws.rowsum, st)));
+    } else {
+        {
+            Timed tm(KK_PREP, st);
+            if (op == OpKind::F16X3)
+                TRY(cu(launch_prep_weights_f16(W, N_out, N_in, (__half *)ws.w_hi, (__half *)ws.w_lo, ws.kpad,
+                                               ws.row_scale, ws.rowsum, st)));
+            else
+                TRY(cu(launch_prep_weights(W, N_out, N_in, op, (__nv_bfloat16 *)ws.w_hi, (__nv_bfloat16 *)ws.w_lo,
+                                           ws.kpad, nullptr, nullptr, 0, nullptr, 0, ws.rowsum, st)));
+        }
+        {
+            Timed tm(KK_BIN, st);
+            TRY(cu(launch_binning(t_in, B, N_in, c, op, false, ws.s_hi, ws.s_lo, ws.kpad, st)));
+        }
     }
     TcEpiArgs a{};
     a.c = c;
@@ -950,8 +975,25 @@ int dstd_timing_enable(int on) {
     for (int k = 0; k < KK_COUNT; ++k) {
         g_timing.ms[k] = 0.0;
         g_timing.n[k] = 0;
+        // a graph may still record these: they are dropped from the list, not reused
+        g_timing.graph[k].clear();
     }
     g_timing.on = on != 0;
+    return DSTD_OK;
+}
+
+int dstd_timing_collect(void) {
+    if (cudaDeviceSynchronize() != cudaSuccess) return DSTD_E_CUDA;
+    std::lock_guard<std::mutex> lk(g_timing.mu);
+    for (int k = 0; k < KK_COUNT; ++k) {
+        for (auto &pr : g_timing.graph[k]) {
+            float ms = 0.f;
+            if (cudaEventElapsedTime(&ms, pr.first, pr.second) == cudaSuccess) {
+                g_timing.ms[k] += ms;
+                g_timing.n[k] += 1;
+            }
+        }
+    }
     return DSTD_OK;
 }
 

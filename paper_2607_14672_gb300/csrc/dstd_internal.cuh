@@ -273,6 +273,12 @@ inline int pad8(int x) { return (x + 7) & ~7; }
 // row sums [R]. One warp per row.
 cudaError_t launch_prep_weights_f16(const float *W, int R, int C, __half *hi, __half *lo, int ldo, float *inv_scale,
                                     float *rowsum, cudaStream_t st);
+// the x3 forward's two operands (binned spike times, fp16 weight split) in
+// one launch: same results as launch_binning (F16X3) and launch_prep_weights_f16
+// with ldo = ld
+cudaError_t launch_fwd_operands_f16(const float *t, int B, int N, const LifConst &c, void *s_hi, void *s_lo, int ld,
+                                    const float *W, int R, __half *w_hi, __half *w_lo, float *inv_scale,
+                                    float *rowsum, cudaStream_t st);
 // W fp32 [R, C] -> hi/lo bf16 [R, ldo] (and optional transpose [C, ldt]),
 // fp32 copy (F32 path), row sums [R].
 cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bfloat16 *hi, __nv_bfloat16 *lo,

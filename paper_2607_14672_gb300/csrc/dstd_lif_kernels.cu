@@ -140,12 +140,11 @@ __device__ __forceinline__ void split_f16(float x, __half &hi, __half &lo) {
 // re-read from memory only for longer rows).
 constexpr int PREP_THREADS = 256, PREP_PER_THREAD = 8;
 
-__global__ void __launch_bounds__(PREP_THREADS) k_prep_weights_f16(const float *__restrict__ W, int R, int C,
-                                                                 __half *hi, __half *lo, int ldo, float *inv_scale,
-                                                                 float *rowsum) {
+// Row r of the forward weight operand (one block of PREP_THREADS threads).
+__device__ __forceinline__ void prep_row_f16(const float *__restrict__ W, int R, int C, __half *hi, __half *lo, int ldo,
+                                             float *inv_scale, float *rowsum, int r) {
     __shared__ float red_max[PREP_THREADS / 32], red_sum[PREP_THREADS / 32];
     __shared__ float sc_sh;
-    const int r = blockIdx.x;
     if (r >= R) return;
     const float *w = W + (long long)r * C;
     float x[PREP_PER_THREAD];
@@ -209,6 +208,12 @@ __global__ void __launch_bounds__(PREP_THREADS) k_prep_weights_f16(const float *
         hi[(long long)r * ldo + j] = h;
         lo[(long long)r * ldo + j] = l;
     }
+}
+
+__global__ void __launch_bounds__(PREP_THREADS) k_prep_weights_f16(const float *__restrict__ W, int R, int C,
+                                                                 __half *hi, __half *lo, int ldo, float *inv_scale,
+                                                                 float *rowsum) {
+    prep_row_f16(W, R, C, hi, lo, ldo, inv_scale, rowsum, blockIdx.x);
 }
 
 cudaError_t launch_prep_weights_f16(const float *W, int R, int C, __half *hi, __half *lo, int ldo, float *inv_scale,
@@ -355,15 +360,13 @@ __device__ __forceinline__ void split16(float x, uint16_t &h, uint16_t &l) {
 // then each thread stores the two weights of its own column (rows m >= M and
 // columns >= N stay zero).
 constexpr int ROWS8_THREADS = 128;
-template <int OP>
-__global__ void __launch_bounds__(ROWS8_THREADS) k_binning_rows8(const float *__restrict__ t, int B, int N,
-                                                                 LifConst c, uint16_t *hi, uint16_t *lo, int ld) {
-    const int b = blockIdx.y;
-    const int col0 = blockIdx.x * ROWS8_THREADS;
-    const int nch = ((ld - col0) < ROWS8_THREADS ? (ld - col0) : ROWS8_THREADS) / 8;  // 16-byte chunks per row
+template <int OP, int NT>
+__device__ __forceinline__ void binning_rows8_block(const float *__restrict__ t, int N, const LifConst &c, uint16_t *hi,
+                                                    uint16_t *lo, int ld, int b, int col0) {
+    const int nch = ((ld - col0) < NT ? (ld - col0) : NT) / 8;  // 16-byte chunks per row
     const long long base = (long long)b * c.Mp * ld + col0;
     const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-    for (int idx = threadIdx.x; idx < c.Mp * nch; idx += ROWS8_THREADS) {
+    for (int idx = threadIdx.x; idx < c.Mp * nch; idx += NT) {
         const int m = idx / nch, cc = idx - m * nch;
         const long long o = base + (long long)m * ld + 8 * cc;
         *reinterpret_cast<uint4 *>(hi + o) = z;
@@ -388,6 +391,43 @@ __global__ void __launch_bounds__(ROWS8_THREADS) k_binning_rows8(const float *__
         hi[o] = h;
         if (OP != 2) lo[o] = l;
     }
+}
+
+template <int OP>
+__global__ void __launch_bounds__(ROWS8_THREADS) k_binning_rows8(const float *__restrict__ t, int B, int N,
+                                                                 LifConst c, uint16_t *hi, uint16_t *lo, int ld) {
+    binning_rows8_block<OP, ROWS8_THREADS>(t, N, c, hi, lo, ld, blockIdx.y, blockIdx.x * ROWS8_THREADS);
+}
+
+// The two operands of the x3 forward contraction in one launch (they do not
+// depend on each other): blocks [0, nbin) bin the spike times (sample
+// blockIdx / nbx, columns of chunk blockIdx % nbx), the rest split weight
+// rows into fp16 hi + lo.
+__global__ void __launch_bounds__(PREP_THREADS) k_fwd_operands_f16(const float *__restrict__ t, int N, LifConst c,
+                                                                 uint16_t *s_hi, uint16_t *s_lo, int ld, int nbx,
+                                                                 int nbin, const float *__restrict__ W, int R,
+                                                                 __half *w_hi, __half *w_lo, float *inv_scale,
+                                                                 float *rowsum) {
+    if ((int)blockIdx.x < nbin) {
+        const int b = blockIdx.x / nbx, cb = blockIdx.x - b * nbx;
+        binning_rows8_block<3, PREP_THREADS>(t, N, c, s_hi, s_lo, ld, b, cb * PREP_THREADS);
+    } else {
+        prep_row_f16(W, R, N, w_hi, w_lo, ld, inv_scale, rowsum, blockIdx.x - nbin);
+    }
+}
+
+cudaError_t launch_fwd_operands_f16(const float *t, int B, int N, const LifConst &c, void *s_hi, void *s_lo, int ld,
+                                    const float *W, int R, __half *w_hi, __half *w_lo, float *inv_scale,
+                                    float *rowsum, cudaStream_t st) {
+    if ((ld % 8) != 0 || ((reinterpret_cast<uintptr_t>(s_hi) | reinterpret_cast<uintptr_t>(s_lo)) & 15) != 0)
+        return cudaErrorInvalidValue;
+    const int nbx = (ld + PREP_THREADS - 1) / PREP_THREADS;
+    const long long nbin = (long long)nbx * B;
+    if (nbin + R > 0x7fffffffLL) return cudaErrorInvalidValue;
+    k_fwd_operands_f16<<<(unsigned)(nbin + R), PREP_THREADS, 0, st>>>(
+        t, N, c, static_cast<uint16_t *>(s_hi), static_cast<uint16_t *>(s_lo), ld, nbx, (int)nbin, W, R, w_hi, w_lo,
+        inv_scale, rowsum);
+    return cudaGetLastError();
 }
 
 // row j, columns (b, m): a warp takes 32 consecutive samples of one input j,

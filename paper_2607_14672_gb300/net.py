@@ -119,7 +119,7 @@ class DenseNet:
             if narrow_layer(n_in, n_out, self.layers[l]["M"], self.math):
                 n += 2                            # few outputs: one fused kernel each way (CUDA cores)
                 continue
-            n += 4                                # fwd: prep + binning + gemm + scan/solve
+            n += 3 if self.math == "x3" else 4    # fwd: [prep +] binning (x3: one launch for both) + gemm + scan
             n += 3 if tc else 4                   # bwd: dw^ + binning^T + dW gemm [+ split-K reduce]
             if l > 0:                             # bwd input times: prep W^T + dS gemm [+ gather]
                 n += 2 if tc else 3

@@ -292,6 +292,50 @@ def test_backward_matches_oracle(math_mode, tau_v, tau_I):
     assert np.all(host(g_t_in)[~np.isfinite(t_in)] == 0)
 
 
+@pytest.mark.parametrize("math_mode", ["f32", "x3"])
+@pytest.mark.parametrize("tau_v,tau_I", TAUS)
+@pytest.mark.parametrize("shape", [(9, 13, 7, 20), (16, 200, 1, 32), (12, 333, 32, 12), (20, 800, 10, 32)])
+def test_few_output_layer_matches_oracle(math_mode, tau_v, tau_I, shape):
+    """Layers with at most 32 outputs run forward and backward on CUDA cores
+    (a sparse sum over the two grid points of each input spike): spike times,
+    masks, dW (with the dead-neuron term) and the input-time gradient against
+    the oracle, over every kernel case, ragged sizes and a single output."""
+    from paper_2607_14672_gb300 import dstd
+    B, N_in, N_out, M = shape
+    t_in, layer = dense_layer(B + 8, N_in, N_out, M, tau_v, tau_I, seed=N_in + N_out, t_offset=0.003,
+                              gammas=(0.05, 0.01, 1e-3), edges=(0.35, 0.8), fire=0.6)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    t_in = _drop_ill_conditioned(t_in, layer)[:B]
+    B = t_in.shape[0]
+    assert B >= 4
+    r = run_fwd(t_in, layer, math_mode)
+    ctx = oracle_forward(t_in, layer["W"], layer)
+    check_times(r["t"], ctx, layer)
+    g = np.random.default_rng(3).normal(1.0, 0.5, r["t"].shape)
+    gup = np.where(np.isfinite(ctx["t"]), g, 0.0)
+    _, gT = olosses.temporal_penalty(ctx["t"], 0.35, 0.8, 0.05, 0.01, 1.0 / B)
+    gW_ref, gt_ref, _ = odstd.backward_dense(ctx, t_in, layer["W"], gup + gT, ctx["T"], ctx["dt"], tau_v, tau_I,
+                                             1.0)
+    _, cnt = olosses.dead_neuron_penalty(ctx["t"], layer["W"].sum(1), 1e-3, 1.0 / B)
+    gW_ref = gW_ref - 1e-3 / B * cnt[:, None]
+    for with_gt in (True, False):
+        g_t_in = torch.full((B, N_in), 7.0, device="cuda") if with_gt else None
+        g_W = torch.full((N_out, N_in), 7.0, device="cuda")
+        dstd.dense_bwd(r["t_dev"], r["W_dev"], r["t_out_dev"], r["saved"], dev(gup), r["p"], math_mode, g_t_in, g_W,
+                       r["ws"])
+        torch.cuda.synchronize()
+        assert rel_l2(host(g_W), gW_ref) <= 1e-3
+        if with_gt:
+            assert rel_l2(host(g_t_in), gt_ref) <= 1e-3
+            assert np.all(host(g_t_in)[~np.isfinite(t_in)] == 0)
+    # the forward's penalty sums, on the spike times the GPU produced
+    Tv, _ = olosses.temporal_penalty(r["t"], 0.35, 0.8, 0.05, 0.01, 1.0 / B)
+    Qv, _ = olosses.dead_neuron_penalty(r["t"], layer["W"].sum(1), 1e-3, 1.0 / B)
+    assert abs(r["pen"][0] - Tv) <= 1e-4 * abs(Tv) + 1e-7
+    assert abs(r["pen"][1] - Qv) <= 1e-4 * abs(Qv) + 1e-7
+    assert r["pen"][2] == (~np.isfinite(r["t"])).sum() and r["pen"][3] == np.isfinite(r["t"]).sum()
+
+
 def test_backward_without_input_gradient():
     from paper_2607_14672_gb300 import dstd
     t_in, layer = dense_layer(8, 64, 96, 16, 0.5, 0.25, seed=23)

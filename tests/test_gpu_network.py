@@ -167,6 +167,30 @@ def test_kernel_timing_counts_launches():
     assert all(ms > 0 for ms, c in tm.values() if c > 0)
 
 
+def test_kernel_timing_inside_a_graph():
+    """Timing on while a step is captured: every launch gets event-record
+    nodes in the graph, and each replay's kernel times are collected."""
+    from paper_2607_14672_gb300 import dstd
+    cfg, n, t0, lab = _cfg2_net("x3", batch=64, keep=np.arange(64))
+    n.step()
+    torch.cuda.synchronize()
+    dstd.timing_enable(True)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            n.step()
+        for _ in range(3):
+            g.replay()
+            dstd.timing_collect()
+    tm = dstd.timing_read()
+    dstd.timing_enable(False)
+    assert sum(c for _, c in tm.values()) == 3 * n.launches_per_step()
+    assert all(ms > 0 for ms, c in tm.values() if c > 0)
+    assert tm["gemm_fwd_scan"][1] == 6 and tm["narrow_bwd"][1] == 3
+
+
 def test_bounded_wait_reports_timeout():
     from paper_2607_14672_gb300 import dstd
     assert dstd.device_status(clear=True) == 0
