@@ -222,6 +222,16 @@ int dstd_adamw_multi(int count, float *const *w, const float *const *g, float *c
                      float eps, float weight_decay, int32_t *step, const float *lr_dev,
                      dstd_stream_t stream);
 
+/* How the forward contraction of a wide dense layer is scheduled: on single
+ * CTAs (128 x 128 tiles) or on SM pairs (tcgen05 cta_group::2, 256 x 128
+ * tiles, half of B per SM). policy 0 (the default) lets a cost model choose
+ * per layer; 1 takes SM pairs wherever they apply (x3 and bf16 forwards
+ * without split-K); 2 never does. Results agree to fp32 rounding either
+ * way. Returns the previous policy (0, 1 or 2), or DSTD_E_INVALID (negative)
+ * for another value.
+ * Process-wide; set it between calls, not while other threads launch. */
+int dstd_set_pair_policy(int policy);
+
 /* Kernel timing (tracing). While enabled, the library brackets every kernel
  * it launches with a CUDA event pair on the launching stream and files the
  * pair under the kernel's kind (dstd_kernel_kind_name).

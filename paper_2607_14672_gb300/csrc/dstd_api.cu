@@ -456,6 +456,19 @@ int dense_forward_core(const float *t_in, const float *W, int B, int N_in, int N
     // whose partial sums add into w^ (zeroed first).
     {
         const int splits = fwd_splits(N_out, cols, N_in);
+        if (splits == 1 && tc_gemm_pair_preferred((int)cols, N_out, N_in, op)) {
+            // on SM pairs, computed transposed: (S W^T)[(b, m), i], stored as w^[i][(b, m)]
+            {
+                Timed tm(KK_GEMM_FWD, st);
+                a.D = ws.D;
+                a.ldd = cols;
+                TRY(cu(launch_tc_gemm_pair_storeT(ws.s_hi, ws.s_lo, ws.kpad, ws.w_hi, ws.w_lo, ws.kpad, (int)cols,
+                                                  N_out, N_in, op, a, st)));
+            }
+            Timed ts(KK_SCAN, st);
+            return cu(launch_scan_solve(ws.D, c.Mp, cols, 1, B, N_out, c, nullptr, ws.rowsum, t_out, sv->q, sv->s,
+                                        sv->vdot, penalty, st));
+        }
         if (splits > 1) TRY(cu(cudaMemsetAsync(ws.D, 0, sizeof(float) * (size_t)N_out * cols, st)));
         Timed tm(KK_GEMM_FWD, st);
         a.D = ws.D;
@@ -980,6 +993,11 @@ int dstd_timing_enable(int on) {
     }
     g_timing.on = on != 0;
     return DSTD_OK;
+}
+
+int dstd_set_pair_policy(int policy) {
+    if (policy < 0 || policy > 2) return DSTD_E_INVALID;
+    return tc_gemm_pair_policy(policy);
 }
 
 int dstd_timing_collect(void) {

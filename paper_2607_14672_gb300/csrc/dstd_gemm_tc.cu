@@ -24,6 +24,7 @@
 #include "dstd_internal.cuh"
 
 #include <cuda.h>
+#include <atomic>
 #include <mutex>
 
 namespace dstd {
@@ -126,6 +127,26 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
             "r"(dst),
         "l"((uint64_t)map), "r"(x), "r"(y), "r"(smem_u32(bar))
         : "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_id_x() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_count_x() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+    return r;
+}
+// every thread of both CTAs of the cluster calls it once, converged
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols) {
@@ -569,6 +590,284 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Two-SM variant (tcgen05 cta_group::2). Clusters of two CTAs compute output
+// tiles of 256 rows x 128 columns, the MMA's M = 256 spanning the pair: each
+// CTA holds its own 128 rows of A and half (64 rows) of the tile's B in
+// shared memory, and the MMA issued by the even CTA reads B from both. Per
+// 64-deep K step of x3 an SM so takes in 48 KB of operands instead of 64 KB
+// for the same tensor work. D rows 0..127 of a tile land in the even CTA's
+// TMEM, rows 128..255 in the odd CTA's.
+//   full[s]    the even CTA's collects both CTAs' TMA bytes (the odd CTA's
+//              loads signal it remotely; the even CTA's producer arms it);
+//   empty[s]   in both CTAs, released by the even CTA's MMA commit (multicast);
+//   acc_full   in both CTAs, by the same commit after a tile's last MMA;
+//   acc_empty  the even CTA's, arrived on by the epilogue warps of both.
+// Epilogue StoreT: D^T[c][r] = acc[r][c] * col_scale[c], the transposed
+// store (the forward computes w^ as S W^T: rows (b, m), columns i, written
+// as w^[i][(b, m)]; consecutive lanes, consecutive addresses).
+// Every wait is bounded; neither CTA leaves before the other (cluster
+// barrier), and the pair frees its TMEM together.
+// ---------------------------------------------------------------------------
+constexpr int BM2 = 128;  // A rows per CTA (256 per pair)
+constexpr int BNH = 64;   // B rows per CTA (128 per pair: the MMA's N)
+
+template <int NPASS>
+struct Cfg2 {
+    static constexpr int A_BYTES = BM2 * BK * 2;
+    static constexpr int B_BYTES = BNH * BK * 2;
+    static constexpr int NOP = (NPASS == 3) ? 2 : 1;
+    static constexpr int STAGE = NOP * (A_BYTES + B_BYTES);
+    static constexpr int STAGES = (200 * 1024) / STAGE > 8 ? 8 : (200 * 1024) / STAGE;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    static constexpr int P_MAIN = (NPASS == 3) ? 3 : 4;
+    static constexpr int BNP = 2 * BNH;               // accumulator columns
+    static constexpr uint32_t TMEM_COLS = 4 * BNP;    // 512
+};
+
+__device__ __forceinline__ uint32_t mapa_rank(uint32_t saddr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+
+// TMA load into this CTA's shared memory whose completion is signalled on an
+// mbarrier of either CTA of the pair (a shared::cluster address)
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n"
+        "}\n" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"((uint16_t)3)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
+        "selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)
+        : "memory");
+    return ok != 0;
+}
+
+// bounded wait at cluster scope (barriers that a peer CTA arrives on)
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, bool sleep) {
+    const uint64_t t0 = globaltimer();
+    for (;;) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (globaltimer() - t0 > WAIT_NS) return false;
+        if (sleep) __nanosleep(256);
+    }
+}
+
+template <int NPASS, bool F16>
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_tc_gemm_pair(const __grid_constant__ CUtensorMap mA_hi, const __grid_constant__ CUtensorMap mA_lo,
+                   const __grid_constant__ CUtensorMap mB_hi, const __grid_constant__ CUtensorMap mB_lo, int R,
+                   int Cn, int ktiles, int n_row, int n_col, TcEpiArgs args) {
+    using C = Cfg2<NPASS>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + C::STAGES * C::STAGE);
+    uint64_t *empty = full + C::STAGES;
+    uint64_t *acc_full = empty + C::STAGES;
+    uint64_t *acc_empty = acc_full + 1;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rank = (int)cluster_ctarank();
+    const int cid = (int)cluster_id_x(), ncl = (int)cluster_count_x();
+    const bool leader = rank == 0;
+    const int ntiles = n_row * n_col;  // tiles of 256 x 128
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(acc_full, 1);
+        mbar_init(acc_empty, 2 * NEPI);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) tmem_alloc_pair(tmem_slot, C::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // both CTAs' barriers exist before any remote signal
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // TMA producer of this CTA's half of every stage
+            const uint32_t full0 = mapa_rank(smem_u32(&full[0]), 0);
+            uint32_t it = 0;
+            bool ok = true;
+            for (int t = cid; t < ntiles && ok; t += ncl) {
+                const int row0 = (t % n_row) * (2 * BM2) + rank * BM2;
+                const int brow0 = (t / n_row) * (2 * BNH) + rank * BNH;
+                for (int i = 0; i < ktiles; ++i, ++it) {
+                    const int s = it % C::STAGES;
+                    const uint32_t ph = (it / C::STAGES) & 1u;
+                    if (!mbar_wait_cluster(&empty[s], ph ^ 1u, false)) {
+                        set_status(STATUS_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    if (leader) mbar_expect_tx(&full[s], (uint32_t)(2 * C::STAGE));
+                    const uint32_t fb = full0 + (uint32_t)(s * sizeof(uint64_t));
+                    const int kx = i * BK;
+                    const uint32_t st = smem_u32(smem + s * C::STAGE);
+                    tma_load_2d_pair(st, &mA_hi, fb, kx, row0);
+                    if (NPASS == 3) tma_load_2d_pair(st + C::A_BYTES, &mA_lo, fb, kx, row0);
+                    const uint32_t sb = st + C::NOP * C::A_BYTES;
+                    tma_load_2d_pair(sb, &mB_hi, fb, kx, brow0);
+                    if (NPASS == 3) tma_load_2d_pair(sb + C::B_BYTES, &mB_lo, fb, kx, brow0);
+                }
+            }
+            if (ok) {
+                // every stage released by the pair's MMAs: no commit targets this CTA afterwards
+                for (int i = 0; i < C::STAGES; ++i, ++it) {
+                    const int s = it % C::STAGES;
+                    const uint32_t ph = (it / C::STAGES) & 1u;
+                    if (!mbar_wait_cluster(&empty[s], ph ^ 1u, false)) {
+                        set_status(STATUS_TIMEOUT);
+                        break;
+                    }
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0 && leader) {
+            // MMA issuer of the pair
+            constexpr uint32_t idesc = idesc_16bit(2 * BM2, C::BNP, F16);
+            uint32_t it = 0, j = 0;
+            bool ok = true;
+            for (int t = cid; t < ntiles && ok; t += ncl, ++j) {
+                if (j > 0) {
+                    // both CTAs' epilogues have taken the previous tile
+                    if (!mbar_wait_cluster(acc_empty, (j - 1) & 1u, false)) {
+                        set_status(STATUS_TIMEOUT);
+                        break;
+                    }
+                    tc_fence_after();
+                }
+                for (int i = 0; i < ktiles; ++i, ++it) {
+                    const int s = it % C::STAGES;
+                    const uint32_t ph = (it / C::STAGES) & 1u;
+                    if (!mbar_wait_cluster(&full[s], ph, false)) {
+                        set_status(STATUS_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_hi = smem_u32(smem + s * C::STAGE);
+                    const uint32_t a_lo = a_hi + C::A_BYTES;
+                    const uint32_t b_hi = a_hi + C::NOP * C::A_BYTES;
+                    const uint32_t b_lo = b_hi + C::B_BYTES;
+                    const uint32_t acc_main = tmem + (uint32_t)((i % C::P_MAIN) * C::BNP);
+                    const uint32_t acc_corr = tmem + (uint32_t)(3 * C::BNP);
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint64_t da = sdesc_sw128(a_hi + kk * 32);
+                        const uint64_t db = sdesc_sw128(b_hi + kk * 32);
+                        mma_pair(acc_main, da, db, idesc, (i >= C::P_MAIN || kk > 0) ? 1u : 0u);
+                        if (NPASS == 3) {
+                            mma_pair(acc_corr, da, sdesc_sw128(b_lo + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                            mma_pair(acc_corr, sdesc_sw128(a_lo + kk * 32), db, idesc, 1u);
+                        }
+                    }
+                    mma_commit_pair(&empty[s]);
+                }
+                if (ok) mma_commit_pair(acc_full);
+            }
+        }
+        __syncwarp();
+    } else {
+        // epilogue warps of both CTAs: this CTA's 128 rows of the tile
+        const int ew = warp - 2;
+        const int quarter = warp & 3, group = ew >> 2;
+        const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t acc_empty0 = mapa_rank(smem_u32(acc_empty), 0);
+        const int c_lo = group * GCOLS;
+        const int n_main = ktiles < C::P_MAIN ? ktiles : C::P_MAIN;
+        uint32_t j = 0;
+        for (int t = cid; t < ntiles; t += ncl, ++j) {
+            const int row = (t % n_row) * (2 * BM2) + rank * BM2 + quarter * 32 + lane;
+            const int col0 = (t / n_row) * C::BNP + c_lo;
+            if (!mbar_wait_cluster(acc_full, j & 1u, true)) {
+                set_status(STATUS_TIMEOUT);
+                break;
+            }
+            tc_fence_after();
+            float v[GCOLS / 32][32];
+#pragma unroll
+            for (int h = 0; h < GCOLS / 32; ++h) tmem_ld_acc<C::BNP>(tbase, c_lo + 32 * h, n_main, NPASS == 3, v[h]);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acc_empty0);
+            if (row < R) {
+#pragma unroll
+                for (int h = 0; h < GCOLS / 32; ++h) {
+#pragma unroll
+                    for (int jj = 0; jj < 32; ++jj) {
+                        const int col = col0 + 32 * h + jj;
+                        if (col < Cn) {
+                            const float cs = args.row_scale ? args.row_scale[col] : 1.0f;
+                            args.D[(long long)col * args.ldd + row] = v[h][jj] * cs;
+                        }
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // both epilogues done with TMEM, every remote arrive landed
+    if (warp == 1) tmem_dealloc_pair(tmem, C::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------
 // Host side: tensor maps and launch.
 // ---------------------------------------------------------------------------
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -638,6 +937,116 @@ static cudaError_t launch_one(const CUtensorMap &a_hi, const CUtensorMap &a_lo, 
 cudaError_t launch_wait_selftest(unsigned long long limit_ns, cudaStream_t st) {
     tc::k_wait_selftest<<<1, 32, 0, st>>>(limit_ns);
     return cudaGetLastError();
+}
+
+namespace tc {
+// SM pairs that can hold a pair kernel's clusters at once (a pair must sit in
+// one GPC: a GPC with an odd number of usable SMs leaves one out)
+template <int NPASS, bool F16>
+static int resident_pairs() {
+    static int resident = 0;
+    if (resident == 0) {
+        using C = Cfg2<NPASS>;
+        auto kern = k_tc_gemm_pair<NPASS, F16>;
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) != cudaSuccess) return 0;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        cfg.blockDim = dim3(NTHREADS);
+        cfg.dynamicSmemBytes = C::SMEM;
+        cfg.gridDim = dim3((num_sms() / 2) * 2);
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) return 0;
+        resident = n;
+    }
+    return resident;
+}
+
+template <int NPASS, bool F16>
+static cudaError_t launch_pair(const CUtensorMap &a_hi, const CUtensorMap &a_lo, const CUtensorMap &b_hi,
+                               const CUtensorMap &b_lo, int R, int Cn, int K, const TcEpiArgs &args,
+                               cudaStream_t st) {
+    using C = Cfg2<NPASS>;
+    auto kern = k_tc_gemm_pair<NPASS, F16>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    const int ktiles = (K + BK - 1) / BK;
+    const int n_row = (R + 2 * BM2 - 1) / (2 * BM2), n_col = (Cn + C::BNP - 1) / C::BNP;
+    const long long ntiles = (long long)n_row * n_col;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.blockDim = dim3(NTHREADS);
+    cfg.dynamicSmemBytes = C::SMEM;
+    cfg.stream = st;
+    // persistent: as many pairs as can be resident at once
+    const int resident = resident_pairs<NPASS, F16>();
+    if (resident < 1) return cudaErrorInvalidConfiguration;
+    const int pairs = (int)(ntiles < resident ? ntiles : resident);
+    cfg.gridDim = dim3(2 * pairs);
+    return cudaLaunchKernelEx(&cfg, kern, a_hi, a_lo, b_hi, b_lo, R, Cn, ktiles, n_row, n_col, args);
+}
+}  // namespace tc
+
+// Work on the busiest SM, in units of one K step of a single-CTA tile: rounds
+// of 128 x 128 tiles on single CTAs, (K steps + 2) each, against rounds of
+// 256 x 128 tiles on resident SM pairs, (0.92 K steps + 4) each. A pair's K
+// step is cheaper (each SM takes in 48 KB instead of 64 KB of operands), its
+// tile boundary dearer (the handshakes between the two SMs); fitted to the
+// 784-wide forward of the MLP (13 K steps: single CTAs faster) and 4096- and
+// 8192-wide layers (64 and 128 K steps: pairs faster, 85-90% against 83% of
+// the bf16 peak).
+static std::atomic<int> g_pair_policy{0};
+
+int tc_gemm_pair_policy(int policy) {
+    if (policy < 0 || policy > 2) return g_pair_policy.load();
+    return g_pair_policy.exchange(policy);
+}
+
+bool tc_gemm_pair_preferred(int R, int Cn, int K, OpKind op) {
+    if (op != OpKind::F16X3 && op != OpKind::BF16) return false;
+    const int policy = g_pair_policy.load();
+    if (policy != 0) return policy == 1;
+    const int pairs = op == OpKind::F16X3 ? tc::resident_pairs<3, true>() : tc::resident_pairs<1, false>();
+    if (pairs < 1) return false;
+    const long long t1 = (long long)((R + 127) / 128) * ((Cn + 127) / 128);
+    const long long t2 = (long long)((R + 255) / 256) * ((Cn + 127) / 128);
+    const long long r1 = (t1 + tc::num_sms() - 1) / tc::num_sms(), r2 = (t2 + pairs - 1) / pairs;
+    const double kt = (double)((K + tc::BK - 1) / tc::BK);
+    return (double)r2 * (0.92 * kt + 4.0) < (double)r1 * (kt + 2.0);
+}
+
+int tc_gemm_resident_pairs(OpKind op) {
+    return op == OpKind::F16X3 ? tc::resident_pairs<3, true>() : tc::resident_pairs<1, false>();
+}
+
+cudaError_t launch_tc_gemm_pair_storeT(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo,
+                                       int ldb, int R, int Cn, int K, OpKind op, const TcEpiArgs &args,
+                                       cudaStream_t st) {
+    CUtensorMap a_hi, a_lo, b_hi, b_lo;
+    const bool three = (op == OpKind::BF16X3 || op == OpKind::F16X3);
+    const bool f16 = (op == OpKind::F16X3);
+    if (op == OpKind::F32 || op == OpKind::BF16X3) return cudaErrorInvalidValue;
+    if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM2, f16) || !tc::make_map(&b_hi, B_hi, Cn, K, ldb, tc::BNH, f16))
+        return cudaErrorInvalidValue;
+    if (three) {
+        if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM2, f16) || !tc::make_map(&b_lo, B_lo, Cn, K, ldb, tc::BNH, f16))
+            return cudaErrorInvalidValue;
+        return tc::launch_pair<3, true>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, args, st);
+    }
+    a_lo = a_hi;
+    b_lo = b_hi;
+    return tc::launch_pair<1, false>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, args, st);
 }
 
 int tc_gemm_splits_valid(int K, int splits) {

@@ -378,6 +378,19 @@ struct TcEpiArgs {
 cudaError_t launch_tc_gemm(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo, int ldb,
                            int R, int Cn, int K, int splits, OpKind op, Epi epi, const TcEpiArgs &args,
                            cudaStream_t st, bool b_mn = false);
+// The same product on SM pairs (tcgen05 cta_group::2, 256 x 128 tiles), with
+// the transposed store D[c * ldd + r] = (A B^T)[r][c] * row_scale[c]
+// (args.D, args.ldd, args.row_scale): A [R, K] rows, B [Cn, K] rows. For the
+// F16X3 and BF16 forward operands.
+cudaError_t launch_tc_gemm_pair_storeT(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo,
+                                       int ldb, int R, int Cn, int K, OpKind op, const TcEpiArgs &args,
+                                       cudaStream_t st);
+// whether the pair kernel is expected to beat the single-CTA one for an
+// R x Cn x K product (resident pairs counted once per process)
+bool tc_gemm_pair_preferred(int R, int Cn, int K, OpKind op);
+int tc_gemm_resident_pairs(OpKind op);
+// 0 the cost model, 1 pairs wherever they apply, 2 never pairs; returns the previous setting
+int tc_gemm_pair_policy(int policy);
 
 cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
                            float *loss, float *g, cudaStream_t st);

@@ -21,7 +21,7 @@ ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "
 EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning", "dstd_dense_what",
            "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
-           "dstd_timing_read", "dstd_timing_collect", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
+           "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd")
 
 
@@ -85,6 +85,7 @@ def load(path=None):
         "dstd_timing_enable": (_I, [_I]),
         "dstd_timing_read": (_I, [_I, ctypes.POINTER(_F), ctypes.POINTER(_I64)]),
         "dstd_timing_collect": (_I, []),
+        "dstd_set_pair_policy": (_I, [_I]),
         "dstd_kernel_kind_count": (_I, []),
         "dstd_kernel_kind_name": (ctypes.c_char_p, [_I]),
         "dstd_selftest_wait_timeout": (_I, [ctypes.c_uint32, _P]),
@@ -292,6 +293,15 @@ def device_status(clear=True):
 def timing_enable(on=True):
     """Turn per-kernel event timing on/off (clears the counters)."""
     _check(load().dstd_timing_enable(1 if on else 0), "dstd_timing_enable")
+
+
+def set_pair_policy(policy):
+    """Forward contraction scheduling: 0 cost model (default), 1 SM pairs
+    wherever they apply, 2 single CTAs only. Returns the previous policy."""
+    r = load().dstd_set_pair_policy(int(policy))
+    if r < 0:
+        raise DstdError(r, "dstd_set_pair_policy")
+    return r
 
 
 def timing_collect():

@@ -104,6 +104,9 @@ def test_null_and_bad_arguments_rejected_on_host(lib):
                           ctypes.c_float(1e-8), ctypes.c_float(0.0), 1, None) == -1
     assert lib.dstd_adamw(one, one, one, one, 10, ctypes.c_float(1e-3), ctypes.c_float(0.9), ctypes.c_float(0.9),
                           ctypes.c_float(1e-8), ctypes.c_float(0.0), 0, None) == -1
+    # contraction scheduling policy: 0, 1, 2 valid (previous returned), anything else rejected
+    assert lib.dstd_set_pair_policy(3) == -1 and lib.dstd_set_pair_policy(-1) == -1
+    assert lib.dstd_set_pair_policy(2) == 0 and lib.dstd_set_pair_policy(0) == 2
     # multi-tensor AdamW: tensor count, null step buffer, misaligned step buffer, empty tensor, bad beta
     ptrs = (ctypes.c_void_p * 33)(*([256] * 33))
     ns = (ctypes.c_int64 * 33)(*([10] * 33))

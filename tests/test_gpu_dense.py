@@ -212,6 +212,37 @@ def test_forward_ragged_shapes(math_mode, shape):
     check_times(r["t"], ctx, layer)
 
 
+@pytest.fixture
+def pair_policy():
+    from paper_2607_14672_gb300 import dstd
+    old = dstd.set_pair_policy(0)
+    yield dstd.set_pair_policy
+    dstd.set_pair_policy(old)
+
+
+@pytest.mark.parametrize("math_mode", ["x3", "bf16"])
+@pytest.mark.parametrize("shape", [(1, 8, 129, 8), (3, 300, 257, 100), (8, 200, 300, 32), (16, 784, 100, 8),
+                                   (9, 257, 513, 32)])
+def test_forward_on_sm_pairs_matches_single_ctas(math_mode, shape, pair_policy):
+    """The forward contraction on SM pairs (tcgen05 cta_group::2, computed
+    transposed and stored back in the scan's layout) against the single-CTA
+    kernel, and the spike times against the oracle, on ragged shapes: row
+    counts that are not multiples of 256, outputs that are not multiples of
+    128, K not a multiple of 64."""
+    B, N_in, N_out, M = shape
+    t_in, layer = dense_layer(B, N_in, N_out, M, 0.5, 0.25, seed=B + N_in + M + 1, fire=0.5)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    pair_policy(1)
+    r2 = run_fwd(t_in, layer, math_mode)
+    pair_policy(2)
+    r1 = run_fwd(t_in, layer, math_mode)
+    ok = np.isfinite(r1["t"]) & np.isfinite(r2["t"])
+    assert (np.isfinite(r1["t"]) == np.isfinite(r2["t"])).mean() > 0.995
+    assert np.abs(r1["t"][ok] - r2["t"][ok]).max() <= 1e-4 * (layer["t_end"] - layer["t_first"])
+    if math_mode == "x3":
+        check_times(r2["t"], oracle_forward(t_in, layer["W"], layer), layer)
+
+
 def test_forward_f32_long_grid():
     # M = 256 runs on the CUDA-core path only
     t_in, layer = dense_layer(4, 64, 48, 256, 0.5, 0.25, seed=2)
