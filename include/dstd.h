@@ -187,6 +187,22 @@ int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const v
                   dstd_math math, float *g_t_in, float *g_W, void *workspace, size_t ws_bytes,
                   dstd_stream_t stream);
 
+/* The output layer's forward followed by the cross-entropy of its spike
+ * times: the results of dstd_dense_fwd and then dstd_ce_loss(t_out, labels,
+ * B, N_out, tau_soft, t_silent, loss, g_t_out). A layer on the few-output
+ * path (at most 32 outputs, fp32 or three-product mode) computes the loss in
+ * the same kernel, one block per sample, and the batch mean in sample order.
+ *  loss: float[2], 8-byte aligned: loss[0] out; loss[1] is the kernel's
+ *        scratch, zero before the first call (each call leaves it zero);
+ *  labels [B] int32 in [0, N_out); g_t_out [B, N_out] out;
+ *  the workspace also holds B floats of per-sample terms.
+ * Errors as dstd_dense_fwd and dstd_ce_loss. */
+int dstd_dense_fwd_ce(const float *t_in, const float *W, int B, int N_in, int N_out,
+                      const dstd_params *p, dstd_math math, float *t_out, void *saved,
+                      float *penalty, void *workspace, size_t ws_bytes, const int32_t *labels,
+                      float tau_soft, float t_silent, float *loss, float *g_t_out,
+                      dstd_stream_t stream);
+
 /* Cross-entropy over softmax(-t/tau_soft) (Eqs. cost_function, L, S_i),
  * mini-batch mean; a silent output enters with the constant time t_silent
  * and passes no gradient.

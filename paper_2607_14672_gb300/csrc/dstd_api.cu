@@ -676,6 +676,42 @@ int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
     return dense_forward_core(t_in, W, B, N_in, N_out, c, op, ws, false, &sv, t_out, penalty, st);
 }
 
+int dstd_dense_fwd_ce(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
+                      dstd_math math, float *t_out, void *saved, float *penalty, void *workspace, size_t ws_bytes,
+                      const int32_t *labels, float tau_soft, float t_silent, float *loss, float *g_t_out,
+                      dstd_stream_t stream) {
+    if (!labels || !loss || !g_t_out) return DSTD_E_INVALID;
+    if (!(tau_soft > 0.0f) || !isfinite(tau_soft) || !isfinite(t_silent)) return DSTD_E_INVALID;
+    if (!t_in || !W || !t_out || !saved || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    if ((reinterpret_cast<uintptr_t>(loss) & 7) != 0) return DSTD_E_INVALID;
+    const OpKind op = op_of(math);
+    if (ws_bytes < fwd_layout(nullptr, B, N_in, N_out, Mp, op, false).bytes || ws_bytes < sizeof(float) * (size_t)B)
+        return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    cudaStream_t st = (cudaStream_t)stream;
+    if (!narrow_layer(N_in, N_out, p->M, op)) {
+        TRY(dstd_dense_fwd(t_in, W, B, N_in, N_out, p, math, t_out, saved, penalty, workspace, ws_bytes, stream));
+        return dstd_ce_loss(t_out, labels, B, N_out, tau_soft, t_silent, loss, g_t_out, stream);
+    }
+    LifConst c = make_const(*p, Mp);
+    Saved sv = saved_view(saved, B, N_out);
+    if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
+    NarrowCe ce;
+    ce.labels = labels;
+    ce.tau_soft = tau_soft;
+    ce.t_silent = t_silent;
+    ce.loss = loss;
+    ce.g = g_t_out;
+    ce.scratch = static_cast<float *>(workspace);
+    Timed tm(KK_NARROW_FWD, st);
+    return cu(launch_narrow_fwd(t_in, W, B, N_in, N_out, c, t_out, sv.q, sv.s, sv.vdot, penalty, st, ce));
+}
+
 int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const void *saved, const float *g_t_out,
                    int B, int N_in, int N_out, const dstd_params *p, dstd_math math, float *g_t_in, float *g_W,
                    void *workspace, size_t ws_bytes, dstd_stream_t stream) {

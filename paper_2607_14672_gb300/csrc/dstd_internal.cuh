@@ -329,8 +329,18 @@ constexpr int kNarrowMaxOut = 32;
 constexpr int kNarrowMaxIn = 4096;       // the forward sorts a sample's inputs in shared memory
 constexpr size_t kNarrowMaxSmem = 200 * 1024;  // and holds W there: its shared memory, at most this
 size_t narrow_fwd_smem(int N_in, int N_out, int M, int Mp);
+// Cross-entropy of the output layer fused into its few-output forward:
+// loss float[2] (loss[1] a ticket: zero before the first call, left zero),
+// g [B, N_out], scratch float[B] (per-sample terms, summed in order by the
+// last block); loss == nullptr: no loss.
+struct NarrowCe {
+    const int32_t *labels = nullptr;
+    float tau_soft = 1.f, t_silent = 0.f;
+    float *loss = nullptr, *g = nullptr, *scratch = nullptr;
+};
 cudaError_t launch_narrow_fwd(const float *t, const float *W, int B, int N_in, int N_out, const LifConst &c,
-                              float *t_out, int *q, float *s, float *vdot, float *penalty, cudaStream_t st);
+                              float *t_out, int *q, float *s, float *vdot, float *penalty, cudaStream_t st,
+                              const NarrowCe &ce = NarrowCe());
 // zeroes g_W, then adds every block's share
 cudaError_t launch_narrow_bwd(const float *t_in, const float *W, const float *t_out, const int *q, const float *s,
                               const float *vdot, const float *g_up, int B, int N_in, int N_out, const LifConst &c,

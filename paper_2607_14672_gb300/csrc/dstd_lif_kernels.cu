@@ -893,7 +893,7 @@ template <int SUB, int NOUT>
 __global__ void __launch_bounds__(NARROW_FWD_THREADS) k_narrow_fwd(const float *__restrict__ t,
                                                                  const float *__restrict__ W, int N_in, int N_out,
                                                                  LifConst c, float *t_out, int *q, float *s,
-                                                                 float *vdot, float *penalty) {
+                                                                 float *vdot, float *penalty, NarrowCe ce) {
     constexpr int NW = NARROW_FWD_THREADS / 32;
     extern __shared__ __align__(16) unsigned char nsm[];
     const int NK = c.M + 2;  // keys 0 .. M, and M + 1 for "no weight"
@@ -1065,6 +1065,42 @@ __global__ void __launch_bounds__(NARROW_FWD_THREADS) k_narrow_fwd(const float *
         finish_neuron(c, st, b, i, N_out, rsum, t_out, q, s, vdot, pacc);
     }
     flush_penalty(pacc, penalty);
+    if (ce.loss == nullptr) return;
+    // cross-entropy over softmax(-t / tau_soft) of this sample (Eqs.
+    // cost_function, L, S_i), one lane per output: a silent output enters
+    // with t_silent and passes no gradient; the batch mean of the per-sample
+    // terms is taken by the block that finishes last, in sample order
+    __syncthreads();  // the sample's t_out (written above) visible to warp 0
+    if (warp != 0) return;
+    const float inv_tau = 1.0f / ce.tau_soft;
+    const int B = gridDim.x, y = ce.labels[b];
+    const float x = lane < N_out ? t_out[(long long)b * N_out + lane] : INFINITY;
+    const bool fin = isfinite(x);
+    const float z = lane < N_out ? -(fin ? x : ce.t_silent) * inv_tau : -INFINITY;
+    float zmax = z;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) zmax = fmaxf(zmax, __shfl_xor_sync(0xffffffffu, zmax, o));
+    const float e = lane < N_out ? expf(z - zmax) : 0.f;
+    const float den = warp_sum(e);
+    const float zy = __shfl_sync(0xffffffffu, z, y & 31);
+    if (lane < N_out)
+        ce.g[(long long)b * N_out + lane] = fin ? (-inv_tau / (float)B) * (e / den - (lane == y ? 1.f : 0.f)) : 0.f;
+    unsigned ticket = 0u;
+    if (lane == 0) {
+        ce.scratch[b] = -(zy - zmax - logf(den)) / (float)B;
+        __threadfence();
+        ticket = atomicAdd(reinterpret_cast<unsigned int *>(ce.loss + 1), 1u);
+    }
+    ticket = __shfl_sync(0xffffffffu, ticket, 0);
+    if (ticket != (unsigned)(B - 1)) return;
+    __threadfence();
+    float sum = 0.f;
+    for (int k = lane; k < B; k += 32) sum += __ldcg(ce.scratch + k);
+    sum = warp_sum(sum);
+    if (lane == 0) {
+        ce.loss[0] = sum;
+        reinterpret_cast<unsigned int *>(ce.loss)[1] = 0u;
+    }
 }
 
 size_t narrow_fwd_smem(int N_in, int N_out, int M, int Mp) {
@@ -1074,7 +1110,8 @@ size_t narrow_fwd_smem(int N_in, int N_out, int M, int Mp) {
 }
 
 cudaError_t launch_narrow_fwd(const float *t, const float *W, int B, int N_in, int N_out, const LifConst &c,
-                              float *t_out, int *q, float *s, float *vdot, float *penalty, cudaStream_t st) {
+                              float *t_out, int *q, float *s, float *vdot, float *penalty, cudaStream_t st,
+                              const NarrowCe &ce) {
     if (N_out < 1 || N_out > kNarrowMaxOut || N_in > kNarrowMaxIn || c.M + 2 > 96) return cudaErrorInvalidValue;
     const size_t smem = narrow_fwd_smem(N_in, N_out, c.M, c.Mp);
     if (smem > kNarrowMaxSmem) return cudaErrorInvalidValue;
@@ -1082,7 +1119,7 @@ cudaError_t launch_narrow_fwd(const float *t, const float *W, int B, int N_in, i
 #define DSTD_NARROW_FWD(S, NO)                                                                                    \
     e = cudaFuncSetAttribute(k_narrow_fwd<S, NO>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);        \
     if (e != cudaSuccess) return e;                                                                                \
-    k_narrow_fwd<S, NO><<<B, NARROW_FWD_THREADS, smem, st>>>(t, W, N_in, N_out, c, t_out, q, s, vdot, penalty);
+    k_narrow_fwd<S, NO><<<B, NARROW_FWD_THREADS, smem, st>>>(t, W, N_in, N_out, c, t_out, q, s, vdot, penalty, ce);
 #define DSTD_NARROW_FWD_NO(S) \
     if (N_out <= 8) {         \
         DSTD_NARROW_FWD(S, 8) \

@@ -19,7 +19,7 @@ ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "
           -6: "no usable sm_103 device"}
 
 EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning", "dstd_dense_what",
-           "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
+           "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_fwd_ce", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd")
@@ -74,6 +74,7 @@ def load(path=None):
         "dstd_dense_what": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _SZ, _P]),
         "dstd_scan_solve": (_I, [_P, _I, _I, _PP, _P, _P, _P, _P, _P]),
         "dstd_dense_fwd": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _P, _SZ, _P]),
+        "dstd_dense_fwd_ce": (_I, [_P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _P, _SZ, _P, _F, _F, _P, _P, _P]),
         "dstd_dense_bwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
         "dstd_ce_loss": (_I, [_P, _P, _I, _I, _F, _F, _P, _P, _P]),
         "dstd_sum_t_loss": (_I, [_P, _I64, _P, _P, _P]),
@@ -184,6 +185,25 @@ def dense_fwd(t_in, W, p, math_mode, t_out, saved, penalty, workspace, stream=No
     _check(load().dstd_dense_fwd(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), MATH[math_mode], _ptr(t_out),
                                  _ptr(saved), _ptr(penalty), _ptr(workspace),
                                  workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_dense_fwd")
+
+
+def dense_fwd_ce(t_in, W, p, math_mode, t_out, saved, penalty, workspace, labels, tau_soft, t_silent, loss,
+                 g_t_out, stream=None):
+    """dense_fwd of the output layer, then the CE loss of its spike times
+    (fused into one kernel on the few-output path). loss: float32[2] device
+    tensor, loss[1] zero before the first call (left zero)."""
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(t_out, "t_out", (B, N_out))
+    _f32(g_t_out, "g_t_out", (B, N_out))
+    if loss.numel() < 2:
+        raise ValueError("dense_fwd_ce: loss must hold 2 floats (value, scratch)")
+    _check(load().dstd_dense_fwd_ce(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), MATH[math_mode],
+                                    _ptr(t_out), _ptr(saved), _ptr(penalty), _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(), _ptr(labels), float(tau_soft),
+                                    float(t_silent), _ptr(loss), _ptr(g_t_out), _stream(stream)), "dstd_dense_fwd_ce")
 
 
 def dense_fwd_noalloc(t_in, W, p, math_mode, t_out, saved, penalty=None, stream=None):

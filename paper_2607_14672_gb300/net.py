@@ -51,7 +51,8 @@ class DenseNet:
         if ws == 0:
             raise ValueError("unsupported layer sizes or constants for the library")
         self.workspace = torch.empty(ws, dtype=torch.uint8, device=dev)
-        self.loss = torch.zeros(1, dtype=torch.float32, device=dev)
+        # (loss value, scratch of the fused output-layer loss: zero between calls)
+        self.loss = torch.zeros(2, dtype=torch.float32, device=dev)
         self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
         self.with_adamw = with_adamw
         if with_adamw:
@@ -87,6 +88,21 @@ class DenseNet:
         else:
             dstd.sum_t_loss(self.t[-1], self.loss, self.g[-1], stream)
 
+    def forward_loss(self, stream=None):
+        """forward, then the loss; with the CE loss the output layer and the
+        loss are one library call (one kernel when the layer has few outputs)."""
+        if self.loss_kind != "ce":
+            self.forward(stream)
+            self.loss_grad(stream)
+            return
+        L = len(self.W)
+        for l in range(L - 1):
+            dstd.dense_fwd(self.layer_input(l), self.W[l], self.p[l], self.math, self.t[l], self.saved[l],
+                           self.penalty[l], self.workspace, stream)
+        dstd.dense_fwd_ce(self.layer_input(L - 1), self.W[L - 1], self.p[L - 1], self.math, self.t[L - 1],
+                          self.saved[L - 1], self.penalty[L - 1], self.workspace, self.labels, self.cfg["tau_soft"],
+                          self.layers[-1]["t_end"], self.loss, self.g[L - 1], stream)
+
     def backward(self, stream=None):
         for l in range(len(self.W) - 1, -1, -1):
             g_in = self.g[l - 1] if l > 0 else None
@@ -99,8 +115,7 @@ class DenseNet:
 
     def step(self, stream=None):
         """One training step: forward, loss, backward (and AdamW if enabled)."""
-        self.forward(stream)
-        self.loss_grad(stream)
+        self.forward_loss(stream)
         self.backward(stream)
         if self.with_adamw:
             self.optimizer(stream=stream)
@@ -113,7 +128,9 @@ class DenseNet:
         """Kernels the library launches per ``step`` (memsets not counted)."""
         tc = self.math != "f32"
         L = len(self.W)
-        n = 1                                     # loss
+        fused_loss = self.loss_kind == "ce" and narrow_layer(self.sizes[-2], self.sizes[-1], self.layers[-1]["M"],
+                                                             self.math)
+        n = 0 if fused_loss else 1                # loss (inside the output layer's kernel when fused)
         for l in range(L):
             n_in, n_out = self.sizes[l], self.sizes[l + 1]
             if narrow_layer(n_in, n_out, self.layers[l]["M"], self.math):

@@ -367,6 +367,45 @@ def test_few_output_layer_matches_oracle(math_mode, tau_v, tau_I, shape):
     assert r["pen"][2] == (~np.isfinite(r["t"])).sum() and r["pen"][3] == np.isfinite(r["t"]).sum()
 
 
+@pytest.mark.parametrize("math_mode", ["f32", "x3"])
+@pytest.mark.parametrize("B,N_in,N_out", [(64, 300, 10), (7, 13, 1), (33, 800, 32), (16, 120, 40)])
+def test_output_layer_with_fused_loss(math_mode, B, N_in, N_out):
+    """dense_fwd_ce (the output layer and its CE loss, one kernel on the
+    few-output path) against dense_fwd followed by ce_loss: the same spike
+    times, the loss and its gradient to fp32 rounding; the loss is the same
+    on a second call (the batch mean has a fixed order) and the scratch word
+    is left zero. (16, 120, 40) has too many outputs for the fused kernel and
+    takes the two calls."""
+    from paper_2607_14672_gb300 import dstd
+    t_in, layer = dense_layer(B, N_in, N_out, 32, 0.5, 0.25, seed=B + N_out, fire=0.8)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    labels = torch.tensor(np.random.default_rng(5).integers(0, N_out, B).astype(np.int32), device="cuda")
+    r = run_fwd(t_in, layer, math_mode)
+    loss_ref = torch.empty(1, device="cuda")
+    g_ref = torch.empty(B, N_out, device="cuda")
+    dstd.ce_loss(r["t_out_dev"], labels, 0.02, layer["t_end"], loss_ref, g_ref)
+    t_out = torch.empty(B, N_out, device="cuda")
+    saved = torch.empty(dstd.dense_saved_bytes(B, N_out), dtype=torch.uint8, device="cuda")
+    pen = torch.empty(4, device="cuda")
+    loss = torch.zeros(2, device="cuda")
+    g = torch.empty(B, N_out, device="cuda")
+    vals = []
+    for _ in range(2):
+        dstd.dense_fwd_ce(r["t_dev"], r["W_dev"], r["p"], math_mode, t_out, saved, pen, r["ws"], labels, 0.02,
+                          layer["t_end"], loss, g)
+        torch.cuda.synchronize()
+        vals.append(host(loss).copy())
+    np.testing.assert_array_equal(host(t_out), r["t"])
+    np.testing.assert_array_equal(host(pen), r["pen"])
+    assert vals[0][0] == vals[1][0] and vals[0][1] == 0.0 and vals[1][1] == 0.0
+    assert vals[0][0] == pytest.approx(host(loss_ref)[0], rel=1e-5)
+    # g = (p - [k = y]) / (tau_soft B): at the label with p near 1 the
+    # difference cancels, so the two evaluations (a butterfly and a serial sum
+    # for the softmax denominator) agree to fp32 rounding of the gradient's
+    # scale 1 / (tau_soft B), not element-wise relatively
+    np.testing.assert_allclose(host(g), host(g_ref), rtol=1e-5, atol=2e-6 / (0.02 * B))
+
+
 def test_backward_without_input_gradient():
     from paper_2607_14672_gb300 import dstd
     t_in, layer = dense_layer(8, 64, 96, 16, 0.5, 0.25, seed=23)
