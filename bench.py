@@ -41,6 +41,9 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--exact", action="store_true",
+                    help="instead of the training step: time the exact (event-driven, Alg. 1) forward against the "
+                         "DSTD forward on the same GPU, per layer shape, and print one JSON line")
     ap.add_argument("--profile", action="store_true",
                     help="only warm-up and the timed replays (for an ncu launch list); no clocks, "
                          "per-kernel timing pass, e2e or CPU baseline")
@@ -475,11 +478,79 @@ def run_ours(args, rank, world, local):
     return 0
 
 
+def run_exact_compare(args, local):
+    """Exact forward (sort + interval sweep, Alg. 1) against the DSTD forward
+    (binning, contraction, scan/solve) of the same layers on one GPU: device
+    time per forward (CUDA events, L2 flushed before each), and how far the
+    two methods' spike times are apart (median over neurons firing in both)."""
+    import numpy as np
+    import torch
+
+    from paper_2607_14672_gb300 import build as _b
+    _b.build()
+    from paper_2607_14672_gb300 import configs, dstd
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    cases = []
+    c2 = configs.config2()
+    t2 = np.asarray(c2["inputs"](), np.float32)
+    cases.append(("784-800-800-10 MLP, layer 1", c2["layers"][0], t2))
+    for N in (1024, 4096):
+        c3 = configs.config3(N, 32)
+        cases.append((f"{N}->{N} layer, M=32", c3["layers"][0], np.asarray(c3["inputs"](), np.float32)))
+    reps = max(3, min(args.steps, 20))
+    out = []
+    stream = torch.cuda.Stream(device=dev)
+    for name, L, t_np in cases:
+        B, N_in = t_np.shape
+        W = torch.tensor(np.asarray(L["W"], np.float32), device=dev)
+        N_out = W.shape[0]
+        t = torch.tensor(t_np, device=dev)
+        p = dstd.params(L, 1.0 / B)
+        ws = torch.empty(dstd.dense_workspace_bytes(B, N_in, N_out, p, "x3"), dtype=torch.uint8, device=dev)
+        wse = torch.empty(dstd.exact_workspace_bytes(B, N_in, N_out), dtype=torch.uint8, device=dev)
+        t_d = torch.empty(B, N_out, device=dev)
+        t_e = torch.empty(B, N_out, device=dev)
+        saved = torch.empty(dstd.dense_saved_bytes(B, N_out), dtype=torch.uint8, device=dev)
+        pen = torch.empty(4, device=dev)
+        runs = {"dstd": lambda: dstd.dense_fwd(t, W, p, "x3", t_d, saved, pen, ws, stream),
+                "exact": lambda: dstd.exact_fwd(t, W, p, t_e, wse, stream)}
+        ms = {}
+        with torch.cuda.stream(stream):
+            for k, fn in runs.items():
+                for _ in range(max(3, args.warmup)):
+                    fn()
+                ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+                for a, b in ev:
+                    flush.zero_()
+                    a.record(stream)
+                    fn()
+                    b.record(stream)
+                stream.synchronize()
+                ms[k] = float(np.median([a.elapsed_time(b) for a, b in ev]))
+        td, te = t_d.cpu().numpy(), t_e.cpu().numpy()
+        both = np.isfinite(td) & np.isfinite(te)
+        out.append({"layer": name, "B": B, "N_in": N_in, "N_out": N_out, "M": L["M"],
+                    "dstd_fwd_ms": ms["dstd"], "exact_fwd_ms": ms["exact"], "exact_over_dstd": ms["exact"] / ms["dstd"],
+                    "fire_dstd": float(np.isfinite(td).mean()), "fire_exact": float(np.isfinite(te).mean()),
+                    "median_abs_dt_fired_both": float(np.median(np.abs(td[both] - te[both]))) if both.any() else None})
+    status = dstd.device_status(clear=True)
+    print(json.dumps({"metric": "exact (event-driven) forward time / DSTD forward time, one GB300", "unit": "ratio",
+                      "higher_is_better": True, "cases": out, "reps": reps, "device_status": status,
+                      "note": "forward only (the GPU exact method has no backward); DSTD in the x3 mode; median of "
+                              "the per-rep CUDA-event times, L2 flushed before each"}), flush=True)
+    return 0 if status == 0 else 1
+
+
 def main():
     args = parse()
     rank, world, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank)
+    if args.exact:
+        return run_exact_compare(args, local) if rank == 0 else 0
     return run_ours(args, rank, world, local)
 
 

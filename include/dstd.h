@@ -238,6 +238,22 @@ int dstd_adamw_multi(int count, float *const *w, const float *const *g, float *c
                      float eps, float weight_decay, int32_t *step, const float *lr_dev,
                      dstd_stream_t stream);
 
+/* The exact (event-driven) first-spike times of one dense layer, Alg. 1 /
+ * Eq. timing_exact: the method DSTD replaces, on the same GPU, for timing
+ * and accuracy comparisons. Per sample the finite input spike times before
+ * p->t_end are sorted; the potential sum_{j<=k} w_ij K(t - t~_j) is walked
+ * interval by interval and the first interval that reaches p->v_th holds
+ * the spike. Spike times are exact up to fp32 (no grid); a neuron that does
+ * not fire before p->t_end gets +inf. Only tau_m, tau_s, v_th and t_end of p
+ * are used (t_first, M only for the root's tolerance). No gradient.
+ *  t_in [B, N_in] (+inf = silent), W [N_out, N_in] fp32, t_out [B, N_out] out;
+ *  workspace of dstd_exact_workspace_bytes (16-byte aligned).
+ * N_in up to 8192 (DSTD_E_UNSUPPORTED beyond). */
+size_t dstd_exact_workspace_bytes(int B, int N_in, int N_out);
+int dstd_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out,
+                   const dstd_params *p, float *t_out, void *workspace, size_t ws_bytes,
+                   dstd_stream_t stream);
+
 /* How the forward contraction of a wide dense layer is scheduled: on single
  * CTAs (128 x 128 tiles) or on SM pairs (tcgen05 cta_group::2, 256 x 128
  * tiles, half of B per SM). policy 0 (the default) lets a cost model choose

@@ -89,12 +89,12 @@ inline int cu(cudaError_t e) { return e == cudaSuccess ? DSTD_OK : DSTD_E_CUDA; 
 // ---------------------------------------------------------------------------
 enum Kind {
     KK_PREP = 0, KK_BIN, KK_BIN_T, KK_GEMM_FWD, KK_SCAN, KK_DWHAT, KK_GEMM_DS, KK_GT, KK_GEMM_DW, KK_REDUCE,
-    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_NARROW_FWD, KK_NARROW_BWD, KK_COUNT
+    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_NARROW_FWD, KK_NARROW_BWD, KK_EXACT_FWD, KK_COUNT
 };
 const char *const kKindNames[KK_COUNT] = {
     "prep_weights", "binning", "binning_T", "gemm_fwd_scan", "scan_solve", "dwhat", "gemm_dS_gradt",
     "gradt_gather", "gemm_dW", "dw_reduce", "loss", "adamw", "binning_public", "what_public", "selftest", "narrow_fwd",
-    "narrow_bwd"};
+    "narrow_bwd", "exact_fwd"};
 
 struct Timing {
     std::mutex mu;
@@ -354,6 +354,31 @@ BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool
     }
     w.bytes = b.off;
     return w;
+}
+
+ExactWs exact_layout(void *base, int B, int N_in, int N_out) {
+    ExactWs w;
+    Bump bp(base);
+    w.Wt = bp.take<float>((size_t)N_in * N_out);
+    w.perm = bp.take<int>((size_t)B * N_in);
+    w.t_start = bp.take<float>((size_t)B * N_in);
+    w.iv = bp.take<float4>((size_t)B * N_in);
+    w.count = bp.take<int>((size_t)B);
+    w.bytes = bp.off;
+    return w;
+}
+
+// sup over s >= 0 of K(s) = e^{-av s} phi(s) (+inf when both rates are 0)
+double kernel_sup(double av, double aI) {
+    if (av > 0.0 && aI > 0.0) {
+        const double lam = aI - av;
+        const double tp = lam == 0.0 ? 1.0 / av : log(aI / av) / lam;
+        const double ph = lam == 0.0 ? tp : -expm1(-lam * tp) / lam;
+        return exp(-av * tp) * ph;
+    }
+    if (av > 0.0) return 1.0 / av;
+    if (aI > 0.0) return 1.0 / aI;
+    return INFINITY;
 }
 
 struct Saved {
@@ -1029,6 +1054,27 @@ int dstd_timing_enable(int on) {
     }
     g_timing.on = on != 0;
     return DSTD_OK;
+}
+
+size_t dstd_exact_workspace_bytes(int B, int N_in, int N_out) {
+    if (check_sizes(B, N_in, N_out) != DSTD_OK || N_in > kExactMaxIn) return 0;
+    return exact_layout(nullptr, B, N_in, N_out).bytes;
+}
+
+int dstd_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p, float *t_out,
+                   void *workspace, size_t ws_bytes, dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    if (N_in > kExactMaxIn) return DSTD_E_UNSUPPORTED;
+    if (!aligned16(workspace)) return DSTD_E_INVALID;
+    if (ws_bytes < exact_layout(nullptr, B, N_in, N_out).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, padded_M(p->M));
+    const double kmax = kernel_sup(c.av, c.aI) * (1.0 + 1e-6);
+    ExactWs ws = exact_layout(workspace, B, N_in, N_out);
+    Timed tm(KK_EXACT_FWD, (cudaStream_t)stream);
+    return cu(launch_exact_fwd(t_in, W, B, N_in, N_out, c, p->t_end, (float)kmax, ws, t_out, (cudaStream_t)stream));
 }
 
 int dstd_set_pair_policy(int policy) {

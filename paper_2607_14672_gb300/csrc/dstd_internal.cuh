@@ -323,6 +323,20 @@ cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const
 // from W, dw^ (operand layout [N_out, ld] over (b, m), hi/lo or hi only) and
 // the per-input bin index / kernel derivatives bw.
 constexpr int kGradtSmallMaxOut = 32;
+// The exact (event-driven) forward, Alg. 1, for comparison with DSTD: W^T,
+// the sorted inputs and their intervals in the workspace (exact_layout).
+constexpr int kExactMaxIn = 8192;  // a sample's inputs are sorted in shared memory
+struct ExactWs {
+    float *Wt = nullptr;       // [N_in][N_out]
+    int *perm = nullptr;       // [B][N_in]: input of the k-th interval
+    float *t_start = nullptr;  // [B][N_in]: its start
+    float4 *iv = nullptr;      // [B][N_in]: e^{-av L}, e^{-aI L}, K(L), L
+    int *count = nullptr;      // [B]: intervals (finite inputs before the window end)
+    size_t bytes = 0;
+};
+cudaError_t launch_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out, const LifConst &c,
+                             float t_end, float kmax, const ExactWs &ws, float *t_out, cudaStream_t st);
+
 // Layers with at most kNarrowMaxOut outputs run forward and backward on CUDA
 // cores in fp32 (sparse over the two grid points of each input spike).
 constexpr int kNarrowMaxOut = 32;

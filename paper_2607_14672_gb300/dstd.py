@@ -22,7 +22,8 @@ EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning
            "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_fwd_ce", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
-           "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd")
+           "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd",
+           "dstd_exact_workspace_bytes", "dstd_exact_fwd")
 
 
 class DstdError(RuntimeError):
@@ -87,6 +88,8 @@ def load(path=None):
         "dstd_timing_read": (_I, [_I, ctypes.POINTER(_F), ctypes.POINTER(_I64)]),
         "dstd_timing_collect": (_I, []),
         "dstd_set_pair_policy": (_I, [_I]),
+        "dstd_exact_workspace_bytes": (_SZ, [_I, _I, _I]),
+        "dstd_exact_fwd": (_I, [_P, _P, _I, _I, _I, _PP, _P, _P, _SZ, _P]),
         "dstd_kernel_kind_count": (_I, []),
         "dstd_kernel_kind_name": (ctypes.c_char_p, [_I]),
         "dstd_selftest_wait_timeout": (_I, [ctypes.c_uint32, _P]),
@@ -313,6 +316,21 @@ def device_status(clear=True):
 def timing_enable(on=True):
     """Turn per-kernel event timing on/off (clears the counters)."""
     _check(load().dstd_timing_enable(1 if on else 0), "dstd_timing_enable")
+
+
+def exact_workspace_bytes(B, N_in, N_out):
+    return load().dstd_exact_workspace_bytes(B, N_in, N_out)
+
+
+def exact_fwd(t_in, W, p, t_out, workspace, stream=None):
+    """Exact (event-driven, Alg. 1) first-spike times of a dense layer."""
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(t_out, "t_out", (B, N_out))
+    _check(load().dstd_exact_fwd(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), _ptr(t_out), _ptr(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_exact_fwd")
 
 
 def set_pair_policy(policy):
