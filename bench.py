@@ -41,6 +41,9 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg4", "cfg5"],
+                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg4 / cfg5: the 9- and 20-layer conv "
+                         "networks (bf16 operands), their training step timed the same way")
     ap.add_argument("--exact", action="store_true",
                     help="instead of the training step: time the exact (event-driven, Alg. 1) forward against the "
                          "DSTD forward on the same GPU, per layer shape, and print one JSON line")
@@ -478,6 +481,106 @@ def run_ours(args, rank, world, local):
     return 0
 
 
+# dense-equivalent tensor flops of one training step of a conv network: the
+# forward contraction of every layer at the padded tile shape, and twice that
+# for the backward (dS and dW), one pass in bf16
+def conv_step_dense_flops(net):
+    tot = 0.0
+    for l, L in enumerate(net.layers):
+        Mp = max(8, 1 << (L["M"] - 1).bit_length())
+        if net.geom[l] is not None:
+            H, W, C, k, st, pad = net.geom[l]
+            Ho, Wo = (H + 2 * pad - k) // st + 1, (W + 2 * pad - k) // st + 1
+            rows, K, n = net.B * Ho * Wo * Mp, k * k * C, net.W[l].shape[0]
+        else:
+            rows, K, n = net.B * Mp, net.W[l].shape[1], net.W[l].shape[0]
+        f = 2.0 * rows * K * n
+        tot += f if l == 0 else 3.0 * f    # layer 1 has no dS
+        if l == 0:
+            tot += f                        # its dW
+    return tot
+
+
+def run_conv(args, local):
+    """Training step (forward, CE loss, backward, AdamW) of the conv network
+    of config 4 or 5, captured in a CUDA graph and replayed K times, L2
+    flushed before each, CUDA events on the stream; per-kind kernel times
+    from a second capture with event nodes."""
+    import numpy as np
+    import torch
+
+    from paper_2607_14672_gb300 import build as _b
+    _b.build()
+    from paper_2607_14672_gb300 import configs, dstd, net
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg = configs.config4() if args.workload == "cfg4" else configs.config5()
+    cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
+    n = net.ConvNet(cfg, device=dev, with_adamw=True)
+    n.set_inputs(np.asarray(cfg["inputs"](), np.float32), cfg["labels"]().astype(np.int32))
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup)):
+            n.step()
+        stream.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            n.step()
+        for _ in range(args.warmup):
+            graph.replay()
+        stream.synchronize()
+    steps = max(2, min(args.steps, 20))
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for a, b in ev:
+            flush.zero_()
+            a.record(stream)
+            graph.replay()
+            b.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    dstd.timing_enable(True)
+    with torch.cuda.stream(stream):
+        gt = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gt, stream=stream):
+            n.step()
+        gt.replay()
+        stream.synchronize()
+        for _ in range(2):
+            flush.zero_()
+            gt.replay()
+            dstd.timing_collect()
+    kt = dstd.timing_read()
+    dstd.timing_enable(False)
+    status = dstd.device_status(clear=True)
+    pk, pk_src = peaks()
+    flops = conv_step_dense_flops(n)
+    dead = [float(x) for x in n.dead_fraction()]
+    B = cfg["batch"]
+    print(json.dumps({
+        "metric": "DSTD conv SNN training step samples/s at 1 GB300", "value": B / (ms / 1000.0),
+        "unit": "samples/s", "n_gpus": 1, "steps": steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "dtype": "bf16 operands, fp32 accumulation and state",
+        "data": "synthetic (seeded intensity maps; random-init weights)",
+        "config": {"workload": cfg["workload"], "global_batch": B, "layers": len(n.layers),
+                   "l2": "flushed (512 MB write) before each timed step"},
+        "tensor": {"dense_flops_per_step": flops, "achieved_tflops": flops / (ms / 1000.0) / 1e12,
+                   "peak": pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
+                   "frac": flops / (ms / 1000.0) / 1e12 / pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
+                   "peak_source": f"{pk_src} bf16 (burst)",
+                   "note": "whole step: every kernel's time in the denominator, the contractions' padded dense "
+                           "flops in the numerator"},
+        "kernel_ms": {k: round(v[0] / 2, 4) for k, v in kt.items() if v[1] > 0},
+        "dead_fraction_per_layer": dead, "clocks": clk, "device_status": status}), flush=True)
+    return 0 if status == 0 else 1
+
+
 def run_exact_compare(args, local):
     """Exact forward (sort + interval sweep, Alg. 1) against the DSTD forward
     (binning, contraction, scan/solve) of the same layers on one GPU: device
@@ -551,6 +654,8 @@ def main():
         return run_reference(args, rank)
     if args.exact:
         return run_exact_compare(args, local) if rank == 0 else 0
+    if args.workload != "cfg2":
+        return run_conv(args, local) if rank == 0 else 0
     return run_ours(args, rank, world, local)
 
 

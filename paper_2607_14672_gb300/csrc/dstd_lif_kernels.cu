@@ -591,9 +591,111 @@ __global__ void k_binning_im2col_cols(const float *__restrict__ t, ConvGeom g, i
     }
 }
 
+// Sparse writers of the im2col operands (as the dense ones): a block zero-
+// fills the Mp rows of one output position over 256 tap columns, or a warp
+// the Mp bins of 32 consecutive positions of one tap, with 16-byte stores,
+// synchronises, and each thread then stores the two weights of its own
+// (position, tap).
+template <int OP>
+__global__ void __launch_bounds__(256) k_binning_im2col_rows8(const float *__restrict__ t, ConvGeom g, int pos0,
+                                                              int npos, LifConst c, uint16_t *hi, uint16_t *lo,
+                                                              int ld) {
+    const int K = g.k * g.k * g.C;
+    const int col0 = blockIdx.x * 256;
+    const int nch = ((ld - col0) < 256 ? (ld - col0) : 256) / 8;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    for (int pl = blockIdx.y; pl < npos; pl += gridDim.y) {
+        const long long base = (long long)pl * c.Mp * ld + col0;
+        for (int idx = threadIdx.x; idx < c.Mp * nch; idx += 256) {
+            const int m = idx / nch, cc = idx - m * nch;
+            const long long o = base + (long long)m * ld + 8 * cc;
+            *reinterpret_cast<uint4 *>(hi + o) = z;
+            if (OP != 2) *reinterpret_cast<uint4 *>(lo + o) = z;
+        }
+        __syncthreads();
+        const int kidx = col0 + threadIdx.x;
+        if (kidx < K) {
+            const float x = im2col_time(t, g, pos0 + pl, kidx);
+            if (isfinite(x)) {
+                const BinW w = bin_weights(c, x, false);
+                uint16_t h, l;
+                if (w.k >= 0 && w.k < c.M) {
+                    split16<OP>(w.wR, h, l);
+                    const long long o = base + (long long)w.k * ld + threadIdx.x;
+                    hi[o] = h;
+                    if (OP != 2) lo[o] = l;
+                }
+                if (w.k + 1 >= 0 && w.k + 1 < c.M) {
+                    split16<OP>(w.wL, h, l);
+                    const long long o = base + (long long)(w.k + 1) * ld + threadIdx.x;
+                    hi[o] = h;
+                    if (OP != 2) lo[o] = l;
+                }
+            }
+        }
+        __syncthreads();  // the next position's zero fill may touch no column before this one's weights are out
+    }
+}
+
+template <int OP>
+__global__ void __launch_bounds__(128) k_binning_im2col_cols8(const float *__restrict__ t, ConvGeom g, int pos0,
+                                                              int npos, LifConst c, uint16_t *hi, uint16_t *lo,
+                                                              int ld) {
+    const int K = g.k * g.k * g.C;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int p0 = (blockIdx.x * 4 + warp) * 32;
+    if (p0 >= npos) return;
+    const int ns = (npos - p0) < 32 ? (npos - p0) : 32;
+    const int nch = ns * c.Mp / 8;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    for (int kidx = blockIdx.y; kidx < K; kidx += gridDim.y) {
+        const long long rowbase = (long long)kidx * ld + (long long)p0 * c.Mp;
+        for (int gq = lane; gq < nch; gq += 32) {
+            *reinterpret_cast<uint4 *>(hi + rowbase + 8 * gq) = z;
+            if (OP != 2) *reinterpret_cast<uint4 *>(lo + rowbase + 8 * gq) = z;
+        }
+        __syncwarp();
+        if (lane < ns) {
+            const float x = im2col_time(t, g, pos0 + p0 + lane, kidx);
+            if (isfinite(x)) {
+                const BinW w = bin_weights(c, x, false);
+                const long long o = rowbase + (long long)lane * c.Mp;
+                uint16_t h, l;
+                if (w.k >= 0 && w.k < c.M) {
+                    split16<OP>(w.wR, h, l);
+                    hi[o + w.k] = h;
+                    if (OP != 2) lo[o + w.k] = l;
+                }
+                if (w.k + 1 >= 0 && w.k + 1 < c.M) {
+                    split16<OP>(w.wL, h, l);
+                    hi[o + w.k + 1] = h;
+                    if (OP != 2) lo[o + w.k + 1] = l;
+                }
+            }
+        }
+        __syncwarp();
+    }
+}
+
 cudaError_t launch_binning_im2col(const float *t, const ConvGeom &g, int pos0, int npos, const LifConst &c,
                                   OpKind op, bool transposed, void *hi, void *lo, int ld, cudaStream_t st) {
     const int K = g.k * g.k * g.C;
+    uint16_t *h16 = static_cast<uint16_t *>(hi), *l16 = static_cast<uint16_t *>(lo);
+    const bool sparse = (ld % 8) == 0 && ((reinterpret_cast<uintptr_t>(hi) | reinterpret_cast<uintptr_t>(lo)) & 15) == 0;
+    if (sparse && !transposed) {
+        dim3 grid((ld + 255) / 256, npos < 65535 ? npos : 65535);
+        if (op == OpKind::F16X3) k_binning_im2col_rows8<3><<<grid, 256, 0, st>>>(t, g, pos0, npos, c, h16, l16, ld);
+        else if (op == OpKind::BF16X3) k_binning_im2col_rows8<1><<<grid, 256, 0, st>>>(t, g, pos0, npos, c, h16, l16, ld);
+        else if (op == OpKind::BF16) k_binning_im2col_rows8<2><<<grid, 256, 0, st>>>(t, g, pos0, npos, c, h16, l16, ld);
+        else return cudaErrorInvalidValue;
+        return cudaGetLastError();
+    }
+    if (sparse && transposed && (op == OpKind::BF16X3 || op == OpKind::BF16)) {
+        dim3 grid((npos + 127) / 128, K < 65535 ? K : 65535);
+        if (op == OpKind::BF16X3) k_binning_im2col_cols8<1><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, h16, l16, ld);
+        else k_binning_im2col_cols8<2><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, h16, l16, ld);
+        return cudaGetLastError();
+    }
     if (!transposed) {
         dim3 grid(blocks_for((ld + 1) / 2, 128), npos < 65535 ? npos : 65535);
         if (op == OpKind::F16X3) k_binning_im2col_rows<3><<<grid, 128, 0, st>>>(t, g, pos0, npos, c, hi, lo, ld);
