@@ -41,8 +41,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg4", "cfg5"],
-                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg4 / cfg5: the 9- and 20-layer conv "
+    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5"],
+                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; cfg4 / cfg5: the 9- and 20-layer conv "
                          "networks (bf16 operands), their training step timed the same way")
     ap.add_argument("--exact", action="store_true",
                     help="instead of the training step: time the exact (event-driven, Alg. 1) forward against the "
@@ -233,17 +233,17 @@ TRAFFIC_PER_LAUNCH = {
     ("gemm_dS_gradt", "x3"): 32.2e6,
     ("scan_solve", "x3"): 26.3e6,
     ("dwhat", "x3"): 3.9e6,
-    ("binning", "x3"): None,            # now also splits the weights: not re-captured yet
+    ("binning", "x3"): 3.37e6,          # k_fwd_operands_f16: binning + the hi/lo split of W
     ("binning_T", "x3"): 0.82e6,
-    ("prep_weights", "x3"): None,       # only the backward's W^T split now: not re-captured yet
+    ("prep_weights", "x3"): 2.57e6,     # the backward's W^T split
     ("loss", "x3"): 0.04e6,
     ("adamw", "x3"): 20.4e6,
-    ("narrow_fwd", "x3"): 0.92e6,
+    ("narrow_fwd", "x3"): 0.93e6,
     ("narrow_bwd", "x3"): 0.97e6,
 }
 
 
-def kind_rooflines(per_kind, sizes, B, M, Mp, npass, math_mode, pk, pk_src):
+def kind_rooflines(per_kind, sizes, B, M, Mp, npass, math_mode, pk, pk_src, first_input_grad=False):
     """Achieved vs peak for each kernel kind of the step.
 
     Contractions are tensor-bound: achieved = the method's flops (2 grid
@@ -279,7 +279,8 @@ def kind_rooflines(per_kind, sizes, B, M, Mp, npass, math_mode, pk, pk_src):
         # forward operands: in x3 the weight split rides in the binning launch
         add(algo_b, "binning" if math_mode == "x3" else "prep_weights", no * ni * 4 + no * pad8(ni) * e)
         add(algo_b, "binning", B * ni * 4 + cols * pad8(ni) * e)
-        if l > 0:
+        in_grad = l > 0 or first_input_grad
+        if in_grad:
             add(algo_b, "prep_weights", no * ni * 4 + ni * pad8(no) * e)   # W^T split for dS
         add(algo_b, "scan_solve", B * no * Mp * 4 + B * no * 16)
         add(algo_b, "dwhat", B * no * 20 + 2 * B * no * Mp * e)
@@ -292,7 +293,7 @@ def kind_rooflines(per_kind, sizes, B, M, Mp, npass, math_mode, pk, pk_src):
         add(dense_f, "gemm_fwd_scan", 2 * npass * r_out * cols * k_in)
         add(algo_f, "gemm_dW", 4 * B * ni * no)
         add(dense_f, "gemm_dW", 2 * npass * r_out * r_in * cols)
-        if l > 0:
+        if in_grad:
             add(algo_f, "gemm_dS_gradt", 4 * B * ni * no)
             add(dense_f, "gemm_dS_gradt", 2 * npass * r_in * cols * k_out)
     out = {}
@@ -581,6 +582,101 @@ def run_conv(args, local):
     return 0 if status == 0 else 1
 
 
+def run_cfg3(args, local):
+    """One dense N -> N layer (config 3: B = 128, tau = (0.4, 0.2), inputs
+    U[0, 1) with 10% silent): forward, sum-of-times loss and backward with the
+    input-time gradient, for several (N, M) and math modes. Each case is
+    captured in a CUDA graph and replayed, L2 flushed before each replay;
+    per-kind kernel times from a second capture with event nodes, and the
+    roofline of each kind at these sizes (operands of 0.1-1 GB, where the
+    memory-bound kernels are no longer latency-bound)."""
+    import numpy as np
+    import torch
+
+    from paper_2607_14672_gb300 import build as _b
+    _b.build()
+    from paper_2607_14672_gb300 import configs, dstd, net
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    pk, pk_src = peaks()
+    cases = [(4096, 32, "x3"), (16384, 32, "x3"), (16384, 128, "x3"), (16384, 128, "bf16")]
+    steps = max(2, min(args.steps, 20))
+    clocks = ClockSampler(local)
+    clocks.start()
+    out = []
+    for N, M, math_mode in cases:
+        cfg = configs.config3(N, M)
+        B = cfg["batch"]
+        n = net.DenseNet(cfg, math_mode, device=dev)
+        n.set_inputs(np.asarray(cfg["inputs"](), np.float32))
+        g_in = torch.empty(B, N, dtype=torch.float32, device=dev)
+
+        def step():
+            dstd.dense_fwd(n.t_in, n.W[0], n.p[0], math_mode, n.t[0], n.saved[0], n.penalty[0], n.workspace, None)
+            dstd.sum_t_loss(n.t[0], n.loss, n.g[0], None)
+            dstd.dense_bwd(n.t_in, n.W[0], n.t[0], n.saved[0], n.g[0], n.p[0], math_mode, g_in, n.gW[0],
+                           n.workspace, None)
+
+        with torch.cuda.stream(stream):
+            for _ in range(max(1, args.warmup)):
+                step()
+            stream.synchronize()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                step()
+            for _ in range(args.warmup):
+                graph.replay()
+            stream.synchronize()
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+            for a, b in ev:
+                flush.zero_()
+                a.record(stream)
+                graph.replay()
+                b.record(stream)
+            stream.synchronize()
+        ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+        dstd.timing_enable(True)
+        with torch.cuda.stream(stream):
+            gt = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gt, stream=stream):
+                step()
+            gt.replay()
+            stream.synchronize()
+            for _ in range(3):
+                flush.zero_()
+                gt.replay()
+                dstd.timing_collect()
+        kt = dstd.timing_read()
+        dstd.timing_enable(False)
+        per_kind = {k: (v[0] / v[1], v[1] // 3) for k, v in kt.items() if v[1] > 0}
+        Mp = max(8, 1 << (M - 1).bit_length())
+        npass = {"x3": 3, "bf16": 1}[math_mode]
+        roofs = kind_rooflines(per_kind, [N, N], B, M, Mp, npass, math_mode, pk, pk_src, first_input_grad=True)
+        keep = ("bound", "achieved", "unit", "frac", "dense_achieved", "dense_frac", "launch_us")
+        out.append({"N": N, "M": M, "math": math_mode, "B": B, "ms_per_step": ms, "samples_per_s": B / (ms / 1e3),
+                    "fired": float(torch.isfinite(n.t[0]).float().mean()),
+                    "kernel_ms": {k: round(v[0], 5) for k, v in per_kind.items()},
+                    "rooflines": {k: {f: (round(r[f], 4) if isinstance(r[f], float) else r[f])
+                                      for f in keep if f in r} for k, r in roofs.items()}})
+        del n, g_in, graph, gt
+        torch.cuda.empty_cache()
+    clk = clocks.stop()
+    status = dstd.device_status(clear=True)
+    print(json.dumps({
+        "metric": "DSTD single dense layer fwd+bwd samples/s at 1 GB300, per-kernel roofline",
+        "unit": "samples/s", "higher_is_better": True, "steps": steps, "warmup": args.warmup,
+        "data": "synthetic (seeded U[0,1) spike times, 10% silent; W = mu + N(0, 1/N))",
+        "config": {"workload": "dense LIF layer N->N, B=128, tau=(0.4,0.2), sum-of-times loss, "
+                               "fwd+bwd incl. the input-time gradient",
+                   "l2": "flushed (512 MB write) before each timed step"},
+        "peaks": {"hbm_gbs": pk.get("hbm_gbs"), "bf16_tflops": pk.get("bf16_tflops"), "source": pk_src},
+        "cases": out, "clocks": clk, "device_status": status}), flush=True)
+    return 0 if status == 0 else 1
+
+
 def run_exact_compare(args, local):
     """Exact forward (sort + interval sweep, Alg. 1) against the DSTD forward
     (binning, contraction, scan/solve) of the same layers on one GPU: device
@@ -654,6 +750,8 @@ def main():
         return run_reference(args, rank)
     if args.exact:
         return run_exact_compare(args, local) if rank == 0 else 0
+    if args.workload == "cfg3":
+        return run_cfg3(args, local) if rank == 0 else 0
     if args.workload != "cfg2":
         return run_conv(args, local) if rank == 0 else 0
     return run_ours(args, rank, world, local)
