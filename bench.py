@@ -41,8 +41,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5"],
-                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; cfg4 / cfg5: the 9- and 20-layer conv "
+    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5", "syn9", "syn20"],
+                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; syn9 / syn20: the paper's Syn-SNN-9 and Syn-SNN-20 (N = 64, batch 50, M = 20); cfg4 / cfg5: the 9- and 20-layer conv "
                          "networks (bf16 operands), their training step timed the same way")
     ap.add_argument("--exact", action="store_true",
                     help="instead of the training step: time the exact (event-driven, Alg. 1) forward against the "
@@ -283,7 +283,8 @@ def kind_rooflines(per_kind, sizes, B, M, Mp, npass, math_mode, pk, pk_src, firs
         if in_grad:
             add(algo_b, "prep_weights", no * ni * 4 + ni * pad8(no) * e)   # W^T split for dS
         add(algo_b, "scan_solve", B * no * Mp * 4 + B * no * 16)
-        add(algo_b, "dwhat", B * no * 20 + 2 * B * no * Mp * e)
+        # dw^ in the (i, (b, m)) layout; the fp32 mode also writes the ((b, m), i) copy
+        add(algo_b, "dwhat", B * no * 20 + (2 if math_mode == "f32" else 1) * B * no * Mp * e)
         add(algo_b, "binning_T", B * ni * 4 + ni * cols * e)
         add(algo_b, "dw_reduce", 3 * no * ni * 4 + no * ni * 4)
         add(algo_b, "adamw", 7 * no * ni * 4)              # read w, g, m, v; write w, m, v
@@ -503,10 +504,10 @@ def conv_step_dense_flops(net):
 
 
 def run_conv(args, local):
-    """Training step (forward, CE loss, backward, AdamW) of the conv network
-    of config 4 or 5, captured in a CUDA graph and replayed K times, L2
-    flushed before each, CUDA events on the stream; per-kind kernel times
-    from a second capture with event nodes."""
+    """Training step (forward, CE loss, backward, AdamW) of a conv network
+    (config 4 or 5, or the paper's Syn-SNN-9 / Syn-SNN-20), captured in a
+    CUDA graph and replayed K times, L2 flushed before each, CUDA events on
+    the stream; per-kind kernel times from a second capture with event nodes."""
     import numpy as np
     import torch
 
@@ -516,7 +517,8 @@ def run_conv(args, local):
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    cfg = configs.config4() if args.workload == "cfg4" else configs.config5()
+    cfg = {"cfg4": configs.config4, "cfg5": configs.config5, "syn9": configs.syn_snn9,
+           "syn20": configs.syn_snn20}[args.workload]()
     cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
     n = net.ConvNet(cfg, device=dev, with_adamw=True)
     n.set_inputs(np.asarray(cfg["inputs"](), np.float32), cfg["labels"]().astype(np.int32))

@@ -203,6 +203,25 @@ int dstd_dense_fwd_ce(const float *t_in, const float *W, int B, int N_in, int N_
                       float tau_soft, float t_silent, float *loss, float *g_t_out,
                       dstd_stream_t stream);
 
+/* Skip-and-delay input of the paper's 20-layer network (App. C.3, Fig.
+ * skip_connection: the third layer of a block also receives the block's input,
+ * delayed by 2 tau_shift). Spike tensors are NHWC, so this is a concatenation
+ * along channels at each of `positions` = B*H*W positions:
+ *   out[p, 0:C_a]       = a[p, :] + delay_a   (+inf stays +inf)
+ *   out[p, C_a:C_a+C_b] = b[p, :]
+ *  a [positions, C_a], b [positions, C_b], out [positions, C_a + C_b]: device
+ *  fp32, caller-owned, out not overlapping a or b. DSTD_E_INVALID for null
+ *  pointers, non-positive sizes or a non-finite delay. */
+int dstd_concat_channels(const float *a, int C_a, float delay_a, const float *b, int C_b, int64_t positions,
+                         float *out, dstd_stream_t stream);
+/* Adjoint of dstd_concat_channels (the delay has unit derivative): from
+ * g [positions, C_a + C_b], writes g_a [positions, C_a] and g_b
+ * [positions, C_b]; either may be NULL (not both). With accumulate_x != 0
+ * the part is added into g_x instead of overwriting it (the block input's
+ * gradient also receives the block's first layer's). */
+int dstd_split_channels(const float *g, int C_a, int C_b, int64_t positions, float *g_a, int accumulate_a,
+                        float *g_b, int accumulate_b, dstd_stream_t stream);
+
 /* Cross-entropy over softmax(-t/tau_soft) (Eqs. cost_function, L, S_i),
  * mini-batch mean; a silent output enters with the constant time t_silent
  * and passes no gradient.
@@ -266,7 +285,10 @@ int dstd_set_pair_policy(int policy);
 
 /* Kernel timing (tracing). While enabled, the library brackets every kernel
  * it launches with a CUDA event pair on the launching stream and files the
- * pair under the kernel's kind (dstd_kernel_kind_name).
+ * pair under the kernel's kind (dstd_kernel_kind_name). Kernels that
+ * otherwise run beside each other on the library's side streams (the layer
+ * backward's operand producers) then run one after another on the caller's
+ * stream, so that each kind's time is that kernel's alone.
  * dstd_timing_enable(on) turns timing on/off and clears the counters.
  * dstd_timing_read(kind, total_ms, launches) synchronises the device and
  * returns the accumulated device time and launch count of one kind. */

@@ -4,9 +4,9 @@ Finds, by bisection with the float64 oracle, the weight mean mu_l for which
 80% of layer l's neurons fire at initialisation on the seed-0 input batch
 (t_offset = 0); layer l sees the previous layer's calibrated output. Prints
 the values that the workload definitions freeze (CFG2_MU, CFG3_MU_TIMES_N,
-CFG4_MU, CFG5_MU). Calls only the oracle and the seeded generators.
+CFG4_MU, CFG5_MU, SYN9_MU, SYN20_MU). Calls only the oracle and the seeded generators.
 
-    python -m oracle.calibrate_configs [2] [3] [4] [5]
+    python -m oracle.calibrate_configs [2] [3] [4] [5] [syn9] [syn20]
 """
 
 import math
@@ -80,15 +80,20 @@ def calibrate_conv(cfg, batch, verbose=True):
     """mu_l for a conv stack (configs 4, 5): w^(mu) = w^(Z) + mu w^(ones) by
     linearity of the contraction, so each bisection step only re-evaluates
     the interval maxima; the chosen mu's spike times feed the next layer."""
-    t = cfg["inputs"](B=batch)
-    mus = []
+    t0 = cfg["inputs"](B=batch)
+    t = t0
+    mus, outs = [], []
     for l, L in enumerate(cfg["layers"], start=1):
         T, dt = dstd.grid(L["t_first"], L["t_end"], L["M"], 0.0)
         tv, ti = L["tau_v"], L["tau_I"]
         B = t.shape[0]
+        if L.get("skip") is not None:     # skip-and-delay input: delayed source first along channels
+            src, delay = L["skip"]
+            t = np.concatenate([(t0 if src < 0 else outs[src]) + delay, t], axis=1)
         if L["kind"] == "conv":
             C, H, Wd = t.shape[1:]
-            Z = synth.normal_weights(1000 + l, L["W"].shape, 0.0, 1.0 / math.sqrt(C * 9))
+            k = L["W"].shape[2]
+            Z = synth.normal_weights(1000 + l, L["W"].shape, 0.0, 1.0 / math.sqrt(C * k * k))
             s = dstd.binning(t.reshape(B, -1), T, dt, tv, ti).reshape(B, L["M"], C, H, Wd)
             A = network.conv_what(s, Z, L["stride"], L["pad"])
             U = network.conv_what(s, np.ones((1,) + Z.shape[1:]), L["stride"], L["pad"])
@@ -105,6 +110,7 @@ def calibrate_conv(cfg, batch, verbose=True):
         mus.append(mu)
         ctx = dstd.solve(A + mu * Ur, T, dt, tv, ti, 1.0)
         t = ctx["t"].reshape((B,) + tuple(shape[1:4])) if L["kind"] == "conv" else ctx["t"]
+        outs.append(t)
         if verbose:
             print(f"layer {l}: mu {mu:.5f}, fired {np.isfinite(ctx['t']).mean():.3f}", flush=True)
     return mus
@@ -122,3 +128,7 @@ if __name__ == "__main__":
         print("CFG4_MU", tuple(round(m, 5) for m in calibrate_conv(configs.config4(), batch=2)))
     if "5" in which:
         print("CFG5_MU", tuple(round(m, 5) for m in calibrate_conv(configs.config5(), batch=1)))
+    if "syn9" in which:
+        print("SYN9_MU", tuple(round(m, 5) for m in calibrate_conv(configs.syn_snn9(mus=(0.0,) * 9), batch=2)))
+    if "syn20" in which:
+        print("SYN20_MU", tuple(round(m, 5) for m in calibrate_conv(configs.syn_snn20(mus=(0.0,) * 20), batch=2)))

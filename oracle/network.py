@@ -14,7 +14,11 @@ the dead-neuron term to dC/dW.
 
 Layer spec (dict): kind ("dense" | "conv"), W, tau_v, tau_I, v_th, t_first,
 t_end, M, t_offset, and for conv stride, pad; penalty constants t_head_l,
-t_tail_l, gamma_head, gamma_tail, gamma_q (missing = 0).
+t_tail_l, gamma_head, gamma_tail, gamma_q (missing = 0); optionally
+skip = (src, delay): the skip-and-delay input of App. C.3 (Fig.
+skip_connection), where the layer sees, along channels, the output of layer
+src (-1 = the network input) delayed by `delay`, followed by the previous
+layer's output.
 Spike tensors: dense [B, N]; conv [B, C, H, W] (channel-major). A dense
 layer after a conv layer flattens in (C, H, W) order.
 """
@@ -137,12 +141,23 @@ def w_rowsum(L):
     return W.reshape(W.shape[0], -1).sum(1)
 
 
+def layer_input(t0, ctxs, l, L):
+    """Input of layer l: the previous output, with a skip layer's delayed
+    source placed first along channels (App. C.3: the third layer of a
+    skip-and-delay block also receives the block's input, 2 tau_shift later)."""
+    x = np.asarray(t0, float) if l == 0 else ctxs[l - 1]["t"]
+    sk = L.get("skip")
+    if sk is None:
+        return x
+    src, delay = sk
+    a = np.asarray(t0, float) if src < 0 else ctxs[src]["t"]
+    return np.concatenate([a + delay, x], axis=1)
+
+
 def forward_net(t0, layers, solver="table"):
-    ctxs, t = [], np.asarray(t0, float)
-    for L in layers:
-        ctx = forward_layer(t, L, solver)
-        ctxs.append(ctx)
-        t = ctx["t"]
+    ctxs = []
+    for l, L in enumerate(layers):
+        ctxs.append(forward_layer(layer_input(t0, ctxs, l, L), L, solver))
     return ctxs
 
 
@@ -175,18 +190,28 @@ def train_objective(t0, layers, labels, tau_soft, solver="table", backward=True)
     if not backward:
         return C, parts, None, ctxs
     grads = [None] * len(layers)
-    g_up = g.reshape(ctxs[-1]["t"].shape)
+    # dC/d(output of layer l) from the layers that read it (and the loss)
+    g_out = [np.zeros(c["t"].shape) for c in ctxs]
+    g_out[-1] = g.reshape(ctxs[-1]["t"].shape)
     for l in range(len(layers) - 1, -1, -1):
         ctx, L = ctxs[l], layers[l]
-        g_t = g_up + gT[l]
+        g_t = g_out[l] + gT[l]
         g_W, g_in = backward_layer(ctx, L, g_t)
         nrm = penalty_norm(ctx)
         W = np.asarray(L["W"], float)
         qg = -L.get("gamma_q", 0.0) * nrm * counts[l]
         g_W = g_W + qg.reshape((-1,) + (1,) * (W.ndim - 1))
         grads[l] = g_W
+        sk = L.get("skip")
+        if sk is not None:
+            # split along channels; the delay has unit derivative
+            src = sk[0]
+            Ca = (np.asarray(t0).shape if src < 0 else ctxs[src]["t"].shape)[1]
+            if src >= 0:
+                g_out[src] = g_out[src] + g_in[:, :Ca]
+            g_in = g_in[:, Ca:]
         if l > 0:
-            g_up = g_in.reshape(ctxs[l - 1]["t"].shape)
+            g_out[l - 1] = g_out[l - 1] + g_in.reshape(ctxs[l - 1]["t"].shape)
     return C, parts, grads, ctxs
 
 

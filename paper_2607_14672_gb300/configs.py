@@ -21,7 +21,7 @@ Layer l's window is [l tau_shift - tau_margin, l tau_shift + tau_width + tau_mar
 and its penalty edges t_head^(l) = l tau_shift + t_head,
 t_tail^(l) = l tau_shift + tau_width - t_tail.
 
-Weight means mu_l (configs 2-5) make about 80% of each layer's neurons fire
+Weight means mu_l (configs 2-5, Syn-SNN-9/20) make about 80% of each layer's neurons fire
 at initialisation on the seed-0 batch with t_offset = 0; they were found once
 by bisection with the oracle (``oracle/calibrate_configs.py``) and are frozen
 here.
@@ -45,6 +45,9 @@ SEED_INPUT, SEED_W, SEED_LABELS, SEED_OFFSET = 0, 1000, 7, 11
 CFG2_MU = (0.03523, 0.01520, 0.01951)
 CFG3_MU_TIMES_N = 17.4
 CFG4_MU = (0.09306, 0.00761, 0.01274, 0.01387, 0.00942, 0.00637, 0.00514, 0.00285, 0.00093)
+SYN9_MU = (0.04479, 0.00758, 0.0125, 0.02298, 0.02083, 0.01099, 0.01407, 0.00318, 0.00084)
+SYN20_MU = (0.28323, 0.00786, 0.01288, 0.00507, 0.01689, 0.02131, 0.00956, 0.00937, 0.01019, 0.00484, 0.01054,
+            0.0105, 0.00636, 0.00449, 0.00506, 0.0024, 0.00522, 0.00541, 0.004, 0.00077)
 CFG5_MU = (0.96918, 0.01896, 0.02438, 0.0258, 0.02676, 0.02719, 0.02923, 0.01346, 0.01353, 0.01343,
            0.01367, 0.01382, 0.01358, 0.01714, 0.00673, 0.00686, 0.00689, 0.00699, 0.00697, 0.00077)
 
@@ -183,6 +186,85 @@ def config5(batch=256, M=64):
         name="cfg5", workload=f"conv LIF TTFS SNN 20 layers on 28x28x1, B={batch}, M={M}, tau=(1.0,0.25), bf16",
         batch=batch, in_shape=(1, 28, 28), loss="ce", tau_soft=SYNFIRE["tau_soft"], n_classes=10, math="bf16",
         inputs=lambda seed=SEED_INPUT, B=batch: synth.intensity_spikes(seed, (B, 1, 28, 28), 0.0, SYNFIRE["tau_in"]),
+        labels=lambda seed=SEED_LABELS, B=batch: synth.labels(seed, B, 10),
+        layers=layers, shapes=shapes)
+
+
+def _conv_k(W, tau, M, l, stride, pad, in_shape, skip=None):
+    d = _conv(W, tau[0], tau[1], M, stride, in_shape, **synfire_layer(l))
+    d["pad"] = pad
+    if skip is not None:
+        d["skip"] = skip
+    return d
+
+
+def syn_snn9(N=64, batch=50, M=20, tau=(INF, INF), mus=None):
+    """Syn-SNN-9 of Tab. architectures on 32x32 colour images:
+    C(N,3,1)-C(N,3,1)-C(N,3,1)-C(N,3,2)-C(2N,3,1)-C(2N,3,1)-C(2N,3,2)-C(2N,5,1)-10,
+    with the input channels doubled (x and 1 - x, App. C.2: 6 input
+    channels); zero-spike padding keeps the size ("same" padding, pad = k // 2):
+    32 -> 16 (layer 4) -> 8 (layer 7), readout 2N*8*8 -> 10. Batch 50 and
+    (tau_m, tau_s) = (inf, inf) as in the paper's experiments; M = 20."""
+    mus = SYN9_MU if mus is None else mus
+    spec = [(N, 3, 1), (N, 3, 1), (N, 3, 1), (N, 3, 2), (2 * N, 3, 1), (2 * N, 3, 1), (2 * N, 3, 2), (2 * N, 5, 1)]
+    C, H = 6, 32
+    layers, shapes = [], []
+    for l, (co, k, st) in enumerate(spec, start=1):
+        W = synth.normal_weights(SEED_W + l, (co, C, k, k), mus[l - 1], 1.0 / math.sqrt(C * k * k))
+        layers.append(_conv_k(W, tau, M, l, st, k // 2, (C, H, H)))
+        H = (H + 2 * (k // 2) - k) // st + 1
+        C = co
+        shapes.append((C, H, H))
+    l = len(spec) + 1
+    W = synth.normal_weights(SEED_W + l, (10, C * H * H), mus[l - 1], 1.0 / math.sqrt(C * H * H))
+    layers.append(_dense(W, tau[0], tau[1], M, **synfire_layer(l)))
+    shapes.append((10,))
+    return dict(
+        name="syn_snn9", workload=f"Syn-SNN-9 (Tab. architectures), N={N}, 32x32x6 input, B={batch}, M={M}, "
+                                  f"tau=({tau[0]},{tau[1]}), bf16",
+        batch=batch, in_shape=(6, 32, 32), loss="ce", tau_soft=SYNFIRE["tau_soft"], n_classes=10, math="bf16",
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.doubled_intensity_spikes(seed, (B, 3, 32, 32), SYNFIRE["tau_in"]),
+        labels=lambda seed=SEED_LABELS, B=batch: synth.labels(seed, B, 10),
+        layers=layers, shapes=shapes)
+
+
+def syn_snn20(N=64, batch=50, M=20, tau=(INF, INF), mus=None, size=28, C_in=1):
+    """Syn-SNN-20 of Tab. architectures on 28x28 grey images:
+    C(N,3,1)-SD2(N)-SD1(N)-SD2(2N)-SD1(2N)-SD2(4N)-SD1(4N)-10.
+    A skip-and-delay block (Fig. skip_connection) is three 3x3 conv layers;
+    the third sees the block's input, delayed by 2 tau_shift, beside the
+    second layer's output (channels concatenated, the delayed input first).
+    In SD2 all three keep N channels and stride 1; in SD1 the third has
+    stride 2 and 2N channels: 28 -> 14 -> 7 -> 4, readout 8N*4*4 -> 10.
+    Batch 50, (tau_m, tau_s) = (inf, inf); M = 20."""
+    mus = SYN20_MU if mus is None else mus
+    spec = [(N, 1, None)]                       # (C_out, stride, skip source) per conv layer
+    width = N
+    for kind, mult in (("SD2", 1), ("SD1", 1), ("SD2", 2), ("SD1", 2), ("SD2", 4), ("SD1", 4)):
+        w = N * mult
+        src = len(spec) - 1                     # index of the block's input layer
+        spec += [(w, 1, None), (w, 1, None), (2 * w if kind == "SD1" else w, 2 if kind == "SD1" else 1, src)]
+    delay = 2 * SYNFIRE["tau_shift"]
+    C, H = C_in, size
+    layers, shapes, outs = [], [], []
+    for l, (co, st, src) in enumerate(spec, start=1):
+        cin = C + (outs[src][0] if src is not None else 0)
+        W = synth.normal_weights(SEED_W + l, (co, cin, 3, 3), mus[l - 1], 1.0 / math.sqrt(cin * 9))
+        layers.append(_conv_k(W, tau, M, l, st, 1, (cin, H, H), None if src is None else (src, delay)))
+        H = (H + 2 - 3) // st + 1
+        C = co
+        outs.append((C, H, H))
+        shapes.append((C, H, H))
+    l = len(spec) + 1
+    W = synth.normal_weights(SEED_W + l, (10, C * H * H), mus[l - 1], 1.0 / math.sqrt(C * H * H))
+    layers.append(_dense(W, tau[0], tau[1], M, **synfire_layer(l)))
+    shapes.append((10,))
+    return dict(
+        name="syn_snn20", workload=f"Syn-SNN-20 (Tab. architectures, skip-and-delay blocks), N={N}, "
+                                   f"{size}x{size}x{C_in} input, B={batch}, M={M}, tau=({tau[0]},{tau[1]}), bf16",
+        batch=batch, in_shape=(C_in, size, size), loss="ce", tau_soft=SYNFIRE["tau_soft"], n_classes=10, math="bf16",
+        inputs=lambda seed=SEED_INPUT, B=batch: synth.intensity_spikes(seed, (B, C_in, size, size), 0.0,
+                                                                       SYNFIRE["tau_in"]),
         labels=lambda seed=SEED_LABELS, B=batch: synth.labels(seed, B, 10),
         layers=layers, shapes=shapes)
 

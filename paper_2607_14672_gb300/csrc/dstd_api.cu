@@ -89,12 +89,13 @@ inline int cu(cudaError_t e) { return e == cudaSuccess ? DSTD_OK : DSTD_E_CUDA; 
 // ---------------------------------------------------------------------------
 enum Kind {
     KK_PREP = 0, KK_BIN, KK_BIN_T, KK_GEMM_FWD, KK_SCAN, KK_DWHAT, KK_GEMM_DS, KK_GT, KK_GEMM_DW, KK_REDUCE,
-    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_NARROW_FWD, KK_NARROW_BWD, KK_EXACT_FWD, KK_COUNT
+    KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_NARROW_FWD, KK_NARROW_BWD, KK_EXACT_FWD, KK_SKIP,
+    KK_COUNT
 };
 const char *const kKindNames[KK_COUNT] = {
     "prep_weights", "binning", "binning_T", "gemm_fwd_scan", "scan_solve", "dwhat", "gemm_dS_gradt",
     "gradt_gather", "gemm_dW", "dw_reduce", "loss", "adamw", "binning_public", "what_public", "selftest", "narrow_fwd",
-    "narrow_bwd", "exact_fwd"};
+    "narrow_bwd", "exact_fwd", "skip_channels"};
 
 struct Timing {
     std::mutex mu;
@@ -202,6 +203,10 @@ struct Fork {
     SideSet *ss = nullptr;
     std::unique_lock<std::mutex> lk;
     explicit Fork(cudaStream_t st) : main(st), side{st, st}, lk(g_side_mu) {
+        // with kernel timing on, everything runs on the caller's stream, one
+        // kernel after another, so that each kind's time is its own (and not
+        // that of kernels sharing the GPU with it)
+        if (g_timing.on) return;
         int dev = 0;
         if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return;
         SideSet &q = g_side[dev];
@@ -857,6 +862,23 @@ int dstd_ce_loss(const float *t_L, const int32_t *labels, int B, int C, float ta
     TRY(device_ok());
     Timed tm(KK_LOSS, (cudaStream_t)stream);
     return cu(launch_ce_loss(t_L, labels, B, C, tau_soft, t_silent, loss, g_t_L, (cudaStream_t)stream));
+}
+
+int dstd_concat_channels(const float *a, int C_a, float delay_a, const float *b, int C_b, int64_t positions,
+                         float *out, dstd_stream_t stream) {
+    if (!a || !b || !out || C_a < 1 || C_b < 1 || positions < 1 || !isfinite(delay_a)) return DSTD_E_INVALID;
+    TRY(device_ok());
+    Timed tm(KK_SKIP, (cudaStream_t)stream);
+    return cu(launch_concat_channels(a, C_a, delay_a, b, C_b, positions, out, (cudaStream_t)stream));
+}
+
+int dstd_split_channels(const float *g, int C_a, int C_b, int64_t positions, float *g_a, int accumulate_a,
+                        float *g_b, int accumulate_b, dstd_stream_t stream) {
+    if (!g || (!g_a && !g_b) || C_a < 1 || C_b < 1 || positions < 1) return DSTD_E_INVALID;
+    TRY(device_ok());
+    Timed tm(KK_SKIP, (cudaStream_t)stream);
+    return cu(launch_split_channels(g, C_a, C_b, positions, g_a, accumulate_a != 0, g_b, accumulate_b != 0,
+                                    (cudaStream_t)stream));
 }
 
 int dstd_sum_t_loss(const float *t, int64_t n, float *loss, float *g, dstd_stream_t stream) {

@@ -419,6 +419,10 @@ int tc_gemm_pair_policy(int policy);
 cudaError_t launch_ce_loss(const float *t, const int32_t *lab, int B, int C, float tau_soft, float t_silent,
                            float *loss, float *g, cudaStream_t st);
 cudaError_t launch_sum_t(const float *t, long long n, float *loss, float *g, cudaStream_t st);
+cudaError_t launch_concat_channels(const float *a, int Ca, float delay, const float *b, int Cb, long long P, float *out,
+                                   cudaStream_t st);
+cudaError_t launch_split_channels(const float *g, int Ca, int Cb, long long P, float *ga, bool acc_a, float *gb,
+                                  bool acc_b, cudaStream_t st);
 cudaError_t launch_adamw(float *w, const float *g, float *m, float *v, long long n, float lr, float b1, float b2,
                          float eps, float wd, int step, cudaStream_t st);
 

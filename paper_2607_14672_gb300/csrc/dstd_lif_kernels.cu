@@ -222,9 +222,110 @@ cudaError_t launch_prep_weights_f16(const float *W, int R, int C, __half *hi, __
     return cudaGetLastError();
 }
 
+// The forward operand in the bf16 modes: row r of W split into bf16 hi (and
+// lo), padded with zeros to ldo columns, and the row's sum; one block per
+// row, two adjacent columns per thread and step (one 4-byte store of a bf16
+// pair per array), the sum reduced in a fixed order.
+__global__ void __launch_bounds__(PREP_THREADS) k_split_rows_bf16(const float *__restrict__ W, int C,
+                                                                  __nv_bfloat16 *hi, __nv_bfloat16 *lo, int ldo,
+                                                                  float *rowsum) {
+    __shared__ float red[PREP_THREADS / 32];
+    const int r = blockIdx.x;
+    const float *w = W + (long long)r * C;
+    float sum = 0.f;
+    for (int j = 2 * threadIdx.x; j < ldo; j += 2 * PREP_THREADS) {
+        const float x0 = j < C ? w[j] : 0.f, x1 = j + 1 < C ? w[j + 1] : 0.f;
+        sum += x0 + x1;
+        __nv_bfloat16 h0, l0, h1, l1;
+        split_bf16(x0, h0, l0);
+        split_bf16(x1, h1, l1);
+        const long long o = (long long)r * ldo + j;
+        *reinterpret_cast<__nv_bfloat162 *>(hi + o) = __halves2bfloat162(h0, h1);
+        if (lo) *reinterpret_cast<__nv_bfloat162 *>(lo + o) = __halves2bfloat162(l0, l1);
+    }
+    for (int j = ldo + threadIdx.x; j < C; j += PREP_THREADS) sum += w[j];  // columns past ldo (none in practice)
+    if (!rowsum) return;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sum;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float t = 0.f;
+        for (int k = 0; k < PREP_THREADS / 32; ++k) t += red[k];
+        rowsum[r] = t;
+    }
+}
+
+// Transposed copies only (W^T split into bf16 hi/lo, or W^T in fp32): one
+// 64 x 64 tile per block, read row by row (two 128-byte rows per warp
+// instruction pair), written as 64 output rows of 64 elements, two elements
+// per lane (one 4-byte store of a bf16 pair), so that a warp writes 128
+// contiguous bytes per instruction and array.
+constexpr int SPLIT_T_TILE = 64;
+__global__ void __launch_bounds__(256) k_split_T(const float *__restrict__ W, int R, int C,
+                                                 __nv_bfloat16 *hiT, __nv_bfloat16 *loT, int ldt, float *f32T,
+                                                 int ldf, int pairs) {
+    __shared__ float tile[SPLIT_T_TILE][SPLIT_T_TILE + 1];
+    const int c0 = blockIdx.x * SPLIT_T_TILE, r0 = blockIdx.y * SPLIT_T_TILE;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+    for (int k = 0; k < SPLIT_T_TILE / 8; ++k) {
+        const int rr = w + 8 * k, r = r0 + rr;
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int cc = c0 + lane + 32 * hh;
+            tile[rr][lane + 32 * hh] = (r < R && cc < C) ? W[(long long)r * C + cc] : 0.0f;
+        }
+    }
+    __syncthreads();
+    const int r = r0 + 2 * lane;
+#pragma unroll
+    for (int k = 0; k < SPLIT_T_TILE / 8; ++k) {
+        const int cl = w + 8 * k, cc = c0 + cl;
+        if (cc >= C) break;
+        const float x0 = tile[2 * lane][cl], x1 = tile[2 * lane + 1][cl];
+        if (hiT && r < ldt) {
+            __nv_bfloat16 h0, l0, h1, l1;
+            split_bf16(x0, h0, l0);
+            split_bf16(x1, h1, l1);
+            const long long o = (long long)cc * ldt + r;
+            if (pairs && r + 1 < ldt) {
+                *reinterpret_cast<__nv_bfloat162 *>(hiT + o) = __halves2bfloat162(h0, h1);
+                if (loT) *reinterpret_cast<__nv_bfloat162 *>(loT + o) = __halves2bfloat162(l0, l1);
+            } else {
+                hiT[o] = h0;
+                if (loT) loT[o] = l0;
+                if (r + 1 < ldt) {
+                    hiT[o + 1] = h1;
+                    if (loT) loT[o + 1] = l1;
+                }
+            }
+        }
+        if (f32T && r < ldf) {
+            const long long o = (long long)cc * ldf + r;
+            f32T[o] = x0;
+            if (r + 1 < ldf) f32T[o + 1] = x1;
+        }
+    }
+}
+
 cudaError_t launch_prep_weights(const float *W, int R, int C, OpKind op, __nv_bfloat16 *hi, __nv_bfloat16 *lo,
                                 int ldo, __nv_bfloat16 *hiT, __nv_bfloat16 *loT, int ldt, float *f32T, int ldf,
                                 float *rowsum, cudaStream_t st) {
+    if (hi && !hiT && !f32T && ldo >= C && ldo % 2 == 0 && ((uintptr_t)hi % 4 == 0) && (!lo || (uintptr_t)lo % 4 == 0)) {
+        k_split_rows_bf16<<<R, PREP_THREADS, 0, st>>>(W, C, hi, lo, ldo, rowsum);
+        return cudaGetLastError();
+    }
+    if (!hi && !rowsum && (hiT || f32T)) {
+        int rr = R;  // output columns to write, padding included
+        if (hiT && ldt > rr) rr = ldt;
+        if (f32T && ldf > rr) rr = ldf;
+        // bf16 pair stores need every output row to start on a 4-byte boundary
+        const int pairs = hiT && (ldt % 2 == 0) && ((uintptr_t)hiT % 4 == 0) && (!loT || (uintptr_t)loT % 4 == 0);
+        dim3 grid((unsigned)((C + SPLIT_T_TILE - 1) / SPLIT_T_TILE), (unsigned)((rr + SPLIT_T_TILE - 1) / SPLIT_T_TILE));
+        k_split_T<<<grid, 256, 0, st>>>(W, R, C, hiT, loT, ldt, f32T, ldf, pairs);
+        return cudaGetLastError();
+    }
     if (rowsum) {
         cudaError_t e = cudaMemsetAsync(rowsum, 0, sizeof(float) * R, st);
         if (e != cudaSuccess) return e;
@@ -1434,12 +1535,110 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
     }
 }
 
+// The same values in the (i, (b, m)) layout only, written row-contiguously:
+// a warp per neuron i and a block per 8 neurons x spb (<= 32) samples. Lane
+// k first takes the scalars of sample b0 + k (coefficient, s, q and the two
+// kernel values next to the spike); then lane f of the warp's (sample,
+// 16-byte chunk) sequence fetches its sample's scalars from the owning lane
+// and writes chunk f, so every store instruction covers up to 512 contiguous
+// bytes of row i (the samples of a row are adjacent: column b Mp + m).
+// Silent neurons are counted per warp and added with one atomic.
+template <int OP>
+__global__ void __launch_bounds__(256) k_dwhat_rows(const float *__restrict__ t_out, const int *__restrict__ qv,
+                                                    const float *__restrict__ sv, const float *__restrict__ vd,
+                                                    const float *__restrict__ g_up, int B, int N, LifConst c,
+                                                    void *a_hi, void *a_lo, int lda, float *count, int spb) {
+    constexpr int EB = OP == 0 ? 4 : 2;
+    constexpr int BPC = 16 / EB;
+    const int lane = threadIdx.x & 31;
+    const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (i >= N) return;
+    const int b0 = blockIdx.y * spb;
+    const int nb = (B - b0) < spb ? (B - b0) : spb;
+    const int cps = c.Mp / BPC;
+    const int total = nb * cps;
+    int pq = c.M;
+    float pcoef = 0.f, ps0 = 0.f, pKq = 0.f, pKq1 = 0.f;
+    if (lane < nb) {
+        const long long idx = (long long)(b0 + lane) * N + i;
+        pq = qv[idx];
+        const float to = t_out[idx], gu = g_up ? g_up[idx] : 0.f, vdi = vd[idx], s0 = sv[idx];
+        if (pq < c.M) {
+            float pv, pg;
+            penalty_T(c, to, pv, pg);
+            pcoef = -(gu + pg) / vdi;
+            ps0 = s0;
+            pKq = kernel_K(c, s0);
+            pKq1 = kernel_K(c, s0 + c.dt);
+        }
+    }
+    if (count) {
+        const int silent = __popc(__ballot_sync(0xffffffffu, lane < nb && pq >= c.M));
+        if (lane == 0 && silent) atomicAdd(&count[i], (float)silent);
+    }
+    const float fv = __expf(c.av * c.dt), fI = __expf(c.aI * c.dt);
+    for (int f0 = 0; f0 < total; f0 += 32) {
+        const int f = f0 + lane;
+        const bool valid = f < total;
+        const int bl = f / cps, ch = f - bl * cps;
+        const int src = valid ? bl : 0;
+        const int q = __shfl_sync(0xffffffffu, pq, src);
+        const float coef = __shfl_sync(0xffffffffu, pcoef, src);
+        const float s0 = __shfl_sync(0xffffffffu, ps0, src);
+        const float Kq = __shfl_sync(0xffffffffu, pKq, src);
+        const float Kq1 = __shfl_sync(0xffffffffu, pKq1, src);
+        if (!valid) continue;
+        const int m0 = ch * BPC;
+        float v[BPC];
+#pragma unroll
+        for (int u = 0; u < BPC; ++u) v[u] = 0.f;
+        if (q < c.M && m0 <= q) {
+            float x = s0 + (float)(q - m0) * c.dt;
+            float ev = __expf(-c.av * x), eI = __expf(-c.aI * x);
+#pragma unroll
+            for (int u = 0; u < BPC; ++u) {
+                const int m = m0 + u;
+                const float Kf = c.lam_zero ? x * ev : (ev - eI) * c.inv_lam;
+                const float K = (m == q) ? Kq : ((m == q - 1) ? Kq1 : Kf);
+                v[u] = (m <= q) ? coef * K : 0.f;
+                ev *= fv;
+                eI *= fI;
+                x -= c.dt;
+            }
+        }
+        const long long o = (long long)i * lda + (long long)(b0 + bl) * c.Mp + m0;
+        if (OP == 0) {
+            *reinterpret_cast<float4 *>((float *)a_hi + o) = make_float4(v[0], v[1], v[2], v[3]);
+        } else {
+            __align__(16) __nv_bfloat16 hh[BPC], ll[BPC];
+#pragma unroll
+            for (int u = 0; u < BPC; ++u) split_bf16(v[u], hh[u], ll[u]);
+            *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + o) = *reinterpret_cast<uint4 *>(hh);
+            if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + o) = *reinterpret_cast<uint4 *>(ll);
+        }
+    }
+}
+
 cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                          int B, int N, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda, void *b_hi,
                          void *b_lo, int ldb, float *silent_count, cudaStream_t st, bool accumulate_count) {
     if (silent_count && !accumulate_count) {
         cudaError_t e = cudaMemsetAsync(silent_count, 0, sizeof(float) * N, st);
         if (e != cudaSuccess) return e;
+    }
+    // samples per block: 64 chunks per warp (two stores per lane and array), at most 32
+    const int cps = c.Mp / (op == OpKind::F32 ? 4 : 8);
+    const int spb = cps >= 32 ? 2 : (64 / cps > 32 ? 32 : 64 / cps);
+    const long long gy = ((long long)B + spb - 1) / spb;
+    if (!b_hi && gy <= 65535) {
+        dim3 grid((unsigned)((N + 7) / 8), (unsigned)gy);
+        if (op == OpKind::F32)
+            k_dwhat_rows<0><<<grid, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, silent_count, spb);
+        else if (op == OpKind::BF16X3)
+            k_dwhat_rows<1><<<grid, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, silent_count, spb);
+        else
+            k_dwhat_rows<2><<<grid, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, silent_count, spb);
+        return cudaGetLastError();
     }
     long long n = 2ll * B * N;  // two lanes per neuron
     unsigned g = blocks_for(n, 256);
@@ -1662,6 +1861,58 @@ __global__ void k_sum_t(const float *__restrict__ t, long long n, float *loss, f
     }
     float v = warp_sum(c);
     if ((threadIdx.x & 31) == 0 && v != 0.f) atomicAdd(loss, v);
+}
+
+// ---------------------------------------------------------------------------
+// Skip-and-delay input (App. C.3, Fig. skip_connection): the third layer of
+// a block sees the block's input, delayed by a fixed time, beside the second
+// layer's output. With NHWC spike tensors (channels innermost) that is a
+// concatenation along channels per position p:
+//   out[p, 0:Ca] = a[p, :] + delay,   out[p, Ca:Ca+Cb] = b[p, :]
+// (+inf stays +inf: a silent input stays silent). Its adjoint splits the
+// gradient back, overwriting or adding into each part.
+// ---------------------------------------------------------------------------
+__global__ void k_concat_channels(const float *__restrict__ a, int Ca, float delay, const float *__restrict__ b,
+                                  int Cb, long long n, float *out) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= n) return;
+    const int Ct = Ca + Cb;
+    const long long p = idx / Ct;
+    const int ch = (int)(idx - p * Ct);
+    out[idx] = ch < Ca ? a[p * Ca + ch] + delay : b[p * Cb + (ch - Ca)];
+}
+
+__global__ void k_split_channels(const float *__restrict__ g, int Ca, int Cb, long long n, float *ga, int acc_a,
+                                 float *gb, int acc_b) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= n) return;
+    const int Ct = Ca + Cb;
+    const long long p = idx / Ct;
+    const int ch = (int)(idx - p * Ct);
+    const float v = g[idx];
+    if (ch < Ca) {
+        if (ga) {
+            float *d = ga + p * Ca + ch;
+            *d = acc_a ? *d + v : v;
+        }
+    } else if (gb) {
+        float *d = gb + p * Cb + (ch - Ca);
+        *d = acc_b ? *d + v : v;
+    }
+}
+
+cudaError_t launch_concat_channels(const float *a, int Ca, float delay, const float *b, int Cb, long long P, float *out,
+                                   cudaStream_t st) {
+    const long long n = P * (Ca + Cb);
+    k_concat_channels<<<blocks_for(n, 256), 256, 0, st>>>(a, Ca, delay, b, Cb, n, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_split_channels(const float *g, int Ca, int Cb, long long P, float *ga, bool acc_a, float *gb,
+                                  bool acc_b, cudaStream_t st) {
+    const long long n = P * (Ca + Cb);
+    k_split_channels<<<blocks_for(n, 256), 256, 0, st>>>(g, Ca, Cb, n, ga, acc_a ? 1 : 0, gb, acc_b ? 1 : 0);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_sum_t(const float *t, long long n, float *loss, float *g, cudaStream_t st) {

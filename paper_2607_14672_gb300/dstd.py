@@ -23,7 +23,7 @@ EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd",
-           "dstd_exact_workspace_bytes", "dstd_exact_fwd")
+           "dstd_exact_workspace_bytes", "dstd_exact_fwd", "dstd_concat_channels", "dstd_split_channels")
 
 
 class DstdError(RuntimeError):
@@ -97,6 +97,8 @@ def load(path=None):
         "dstd_conv_workspace_bytes": (_SZ, [_I, _I, _I, _I, _I, _I, _I, _I, _PP, _I]),
         "dstd_conv_fwd": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _P, _SZ, _P]),
         "dstd_conv_bwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
+        "dstd_concat_channels": (_I, [_P, _I, _F, _P, _I, _I64, _P, _P]),
+        "dstd_split_channels": (_I, [_P, _I, _I, _I64, _P, _I, _P, _I, _P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -276,6 +278,30 @@ def ce_loss(t_L, labels, tau_soft, t_silent, loss, g_t_L, stream=None):
     _f32(t_L, "t_L")
     _check(load().dstd_ce_loss(_ptr(t_L), _ptr(labels), B, C, float(tau_soft), float(t_silent), _ptr(loss),
                                _ptr(g_t_L), _stream(stream)), "dstd_ce_loss")
+
+
+def concat_channels(a, b, delay_a, out, stream=None):
+    """out[..., :C_a] = a + delay_a, out[..., C_a:] = b (channels innermost)."""
+    for x, nm in ((a, "a"), (b, "b"), (out, "out")):
+        _f32(x, nm)
+    Ca, Cb = a.shape[-1], b.shape[-1]
+    P = a.numel() // Ca
+    if b.numel() != P * Cb or out.numel() != P * (Ca + Cb):
+        raise ValueError("concat_channels: a, b and out disagree on the number of positions")
+    _check(load().dstd_concat_channels(_ptr(a), Ca, float(delay_a), _ptr(b), Cb, P, _ptr(out),
+                                       _stream(stream)), "dstd_concat_channels")
+
+
+def split_channels(g, C_a, g_a=None, accumulate_a=False, g_b=None, accumulate_b=False, stream=None):
+    """Adjoint of concat_channels: g[..., :C_a] into g_a, g[..., C_a:] into g_b
+    (overwriting, or adding with accumulate_*); either target may be None."""
+    _f32(g, "g")
+    Ct = g.shape[-1]
+    Cb = Ct - C_a
+    P = g.numel() // Ct
+    _check(load().dstd_split_channels(_ptr(g), int(C_a), int(Cb), P, _ptr(g_a) if g_a is not None else None,
+                                      int(bool(accumulate_a)), _ptr(g_b) if g_b is not None else None,
+                                      int(bool(accumulate_b)), _stream(stream)), "dstd_split_channels")
 
 
 def sum_t_loss(t, loss, g, stream=None):

@@ -165,10 +165,24 @@ class ConvNet:
         C, H, Wd = cfg["in_shape"]
         self.in_shape = (H, Wd, C)
         self.W, self.p, self.t, self.g, self.saved, self.geom = [], [], [], [], [], []
+        # skip-and-delay layers (App. C.3): per layer, (source layer or -1, delay,
+        # concatenated input, its gradient), else None
+        self.skip = []
         ws = 0
         shape = (H, Wd, C)
-        for L in self.layers:
+        for l, L in enumerate(self.layers):
             Wl = torch.tensor(L["W"], dtype=torch.float32)
+            sk = L.get("skip")
+            if sk is not None:
+                src, delay = int(sk[0]), float(sk[1])
+                s_shape = (H, Wd, C) if src < 0 else tuple(self.t[src].shape[1:])
+                if s_shape[:2] != shape[:2]:
+                    raise ValueError(f"layer {l}: skip source and previous output differ in size")
+                shape = (shape[0], shape[1], s_shape[2] + shape[2])
+                cat = torch.empty((B,) + shape, dtype=torch.float32, device=dev)
+                self.skip.append((src, delay, cat, torch.empty_like(cat), s_shape[2]))
+            else:
+                self.skip.append(None)
             if L["kind"] == "conv":
                 Hh, Ww, Cc = shape
                 k, st, pad = Wl.shape[2], L["stride"], L["pad"]
@@ -223,10 +237,17 @@ class ConvNet:
             self.labels.copy_(torch.as_tensor(labels, dtype=torch.int32), non_blocking=True)
 
     def layer_input(self, l):
+        if self.skip[l] is not None:
+            return self.skip[l][2]
         return self.t_in if l == 0 else self.t[l - 1]
 
     def forward(self, stream=None):
         for l, L in enumerate(self.layers):
+            sk = self.skip[l]
+            if sk is not None:
+                src, delay, cat = sk[0], sk[1], sk[2]
+                dstd.concat_channels(self.t_in if src < 0 else self.t[src], self.t_in if l == 0 else self.t[l - 1],
+                                     delay, cat, stream)
             x = self.layer_input(l)
             if self.geom[l] is not None:
                 _, _, _, k, st, pad = self.geom[l]
@@ -241,9 +262,18 @@ class ConvNet:
                      self.g[-1], stream)
 
     def backward(self, stream=None):
+        """Layers in reverse. A layer's input gradient overwrites the previous
+        output's; a skip layer's goes to its concatenated input and is split:
+        the previous layer's part overwrites, and the delayed source's part
+        is added into the source's gradient once the layer after the source
+        (the block's first layer) has written it."""
         for l in range(len(self.layers) - 1, -1, -1):
             x = self.layer_input(l)
-            g_in = self.g[l - 1] if l > 0 else None
+            sk = self.skip[l]
+            if sk is not None:
+                g_in = sk[3]
+            else:
+                g_in = self.g[l - 1] if l > 0 else None
             if self.geom[l] is not None:
                 _, _, _, k, st, pad = self.geom[l]
                 dstd.conv_bwd(x, self.W[l], self.t[l], self.saved[l], self.g[l], st, pad, self.p[l], self.math,
@@ -252,6 +282,13 @@ class ConvNet:
                 dstd.dense_bwd(x.reshape(self.B, -1), self.W[l], self.t[l], self.saved[l], self.g[l], self.p[l],
                                self.math, None if g_in is None else g_in.reshape(self.B, -1), self.gW[l],
                                self.workspace, stream)
+            if sk is not None and l > 0:
+                dstd.split_channels(sk[3], sk[4], g_b=self.g[l - 1], stream=stream)
+            # skip layers that read the output of layer l - 1: add their part now
+            for m in range(l, len(self.layers)):
+                sm = self.skip[m]
+                if sm is not None and sm[0] == l - 1 and l > 0:
+                    dstd.split_channels(sm[3], sm[4], g_a=self.g[l - 1], accumulate_a=True, stream=stream)
 
     def optimizer(self, lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=1e-2, stream=None):
         dstd.adamw_multi(self.W, self.gW, self.m, self.v, lr, betas[0], betas[1], eps, weight_decay,

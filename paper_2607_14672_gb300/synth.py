@@ -38,6 +38,15 @@ def intensity_spikes(seed, shape, zero_frac=0.0, tau_in=1.0):
     return np.where(x > 0.0, tau_in * (1.0 - x), np.inf)
 
 
+def doubled_intensity_spikes(seed, shape, tau_in=1.0):
+    """Colour-image input with the channel doubling of App. C.2: x ~ U[0, 1)
+    of shape (B, C, H, W), channels C..2C-1 hold 1 - x, and every pixel is
+    encoded as t = tau_in (1 - x) (so no input is silent)."""
+    x = rng(seed).random(size=shape)
+    x2 = np.concatenate([x, 1.0 - x], axis=1)
+    return tau_in * (1.0 - x2)
+
+
 def normal_weights(seed, shape, mean=0.0, std=1.0):
     return rng(seed).normal(mean, std, size=shape)
 

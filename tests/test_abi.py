@@ -106,6 +106,12 @@ def test_null_and_bad_arguments_rejected_on_host(lib):
                           ctypes.c_float(1e-8), ctypes.c_float(0.0), 0, None) == -1
     # contraction scheduling policy: 0, 1, 2 valid (previous returned), anything else rejected
     assert lib.dstd_set_pair_policy(3) == -1 and lib.dstd_set_pair_policy(-1) == -1
+    # skip-and-delay channel concatenation and its adjoint
+    assert lib.dstd_concat_channels(None, 4, ctypes.c_float(0.2), one, 4, 10, one, None) == -1
+    assert lib.dstd_concat_channels(one, 0, ctypes.c_float(0.2), one, 4, 10, one, None) == -1
+    assert lib.dstd_concat_channels(one, 4, ctypes.c_float(float("inf")), one, 4, 10, one, None) == -1
+    assert lib.dstd_split_channels(one, 4, 4, 10, None, 0, None, 0, None) == -1
+    assert lib.dstd_split_channels(one, 4, 4, 0, one, 0, one, 0, None) == -1
     assert lib.dstd_set_pair_policy(2) == 0 and lib.dstd_set_pair_policy(0) == 2
     # multi-tensor AdamW: tensor count, null step buffer, misaligned step buffer, empty tensor, bad beta
     ptrs = (ctypes.c_void_p * 33)(*([256] * 33))

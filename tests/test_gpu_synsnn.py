@@ -1,0 +1,151 @@
+"""GPU parity of the paper's two network architectures (Tab. architectures)
+against the float64 oracle: Syn-SNN-9 (a 5x5 layer, the doubled colour
+input of App. C.2) and Syn-SNN-20 (skip-and-delay blocks, App. C.3, Fig.
+skip_connection), built by ``net.ConvNet`` from the library's calls.
+
+The networks run at a reduced width (N = 4) so that the oracle checks every
+neuron; the architecture, strides, kernel sizes, skip wiring and delays are
+those of the full networks. Weight means come from the oracle's calibration
+(80% firing per layer), 3% larger so that no neuron sits at the threshold.
+The contraction runs in the three-product mode (fp32 accuracy), so spike
+times must agree within 1e-4 T_max and masks exactly away from the
+threshold; whole-network weight gradients within 1e-3 relative L2.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from helpers import f32, rel_l2
+from oracle import calibrate_configs as ocal, network as onet
+
+pytestmark = pytest.mark.gpu
+
+MARGIN = 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    from paper_2607_14672_gb300 import build, dstd
+    build.build()
+    dstd.load()
+    assert dstd.device_status(clear=True) == 0
+    yield
+    assert dstd.device_status(clear=True) == 0
+
+
+def host(x):
+    return x.detach().cpu().numpy().astype(np.float64)
+
+
+def nchw(t):
+    return t.transpose(0, 3, 1, 2) if t.ndim == 4 else t
+
+
+def nhwc(t):
+    return np.ascontiguousarray(t.transpose(0, 2, 3, 1)) if t.ndim == 4 else t
+
+
+def tiny(name):
+    from paper_2607_14672_gb300 import configs
+    if name == "syn20":
+        mk = lambda mus: configs.syn_snn20(N=4, batch=4, M=12, size=8, mus=mus)
+        n_layers = 20
+    else:
+        mk = lambda mus: configs.syn_snn9(N=4, batch=2, M=12, mus=mus)
+        n_layers = 9
+    mus = ocal.calibrate_conv(mk((0.0,) * n_layers), batch=mk((0.0,) * n_layers)["batch"], verbose=False)
+    cfg = mk(tuple(1.03 * m for m in mus))
+    cfg["layers"] = [dict(L, W=f32(L["W"])) for L in cfg["layers"]]
+    return cfg
+
+
+def gpu_net(cfg, seed, with_step):
+    from paper_2607_14672_gb300 import dstd, net
+    n = net.ConvNet(cfg, math_mode="x3", with_adamw=False)
+    t0 = f32(cfg["inputs"](seed=seed))
+    lab = cfg["labels"]()
+    n.set_inputs(t0.astype(np.float32), lab)
+    if with_step:
+        n.step()
+    else:
+        n.forward()
+    torch.cuda.synchronize()
+    assert dstd.device_status(clear=True) == 0
+    return n, t0, lab
+
+
+def test_concat_and_split_channels_bit_exact():
+    from paper_2607_14672_gb300 import dstd
+    g = np.random.default_rng(3)
+    P, Ca, Cb = 1000, 24, 40
+    a = np.where(g.random((P, Ca)) < 0.2, np.inf, g.uniform(0, 1, (P, Ca))).astype(np.float32)
+    b = np.where(g.random((P, Cb)) < 0.2, np.inf, g.uniform(0, 1, (P, Cb))).astype(np.float32)
+    out = torch.empty(P, Ca + Cb, device="cuda")
+    dstd.concat_channels(torch.tensor(a, device="cuda"), torch.tensor(b, device="cuda"), 0.2, out)
+    ref = np.concatenate([a + np.float32(0.2), b], axis=1)
+    np.testing.assert_array_equal(out.cpu().numpy(), ref)
+    gc = g.normal(size=(P, Ca + Cb)).astype(np.float32)
+    ga0 = g.normal(size=(P, Ca)).astype(np.float32)
+    ga = torch.tensor(ga0, device="cuda")
+    gb = torch.full((P, Cb), 7.0, device="cuda")
+    gct = torch.tensor(gc, device="cuda")
+    dstd.split_channels(gct, Ca, g_b=gb)                               # overwrite
+    dstd.split_channels(gct, Ca, g_a=ga, accumulate_a=True)            # add
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(gb.cpu().numpy(), gc[:, Ca:])
+    np.testing.assert_array_equal(ga.cpu().numpy(), ga0 + gc[:, :Ca])
+
+
+@pytest.mark.parametrize("name", ["syn9", "syn20"])
+def test_paper_architecture_layers_match_oracle(name):
+    """Every layer of the network, teacher-forced: the oracle layer sees the
+    GPU's own input to that layer, rebuilt on the host (the delayed skip
+    source first, then the previous output)."""
+    cfg = tiny(name)
+    n, t0, _ = gpu_net(cfg, seed=2, with_step=False)
+    outs = [nchw(host(t)) for t in n.t]
+    checked = 0
+    for l, L in enumerate(cfg["layers"]):
+        x = t0 if l == 0 else outs[l - 1]
+        sk = L.get("skip")
+        if sk is not None:
+            src, delay = sk
+            a = t0 if src < 0 else outs[src]
+            cat = np.concatenate([f32(np.float32(a) + np.float32(delay)), x], axis=1)
+            # the GPU's concatenated input is exactly that (fp32 addition)
+            np.testing.assert_array_equal(nchw(host(n.skip[l][2])), cat)
+            x = cat
+        ctx = onet.forward_layer(x, L)
+        tg = outs[l].reshape(ctx["t"].shape)
+        ok = np.abs(ctx["vpeak"] - L["v_th"]) > MARGIN
+        fg, fo = np.isfinite(tg), np.isfinite(ctx["t"])
+        assert not (ok & (fg != fo)).any(), (l, int((ok & (fg != fo)).sum()))
+        both = ok & fg & fo
+        assert both.sum() > 0.2 * tg.size, l
+        assert np.abs(tg[both] - ctx["t"][both]).max() <= 1e-4 * (L["t_end"] - L["t_first"]), l
+        checked += 1
+    assert checked == len(cfg["layers"])
+
+
+def test_syn20_gradients_match_oracle():
+    """One training step (forward, CE + T + Q, backward) of the 20-layer
+    network with skip-and-delay blocks: the skip's gradient reaches the
+    block's input twice (through the block's first layer and through the
+    skip), and every layer's dC/dW must match the oracle's."""
+    cfg = tiny("syn20")
+    n, t0, lab = gpu_net(cfg, seed=2, with_step=True)
+    C, parts, grads, ctxs = onet.train_objective(t0, cfg["layers"], lab, cfg["tau_soft"])
+    for l, ctx in enumerate(ctxs):
+        assert np.abs(ctx["vpeak"] - 1.0).min() > MARGIN        # no neuron at the threshold
+        tg = nchw(host(n.t[l])).reshape(ctx["t"].shape)
+        np.testing.assert_array_equal(np.isfinite(tg), np.isfinite(ctx["t"]))
+    assert float(n.loss[0]) == pytest.approx(parts["ce"], rel=1e-4)
+    for l, L in enumerate(cfg["layers"]):
+        gW = host(n.gW[l])
+        if L["kind"] == "conv":
+            gW = gW.transpose(0, 3, 1, 2)
+        else:
+            C_, H_, W_ = ctxs[l - 1]["t"].shape[1:]
+            gW = gW.reshape(gW.shape[0], H_, W_, C_).transpose(0, 3, 1, 2).reshape(gW.shape[0], -1)
+        assert rel_l2(gW, grads[l]) <= 1e-3, (l, rel_l2(gW, grads[l]))

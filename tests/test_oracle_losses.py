@@ -110,10 +110,10 @@ def _conv_as_dense(Wc, C, H, Wd, stride, pad):
     return D
 
 
-@pytest.mark.parametrize("stride,pad", [(1, 1), (2, 1), (1, 0)])
-def test_conv_equals_expanded_dense(stride, pad):
+@pytest.mark.parametrize("stride,pad,k", [(1, 1, 3), (2, 1, 3), (1, 0, 3), (1, 2, 5)])
+def test_conv_equals_expanded_dense(stride, pad, k):
     g = np.random.default_rng(3)
-    B, C, H, Wd, O, k = 2, 3, 6, 5, 4, 3
+    B, C, H, Wd, O = 2, 3, 6, 5, 4
     t_in = g.uniform(0, 1, (B, C, H, Wd))
     t_in[g.random(t_in.shape) < 0.2] = INF
     Wc = g.normal(1.0, 1.0, (O, C, k, k))
@@ -177,6 +177,82 @@ def test_network_gradients_by_finite_differences():
             fd[idx] = (network.train_objective(t0, lp, lab, 0.05, backward=False)[0]
                        - network.train_objective(t0, lm, lab, 0.05, backward=False)[0]) / (2 * h)
         assert np.linalg.norm(grads[l] - fd) <= 1e-6 * np.linalg.norm(fd) + 1e-10, l
+
+
+def _skip_net(seed, B=2):
+    """conv 2->3 (3x3) - conv 3->3 (5x5, pad 2) - conv 6->4 (3x3, stride 2) whose
+    input is layer 1's output delayed by 0.2 beside layer 2's (App. C.3) -
+    dense readout; synfire windows as in App. C.1."""
+    g = np.random.default_rng(seed)
+    C0, H = 2, 5
+    specs = [(3, C0, 3, 1, 1, None), (3, 3, 5, 1, 2, None), (4, 6, 3, 2, 1, (0, 0.2))]
+    layers = []
+    for l, (O, C, k, st, pad, skip) in enumerate(specs, start=1):
+        wp = losses.window_params(l, 0.1, 1.0, 0.1, 0.2, 0.2)
+        L = dict(kind="conv", W=g.normal(0.9, 0.5, (O, C, k, k)), tau_v=0.5, tau_I=0.25, v_th=1.0,
+                 t_first=wp["t_first"], t_end=wp["t_end"], M=10, t_offset=0.011 * (-1) ** l, stride=st, pad=pad,
+                 t_head_l=wp["t_head_l"], t_tail_l=wp["t_tail_l"], gamma_head=0.05, gamma_tail=0.01, gamma_q=1e-2)
+        if skip is not None:
+            L["skip"] = skip
+        layers.append(L)
+    wp = losses.window_params(4, 0.1, 1.0, 0.1, 0.2, 0.2)
+    layers.append(dict(kind="dense", W=g.normal(0.5, 0.5, (3, 4 * 3 * 3)), tau_v=0.5, tau_I=0.25, v_th=1.0,
+                       t_first=wp["t_first"], t_end=wp["t_end"], M=10, t_offset=0.0, t_head_l=wp["t_head_l"],
+                       t_tail_l=wp["t_tail_l"], gamma_head=0.05, gamma_tail=0.01, gamma_q=1e-2))
+    t0 = g.uniform(0, 1, (B, C0, H, H))
+    t0[g.random(t0.shape) < 0.2] = INF
+    return t0, layers, g.integers(0, 3, B)
+
+
+def test_skip_input_is_delayed_source_then_previous():
+    # the skip layer's w^ must be the sum of two separate contractions: the
+    # first C_a filter channels over layer 1's spikes 0.2 later, the rest over
+    # layer 2's spikes (a swapped order or a delay of the wrong sign differs)
+    t0, layers, _ = _skip_net(21)
+    ctxs = network.forward_net(t0, layers)
+    L = layers[2]
+    T, dt = network.layer_grid(L)
+    B = t0.shape[0]
+
+    def bins(t):
+        return dstd.binning(t.reshape(B, -1), T, dt, L["tau_v"], L["tau_I"]).reshape((B, L["M"]) + t.shape[1:])
+
+    a, b = ctxs[0]["t"] + 0.2, ctxs[1]["t"]
+    assert np.isfinite(a).sum() > 10 and np.isfinite(b).sum() > 10
+    Ca = a.shape[1]
+    what = (network.conv_what(bins(a), L["W"][:, :Ca], 2, 1) + network.conv_what(bins(b), L["W"][:, Ca:], 2, 1))
+    np.testing.assert_allclose(ctxs[2]["what"], what, rtol=1e-12, atol=1e-12)
+    ref = dstd.solve(what.reshape(B, -1, L["M"]), T, dt, L["tau_v"], L["tau_I"], 1.0)
+    t2 = ctxs[2]["t"].reshape(B, -1)
+    np.testing.assert_array_equal(np.isfinite(t2), np.isfinite(ref["t"]))
+    fin = np.isfinite(t2)
+    assert fin.sum() > 5
+    np.testing.assert_allclose(t2[fin], ref["t"][fin], rtol=0, atol=1e-12)
+
+
+def test_skip_network_gradients_by_finite_differences():
+    t0, layers, lab = _skip_net(22)
+    C, parts, grads, ctxs = network.train_objective(t0, layers, lab, 0.05)
+    assert all(np.isfinite(c["t"]).sum() >= 3 for c in ctxs)
+    h = 1e-7
+    g = np.random.default_rng(5)
+    for l, L in enumerate(layers):
+        # 12 sampled weights per layer (the whole gradient would take long)
+        flat = [tuple(int(v) for v in np.unravel_index(i, L["W"].shape))
+                for i in g.choice(L["W"].size, 12, replace=False)]
+        for idx in flat:
+            Wp, Wm = L["W"].copy(), L["W"].copy()
+            Wp[idx] += h
+            Wm[idx] -= h
+            lp = [dict(x) for x in layers]
+            lm = [dict(x) for x in layers]
+            lp[l]["W"], lm[l]["W"] = Wp, Wm
+            fd = (network.train_objective(t0, lp, lab, 0.05, backward=False)[0]
+                  - network.train_objective(t0, lm, lab, 0.05, backward=False)[0]) / (2 * h)
+            assert abs(grads[l][idx] - fd) <= 1e-6 * max(1.0, abs(fd)), (l, idx, grads[l][idx], fd)
+    # the skip gradient reaches layer 1 twice (through layer 2 and the skip):
+    # dropping the skip's part changes layer 1's gradient
+    assert np.linalg.norm(grads[0]) > 0
 
 
 def test_e_rmse():
