@@ -203,6 +203,37 @@ int dstd_dense_fwd_ce(const float *t_in, const float *W, int B, int N_in, int N_
                       float tau_soft, float t_silent, float *loss, float *g_t_out,
                       dstd_stream_t stream);
 
+/* Multi-spike layers (App. D, Eq. Vmem_multiSpikes): a neuron may fire up to
+ * F_out times in the window; at each spike its membrane potential is reset to
+ * 0 and its synaptic current kept. Each input spike is discretised on its
+ * own and the grid weights of an input's spikes are summed, so w^ = W s is
+ * the same contraction; the spikes of a neuron are found one after another
+ * (after spike k the rest of its interval is tested again from v = 0).
+ *  t_in  [B, N_in, F_in]   spike times of each input, +inf = none (any order);
+ *  t_out [B, N_out, F_out] out: ascending, +inf after a neuron's last spike;
+ *  saved dstd_ms_saved_bytes(B, N_out, F_out) bytes (bin, current and dv^/dt
+ *        at every spike), written by the forward and read by the backward;
+ *  g_t_out [B, N_out, F_out] dC/dt_out (entries after the last spike ignored);
+ *  g_t_in  [B, N_in, F_in] out (may be NULL): dC/dt of every input spike, 0
+ *        for +inf entries; g_W [N_out, N_in] out (overwritten).
+ * Backward: the implicit function theorem per spike; spike k depends on w^
+ * both directly and through the spike k - 1 it was reset at, and the
+ * adjoints run from the last spike back to the first.
+ * 1 <= F_in, F_out <= 8 (DSTD_E_UNSUPPORTED above); tensor-core modes only
+ * (DSTD_MATH_F32 gives DSTD_E_UNSUPPORTED). The temporal and dead-neuron
+ * penalties are not defined for this regime: the params' penalty fields are
+ * not used. Other errors as dstd_dense_fwd / dstd_dense_bwd. */
+size_t dstd_ms_saved_bytes(int B, int N_out, int F_out);
+size_t dstd_ms_workspace_bytes(int B, int N_in, int N_out, int F_in, int F_out, const dstd_params *p,
+                               dstd_math math);
+int dstd_dense_fwd_ms(const float *t_in, const float *W, int B, int N_in, int N_out, int F_in, int F_out,
+                      const dstd_params *p, dstd_math math, float *t_out, void *saved, void *workspace,
+                      size_t ws_bytes, dstd_stream_t stream);
+int dstd_dense_bwd_ms(const float *t_in, const float *W, const float *t_out, const void *saved,
+                      const float *g_t_out, int B, int N_in, int N_out, int F_in, int F_out, const dstd_params *p,
+                      dstd_math math, float *g_t_in, float *g_W, void *workspace, size_t ws_bytes,
+                      dstd_stream_t stream);
+
 /* Skip-and-delay input of the paper's 20-layer network (App. C.3, Fig.
  * skip_connection: the third layer of a block also receives the block's input,
  * delayed by 2 tau_shift). Spike tensors are NHWC, so this is a concatenation

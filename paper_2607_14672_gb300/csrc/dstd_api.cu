@@ -1099,6 +1099,186 @@ int dstd_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
     return cu(launch_exact_fwd(t_in, W, B, N_in, N_out, c, p->t_end, (float)kmax, ws, t_out, (cudaStream_t)stream));
 }
 
+// ---------------------------------------------------------------------------
+// Multi-spike layers (App. D): the forward operands and the contraction of
+// the tensor-core modes, the scan with reset, and a backward whose dS is
+// stored (each input spike gathers its own two bins).
+// ---------------------------------------------------------------------------
+struct MsSaved {
+    int *q;
+    float *I, *vdot;
+};
+MsSaved ms_saved_view(void *saved, int B, int N_out, int F) {
+    Bump b(saved);
+    MsSaved v;
+    v.q = b.take<int>((size_t)B * N_out * F);
+    v.I = b.take<float>((size_t)B * N_out * F);
+    v.vdot = b.take<float>((size_t)B * N_out * F);
+    return v;
+}
+
+struct MsBwdWs {
+    __nv_bfloat16 *wt_hi = nullptr, *wt_lo = nullptr, *dA_hi = nullptr, *dA_lo = nullptr, *dB_hi = nullptr,
+                  *dB_lo = nullptr, *sT_hi = nullptr, *sT_lo = nullptr;
+    float *DS = nullptr;
+    int ldt = 0, ldn = 0, ldbm = 0, splits = 1;
+    size_t bytes = 0;
+};
+MsBwdWs ms_bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool need_gt) {
+    MsBwdWs w;
+    Bump b(base);
+    const long long cols = (long long)B * Mp;
+    const bool three = op == OpKind::BF16X3;
+    w.ldt = pad8(N_out);
+    w.ldn = pad8(N_out);
+    w.ldbm = pad8((int)cols);
+    w.splits = dw_splits(N_in, N_out, (int)cols, op);
+    w.dA_hi = b.take<__nv_bfloat16>((size_t)N_out * w.ldbm);
+    if (three) w.dA_lo = b.take<__nv_bfloat16>((size_t)N_out * w.ldbm);
+    w.sT_hi = b.take<__nv_bfloat16>((size_t)N_in * w.ldbm);
+    if (three) w.sT_lo = b.take<__nv_bfloat16>((size_t)N_in * w.ldbm);
+    if (need_gt) {
+        w.dB_hi = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
+        if (three) w.dB_lo = b.take<__nv_bfloat16>((size_t)cols * w.ldn);
+        w.wt_hi = b.take<__nv_bfloat16>((size_t)N_in * w.ldt);
+        if (three) w.wt_lo = b.take<__nv_bfloat16>((size_t)N_in * w.ldt);
+        w.DS = b.take<float>((size_t)N_in * cols);
+    }
+    w.bytes = b.off;
+    return w;
+}
+
+int check_ms(int F_in, int F_out, dstd_math math) {
+    if (F_in < 1 || F_out < 1) return DSTD_E_INVALID;
+    if (F_in > kMsMaxSpikes || F_out > kMsMaxSpikes) return DSTD_E_UNSUPPORTED;
+    if (math == DSTD_MATH_F32) return DSTD_E_UNSUPPORTED;
+    return DSTD_OK;
+}
+
+size_t dstd_ms_saved_bytes(int B, int N_out, int F_out) {
+    if (B < 1 || N_out < 1 || F_out < 1 || F_out > kMsMaxSpikes) return 0;
+    Bump b(nullptr);
+    b.take<int>((size_t)B * N_out * F_out);
+    b.take<float>((size_t)B * N_out * F_out);
+    b.take<float>((size_t)B * N_out * F_out);
+    return b.off;
+}
+
+size_t dstd_ms_workspace_bytes(int B, int N_in, int N_out, int F_in, int F_out, const dstd_params *p,
+                               dstd_math math) {
+    if (check_sizes(B, N_in, N_out) != DSTD_OK || check_params(p) != DSTD_OK) return 0;
+    if (check_ms(F_in, F_out, math) != DSTD_OK) return 0;
+    const int Mp = padded_M(p->M);
+    if (check_math(math, Mp) != DSTD_OK) return 0;
+    const size_t f = fwd_layout(nullptr, B, N_in, N_out, Mp, op_of(math), true).bytes;
+    const size_t g = ms_bwd_layout(nullptr, B, N_in, N_out, Mp, bwd_op_of(math), true).bytes;
+    return f > g ? f : g;
+}
+
+int dstd_dense_fwd_ms(const float *t_in, const float *W, int B, int N_in, int N_out, int F_in, int F_out,
+                      const dstd_params *p, dstd_math math, float *t_out, void *saved, void *workspace,
+                      size_t ws_bytes, dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    TRY(check_ms(F_in, F_out, math));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    const OpKind op = op_of(math);
+    if (ws_bytes < fwd_layout(nullptr, B, N_in, N_out, Mp, op, true).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    FwdWs ws = fwd_layout(workspace, B, N_in, N_out, Mp, op, true);
+    MsSaved sv = ms_saved_view(saved, B, N_out, F_out);
+    const long long cols = (long long)B * Mp;
+    {
+        Timed tm(KK_PREP, st);
+        if (op == OpKind::F16X3)
+            TRY(cu(launch_prep_weights_f16(W, N_out, N_in, (__half *)ws.w_hi, (__half *)ws.w_lo, ws.kpad,
+                                           ws.row_scale, ws.rowsum, st)));
+        else
+            TRY(cu(launch_prep_weights(W, N_out, N_in, op, (__nv_bfloat16 *)ws.w_hi, (__nv_bfloat16 *)ws.w_lo,
+                                       ws.kpad, nullptr, nullptr, 0, nullptr, 0, ws.rowsum, st)));
+    }
+    {
+        Timed tm(KK_BIN, st);
+        TRY(cu(launch_binning_ms(t_in, B, N_in, F_in, c, op, false, ws.s_hi, ws.s_lo, ws.kpad, st)));
+    }
+    {
+        const int splits = fwd_splits(N_out, cols, N_in);
+        if (splits > 1) TRY(cu(cudaMemsetAsync(ws.D, 0, sizeof(float) * (size_t)N_out * cols, st)));
+        TcEpiArgs a{};
+        a.row_scale = ws.row_scale;
+        a.D = ws.D;
+        a.ldd = cols;
+        a.atomic = splits > 1;
+        Timed tm(KK_GEMM_FWD, st);
+        TRY(cu(launch_tc_gemm(ws.w_hi, ws.w_lo, ws.kpad, ws.s_hi, ws.s_lo, ws.kpad, N_out, (int)cols, N_in, splits,
+                              op, Epi::Store, a, st)));
+    }
+    Timed tm(KK_SCAN, st);
+    return cu(launch_scan_ms(ws.D, Mp, cols, B, N_out, c, F_out, t_out, sv.q, sv.I, sv.vdot, st));
+}
+
+int dstd_dense_bwd_ms(const float *t_in, const float *W, const float *t_out, const void *saved,
+                      const float *g_t_out, int B, int N_in, int N_out, int F_in, int F_out, const dstd_params *p,
+                      dstd_math math, float *g_t_in, float *g_W, void *workspace, size_t ws_bytes,
+                      dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !saved || !g_W || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    TRY(check_ms(F_in, F_out, math));
+    const int Mp = padded_M(p->M);
+    TRY(check_math(math, Mp));
+    if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
+    const OpKind op = bwd_op_of(math);
+    const bool need_gt = g_t_in != nullptr;
+    if (ws_bytes < ms_bwd_layout(nullptr, B, N_in, N_out, Mp, op, need_gt).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, Mp);
+    cudaStream_t st = (cudaStream_t)stream;
+    MsBwdWs ws = ms_bwd_layout(workspace, B, N_in, N_out, Mp, op, need_gt);
+    MsSaved sv = ms_saved_view(const_cast<void *>(saved), B, N_out, F_out);
+    const long long cols = (long long)B * Mp;
+    {
+        Timed tm(KK_DWHAT, st);
+        TRY(cu(launch_dwhat_ms(t_out, sv.q, sv.I, sv.vdot, g_t_out, B, N_out, F_out, c, op, ws.dA_hi, ws.dA_lo,
+                               ws.ldbm, ws.dB_hi, ws.dB_lo, ws.ldn, st)));
+    }
+    if (need_gt) {
+        {
+            Timed tm(KK_PREP, st);
+            TRY(cu(launch_prep_weights(W, N_out, N_in, op, nullptr, nullptr, 0, ws.wt_hi, ws.wt_lo, ws.ldt, nullptr,
+                                       0, nullptr, st)));
+        }
+        {
+            // dS[j, (b, m)] = sum_i W_ij dw^_i(b, m), stored in fp32
+            TcEpiArgs a{};
+            a.D = ws.DS;
+            a.ldd = cols;
+            Timed tm(KK_GEMM_DS, st);
+            TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dB_hi, ws.dB_lo, ws.ldn, N_in, (int)cols, N_out, 1,
+                                  op, Epi::Store, a, st)));
+        }
+        Timed tm(KK_GT, st);
+        TRY(cu(launch_gt_ms(ws.DS, cols, t_in, B, N_in, F_in, c, g_t_in, st)));
+    }
+    {
+        Timed tm(KK_BIN_T, st);
+        TRY(cu(launch_binning_ms(t_in, B, N_in, F_in, c, op, true, ws.sT_hi, ws.sT_lo, ws.ldbm, st)));
+    }
+    TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)N_out * N_in, st)));
+    TcEpiArgs a{};
+    a.D = g_W;
+    a.ldd = N_in;
+    a.atomic = 1;
+    Timed tm(KK_GEMM_DW, st);
+    return cu(launch_tc_gemm(ws.dA_hi, ws.dA_lo, ws.ldbm, ws.sT_hi, ws.sT_lo, ws.ldbm, N_out, N_in, (int)cols,
+                             ws.splits, op, Epi::Store, a, st));
+}
+
 int dstd_set_pair_policy(int policy) {
     if (policy < 0 || policy > 2) return DSTD_E_INVALID;
     return tc_gemm_pair_policy(policy);

@@ -325,6 +325,18 @@ cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const
 constexpr int kGradtSmallMaxOut = 32;
 // The exact (event-driven) forward, Alg. 1, for comparison with DSTD: W^T,
 // the sorted inputs and their intervals in the workspace (exact_layout).
+// multi-spike regime (App. D): at most this many spikes per neuron, in and out
+constexpr int kMsMaxSpikes = 8;
+cudaError_t launch_binning_ms(const float *t, int B, int N, int F, const LifConst &c, OpKind op, bool transposed,
+                              void *hi, void *lo, int ld, cudaStream_t st);
+cudaError_t launch_scan_ms(const float *what, long long sb, long long si, int B, int N, const LifConst &c, int F,
+                           float *t_out, int *q, float *I, float *vd, cudaStream_t st);
+cudaError_t launch_dwhat_ms(const float *t_out, const int *q, const float *I, const float *vd, const float *g_up,
+                            int B, int N, int F, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda,
+                            void *b_hi, void *b_lo, int ldb, cudaStream_t st);
+cudaError_t launch_gt_ms(const float *D, long long ldd, const float *t_in, int B, int N, int F, const LifConst &c,
+                         float *g_t_in, cudaStream_t st);
+
 constexpr int kExactMaxIn = 8192;  // a sample's inputs are sorted in shared memory
 struct ExactWs {
     float *Wt = nullptr;       // [N_in][N_out]

@@ -23,7 +23,8 @@ EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd",
-           "dstd_exact_workspace_bytes", "dstd_exact_fwd", "dstd_concat_channels", "dstd_split_channels")
+           "dstd_exact_workspace_bytes", "dstd_exact_fwd", "dstd_concat_channels", "dstd_split_channels",
+           "dstd_ms_saved_bytes", "dstd_ms_workspace_bytes", "dstd_dense_fwd_ms", "dstd_dense_bwd_ms")
 
 
 class DstdError(RuntimeError):
@@ -98,6 +99,10 @@ def load(path=None):
         "dstd_conv_fwd": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _P, _SZ, _P]),
         "dstd_conv_bwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
         "dstd_concat_channels": (_I, [_P, _I, _F, _P, _I, _I64, _P, _P]),
+        "dstd_ms_saved_bytes": (_SZ, [_I, _I, _I]),
+        "dstd_ms_workspace_bytes": (_SZ, [_I, _I, _I, _I, _I, _PP, _I]),
+        "dstd_dense_fwd_ms": (_I, [_P, _P, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
+        "dstd_dense_bwd_ms": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _PP, _I, _P, _P, _P, _SZ, _P]),
         "dstd_split_channels": (_I, [_P, _I, _I, _I64, _P, _I, _P, _I, _P]),
     }
     for name, (res, args) in sig.items():
@@ -278,6 +283,35 @@ def ce_loss(t_L, labels, tau_soft, t_silent, loss, g_t_L, stream=None):
     _f32(t_L, "t_L")
     _check(load().dstd_ce_loss(_ptr(t_L), _ptr(labels), B, C, float(tau_soft), float(t_silent), _ptr(loss),
                                _ptr(g_t_L), _stream(stream)), "dstd_ce_loss")
+
+
+def ms_saved_bytes(B, N_out, F_out):
+    return load().dstd_ms_saved_bytes(B, N_out, F_out)
+
+
+def ms_workspace_bytes(B, N_in, N_out, F_in, F_out, p, math="x3"):
+    return load().dstd_ms_workspace_bytes(B, N_in, N_out, F_in, F_out, ctypes.byref(p), MATH[math])
+
+
+def dense_fwd_ms(t_in, W, p, math, t_out, saved, workspace, stream=None):
+    """Multi-spike layer forward: t_in [B, N_in, F_in] -> t_out [B, N_out, F_out]."""
+    B, N_in, F_in = t_in.shape
+    N_out, F_out = t_out.shape[1], t_out.shape[2]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(t_out, "t_out", (B, N_out, F_out))
+    _check(load().dstd_dense_fwd_ms(_ptr(t_in), _ptr(W), B, N_in, N_out, F_in, F_out, ctypes.byref(p), MATH[math],
+                                    _ptr(t_out), _ptr(saved), _ptr(workspace), workspace.numel(), _stream(stream)),
+           "dstd_dense_fwd_ms")
+
+
+def dense_bwd_ms(t_in, W, t_out, saved, g_t_out, p, math, g_t_in, g_W, workspace, stream=None):
+    """Multi-spike layer backward (g_t_in may be None)."""
+    B, N_in, F_in = t_in.shape
+    N_out, F_out = t_out.shape[1], t_out.shape[2]
+    _check(load().dstd_dense_bwd_ms(_ptr(t_in), _ptr(W), _ptr(t_out), _ptr(saved), _ptr(g_t_out), B, N_in, N_out,
+                                    F_in, F_out, ctypes.byref(p), MATH[math], _ptr(g_t_in), _ptr(g_W),
+                                    _ptr(workspace), workspace.numel(), _stream(stream)), "dstd_dense_bwd_ms")
 
 
 def concat_channels(a, b, delay_a, out, stream=None):
