@@ -41,8 +41,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5", "syn9", "syn20"],
-                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; syn9 / syn20: the paper's Syn-SNN-9 and Syn-SNN-20 (N = 64, batch 50, M = 20); cfg4 / cfg5: the 9- and 20-layer conv "
+    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5", "syn9", "syn20", "ms"],
+                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; syn9 / syn20: the paper's Syn-SNN-9 and Syn-SNN-20 (N = 64, batch 50, M = 20); ms: the multi-spike layer (App. D) against the first-spike layer of the same size; cfg4 / cfg5: the 9- and 20-layer conv "
                          "networks (bf16 operands), their training step timed the same way")
     ap.add_argument("--exact", action="store_true",
                     help="instead of the training step: time the exact (event-driven, Alg. 1) forward against the "
@@ -679,6 +679,92 @@ def run_cfg3(args, local):
     return 0 if status == 0 else 1
 
 
+def run_multispike(args, local):
+    """Multi-spike layers (App. D): forward + backward (with the input-time
+    gradient) of a dense layer whose inputs carry up to F spikes and whose
+    neurons fire up to F times, against the first-spike layer of the same
+    size; CUDA events around each pass, L2 flushed before each, per-kind
+    kernel times from the library's event timing."""
+    import numpy as np
+    import torch
+
+    from paper_2607_14672_gb300 import build as _b
+    _b.build()
+    from paper_2607_14672_gb300 import dstd, synth
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    reps = max(3, min(args.steps, 20))
+    out = []
+    for (B, N, M, F) in ((256, 800, 32, 4), (128, 4096, 32, 4)):
+        L = dict(tau_v=0.5, tau_I=0.25, v_th=1.0, t_first=0.0, t_end=1.2, M=M, t_offset=0.0)
+        p = dstd.params(L, 0.0)
+        t = np.sort(synth.uniform_spikes(0, (B, N, F), 0.0, 1.0, 0.25), axis=-1).astype(np.float32)
+        W = synth.normal_weights(1001, (N, N), 6.0 / N, 1.0 / math.sqrt(N)).astype(np.float32)
+        t_in = torch.tensor(t, device=dev)
+        Wd = torch.tensor(W, device=dev)
+        ws = torch.empty(dstd.ms_workspace_bytes(B, N, N, F, F, p, "x3"), dtype=torch.uint8, device=dev)
+        saved = torch.empty(dstd.ms_saved_bytes(B, N, F), dtype=torch.uint8, device=dev)
+        t_out = torch.empty(B, N, F, device=dev)
+        g_up = torch.ones(B, N, F, device=dev)
+        g_in = torch.empty_like(t_in)
+        g_W = torch.empty_like(Wd)
+        # the first-spike layer on the first spike of each input
+        t1 = t_in[..., 0].contiguous()
+        ws1 = torch.empty(dstd.dense_workspace_bytes(B, N, N, p, "x3"), dtype=torch.uint8, device=dev)
+        sv1 = torch.empty(dstd.dense_saved_bytes(B, N), dtype=torch.uint8, device=dev)
+        to1 = torch.empty(B, N, device=dev)
+        g1 = torch.ones(B, N, device=dev)
+        gi1 = torch.empty_like(t1)
+        pen = torch.empty(4, device=dev)
+        runs = {
+            "ms_fwd": lambda: dstd.dense_fwd_ms(t_in, Wd, p, "x3", t_out, saved, ws, stream),
+            "ms_bwd": lambda: dstd.dense_bwd_ms(t_in, Wd, t_out, saved, g_up, p, "x3", g_in, g_W, ws, stream),
+            "ttfs_fwd": lambda: dstd.dense_fwd(t1, Wd, p, "x3", to1, sv1, pen, ws1, stream),
+            "ttfs_bwd": lambda: dstd.dense_bwd(t1, Wd, to1, sv1, g1, p, "x3", gi1, g_W, ws1, stream),
+        }
+        ms = {}
+        with torch.cuda.stream(stream):
+            for k, fn in runs.items():
+                if k.endswith("bwd"):
+                    runs[k.replace("bwd", "fwd")]()
+                for _ in range(max(3, args.warmup)):
+                    fn()
+                ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+                for a, b in ev:
+                    flush.zero_()
+                    a.record(stream)
+                    fn()
+                    b.record(stream)
+                stream.synchronize()
+                ms[k] = float(np.median([a.elapsed_time(b) for a, b in ev]))
+        dstd.timing_enable(True)
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            runs["ms_fwd"]()
+            flush.zero_()
+            runs["ms_bwd"]()
+        kt = dstd.timing_read()
+        dstd.timing_enable(False)
+        runs["ms_fwd"]()
+        torch.cuda.synchronize()
+        n = torch.isfinite(t_out).sum(-1).float()
+        out.append({"B": B, "N_in": N, "N_out": N, "M": M, "F_in": F, "F_out": F, "ms": ms,
+                    "ms_over_ttfs_fwd_bwd": (ms["ms_fwd"] + ms["ms_bwd"]) / (ms["ttfs_fwd"] + ms["ttfs_bwd"]),
+                    "mean_spikes_per_neuron": float(n.mean()), "share_at_cap": float((n == F).float().mean()),
+                    "kernel_ms": {k: round(v[0], 4) for k, v in kt.items() if v[1] > 0}})
+    status = dstd.device_status(clear=True)
+    print(json.dumps({"metric": "multi-spike DSTD layer fwd+bwd time vs the first-spike layer, one GB300",
+                      "unit": "ms", "higher_is_better": False, "cases": out, "reps": reps,
+                      "config": {"workload": "dense LIF layer N->N, up to F spikes per input and per neuron "
+                                             "(reset v, keep I), tau=(0.5,0.25), x3",
+                                 "l2": "flushed before each timed pass"},
+                      "device_status": status}), flush=True)
+    return 0 if status == 0 else 1
+
+
 def run_exact_compare(args, local):
     """Exact forward (sort + interval sweep, Alg. 1) against the DSTD forward
     (binning, contraction, scan/solve) of the same layers on one GPU: device
@@ -754,6 +840,8 @@ def main():
         return run_exact_compare(args, local) if rank == 0 else 0
     if args.workload == "cfg3":
         return run_cfg3(args, local) if rank == 0 else 0
+    if args.workload == "ms":
+        return run_multispike(args, local) if rank == 0 else 0
     if args.workload != "cfg2":
         return run_conv(args, local) if rank == 0 else 0
     return run_ours(args, rank, world, local)
