@@ -60,6 +60,32 @@ def dist_env():
     return rank, world, local
 
 
+def rank_batch(cfg, rank):
+    """The synthetic batch of one rank: its own input and label seeds, so
+    that every replica trains on different data (weak scaling)."""
+    import numpy as np
+    from paper_2607_14672_gb300 import configs
+    t0 = np.asarray(cfg["inputs"](seed=configs.SEED_INPUT + rank), np.float32)
+    lab = cfg["labels"](seed=configs.SEED_LABELS + rank).astype(np.int32)
+    return t0, lab
+
+
+def max_over_ranks(ms, world, device=None):
+    """The slowest rank's step time (the job's step time)."""
+    if world == 1:
+        return float(ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world, per_rank_batch, ms):
+    """Samples per second of the whole job: every rank's batch per step time."""
+    return world * per_rank_batch / (ms / 1000.0)
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -336,8 +362,7 @@ def run_ours(args, rank, world, local):
     cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
     B = cfg["batch"]
     n = net.DenseNet(cfg, args.math, device=dev, with_adamw=True)
-    t0 = np.asarray(cfg["inputs"](seed=configs.SEED_INPUT + rank), np.float32)
-    lab = cfg["labels"](seed=configs.SEED_LABELS + rank).astype(np.int32)
+    t0, lab = rank_batch(cfg, rank)
     n.set_inputs(t0, lab)
     stream = torch.cuda.Stream(device=dev)
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > L2
@@ -384,11 +409,8 @@ def run_ours(args, rank, world, local):
     clk = clocks.stop()
     ms_steps = [a.elapsed_time(b) for a, b in ev]
     ms = sum(ms_steps) / len(ms_steps)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
-    value = world * B / (ms / 1000.0)
+    ms = max_over_ranks(ms, world, dev)
+    value = job_throughput(world, B, ms)
     status = dstd.device_status(clear=True)
     if args.profile:
         if rank == 0:
@@ -434,7 +456,7 @@ def run_ours(args, rank, world, local):
             stream.synchronize()
             _ = float(loss_h[0])
         e2e_ms = (time.perf_counter() - t_e) * 1000.0 / n_e2e
-    e2e = {"value": world * B / (e2e_ms / 1000.0), "unit": UNIT,
+    e2e = {"value": job_throughput(world, B, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": int(pin_t.numel() * 4 + pin_l.numel() * 4), "d2h_bytes_per_step": 4,
            "ms_per_step": e2e_ms, "path": "DenseNet.step captured in a CUDA graph, replayed per step"}
 
