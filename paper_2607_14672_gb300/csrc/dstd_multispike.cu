@@ -78,16 +78,41 @@ __global__ void k_binning_ms_rows(const float *__restrict__ t, int B, int N, int
     for (int m = 0; m < c.Mp; ++m) ms_store<OP>(hi, lo, ((long long)b * c.Mp + m) * ld + j, ms_value(c, bins, m));
 }
 
+// a warp per (input j, sample b): lane f < F discretises spike f, the warp
+// shares the results, and lane l writes bins l, l + 32, ... of the row
+// segment (contiguous: column b*Mp + m)
 template <int OP>
-__global__ void k_binning_ms_cols(const float *__restrict__ t, int B, int N, int F, LifConst c, void *hi, void *lo,
-                                  int ld) {
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= (long long)B * N) return;
-    const int j = (int)(idx / B), b = (int)(idx % B);  // consecutive threads: consecutive samples of one row
+__global__ void __launch_bounds__(256) k_binning_ms_cols(const float *__restrict__ t, int B, int N, int F, LifConst c,
+                                                         void *hi, void *lo, int ld) {
+    const int lane = threadIdx.x & 31;
+    const int j = blockIdx.x;
+    const int b = blockIdx.y * 8 + (threadIdx.x >> 5);
+    if (b >= B) return;
+    int kf = -100;
+    float wr = 0.f, wl = 0.f;
+    if (lane < F) {
+        const float x = t[((long long)b * N + j) * F + lane];
+        if (isfinite(x)) {
+            const BinW w = bin_weights(c, x, false);
+            kf = w.k;
+            wr = w.wR;
+            wl = w.wL;
+        }
+    }
     MsBins bins;
-    ms_bins(c, t + ((long long)b * N + j) * F, F, bins);
+    bins.n = 0;
+    for (int f = 0; f < F; ++f) {
+        const int k = __shfl_sync(0xffffffffu, kf, f);
+        const float r = __shfl_sync(0xffffffffu, wr, f), l = __shfl_sync(0xffffffffu, wl, f);
+        if (k != -100) {
+            bins.k[bins.n] = k;
+            bins.wR[bins.n] = r;
+            bins.wL[bins.n] = l;
+            ++bins.n;
+        }
+    }
     const long long o = (long long)j * ld + (long long)b * c.Mp;
-    for (int m = 0; m < c.Mp; ++m) ms_store<OP>(hi, lo, o + m, ms_value(c, bins, m));
+    for (int m = lane; m < c.Mp; m += 32) ms_store<OP>(hi, lo, o + m, ms_value(c, bins, m));
 }
 
 cudaError_t launch_binning_ms(const float *t, int B, int N, int F, const LifConst &c, OpKind op, bool transposed,
@@ -95,7 +120,8 @@ cudaError_t launch_binning_ms(const float *t, int B, int N, int F, const LifCons
     if (F < 1 || F > kMsMaxSpikes) return cudaErrorInvalidValue;
 #define DSTD_MS_BIN(OPV)                                                                                        \
     if (transposed)                                                                                             \
-        k_binning_ms_cols<OPV><<<ms_blocks((long long)B * N, 256), 256, 0, st>>>(t, B, N, F, c, hi, lo, ld);   \
+        k_binning_ms_cols<OPV><<<dim3((unsigned)N, (unsigned)((B + 7) / 8)), 256, 0, st>>>(t, B, N, F, c, hi,  \
+                                                                                           lo, ld);             \
     else                                                                                                        \
         k_binning_ms_rows<OPV><<<dim3((unsigned)((ld + 127) / 128), (unsigned)B), 128, 0, st>>>(t, B, N, F, c, \
                                                                                                 hi, lo, ld);
@@ -118,7 +144,7 @@ cudaError_t launch_binning_ms(const float *t, int B, int N, int F, const LifCons
 // t = +inf, q = M after the last spike.
 __global__ void __launch_bounds__(256) k_scan_ms(const float *__restrict__ what, long long sb, long long si, int B,
                                                  int N, LifConst c, int F, float *t_out, int *q_out, float *I_out,
-                                                 float *vd_out) {
+                                                 float *vd_out, int vec4) {
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)B * N) return;
     const int b = (int)(idx / N), i = (int)(idx % N);
@@ -126,8 +152,26 @@ __global__ void __launch_bounds__(256) k_scan_ms(const float *__restrict__ what,
     float v = 0.f, I = 0.f;
     int nk = 0;
     const long long o = idx * F;
+    float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int m = 0; m < c.M && nk < F; ++m) {
-        float v0 = v, I0 = I + w[m];
+        if (vec4) {
+            if ((m & 3) == 0) w4 = __ldg(reinterpret_cast<const float4 *>(w + m));
+        }
+        const float wm = vec4 ? ((m & 3) == 0 ? w4.x : (m & 3) == 1 ? w4.y : (m & 3) == 2 ? w4.z : w4.w) : w[m];
+        float v0 = v, I0 = I + wm;
+        // a whole interval with no spike in it yet: the cheap tests of the
+        // first-spike scan decide whether the exact test is needed
+        {
+            const float ve = fmaf(c.KD, I0, c.rv * v0);
+            const bool endp = ve >= c.vth;
+            const bool peak = (fmaf(-c.av, v0, I0) > 0.0f) & (fmaf(-c.av, ve, c.rI * I0) < 0.0f) &
+                              (fmaf(fmaxf(I0, 0.0f), c.Kmax, fmaxf(v0, 0.0f)) >= c.vth);
+            if (!(endp | peak)) {
+                v = ve;
+                I = c.rI * I0;
+                continue;
+            }
+        }
         float L = c.dt, start = c.T0 + (float)m * c.dt;
         // at most F spikes in all, so the inner loop ends
         while (nk < F) {
@@ -164,7 +208,9 @@ __global__ void __launch_bounds__(256) k_scan_ms(const float *__restrict__ what,
 cudaError_t launch_scan_ms(const float *what, long long sb, long long si, int B, int N, const LifConst &c, int F,
                            float *t_out, int *q, float *I, float *vd, cudaStream_t st) {
     if (F < 1 || F > kMsMaxSpikes) return cudaErrorInvalidValue;
-    k_scan_ms<<<ms_blocks((long long)B * N, 256), 256, 0, st>>>(what, sb, si, B, N, c, F, t_out, q, I, vd);
+    // 16-byte loads when every row of bins starts on a 16-byte boundary
+    const int vec4 = (sb % 4 == 0) && (si % 4 == 0) && (reinterpret_cast<uintptr_t>(what) % 16 == 0) && (c.Mp % 4 == 0);
+    k_scan_ms<<<ms_blocks((long long)B * N, 256), 256, 0, st>>>(what, sb, si, B, N, c, F, t_out, q, I, vd, vec4);
     return cudaGetLastError();
 }
 
@@ -176,59 +222,94 @@ cudaError_t launch_scan_ms(const float *what, long long sb, long long si, int B,
 //             dt_k/dt_{k-1} = -I_{k-1} [(av - aI) K(s) - e^{-aI s}] / v'_k, s = t_k - t_{k-1}
 // (the current kept through the reset decays at aI; dK/ds = -av K + e^{-aI s}).
 // The adjoints a_k = dC/dt_k + a_{k+1} dt_{k+1}/dt_k run from the last
-// spike back; dC/dw^_m = sum_k a_k dt_k/dw^_m. Writes the (i, (b, m)) layout
-// and the ((b, m), i) one (row stride ldb), zero after the last spike.
+// spike back; dC/dw^_m = sum_k a_k dt_k/dw^_m.
+//
+// A block takes 32 neurons of one sample: thread i < 32 runs neuron i's
+// adjoints into shared memory, the block fills a [Mp][32] tile of dC/dw^
+// (zero after a neuron's last spike), and writes it to both layouts with
+// contiguous stores: the (i, (b, m)) rows (a warp per neuron, lanes over m)
+// and, when b_hi is given, the ((b, m), i) rows (lanes over the 32 neurons).
+constexpr int MS_DW_NEURONS = 32;
 template <int OP>
 __global__ void __launch_bounds__(256) k_dwhat_ms(const float *__restrict__ t_out, const int *__restrict__ qv,
                                                   const float *__restrict__ Iv, const float *__restrict__ vdv,
                                                   const float *__restrict__ g_up, int B, int N, int F, LifConst c,
                                                   void *a_hi, void *a_lo, int lda, void *b_hi, void *b_lo, int ldb) {
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= (long long)B * N) return;
-    const int b = (int)(idx / N), i = (int)(idx % N);
-    const long long o = idx * F;
-    float tk[kMsMaxSpikes], Ik[kMsMaxSpikes], coef[kMsMaxSpikes];
-    int qk[kMsMaxSpikes];
-    int n = 0;
-    for (int k = 0; k < F; ++k) {
-        if (qv[o + k] >= c.M) break;
-        tk[k] = t_out[o + k];
-        qk[k] = qv[o + k];
-        Ik[k] = Iv[o + k];
-        coef[k] = g_up ? g_up[o + k] : 0.f;
-        n = k + 1;
-    }
-    // adjoints, last spike first; coef_k = -a_k / v'_k
-    for (int k = n - 1; k >= 0; --k) {
-        const float vd = vdv[o + k];
-        coef[k] = -coef[k] / vd;
-        if (k > 0) {
-            const float s = tk[k] - tk[k - 1];
-            const float dv_dprev = Ik[k - 1] * fmaf(c.av - c.aI, kernel_K(c, s), -expf(-c.aI * s));
-            coef[k - 1] += coef[k] * dv_dprev;  // a_{k-1} += a_k (-dv_dprev / v'_k)
-        }
-    }
-    // the shared factor of spike k >= 1 over the bins before spike k - 1
-    float Kk[kMsMaxSpikes];
-    for (int k = 1; k < n; ++k) Kk[k] = kernel_K(c, tk[k] - tk[k - 1]);
-    const int last = n > 0 ? qk[n - 1] : -1;
-    const long long oa = (long long)i * lda + (long long)b * c.Mp;
-    for (int m = 0; m < c.Mp; ++m) {
-        float val = 0.f;
-        if (m <= last) {
-            const float Tm = c.T0 + (float)m * c.dt;
+    extern __shared__ __align__(16) float dsm[];
+    float *tile = dsm;                                        // [Mp][33]
+    float *stk = tile + c.Mp * (MS_DW_NEURONS + 1);           // [32][F] spike times
+    float *scf = stk + MS_DW_NEURONS * F;                     // [32][F] coefficients -a_k / v'_k
+    float *sKk = scf + MS_DW_NEURONS * F;                     // [32][F] K(t_k - t_{k-1})
+    int *sq = reinterpret_cast<int *>(sKk + MS_DW_NEURONS * F);  // [32][F] bins
+    int *sn = sq + MS_DW_NEURONS * F;                         // [32] spike counts
+    const int b = blockIdx.y;
+    const int i0 = blockIdx.x * MS_DW_NEURONS;
+    const int tid = threadIdx.x;
+    if (tid < MS_DW_NEURONS) {
+        const int i = i0 + tid;
+        int n = 0;
+        if (i < N) {
+            const long long o = ((long long)b * N + i) * F;
+            float tk[kMsMaxSpikes], Ik[kMsMaxSpikes], coef[kMsMaxSpikes];
+            for (int k = 0; k < F; ++k) {
+                if (qv[o + k] >= c.M) break;
+                tk[k] = t_out[o + k];
+                Ik[k] = Iv[o + k];
+                coef[k] = g_up ? g_up[o + k] : 0.f;
+                sq[tid * F + k] = qv[o + k];
+                n = k + 1;
+            }
+            // adjoints, last spike first; coef_k = -a_k / v'_k
+            for (int k = n - 1; k >= 0; --k) {
+                coef[k] = -coef[k] / vdv[o + k];
+                if (k > 0) {
+                    const float s = tk[k] - tk[k - 1];
+                    const float dv_dprev = Ik[k - 1] * fmaf(c.av - c.aI, kernel_K(c, s), -expf(-c.aI * s));
+                    coef[k - 1] += coef[k] * dv_dprev;  // a_{k-1} += a_k (-dv_dprev / v'_k)
+                }
+            }
             for (int k = 0; k < n; ++k) {
-                if (m > qk[k]) continue;
-                float basis;
-                if (k > 0 && m <= qk[k - 1])
-                    basis = expf(-c.aI * (tk[k - 1] - Tm)) * Kk[k];
-                else
-                    basis = kernel_K(c, tk[k] - Tm);
-                val = fmaf(coef[k], basis, val);
+                stk[tid * F + k] = tk[k];
+                scf[tid * F + k] = coef[k];
+                sKk[tid * F + k] = k > 0 ? kernel_K(c, tk[k] - tk[k - 1]) : 0.f;
             }
         }
-        ms_store<OP>(a_hi, a_lo, oa + m, val);
-        if (b_hi) ms_store<OP>(b_hi, b_lo, ((long long)b * c.Mp + m) * ldb + i, val);
+        sn[tid] = n;
+    }
+    __syncthreads();
+    // the tile: thread (neuron il, bins m = row, row + 8, ...)
+    for (int e = tid; e < c.Mp * MS_DW_NEURONS; e += blockDim.x) {
+        const int il = e % MS_DW_NEURONS, m = e / MS_DW_NEURONS;
+        const int n = sn[il];
+        float val = 0.f;
+        if (n > 0 && m <= sq[il * F + n - 1]) {
+            const float Tm = c.T0 + (float)m * c.dt;
+            for (int k = 0; k < n; ++k) {
+                const int qk = sq[il * F + k];
+                if (m > qk) continue;
+                float basis;
+                if (k > 0 && m <= sq[il * F + k - 1])
+                    basis = expf(-c.aI * (stk[il * F + k - 1] - Tm)) * sKk[il * F + k];
+                else
+                    basis = kernel_K(c, stk[il * F + k] - Tm);
+                val = fmaf(scf[il * F + k], basis, val);
+            }
+        }
+        tile[m * (MS_DW_NEURONS + 1) + il] = val;
+    }
+    __syncthreads();
+    const int lane = tid & 31, warp = tid >> 5;
+    for (int il = warp; il < MS_DW_NEURONS; il += blockDim.x / 32) {
+        const int i = i0 + il;
+        if (i >= N) break;
+        const long long oa = (long long)i * lda + (long long)b * c.Mp;
+        for (int m = lane; m < c.Mp; m += 32) ms_store<OP>(a_hi, a_lo, oa + m, tile[m * (MS_DW_NEURONS + 1) + il]);
+    }
+    if (b_hi) {
+        const int i = i0 + lane;
+        if (i < N)
+            for (int m = warp; m < c.Mp; m += blockDim.x / 32)
+                ms_store<OP>(b_hi, b_lo, ((long long)b * c.Mp + m) * ldb + i, tile[m * (MS_DW_NEURONS + 1) + lane]);
     }
 }
 
@@ -236,13 +317,14 @@ cudaError_t launch_dwhat_ms(const float *t_out, const int *q, const float *I, co
                             int B, int N, int F, const LifConst &c, OpKind op, void *a_hi, void *a_lo, int lda,
                             void *b_hi, void *b_lo, int ldb, cudaStream_t st) {
     if (F < 1 || F > kMsMaxSpikes) return cudaErrorInvalidValue;
-    const unsigned g = ms_blocks((long long)B * N, 256);
+    const size_t smem = sizeof(float) * ((size_t)c.Mp * (MS_DW_NEURONS + 1) + 4 * MS_DW_NEURONS * F + MS_DW_NEURONS);
+    const dim3 g((unsigned)((N + MS_DW_NEURONS - 1) / MS_DW_NEURONS), (unsigned)B);
     if (op == OpKind::F32)
-        k_dwhat_ms<0><<<g, 256, 0, st>>>(t_out, q, I, vd, g_up, B, N, F, c, a_hi, a_lo, lda, b_hi, b_lo, ldb);
+        k_dwhat_ms<0><<<g, 256, smem, st>>>(t_out, q, I, vd, g_up, B, N, F, c, a_hi, a_lo, lda, b_hi, b_lo, ldb);
     else if (op == OpKind::BF16X3)
-        k_dwhat_ms<1><<<g, 256, 0, st>>>(t_out, q, I, vd, g_up, B, N, F, c, a_hi, a_lo, lda, b_hi, b_lo, ldb);
+        k_dwhat_ms<1><<<g, 256, smem, st>>>(t_out, q, I, vd, g_up, B, N, F, c, a_hi, a_lo, lda, b_hi, b_lo, ldb);
     else
-        k_dwhat_ms<2><<<g, 256, 0, st>>>(t_out, q, I, vd, g_up, B, N, F, c, a_hi, a_lo, lda, b_hi, b_lo, ldb);
+        k_dwhat_ms<2><<<g, 256, smem, st>>>(t_out, q, I, vd, g_up, B, N, F, c, a_hi, a_lo, lda, b_hi, b_lo, ldb);
     return cudaGetLastError();
 }
 
