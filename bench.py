@@ -44,6 +44,8 @@ def parse():
     ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5", "syn9", "syn20", "ms"],
                     help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; syn9 / syn20: the paper's Syn-SNN-9 and Syn-SNN-20 (N = 64, batch 50, M = 20); ms: the multi-spike layer (App. D) against the first-spike layer of the same size; cfg4 / cfg5: the 9- and 20-layer conv "
                          "networks (bf16 operands), their training step timed the same way")
+    ap.add_argument("--cfg3-cases", default="4096:32:x3,16384:32:x3,16384:128:x3,16384:128:bf16",
+                    help="with --workload cfg3: the (N:M:math) cases to run, comma-separated")
     ap.add_argument("--exact", action="store_true",
                     help="instead of the training step: time the exact (event-driven, Alg. 1) forward against the "
                          "DSTD forward on the same GPU, per layer shape, and print one JSON line")
@@ -626,7 +628,7 @@ def run_cfg3(args, local):
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     stream = torch.cuda.Stream(device=dev)
     pk, pk_src = peaks()
-    cases = [(4096, 32, "x3"), (16384, 32, "x3"), (16384, 128, "x3"), (16384, 128, "bf16")]
+    cases = [(int(n), int(m), mm) for n, m, mm in (c.split(":") for c in args.cfg3_cases.split(","))]
     steps = max(2, min(args.steps, 20))
     clocks = ClockSampler(local)
     clocks.start()
