@@ -106,6 +106,21 @@ def test_null_and_bad_arguments_rejected_on_host(lib):
                           ctypes.c_float(1e-8), ctypes.c_float(0.0), 0, None) == -1
     # contraction scheduling policy: 0, 1, 2 valid (previous returned), anything else rejected
     assert lib.dstd_set_pair_policy(3) == -1 and lib.dstd_set_pair_policy(-1) == -1
+    # multi-spike layers: spike counts 1..8, tensor-core modes only, checked before any device call
+    ms_args = lambda Fi, Fo, math: (one, one, 8, 16, 16, Fi, Fo, p, math, one, one, one, 1 << 30, None)
+    assert lib.dstd_dense_fwd_ms(*ms_args(0, 2, 1)) == -1
+    assert lib.dstd_dense_fwd_ms(*ms_args(2, 0, 1)) == -1
+    assert lib.dstd_dense_fwd_ms(*ms_args(9, 2, 1)) == -2
+    assert lib.dstd_dense_fwd_ms(*ms_args(2, 9, 1)) == -2
+    assert lib.dstd_dense_fwd_ms(*ms_args(2, 2, 0)) == -2                     # fp32 CUDA-core mode
+    assert lib.dstd_dense_bwd_ms(one, one, one, one, one, 8, 16, 16, 2, 9, p, 1, None, one, one, 1 << 30,
+                                 None) == -2
+    assert lib.dstd_dense_bwd_ms(one, one, one, one, one, 8, 16, 16, 2, 2, p, 1, None, None, one, 1 << 30,
+                                 None) == -1                                   # no g_W
+    assert lib.dstd_ms_saved_bytes(8, 16, 0) == 0 and lib.dstd_ms_saved_bytes(8, 16, 9) == 0
+    assert lib.dstd_ms_saved_bytes(8, 16, 3) >= 8 * 16 * 3 * 12
+    assert lib.dstd_ms_workspace_bytes(8, 16, 16, 2, 2, p, 0) == 0
+    assert lib.dstd_ms_workspace_bytes(8, 16, 16, 2, 2, p, 1) > 0
     # skip-and-delay channel concatenation and its adjoint
     assert lib.dstd_concat_channels(None, 4, ctypes.c_float(0.2), one, 4, 10, one, None) == -1
     assert lib.dstd_concat_channels(one, 0, ctypes.c_float(0.2), one, 4, 10, one, None) == -1
