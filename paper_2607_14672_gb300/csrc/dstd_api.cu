@@ -324,6 +324,26 @@ int dw_splits(int N_in, int N_out, int K, OpKind op) {
     return best;
 }
 
+// whether dW runs on SM pairs (transposed, no split-K) rather than on
+// single CTAs with the split-K factor of dw_splits: the same cost units as
+// both (rounds of work x K slices per item, plus fill and drain), with the
+// pair's 256 x 128 tiles, resident pairs and a pair K slice at 0.92 of a
+// single CTA's (measured); the scheduling policy can force either
+bool dw_on_pairs(int N_in, int N_out, int K, OpKind op) {
+    const int policy = tc_gemm_pair_policy(-1);
+    if (policy == 1) return true;
+    if (policy == 2) return false;
+    const int s = dw_splits(N_in, N_out, K, op);
+    const long long kt = (K + 63) / 64;
+    const long long tiles = (long long)((N_out + 127) / 128) * ((N_in + 127) / 128);
+    const double single = (double)((tiles * s + 151) / 152) * (double)((kt + s - 1) / s + 2);
+    const long long pairs = tc_gemm_resident_pairs(op);
+    if (pairs < 1) return false;
+    const long long t2 = (long long)((N_in + 255) / 256) * ((N_out + 127) / 128);
+    const double pair = (double)((t2 + pairs - 1) / pairs) * (0.92 * (double)kt + 4.0);
+    return pair < single;
+}
+
 BwdWs bwd_layout(void *base, int B, int N_in, int N_out, int Mp, OpKind op, bool need_gt) {
     BwdWs w;
     Bump b(base);
@@ -841,6 +861,21 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
         // dw^ read transposed from its dW layout [N_out, B*Mp]
         TRY(cu(launch_tc_gemm(ws.wt_hi, ws.wt_lo, ws.ldt, ws.dA_hi, ws.dA_lo, ws.ldbm, N_in, (int)cols, N_out, 1, op,
                               Epi::GradT, a, st, true)));
+    }
+    if (dw_on_pairs(N_in, N_out, (int)cols, op)) {
+        // on SM pairs, computed transposed: (s^T dw^)[j, i] stored as dW[i][j];
+        // then the dead-neuron term qcoef * count_i added in place
+        TcEpiArgs a{};
+        a.D = g_W;
+        a.ldd = N_in;
+        {
+            Timed tm(KK_GEMM_DW, st);
+            TRY(cu(launch_tc_gemm_pair_storeT(ws.sT_hi, ws.sT_lo, ws.ldbm, ws.dA_hi, ws.dA_lo, ws.ldbm, N_in, N_out,
+                                              (int)cols, op, a, st)));
+        }
+        if (qcoef == 0.0f) return DSTD_OK;
+        Timed tm(KK_REDUCE, st);
+        return cu(launch_dw_reduce(g_W, 1, 0, N_in, N_out, N_in, ws.count, qcoef, g_W, st, false));
     }
     // dW = dw^T s: the split-K slices add into g_W (zeroed above); split 0
     // also adds the dead-neuron term qcoef * count_i

@@ -1017,7 +1017,7 @@ bool tc_gemm_pair_preferred(int R, int Cn, int K, OpKind op) {
     if (op != OpKind::F16X3 && op != OpKind::BF16) return false;
     const int policy = g_pair_policy.load();
     if (policy != 0) return policy == 1;
-    const int pairs = op == OpKind::F16X3 ? tc::resident_pairs<3, true>() : tc::resident_pairs<1, false>();
+    const int pairs = tc_gemm_resident_pairs(op);
     if (pairs < 1) return false;
     const long long t1 = (long long)((R + 127) / 128) * ((Cn + 127) / 128);
     const long long t2 = (long long)((R + 255) / 256) * ((Cn + 127) / 128);
@@ -1027,7 +1027,9 @@ bool tc_gemm_pair_preferred(int R, int Cn, int K, OpKind op) {
 }
 
 int tc_gemm_resident_pairs(OpKind op) {
-    return op == OpKind::F16X3 ? tc::resident_pairs<3, true>() : tc::resident_pairs<1, false>();
+    return op == OpKind::F16X3    ? tc::resident_pairs<3, true>()
+           : op == OpKind::BF16X3 ? tc::resident_pairs<3, false>()
+                                  : tc::resident_pairs<1, false>();
 }
 
 cudaError_t launch_tc_gemm_pair_storeT(const void *A_hi, const void *A_lo, int lda, const void *B_hi, const void *B_lo,
@@ -1036,13 +1038,14 @@ cudaError_t launch_tc_gemm_pair_storeT(const void *A_hi, const void *A_lo, int l
     CUtensorMap a_hi, a_lo, b_hi, b_lo;
     const bool three = (op == OpKind::BF16X3 || op == OpKind::F16X3);
     const bool f16 = (op == OpKind::F16X3);
-    if (op == OpKind::F32 || op == OpKind::BF16X3) return cudaErrorInvalidValue;
+    if (op == OpKind::F32) return cudaErrorInvalidValue;
     if (!tc::make_map(&a_hi, A_hi, R, K, lda, tc::BM2, f16) || !tc::make_map(&b_hi, B_hi, Cn, K, ldb, tc::BNH, f16))
         return cudaErrorInvalidValue;
     if (three) {
         if (!tc::make_map(&a_lo, A_lo, R, K, lda, tc::BM2, f16) || !tc::make_map(&b_lo, B_lo, Cn, K, ldb, tc::BNH, f16))
             return cudaErrorInvalidValue;
-        return tc::launch_pair<3, true>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, args, st);
+        return f16 ? tc::launch_pair<3, true>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, args, st)
+                   : tc::launch_pair<3, false>(a_hi, a_lo, b_hi, b_lo, R, Cn, K, args, st);
     }
     a_lo = a_hi;
     b_lo = b_hi;

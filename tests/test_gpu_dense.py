@@ -406,6 +406,41 @@ def test_output_layer_with_fused_loss(math_mode, B, N_in, N_out):
     np.testing.assert_allclose(host(g), host(g_ref), rtol=1e-5, atol=2e-6 / (0.02 * B))
 
 
+@pytest.mark.parametrize("math_mode", ["x3", "bf16"])
+def test_backward_dW_on_sm_pairs_matches_single_ctas(math_mode, pair_policy):
+    """dW on SM pairs (computed transposed, s^T dw^, stored as dW, with the
+    dead-neuron term added afterwards) against the single-CTA split-K
+    contraction and the oracle; 140 inputs and 150 outputs are not multiples
+    of the 256 x 128 pair tile."""
+    from paper_2607_14672_gb300 import dstd
+    t_in, layer = dense_layer(24, 140, 150, 32, 0.5, 0.25, seed=17, t_offset=0.007,
+                              gammas=(0.05, 0.01, 1e-3), edges=(0.35, 0.8), fire=0.6)
+    t_in, layer["W"] = f32(t_in), f32(layer["W"])
+    t_in = _drop_ill_conditioned(t_in, layer)
+    B = t_in.shape[0]
+    out = {}
+    for policy in (1, 2):
+        pair_policy(policy)
+        r = run_fwd(t_in, layer, math_mode)
+        ctx = oracle_forward(t_in, layer["W"], layer)
+        gup = np.where(np.isfinite(ctx["t"]) & np.isfinite(r["t"]), 1.0, 0.0)
+        g_W = torch.empty(150, 140, device="cuda")
+        dstd.dense_bwd(r["t_dev"], r["W_dev"], r["t_out_dev"], r["saved"], dev(gup), r["p"], math_mode, None, g_W,
+                       r["ws"])
+        torch.cuda.synchronize()
+        assert dstd.device_status(clear=True) == 0
+        out[policy] = (host(g_W), gup, ctx, r)
+    assert rel_l2(out[1][0], out[2][0]) <= (1e-5 if math_mode == "x3" else 2e-2)
+    if math_mode == "x3":
+        gW, gup, ctx, r = out[1]
+        _, gT = olosses.temporal_penalty(ctx["t"], 0.35, 0.8, 0.05, 0.01, 1.0 / B)
+        gW_ref, _, _ = odstd.backward_dense(ctx, t_in, layer["W"], gup + np.where(np.isfinite(ctx["t"]), gT, 0.0),
+                                            ctx["T"], ctx["dt"], 0.5, 0.25, 1.0)
+        _, cnt = olosses.dead_neuron_penalty(ctx["t"], layer["W"].sum(1), 1e-3, 1.0 / B)
+        gW_ref = gW_ref - 1e-3 / B * cnt[:, None]
+        assert rel_l2(gW, gW_ref) <= 1e-3
+
+
 def test_backward_without_input_gradient():
     from paper_2607_14672_gb300 import dstd
     t_in, layer = dense_layer(8, 64, 96, 16, 0.5, 0.25, seed=23)
