@@ -549,6 +549,10 @@ def run_conv(args, local):
     stream = torch.cuda.Stream(device=dev)
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     with torch.cuda.stream(stream):
+        # silent share per layer at initialisation (before any optimizer step)
+        n.forward()
+        stream.synchronize()
+        dead_init = [float(x) for x in n.dead_fraction()]
         for _ in range(max(1, args.warmup)):
             n.step()
         stream.synchronize()
@@ -604,7 +608,10 @@ def run_conv(args, local):
                    "note": "whole step: every kernel's time in the denominator, the contractions' padded dense "
                            "flops in the numerator"},
         "kernel_ms": {k: round(v[0] / 2, 4) for k, v in kt.items() if v[1] > 0},
-        "dead_fraction_per_layer": dead, "clocks": clk, "device_status": status}), flush=True)
+        "dead_fraction_per_layer": {"at_init": dead_init, "after_steps": dead,
+                                    "note": "after_steps follows the warm-up and timed steps, each with an AdamW "
+                                            "update on random labels"},
+        "clocks": clk, "device_status": status}), flush=True)
     return 0 if status == 0 else 1
 
 
