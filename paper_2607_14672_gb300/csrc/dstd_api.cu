@@ -333,6 +333,7 @@ bool dw_on_pairs(int N_in, int N_out, int K, OpKind op) {
     const int policy = tc_gemm_pair_policy(-1);
     if (policy == 1) return true;
     if (policy == 2) return false;
+    if (N_in < 256 || N_out < 256) return false;  // a narrow side leaves the pair's 256 x 128 tiles mostly padding
     const int s = dw_splits(N_in, N_out, K, op);
     const long long kt = (K + 63) / 64;
     const long long tiles = (long long)((N_out + 127) / 128) * ((N_in + 127) / 128);
