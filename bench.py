@@ -1,18 +1,25 @@
 #!/usr/bin/env python
 """Benchmark: DSTD LIF forward+backward samples/s on one GB300.
 
-Workload (default): the 3-layer dense TTFS MLP 784-800-800-10, batch 256,
-M = 32 DSTD steps, (tau_m, tau_s) = (0.5, 0.25), synfire windows, CE + T +
-gamma_Q Q; one step = forward of all layers, loss, backward of all layers
+Workload (default): the 20-layer convolutional TTFS SNN on 28x28x1 inputs
+(19 3x3 conv layers with 64/128/256 channels, stride 2 at layers 7 and 14,
+a dense 12544 -> 10 readout), batch 256, M = 64 DSTD steps, (tau_m, tau_s) =
+(1.0, 0.25), staggered synfire windows, CE + T + gamma_Q Q, bf16 contraction
+operands with fp32 accumulation and state. One step = forward of every
+layer, loss, backward of every layer and one AdamW update of every weight
 (the whole hot path: binning, contraction, scan/solve/select, dw^, both
-backward contractions). Synthetic seeded inputs of the shape of 28x28
-images (60% zero pixels, t = 1 - x); random-init weights of that
-architecture. L2 (129 MB) is flushed before every timed step.
+backward contractions with the input-time gradient). Synthetic seeded inputs
+of the shape of 28x28 intensity maps (t = 1 - x); random-init weights of
+that architecture with calibrated means. The weights and optimizer state
+are put back to their initial values before every timed step (outside the
+timed region), so every step trains the calibrated network. L2 (129 MB) is
+flushed before every timed step.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload cfg5|cfg4|syn9|syn20|cfg2|cfg3|ms] [--exact]
 
 One JSON line on stdout (rank 0). ``--impl reference`` times the float64
-CPU oracle on the host cores instead.
+CPU oracle on the host cores instead (one layer shape per step).
 """
 
 import argparse
@@ -24,25 +31,28 @@ import sys
 import threading
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "DSTD LIF fwd+bwd samples/s at 1 GB300; % of tensor/HBM roofline; peak mem"
 UNIT = "samples/s"
 WORKLOAD = "dense LIF TTFS MLP 784-800-800-10, B=256, M=32, tau=(0.5,0.25), synfire CE+T+Q, fwd+bwd+AdamW"
+CONV_WORKLOADS = ("cfg4", "cfg5", "syn9", "syn20")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"])
+    ap.add_argument("--math", default="x3", choices=["x3", "bf16", "f32"], help="contraction mode of --workload cfg2")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="cfg2", choices=["cfg2", "cfg3", "cfg4", "cfg5", "syn9", "syn20", "ms"],
-                    help="cfg2: the 784-800-800-10 MLP (the headline line); cfg3: one N->N layer at several (N, M), per-kernel rooflines; syn9 / syn20: the paper's Syn-SNN-9 and Syn-SNN-20 (N = 64, batch 50, M = 20); ms: the multi-spike layer (App. D) against the first-spike layer of the same size; cfg4 / cfg5: the 9- and 20-layer conv "
+    ap.add_argument("--workload", default="cfg5", choices=["cfg2", "cfg3", "cfg4", "cfg5", "syn9", "syn20", "ms"],
+                    help="cfg5: the 20-layer conv network (the headline line); cfg2: the 784-800-800-10 MLP; cfg3: one N->N layer at several (N, M), per-kernel rooflines; syn9 / syn20: the paper's Syn-SNN-9 and Syn-SNN-20 (N = 64, batch 50, M = 20); ms: the multi-spike layer (App. D) against the first-spike layer of the same size; cfg4 / cfg5: the 9- and 20-layer conv "
                          "networks (bf16 operands), their training step timed the same way")
     ap.add_argument("--cfg3-cases", default="4096:32:x3,16384:32:x3,16384:128:x3,16384:128:bf16",
                     help="with --workload cfg3: the (N:M:math) cases to run, comma-separated")
@@ -160,29 +170,208 @@ def oracle_throughput(samples_per_worker=8, max_workers=16):
 
 
 def run_reference(args, rank):
+    """The float64 oracle on the host cores, on the same workload and metric."""
     if rank != 0:
         return 0
+    if args.workload in CONV_WORKLOADS:
+        return run_reference_conv(args)
     t_all = time.perf_counter()
     pool = OraclePool()
     per = 2
-    tot_n, tot_t = 0, 0.0
+    tot_n, tot_t, walls = 0, 0.0, []
     try:
         for k in range(args.warmup + args.steps):
+            t_s = time.perf_counter()
             n, wall = pool.run(per)
             if k >= args.warmup:
                 tot_n += n
                 tot_t += wall
+                walls.append(time.perf_counter() - t_s)
     finally:
         pool.close()
     v = tot_n / tot_t
-    ms = 256 / v * 1000.0
+    ms = 1000.0 * sum(walls) / len(walls)
     base = {"value": v, "unit": UNIT, "cores": pool.workers, "kind": "oracle",
             "sample": f"each step {per * pool.workers} of the 256 samples ({per} per worker), float64 NumPy fwd+bwd"
-                      f" of all 3 layers + CE/T/Q on {pool.workers} spawned single-threaded workers"}
+                      f" of all 3 layers + CE/T/Q on {pool.workers} spawned single-threaded workers; value = samples "
+                      f"/ slowest worker's compute time, ms_per_step = measured wall time of a step"}
     line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD + " (oracle on host cores)", "global_batch": 256},
+            "config": {"workload": WORKLOAD + " (oracle on host cores)", "global_batch": per * pool.workers},
+            "impl": "reference", "cpu_baseline": base,
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "wall_s": time.perf_counter() - t_all}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on the conv networks: one image through one layer shape per task
+# ---------------------------------------------------------------------------
+def conv_workload(name, batch=None):
+    from paper_2607_14672_gb300 import configs
+    mk = {"cfg4": configs.config4, "cfg5": configs.config5, "syn9": configs.syn_snn9,
+          "syn20": configs.syn_snn20}[name]
+    cfg = mk() if batch is None else mk(batch=batch)
+    return configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
+
+
+def _layer_in_shape(cfg, l):
+    """(C, H, W) of layer l's input (the concatenated input of a skip layer)."""
+    L = cfg["layers"][l]
+    if L["kind"] == "conv":
+        return tuple(L["in_shape"])
+    return (int(L["W"].shape[1]),)
+
+
+def conv_layer_groups(cfg):
+    """Layers of the same shape (kind, input shape, filter, stride): {key: [layer indices]}."""
+    groups = {}
+    for l, L in enumerate(cfg["layers"]):
+        key = (L["kind"], _layer_in_shape(cfg, l), tuple(np.asarray(L["W"]).shape), L.get("stride", 1),
+               L.get("pad", 0))
+        groups.setdefault(key, []).append(l)
+    return groups
+
+
+_LAYER_CFG = {}
+
+
+def _oracle_layer_task(args):
+    """Oracle forward + backward of one image through layer l of a conv
+    workload (Alg. 2 body, its IFT backward, T and Q terms; the readout with
+    the CE loss). Layer l > 0 sees spike times drawn over the previous
+    layer's window with a quarter silent (its cost does not depend on the
+    values). Returns the seconds of oracle work."""
+    name, l, img = args
+    from oracle import losses, network
+    if name not in _LAYER_CFG:
+        _LAYER_CFG[name] = conv_workload(name)
+    cfg = _LAYER_CFG[name]
+    L = cfg["layers"][l]
+    shp = _layer_in_shape(cfg, l)
+    g = np.random.default_rng(100 + l)
+    if l == 0:
+        x = np.asarray(cfg["inputs"](), np.float32).astype(np.float64)[img:img + 1]
+    else:
+        P = cfg["layers"][l - 1]
+        x = g.uniform(P["t_first"] + 0.2, P["t_end"], (1,) + shp)
+        x[g.random(x.shape) < 0.25] = np.inf
+    t = time.perf_counter()
+    ctx = network.forward_layer(x, L)
+    nrm = network.penalty_norm(ctx)
+    if l == len(cfg["layers"]) - 1:
+        _, g_t = losses.ce_loss(ctx["t"].reshape(1, -1), cfg["labels"]()[img:img + 1], cfg["tau_soft"],
+                                t_silent=L["t_end"])
+        g_t = g_t.reshape(ctx["t"].shape)
+    else:
+        g_t = g.normal(0.0, 1.0, ctx["t"].shape)
+    _, gT = losses.temporal_penalty(ctx["t"], L.get("t_head_l", 0.0), L.get("t_tail_l", 0.0),
+                                    L.get("gamma_head", 0.0), L.get("gamma_tail", 0.0), nrm)
+    network.backward_layer(ctx, L, g_t + gT)
+    return time.perf_counter() - t
+
+
+def _spawn_pool(n):
+    import multiprocessing as mp
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[v] = "1"
+    return mp.get_context("spawn").Pool(n)
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def oracle_conv_baseline(name, max_workers=16):
+    """cpu_baseline of a conv workload: every distinct layer shape timed once
+    (one image, forward + backward), the shapes in parallel on single-threaded
+    spawned workers; one image's time is the sum over the network's layers of
+    its shape's time, and the value is the throughput of that many cores
+    each taking an image through the network."""
+    cfg = conv_workload(name)
+    groups = conv_layer_groups(cfg)
+    keys = list(groups)
+    workers = max(1, min(host_cores(), max_workers, len(keys)))
+    pool = _spawn_pool(workers)
+    try:
+        secs = pool.map(_oracle_layer_task, [(name, groups[k][0], 0) for k in keys])
+    finally:
+        pool.close()
+        pool.join()
+    per_image = sum(t * len(groups[k]) for k, t in zip(keys, secs))
+    return {"value": workers / per_image, "unit": UNIT, "cores": workers, "kind": "oracle",
+            "sample": f"one image through each of the {len(keys)} distinct layer shapes of the {len(cfg['layers'])}"
+                      f"-layer network (float64 NumPy forward + backward, penalties, CE at the readout), the shapes "
+                      f"in parallel on {workers} spawned single-threaded workers ({max(secs):.1f} s wall); one image "
+                      f"= {per_image:.1f} s of oracle work (each layer timed at its shape), value = {workers} cores / "
+                      f"that", "per_image_s": per_image}
+
+
+def run_reference_conv(args):
+    """--impl reference on a conv workload: each step runs one layer shape of
+    the network (cycling through the shapes, cheapest first) for one image on
+    every worker (a different image each); the value is the worker count over
+    one image's time through the whole network, each layer at its shape's
+    mean measured time (shapes that a run of fewer steps than shapes did not
+    reach are timed once after the timed steps)."""
+    t_all = time.perf_counter()
+    name = args.workload
+    cfg = conv_workload(name)
+    groups = conv_layer_groups(cfg)
+    keys = list(groups)
+    workers = max(1, min(host_cores(), 16))
+    pool = _spawn_pool(workers)
+
+    def flops(k):
+        L = cfg["layers"][groups[k][0]]
+        W = np.asarray(L["W"])
+        shp = _layer_in_shape(cfg, groups[k][0])
+        if L["kind"] == "conv":
+            H = (shp[1] + 2 * L["pad"] - W.shape[2]) // L["stride"] + 1
+            return float(H * H * W.size)
+        return float(W.size)
+
+    warm_key = min(keys, key=flops)
+    order = sorted(keys, key=flops)
+    times, walls = {}, []
+    try:
+        for k in range(args.warmup):
+            pool.map(_oracle_layer_task, [(name, groups[warm_key][0], i) for i in range(workers)])
+        for k in range(args.steps):
+            key = order[k % len(order)]
+            t_s = time.perf_counter()
+            secs = pool.map(_oracle_layer_task, [(name, groups[key][0], i) for i in range(workers)])
+            walls.append(time.perf_counter() - t_s)
+            times.setdefault(key, []).extend(secs)
+        reached = len(times)
+        # shapes a short run did not reach: timed once after the timed steps
+        missing = [k for k in keys if k not in times]
+        if missing:
+            secs = pool.map(_oracle_layer_task, [(name, groups[k][0], 0) for k in missing])
+            for k, t in zip(missing, secs):
+                times[k] = [t]
+    finally:
+        pool.close()
+        pool.join()
+    mean = {k: float(np.mean(v)) for k, v in times.items()}
+    per_image = sum(len(groups[k]) * mean[k] for k in keys)
+    v = workers / per_image
+    ms = 1000.0 * float(np.mean(walls))
+    base = {"value": v, "unit": UNIT, "cores": workers, "kind": "oracle",
+            "sample": f"each step: one image per worker through one of the {len(keys)} distinct layer shapes "
+                      f"(forward + backward), cycling cheapest first; {reached} shapes reached by the timed steps (the rest "
+                      f"timed once after them); one image through "
+                      f"the network = {per_image:.1f} s of oracle work; ms_per_step = measured wall time of a step"}
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg["workload"] + " (oracle on host cores)", "global_batch": cfg["batch"],
+                       "per_step_sample": f"{workers} images x 1 layer shape"},
             "impl": "reference", "cpu_baseline": base,
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "wall_s": time.perf_counter() - t_all}
@@ -507,111 +696,324 @@ def run_ours(args, rank, world, local):
     return 0
 
 
-# dense-equivalent tensor flops of one training step of a conv network: the
-# forward contraction of every layer at the padded tile shape, and twice that
-# for the backward (dS and dW), one pass in bf16
-def conv_step_dense_flops(net):
-    tot = 0.0
-    for l, L in enumerate(net.layers):
-        Mp = max(8, 1 << (L["M"] - 1).bit_length())
-        if net.geom[l] is not None:
-            H, W, C, k, st, pad = net.geom[l]
-            Ho, Wo = (H + 2 * pad - k) // st + 1, (W + 2 * pad - k) // st + 1
-            rows, K, n = net.B * Ho * Wo * Mp, k * k * C, net.W[l].shape[0]
+def _padded_m(M):
+    return max(8, 1 << (int(M) - 1).bit_length())
+
+
+def conv_step_units(n):
+    """Algorithmic work of one training step of a conv network, per kernel
+    kind (SURVEY 8(d) units, summed over the layers):
+      contractions  4 x positions x k^2 C_in x C_out flops each (two grid
+                    weights per input spike), with the dense tensor-core
+                    flops of the binned formulation beside them;
+      binning       read the input spike times (4 B), write the binned
+                    operand in the NHWC + grid-step layout (M x 2 B each);
+      scan/solve    read w^ (positions x M_p x C_out x 4 B), write 16 B per neuron;
+      dw^           read 20 B per neuron, write positions x M_p x C_out x 2 B;
+      weight prep   read W (4 B), write its bf16 copy (forward and, where the
+                    input gradient is needed, the transposed one);
+      AdamW         28 B per weight.
+    The dense readout counts as a dense layer (its own kinds on the
+    few-output path). Returns (flops, dense_flops, bytes) dicts."""
+    from paper_2607_14672_gb300.net import narrow_layer
+    algo_f, dense_f, algo_b = {}, {}, {}
+
+    def add(d, k, v):
+        d[k] = d.get(k, 0.0) + float(v)
+
+    B = n.B
+    for l, L in enumerate(n.layers):
+        M = int(L["M"])
+        Mp = _padded_m(M)
+        O = int(n.W[l].shape[0])
+        if n.geom[l] is not None:
+            H, Wd, C, k, st, pad = n.geom[l]
+            Ho, Wo = (H + 2 * pad - k) // st + 1, (Wd + 2 * pad - k) // st + 1
+            P, Pin, K = B * Ho * Wo, B * H * Wd * C, k * k * C
+            f, df = 4.0 * P * K * O, 2.0 * P * Mp * K * O
+            kinds = ["gemm_fwd_scan", "gemm_dW"] + (["gemm_dS_gradt"] if l > 0 else [])
+            for kk in kinds:
+                add(algo_f, kk, f)
+                add(dense_f, kk, df)
+            add(algo_b, "binning", Pin * 4 + Pin * M * 2)
+            add(algo_b, "binning_T", Pin * 4 + Pin * M * 2)
+            add(algo_b, "scan_solve", P * O * Mp * 4 + P * O * 16)
+            add(algo_b, "dwhat", P * O * 20 + P * O * Mp * 2)
+            add(algo_b, "prep_weights", (O * K * 6) * (2 if l > 0 else 1))
+            add(algo_b, "adamw", 28 * O * K)
         else:
-            rows, K, n = net.B * Mp, net.W[l].shape[1], net.W[l].shape[0]
-        f = 2.0 * rows * K * n
-        tot += f if l == 0 else 3.0 * f    # layer 1 has no dS
-        if l == 0:
-            tot += f                        # its dW
-    return tot
+            ni = int(n.W[l].shape[1])
+            if narrow_layer(ni, O, M, n.math):
+                add(algo_b, "narrow_fwd", B * ni * 4 + O * ni * 4 + 16 * B * O)
+                add(algo_b, "narrow_bwd", B * ni * 4 + O * ni * 4 + 20 * B * O + B * ni * 4 + O * ni * 4)
+            else:
+                f, df = 4.0 * B * ni * O, 2.0 * B * Mp * ni * ((O + 127) // 128 * 128)
+                for kk in ("gemm_fwd_scan", "gemm_dW", "gemm_dS_gradt"):
+                    add(algo_f, kk, f)
+                    add(dense_f, kk, df)
+                add(algo_b, "binning", B * ni * 4 + B * M * ni * 2)
+                add(algo_b, "binning_T", B * ni * 4 + B * M * ni * 2)
+                add(algo_b, "scan_solve", B * O * Mp * 4 + B * O * 16)
+                add(algo_b, "dwhat", B * O * 20 + B * O * Mp * 2)
+                add(algo_b, "prep_weights", O * ni * 12)
+            add(algo_b, "adamw", 28 * O * ni)
+    return algo_f, dense_f, algo_b
 
 
-def run_conv(args, local):
+def conv_rooflines(n, per_kind, pk, pk_src, sustained=False):
+    """Achieved against the measured peak for every kernel kind of the step:
+    the kind's algorithmic work per step over its device time per step."""
+    algo_f, dense_f, algo_b = conv_step_units(n)
+    hbm = pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    key = "bf16_tflops_sustained" if sustained else "bf16_tflops"
+    tc = pk.get(key, FALLBACK_PEAKS[key])
+    out = {}
+    for k, (ms, launches) in per_kind.items():
+        t = ms / 1000.0
+        if t <= 0:
+            continue
+        if k in algo_f:
+            a = algo_f[k] / t / 1e12
+            d = dense_f[k] / t / 1e12
+            out[k] = {"bound": "tensor", "achieved": a, "peak": tc, "unit": "TFLOP/s", "frac": a / tc,
+                      "dense_achieved": d, "dense_frac": d / tc, "per_launch_flops": algo_f[k] / max(launches, 1),
+                      "per_launch_dense_flops": dense_f[k] / max(launches, 1), "launches": launches,
+                      "peak_source": f"{pk_src} bf16 ({'sustained' if sustained else 'burst'})",
+                      "launch_us": ms * 1000.0 / max(launches, 1)}
+        elif k in algo_b:
+            a = algo_b[k] / t / 1e9
+            out[k] = {"bound": "hbm", "achieved": a, "peak": hbm, "unit": "GB/s", "frac": a / hbm,
+                      "per_launch_bytes": algo_b[k] / max(launches, 1), "launches": launches,
+                      "peak_source": f"{pk_src} copy", "launch_us": ms * 1000.0 / max(launches, 1)}
+    return out
+
+
+def exact_candidate_bytes(n):
+    """The exact method's retained candidates for a backward (16 B per sample
+    x neuron x input, Tab. computational_complexity), over the network."""
+    tot = 0
+    for l, L in enumerate(n.layers):
+        O = int(n.W[l].shape[0])
+        if n.geom[l] is not None:
+            H, Wd, C, k, st, pad = n.geom[l]
+            Ho, Wo = (H + 2 * pad - k) // st + 1, (Wd + 2 * pad - k) // st + 1
+            tot += n.B * Ho * Wo * O * k * k * C * 16
+        else:
+            tot += n.B * O * int(n.W[l].shape[1]) * 16
+    return int(tot)
+
+
+def measure_cfg2(dev, stream, flush, steps=20, warmup=3):
+    """The 784-800-800-10 MLP step (x3), timed like the headline: a compact line."""
+    import torch
+    from paper_2607_14672_gb300 import configs, net
+    cfg = configs.config2()
+    cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
+    n = net.DenseNet(cfg, "x3", device=dev, with_adamw=True)
+    t0, lab = rank_batch(cfg, 0)
+    n.set_inputs(t0, lab)
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            n.step()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            n.step()
+        for _ in range(warmup):
+            g.replay()
+        stream.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in ev:
+            flush.zero_()
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+        stream.synchronize()
+    ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    return {"workload": WORKLOAD, "value": cfg["batch"] / (ms / 1000.0), "unit": UNIT, "ms_per_step": ms,
+            "steps": steps, "math": "x3 (fp32-accurate three-product bf16/fp16 split)",
+            "l2": "flushed (512 MB write) before each timed step"}
+
+
+def run_conv(args, rank, world, local):
     """Training step (forward, CE loss, backward, AdamW) of a conv network
-    (config 4 or 5, or the paper's Syn-SNN-9 / Syn-SNN-20), captured in a
-    CUDA graph and replayed K times, L2 flushed before each, CUDA events on
-    the stream; per-kind kernel times from a second capture with event nodes."""
-    import numpy as np
+    (config 5 by default; config 4, Syn-SNN-9 / Syn-SNN-20), captured in a
+    CUDA graph and replayed K times with CUDA events on the stream, L2
+    flushed and the weights and optimizer state put back to their initial
+    values before each (outside the events); per-kind kernel times from a
+    second capture with event nodes; end to end through the public API with
+    the inputs copied in and the loss read back every step."""
     import torch
 
     from paper_2607_14672_gb300 import build as _b
     _b.build()
-    from paper_2607_14672_gb300 import configs, dstd, net
+    from paper_2607_14672_gb300 import dstd, net
 
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    cfg = {"cfg4": configs.config4, "cfg5": configs.config5, "syn9": configs.syn_snn9,
-           "syn20": configs.syn_snn20}[args.workload]()
-    cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
+    cfg = conv_workload(args.workload)
+    B = cfg["batch"]
     n = net.ConvNet(cfg, device=dev, with_adamw=True)
-    n.set_inputs(np.asarray(cfg["inputs"](), np.float32), cfg["labels"]().astype(np.int32))
+    t0, lab = rank_batch(cfg, rank)
+    n.set_inputs(t0, lab)
     stream = torch.cuda.Stream(device=dev)
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    init = [(x, x.clone()) for x in list(n.W) + list(n.m) + list(n.v)] + [(n.adam_state, n.adam_state.clone())]
+
+    def restore():
+        for dst, src in init:
+            dst.copy_(src, non_blocking=True)
+
     with torch.cuda.stream(stream):
-        # silent share per layer at initialisation (before any optimizer step)
         n.forward()
         stream.synchronize()
         dead_init = [float(x) for x in n.dead_fraction()]
         for _ in range(max(1, args.warmup)):
             n.step()
-        stream.synchronize()
+        restore()
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
             n.step()
         for _ in range(args.warmup):
+            restore()
             graph.replay()
         stream.synchronize()
-    steps = max(2, min(args.steps, 20))
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    status = dstd.device_status(clear=True)
+    if status != 0:
+        raise RuntimeError(f"device status {status} after warm-up")
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     clocks = ClockSampler(local)
-    clocks.start()
+    if not args.profile:
+        clocks.start()
+        with torch.cuda.stream(stream):
+            t_load = time.time()
+            while time.time() - t_load < 0.5:
+                restore()
+                graph.replay()
+                stream.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         for a, b in ev:
             flush.zero_()
+            restore()
             a.record(stream)
             graph.replay()
             b.record(stream)
     torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
     clk = clocks.stop()
     ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    ms = max_over_ranks(ms, world, dev)
+    value = job_throughput(world, B, ms)
+    dead_after = [float(x) for x in n.dead_fraction()]
+    status = dstd.device_status(clear=True)
+    if args.profile:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": value, "unit": UNIT, "ms_per_step": ms, "steps": args.steps,
+                              "warmup": args.warmup, "profile_run": True, "device_status": status}), flush=True)
+        return 0 if status == 0 else 1
+
+    # per-kind device times: the step captured again with event nodes around every launch
+    n_kt = 2
     dstd.timing_enable(True)
     with torch.cuda.stream(stream):
         gt = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gt, stream=stream):
             n.step()
+        restore()
         gt.replay()
         stream.synchronize()
-        for _ in range(2):
+        for _ in range(n_kt):
             flush.zero_()
+            restore()
             gt.replay()
             dstd.timing_collect()
     kt = dstd.timing_read()
     dstd.timing_enable(False)
-    status = dstd.device_status(clear=True)
+    per_kind = {k: (v[0] / n_kt, v[1] // n_kt) for k, v in kt.items() if v[1] > 0}
+    launches_per_step = sum(c for _, c in per_kind.values())
+
+    # end to end through the public API: pinned H2D of the inputs and labels,
+    # the step, D2H of the loss, every step
+    pin_t = torch.from_numpy(np.ascontiguousarray(np.asarray(t0, np.float32).transpose(0, 2, 3, 1))).pin_memory()
+    pin_l = torch.from_numpy(np.asarray(lab, np.int32)).pin_memory()
+    loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
+    n_e2e = max(2, min(args.steps, 10))
+    e2e_s = 0.0
+    with torch.cuda.stream(stream):
+        for _ in range(n_e2e):
+            restore()
+            stream.synchronize()
+            t_s = time.perf_counter()
+            n.t_in.copy_(pin_t, non_blocking=True)
+            n.labels.copy_(pin_l, non_blocking=True)
+            graph.replay()
+            loss_h.copy_(n.loss[:1], non_blocking=True)
+            stream.synchronize()
+            _ = float(loss_h[0])
+            e2e_s += time.perf_counter() - t_s
+    e2e_ms = 1000.0 * e2e_s / n_e2e
+    e2e = {"value": job_throughput(world, B, e2e_ms), "unit": UNIT, "ms_per_step": e2e_ms,
+           "h2d_bytes_per_step": int(pin_t.numel() * 4 + pin_l.numel() * 4), "d2h_bytes_per_step": 4,
+           "path": "ConvNet.step (public ctypes API) captured in a CUDA graph, replayed per step, host clock"}
+
     pk, pk_src = peaks()
-    flops = conv_step_dense_flops(n)
-    dead = [float(x) for x in n.dead_fraction()]
-    B = cfg["batch"]
-    print(json.dumps({
-        "metric": "DSTD conv SNN training step samples/s at 1 GB300", "value": B / (ms / 1000.0),
-        "unit": "samples/s", "n_gpus": 1, "steps": steps, "warmup": args.warmup, "ms_per_step": ms,
-        "higher_is_better": True, "dtype": "bf16 operands, fp32 accumulation and state",
-        "data": "synthetic (seeded intensity maps; random-init weights)",
-        "config": {"workload": cfg["workload"], "global_batch": B, "layers": len(n.layers),
-                   "l2": "flushed (512 MB write) before each timed step"},
-        "tensor": {"dense_flops_per_step": flops, "achieved_tflops": flops / (ms / 1000.0) / 1e12,
-                   "peak": pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
-                   "frac": flops / (ms / 1000.0) / 1e12 / pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]),
-                   "peak_source": f"{pk_src} bf16 (burst)",
-                   "note": "whole step: every kernel's time in the denominator, the contractions' padded dense "
-                           "flops in the numerator"},
-        "kernel_ms": {k: round(v[0] / 2, 4) for k, v in kt.items() if v[1] > 0},
-        "dead_fraction_per_layer": {"at_init": dead_init, "after_steps": dead,
-                                    "note": "after_steps follows the warm-up and timed steps, each with an AdamW "
-                                            "update on random labels"},
-        "clocks": clk, "device_status": status}), flush=True)
+    rooflines = conv_rooflines(n, per_kind, pk, pk_src)
+    dom = max(per_kind, key=lambda k: per_kind[k][0])
+    roof = dict(rooflines.get(dom, {"bound": None, "achieved": None, "peak": None, "unit": None, "frac": None}))
+    roof["kernel"] = dom
+    roof["share_of_step"] = per_kind[dom][0] / sum(v[0] for v in per_kind.values())
+    roof["traffic"] = None
+    roof["traffic_note"] = "DRAM bytes per launch of this kernel: profiles/ (ncu), not measured in this run"
+    algo_f, dense_f, _ = conv_step_units(n)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded intensity maps, t = 1 - x; random-init weights with calibrated means)",
+            "config": {"workload": cfg["workload"], "global_batch": B * world, "per_gpu_batch": B,
+                       "M": int(cfg["layers"][0]["M"]), "layers": len(n.layers),
+                       "arithmetic": "bf16 contraction operands, fp32 accumulation, fp32 state and solve",
+                       "l2": "flushed (512 MB write) before each timed step",
+                       "state": "weights and AdamW state put back to their initial values before each timed step "
+                                "(outside the timed region)",
+                       "parallelism": "replicas" if world > 1 else "single"},
+            "roofline": roof, "rooflines": rooflines, "clocks": clk, "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps,
+            "gpu_launches_counted": {"per_step": launches_per_step, "how": "event nodes of a timing capture"},
+            "kernel_ms": {k: round(v[0], 4) for k, v in per_kind.items()},
+            "tensor": {"algorithmic_flops_per_step": sum(algo_f.values()),
+                       "dense_flops_per_step": sum(dense_f.values()),
+                       "step_algorithmic_tflops": sum(algo_f.values()) / (ms / 1000.0) / 1e12,
+                       "step_dense_tflops": sum(dense_f.values()) / (ms / 1000.0) / 1e12},
+            "memory": {"peak_allocated_bytes": int(torch.cuda.max_memory_allocated(dev)) - flush.numel(),
+                       "workspace_bytes": int(n.workspace.numel()),
+                       "saved_state_bytes": int(sum(x.numel() for x in n.saved) + sum(x.numel() * 4 for x in n.t)),
+                       "exact_candidate_bytes": exact_candidate_bytes(n),
+                       "note": "peak excludes the L2-flush buffer; exact = the exact method's retained candidates "
+                               "(16 B per sample x neuron x input, Tab. computational_complexity)"},
+            "dead_fraction_per_layer": {"at_init": dead_init, "after_timed_steps": dead_after},
+            "device_status": status}
+    if rank == 0 and world == 1:
+        if args.workload == "cfg5":
+            try:
+                line["also"] = {"cfg2": measure_cfg2(dev, stream, flush)}
+            except Exception as e:
+                line["also"] = {"cfg2": {"error": repr(e)}}
+        if not args.no_cpu_baseline:
+            try:
+                line["cpu_baseline"] = oracle_conv_baseline(args.workload)
+            except Exception as e:  # the baseline is reported, never fatal
+                line["cpu_baseline"] = {"value": None, "error": repr(e)}
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
     return 0 if status == 0 else 1
 
 
@@ -873,8 +1275,8 @@ def main():
         return run_cfg3(args, local) if rank == 0 else 0
     if args.workload == "ms":
         return run_multispike(args, local) if rank == 0 else 0
-    if args.workload != "cfg2":
-        return run_conv(args, local) if rank == 0 else 0
+    if args.workload in CONV_WORKLOADS:
+        return run_conv(args, rank, world, local)
     return run_ours(args, rank, world, local)
 
 

@@ -12,7 +12,7 @@ Parity status: pinned.
     to the exact method as M grows (App. E.1).
   * ``backward_*``: central finite differences of the float64 forward.
 
-Readings where the paper is silent or garbled (listed in the design notes):
+Readings where the paper is silent or garbled (the CUDA path takes the same ones):
   R1  candidates q = 0..M-1 on [T_q, T_{q+1}); no crossing by T_M = silent;
       so only w^_m for m = 0..M-1 can matter and the bin axis has M entries.
   R2  Eq. DSTD_kernel is applied literally for m = 0..M-1: a spike earlier

@@ -17,7 +17,7 @@ Cost (Eq. cost_function), per sample and averaged over the mini-batch:
   Q  dead-neuron term (Eq. dead_neuron_penalty): -sum_{i,l} 1{t_i = inf} sum_j w_ij.
   For convolutional layers T and Q are divided by the spatial size.
 
-Readings (listed in the design notes):
+Readings where the paper is silent (the CUDA path takes the same ones):
   R7  T skips silent neurons (the paper notes T gives them no gradient);
       in L a silent output enters with the constant time ``t_silent`` (the
       output layer's window end), so the loss stays finite and a silent

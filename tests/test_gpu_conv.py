@@ -138,3 +138,82 @@ def test_conv_chunked_matches_unchunked():
         torch.cuda.synchronize()
         gWs.append(host(g_W))
     assert rel_l2(gWs[0], sum(gWs[1:])) <= 1e-5
+
+
+# ---------------------------------------------------------------------------
+# bf16 (the conv workloads' precision) against the oracle on bf16-rounded
+# contraction operands (reading R9): s and W in the forward; dw^, s and W in
+# the backward. Layer shapes, tau and M of configs 4 and 5 at a reduced image
+# size (the oracle's contraction is a plain per-tap einsum), B = 2.
+# ---------------------------------------------------------------------------
+BF16_CASES = [
+    # C_in, H, C_out, stride, tau, M
+    (3, 16, 64, 1, (INF, INF), 32),       # config 4, layer 1
+    (64, 16, 64, 2, (INF, INF), 32),      # config 4, layer 2
+    (64, 8, 128, 1, (INF, INF), 32),      # config 4, layer 3
+    (256, 4, 512, 1, (INF, INF), 32),     # config 4, layer 7
+    (1, 12, 64, 1, (1.0, 0.25), 64),      # config 5, layer 1
+    (64, 10, 64, 1, (1.0, 0.25), 64),     # config 5, layers 2-6
+    (64, 10, 128, 2, (1.0, 0.25), 64),    # config 5, layer 7
+    (128, 6, 128, 1, (1.0, 0.25), 64),    # config 5, layers 8-13
+    (128, 6, 256, 2, (1.0, 0.25), 64),    # config 5, layer 14
+    (256, 4, 256, 1, (1.0, 0.25), 64),    # config 5, layers 15-19
+]
+
+
+@pytest.mark.parametrize("C,H,O,stride,tau,M", BF16_CASES)
+def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
+    from paper_2607_14672_gb300 import dstd
+    from helpers import (bf16, bf16_potential_bound, check_bf16_times, conv_neurons, grid_of, kernel_max)
+    B = 2
+    t, L = conv_case(B, C, H, O, 3, stride, 1, M, tau, seed=7 * C + H + O, wmean=WMEAN64[tau] * 64 / C,
+                     gammas=(0.05, 0.01, 1e-3), silent=0.1)
+    r = run_conv_fwd(t, L, "bf16")
+    T, dt = grid_of(L)
+    tv, ti = tau
+    s = odstd.binning(t.reshape(B, -1), T, dt, tv, ti).reshape(B, M, C, H, H)
+    what = onet.conv_what(bf16(s), bf16(L["W"]), stride, 1)
+    _, _, Ho, Wo, _ = what.shape
+    flat = odstd.solve(what.reshape(B, O * Ho * Wo, M), T, dt, tv, ti, 1.0)
+    ctx = {k: flat[k].reshape(B, O, Ho, Wo) for k in ("t", "q", "vpeak", "vdot", "fired")}
+    kmax = kernel_max(T, tv, ti)
+
+    def bound(idx):
+        b, o, y, x = np.unravel_index(idx, (B, O, Ho, Wo))
+        nc = conv_neurons(t, L, list(zip(b, o, y, x)))
+        return bf16_potential_bound(nc["s"], nc["w"], ctx["q"].ravel()[idx], ctx["t"].ravel()[idx], T, tv, ti,
+                                    kmax)
+
+    n_cmp, n_bound = check_bf16_times(r["t"], ctx, L, bound)
+    assert n_cmp > 0.2 * r["t"].size
+    assert n_bound <= 0.01 * r["t"].size
+
+    # backward: random upstream gradient; the neurons whose spike state is
+    # ill-conditioned (near the threshold, or outside the base tolerance)
+    # get none, on either side
+    Tmax = L["t_end"] - L["t_first"]
+    fo, fg = np.isfinite(ctx["t"]), np.isfinite(r["t"])
+    gap = np.where(fo & fg, np.abs(np.where(fo & fg, r["t"] - ctx["t"], 0.0)), 0.0)
+    ill = (np.abs(ctx["vpeak"] - 1.0) <= 1e-5) | (fo != fg) | (gap > 1e-4 * Tmax)
+    nrm = 1.0 / (B * Ho * Wo)
+    g = np.random.default_rng(C + O).normal(0.0, 1.0, ctx["t"].shape)
+    _, pg = olosses.temporal_penalty(r["t"], 0.35, 0.8, 0.05, 0.01, nrm)
+    _, gT = olosses.temporal_penalty(ctx["t"], 0.35, 0.8, 0.05, 0.01, nrm)
+    g_gpu = np.where(ill, -pg, g)
+    g_ora = np.where(ill, 0.0, g + gT)
+    g_t_in = torch.empty_like(r["t_in"])
+    g_W = torch.empty_like(r["W"])
+    dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g_gpu.transpose(0, 2, 3, 1)), stride, 1, r["p"],
+                  "bf16", g_t_in, g_W, r["ws"])
+    torch.cuda.synchronize()
+    assert dstd.device_status(clear=True) == 0
+    fl = {k: ctx[k].reshape(B, -1) for k in ("t", "q", "vdot", "fired")}
+    gw = odstd.solve_backward(fl, g_ora.reshape(B, -1), T, dt, tv, ti, 1.0).reshape(B, O, Ho, Wo, M)
+    gW, gs = onet.conv_what_adjoint(bf16(gw), bf16(s), bf16(L["W"]), stride, 1)
+    ds = odstd.binning(t.reshape(B, -1), T, dt, tv, ti, derivative=True).reshape(gs.shape)
+    gin = np.sum(gs * ds, axis=1)
+    cnt = (~fg).sum((0, 2, 3))
+    gW = gW - 1e-3 * nrm * cnt[:, None, None, None]
+    assert rel_l2(host(g_W).transpose(0, 3, 1, 2), gW) <= 1e-3
+    assert rel_l2(host(g_t_in).transpose(0, 3, 1, 2), gin) <= 1e-3
+    assert np.all(host(g_t_in).transpose(0, 3, 1, 2)[~np.isfinite(t)] == 0)

@@ -1,22 +1,28 @@
 """GPU parity of the convolutional networks (configs 4 and 5) against the
-float64 oracle, at their full batch in bf16 (the workloads' precision).
+float64 oracle, in bf16 (the workloads' precision).
 
-The GPU runs whole training steps (forward, CE + T + Q, backward, AdamW) on
-the full batch. Parity is checked layer by layer with teacher forcing (each
-oracle layer is fed the GPU's input to that layer), on the oracle run with
-bf16-rounded contraction operands (reading R9):
+The GPU runs whole training steps (forward, CE + T + Q, backward, AdamW).
+Parity is checked layer by layer with teacher forcing (each oracle layer is
+fed the GPU's input to that layer), on the oracle run with bf16-rounded
+contraction operands (reading R9):
 
-* config 4 (tau = (inf, inf), closed-form solve): every neuron of two images
-  of every layer, plus a free-running oracle pass of those images whose
-  per-layer firing fractions and loss terms must agree;
-* config 5 (tau = (1.0, 0.25), numeric solve): 192 sampled neurons per layer,
-  each recomputed from its 3x3 receptive field, and the per-layer silent
-  (dead) share on those neurons.
+* config 4 (tau = (inf, inf), closed-form solve), full batch: every neuron of
+  two images of every layer, plus a free-running oracle pass of those images
+  whose per-layer firing fractions must agree;
+* config 5 (tau = (1.0, 0.25), numeric solve), full batch: 192 sampled
+  neurons per layer, each recomputed from its 3x3 receptive field, and the
+  per-layer silent (dead) share on those neurons;
+* gradients of both networks at full width (batch 4): for every conv layer,
+  the weight gradient of one output channel (a sum over every position of
+  every image) and the input-time gradient of every channel at two input
+  positions, each within 1e-3 relative L2 of the oracle.
 
-bf16 operands: s is rounded from fp32 on the GPU and from float64 in the
-oracle, which can differ by one bf16 step in a single term; as in the dense
-bf16 test the time tolerance is 5e-4 T_max and the near-threshold margin
-1e-3 (R9).
+Spike times meet |dt| <= 1e-4 T_max and masks agree outside the 1e-5 band
+around the threshold, except where a neuron's own bound on the bf16
+difference allows more (``helpers.check_bf16_times``): a grid weight that
+lies within a few fp32 ulps of a bf16 rounding midpoint may round to the
+other neighbour on the GPU (fp32) than in the oracle (float64), and the
+tensor core accumulates the exact bf16 products in fp32.
 """
 
 import math
@@ -25,12 +31,11 @@ import numpy as np
 import pytest
 import torch
 
-from helpers import bf16, grid_of, oracle_forward
-from oracle import dstd as odstd, network as onet
+from helpers import (bf16, check_bf16_times, conv_neurons, decode_saved, dense_bound_fn, grid_of, neuron_bound_fn,
+                     oracle_forward, receptive_fields, rel_l2)
+from oracle import dstd as odstd, losses as olosses, network as onet
 
 pytestmark = pytest.mark.gpu
-
-TOL_SCALE, MARGIN = 5.0, 1e-3
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -74,35 +79,37 @@ def oracle_conv_layer(x, L, operand_round=bf16):
     what = onet.conv_what(operand_round(s), operand_round(np.asarray(L["W"], np.float32)), L["stride"], L["pad"])
     _, O, Ho, Wo, M = what.shape
     ctx = odstd.solve(what.reshape(B, O * Ho * Wo, M), T, dt, tv, ti, V)
-    return {k: ctx[k].reshape(B, O, Ho, Wo) for k in ("t", "vpeak", "q")}
+    out = {k: ctx[k].reshape(B, O, Ho, Wo) for k in ("t", "vpeak", "q", "vdot", "fired")}
+    out["T"], out["dt"] = T, dt
+    return out
 
 
-def oracle_conv_neurons(x, L, idx, operand_round=bf16):
-    """Oracle output of the conv neurons idx = [(b, o, y, x)], each from its k x k receptive field."""
-    T, dt = grid_of(L)
-    tv, ti, V = L["tau_v"], L["tau_I"], L["v_th"]
+def conv_layer_bound_fn(x, ctx, L):
+    """Per-neuron bf16 bound of a whole-layer oracle context (receptive fields of the flagged neurons only)."""
+    from helpers import bf16_potential_bound, kernel_max
+    shape = ctx["t"].shape
+    kmax = kernel_max(ctx["T"], L["tau_v"], L["tau_I"])
+
+    def fn(idx):
+        b, o, y, xx = np.unravel_index(idx, shape)
+        nc = conv_neurons(x, L, list(zip(b, o, y, xx)))
+        return bf16_potential_bound(nc["s"], nc["w"], ctx["q"].ravel()[idx], ctx["t"].ravel()[idx], ctx["T"],
+                                    L["tau_v"], L["tau_I"], kmax)
+    return fn
+
+
+def compare_layer(t_gpu, ctx, L, bound_fn, min_cmp=0.9):
+    n_cmp, n_bound = check_bf16_times(t_gpu, ctx, L, bound_fn)
+    ok = np.abs(np.asarray(ctx["vpeak"]) - L["v_th"]) > 1e-5
+    assert ok.sum() > min_cmp * np.asarray(t_gpu).size
+    assert n_bound <= 0.01 * np.asarray(t_gpu).size
+    return n_cmp
+
+
+def dense_readout_ctx(x, L):
     W = np.asarray(L["W"], np.float32).astype(np.float64)
-    k, st, pad = W.shape[2], L["stride"], L["pad"]
-    xp = np.pad(x, ((0, 0), (0, 0), (pad, pad), (pad, pad)), constant_values=np.inf)
-    patches = np.stack([xp[b, :, y * st:y * st + k, xx * st:xx * st + k] for (b, o, y, xx) in idx])
-    n = len(idx)
-    s = odstd.binning(patches.reshape(n, -1), T, dt, tv, ti)          # [n, M, C k k]
-    Wsel = W[[o for (_, o, _, _) in idx]].reshape(n, -1)
-    what = np.einsum("nmj,nj->nm", operand_round(s), operand_round(Wsel))
-    ctx = odstd.solve(what[None], T, dt, tv, ti, V)
-    return {key: ctx[key][0] for key in ("t", "vpeak", "q")}
-
-
-def compare(t_gpu, t_ora, vpeak, L, min_both=0.2):
-    """Masks equal away from the threshold; times within TOL_SCALE 1e-4 T_max."""
-    ok = np.abs(vpeak - L["v_th"]) > MARGIN
-    fg, fo = np.isfinite(t_gpu), np.isfinite(t_ora)
-    assert not (ok & (fg != fo)).any(), f"{int((ok & (fg != fo)).sum())} mask flips away from threshold"
-    both = ok & fg & fo
-    if both.any():
-        err = np.abs(t_gpu[both] - t_ora[both]).max()
-        assert err <= TOL_SCALE * 1e-4 * (L["t_end"] - L["t_first"]), err
-    return int(both.sum()), int(ok.sum())
+    ctx = oracle_forward(x.reshape(x.shape[0], -1), W, L, operand_round=bf16)
+    return ctx, dense_bound_fn(ctx, W, L)
 
 
 def test_cfg4_conv_network_layers_match_oracle():
@@ -114,11 +121,10 @@ def test_cfg4_conv_network_layers_match_oracle():
         t_gpu = to_nchw(host(n.t[l]))[imgs]
         if L["kind"] == "conv":
             ctx = oracle_conv_layer(x, L)
+            fn = conv_layer_bound_fn(x, ctx, L)
         else:
-            ctx = oracle_forward(x.reshape(len(imgs), -1), np.asarray(L["W"], np.float32).astype(np.float64), L,
-                                 operand_round=bf16)
-        both, ok = compare(t_gpu, ctx["t"], ctx["vpeak"], L)
-        assert ok > 0.9 * t_gpu.size
+            ctx, fn = dense_readout_ctx(x, L)
+        compare_layer(t_gpu, ctx, L, fn)
         x = t_gpu                                   # teacher forcing: next layer sees the GPU's output
     # every layer fires, and the whole batch's dead share is recorded by the counters
     dead = n.dead_fraction()
@@ -154,20 +160,143 @@ def test_cfg5_conv_network_sampled_neurons_match_oracle():
             _, O, Ho, Wo = t_gpu.shape
             idx = [(bi, int(rng.integers(O)), int(rng.integers(Ho)), int(rng.integers(Wo)))
                    for bi in range(len(imgs)) for _ in range(96)]
-            ctx = oracle_conv_neurons(x, L, idx)
+            ctx = conv_neurons(x, L, idx)
+            fn = neuron_bound_fn(ctx, L)
             tg = np.array([t_gpu[imgs[b], o, y, xx] for (b, o, y, xx) in idx])
         else:
-            ctx = oracle_forward(x.reshape(len(imgs), -1), np.asarray(L["W"], np.float32).astype(np.float64), L,
-                                 operand_round=bf16)
+            ctx, fn = dense_readout_ctx(x, L)
             tg = t_gpu[imgs]
-        both, ok = compare(tg, ctx["t"], ctx["vpeak"], L)
-        assert ok > 0.9 * tg.size
+        compare_layer(tg, ctx, L, fn)
         # dead (silent) share on the sampled neurons, away from the threshold
-        okm = np.abs(ctx["vpeak"] - L["v_th"]) > MARGIN
-        assert np.mean(~np.isfinite(tg[okm])) == pytest.approx(np.mean(~np.isfinite(ctx["t"][okm])), abs=1e-12)
+        okm = np.abs(ctx["vpeak"] - L["v_th"]) > 1e-5
+        assert abs(np.mean(~np.isfinite(tg[okm])) - np.mean(~np.isfinite(ctx["t"][okm]))) <= 2.0 / okm.sum()
         x_all = t_gpu                               # teacher forcing
     for g in n.gW:
         assert torch.isfinite(g).all()
+
+
+# ---------------------------------------------------------------------------
+# gradients at full width (every conv layer of configs 4 and 5, batch 4)
+# ---------------------------------------------------------------------------
+def gpu_state(n, l):
+    """The GPU's spike state of layer l as [B, O, Ho, Wo] arrays (t, q, dv^/dt)."""
+    t = host(n.t[l])
+    B, Ho, Wo, O = t.shape
+    q, _, vd = decode_saved(n.saved[l].cpu().numpy(), B * Ho * Wo, O)
+    tr = lambda a: np.asarray(a, float).reshape(B, Ho, Wo, O).transpose(0, 3, 1, 2)
+    return to_nchw(t), tr(q), tr(vd)
+
+
+def with_gpu_state(ctx, gstate, L):
+    """Neurons whose spike state is ill-conditioned (near the threshold, a
+    firing mismatch, or a time gap beyond the base tolerance) take the GPU's
+    state (t, q, dv^/dt) before the backward: their gradient is then the
+    oracle's formula at the GPU's spike, the rest the oracle's own."""
+    tg, qg, vdg = gstate
+    Tmax = L["t_end"] - L["t_first"]
+    fo, fg = np.isfinite(ctx["t"]), np.isfinite(tg)
+    gap = np.where(fo & fg, np.abs(np.where(fo & fg, tg - ctx["t"], 0.0)), 0.0)
+    ill = (np.abs(ctx["vpeak"] - L["v_th"]) <= 1e-5) | (fo != fg) | (gap > 1e-4 * Tmax)
+    out = dict(ctx)
+    out["t"] = np.where(ill, tg, ctx["t"])
+    out["q"] = np.where(ill, qg, ctx["q"]).astype(int)
+    out["vdot"] = np.where(ill, vdg, ctx["vdot"])
+    out["fired"] = np.isfinite(out["t"])
+    return out, ill
+
+
+def oracle_dW_row(x, L, o, g_up, gstate, nrm):
+    """dC/dW[o] of a conv layer (oracle steps on bf16-rounded operands): the
+    layer's output channel o at every position of every image, its IFT
+    backward with the upstream gradient plus T', the adjoint contraction, and
+    the dead-neuron term."""
+    T, dt = grid_of(L)
+    tv, ti, V = L["tau_v"], L["tau_I"], L["v_th"]
+    B, C, H, Wd = x.shape
+    W = np.asarray(L["W"], np.float32).astype(np.float64)[o:o + 1]
+    s = odstd.binning(x.reshape(B, -1), T, dt, tv, ti).reshape(B, L["M"], C, H, Wd)
+    what = onet.conv_what(bf16(s), bf16(W), L["stride"], L["pad"])
+    _, _, Ho, Wo, M = what.shape
+    fl = odstd.solve(what.reshape(B, Ho * Wo, M), T, dt, tv, ti, V)
+    ctx = {k: fl[k].reshape(B, Ho, Wo) for k in ("t", "q", "vpeak", "vdot", "fired")}
+    ctx, ill = with_gpu_state(ctx, tuple(a[:, o] for a in gstate), L)
+    _, gT = olosses.temporal_penalty(ctx["t"], L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], nrm)
+    flat = {k: ctx[k].reshape(B, -1) for k in ("t", "q", "vdot", "fired")}
+    gw = odstd.solve_backward(flat, (g_up[:, o] + gT).reshape(B, -1), T, dt, tv, ti, V)
+    gW, _ = onet.conv_what_adjoint(bf16(gw.reshape(B, 1, Ho, Wo, M)), bf16(s), bf16(W), L["stride"], L["pad"])
+    cnt = float((~ctx["fired"]).sum())
+    return gW[0] - L["gamma_q"] * nrm * cnt, int(ill.sum())
+
+
+def oracle_input_grad(x, L, b, yi, xi, g_up, gstate, nrm):
+    """dC/dt_in of every channel of input position (b, yi, xi): the output
+    neurons whose receptive field holds it (all channels), their IFT backward,
+    then sum_m (sum_o W dw^) ds/dt (Tab. DSTD_kernels' derivative)."""
+    T, dt = grid_of(L)
+    tv, ti, V = L["tau_v"], L["tau_I"], L["v_th"]
+    W = np.asarray(L["W"], np.float32).astype(np.float64)
+    O, C, k, _ = W.shape
+    st, pad = L["stride"], L["pad"]
+    _, _, Ho, Wo = gstate[0].shape
+    taps = [(y, xx, yi - y * st + pad, xi - xx * st + pad) for y in range(Ho) for xx in range(Wo)
+            if 0 <= yi - y * st + pad < k and 0 <= xi - xx * st + pad < k]
+    rf = receptive_fields(x, k, st, pad, [(b, y, xx) for (y, xx, _, _) in taps])
+    s = odstd.binning(rf, T, dt, tv, ti)                                   # [P, M, K]
+    w2 = bf16(W.reshape(O, -1))
+    what = np.matmul(bf16(s), w2.T).transpose(0, 2, 1)                     # [P, O, M]
+    fl = odstd.solve(what, T, dt, tv, ti, V)
+    g = np.stack([g_up[b, :, y, xx] for (y, xx, _, _) in taps])           # [P, O]
+    gs = tuple(np.stack([a[b, :, y, xx] for (y, xx, _, _) in taps]) for a in gstate)
+    ctx, _ = with_gpu_state({k: fl[k] for k in ("t", "q", "vpeak", "vdot", "fired")}, gs, L)
+    _, gT = olosses.temporal_penalty(ctx["t"], L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], nrm)
+    gw = bf16(odstd.solve_backward(ctx, g + gT, T, dt, tv, ti, V))          # [P, O, M]
+    dS = sum(bf16(W[:, :, kh, kw]).T @ gw[p] for p, (_, _, kh, kw) in enumerate(taps))   # [C, M]
+    ds = odstd.binning(x[b, :, yi, xi], T, dt, tv, ti, derivative=True)    # [M, C]
+    return np.sum(dS * ds.T, axis=1)
+
+
+def check_network_gradients(cfg, seed):
+    from paper_2607_14672_gb300 import dstd
+    cfg, n, t0, lab = run_net(cfg)
+    rng = np.random.default_rng(seed)
+    B = n.B
+    worst = []
+    for l, L in enumerate(cfg["layers"]):
+        if L["kind"] != "conv":
+            continue
+        x = to_nchw(host(n.layer_input(l)))
+        g_up = to_nchw(host(n.g[l]))
+        gstate = gpu_state(n, l)
+        _, O, Ho, Wo = gstate[0].shape
+        nrm = 1.0 / (B * Ho * Wo)
+        o = int(rng.integers(O))
+        ref, n_ill = oracle_dW_row(x, L, o, g_up, gstate, nrm)
+        got = host(n.gW[l])[o].transpose(2, 0, 1)                          # [k, k, C] -> [C, k, k]
+        e_w = rel_l2(got, ref)
+        assert e_w <= 1e-3, (l, o, e_w, n_ill)
+        if l == 0:
+            worst.append((l, e_w, None))
+            continue
+        H, Wd = x.shape[2], x.shape[3]
+        got_g, ref_g = [], []
+        for (b, yi, xi) in [(0, 0, 0), (B - 1, int(rng.integers(1, H - 1)), int(rng.integers(1, Wd - 1)))]:
+            ref_g.append(oracle_input_grad(x, L, b, yi, xi, g_up, gstate, nrm))
+            got_g.append(to_nchw(host(n.g[l - 1]))[b, :, yi, xi])
+        e_g = rel_l2(np.concatenate(got_g), np.concatenate(ref_g))
+        assert e_g <= 1e-3, (l, e_g)
+        worst.append((l, e_w, e_g))
+    assert dstd.device_status(clear=True) == 0
+    return worst
+
+
+def test_cfg4_gradients_full_width_match_oracle():
+    from paper_2607_14672_gb300 import configs
+    print(check_network_gradients(configs.config4(batch=4), 41))
+
+
+def test_cfg5_gradients_full_width_match_oracle():
+    from paper_2607_14672_gb300 import configs
+    print(check_network_gradients(configs.config5(batch=4), 51))
 
 
 @pytest.mark.parametrize("shape,tau,seed", [((64, 16, 128, 1), (math.inf, math.inf), 4),

@@ -196,9 +196,13 @@ def test_forward_bf16_matches_rounded_oracle():
     t_in, layer["W"] = f32(t_in), f32(layer["W"])
     r = run_fwd(t_in, layer, "bf16")
     ctx = oracle_forward(t_in, layer["W"], layer, operand_round=bf16)
-    # bf16 operands: s is rounded from fp32 on the GPU and from fp64 in the
-    # oracle, which can differ by one bf16 step; tolerance and margin widen.
-    assert check_times(r["t"], ctx, layer, tol_scale=5.0, margin=1e-3) > 1500
+    # the benchmark spec's tolerance, widened only by each neuron's own bound on the
+    # legitimate bf16 difference (a grid weight at a rounding midpoint, fp32
+    # accumulation of the products): helpers.check_bf16_times
+    from helpers import check_bf16_times, dense_bound_fn
+    n_cmp, n_bound = check_bf16_times(r["t"], ctx, layer, dense_bound_fn(ctx, layer["W"], layer))
+    assert n_cmp > 1500
+    assert n_bound <= 0.01 * r["t"].size
 
 
 @pytest.mark.parametrize("math_mode", ["f32", "x3"])

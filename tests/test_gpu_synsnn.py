@@ -149,3 +149,44 @@ def test_syn20_gradients_match_oracle():
             C_, H_, W_ = ctxs[l - 1]["t"].shape[1:]
             gW = gW.reshape(gW.shape[0], H_, W_, C_).transpose(0, 3, 1, 2).reshape(gW.shape[0], -1)
         assert rel_l2(gW, grads[l]) <= 1e-3, (l, rel_l2(gW, grads[l]))
+
+
+@pytest.mark.parametrize("name", ["syn9", "syn20"])
+def test_paper_architecture_full_size_sampled_bf16(name):
+    """The benchmarked networks: N = 64, batch 50, M = 20, bf16 operands.
+    Every layer, teacher-forced (the oracle sees the GPU's input to the
+    layer, the skip layers' concatenated input included), on 192 sampled
+    neurons recomputed from their receptive fields (the 5x5 layer's too),
+    against the oracle on bf16-rounded operands (reading R9), with the
+    per-neuron bf16 bound of ``helpers.check_bf16_times``; the readout in
+    full."""
+    from paper_2607_14672_gb300 import configs, dstd, net
+    from helpers import bf16, check_bf16_times, conv_neurons, dense_bound_fn, neuron_bound_fn, oracle_forward
+    cfg = configs.syn_snn9() if name == "syn9" else configs.syn_snn20()
+    cfg = configs.with_offsets(cfg, configs.draw_offsets(cfg["layers"]))
+    n = net.ConvNet(cfg, math_mode="bf16", with_adamw=False)
+    t0 = f32(cfg["inputs"]())
+    n.set_inputs(t0.astype(np.float32), cfg["labels"]())
+    n.forward()
+    torch.cuda.synchronize()
+    assert dstd.device_status(clear=True) == 0
+    rng = np.random.default_rng(9)
+    imgs = [0, n.B - 1]
+    for l, L in enumerate(cfg["layers"]):
+        x = nchw(host(n.layer_input(l)))[imgs]
+        tg_all = nchw(host(n.t[l]))
+        if L["kind"] == "conv":
+            _, O, Ho, Wo = tg_all.shape
+            idx = [(bi, int(rng.integers(O)), int(rng.integers(Ho)), int(rng.integers(Wo)))
+                   for bi in range(len(imgs)) for _ in range(96)]
+            ctx = conv_neurons(x, L, idx)
+            fn = neuron_bound_fn(ctx, L)
+            tg = np.array([tg_all[imgs[b], o, y, xx] for (b, o, y, xx) in idx])
+        else:
+            W = np.asarray(L["W"], np.float32).astype(np.float64)
+            ctx = oracle_forward(x.reshape(len(imgs), -1), W, L, operand_round=bf16)
+            fn = dense_bound_fn(ctx, W, L)
+            tg = tg_all[imgs]
+        n_cmp, n_bound = check_bf16_times(tg, ctx, L, fn)
+        assert n_cmp > 0.1 * tg.size, (l, n_cmp)
+        assert n_bound <= max(2, 0.02 * tg.size), (l, n_bound)
