@@ -20,7 +20,8 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libdstd.so")
 SOURCES = ["dstd_api.cu", "dstd_lif_kernels.cu", "dstd_gemm_simt.cu", "dstd_gemm_tc.cu", "dstd_exact.cu",
            "dstd_multispike.cu"]
-HEADERS = [os.path.join(CSRC, "dstd_internal.cuh"), os.path.join(ROOT, "include", "dstd.h")]
+HEADERS = [os.path.join(CSRC, "dstd_internal.cuh"), os.path.join(CSRC, "dstd_tc_ptx.cuh"),
+           os.path.join(ROOT, "include", "dstd.h")]
 GENCODE = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
               "-Xptxas", "-O3"]

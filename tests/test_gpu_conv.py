@@ -38,11 +38,11 @@ def host(x):
     return x.detach().cpu().numpy().astype(np.float64)
 
 
-def conv_case(B, C, H, O, k, stride, pad, M, tau, seed, wmean, gammas=(0.0, 0.0, 0.0), silent=0.3):
+def conv_case(B, C, H, O, k, stride, pad, M, tau, seed, wmean, gammas=(0.0, 0.0, 0.0), silent=0.3, t_offset=0.011):
     g = np.random.default_rng(seed)
     t = f32(np.where(g.random((B, C, H, H)) < silent, INF, g.uniform(0, 1, (B, C, H, H))))
     W = f32(g.normal(wmean, 1.0 / math.sqrt(C * k * k), (O, C, k, k)))
-    L = dict(kind="conv", W=W, tau_v=tau[0], tau_I=tau[1], v_th=1.0, t_first=0.0, t_end=1.2, M=M, t_offset=0.011,
+    L = dict(kind="conv", W=W, tau_v=tau[0], tau_I=tau[1], v_th=1.0, t_first=0.0, t_end=1.2, M=M, t_offset=t_offset,
              stride=stride, pad=pad, t_head_l=0.35, t_tail_l=0.8, gamma_head=gammas[0], gamma_tail=gammas[1],
              gamma_q=gammas[2])
     return t, L
@@ -145,6 +145,13 @@ def test_conv_chunked_matches_unchunked():
 # contraction operands (reading R9): s and W in the forward; dw^, s and W in
 # the backward. Layer shapes, tau and M of configs 4 and 5 at a reduced image
 # size (the oracle's contraction is a plain per-tap einsum), B = 2.
+#
+# The backward is compared at the GPU's own spike state (t, q, dv^/dt from
+# the saved buffer), which the forward check has just held to the
+# tolerance: the input-time gradient is a difference of dS at the two grid
+# points around each input spike (for tau = (inf, inf) exactly (dS_{k+1} -
+# dS_k) / dt), so it magnifies a spike-time difference by about T / dt, and
+# bf16 operands legitimately move spike times by a few 1e-6.
 # ---------------------------------------------------------------------------
 BF16_CASES = [
     # C_in, H, C_out, stride, tau, M
@@ -161,13 +168,22 @@ BF16_CASES = [
 ]
 
 
+def gpu_spike_state(r, B, O, Ho, Wo):
+    """The GPU's spike state of a conv layer as an oracle context [B, O, Ho, Wo]."""
+    from helpers import decode_saved
+    q, _, vd = decode_saved(r["saved"].cpu().numpy(), B * Ho * Wo, O)
+    tr = lambda a: np.asarray(a, float).reshape(B, Ho, Wo, O).transpose(0, 3, 1, 2)
+    t = np.asarray(r["t"], float)
+    return {"t": t, "q": tr(q).astype(int), "vdot": tr(vd), "fired": np.isfinite(t)}
+
+
 @pytest.mark.parametrize("C,H,O,stride,tau,M", BF16_CASES)
 def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
     from paper_2607_14672_gb300 import dstd
     from helpers import (bf16, bf16_potential_bound, check_bf16_times, conv_neurons, grid_of, kernel_max)
     B = 2
     t, L = conv_case(B, C, H, O, 3, stride, 1, M, tau, seed=7 * C + H + O, wmean=WMEAN64[tau] * 64 / C,
-                     gammas=(0.05, 0.01, 1e-3), silent=0.1)
+                     gammas=(0.05, 0.01, 1e-3), silent=0.1, t_offset=0.3 * 1.2 / M)
     r = run_conv_fwd(t, L, "bf16")
     T, dt = grid_of(L)
     tv, ti = tau
@@ -188,32 +204,26 @@ def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
     assert n_cmp > 0.2 * r["t"].size
     assert n_bound <= 0.01 * r["t"].size
 
-    # backward: random upstream gradient; the neurons whose spike state is
-    # ill-conditioned (near the threshold, or outside the base tolerance)
-    # get none, on either side
-    Tmax = L["t_end"] - L["t_first"]
-    fo, fg = np.isfinite(ctx["t"]), np.isfinite(r["t"])
-    gap = np.where(fo & fg, np.abs(np.where(fo & fg, r["t"] - ctx["t"], 0.0)), 0.0)
-    ill = (np.abs(ctx["vpeak"] - 1.0) <= 1e-5) | (fo != fg) | (gap > 1e-4 * Tmax)
+    # backward at the GPU's spike state: random upstream gradient on every
+    # neuron (the penalty gradient T' is added on both sides from the GPU's times)
+    gs = gpu_spike_state(r, B, O, Ho, Wo)
     nrm = 1.0 / (B * Ho * Wo)
-    g = np.random.default_rng(C + O).normal(0.0, 1.0, ctx["t"].shape)
-    _, pg = olosses.temporal_penalty(r["t"], 0.35, 0.8, 0.05, 0.01, nrm)
-    _, gT = olosses.temporal_penalty(ctx["t"], 0.35, 0.8, 0.05, 0.01, nrm)
-    g_gpu = np.where(ill, -pg, g)
-    g_ora = np.where(ill, 0.0, g + gT)
+    g = np.random.default_rng(C + O).normal(0.0, 1.0, gs["t"].shape)
+    _, gT = olosses.temporal_penalty(gs["t"], 0.35, 0.8, 0.05, 0.01, nrm)
     g_t_in = torch.empty_like(r["t_in"])
     g_W = torch.empty_like(r["W"])
-    dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g_gpu.transpose(0, 2, 3, 1)), stride, 1, r["p"],
+    dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g.transpose(0, 2, 3, 1)), stride, 1, r["p"],
                   "bf16", g_t_in, g_W, r["ws"])
     torch.cuda.synchronize()
     assert dstd.device_status(clear=True) == 0
-    fl = {k: ctx[k].reshape(B, -1) for k in ("t", "q", "vdot", "fired")}
-    gw = odstd.solve_backward(fl, g_ora.reshape(B, -1), T, dt, tv, ti, 1.0).reshape(B, O, Ho, Wo, M)
-    gW, gs = onet.conv_what_adjoint(bf16(gw), bf16(s), bf16(L["W"]), stride, 1)
-    ds = odstd.binning(t.reshape(B, -1), T, dt, tv, ti, derivative=True).reshape(gs.shape)
-    gin = np.sum(gs * ds, axis=1)
-    cnt = (~fg).sum((0, 2, 3))
+    fl = {k: gs[k].reshape(B, -1) for k in ("t", "q", "vdot", "fired")}
+    gw = odstd.solve_backward(fl, (g + gT).reshape(B, -1), T, dt, tv, ti, 1.0).reshape(B, O, Ho, Wo, M)
+    gW, gsum = onet.conv_what_adjoint(bf16(gw), bf16(s), bf16(L["W"]), stride, 1)
+    ds = odstd.binning(t.reshape(B, -1), T, dt, tv, ti, derivative=True).reshape(gsum.shape)
+    gin = np.sum(gsum * ds, axis=1)
+    cnt = (~gs["fired"]).sum((0, 2, 3))
     gW = gW - 1e-3 * nrm * cnt[:, None, None, None]
-    assert rel_l2(host(g_W).transpose(0, 3, 1, 2), gW) <= 1e-3
-    assert rel_l2(host(g_t_in).transpose(0, 3, 1, 2), gin) <= 1e-3
+    e_w = rel_l2(host(g_W).transpose(0, 3, 1, 2), gW)
+    e_g = rel_l2(host(g_t_in).transpose(0, 3, 1, 2), gin)
+    assert e_w <= 1e-3 and e_g <= 1e-3, (e_w, e_g)
     assert np.all(host(g_t_in).transpose(0, 3, 1, 2)[~np.isfinite(t)] == 0)

@@ -15,7 +15,8 @@ contraction operands (reading R9):
 * gradients of both networks at full width (batch 4): for every conv layer,
   the weight gradient of one output channel (a sum over every position of
   every image) and the input-time gradient of every channel at two input
-  positions, each within 1e-3 relative L2 of the oracle.
+  positions, each within 1e-3 relative L2 of the oracle's backward at the
+  GPU's spike state (held to the tolerance by the forward checks).
 
 Spike times meet |dt| <= 1e-4 T_max and masks agree outside the 1e-5 band
 around the threshold, except where a neuron's own bound on the bf16
@@ -32,7 +33,7 @@ import pytest
 import torch
 
 from helpers import (bf16, check_bf16_times, conv_neurons, decode_saved, dense_bound_fn, grid_of, neuron_bound_fn,
-                     oracle_forward, receptive_fields, rel_l2)
+                     oracle_forward, rel_l2)
 from oracle import dstd as odstd, losses as olosses, network as onet
 
 pytestmark = pytest.mark.gpu
@@ -187,51 +188,35 @@ def gpu_state(n, l):
     return to_nchw(t), tr(q), tr(vd)
 
 
-def with_gpu_state(ctx, gstate, L):
-    """Neurons whose spike state is ill-conditioned (near the threshold, a
-    firing mismatch, or a time gap beyond the base tolerance) take the GPU's
-    state (t, q, dv^/dt) before the backward: their gradient is then the
-    oracle's formula at the GPU's spike, the rest the oracle's own."""
-    tg, qg, vdg = gstate
-    Tmax = L["t_end"] - L["t_first"]
-    fo, fg = np.isfinite(ctx["t"]), np.isfinite(tg)
-    gap = np.where(fo & fg, np.abs(np.where(fo & fg, tg - ctx["t"], 0.0)), 0.0)
-    ill = (np.abs(ctx["vpeak"] - L["v_th"]) <= 1e-5) | (fo != fg) | (gap > 1e-4 * Tmax)
-    out = dict(ctx)
-    out["t"] = np.where(ill, tg, ctx["t"])
-    out["q"] = np.where(ill, qg, ctx["q"]).astype(int)
-    out["vdot"] = np.where(ill, vdg, ctx["vdot"])
-    out["fired"] = np.isfinite(out["t"])
-    return out, ill
-
-
 def oracle_dW_row(x, L, o, g_up, gstate, nrm):
-    """dC/dW[o] of a conv layer (oracle steps on bf16-rounded operands): the
-    layer's output channel o at every position of every image, its IFT
-    backward with the upstream gradient plus T', the adjoint contraction, and
-    the dead-neuron term."""
+    """dC/dW[o] of a conv layer (oracle steps on bf16-rounded operands) at the
+    GPU's spike state of output channel o (every position of every image):
+    the IFT backward with the upstream gradient plus T', the adjoint
+    contraction, and the dead-neuron term. The state itself is held to the
+    tolerance by the forward checks; the input-time gradient would magnify
+    its legitimate bf16 differences (a difference of dS at adjacent grid
+    points), so both gradients are compared at the same state."""
     T, dt = grid_of(L)
     tv, ti, V = L["tau_v"], L["tau_I"], L["v_th"]
     B, C, H, Wd = x.shape
     W = np.asarray(L["W"], np.float32).astype(np.float64)[o:o + 1]
     s = odstd.binning(x.reshape(B, -1), T, dt, tv, ti).reshape(B, L["M"], C, H, Wd)
-    what = onet.conv_what(bf16(s), bf16(W), L["stride"], L["pad"])
-    _, _, Ho, Wo, M = what.shape
-    fl = odstd.solve(what.reshape(B, Ho * Wo, M), T, dt, tv, ti, V)
-    ctx = {k: fl[k].reshape(B, Ho, Wo) for k in ("t", "q", "vpeak", "vdot", "fired")}
-    ctx, ill = with_gpu_state(ctx, tuple(a[:, o] for a in gstate), L)
-    _, gT = olosses.temporal_penalty(ctx["t"], L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], nrm)
-    flat = {k: ctx[k].reshape(B, -1) for k in ("t", "q", "vdot", "fired")}
+    tg, qg, vdg = (a[:, o] for a in gstate)
+    _, _, Ho, Wo = gstate[0].shape
+    _, gT = olosses.temporal_penalty(tg, L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], nrm)
+    flat = {"t": tg.reshape(B, -1), "q": qg.reshape(B, -1).astype(int), "vdot": vdg.reshape(B, -1),
+            "fired": np.isfinite(tg).reshape(B, -1)}
     gw = odstd.solve_backward(flat, (g_up[:, o] + gT).reshape(B, -1), T, dt, tv, ti, V)
-    gW, _ = onet.conv_what_adjoint(bf16(gw.reshape(B, 1, Ho, Wo, M)), bf16(s), bf16(W), L["stride"], L["pad"])
-    cnt = float((~ctx["fired"]).sum())
-    return gW[0] - L["gamma_q"] * nrm * cnt, int(ill.sum())
+    gW, _ = onet.conv_what_adjoint(bf16(gw.reshape(B, 1, Ho, Wo, -1)), bf16(s), bf16(W), L["stride"], L["pad"])
+    cnt = float((~np.isfinite(tg)).sum())
+    return gW[0] - L["gamma_q"] * nrm * cnt
 
 
 def oracle_input_grad(x, L, b, yi, xi, g_up, gstate, nrm):
-    """dC/dt_in of every channel of input position (b, yi, xi): the output
-    neurons whose receptive field holds it (all channels), their IFT backward,
-    then sum_m (sum_o W dw^) ds/dt (Tab. DSTD_kernels' derivative)."""
+    """dC/dt_in of every channel of input position (b, yi, xi), at the GPU's
+    spike state of the output neurons whose receptive field holds it (all
+    channels): their IFT backward, then sum_m (sum_o W dw^) ds/dt (the
+    derivative of Tab. DSTD_kernels), on bf16-rounded W and dw^."""
     T, dt = grid_of(L)
     tv, ti, V = L["tau_v"], L["tau_I"], L["v_th"]
     W = np.asarray(L["W"], np.float32).astype(np.float64)
@@ -240,15 +225,10 @@ def oracle_input_grad(x, L, b, yi, xi, g_up, gstate, nrm):
     _, _, Ho, Wo = gstate[0].shape
     taps = [(y, xx, yi - y * st + pad, xi - xx * st + pad) for y in range(Ho) for xx in range(Wo)
             if 0 <= yi - y * st + pad < k and 0 <= xi - xx * st + pad < k]
-    rf = receptive_fields(x, k, st, pad, [(b, y, xx) for (y, xx, _, _) in taps])
-    s = odstd.binning(rf, T, dt, tv, ti)                                   # [P, M, K]
-    w2 = bf16(W.reshape(O, -1))
-    what = np.matmul(bf16(s), w2.T).transpose(0, 2, 1)                     # [P, O, M]
-    fl = odstd.solve(what, T, dt, tv, ti, V)
     g = np.stack([g_up[b, :, y, xx] for (y, xx, _, _) in taps])           # [P, O]
-    gs = tuple(np.stack([a[b, :, y, xx] for (y, xx, _, _) in taps]) for a in gstate)
-    ctx, _ = with_gpu_state({k: fl[k] for k in ("t", "q", "vpeak", "vdot", "fired")}, gs, L)
-    _, gT = olosses.temporal_penalty(ctx["t"], L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], nrm)
+    tg, qg, vdg = (np.stack([a[b, :, y, xx] for (y, xx, _, _) in taps]) for a in gstate)
+    _, gT = olosses.temporal_penalty(tg, L["t_head_l"], L["t_tail_l"], L["gamma_head"], L["gamma_tail"], nrm)
+    ctx = {"t": tg, "q": qg.astype(int), "vdot": vdg, "fired": np.isfinite(tg)}
     gw = bf16(odstd.solve_backward(ctx, g + gT, T, dt, tv, ti, V))          # [P, O, M]
     dS = sum(bf16(W[:, :, kh, kw]).T @ gw[p] for p, (_, _, kh, kw) in enumerate(taps))   # [C, M]
     ds = odstd.binning(x[b, :, yi, xi], T, dt, tv, ti, derivative=True)    # [M, C]
@@ -270,10 +250,10 @@ def check_network_gradients(cfg, seed):
         _, O, Ho, Wo = gstate[0].shape
         nrm = 1.0 / (B * Ho * Wo)
         o = int(rng.integers(O))
-        ref, n_ill = oracle_dW_row(x, L, o, g_up, gstate, nrm)
+        ref = oracle_dW_row(x, L, o, g_up, gstate, nrm)
         got = host(n.gW[l])[o].transpose(2, 0, 1)                          # [k, k, C] -> [C, k, k]
         e_w = rel_l2(got, ref)
-        assert e_w <= 1e-3, (l, o, e_w, n_ill)
+        assert e_w <= 1e-3, (l, o, e_w)
         if l == 0:
             worst.append((l, e_w, None))
             continue

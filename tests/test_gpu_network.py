@@ -254,8 +254,9 @@ def test_cfg3_backward_full_size_sampled(math_mode):
     epilogue; several persistent rounds of tiles). Checked against oracle
     steps on 8 sampled rows of dW (each a sum over every sample) and on the
     whole input-time gradient of 2 samples, within 1e-3 relative L2. bf16 runs
-    the oracle on bf16-rounded contraction operands (reading R9). Neurons
-    whose spike state is ill-conditioned take the GPU's state first."""
+    the oracle on bf16-rounded contraction operands (reading R9). The oracle's
+    backward runs at the GPU's spike state (the forward tests hold it to the
+    tolerance)."""
     from paper_2607_14672_gb300 import configs, dstd, net
     from helpers import bf16, decode_saved
     N, M = 16384, 128
@@ -278,38 +279,31 @@ def test_cfg3_backward_full_size_sampled(math_mode):
     tv, ti = L["tau_v"], L["tau_I"]
     tg = host(n.t[0])
     qg, _, vdg = decode_saved(n.saved[0].cpu().numpy(), B, N)
-    Tmax = configs.t_max(L)
 
-    def state(what, b, cols):
-        ctx = odstd.solve(what, T, dt, tv, ti, 1.0)
-        t_gpu, q_gpu, vd_gpu = tg[b][..., cols], qg[b][..., cols], vdg[b][..., cols]
-        fo, fg = np.isfinite(ctx["t"]), np.isfinite(t_gpu)
-        gap = np.where(fo & fg, np.abs(np.where(fo & fg, t_gpu - ctx["t"], 0.0)), 0.0)
-        ill = (np.abs(ctx["vpeak"] - 1.0) <= 1e-5) | (fo != fg) | (gap > 1e-4 * Tmax)
-        ctx["t"] = np.where(ill, t_gpu, ctx["t"])
-        ctx["q"] = np.where(ill, q_gpu, ctx["q"]).astype(int)
-        ctx["vdot"] = np.where(ill, vd_gpu, ctx["vdot"])
-        ctx["fired"] = np.isfinite(ctx["t"])
-        return ctx, int(ill.sum())
+    def state(b, cols):
+        """The GPU's spike state of sample b's neurons cols (held to the
+        tolerance by the forward tests): the input-time gradient magnifies
+        spike-time differences by about T / dt, so the backward is compared
+        at the same state."""
+        t = tg[b][cols][None]
+        return {"t": t, "q": qg[b][cols][None].astype(int), "vdot": vdg[b][cols][None], "fired": np.isfinite(t)}
 
     # dW rows: every sample's contribution
     g = np.random.default_rng(3)
     rows = np.sort(g.choice(N, 8, replace=False))
     gW_ref = np.zeros((len(rows), N))
     for b in range(B):
-        s_b = odstd.binning(t0[b], T, dt, tv, ti)                         # [M, N]
-        sr = rnd(s_b)
-        ctx, _ = state((Wr[rows] @ sr.T)[None], b, rows)
+        sr = rnd(odstd.binning(t0[b], T, dt, tv, ti))                     # [M, N]
+        ctx = state(b, rows)
         gw = odstd.solve_backward(ctx, ctx["fired"].astype(float), T, dt, tv, ti, 1.0)[0]   # [8, M]
         gW_ref += rnd(gw) @ sr
     e_w = rel_l2(host(n.gW[0])[rows], gW_ref)
     assert e_w <= 1e-3, e_w
     # input-time gradient of two whole samples: every neuron's dw^, then W^T
     for b in (0, B - 1):
-        s_b = odstd.binning(t0[b], T, dt, tv, ti)
-        ctx, n_ill = state((Wr @ rnd(s_b).T)[None], b, slice(None))
+        ctx = state(b, slice(None))
         gw = odstd.solve_backward(ctx, ctx["fired"].astype(float), T, dt, tv, ti, 1.0)[0]    # [N, M]
         dS = rnd(gw).T @ Wr                                                # [M, N]
         ref = np.sum(dS * odstd.binning(t0[b], T, dt, tv, ti, derivative=True), axis=0)
         e_g = rel_l2(host(g_in)[b], ref)
-        assert e_g <= 1e-3, (b, e_g, n_ill)
+        assert e_g <= 1e-3, (b, e_g)
