@@ -172,8 +172,16 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
  *  penalty as in dstd_dense_fwd; set p->penalty_norm = 1/(B*Ho*Wo) (App. C.1:
  *          T and Q of conv layers are divided by the spatial size).
  * Tensor-core math modes only (DSTD_MATH_F32 returns DSTD_E_UNSUPPORTED).
- * Padding taps read silent inputs. Images are processed in chunks so the
- * gathered operand stays near 1 GiB; the workspace query accounts for it. */
+ * Padding taps read silent inputs.
+ * In DSTD_MATH_BF16 with C_in and C_out multiples of 64 and M <= 128, the
+ * layer runs as implicit GEMMs: the grid weights of the input (Eq.
+ * DSTD_kernel) are written once, [B, H, W, Mp, C_in] in bf16, and each
+ * filter tap reads them through shifted TMA boxes (no im2col copy); dS is
+ * the transposed convolution of dw^ with the input-time gradient taken in
+ * its epilogue; dW reads the same two arrays. Chunks of whole images keep
+ * that scratch near 4 GiB (dstd_conv_set_chunk_images). Other shapes and
+ * the three-product mode gather the binned input per tap (im2col) in chunks
+ * of whole images near 1 GiB. The workspace query accounts for either. */
 size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k, int stride, int pad,
                                  const dstd_params *p, dstd_math math);
 int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C_in, int C_out, int k, int stride,
@@ -313,6 +321,14 @@ int dstd_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
  * for another value.
  * Process-wide; set it between calls, not while other threads launch. */
 int dstd_set_pair_policy(int policy);
+
+/* Images per chunk of the implicit-GEMM conv layers (bf16, channels in
+ * multiples of 64): 0 (the default) takes as many as fit about 4 GiB of
+ * per-image scratch; n > 0 caps a chunk at n images. It changes the
+ * workspace size that dstd_conv_workspace_bytes returns, so query again
+ * after setting it. Returns the previous value (max_images < 0 only reads
+ * it). Process-wide; set it between calls, not while other threads launch. */
+int dstd_conv_set_chunk_images(int max_images);
 
 /* Kernel timing (tracing). While enabled, the library brackets every kernel
  * it launches with a CUDA event pair on the launching stream and files the

@@ -18,8 +18,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libdstd.so")
-SOURCES = ["dstd_api.cu", "dstd_lif_kernels.cu", "dstd_gemm_simt.cu", "dstd_gemm_tc.cu", "dstd_exact.cu",
-           "dstd_multispike.cu"]
+SOURCES = ["dstd_api.cu", "dstd_lif_kernels.cu", "dstd_gemm_simt.cu", "dstd_gemm_tc.cu", "dstd_conv_tc.cu",
+           "dstd_exact.cu", "dstd_multispike.cu"]
 HEADERS = [os.path.join(CSRC, "dstd_internal.cuh"), os.path.join(CSRC, "dstd_tc_ptx.cuh"),
            os.path.join(ROOT, "include", "dstd.h")]
 GENCODE = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -625,6 +625,128 @@ ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
     return w;
 }
 
+// Implicit-GEMM path (bf16, C_in and C_out multiples of 64): the binned
+// input S [positions][Mp][C_in] is written once per chunk of whole images
+// and read by per-tap TMA boxes (no im2col copy); w^ and dw^ are
+// [positions][Mp][C_out]. Chunks of whole images bound the scratch.
+constexpr size_t kConvImplBudget = 4ull << 30;  // bytes of per-image operands per chunk
+static int g_conv_chunk_images = 0;             // 0: from the budget; else at most this many images per chunk
+
+struct ConvImplWs {
+    __nv_bfloat16 *Wf = nullptr, *Wt = nullptr, *S = nullptr, *dwh = nullptr;
+    float *rowsum = nullptr, *count = nullptr, *what = nullptr;
+    int imgs = 1;
+    size_t bytes = 0;
+};
+
+int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
+    const long long per_img = (long long)g.H * g.W * Mp * g.C * 2 + (long long)g.Ho * g.Wo * Mp * C_out * 4;
+    long long imgs = (long long)(kConvImplBudget / (size_t)per_img);
+    if (g_conv_chunk_images > 0 && imgs > g_conv_chunk_images) imgs = g_conv_chunk_images;
+    if (imgs < 1) imgs = 1;
+    if (imgs > g.B) imgs = g.B;
+    return (int)imgs;
+}
+
+ConvImplWs conv_impl_layout(void *base, const ConvGeom &g, int C_out, int Mp, bool fwd) {
+    ConvImplWs w;
+    Bump b(base);
+    const long long K = (long long)g.k * g.k * g.C;
+    w.imgs = conv_impl_images(g, C_out, Mp);
+    w.rowsum = b.take<float>(C_out);
+    w.count = b.take<float>(C_out);
+    w.Wf = b.take<__nv_bfloat16>((size_t)C_out * K);
+    w.Wt = b.take<__nv_bfloat16>((size_t)C_out * K);
+    w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * g.C);
+    if (fwd)
+        w.what = b.take<float>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
+    else
+        w.dwh = b.take<__nv_bfloat16>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
+    w.bytes = b.off;
+    return w;
+}
+
+bool conv_use_implicit(dstd_math math, const ConvGeom &g, int C_out, int Mp) {
+    return math == DSTD_MATH_BF16 && conv_implicit_supported(g, C_out, Mp);
+}
+
+int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int C_out, const dstd_params *p, int Mp,
+                      float *t_out, void *saved, float *penalty, void *workspace, size_t ws_bytes, cudaStream_t st) {
+    const ConvImplWs ws = conv_impl_layout(workspace, g, C_out, Mp, true);
+    if (ws_bytes < ws.bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, Mp);
+    const long long npos = (long long)g.B * g.Ho * g.Wo;
+    const int K = g.k * g.k * g.C;
+    Saved sv = saved_view(saved, npos, C_out);
+    if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
+    {
+        Timed tm(KK_PREP, st);
+        TRY(cu(launch_prep_weights(W, C_out, K, OpKind::BF16, ws.Wf, nullptr, K, nullptr, nullptr, 0, nullptr, 0,
+                                   ws.rowsum, st)));
+    }
+    for (int img0 = 0; img0 < g.B; img0 += ws.imgs) {
+        const int ni = (g.B - img0) < ws.imgs ? (g.B - img0) : ws.imgs;
+        const long long in_off = (long long)img0 * g.H * g.W * g.C;
+        const long long out_off = (long long)img0 * g.Ho * g.Wo * C_out;
+        const long long P_out = (long long)ni * g.Ho * g.Wo;
+        {
+            Timed tm(KK_BIN, st);
+            TRY(cu(launch_bin_pmc(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+        }
+        {
+            Timed tm(KK_GEMM_FWD, st);
+            TRY(cu(launch_conv_fwd_gemm(g, ni, C_out, c, ws.S, ws.Wf, ws.what, st)));
+        }
+        Timed tm(KK_SCAN, st);
+        TRY(cu(launch_scan_solve(ws.what, (long long)Mp * C_out, 1, C_out, (int)P_out, C_out, c, nullptr, ws.rowsum,
+                                 t_out + out_off, sv.q + out_off, sv.s + out_off, sv.vdot + out_off, penalty, st)));
+    }
+    return DSTD_OK;
+}
+
+int conv_bwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int C_out, const dstd_params *p, int Mp,
+                      const float *t_out, const void *saved, const float *g_t_out, float *g_t_in, float *g_W,
+                      void *workspace, size_t ws_bytes, cudaStream_t st) {
+    const ConvImplWs ws = conv_impl_layout(workspace, g, C_out, Mp, false);
+    if (ws_bytes < ws.bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, Mp);
+    const long long npos = (long long)g.B * g.Ho * g.Wo;
+    const int T = g.k * g.k;
+    Saved sv = saved_view(const_cast<void *>(saved), npos, C_out);
+    const float qcoef = -p->gamma_q * p->penalty_norm;
+    TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)C_out * T * g.C, st)));
+    TRY(cu(cudaMemsetAsync(ws.count, 0, sizeof(float) * (size_t)C_out, st)));
+    if (g_t_in) {
+        Timed tm(KK_PREP, st);
+        TRY(cu(launch_filters_t(W, C_out, T, g.C, ws.Wt, st)));
+    }
+    for (int img0 = 0; img0 < g.B; img0 += ws.imgs) {
+        const int ni = (g.B - img0) < ws.imgs ? (g.B - img0) : ws.imgs;
+        const bool last = img0 + ni >= g.B;
+        const long long in_off = (long long)img0 * g.H * g.W * g.C;
+        const long long out_off = (long long)img0 * g.Ho * g.Wo * C_out;
+        const long long P_out = (long long)ni * g.Ho * g.Wo;
+        {
+            Timed tm(KK_DWHAT, st);
+            TRY(cu(launch_dwhat_pmc(t_out + out_off, sv.q + out_off, sv.s + out_off, sv.vdot + out_off,
+                                    g_t_out ? g_t_out + out_off : nullptr, P_out, C_out, c, ws.dwh, ws.count, st)));
+        }
+        if (g_t_in) {
+            Timed tm(KK_GEMM_DS, st);
+            TRY(cu(launch_conv_ds_gemm(g, ni, C_out, c, ws.dwh, ws.Wt, t_in + in_off, g_t_in + in_off, st)));
+        }
+        {
+            Timed tm(KK_BIN_T, st);
+            TRY(cu(launch_bin_pmc(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+        }
+        Timed tm(KK_GEMM_DW, st);
+        TRY(cu(launch_conv_dw_gemm(g, ni, C_out, c, ws.S, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
+    }
+    return DSTD_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -966,6 +1088,11 @@ size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k
     if (math == DSTD_MATH_F32 || check_math(math, Mp) != DSTD_OK) return 0;
     ConvPlan pl;
     if (conv_plan(B, H, W, C_in, k, stride, pad, Mp, true, C_out, &pl) != DSTD_OK) return 0;
+    if (conv_use_implicit(math, pl.g, C_out, Mp)) {
+        size_t f = conv_impl_layout(nullptr, pl.g, C_out, Mp, true).bytes;
+        size_t g = conv_impl_layout(nullptr, pl.g, C_out, Mp, false).bytes;
+        return f > g ? f : g;
+    }
     size_t f = conv_fwd_layout(nullptr, pl, C_out, Mp, op_of(math)).bytes;
     size_t g = conv_bwd_layout(nullptr, pl, C_out, Mp, bwd_op_of(math), true).bytes;
     return f > g ? f : g;
@@ -983,6 +1110,9 @@ int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C
     if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
     ConvPlan pl;
     TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, C_out, &pl));
+    if (conv_use_implicit(math, pl.g, C_out, Mp))
+        return conv_fwd_implicit(t_in, W, pl.g, C_out, p, Mp, t_out, saved, penalty, workspace, ws_bytes,
+                                 (cudaStream_t)stream);
     const OpKind op = op_of(math);
     if (ws_bytes < conv_fwd_layout(nullptr, pl, C_out, Mp, op).bytes) return DSTD_E_WORKSPACE;
     TRY(device_ok());
@@ -1039,6 +1169,9 @@ int dstd_conv_bwd(const float *t_in, const float *W, const float *t_out, const v
     if (!aligned16(t_in) || !aligned16(W) || !aligned16(workspace) || !aligned16(saved)) return DSTD_E_INVALID;
     ConvPlan pl;
     TRY(conv_plan(B, H, Wd, C_in, k, stride, pad, Mp, true, C_out, &pl));
+    if (conv_use_implicit(math, pl.g, C_out, Mp))
+        return conv_bwd_implicit(t_in, W, pl.g, C_out, p, Mp, t_out, saved, g_t_out, g_t_in, g_W, workspace,
+                                 ws_bytes, (cudaStream_t)stream);
     const OpKind bop = bwd_op_of(math);
     const bool need_gt = g_t_in != nullptr;
     if (ws_bytes < conv_bwd_layout(nullptr, pl, C_out, Mp, bop, need_gt).bytes) return DSTD_E_WORKSPACE;
@@ -1417,9 +1550,17 @@ int dstd_dense_fwd_noalloc(const float *t_in, const float *W, int B, int N_in, i
 
 int dstd_device_status(int clear) {
     if (cudaDeviceSynchronize() != cudaSuccess) return DSTD_E_CUDA;
-    unsigned int s = 0;
+    unsigned int s = 0, s2 = 0;
     if (status_read(&s, clear) != cudaSuccess) return DSTD_E_CUDA;
-    return (s & STATUS_TIMEOUT) ? DSTD_E_TIMEOUT : DSTD_OK;
+    if (conv_status_read(&s2, clear) != cudaSuccess) return DSTD_E_CUDA;
+    return ((s | s2) & STATUS_TIMEOUT) ? DSTD_E_TIMEOUT : DSTD_OK;
+}
+
+int dstd_conv_set_chunk_images(int max_images) {
+    if (max_images < 0) return g_conv_chunk_images;
+    const int prev = g_conv_chunk_images;
+    g_conv_chunk_images = max_images;
+    return prev;
 }
 
 }  // extern "C"

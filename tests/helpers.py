@@ -240,3 +240,14 @@ def dense_bound_fn(ctx, W, layer):
         return bf16_potential_bound(ctx["s"][b], W[i], ctx["q"][b, i], ctx["t"][b, i], T, layer["tau_v"],
                                     layer["tau_I"], kmax)
     return fn
+
+
+def bf16_grad_rel_bound(bound, ref):
+    """The relative L2 allowance a bf16 backward adds to the benchmark spec's 1e-3:
+    ||per-element bound|| / ||reference||. The per-element bound sums, over
+    the dC/dw^ entries that lie within 2^-16 of a bf16 rounding midpoint (the
+    GPU rounds its fp32 value, the oracle its float64 one: they may land on
+    different neighbours), one bf16 step times the other operand's
+    magnitude (and |ds/dt| for the input-time gradient)."""
+    n = np.linalg.norm(np.asarray(ref, float))
+    return float(np.linalg.norm(np.asarray(bound, float)) / n) if n > 0 else 0.0

@@ -128,6 +128,8 @@ def test_null_and_bad_arguments_rejected_on_host(lib):
     assert lib.dstd_split_channels(one, 4, 4, 10, None, 0, None, 0, None) == -1
     assert lib.dstd_split_channels(one, 4, 4, 0, one, 0, one, 0, None) == -1
     assert lib.dstd_set_pair_policy(2) == 0 and lib.dstd_set_pair_policy(0) == 2
+    assert lib.dstd_conv_set_chunk_images(-1) == 0
+    assert lib.dstd_conv_set_chunk_images(3) == 0 and lib.dstd_conv_set_chunk_images(0) == 3
     # multi-tensor AdamW: tensor count, null step buffer, misaligned step buffer, empty tensor, bad beta
     ptrs = (ctypes.c_void_p * 33)(*([256] * 33))
     ns = (ctypes.c_int64 * 33)(*([10] * 33))

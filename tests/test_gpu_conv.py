@@ -151,7 +151,10 @@ def test_conv_chunked_matches_unchunked():
 # tolerance: the input-time gradient is a difference of dS at the two grid
 # points around each input spike (for tau = (inf, inf) exactly (dS_{k+1} -
 # dS_k) / dt), so it magnifies a spike-time difference by about T / dt, and
-# bf16 operands legitimately move spike times by a few 1e-6.
+# bf16 operands legitimately move spike times by a few 1e-6. Likewise a
+# dw^ entry at a bf16 rounding midpoint may round to either neighbour (fp32
+# on the GPU, float64 in the oracle): the tolerance is 1e-3 plus that
+# entry-wise bound (helpers.bf16_grad_rel_bound).
 # ---------------------------------------------------------------------------
 BF16_CASES = [
     # C_in, H, C_out, stride, tau, M
@@ -180,7 +183,8 @@ def gpu_spike_state(r, B, O, Ho, Wo):
 @pytest.mark.parametrize("C,H,O,stride,tau,M", BF16_CASES)
 def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
     from paper_2607_14672_gb300 import dstd
-    from helpers import (bf16, bf16_potential_bound, check_bf16_times, conv_neurons, grid_of, kernel_max)
+    from helpers import (bf16, bf16_ambiguous_ulp, bf16_grad_rel_bound, bf16_potential_bound, check_bf16_times,
+                         conv_neurons, grid_of, kernel_max)
     B = 2
     t, L = conv_case(B, C, H, O, 3, stride, 1, M, tau, seed=7 * C + H + O, wmean=WMEAN64[tau] * 64 / C,
                      gammas=(0.05, 0.01, 1e-3), silent=0.1, t_offset=0.3 * 1.2 / M)
@@ -223,7 +227,44 @@ def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
     gin = np.sum(gsum * ds, axis=1)
     cnt = (~gs["fired"]).sum((0, 2, 3))
     gW = gW - 1e-3 * nrm * cnt[:, None, None, None]
+    # dw^ entries at a bf16 rounding midpoint may round either way (bf16_grad_rel_bound)
+    bW, bs = onet.conv_what_adjoint(bf16_ambiguous_ulp(gw, 2.0 ** -16), np.abs(bf16(s)), np.abs(bf16(L["W"])),
+                                    stride, 1)
+    b_in = np.sum(bs * np.abs(ds), axis=1)
     e_w = rel_l2(host(g_W).transpose(0, 3, 1, 2), gW)
     e_g = rel_l2(host(g_t_in).transpose(0, 3, 1, 2), gin)
-    assert e_w <= 1e-3 and e_g <= 1e-3, (e_w, e_g)
+    a_w, a_g = bf16_grad_rel_bound(bW, gW), bf16_grad_rel_bound(b_in, gin)
+    assert e_w <= 1e-3 + a_w and e_g <= 1e-3 + a_g, (e_w, a_w, e_g, a_g)
     assert np.all(host(g_t_in).transpose(0, 3, 1, 2)[~np.isfinite(t)] == 0)
+
+
+def test_conv_bf16_chunks_agree():
+    """The implicit-GEMM path in chunks of whole images (1, 2 and 3 images
+    per chunk, the last one ragged) against one chunk: the forward of an
+    image does not depend on the chunk it falls in (bitwise), and dW sums
+    the chunks' contributions (fp32 atomics: rounding order only)."""
+    from paper_2607_14672_gb300 import dstd
+    t, L = conv_case(5, 64, 10, 128, 3, 2, 1, 64, (1.0, 0.25), seed=21, wmean=WMEAN64[(1.0, 0.25)],
+                     gammas=(0.05, 0.01, 1e-3), t_offset=0.005)
+    outs = []
+    prev = dstd.conv_set_chunk_images(0)
+    try:
+        for cap in (0, 1, 2, 3):
+            dstd.conv_set_chunk_images(cap)
+            r = run_conv_fwd(t, L, "bf16")
+            g = np.where(np.isfinite(r["t"]), 1.0, 0.0)
+            g_t_in = torch.empty_like(r["t_in"])
+            g_W = torch.empty_like(r["W"])
+            dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g.transpose(0, 2, 3, 1)), 2, 1, r["p"],
+                          "bf16", g_t_in, g_W, r["ws"])
+            torch.cuda.synchronize()
+            assert dstd.device_status(clear=True) == 0
+            outs.append((r["t"], host(g_t_in), host(g_W)))
+    finally:
+        dstd.conv_set_chunk_images(prev)
+    t0, gi0, gw0 = outs[0]
+    assert np.isfinite(t0).mean() > 0.2
+    for tt, gi, gw in outs[1:]:
+        np.testing.assert_array_equal(tt, t0)
+        assert rel_l2(gi, gi0) <= 1e-6
+        assert rel_l2(gw, gw0) <= 1e-5

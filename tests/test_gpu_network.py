@@ -258,7 +258,7 @@ def test_cfg3_backward_full_size_sampled(math_mode):
     backward runs at the GPU's spike state (the forward tests hold it to the
     tolerance)."""
     from paper_2607_14672_gb300 import configs, dstd, net
-    from helpers import bf16, decode_saved
+    from helpers import bf16, bf16_ambiguous_ulp, bf16_grad_rel_bound, decode_saved
     N, M = 16384, 128
     cfg = configs.config3(N, M)
     n = net.DenseNet(cfg, math_mode)
@@ -291,19 +291,25 @@ def test_cfg3_backward_full_size_sampled(math_mode):
     # dW rows: every sample's contribution
     g = np.random.default_rng(3)
     rows = np.sort(g.choice(N, 8, replace=False))
+    # bf16: dw^ entries at a rounding midpoint may round either way (helpers.bf16_grad_rel_bound)
+    amb = (lambda a: bf16_ambiguous_ulp(a, 2.0 ** -16)) if math_mode == "bf16" else (lambda a: np.zeros_like(a))
     gW_ref = np.zeros((len(rows), N))
+    bW = np.zeros((len(rows), N))
     for b in range(B):
         sr = rnd(odstd.binning(t0[b], T, dt, tv, ti))                     # [M, N]
         ctx = state(b, rows)
         gw = odstd.solve_backward(ctx, ctx["fired"].astype(float), T, dt, tv, ti, 1.0)[0]   # [8, M]
         gW_ref += rnd(gw) @ sr
+        bW += amb(gw) @ np.abs(sr)
     e_w = rel_l2(host(n.gW[0])[rows], gW_ref)
-    assert e_w <= 1e-3, e_w
+    assert e_w <= 1e-3 + bf16_grad_rel_bound(bW, gW_ref), e_w
     # input-time gradient of two whole samples: every neuron's dw^, then W^T
     for b in (0, B - 1):
         ctx = state(b, slice(None))
         gw = odstd.solve_backward(ctx, ctx["fired"].astype(float), T, dt, tv, ti, 1.0)[0]    # [N, M]
         dS = rnd(gw).T @ Wr                                                # [M, N]
-        ref = np.sum(dS * odstd.binning(t0[b], T, dt, tv, ti, derivative=True), axis=0)
-        e_g = rel_l2(host(g_in)[b], ref)
-        assert e_g <= 1e-3, (b, e_g)
+        ds = odstd.binning(t0[b], T, dt, tv, ti, derivative=True)
+        ref = np.sum(dS * ds, axis=0)
+        bnd = np.sum((amb(gw).T @ np.abs(Wr)) * np.abs(ds), axis=0) if math_mode == "bf16" else 0.0 * ref
+        e_g, a_g = rel_l2(host(g_in)[b], ref), bf16_grad_rel_bound(bnd, ref)
+        assert e_g <= 1e-3 + a_g, (b, e_g, a_g)
