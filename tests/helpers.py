@@ -120,30 +120,33 @@ def bf16_ambiguous_ulp(x, rel=2.0 ** -18):
     return np.where(amb, u, 0.0)
 
 
-def bf16_potential_bound(s, w, q, t, T, tau_v, tau_I, kmax):
-    """Bound on |v^_gpu - v^_oracle| of bf16-operand neurons from two sources.
+def bf16_potential_bound(s, w, q, t, T, tau_v, tau_I, kmax, v_th=1.0):
+    """Bound on |v^_gpu - v^_oracle| of bf16-operand neurons.
 
     s [n, M, K] grid weights (float64, unrounded), w [n, K] weights, q [n]
-    spike interval (M when silent), t [n] oracle spike time. (1) grid weights
-    that may round to the other bf16 neighbour (``bf16_ambiguous_ulp``); (2)
-    the fp32 accumulation of the exact bf16 x bf16 products: at most
-    (nnz - 1) 2^-23 sum |terms| per grid point with nnz nonzero terms
-    (the standard recursive-summation bound, with 2^-23 allowing truncating
-    adds). Returns (bound at the spike, bound over the whole window).
+    spike interval (M when silent), t [n] oracle spike time. Per grid point:
+    (1) grid weights that may round to the other bf16 neighbour
+    (``bf16_ambiguous_ulp``); (2) the fp32 accumulation of the exact bf16 x
+    bf16 products, at most (nnz - 1) 2^-23 sum |terms| with nnz nonzero
+    terms (the recursive-summation bound; 2^-23 allows truncating adds);
+    (3) the fp32 scan of the state over at most M grid steps, four roundings
+    each: M 2^-22 sum |terms|. At the spike, also the root's stopping
+    tolerance, |v^ - v_th| <= 4e-7 v_th. Returns (bound at the spike, bound
+    over the whole window).
     """
     from oracle import lif
     aw = np.abs(np.asarray(w, float))[:, None, :]
     amb = np.sum(bf16_ambiguous_ulp(s) * aw, -1)                          # [n, M]
     terms = np.abs(bf16(s)) * aw
     nnz = np.count_nonzero(terms, -1)
-    acc = 2.0 ** -23 * np.maximum(nnz - 1, 0) * terms.sum(-1)
-    per_m = amb + acc
     M = s.shape[1]
+    arith = (2.0 ** -23 * np.maximum(nnz - 1, 0) + M * 2.0 ** -22) * terms.sum(-1)
+    per_m = amb + arith
     fired = q < M
     ts = np.where(fired, t, T[0])
     Km = lif.K(ts[:, None] - T[None, :M], tau_v, tau_I)
     upto = np.arange(M)[None, :] <= np.minimum(q, M - 1)[:, None]
-    at_spike = np.sum(np.where(upto & fired[:, None], per_m * Km, 0.0), -1)
+    at_spike = np.sum(np.where(upto & fired[:, None], per_m * Km, 0.0), -1) + 4e-7 * v_th
     return at_spike, kmax * per_m.sum(-1)
 
 
