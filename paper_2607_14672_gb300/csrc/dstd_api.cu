@@ -626,21 +626,24 @@ ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
 }
 
 // Implicit-GEMM path (bf16, C_in and C_out multiples of 64): the binned
-// input S [positions][Mp][C_in] is written once per chunk of whole images
-// and read by per-tap TMA boxes (no im2col copy); w^ and dw^ are
-// [positions][Mp][C_out]. Chunks of whole images bound the scratch.
+// input is one 8-byte record per input spike (grid step and its two
+// weights), from which the forward and dW contractions generate their
+// operand tiles in shared memory (no binned or im2col array in memory); w^
+// and dw^ are [positions][Mp][C_out]. Chunks of whole images bound the
+// scratch.
 constexpr size_t kConvImplBudget = 4ull << 30;  // bytes of per-image operands per chunk
 static int g_conv_chunk_images = 0;             // 0: from the budget; else at most this many images per chunk
 
 struct ConvImplWs {
-    __nv_bfloat16 *Wf = nullptr, *Wt = nullptr, *S = nullptr, *dwh = nullptr;
+    __nv_bfloat16 *Wf = nullptr, *Wt = nullptr, *dwh = nullptr;
+    uint2 *rec = nullptr;
     float *rowsum = nullptr, *count = nullptr, *what = nullptr;
     int imgs = 1;
     size_t bytes = 0;
 };
 
 int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
-    const long long per_img = (long long)g.H * g.W * Mp * g.C * 2 + (long long)g.Ho * g.Wo * Mp * C_out * 4;
+    const long long per_img = (long long)g.H * g.W * g.C * 8 + (long long)g.Ho * g.Wo * Mp * C_out * 4;
     long long imgs = (long long)(kConvImplBudget / (size_t)per_img);
     if (g_conv_chunk_images > 0 && imgs > g_conv_chunk_images) imgs = g_conv_chunk_images;
     if (imgs < 1) imgs = 1;
@@ -657,7 +660,7 @@ ConvImplWs conv_impl_layout(void *base, const ConvGeom &g, int C_out, int Mp, bo
     w.count = b.take<float>(C_out);
     w.Wf = b.take<__nv_bfloat16>((size_t)C_out * K);
     w.Wt = b.take<__nv_bfloat16>((size_t)C_out * K);
-    w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * g.C);
+    w.rec = b.take<uint2>((size_t)w.imgs * g.H * g.W * g.C);
     if (fwd)
         w.what = b.take<float>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
     else
@@ -692,11 +695,11 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         const long long P_out = (long long)ni * g.Ho * g.Wo;
         {
             Timed tm(KK_BIN, st);
-            TRY(cu(launch_bin_pmc(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+            TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
         {
             Timed tm(KK_GEMM_FWD, st);
-            TRY(cu(launch_conv_fwd_gemm(g, ni, C_out, c, ws.S, ws.Wf, ws.what, st)));
+            TRY(cu(launch_conv_fwd_gen(g, ni, C_out, c, ws.rec, ws.Wf, ws.what, st)));
         }
         Timed tm(KK_SCAN, st);
         TRY(cu(launch_scan_solve(ws.what, (long long)Mp * C_out, 1, C_out, (int)P_out, C_out, c, nullptr, ws.rowsum,
@@ -739,10 +742,10 @@ int conv_bwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         }
         {
             Timed tm(KK_BIN_T, st);
-            TRY(cu(launch_bin_pmc(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+            TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
         Timed tm(KK_GEMM_DW, st);
-        TRY(cu(launch_conv_dw_gemm(g, ni, C_out, c, ws.S, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
+        TRY(cu(launch_conv_dw_gen(g, ni, C_out, c, ws.rec, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
     }
     return DSTD_OK;
 }

@@ -318,6 +318,15 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
 cudaError_t launch_conv_dw_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
                                 const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
                                 cudaStream_t st);
+// the binned operand generated on chip: one 8-byte record per input
+// (grid step, bf16 pair of its two weights), then the forward and dW
+// contractions write the operand tiles in shared memory from the records
+cudaError_t launch_bin_rec(const float *t, long long n, const LifConst &c, uint2 *rec, cudaStream_t st);
+cudaError_t launch_conv_fwd_gen(const ConvGeom &g, int ni, int C_out, const LifConst &c, const uint2 *rec,
+                                const __nv_bfloat16 *Wf, float *what, cudaStream_t st);
+cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifConst &c, const uint2 *rec,
+                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
+                               cudaStream_t st);
 cudaError_t conv_status_read(unsigned int *out, int clear);
 // im2col binning of positions [pos0, pos0 + npos): the grid weights of the
 // input spike under each filter tap. !transposed: [npos*Mp, ld] (row (pos, m),
