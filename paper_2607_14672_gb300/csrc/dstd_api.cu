@@ -629,7 +629,7 @@ ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
 // input is one 8-byte record per input spike (grid step and its two
 // weights), from which the forward and dW contractions generate their
 // operand tiles in shared memory (no binned or im2col array in memory); w^
-// and dw^ are [positions][Mp][C_out]. Chunks of whole images bound the
+// is [positions][C_out][Mp] and dw^ [positions][Mp][C_out]. Chunks of whole images bound the
 // scratch.
 constexpr size_t kConvImplBudget = 4ull << 30;  // bytes of per-image operands per chunk
 static int g_conv_chunk_images = 0;             // 0: from the budget; else at most this many images per chunk
@@ -702,7 +702,7 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
             TRY(cu(launch_conv_fwd_gen(g, ni, C_out, c, ws.rec, ws.Wf, ws.what, st)));
         }
         Timed tm(KK_SCAN, st);
-        TRY(cu(launch_scan_solve(ws.what, (long long)Mp * C_out, 1, C_out, (int)P_out, C_out, c, nullptr, ws.rowsum,
+        TRY(cu(launch_scan_solve(ws.what, (long long)Mp * C_out, Mp, 1, (int)P_out, C_out, c, nullptr, ws.rowsum,
                                  t_out + out_off, sv.q + out_off, sv.s + out_off, sv.vdot + out_off, penalty, st)));
     }
     return DSTD_OK;

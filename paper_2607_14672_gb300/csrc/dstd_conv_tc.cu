@@ -1,31 +1,29 @@
 // Convolutional DSTD layer as implicit GEMMs on sm_103a (bf16 operands,
-// tcgen05 + TMA), with no im2col operand.
+// tcgen05), with no im2col operand and no binned array in memory.
 //
 // Layouts (a chunk of whole images, NHWC positions p = (b*H + y)*W + x):
-//   S     [P_in][Mp][C_in]   bf16  grid weights of the input spikes (Eq.
-//                                  DSTD_kernel): row (p, m), channel innermost
-//   w^    [P_out][Mp][C_out] fp32  the forward contraction (Eq. DSTD)
+//   rec   [P_in][C_in]       8 B   per input spike: grid step k and the bf16
+//                                  pair of its two weights (Eq. DSTD_kernel)
+//   w^    [P_out][C_out][Mp] fp32  the forward contraction (Eq. DSTD), the
+//                                  Mp grid steps of a neuron contiguous
 //   dw^   [P_out][Mp][C_out] bf16  dC/dw^ (implicit-function theorem)
 //   Wf    [C_out][k k C_in]  bf16  filters, taps (kh, kw) then channels
 //   Wt    [C_in][k k C_out]  bf16  the same filters transposed
-// A row (p, m) holds 64 channels per 128-byte swizzled line, so one TMA box
-// of a 5-D tensor map (channel, m, x, y, b) = (64, Mp, 1, 1, 1) is the
-// K-major operand slice of one position for one filter tap: the tap shifts
-// the (x, y) coordinates, and coordinates outside the image read zeros,
-// which is the silent padding. Nothing is gathered or expanded in memory.
 //
-//   forward  w^[(p, m), o]  = sum_{tap, c} S[(p + tap), m, c] Wf[o, tap, c]
+//   forward  w^[(p, m), o]  = sum_{tap, c} S[(p + tap), m, c] Wf[o, tap, c]:
+//            the binned operand S is generated in shared memory from the
+//            records of the inputs each tap reads (two nonzeros per input)
 //   dS       dS[(p', m), c] = sum_{tap, o} dw^[(p' - tap) / s, m, o] Wt[c, tap, o]
-//            (the transposed convolution; taps whose output position is not
-//            on the stride grid read zeros), consumed in the epilogue:
-//            dC/dt_j = sum_{m in {k, k+1}} dS[(p', m), c] ds_jm/dt_j
+//            (the transposed convolution; one TMA box of a 5-D tensor map
+//            (channel, m, x, y, b) per position and tap, coordinates outside
+//            the image or off the stride grid read zeros), consumed in the
+//            epilogue: dC/dt_j = sum_{m in {k, k+1}} dS[(p', m), c] ds_jm/dt_j
 //   dW       dW[o, tap, c]  = sum_{(p, m)} dw^[(p, m), o] S[(p + tap), m, c]
-//            (both operands MN-major, K = positions x grid steps, split-K)
+//            (both operands MN-major, S generated on chip, split-K)
 //
-// One thread issues tcgen05.mma (M = 128, N = BN <= 256, K = 16) into one of
-// two TMEM accumulators, so the epilogue of a tile overlaps the MMAs of the
-// next. Every mbarrier wait is bounded; an expired wait sets this unit's
-// status word, the role stops, and the CTA still frees its TMEM.
+// One thread issues tcgen05.mma (M = 128, N = BN <= 256, K = 16) into TMEM
+// accumulators. Every mbarrier wait is bounded; an expired wait sets this
+// unit's status word, the role stops, and the CTA still frees its TMEM.
 #include "dstd_internal.cuh"
 #include "dstd_tc_ptx.cuh"
 
@@ -62,50 +60,6 @@ static int conv_num_sms() {
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<const uint32_t *>(&h);
-}
-
-// ---------------------------------------------------------------------------
-// Binning (Eq. DSTD_kernel) into S [P][Mp][C]: a thread takes 8 channels of
-// one position, computes their grid step and two weights, then writes the
-// position's Mp rows of those channels (16 bytes per row, zeros away from the
-// two grid points; a warp's store covers whole 128-byte lines).
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_bin_pmc(const float *__restrict__ t, long long P, int C, LifConst c,
-                                                 __nv_bfloat16 *__restrict__ S) {
-    const int groups = C >> 3;
-    const long long n = P * groups;
-    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const long long p = idx / groups;
-        const int c0 = (int)(idx - p * groups) * 8;
-        int k[8];
-        float wR[8], wL[8];
-        const float4 a = __ldg(reinterpret_cast<const float4 *>(t + p * C + c0));
-        const float4 b = __ldg(reinterpret_cast<const float4 *>(t + p * C + c0 + 4));
-        const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            k[u] = -100;
-            wR[u] = wL[u] = 0.f;
-            if (isfinite(x[u])) {
-                const BinW w = bin_weights(c, x[u], false);
-                k[u] = w.k;
-                wR[u] = w.wR;
-                wL[u] = w.wL;
-            }
-        }
-        uint4 *dst = reinterpret_cast<uint4 *>(S + p * (long long)c.Mp * C + c0);
-        const int step = C >> 3;  // uint4 per row
-        for (int m = 0; m < c.Mp; ++m) {
-            float v[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-                v[u] = (m < c.M) ? ((m == k[u]) ? wR[u] : ((m == k[u] + 1) ? wL[u] : 0.f)) : 0.f;
-            dst[(long long)m * step] =
-                make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
-                           pack_bf16x2(v[6], v[7]));
-        }
-    }
 }
 
 // ---------------------------------------------------------------------------
@@ -227,7 +181,7 @@ struct ConvGemmArgs {
     int Mp;
     int P_rows;          // row positions (forward: ni Ho Wo; dS: ni H W; dW: K positions ni Ho Wo)
     int n_row, n_col, n_split, kt_per_split, ktiles;
-    float *what;         // forward: w^ [P_out][Mp][C_out]
+    float *what;         // forward: w^ [P_out][C_out][Mp]
     const float *t_in;   // dS: layer input spike times [P_in][C_in]
     float *g_t_in;       // dS: [P_in][C_in], zeroed, accumulated
     float *g_W;          // dW: [C_out][k k C_in], accumulated
@@ -239,12 +193,12 @@ struct ConvGemmArgs {
     LifConst c;
 };
 
-template <int BN, int MODE>  // MODE 0 forward, 1 dS, 2 dW
+template <int BN>
 struct ConvCfg {
-    static constexpr int A_BYTES = 128 * 128;          // 128 rows (or MN) x 64 k of bf16
+    static constexpr int A_BYTES = 128 * 128;          // 128 rows x 64 k of bf16
     static constexpr int B_BYTES = BN * 128;
     static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int EPI_BYTES = MODE == 1 ? CONV_NEPI * 32 * EPI_LD * 4 : 0;
+    static constexpr int EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
     static constexpr int STAGES_RAW = (CONV_SMEM_BUDGET - EPI_BYTES) / STAGE;
     static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
     static constexpr int SMEM = STAGES * STAGE + EPI_BYTES + 1024 + 256;
@@ -262,11 +216,10 @@ __device__ __forceinline__ void pos_decode(int p, int h, int w, int &b, int &y, 
     x = r - y * w;
 }
 
-// Source coordinates (x, y, b) of the A box of row position p and tap
-// (kh, kw). Forward: the input position the tap reads. dS: the output
-// position whose tap reads p, when p - tap is on the stride grid. Anything
-// out of range is left outside the tensor, where TMA reads zeros.
-template <int MODE>
+// Source coordinates (x, y, b) of the dS A box of input position p and tap
+// (kh, kw): the output position whose tap reads p, when p - tap is on the
+// stride grid. Anything out of range is left outside the tensor, where TMA
+// reads zeros.
 __device__ __forceinline__ void conv_src(const ConvGemmArgs &a, int p, int kh, int kw, int &sx, int &sy, int &sb) {
     if (p >= a.P_rows) {
         sx = 0;
@@ -275,39 +228,33 @@ __device__ __forceinline__ void conv_src(const ConvGemmArgs &a, int p, int kh, i
         return;
     }
     int b, y, x;
-    if (MODE == 1) {
-        pos_decode(p, a.H, a.W, b, y, x);
-        const int ny = y + a.pad - kh, nx = x + a.pad - kw;
-        sb = b;
-        if (ny % a.stride != 0 || nx % a.stride != 0) {
-            sx = 0;
-            sy = -1;
-        } else {
-            sy = ny / a.stride;
-            sx = nx / a.stride;
-        }
+    pos_decode(p, a.H, a.W, b, y, x);
+    const int ny = y + a.pad - kh, nx = x + a.pad - kw;
+    sb = b;
+    if (ny % a.stride != 0 || nx % a.stride != 0) {
+        sx = 0;
+        sy = -1;
     } else {
-        pos_decode(p, a.Ho, a.Wo, b, y, x);
-        sb = b;
-        sy = y * a.stride + kh - a.pad;
-        sx = x * a.stride + kw - a.pad;
+        sy = ny / a.stride;
+        sx = nx / a.stride;
     }
 }
 
 // ---------------------------------------------------------------------------
-// Forward and dS: rows (position, m) of 128 per tile (128 / Mp positions),
-// columns BN of the n_total channels; K = k k taps x blocks of 64 channels of
-// the source activation. Persistent: CTA b takes tiles b, b + grid, ...
+// dS with the input-time gradient: rows (input position, m) of 128 per tile
+// (128 / Mp positions), columns BN of the C_in channels; K = k k taps x
+// blocks of 64 output channels of dw^ (the transposed convolution).
+// Persistent: CTA b takes tiles b, b + grid, ...
 //   warp 0  TMA producer (one lane): the 128/Mp position boxes of A, B's box
 //   warp 1  TMEM allocation and MMA issue (one lane)
 //   warps 2-9  epilogue: warp w reads TMEM lane quarter w % 4, 32-column
 //              chunks (w - 2) / 4, +2, ... of the tile
 // Barriers: full/empty per stage; acc_full/acc_empty per accumulator (two).
 // ---------------------------------------------------------------------------
-template <int BN, int MODE>
+template <int BN>
 __global__ void __launch_bounds__(CONV_THREADS, 1)
-    k_conv_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a) {
-    using Cfg = ConvCfg<BN, MODE>;
+    k_conv_ds(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a) {
+    using Cfg = ConvCfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     float *epi = reinterpret_cast<float *>(smem + Cfg::STAGES * Cfg::STAGE);
@@ -321,7 +268,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
     const int ntiles = a.n_row * a.n_col;
     const int Mp = a.Mp;
     const int ppt = 128 / Mp;  // positions per tile
-    const int c_red = MODE == 0 ? a.C_in : a.C_out;
+    const int c_red = a.C_out;
     const int ncb = c_red >> 6;
 
     if (threadIdx.x == 0) {
@@ -351,7 +298,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
                     const int s = it % Cfg::STAGES;
                     const uint32_t ph = (it / Cfg::STAGES) & 1u;
-                    if (!tc::mbar_wait(&empty[s], ph ^ 1u)) {
+                    if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
@@ -362,7 +309,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     const uint32_t st = tc::smem_u32(smem + s * Cfg::STAGE);
                     for (int pp = 0; pp < ppt; ++pp) {
                         int sx, sy, sb;
-                        conv_src<MODE>(a, rt * ppt + pp, kh, kw, sx, sy, sb);
+                        conv_src(a, rt * ppt + pp, kh, kw, sx, sy, sb);
                         tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, sb);
                     }
                     tc::tma_load_2d(st + Cfg::A_BYTES, &mapB, &full[s], tap * c_red + cb * 64, ct * BN);
@@ -371,7 +318,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             // loads still in flight (after an expired wait) land before the CTA exits
             const uint32_t n_drain = it < (uint32_t)Cfg::STAGES ? it : (uint32_t)Cfg::STAGES;
             for (uint32_t i = it - n_drain; i < it; ++i)
-                tc::mbar_wait(&full[i % Cfg::STAGES], (i / Cfg::STAGES) & 1u);
+                tc::mbar_wait_spin(&full[i % Cfg::STAGES], (i / Cfg::STAGES) & 1u);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -382,7 +329,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
                 const uint32_t buf = j & 1u;
                 if (j >= 2) {
-                    if (!tc::mbar_wait(&acc_empty[buf], ((j >> 1) + 1u) & 1u)) {
+                    if (!tc::mbar_wait_spin(&acc_empty[buf], ((j >> 1) + 1u) & 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         break;
                     }
@@ -392,7 +339,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
                     const int s = it % Cfg::STAGES;
                     const uint32_t ph = (it / Cfg::STAGES) & 1u;
-                    if (!tc::mbar_wait(&full[s], ph)) {
+                    if (!tc::mbar_wait_spin(&full[s], ph)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
@@ -431,14 +378,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 float v[32];
                 tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
                 const int col0 = ct * BN + cc * 32;
-                if (MODE == 0) {
-                    if (p < a.P_rows) {
-                        float *dst = a.what + ((long long)p * Mp + (r % Mp)) * a.C_out + col0;
-#pragma unroll
-                        for (int u = 0; u < 32; u += 4)
-                            *reinterpret_cast<float4 *>(dst + u) = make_float4(v[u], v[u + 1], v[u + 2], v[u + 3]);
-                    }
-                } else {
+                {
                     // dS: lane m of the warp holds grid step m_base + m of 32
                     // channels; transpose through shared memory so that lane
                     // u owns channel col0 + u and reads its two grid steps
@@ -471,201 +411,17 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
-// dW: rows = (tap, channel) of the filters in blocks of 64 (two per tile),
-// columns = BN output channels, K = (output position, m) in steps of 64
-// (64 / Mp positions). Both operands MN-major, straight from S and dw^:
-//   A  S at the input position each row block's tap reads (two boxes of 64
-//      channels), 64 k-rows each;
-//   B  dw^ at the output positions (BN / 64 boxes of 64 channels).
-// Split-K over positions; every split adds its tile into g_W atomically
-// (split 0 also adds the dead-neuron term qcoef * count[o]).
-// ---------------------------------------------------------------------------
-template <int BN>
-__global__ void __launch_bounds__(CONV_THREADS, 1)
-    k_conv_dw(const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD, ConvGemmArgs a) {
-    using Cfg = ConvCfg<BN, 2>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + Cfg::STAGES * Cfg::STAGE);
-    uint64_t *empty = full + Cfg::STAGES;
-    uint64_t *acc_full = empty + Cfg::STAGES;
-    uint64_t *acc_empty = acc_full + 2;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int ntiles = a.n_row * a.n_col * a.n_split;
-    const int Mp = a.Mp;
-    const int kpos = 64 / Mp;        // positions per K step
-    const int ncb = a.C_in >> 6;     // channel blocks per tap
-    const int nrb = a.k * a.k * ncb; // row blocks of 64
-    const int Ktot = a.k * a.k * a.C_in;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < Cfg::STAGES; ++s) {
-            tc::mbar_init(&full[s], 1);
-            tc::mbar_init(&empty[s], 1);
-        }
-        for (int u = 0; u < 2; ++u) {
-            tc::mbar_init(&acc_full[u], 1);
-            tc::mbar_init(&acc_empty[u], CONV_NEPI);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    }
-    if (warp == 1) tc::tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
-
-    // tile t -> (split, row tile, column tile); K steps [kt0, kt0 + nkt)
-    auto decode = [&](int t, int &rt, int &ct, int &kt0, int &nkt) {
-        const int per = a.n_row * a.n_col;
-        const int sp = t / per, rem = t - sp * per;
-        rt = rem / a.n_col;
-        ct = rem - rt * a.n_col;
-        kt0 = sp * a.kt_per_split;
-        nkt = a.ktiles - kt0;
-        if (nkt > a.kt_per_split) nkt = a.kt_per_split;
-    };
-
-    if (warp == 0) {
-        if (lane == 0) {
-            uint32_t it = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-                int rt, ct, kt0, nkt;
-                decode(t, rt, ct, kt0, nkt);
-                for (int i = 0; i < nkt; ++i, ++it) {
-                    const int s = it % Cfg::STAGES;
-                    const uint32_t ph = (it / Cfg::STAGES) & 1u;
-                    if (!tc::mbar_wait(&empty[s], ph ^ 1u)) {
-                        conv_set_status(STATUS_TIMEOUT);
-                        ok = false;
-                        break;
-                    }
-                    tc::mbar_expect_tx(&full[s], (uint32_t)Cfg::STAGE);
-                    const uint32_t st = tc::smem_u32(smem + s * Cfg::STAGE);
-                    const int kt = kt0 + i;
-                    for (int kp = 0; kp < kpos; ++kp) {
-                        const int p = kt * kpos + kp;  // output position of these k-rows
-                        int b, y, x;
-                        const bool in = p < a.P_rows;
-                        if (in) pos_decode(p, a.Ho, a.Wo, b, y, x);
-                        // A: the two row blocks' taps at input positions
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const int rb = 2 * rt + h;
-                            int sx = 0, sy = 0, sbi = a.ni, cb = 0;
-                            if (in && rb < nrb) {
-                                const int tap = rb / ncb;
-                                cb = rb - tap * ncb;
-                                const int kh = tap / a.k, kw = tap - kh * a.k;
-                                sx = x * a.stride + kw - a.pad;
-                                sy = y * a.stride + kh - a.pad;
-                                sbi = b;
-                            }
-                            tma_load_5d(st + h * 8192 + kp * Mp * 128, &mapS, &full[s], cb * 64, 0, sx, sy, sbi);
-                        }
-                        // B: dw^ of the output position, BN / 64 channel boxes
-                        for (int g = 0; g < BN / 64; ++g)
-                            tma_load_5d(st + Cfg::A_BYTES + g * 8192 + kp * Mp * 128, &mapD, &full[s],
-                                        ct * BN + g * 64, 0, in ? x : 0, in ? y : 0, in ? b : a.ni);
-                    }
-                }
-            }
-            const uint32_t n_drain = it < (uint32_t)Cfg::STAGES ? it : (uint32_t)Cfg::STAGES;
-            for (uint32_t i = it - n_drain; i < it; ++i)
-                tc::mbar_wait(&full[i % Cfg::STAGES], (i / Cfg::STAGES) & 1u);
-        }
-        __syncwarp();
-    } else if (warp == 1) {
-        if (lane == 0) {
-            constexpr uint32_t idesc = idesc_bf16(128, BN, true, true);
-            uint32_t it = 0, j = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
-                int rt, ct, kt0, nkt;
-                decode(t, rt, ct, kt0, nkt);
-                const uint32_t buf = j & 1u;
-                if (j >= 2) {
-                    if (!tc::mbar_wait(&acc_empty[buf], ((j >> 1) + 1u) & 1u)) {
-                        conv_set_status(STATUS_TIMEOUT);
-                        break;
-                    }
-                    tc::tc_fence_after();
-                }
-                const uint32_t acc = tmem + buf * BN;
-                for (int i = 0; i < nkt; ++i, ++it) {
-                    const int s = it % Cfg::STAGES;
-                    const uint32_t ph = (it / Cfg::STAGES) & 1u;
-                    if (!tc::mbar_wait(&full[s], ph)) {
-                        conv_set_status(STATUS_TIMEOUT);
-                        ok = false;
-                        break;
-                    }
-                    tc::tc_fence_after();
-                    const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE);
-                    const uint32_t sbb = sa + Cfg::A_BYTES;
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        tc::mma_bf16(acc, tc::sdesc_sw128_mn(sa + kk * 2048, 8192), tc::sdesc_sw128_mn(sbb + kk * 2048, 8192),
-                                     idesc, (i > 0 || kk > 0) ? 1u : 0u);
-                    tc::mma_commit(&empty[s]);
-                }
-                if (ok) tc::mma_commit(&acc_full[buf]);
-            }
-        }
-        __syncwarp();
-    } else {
-        const int quarter = warp & 3, group = (warp - 2) >> 2;
-        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-        const int r = quarter * 32 + lane;
-        uint32_t j = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
-            int rt, ct, kt0, nkt;
-            decode(t, rt, ct, kt0, nkt);
-            const uint32_t buf = j & 1u;
-            if (!tc::mbar_wait_sleep(&acc_full[buf], (j >> 1) & 1u)) {
-                conv_set_status(STATUS_TIMEOUT);
-                break;
-            }
-            tc::tc_fence_after();
-            const int kidx = rt * 128 + r;  // (tap, channel) of this lane
-            const bool first = kt0 == 0;
-            for (int cc = group; cc < BN / 32; cc += 2) {
-                float v[32];
-                tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
-                if (kidx < Ktot) {
-                    const int o0 = ct * BN + cc * 32;
-#pragma unroll
-                    for (int u = 0; u < 32; ++u) {
-                        const float add = (first && a.count) ? a.qcoef * a.count[o0 + u] : 0.f;
-                        atomicAdd(a.g_W + (long long)(o0 + u) * Ktot + kidx, v[u] + add);
-                    }
-                }
-            }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
-        }
-    }
-    tc::tc_fence_before();
-    __syncthreads();
-    if (warp == 1) tc::tmem_dealloc(tmem, Cfg::TMEM_COLS);
-}
-
-// ---------------------------------------------------------------------------
 // Binned operand generated on chip (the compact support of K_DSTD: each
 // input spike has two nonzero grid weights among Mp). The binning writes
 // one 8-byte record per input, rec[p][c] = (grid step k, bf16 pair (w at
-// T_k, w at T_{k+1})), k = -128 when silent. Per K step the TMA producer
-// copies the records the tile needs (64 per position and tap) into the stage;
-// four generator warps then write each record's two nonzeros into the
-// swizzled A tile that the tensor core reads. Each thread owns fixed columns
-// of the tile, so before writing it erases the two entries it wrote the last
-// time it used that stage (all stages start zeroed): 4 two-byte shared
-// stores per input instead of 16 KB of operand per K step from L2.
+// T_k, w at T_{k+1})), k = -128 when silent. Generator warps load the
+// records a K step needs (64 consecutive per position and tap: a warp reads
+// 256 contiguous bytes) several K steps ahead and write each record's two
+// nonzeros into the swizzled A tile that the tensor core reads. Each thread
+// owns fixed columns of the tile, so before writing it erases the two
+// entries it wrote the last time it used that stage (all stages start
+// zeroed): 4 two-byte shared stores per input instead of 16 KB of operand
+// per K step from L2.
 // ---------------------------------------------------------------------------
 constexpr int REC_SILENT = -128;
 
@@ -682,12 +438,11 @@ __global__ void __launch_bounds__(256) k_bin_rec(const float *__restrict__ t, lo
     }
 }
 
-__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map, uint64_t *bar, int c, int x, int y,
-                                            int b) {
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint64_t *bar, int c, int m, int p) {
     asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
-        "l"((uint64_t)map), "r"(c), "r"(x), "r"(y), "r"(b), "r"(tc::smem_u32(bar))
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(c), "r"(m), "r"(p), "r"(tc::smem_u32(bar))
         : "memory");
 }
 
@@ -730,36 +485,43 @@ __device__ __forceinline__ void gen_put_mn(uint32_t tile, int kr0, int c, int ko
     }
 }
 
-constexpr int GEN_WARPS = 4;
-constexpr int GEN_THREADS = (2 + CONV_NEPI + GEN_WARPS) * 32;  // 448
+constexpr int GEN_WARPS = 4;                                    // per generator group (one K step)
+constexpr int GEN_THREADS = (2 + CONV_NEPI + GEN_WARPS) * 32;  // 448: dW, one group
+constexpr int FWD_GEN_GROUPS = 4;                               // forward: K steps generated at once
+constexpr int FWD_THREADS = (2 + CONV_NEPI + GEN_WARPS * FWD_GEN_GROUPS) * 32;  // 832
 
-// shared-memory plan of the generated-operand kernels: per stage the A tile,
-// the B tile (unless resident) and the records; the stage count and the
+// shared-memory plan of the generated-operand forward: per stage the A tile
+// and the B tile (unless the filters are resident); the stage count and the
 // resident bytes are chosen on the host (ConvGemmArgs::nst, ::res_bytes)
 template <int BN, bool RES>
 struct GenFwdCfg {
     static constexpr int A_BYTES = 128 * 128;
     static constexpr int B_BYTES = RES ? 0 : BN * 128;
-    static constexpr int R_BYTES = 2048;            // up to 4 positions x 64 records x 8 B
-    static constexpr int STAGE = A_BYTES + B_BYTES + R_BYTES;
+    static constexpr int STAGE = A_BYTES + B_BYTES;
     static constexpr int MAX_STAGES = 8;
     static constexpr int PREV_BYTES = MAX_STAGES * 256 * 2;  // last grid step written, per stage and slot
     static constexpr uint32_t TMEM_COLS = 2 * BN;
-    static __host__ __device__ int smem(int nst, int res_bytes) { return nst * STAGE + res_bytes + PREV_BYTES + 1024 + 256; }
+    static __host__ __device__ int smem(int nst, int res_bytes) {
+        return nst * STAGE + res_bytes + PREV_BYTES + 1024 + 256;
+    }
 };
 constexpr int GEN_SMEM_MAX = 225 * 1024;
+constexpr int GEN_AHEAD = 8;  // K steps of records a generator thread loads ahead
 
-// Forward with the binned operand generated on chip. Warps: 0 TMA (records,
-// and the filter tiles unless RES: then all of them once, resident), 1 MMA,
-// 2-9 epilogue (w^ rows as k_conv_gemm), 10-13 generators.
+// Forward with the binned operand generated on chip. Warps: 0 TMA (the
+// filter tiles per K step, or all of them once when RES), 1 MMA, 2-9
+// epilogue (w^ rows), 10-13 generators. A generator thread owns slots
+// (position pp, channel c) g and g + 128 of the tile; it loads their records
+// GEN_AHEAD K steps ahead (a warp reads 32 consecutive records), waits until
+// the stage's previous MMAs are done, writes the A tile, and arrives.
 template <int BN, bool RES>
-__global__ void __launch_bounds__(GEN_THREADS, 1)
-    k_conv_fwd_gen(const __grid_constant__ CUtensorMap mapR, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a) {
+__global__ void __launch_bounds__(FWD_THREADS, 1)
+    k_conv_fwd_gen(const uint2 *__restrict__ rec, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a) {
     using Cfg = GenFwdCfg<BN, RES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int NST = a.nst;
-    uint8_t *bres = smem + NST * Cfg::STAGE;                           // resident filters (RES)
+    uint8_t *bres = smem + NST * Cfg::STAGE;  // resident filters (RES)
     int16_t *prevk = reinterpret_cast<int16_t *>(bres + a.res_bytes);
     uint64_t *full_t = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(prevk) + Cfg::PREV_BYTES);
     uint64_t *full_a = full_t + Cfg::MAX_STAGES;
@@ -775,7 +537,6 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
     const int ppt = 128 / Mp;
     const int ncb = a.C_in >> 6;
 
-    // zero every stage's A tile and mark every slot unwritten
     for (int i = threadIdx.x; i < NST * (Cfg::A_BYTES / 16); i += blockDim.x) {
         const int st = i / (Cfg::A_BYTES / 16), off = i - st * (Cfg::A_BYTES / 16);
         reinterpret_cast<uint4 *>(smem + st * Cfg::STAGE)[off] = make_uint4(0u, 0u, 0u, 0u);
@@ -810,37 +571,30 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
                     const int tap = kt / ncb, cb = kt - tap * ncb;
                     tc::tma_load_2d(tc::smem_u32(bres + kt * BN * 128), &mapB, bres_full, tap * a.C_in + cb * 64, 0);
                 }
-            }
-            uint32_t it = 0;
-            bool ok = true;
-            const uint32_t tx = (uint32_t)(ppt * 512 + Cfg::B_BYTES);
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-                const int rt = t / a.n_col, ct = t - rt * a.n_col;
-                for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
-                    if (!tc::mbar_wait(&empty[s], ph ^ 1u)) {
-                        conv_set_status(STATUS_TIMEOUT);
-                        ok = false;
-                        break;
+                tc::mbar_wait_spin(bres_full, 0);
+            } else {
+                uint32_t it = 0;
+                bool ok = true;
+                for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                    const int ct = t % a.n_col;
+                    for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
+                        const int s = it % NST;
+                        const uint32_t ph = (it / NST) & 1u;
+                        if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
+                            conv_set_status(STATUS_TIMEOUT);
+                            ok = false;
+                            break;
+                        }
+                        tc::mbar_expect_tx(&full_t[s], (uint32_t)Cfg::B_BYTES);
+                        const int tap = kt / ncb, cb = kt - tap * ncb;
+                        tc::tma_load_2d(tc::smem_u32(smem + s * Cfg::STAGE + Cfg::A_BYTES), &mapB, &full_t[s],
+                                        tap * a.C_in + cb * 64, ct * BN);
                     }
-                    tc::mbar_expect_tx(&full_t[s], tx);
-                    const int tap = kt / ncb, cb = kt - tap * ncb;
-                    const int kh = tap / a.k, kw = tap - kh * a.k;
-                    const uint32_t st = tc::smem_u32(smem + s * Cfg::STAGE);
-                    const uint32_t sr = st + Cfg::A_BYTES + Cfg::B_BYTES;
-                    for (int pp = 0; pp < ppt; ++pp) {
-                        int sx, sy, sb;
-                        conv_src<0>(a, rt * ppt + pp, kh, kw, sx, sy, sb);
-                        tma_load_4d(sr + pp * 512, &mapR, &full_t[s], 2 * cb * 64, sx, sy, sb);
-                    }
-                    if (!RES) tc::tma_load_2d(st + Cfg::A_BYTES, &mapB, &full_t[s], tap * a.C_in + cb * 64, ct * BN);
                 }
+                const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
+                for (uint32_t i = it - n_drain; i < it; ++i)
+                    tc::mbar_wait_spin(&full_t[i % NST], (i / NST) & 1u);
             }
-            const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
-            for (uint32_t i = it - n_drain; i < it; ++i)
-                tc::mbar_wait(&full_t[i % NST], (i / NST) & 1u);
-            if (RES) tc::mbar_wait(bres_full, 0);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -848,14 +602,14 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
             constexpr uint32_t idesc = idesc_bf16(128, BN, false, false);
             uint32_t it = 0, j = 0;
             bool ok = true;
-            if (RES && !tc::mbar_wait(bres_full, 0)) {
+            if (RES && !tc::mbar_wait_spin(bres_full, 0)) {
                 conv_set_status(STATUS_TIMEOUT);
                 ok = false;
             }
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
                 const uint32_t buf = j & 1u;
                 if (j >= 2) {
-                    if (!tc::mbar_wait(&acc_empty[buf], ((j >> 1) + 1u) & 1u)) {
+                    if (!tc::mbar_wait_spin(&acc_empty[buf], ((j >> 1) + 1u) & 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         break;
                     }
@@ -865,7 +619,7 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
                 for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
                     const int s = it % NST;
                     const uint32_t ph = (it / NST) & 1u;
-                    if (!tc::mbar_wait(&full_t[s], ph) || !tc::mbar_wait(&full_a[s], ph)) {
+                    if ((!RES && !tc::mbar_wait_spin(&full_t[s], ph)) || !tc::mbar_wait_spin(&full_a[s], ph)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
@@ -902,10 +656,11 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
                 float v[32];
                 tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
                 if (p < a.P_rows) {
-                    float *dst = a.what + ((long long)p * Mp + (r % Mp)) * a.C_out + ct * BN + cc * 32;
+                    // w^ [p][o][m]: for each neuron o the warp's 32 lanes hold 32
+                    // consecutive grid steps, one 128-byte line per store
+                    float *dst = a.what + ((long long)p * a.C_out + ct * BN + cc * 32) * Mp + (r % Mp);
 #pragma unroll
-                    for (int u = 0; u < 32; u += 4)
-                        *reinterpret_cast<float4 *>(dst + u) = make_float4(v[u], v[u + 1], v[u + 2], v[u + 3]);
+                    for (int u = 0; u < 32; ++u) __stcs(dst + (long long)u * Mp, v[u]);
                 }
             }
             tc::tc_fence_before();
@@ -913,34 +668,95 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
             if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
         }
     } else {
-        // generators: thread g owns slots g, g + 128, ... (slot = position
-        // pp x 64 + channel c of the tile) in every stage
-        const int g = threadIdx.x - (2 + CONV_NEPI) * 32;
+        // generator group grp (4 warps) takes K steps it = grp, grp + 4, ...;
+        // the stage count is a multiple of 4, so a stage always belongs to the
+        // same group and each of its slots to the same thread
+        const int gw = warp - (2 + CONV_NEPI);
+        const int grp = gw / GEN_WARPS;
+        const int g = (gw % GEN_WARPS) * 32 + lane;
         const int nslots = ppt * 64;
-        uint32_t it = 0;
+        uint2 q[GEN_AHEAD][2];
+        // the K step whose records load next (tile la_t, step la_kt), and the
+        // decoded positions of this thread's two slots in tile la_t
+        int la_t = blockIdx.x, la_kt = grp;
+        while (la_kt >= a.ktiles && la_t < ntiles) {
+            la_kt -= a.ktiles;
+            la_t += gridDim.x;
+        }
+        int pc_t = -1, pb[2] = {0, 0}, py[2] = {0, 0}, px[2] = {0, 0};
+        auto load_next = [&](uint2(&dst)[2]) {
+            if (la_t < ntiles && la_t != pc_t) {
+                pc_t = la_t;
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int p = (la_t / a.n_col) * ppt + ((g + u * 128) >> 6);
+                    if (p < a.P_rows) pos_decode(p, a.Ho, a.Wo, pb[u], py[u], px[u]);
+                    else pb[u] = a.ni;
+                }
+            }
+            const int tap = la_kt / ncb, cb = la_kt - tap * ncb;
+            const int kh = tap / a.k, kw = tap - kh * a.k;
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int slot = g + u * 128;
+                dst[u] = make_uint2((uint32_t)REC_SILENT, 0u);
+                const int sy = py[u] * a.stride + kh - a.pad, sx = px[u] * a.stride + kw - a.pad;
+                if (la_t < ntiles && slot < nslots && pb[u] < a.ni && sx >= 0 && sx < a.W && sy >= 0 && sy < a.H)
+                    dst[u] = __ldg(rec + (((long long)pb[u] * a.H + sy) * a.W + sx) * a.C_in + cb * 64 + (slot & 63));
+            }
+            la_kt += FWD_GEN_GROUPS;
+            while (la_kt >= a.ktiles && la_t < ntiles) {
+                la_kt -= a.ktiles;
+                la_t += gridDim.x;
+            }
+        };
+#pragma unroll
+        for (int d = 0; d < GEN_AHEAD; ++d) load_next(q[d]);
+        uint32_t it = grp;
+        int cur_t = blockIdx.x, cur_kt = grp;
+        while (cur_kt >= a.ktiles && cur_t < ntiles) {
+            cur_kt -= a.ktiles;
+            cur_t += gridDim.x;
+        }
         bool ok = true;
-        for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-            for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
-                const int s = it % NST;
-                const uint32_t ph = (it / NST) & 1u;
-                if (!tc::mbar_wait(&full_t[s], ph)) {
-                    conv_set_status(STATUS_TIMEOUT);
-                    ok = false;
-                    break;
+        while (cur_t < ntiles && ok) {
+#pragma unroll
+            for (int d = 0; d < GEN_AHEAD; ++d) {
+                if (cur_t < ntiles && ok) {
+                    const int s = it % NST;
+                    const uint32_t ph = (it / NST) & 1u;
+                    int w_ok = 1;
+                    // generators run ahead of the MMAs: park (suspend hint) rather
+                    // than poll, which would take shared-memory cycles from the
+                    // tensor core's operand reads
+                    if (lane == 0) w_ok = tc::mbar_wait(&empty[s], ph ^ 1u) ? 1 : 0;
+                    w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+                    if (!w_ok) {
+                        if (lane == 0) conv_set_status(STATUS_TIMEOUT);
+                        ok = false;
+                    } else {
+                        const uint32_t tile = tc::smem_u32(smem + s * Cfg::STAGE);
+#pragma unroll
+                        for (int u = 0; u < 2; ++u) {
+                            const int slot = g + u * 128;
+                            if (slot < nslots) {
+                                int16_t *pk = prevk + s * 256 + slot;
+                                gen_put(tile, (slot >> 6) * Mp, slot & 63, (int)*pk, q[d][u], a.c.M);
+                                *pk = (int16_t)(int)q[d][u].x;
+                            }
+                        }
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(&full_a[s]);
+                        load_next(q[d]);
+                        it += FWD_GEN_GROUPS;
+                        cur_kt += FWD_GEN_GROUPS;
+                        while (cur_kt >= a.ktiles && cur_t < ntiles) {
+                            cur_kt -= a.ktiles;
+                            cur_t += gridDim.x;
+                        }
+                    }
                 }
-                uint8_t *st = smem + s * Cfg::STAGE;
-                const uint32_t tile = tc::smem_u32(st);
-                const uint2 *rec = reinterpret_cast<const uint2 *>(st + Cfg::A_BYTES + Cfg::B_BYTES);
-                for (int slot = g; slot < nslots; slot += GEN_WARPS * 32) {
-                    const int pp = slot >> 6, c = slot & 63;
-                    const uint2 r = rec[slot];
-                    int16_t *pk = prevk + s * 256 + slot;
-                    gen_put(tile, pp * Mp, c, (int)*pk, r, a.c.M);
-                    *pk = (int16_t)(int)r.x;
-                }
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                __syncwarp();
-                if (lane == 0) tc::mbar_arrive(&full_a[s]);
             }
         }
     }
@@ -952,38 +768,60 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
 // ---------------------------------------------------------------------------
 // dW with the binned operand generated on chip: a CTA tile is G row tiles
 // (128 filter rows (tap, channel) each, two 64-channel row blocks) by BN
-// output channels over a range of K = (output position, m). Per K step it
-// stages one dw^ tile (MN-major, by TMA) and the records of the G row
-// tiles' inputs, the generators write the G MN-major A tiles, and G MMAs
-// (one TMEM accumulator each) reuse the dw^ tile. Split-K over positions;
-// each split adds its tiles into g_W atomically (split 0 also the
-// dead-neuron term).
+// output channels over a range of K = (output position, m). Per K step the
+// TMA producer stages one dw^ tile (MN-major: BN / 64 boxes of a 3-D view
+// (channel, m, position), 64 k-rows each); the generators write the G
+// MN-major A tiles from the records of the G row tiles' inputs (loaded
+// DW_AHEAD K steps ahead), and G MMAs (one TMEM accumulator each) reuse the
+// dw^ tile. Split-K over positions; each split adds its tiles into g_W
+// atomically (split 0 also the dead-neuron term).
 // ---------------------------------------------------------------------------
 constexpr int DWG_MAX_G = 8;
 constexpr int DWG_MAX_STAGES = 4;
+constexpr int DW_AHEAD = 2;
+constexpr int DW_MAX_SPT = 8;   // slots per generator thread: G kpos <= 8
+constexpr int DW_GEN_GROUPS = 2;  // K steps generated at once
+constexpr int DW_THREADS = (2 + CONV_NEPI + GEN_WARPS * DW_GEN_GROUPS) * 32;  // 576
 
 template <int BN>
 struct GenDwCfg {
     static constexpr int B_BYTES = BN * 128;
-    static __host__ __device__ int stage(int G, int kpos) { return G * (128 * 128 + 2 * kpos * 512) + B_BYTES; }
+    static __host__ __device__ int stage(int G) { return G * 128 * 128 + B_BYTES; }
     static __host__ __device__ int prev_bytes(int nst, int G, int kpos) { return nst * G * 128 * kpos * 2; }
     static __host__ __device__ int smem(int nst, int G, int kpos) {
-        return nst * stage(G, kpos) + prev_bytes(nst, G, kpos) + 1024 + 256;
+        return nst * stage(G) + prev_bytes(nst, G, kpos) + 1024 + 256;
     }
 };
 
+// record of slot (row block u of the group, position kp, channel c) at K step kt
+__device__ __forceinline__ uint2 dw_record(const ConvGemmArgs &a, const uint2 *__restrict__ rec, int rg, int G, int kt,
+                                           int u, int kp, int c) {
+    const int kpos = 64 / a.Mp;
+    const int ncb = a.C_in >> 6;
+    const int rb = rg * 2 * G + u;
+    const int p = kt * kpos + kp;
+    if (p >= a.P_rows || rb >= a.k * a.k * ncb) return make_uint2((uint32_t)REC_SILENT, 0u);
+    int b, y, x;
+    pos_decode(p, a.Ho, a.Wo, b, y, x);
+    const int tap = rb / ncb, cb = rb - tap * ncb;
+    const int kh = tap / a.k, kw = tap - kh * a.k;
+    const int sx = x * a.stride + kw - a.pad, sy = y * a.stride + kh - a.pad;
+    if (sx < 0 || sx >= a.W || sy < 0 || sy >= a.H) return make_uint2((uint32_t)REC_SILENT, 0u);
+    return __ldg(rec + (((long long)b * a.H + sy) * a.W + sx) * a.C_in + cb * 64 + c);
+}
+
 template <int BN>
-__global__ void __launch_bounds__(GEN_THREADS, 1)
-    k_conv_dw_gen(const __grid_constant__ CUtensorMap mapR, const __grid_constant__ CUtensorMap mapD, ConvGemmArgs a) {
+__global__ void __launch_bounds__(DW_THREADS, 1)
+    k_conv_dw_gen(const uint2 *__restrict__ rec, const __grid_constant__ CUtensorMap mapD, ConvGemmArgs a) {
     using Cfg = GenDwCfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int G = a.groups, NST = a.nst;
     const int Mp = a.Mp;
     const int kpos = 64 / Mp;
-    const int STG = Cfg::stage(G, kpos);
+    const int STG = Cfg::stage(G);
     const int a_bytes = G * 128 * 128;
-    const int slots = G * 128 * kpos;                 // (row tile, row block, position, channel)
+    const int slots = G * 128 * kpos;  // (row block u of the group, position kp, channel c)
     int16_t *prevk = reinterpret_cast<int16_t *>(smem + NST * STG);
     uint64_t *full_t = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(prevk) + Cfg::prev_bytes(NST, G, kpos));
     uint64_t *full_a = full_t + DWG_MAX_STAGES;
@@ -993,10 +831,8 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n_grp = a.n_row;                        // row groups of G row tiles
+    const int n_grp = a.n_row;  // row groups of G row tiles
     const int ntiles = n_grp * a.n_col * a.n_split;
-    const int ncb = a.C_in >> 6;
-    const int nrb = a.k * a.k * ncb;
     const int Ktot = a.k * a.k * a.C_in;
     uint32_t tcols = 32;
     while ((int)tcols < G * BN) tcols <<= 1;
@@ -1037,48 +873,25 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
         if (lane == 0) {
             uint32_t it = 0;
             bool ok = true;
-            const uint32_t tx = (uint32_t)(G * 2 * kpos * 512 + Cfg::B_BYTES);
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
                 int rg, ct, kt0, nkt;
                 decode(t, rg, ct, kt0, nkt);
                 for (int i = 0; i < nkt; ++i, ++it) {
                     const int s = it % NST;
                     const uint32_t ph = (it / NST) & 1u;
-                    if (!tc::mbar_wait(&empty[s], ph ^ 1u)) {
+                    if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
                     }
-                    tc::mbar_expect_tx(&full_t[s], tx);
-                    const uint32_t st = tc::smem_u32(smem + s * STG);
-                    const uint32_t sr = st + a_bytes + Cfg::B_BYTES;
-                    const int kt = kt0 + i;
-                    for (int kp = 0; kp < kpos; ++kp) {
-                        const int p = kt * kpos + kp;
-                        const bool in = p < a.P_rows;
-                        int b = 0, y = 0, x = 0;
-                        if (in) pos_decode(p, a.Ho, a.Wo, b, y, x);
-                        for (int u = 0; u < 2 * G; ++u) {
-                            const int rb = rg * 2 * G + u;
-                            int sx = 0, sy = 0, sbi = a.ni, cb = 0;
-                            if (in && rb < nrb) {
-                                const int tap = rb / ncb;
-                                cb = rb - tap * ncb;
-                                const int kh = tap / a.k, kw = tap - kh * a.k;
-                                sx = x * a.stride + kw - a.pad;
-                                sy = y * a.stride + kh - a.pad;
-                                sbi = b;
-                            }
-                            tma_load_4d(sr + (u * kpos + kp) * 512, &mapR, &full_t[s], 2 * cb * 64, sx, sy, sbi);
-                        }
-                        for (int gq = 0; gq < BN / 64; ++gq)
-                            tma_load_5d(st + a_bytes + gq * 8192 + kp * Mp * 128, &mapD, &full_t[s], ct * BN + gq * 64,
-                                        0, in ? x : 0, in ? y : 0, in ? b : a.ni);
-                    }
+                    tc::mbar_expect_tx(&full_t[s], (uint32_t)Cfg::B_BYTES);
+                    const uint32_t sb = tc::smem_u32(smem + s * STG + a_bytes);
+                    for (int gq = 0; gq < BN / 64; ++gq)
+                        tma_load_3d(sb + gq * 8192, &mapD, &full_t[s], ct * BN + gq * 64, 0, (kt0 + i) * kpos);
                 }
             }
             const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
-            for (uint32_t i = it - n_drain; i < it; ++i) tc::mbar_wait(&full_t[i % NST], (i / NST) & 1u);
+            for (uint32_t i = it - n_drain; i < it; ++i) tc::mbar_wait_spin(&full_t[i % NST], (i / NST) & 1u);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -1090,7 +903,7 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
                 int rg, ct, kt0, nkt;
                 decode(t, rg, ct, kt0, nkt);
                 if (j >= 1) {
-                    if (!tc::mbar_wait(acc_empty, (j - 1) & 1u)) {
+                    if (!tc::mbar_wait_spin(acc_empty, (j - 1) & 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         break;
                     }
@@ -1099,7 +912,7 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
                 for (int i = 0; i < nkt; ++i, ++it) {
                     const int s = it % NST;
                     const uint32_t ph = (it / NST) & 1u;
-                    if (!tc::mbar_wait(&full_t[s], ph) || !tc::mbar_wait(&full_a[s], ph)) {
+                    if (!tc::mbar_wait_spin(&full_t[s], ph) || !tc::mbar_wait_spin(&full_a[s], ph)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
@@ -1153,35 +966,84 @@ __global__ void __launch_bounds__(GEN_THREADS, 1)
             if (lane == 0) tc::mbar_arrive(acc_empty);
         }
     } else {
-        const int g = threadIdx.x - (2 + CONV_NEPI) * 32;
-        uint32_t it = 0;
+        // generator group grp (4 warps) takes K steps it = grp, grp + 2, ...
+        // (the stage count is even: a stage and its slots keep their owners)
+        const int gw = warp - (2 + CONV_NEPI);
+        const int grp = gw / GEN_WARPS;
+        const int g = (gw % GEN_WARPS) * 32 + lane;
+        // advance a (tile, step) position by n K steps of this CTA's sequence
+        auto advance = [&](int &t, int &i, int n) {
+            while (t < ntiles && n > 0) {
+                int rg, ct, kt0, nkt;
+                decode(t, rg, ct, kt0, nkt);
+                const int left = nkt - i;
+                if (n < left) {
+                    i += n;
+                    n = 0;
+                } else {
+                    n -= left;
+                    i = 0;
+                    t += gridDim.x;
+                }
+            }
+        };
+        uint2 q[DW_AHEAD][DW_MAX_SPT];
+        int la_t = blockIdx.x, la_i = 0;  // the K step whose records load next
+        advance(la_t, la_i, grp);
+        auto load_next = [&](uint2(&dst)[DW_MAX_SPT]) {
+            int rg = 0, ct, kt0 = 0, nkt = 0;
+            if (la_t < ntiles) decode(la_t, rg, ct, kt0, nkt);
+#pragma unroll
+            for (int v = 0; v < DW_MAX_SPT; ++v) {
+                const int slot = g + v * 128;
+                dst[v] = make_uint2((uint32_t)REC_SILENT, 0u);
+                if (la_t < ntiles && slot < slots) {
+                    const int c = slot & 63, qq = slot >> 6;
+                    dst[v] = dw_record(a, rec, rg, G, kt0 + la_i, qq / kpos, qq % kpos, c);
+                }
+            }
+            advance(la_t, la_i, DW_GEN_GROUPS);
+        };
+#pragma unroll
+        for (int d = 0; d < DW_AHEAD; ++d) load_next(q[d]);
+        uint32_t it = grp;
+        int cur_t = blockIdx.x, cur_i = 0;
+        advance(cur_t, cur_i, grp);
         bool ok = true;
-        for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-            int rg, ct, kt0, nkt;
-            decode(t, rg, ct, kt0, nkt);
-            for (int i = 0; i < nkt; ++i, ++it) {
-                const int s = it % NST;
-                const uint32_t ph = (it / NST) & 1u;
-                if (!tc::mbar_wait(&full_t[s], ph)) {
-                    conv_set_status(STATUS_TIMEOUT);
-                    ok = false;
-                    break;
+        while (cur_t < ntiles && ok) {
+#pragma unroll
+            for (int d = 0; d < DW_AHEAD; ++d) {
+                if (cur_t < ntiles && ok) {
+                    const int s = it % NST;
+                    const uint32_t ph = (it / NST) & 1u;
+                    int w_ok = 1;
+                    if (lane == 0) w_ok = tc::mbar_wait(&empty[s], ph ^ 1u) ? 1 : 0;
+                    w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+                    if (!w_ok) {
+                        if (lane == 0) conv_set_status(STATUS_TIMEOUT);
+                        ok = false;
+                    } else {
+                        const uint32_t tile0 = tc::smem_u32(smem + s * STG);
+#pragma unroll
+                        for (int v = 0; v < DW_MAX_SPT; ++v) {
+                            const int slot = g + v * 128;
+                            if (slot < slots) {
+                                const int c = slot & 63, qq = slot >> 6;
+                                const int kp = qq % kpos, u = qq / kpos;
+                                int16_t *pk = prevk + s * slots + slot;
+                                gen_put_mn(tile0 + (u >> 1) * 16384 + (u & 1) * 8192, kp * Mp, c, (int)*pk, q[d][v],
+                                           a.c.M);
+                                *pk = (int16_t)(int)q[d][v].x;
+                            }
+                        }
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        __syncwarp();
+                        if (lane == 0) tc::mbar_arrive(&full_a[s]);
+                        load_next(q[d]);
+                        it += DW_GEN_GROUPS;
+                        advance(cur_t, cur_i, DW_GEN_GROUPS);
+                    }
                 }
-                uint8_t *st = smem + s * STG;
-                const uint32_t tile0 = tc::smem_u32(st);
-                const uint2 *rec = reinterpret_cast<const uint2 *>(st + a_bytes + Cfg::B_BYTES);
-                for (int slot = g; slot < slots; slot += GEN_WARPS * 32) {
-                    // slot = ((u = 2 row tile + block) kpos + kp) 64 + c
-                    const int c = slot & 63, q = slot >> 6;
-                    const int kp = q % kpos, u = q / kpos;
-                    const uint2 r = rec[slot];
-                    int16_t *pk = prevk + s * slots + slot;
-                    gen_put_mn(tile0 + (u >> 1) * 16384 + (u & 1) * 8192, kp * Mp, c, (int)*pk, r, a.c.M);
-                    *pk = (int16_t)(int)r.x;
-                }
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                __syncwarp();
-                if (lane == 0) tc::mbar_arrive(&full_a[s]);
             }
         }
     }
@@ -1241,43 +1103,44 @@ static bool map_mat(CUtensorMap *m, const void *ptr, int rows, int cols, int box
 
 static int pick_bn(int n) { return (n % 256 == 0) ? 256 : ((n % 128 == 0) ? 128 : 64); }
 
-// records [ni][h][w][C] of 8 bytes as a 4-D map of 32-bit words (2C, w, h,
-// ni), boxes of 64 records of one position, no swizzle, zeros outside
-static bool map_rec(CUtensorMap *m, const void *ptr, int ni, int h, int w, int C) {
-    EncodeFn enc = conv_encode();
-    if (!enc) return false;
-    cuuint64_t dims[4] = {(cuuint64_t)2 * C, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)ni};
-    cuuint64_t strides[3] = {(cuuint64_t)C * 8, (cuuint64_t)w * C * 8, (cuuint64_t)h * w * C * 8};
-    cuuint32_t box[4] = {128, 1, 1, 1};
-    cuuint32_t es[4] = {1, 1, 1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, const_cast<void *>(ptr), dims, strides, box, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int BN, bool RES>
-static cudaError_t launch_fwd_gen_bn(const CUtensorMap &mR, const CUtensorMap &mB, ConvGemmArgs a, cudaStream_t st) {
+static cudaError_t launch_fwd_gen_bn(const uint2 *rec, const CUtensorMap &mB, ConvGemmArgs a, cudaStream_t st) {
     using Cfg = GenFwdCfg<BN, RES>;
     const int fixed = a.res_bytes + Cfg::PREV_BYTES + 1024 + 256;
     int nst = (GEN_SMEM_MAX - fixed) / Cfg::STAGE;
     if (nst > Cfg::MAX_STAGES) nst = Cfg::MAX_STAGES;
-    if (nst < 2) return cudaErrorInvalidConfiguration;
+    nst -= nst % FWD_GEN_GROUPS;  // each stage belongs to one generator group
+    if (nst < FWD_GEN_GROUPS) return cudaErrorInvalidConfiguration;
     a.nst = nst;
     const int smem = Cfg::smem(nst, a.res_bytes);
     cudaError_t e = cudaFuncSetAttribute(k_conv_fwd_gen<BN, RES>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ntiles = a.n_row * a.n_col;
     const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_fwd_gen<BN, RES><<<grid, GEN_THREADS, smem, st>>>(mR, mB, a);
+    k_conv_fwd_gen<BN, RES><<<grid, FWD_THREADS, smem, st>>>(rec, mB, a);
     return cudaGetLastError();
 }
 
+// dw^ [P][Mp][C] bf16 as a 3-D map (C, Mp, P), boxes of (64, Mp, 64 / Mp):
+// the 64 k-rows (position, m) of one K step of dW, 128-byte swizzle
+static bool map_act3(CUtensorMap *m, const void *ptr, long long P, int Mp, int C) {
+    EncodeFn enc = conv_encode();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)C, (cuuint64_t)Mp, (cuuint64_t)P};
+    cuuint64_t strides[2] = {(cuuint64_t)C * 2, (cuuint64_t)Mp * C * 2};
+    cuuint32_t box[3] = {64, (cuuint32_t)Mp, (cuuint32_t)(64 / Mp)};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN>
-static cudaError_t launch_dw_gen_bn(const CUtensorMap &mR, const CUtensorMap &mD, ConvGemmArgs a, cudaStream_t st) {
+static cudaError_t launch_dw_gen_bn(const uint2 *rec, const CUtensorMap &mD, ConvGemmArgs a, cudaStream_t st) {
     using Cfg = GenDwCfg<BN>;
     const int kpos = 64 / a.Mp;
     int nst = DWG_MAX_STAGES;
-    while (nst > 2 && Cfg::smem(nst, a.groups, kpos) > GEN_SMEM_MAX) --nst;
+    while (nst > DW_GEN_GROUPS && Cfg::smem(nst, a.groups, kpos) > GEN_SMEM_MAX) nst -= DW_GEN_GROUPS;
     if (Cfg::smem(nst, a.groups, kpos) > GEN_SMEM_MAX) return cudaErrorInvalidConfiguration;
     a.nst = nst;
     const int smem = Cfg::smem(nst, a.groups, kpos);
@@ -1285,29 +1148,18 @@ static cudaError_t launch_dw_gen_bn(const CUtensorMap &mR, const CUtensorMap &mD
     if (e != cudaSuccess) return e;
     const int ntiles = a.n_row * a.n_col * a.n_split;
     const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_dw_gen<BN><<<grid, GEN_THREADS, smem, st>>>(mR, mD, a);
-    return cudaGetLastError();
-}
-
-template <int BN, int MODE>
-static cudaError_t launch_gemm_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, cudaStream_t st) {
-    using Cfg = ConvCfg<BN, MODE>;
-    cudaError_t e = cudaFuncSetAttribute(k_conv_gemm<BN, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (e != cudaSuccess) return e;
-    const int ntiles = a.n_row * a.n_col;
-    const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_gemm<BN, MODE><<<grid, CONV_THREADS, Cfg::SMEM, st>>>(mA, mB, a);
+    k_conv_dw_gen<BN><<<grid, DW_THREADS, smem, st>>>(rec, mD, a);
     return cudaGetLastError();
 }
 
 template <int BN>
-static cudaError_t launch_dw_bn(const CUtensorMap &mS, const CUtensorMap &mD, ConvGemmArgs a, cudaStream_t st) {
-    using Cfg = ConvCfg<BN, 2>;
-    cudaError_t e = cudaFuncSetAttribute(k_conv_dw<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+static cudaError_t launch_ds_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, cudaStream_t st) {
+    using Cfg = ConvCfg<BN>;
+    cudaError_t e = cudaFuncSetAttribute(k_conv_ds<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
-    const int ntiles = a.n_row * a.n_col * a.n_split;
+    const int ntiles = a.n_row * a.n_col;
     const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_dw<BN><<<grid, CONV_THREADS, Cfg::SMEM, st>>>(mS, mD, a);
+    k_conv_ds<BN><<<grid, CONV_THREADS, Cfg::SMEM, st>>>(mA, mB, a);
     return cudaGetLastError();
 }
 
@@ -1334,17 +1186,6 @@ bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp) {
            g.C * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
 }
 
-cudaError_t launch_bin_pmc(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st) {
-    if (C % 8 != 0) return cudaErrorInvalidValue;
-    const long long n = P * (C / 8);
-    long long blocks = (n + 255) / 256;
-    const long long cap = 8ll * conv_num_sms();
-    if (blocks > cap) blocks = cap;
-    if (blocks < 1) blocks = 1;
-    k_bin_pmc<<<(unsigned)blocks, 256, 0, st>>>(t, P, C, c, S);
-    return cudaGetLastError();
-}
-
 cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                              long long P, int C, const LifConst &c, __nv_bfloat16 *D, float *count,
                              cudaStream_t st) {
@@ -1367,28 +1208,6 @@ cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, __nv_bf
     return cudaGetLastError();
 }
 
-// forward contraction of ni images: S [ni H W][Mp][C_in], Wf [C_out][k k C_in]
-// -> w^ [ni Ho Wo][Mp][C_out]
-cudaError_t launch_conv_fwd_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                                 const __nv_bfloat16 *Wf, float *what, cudaStream_t st) {
-    ConvGemmArgs a = base_args(g, ni, c);
-    a.C_out = C_out;
-    a.P_rows = ni * g.Ho * g.Wo;
-    const int BN = pick_bn(C_out);
-    a.n_row = (a.P_rows + (128 / c.Mp) - 1) / (128 / c.Mp);
-    a.n_col = C_out / BN;
-    a.ktiles = g.k * g.k * (g.C / 64);
-    a.what = what;
-    CUtensorMap mA, mB;
-    if (!map_act(&mA, S, ni, g.H, g.W, c.Mp, g.C) || !map_mat(&mB, Wf, C_out, g.k * g.k * g.C, BN))
-        return cudaErrorInvalidValue;
-    switch (BN) {
-        case 256: return launch_gemm_bn<256, 0>(mA, mB, a, st);
-        case 128: return launch_gemm_bn<128, 0>(mA, mB, a, st);
-        default: return launch_gemm_bn<64, 0>(mA, mB, a, st);
-    }
-}
-
 // dS of ni images with the input-time gradient: dw^ [ni Ho Wo][Mp][C_out],
 // Wt [C_in][k k C_out], t_in [ni H W][C_in] -> g_t_in (zeroed first)
 cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *dW_hat,
@@ -1408,44 +1227,9 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out) || !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))
         return cudaErrorInvalidValue;
     switch (BN) {
-        case 256: return launch_gemm_bn<256, 1>(mA, mB, a, st);
-        case 128: return launch_gemm_bn<128, 1>(mA, mB, a, st);
-        default: return launch_gemm_bn<64, 1>(mA, mB, a, st);
-    }
-}
-
-// dW over ni images added into g_W [C_out][k k C_in] (zeroed by the caller
-// before the first chunk); count (may be null) adds qcoef * count[o] once
-cudaError_t launch_conv_dw_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                                const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
-                                cudaStream_t st) {
-    ConvGemmArgs a = base_args(g, ni, c);
-    a.C_out = C_out;
-    a.P_rows = ni * g.Ho * g.Wo;
-    const int BN = pick_bn(C_out);
-    const int Ktot = g.k * g.k * g.C;
-    a.n_row = (Ktot / 64 + 1) / 2;
-    a.n_col = C_out / BN;
-    const int kpos = 64 / c.Mp;
-    a.ktiles = (a.P_rows + kpos - 1) / kpos;
-    // split-K: about two tiles per SM, at least 16 K steps each
-    const int tiles = a.n_row * a.n_col;
-    int splits = (2 * conv_num_sms() + tiles - 1) / tiles;
-    const int max_splits = (a.ktiles + 15) / 16;
-    if (splits > max_splits) splits = max_splits;
-    if (splits < 1) splits = 1;
-    a.kt_per_split = (a.ktiles + splits - 1) / splits;
-    a.n_split = (a.ktiles + a.kt_per_split - 1) / a.kt_per_split;
-    a.g_W = g_W;
-    a.count = count;
-    a.qcoef = qcoef;
-    CUtensorMap mS, mD;
-    if (!map_act(&mS, S, ni, g.H, g.W, c.Mp, g.C) || !map_act(&mD, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out))
-        return cudaErrorInvalidValue;
-    switch (BN) {
-        case 256: return launch_dw_bn<256>(mS, mD, a, st);
-        case 128: return launch_dw_bn<128>(mS, mD, a, st);
-        default: return launch_dw_bn<64>(mS, mD, a, st);
+        case 256: return launch_ds_bn<256>(mA, mB, a, st);
+        case 128: return launch_ds_bn<128>(mA, mB, a, st);
+        default: return launch_ds_bn<64>(mA, mB, a, st);
     }
 }
 
@@ -1474,20 +1258,19 @@ cudaError_t launch_conv_fwd_gen(const ConvGeom &g, int ni, int C_out, const LifC
     const long long res = (long long)a.ktiles * BN * 128;
     const bool resident = a.n_col == 1 && res <= 144 * 1024;
     a.res_bytes = resident ? (int)res : 0;
-    CUtensorMap mR, mB;
-    if (!map_rec(&mR, rec, ni, g.H, g.W, g.C) || !map_mat(&mB, Wf, C_out, g.k * g.k * g.C, BN))
-        return cudaErrorInvalidValue;
+    CUtensorMap mB;
+    if (!map_mat(&mB, Wf, C_out, g.k * g.k * g.C, BN)) return cudaErrorInvalidValue;
     if (resident) {
         switch (BN) {
-            case 256: return launch_fwd_gen_bn<256, true>(mR, mB, a, st);
-            case 128: return launch_fwd_gen_bn<128, true>(mR, mB, a, st);
-            default: return launch_fwd_gen_bn<64, true>(mR, mB, a, st);
+            case 256: return launch_fwd_gen_bn<256, true>(rec, mB, a, st);
+            case 128: return launch_fwd_gen_bn<128, true>(rec, mB, a, st);
+            default: return launch_fwd_gen_bn<64, true>(rec, mB, a, st);
         }
     }
     switch (BN) {
-        case 256: return launch_fwd_gen_bn<256, false>(mR, mB, a, st);
-        case 128: return launch_fwd_gen_bn<128, false>(mR, mB, a, st);
-        default: return launch_fwd_gen_bn<64, false>(mR, mB, a, st);
+        case 256: return launch_fwd_gen_bn<256, false>(rec, mB, a, st);
+        case 128: return launch_fwd_gen_bn<128, false>(rec, mB, a, st);
+        default: return launch_fwd_gen_bn<64, false>(rec, mB, a, st);
     }
 }
 
@@ -1505,6 +1288,7 @@ cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifCo
     int gmax = 512 / BN;
     if (gmax > DWG_MAX_G) gmax = DWG_MAX_G;
     const int kpos = 64 / c.Mp;
+    if (gmax * kpos > DW_MAX_SPT) gmax = DW_MAX_SPT / kpos;
     // shared memory: at least two stages of G tiles
     auto smem2 = [&](int G) {
         return BN == 256 ? GenDwCfg<256>::smem(2, G, kpos)
@@ -1526,13 +1310,12 @@ cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifCo
     a.g_W = g_W;
     a.count = count;
     a.qcoef = qcoef;
-    CUtensorMap mR, mD;
-    if (!map_rec(&mR, rec, ni, g.H, g.W, g.C) || !map_act(&mD, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out))
-        return cudaErrorInvalidValue;
+    CUtensorMap mD;
+    if (!map_act3(&mD, dW_hat, (long long)a.P_rows, c.Mp, C_out)) return cudaErrorInvalidValue;
     switch (BN) {
-        case 256: return launch_dw_gen_bn<256>(mR, mD, a, st);
-        case 128: return launch_dw_gen_bn<128>(mR, mD, a, st);
-        default: return launch_dw_gen_bn<64>(mR, mD, a, st);
+        case 256: return launch_dw_gen_bn<256>(rec, mD, a, st);
+        case 128: return launch_dw_gen_bn<128>(rec, mD, a, st);
+        default: return launch_dw_gen_bn<64>(rec, mD, a, st);
     }
 }
 

@@ -300,27 +300,25 @@ struct ConvGeom {
     int B, H, W, C, Ho, Wo, k, s, p;
 };
 // Implicit-GEMM conv layer in bf16 (dstd_conv_tc.cu), for C_in and C_out
-// multiples of 64 and Mp in {32, 64, 128}: activations [positions][Mp][C]
-// (channel innermost), no im2col operand. ni = images of the chunk.
+// multiples of 64 and Mp in {32, 64, 128}: no im2col operand. ni = images of
+// the chunk; positions NHWC.
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp);
-// t [P][C] -> S [P][Mp][C] bf16 (C a multiple of 8)
-cudaError_t launch_bin_pmc(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st);
 // dw^ [P][Mp][C] bf16 from the saved state [P][C]; silent counts per channel
 // added into count (zeroed by the caller)
 cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                              long long P, int C, const LifConst &c, __nv_bfloat16 *D, float *count, cudaStream_t st);
 // filters [C_out][T][C_in] fp32 -> [C_in][T][C_out] bf16
 cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, __nv_bfloat16 *Wt, cudaStream_t st);
-cudaError_t launch_conv_fwd_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                                 const __nv_bfloat16 *Wf, float *what, cudaStream_t st);
+// dS of ni images (the transposed convolution of dw^ [ni Ho Wo][Mp][C_out]
+// with Wt [C_in][k k C_out]) with the input-time gradient in the epilogue:
+// g_t_in [ni H W][C_in] (zeroed first) from t_in [ni H W][C_in]
 cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *dW_hat,
                                 const __nv_bfloat16 *Wt, const float *t_in, float *g_t_in, cudaStream_t st);
-cudaError_t launch_conv_dw_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                                const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
-                                cudaStream_t st);
 // the binned operand generated on chip: one 8-byte record per input
-// (grid step, bf16 pair of its two weights), then the forward and dW
-// contractions write the operand tiles in shared memory from the records
+// (grid step, bf16 pair of its two weights), then the forward (w^ [ni Ho
+// Wo][C_out][Mp] fp32) and dW (added into g_W [C_out][k k C_in], zeroed by
+// the caller before the first chunk) contractions write their operand
+// tiles in shared memory from the records
 cudaError_t launch_bin_rec(const float *t, long long n, const LifConst &c, uint2 *rec, cudaStream_t st);
 cudaError_t launch_conv_fwd_gen(const ConvGeom &g, int ni, int C_out, const LifConst &c, const uint2 *rec,
                                 const __nv_bfloat16 *Wf, float *what, cudaStream_t st);

@@ -53,6 +53,36 @@ static __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t par
     return ok != 0;
 }
 
+// try_wait without a suspend-time hint: returns after the implementation's
+// own short time limit, so a thread that polls in a loop reacts to the
+// phase change within a few cycles
+static __device__ __forceinline__ bool mbar_try_wait_now(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// bounded spin wait for the threads on a pipeline's critical path (TMA
+// producer, MMA issuer, operand generators): false after limit_ns
+static __device__ __forceinline__ bool mbar_wait_spin(uint64_t *bar, uint32_t parity,
+                                                      unsigned long long limit_ns = WAIT_NS) {
+    if (mbar_try_wait_now(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    for (;;) {
+        for (int i = 0; i < 32; ++i)
+            if (mbar_try_wait_now(bar, parity)) return true;
+        if (globaltimer() - t0 > limit_ns) return false;
+    }
+}
+
 // bounded wait: false if the phase did not complete within limit_ns
 static __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
                                           unsigned long long limit_ns = WAIT_NS) {
