@@ -138,8 +138,11 @@ int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
  * t_in, W, t_out, saved and penalty. (The paper has no counterpart: this is
  * a deployment convenience of this library.)
  * Scratch: a fixed 64 MiB array in device memory, part of the library's
- * image, present on every GPU that loads the library until the process
- * exits. A call whose scratch need (dstd_dense_workspace_bytes' forward part)
+ * image. With CUDA's lazy module loading it is taken on a device when the
+ * library's module is first loaded there (the first launch of any of its
+ * kernels, or this function's address lookup), by every process that uses
+ * the library on that device whether or not it calls this function, and it
+ * stays until the process exits. A call whose scratch need (dstd_dense_workspace_bytes' forward part)
  * exceeds 64 MiB returns DSTD_E_WORKSPACE and launches nothing; the 784-800
  * and 800-800 layers at B = 256, M = 32 fit. No call allocates or frees.
  * Every call uses the same array, which keeps whatever the previous call
@@ -147,7 +150,10 @@ int dstd_dense_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
  * that can overlap on the GPU (different streams, or different host threads)
  * race; serialise them. The first call on each device looks up the array's
  * device address (cudaGetSymbolAddress) with that device current; make that
- * first call before starting any stream capture. */
+ * first call before starting any stream capture. The address is kept per
+ * device for the life of the process: it belongs to the device's primary
+ * context, so calls must come from that context (the runtime API's default),
+ * and not after a cudaDeviceReset. */
 int dstd_dense_fwd_noalloc(const float *t_in, const float *W, int B, int N_in, int N_out, const dstd_params *p,
                            dstd_math math, float *t_out, void *saved, float *penalty, dstd_stream_t stream);
 

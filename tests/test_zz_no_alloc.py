@@ -29,7 +29,10 @@ def _both(t_in, W, layer, B, math_mode):
     from paper_2607_14672_gb300 import dstd
     N_out, N_in = W.shape
     p = dstd.params(layer, 1.0 / B)
-    ws = torch.empty(dstd.dense_workspace_bytes(B, N_in, N_out, p, math_mode), dtype=torch.uint8, device="cuda")
+    # the workspace starts full of 0xFF bytes, so a forward that read scratch
+    # it had not written would differ from the allocation-free one
+    ws = torch.full((dstd.dense_workspace_bytes(B, N_in, N_out, p, math_mode),), 255, dtype=torch.uint8,
+                    device="cuda")
     nsv = dstd.dense_saved_bytes(B, N_out)
     out = []
     for noalloc in (False, True):
@@ -88,3 +91,24 @@ def test_noalloc_rejects_oversized_layers():
         dstd.dense_fwd_noalloc(t_in, W, p, "x3", t_out, saved)
     assert e.value.code == -3
     assert dstd.device_status(clear=True) == 0
+
+
+@pytest.mark.parametrize("math_mode", ["x3", "bf16"])
+def test_noalloc_ragged_width_after_a_larger_layer(math_mode):
+    """A layer whose input width is not a multiple of 8 (100 -> 300: its
+    operand rows are padded to 104 columns) right after a larger layer has
+    filled the shared scratch: the padding columns must not carry the
+    earlier call's values into the result."""
+    from paper_2607_14672_gb300 import configs, synth
+    cfg = configs.config2(batch=256)
+    B = 256
+    L1 = cfg["layers"][0]
+    t0 = torch.tensor(np.asarray(cfg["inputs"](B=B), np.float32), device="cuda")
+    W1 = torch.tensor(np.asarray(L1["W"], np.float32), device="cuda")
+    r1 = _both(t0, W1, L1, B, math_mode)          # 784 -> 800 fills the scratch first
+    _check(r1[0], r1[1], L1)
+    L = dict(L1)
+    t_small = torch.tensor(np.asarray(synth.uniform_spikes(5, (B, 100), 0.0, 1.0, 0.2), np.float32), device="cuda")
+    W_small = torch.tensor(np.asarray(synth.normal_weights(1005, (300, 100), 0.12, 0.1), np.float32), device="cuda")
+    r2 = _both(t_small, W_small, L, B, math_mode)
+    _check(r2[0], r2[1], L)
