@@ -193,20 +193,6 @@ struct ConvGemmArgs {
     LifConst c;
 };
 
-template <int BN>
-struct ConvCfg {
-    static constexpr int A_BYTES = 128 * 128;          // 128 rows x 64 k of bf16
-    static constexpr int B_BYTES = BN * 128;
-    static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
-    static constexpr int STAGES_RAW = (CONV_SMEM_BUDGET - EPI_BYTES) / STAGE;
-    static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
-    static constexpr int SMEM = STAGES * STAGE + EPI_BYTES + 1024 + 256;
-    static constexpr uint32_t TMEM_COLS = 2 * BN;
-    static_assert(STAGES >= 2, "at least two stages");
-    static_assert(BN == 64 || BN == 128 || BN == 256, "BN");
-};
-
 // position p of an (ni, h, w) grid -> (b, y, x)
 __device__ __forceinline__ void pos_decode(int p, int h, int w, int &b, int &y, int &x) {
     const int hw = h * w;
@@ -240,39 +226,58 @@ __device__ __forceinline__ void conv_src(const ConvGemmArgs &a, int p, int kh, i
     }
 }
 
+// shared-memory plan of dS: a stage ("unit") holds the A operand of one
+// (tap, channel block) (per-position boxes, 16 KB) or, with row boxes, of
+// one (filter row kh, channel block) for all k taps of that row ((128/Mp +
+// k - 1) positions of Mp rows), and the B tiles of its taps unless the
+// transposed filters are resident; sizes are chosen on the host
+struct DsPlan {
+    int a_bytes, b_bytes, stage, res_bytes, nst, units, taps_per_unit;
+};
+constexpr int DS_MAX_STAGES = 8;
+constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
+
 // ---------------------------------------------------------------------------
 // dS with the input-time gradient: rows (input position, m) of 128 per tile
 // (128 / Mp positions), columns BN of the C_in channels; K = k k taps x
 // blocks of 64 output channels of dw^ (the transposed convolution).
 // Persistent: CTA b takes tiles b, b + grid, ...
-//   warp 0  TMA producer (one lane): the 128/Mp position boxes of A, B's box
+//   warp 0  TMA producer (one lane): A boxes and the B tiles (or, with RES,
+//           every B tile once)
 //   warp 1  TMEM allocation and MMA issue (one lane)
 //   warps 2-9  epilogue: warp w reads TMEM lane quarter w % 4, 32-column
 //              chunks (w - 2) / 4, +2, ... of the tile
-// Barriers: full/empty per stage; acc_full/acc_empty per accumulator (two).
+// ROWBOX (stride 1, tiles within one image row): one box of 128/Mp + k - 1
+// positions per (kh, channel block) serves all k taps kw of that filter row;
+// tap kw's A tile starts (k - 1 - kw) positions into it.
+// Barriers: full/empty per unit; acc_full/acc_empty per accumulator (two).
 // ---------------------------------------------------------------------------
-template <int BN>
+template <int BN, bool ROWBOX, bool RES>
 __global__ void __launch_bounds__(CONV_THREADS, 1)
-    k_conv_ds(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a) {
-    using Cfg = ConvCfg<BN>;
+    k_conv_ds(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a,
+              DsPlan pl) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    float *epi = reinterpret_cast<float *>(smem + Cfg::STAGES * Cfg::STAGE);
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + Cfg::STAGES * Cfg::STAGE + Cfg::EPI_BYTES);
-    uint64_t *empty = full + Cfg::STAGES;
-    uint64_t *acc_full = empty + Cfg::STAGES;  // [2]
-    uint64_t *acc_empty = acc_full + 2;       // [2]
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
+    const int NST = pl.nst;
+    uint8_t *bres = smem + NST * pl.stage;
+    float *epi = reinterpret_cast<float *>(bres + pl.res_bytes);
+    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + DS_EPI_BYTES);
+    uint64_t *empty = full + DS_MAX_STAGES;
+    uint64_t *acc_full = empty + DS_MAX_STAGES;  // [2]
+    uint64_t *acc_empty = acc_full + 2;          // [2]
+    uint64_t *bres_full = acc_empty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bres_full + 1);
+    constexpr uint32_t TMEM_COLS = 2 * BN;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int ntiles = a.n_row * a.n_col;
     const int Mp = a.Mp;
     const int ppt = 128 / Mp;  // positions per tile
-    const int c_red = a.C_out;
-    const int ncb = c_red >> 6;
+    const int ncb = a.C_out >> 6;
+    const int k = a.k;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < Cfg::STAGES; ++s) {
+        for (int s = 0; s < NST; ++s) {
             tc::mbar_init(&full[s], 1);
             tc::mbar_init(&empty[s], 1);
         }
@@ -280,10 +285,11 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             tc::mbar_init(&acc_full[u], 1);
             tc::mbar_init(&acc_empty[u], CONV_NEPI);
         }
+        tc::mbar_init(bres_full, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
-    if (warp == 1) tc::tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+    if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
@@ -291,34 +297,54 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
 
     if (warp == 0) {
         if (lane == 0) {
+            if (RES) {
+                // every (tap, channel block) B tile of the single column tile, once
+                const int nslices = k * k * ncb;
+                tc::mbar_expect_tx(bres_full, (uint32_t)(nslices * BN * 128));
+                for (int q = 0; q < nslices; ++q) {
+                    const int tap = q / ncb, cb = q - tap * ncb;
+                    tc::tma_load_2d(tc::smem_u32(bres + q * BN * 128), &mapB, bres_full, tap * a.C_out + cb * 64, 0);
+                }
+            }
             uint32_t it = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
                 const int rt = t / a.n_col, ct = t - rt * a.n_col;
-                for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
-                    const int s = it % Cfg::STAGES;
-                    const uint32_t ph = (it / Cfg::STAGES) & 1u;
+                int b0 = 0, y0 = 0, x0 = 0;
+                if (ROWBOX) pos_decode(rt * ppt, a.H, a.W, b0, y0, x0);
+                for (int u = 0; u < pl.units; ++u, ++it) {
+                    const int s = it % NST;
+                    const uint32_t ph = (it / NST) & 1u;
                     if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
                     }
-                    tc::mbar_expect_tx(&full[s], (uint32_t)Cfg::STAGE);
-                    const int tap = kt / ncb, cb = kt - tap * ncb;
-                    const int kh = tap / a.k, kw = tap - kh * a.k;
-                    const uint32_t st = tc::smem_u32(smem + s * Cfg::STAGE);
-                    for (int pp = 0; pp < ppt; ++pp) {
-                        int sx, sy, sb;
-                        conv_src(a, rt * ppt + pp, kh, kw, sx, sy, sb);
-                        tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, sb);
+                    tc::mbar_expect_tx(&full[s], (uint32_t)(pl.a_bytes + pl.b_bytes));
+                    const uint32_t st = tc::smem_u32(smem + s * pl.stage);
+                    if (ROWBOX) {
+                        // unit u = (kh, cb): output positions x0 + pad - (k - 1) .. of row y0 + pad - kh
+                        const int kh = u / ncb, cb = u - kh * ncb;
+                        tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 + a.pad - (k - 1), y0 + a.pad - kh, b0);
+                        if (!RES)
+                            for (int kw = 0; kw < k; ++kw)
+                                tc::tma_load_2d(st + pl.a_bytes + kw * BN * 128, &mapB, &full[s],
+                                                (kh * k + kw) * a.C_out + cb * 64, ct * BN);
+                    } else {
+                        const int tap = u / ncb, cb = u - tap * ncb;
+                        const int kh = tap / k, kw = tap - kh * k;
+                        for (int pp = 0; pp < ppt; ++pp) {
+                            int sx, sy, sb;
+                            conv_src(a, rt * ppt + pp, kh, kw, sx, sy, sb);
+                            tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, sb);
+                        }
+                        if (!RES) tc::tma_load_2d(st + pl.a_bytes, &mapB, &full[s], tap * a.C_out + cb * 64, ct * BN);
                     }
-                    tc::tma_load_2d(st + Cfg::A_BYTES, &mapB, &full[s], tap * c_red + cb * 64, ct * BN);
                 }
             }
-            // loads still in flight (after an expired wait) land before the CTA exits
-            const uint32_t n_drain = it < (uint32_t)Cfg::STAGES ? it : (uint32_t)Cfg::STAGES;
-            for (uint32_t i = it - n_drain; i < it; ++i)
-                tc::mbar_wait_spin(&full[i % Cfg::STAGES], (i / Cfg::STAGES) & 1u);
+            const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
+            for (uint32_t i = it - n_drain; i < it; ++i) tc::mbar_wait_spin(&full[i % NST], (i / NST) & 1u);
+            if (RES) tc::mbar_wait_spin(bres_full, 0);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -326,6 +352,11 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             constexpr uint32_t idesc = idesc_bf16(128, BN, false, false);
             uint32_t it = 0, j = 0;
             bool ok = true;
+            if (RES && !tc::mbar_wait_spin(bres_full, 0)) {
+                conv_set_status(STATUS_TIMEOUT);
+                ok = false;
+            }
+            const int tpu = ROWBOX ? k : 1;  // taps per unit
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
                 const uint32_t buf = j & 1u;
                 if (j >= 2) {
@@ -336,21 +367,36 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     tc::tc_fence_after();
                 }
                 const uint32_t acc = tmem + buf * BN;
-                for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
-                    const int s = it % Cfg::STAGES;
-                    const uint32_t ph = (it / Cfg::STAGES) & 1u;
+                for (int u = 0; u < pl.units; ++u, ++it) {
+                    const int s = it % NST;
+                    const uint32_t ph = (it / NST) & 1u;
                     if (!tc::mbar_wait_spin(&full[s], ph)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
                         break;
                     }
                     tc::tc_fence_after();
-                    const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE);
-                    const uint32_t sbb = sa + Cfg::A_BYTES;
+                    const uint32_t sa = tc::smem_u32(smem + s * pl.stage);
+                    for (int v = 0; v < tpu; ++v) {
+                        int tap, cb;
+                        uint32_t abase;
+                        if (ROWBOX) {
+                            const int kh = u / ncb;
+                            cb = u - kh * ncb;
+                            tap = kh * k + v;
+                            abase = sa + (uint32_t)((k - 1 - v) * Mp * 128);
+                        } else {
+                            tap = u / ncb;
+                            cb = u - tap * ncb;
+                            abase = sa;
+                        }
+                        const uint32_t bbase = RES ? tc::smem_u32(bres + (tap * ncb + cb) * BN * 128)
+                                                   : sa + (uint32_t)(pl.a_bytes + v * BN * 128);
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        tc::mma_bf16(acc, tc::sdesc_sw128(sa + kk * 32), tc::sdesc_sw128(sbb + kk * 32), idesc,
-                                     (kt > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc::mma_bf16(acc, tc::sdesc_sw128(abase + kk * 32), tc::sdesc_sw128(bbase + kk * 32), idesc,
+                                         (u > 0 || v > 0 || kk > 0) ? 1u : 0u);
+                    }
                     tc::mma_commit(&empty[s]);
                 }
                 if (ok) tc::mma_commit(&acc_full[buf]);
@@ -361,44 +407,57 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         const int quarter = warp & 3, group = (warp - 2) >> 2;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
         float *tb = epi + (warp - 2) * 32 * EPI_LD;
-        const int r = quarter * 32 + lane;       // tile row of this lane
         const int pp = (quarter * 32) / Mp;      // position of this warp's rows (Mp >= 32)
         const int m_base = (quarter * 32) % Mp;  // first grid step of this warp's rows
+        constexpr int NCH = BN / 64;             // 32-column chunks of this warp
         uint32_t j = 0;
         for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
             const int rt = t / a.n_col, ct = t - rt * a.n_col;
             const uint32_t buf = j & 1u;
+            const int p = rt * ppt + pp;
+            // the grid step and the two kernel derivatives of the input each
+            // lane will own, loaded while the tile's MMAs run
+            int wk[NCH];
+            float wdR[NCH], wdL[NCH];
+#pragma unroll
+            for (int h = 0; h < NCH; ++h) {
+                wk[h] = -1000;
+                wdR[h] = wdL[h] = 0.f;
+                const int col0 = ct * BN + (group + 2 * h) * 32;
+                if (p < a.P_rows) {
+                    const float x = __ldg(a.t_in + (long long)p * a.C_in + col0 + lane);
+                    if (isfinite(x)) {
+                        const BinW w = bin_weights(a.c, x, true);
+                        wk[h] = w.k;
+                        wdR[h] = w.dR;
+                        wdL[h] = w.dL;
+                    }
+                }
+            }
             if (!tc::mbar_wait_sleep(&acc_full[buf], (j >> 1) & 1u)) {
                 conv_set_status(STATUS_TIMEOUT);
                 break;
             }
             tc::tc_fence_after();
-            const int p = rt * ppt + pp;
-            for (int cc = group; cc < BN / 32; cc += 2) {
+#pragma unroll
+            for (int h = 0; h < NCH; ++h) {
+                const int cc = group + 2 * h;
                 float v[32];
                 tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
-                const int col0 = ct * BN + cc * 32;
-                {
-                    // dS: lane m of the warp holds grid step m_base + m of 32
-                    // channels; transpose through shared memory so that lane
-                    // u owns channel col0 + u and reads its two grid steps
+                // lane m of the warp holds grid step m_base + m of 32 channels;
+                // transpose through shared memory so that lane u owns channel
+                // col0 + u and reads its two grid steps
 #pragma unroll
-                    for (int u = 0; u < 32; ++u) tb[lane * EPI_LD + u] = v[u];
-                    __syncwarp();
-                    if (p < a.P_rows) {
-                        const long long e = (long long)p * a.C_in + col0 + lane;
-                        const float x = __ldg(a.t_in + e);
-                        if (isfinite(x)) {
-                            const BinW w = bin_weights(a.c, x, true);
-                            float g = 0.f;
-                            const int k0 = w.k - m_base, k1 = w.k + 1 - m_base;
-                            if (k0 >= 0 && k0 < 32 && w.k < a.c.M) g = fmaf(tb[k0 * EPI_LD + lane], w.dR, g);
-                            if (k1 >= 0 && k1 < 32 && w.k + 1 < a.c.M) g = fmaf(tb[k1 * EPI_LD + lane], w.dL, g);
-                            if (g != 0.f) atomicAdd(a.g_t_in + e, g);
-                        }
-                    }
-                    __syncwarp();
+                for (int u = 0; u < 32; ++u) tb[lane * EPI_LD + u] = v[u];
+                __syncwarp();
+                if (p < a.P_rows && wk[h] > -1000) {
+                    float g = 0.f;
+                    const int k0 = wk[h] - m_base, k1 = wk[h] + 1 - m_base;
+                    if (k0 >= 0 && k0 < 32 && wk[h] < a.c.M) g = fmaf(tb[k0 * EPI_LD + lane], wdR[h], g);
+                    if (k1 >= 0 && k1 < 32 && wk[h] + 1 < a.c.M) g = fmaf(tb[k1 * EPI_LD + lane], wdL[h], g);
+                    if (g != 0.f) atomicAdd(a.g_t_in + (long long)p * a.C_in + ct * BN + cc * 32 + lane, g);
                 }
+                __syncwarp();
             }
             tc::tc_fence_before();
             __syncwarp();
@@ -407,7 +466,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
     }
     tc::tc_fence_before();
     __syncthreads();
-    if (warp == 1) tc::tmem_dealloc(tmem, Cfg::TMEM_COLS);
+    if (warp == 1) tc::tmem_dealloc(tmem, TMEM_COLS);
 }
 
 // ---------------------------------------------------------------------------
@@ -1074,14 +1133,14 @@ static EncodeFn conv_encode() {
 }
 
 // activation [ni][h][w][Mp][C] bf16 as a 5-D map (C, Mp, w, h, ni), boxes of
-// (64, Mp, 1, 1, 1), 128-byte swizzle, zeros outside
-static bool map_act(CUtensorMap *m, const void *ptr, int ni, int h, int w, int Mp, int C) {
+// (64, Mp, box_x, 1, 1), 128-byte swizzle, zeros outside
+static bool map_act(CUtensorMap *m, const void *ptr, int ni, int h, int w, int Mp, int C, int box_x = 1) {
     EncodeFn enc = conv_encode();
     if (!enc) return false;
     cuuint64_t dims[5] = {(cuuint64_t)C, (cuuint64_t)Mp, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)ni};
     cuuint64_t strides[4] = {(cuuint64_t)C * 2, (cuuint64_t)Mp * C * 2, (cuuint64_t)w * Mp * C * 2,
                              (cuuint64_t)h * w * Mp * C * 2};
-    cuuint32_t box[5] = {64, (cuuint32_t)Mp, 1, 1, 1};
+    cuuint32_t box[5] = {64, (cuuint32_t)Mp, (cuuint32_t)box_x, 1, 1};
     cuuint32_t es[5] = {1, 1, 1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(ptr), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1152,14 +1211,16 @@ static cudaError_t launch_dw_gen_bn(const uint2 *rec, const CUtensorMap &mD, Con
     return cudaGetLastError();
 }
 
-template <int BN>
-static cudaError_t launch_ds_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, cudaStream_t st) {
-    using Cfg = ConvCfg<BN>;
-    cudaError_t e = cudaFuncSetAttribute(k_conv_ds<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+template <int BN, bool ROWBOX, bool RES>
+static cudaError_t launch_ds_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
+                                cudaStream_t st) {
+    const int smem = pl.nst * pl.stage + pl.res_bytes + DS_EPI_BYTES + 1024 + 256;
+    cudaError_t e =
+        cudaFuncSetAttribute(k_conv_ds<BN, ROWBOX, RES>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ntiles = a.n_row * a.n_col;
     const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_ds<BN><<<grid, CONV_THREADS, Cfg::SMEM, st>>>(mA, mB, a);
+    k_conv_ds<BN, ROWBOX, RES><<<grid, CONV_THREADS, smem, st>>>(mA, mB, a, pl);
     return cudaGetLastError();
 }
 
@@ -1216,21 +1277,49 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     a.C_out = C_out;
     a.P_rows = ni * g.H * g.W;
     const int BN = pick_bn(g.C);
-    a.n_row = (a.P_rows + (128 / c.Mp) - 1) / (128 / c.Mp);
+    const int ppt = 128 / c.Mp;
+    const int ncb = C_out / 64;
+    a.n_row = (a.P_rows + ppt - 1) / ppt;
     a.n_col = g.C / BN;
-    a.ktiles = g.k * g.k * (C_out / 64);
     a.t_in = t_in;
     a.g_t_in = g_t_in;
     cudaError_t e = cudaMemsetAsync(g_t_in, 0, sizeof(float) * (size_t)a.P_rows * g.C, st);
     if (e != cudaSuccess) return e;
+    // resident transposed filters when they are small; one box per filter row
+    // at stride 1 when every tile lies within one image row
+    const long long res = (long long)g.k * g.k * ncb * BN * 128;
+    const bool resident = a.n_col == 1 && res <= 80 * 1024;
+    auto plan = [&](bool rowbox) {
+        DsPlan pl{};
+        pl.taps_per_unit = rowbox ? g.k : 1;
+        pl.a_bytes = rowbox ? (ppt + g.k - 1) * c.Mp * 128 : 128 * 128;
+        pl.b_bytes = resident ? 0 : pl.taps_per_unit * BN * 128;
+        pl.stage = (pl.a_bytes + pl.b_bytes + 1023) & ~1023;
+        pl.res_bytes = resident ? (int)res : 0;
+        pl.units = (rowbox ? g.k : g.k * g.k) * ncb;
+        int nst = (GEN_SMEM_MAX - pl.res_bytes - DS_EPI_BYTES - 1280) / pl.stage;
+        pl.nst = nst > DS_MAX_STAGES ? DS_MAX_STAGES : nst;
+        return pl;
+    };
+    const bool row_ok = g.s == 1 && g.W % ppt == 0 && ppt + g.k - 1 <= 256;
+    DsPlan pl = plan(row_ok);
+    bool rowbox = row_ok && pl.nst >= 3;
+    if (!rowbox) pl = plan(false);
+    if (pl.nst < 2) return cudaErrorInvalidConfiguration;
     CUtensorMap mA, mB;
-    if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out) || !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))
+    if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, rowbox ? ppt + g.k - 1 : 1) ||
+        !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))
         return cudaErrorInvalidValue;
+#define DSTD_DS(BNV)                                                                                   \
+    if (rowbox) return resident ? launch_ds_bn<BNV, true, true>(mA, mB, a, pl, st)                     \
+                                : launch_ds_bn<BNV, true, false>(mA, mB, a, pl, st);                   \
+    return resident ? launch_ds_bn<BNV, false, true>(mA, mB, a, pl, st) : launch_ds_bn<BNV, false, false>(mA, mB, a, pl, st);
     switch (BN) {
-        case 256: return launch_ds_bn<256>(mA, mB, a, st);
-        case 128: return launch_ds_bn<128>(mA, mB, a, st);
-        default: return launch_ds_bn<64>(mA, mB, a, st);
+        case 256: { DSTD_DS(256) }
+        case 128: { DSTD_DS(128) }
+        default: { DSTD_DS(64) }
     }
+#undef DSTD_DS
 }
 
 cudaError_t launch_bin_rec(const float *t, long long n, const LifConst &c, uint2 *rec, cudaStream_t st) {
