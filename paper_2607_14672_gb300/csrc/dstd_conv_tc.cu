@@ -202,38 +202,43 @@ __device__ __forceinline__ void pos_decode(int p, int h, int w, int &b, int &y, 
     x = r - y * w;
 }
 
-// Source coordinates (x, y, b) of the dS A box of input position p and tap
-// (kh, kw): the output position whose tap reads p, when p - tap is on the
-// stride grid. Anything out of range is left outside the tensor, where TMA
-// reads zeros.
-__device__ __forceinline__ void conv_src(const ConvGemmArgs &a, int p, int kh, int kw, int &sx, int &sy, int &sb) {
-    if (p >= a.P_rows) {
-        sx = 0;
-        sy = 0;
-        sb = a.ni;
-        return;
-    }
-    int b, y, x;
-    pos_decode(p, a.H, a.W, b, y, x);
-    const int ny = y + a.pad - kh, nx = x + a.pad - kw;
-    sb = b;
-    if (ny % a.stride != 0 || nx % a.stride != 0) {
-        sx = 0;
-        sy = -1;
-    } else {
-        sy = ny / a.stride;
-        sx = nx / a.stride;
-    }
-}
-
-// shared-memory plan of dS: a stage ("unit") holds the A operand of one
-// (tap, channel block) (per-position boxes, 16 KB) or, with row boxes, of
-// one (filter row kh, channel block) for all k taps of that row ((128/Mp +
-// k - 1) positions of Mp rows), and the B tiles of its taps unless the
-// transposed filters are resident; sizes are chosen on the host
+// dS row tiles group the input positions by stride class (y mod s, x mod s):
+// every position of a class is reached by the same taps, those whose offset
+// lands on the stride grid, so a tile multiplies only those. Class c holds
+// the positions y = py + ps yy, x = px + ps xx of every image, in image-major
+// order; with stride 1 the one class is the identity order.
+constexpr int DS_MAX_CLS = 4;
+struct DsClass {
+    int py, px;    // class offsets
+    int Hc, Wc;    // class grid of one image
+    int count;     // positions of the class over all images
+    int tile0;     // first row tile of the class
+    int kh0, kw0;  // first tap row / column that reaches the class
+    int nkh, nkw;  // taps reaching it: rows kh0, kh0 + ts, ..., columns alike
+};
 struct DsPlan {
     int a_bytes, b_bytes, stage, res_bytes, nst, units, taps_per_unit;
+    int ncls, ps, ts;  // classes, position step within a class, tap step
+    DsClass cls[DS_MAX_CLS];
 };
+
+__device__ __forceinline__ int ds_class(const DsPlan &pl, int rt) {
+    int c = 0;
+    while (c + 1 < pl.ncls && rt >= pl.cls[c + 1].tile0) ++c;
+    return c;
+}
+
+// input position held by row slot pp of row tile rt (of class c), or -1
+__device__ __forceinline__ int ds_pos(const ConvGemmArgs &a, const DsPlan &pl, int c, int rt, int pp, int ppt) {
+    const DsClass &q = pl.cls[c];
+    const int j = (rt - q.tile0) * ppt + pp;
+    if (j >= q.count) return -1;
+    const int per = q.Hc * q.Wc;
+    const int b = j / per, r = j - b * per;
+    const int yy = r / q.Wc, xx = r - yy * q.Wc;
+    return (b * a.H + q.py + pl.ps * yy) * a.W + q.px + pl.ps * xx;
+}
+
 constexpr int DS_MAX_STAGES = 8;
 constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
 
@@ -255,7 +260,7 @@ constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
 template <int BN, bool ROWBOX, bool RES>
 __global__ void __launch_bounds__(CONV_THREADS, 1)
     k_conv_ds(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a,
-              DsPlan pl) {
+              const __grid_constant__ DsPlan pl) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int NST = pl.nst;
@@ -306,41 +311,84 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     tc::tma_load_2d(tc::smem_u32(bres + q * BN * 128), &mapB, bres_full, tap * a.C_out + cb * 64, 0);
                 }
             }
-            uint32_t it = 0;
+            // one thread issues every copy: the loops below keep its work per
+            // unit to a few additions (positions decoded once per tile, stage
+            // and phase counted, taps stepped)
+            uint32_t it = 0;  // units issued
+            int s = 0;
+            uint32_t ph = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
                 const int rt = t / a.n_col, ct = t - rt * a.n_col;
+                const DsClass &q = pl.cls[ds_class(pl, rt)];
                 int b0 = 0, y0 = 0, x0 = 0;
-                if (ROWBOX) pos_decode(rt * ppt, a.H, a.W, b0, y0, x0);
-                for (int u = 0; u < pl.units; ++u, ++it) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
-                    if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
-                        conv_set_status(STATUS_TIMEOUT);
-                        ok = false;
-                        break;
-                    }
-                    tc::mbar_expect_tx(&full[s], (uint32_t)(pl.a_bytes + pl.b_bytes));
-                    const uint32_t st = tc::smem_u32(smem + s * pl.stage);
-                    if (ROWBOX) {
-                        // unit u = (kh, cb): output positions x0 + pad - (k - 1) .. of row y0 + pad - kh
-                        const int kh = u / ncb, cb = u - kh * ncb;
-                        tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 + a.pad - (k - 1), y0 + a.pad - kh, b0);
-                        if (!RES)
-                            for (int kw = 0; kw < k; ++kw)
-                                tc::tma_load_2d(st + pl.a_bytes + kw * BN * 128, &mapB, &full[s],
-                                                (kh * k + kw) * a.C_out + cb * 64, ct * BN);
-                    } else {
-                        const int tap = u / ncb, cb = u - tap * ncb;
-                        const int kh = tap / k, kw = tap - kh * k;
-                        for (int pp = 0; pp < ppt; ++pp) {
-                            int sx, sy, sb;
-                            conv_src(a, rt * ppt + pp, kh, kw, sx, sy, sb);
-                            tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, sb);
+                int pb[4], pyy[4], pxx[4];  // image and class coordinates of the tile's positions
+                if (ROWBOX) {
+                    pos_decode(rt * ppt, a.H, a.W, b0, y0, x0);
+                } else {
+#pragma unroll
+                    for (int pp = 0; pp < 4; ++pp) {
+                        pb[pp] = a.ni;  // padding row: a box outside the tensor (zeros)
+                        pyy[pp] = pxx[pp] = 0;
+                        const int jj = (rt - q.tile0) * ppt + pp;
+                        if (pp < ppt && jj < q.count) {
+                            const int per = q.Hc * q.Wc;
+                            pb[pp] = jj / per;
+                            const int r = jj - pb[pp] * per;
+                            pyy[pp] = r / q.Wc;
+                            pxx[pp] = r - pyy[pp] * q.Wc;
                         }
-                        if (!RES) tc::tma_load_2d(st + pl.a_bytes, &mapB, &full[s], tap * a.C_out + cb * 64, ct * BN);
                     }
                 }
+                // class coordinates: tap (kh0 + ih ts, kw0 + iw ts) reads output
+                // position (yy + by0 - ih, xx + bx0 - iw)
+                const bool cls_order = pl.ps == a.stride;
+                const int by0 = cls_order ? (q.py + a.pad - q.kh0) / pl.ts : 0;
+                const int bx0 = cls_order ? (q.px + a.pad - q.kw0) / pl.ts : 0;
+                const int nkh = ROWBOX ? k : q.nkh, nkw = ROWBOX ? 1 : q.nkw;
+                for (int ih = 0; ih < nkh && ok; ++ih)
+                    for (int iw = 0; iw < nkw && ok; ++iw)
+                        for (int cb = 0; cb < ncb; ++cb, ++it) {
+                            if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
+                                conv_set_status(STATUS_TIMEOUT);
+                                ok = false;
+                                break;
+                            }
+                            tc::mbar_expect_tx(&full[s], (uint32_t)(pl.a_bytes + pl.b_bytes));
+                            const uint32_t st = tc::smem_u32(smem + s * pl.stage);
+                            if (ROWBOX) {
+                                // unit (kh, cb): output positions x0 + pad - (k - 1) .. of row y0 + pad - kh
+                                tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 + a.pad - (k - 1), y0 + a.pad - ih, b0);
+                                if (!RES)
+                                    for (int kw = 0; kw < k; ++kw)
+                                        tc::tma_load_2d(st + pl.a_bytes + kw * BN * 128, &mapB, &full[s],
+                                                        (ih * k + kw) * a.C_out + cb * 64, ct * BN);
+                            } else {
+                                const int kh = q.kh0 + ih * pl.ts, kw = q.kw0 + iw * pl.ts;
+#pragma unroll
+                                for (int pp = 0; pp < 4; ++pp) {
+                                    if (pp >= ppt) break;
+                                    int sx, sy;
+                                    if (cls_order) {
+                                        sy = pyy[pp] + by0 - ih;
+                                        sx = pxx[pp] + bx0 - iw;
+                                    } else {  // identity order (stride above 2): off-grid taps read zeros
+                                        const int ny = pyy[pp] + a.pad - kh, nx = pxx[pp] + a.pad - kw;
+                                        const bool on = ny % a.stride == 0 && nx % a.stride == 0;
+                                        sy = on ? ny / a.stride : -1;
+                                        sx = on ? nx / a.stride : 0;
+                                    }
+                                    tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, pb[pp]);
+                                }
+                                if (!RES)
+                                    tc::tma_load_2d(st + pl.a_bytes, &mapB, &full[s], (kh * k + kw) * a.C_out + cb * 64,
+                                                    ct * BN);
+                            }
+                            if (++s == NST) {
+                                s = 0;
+                                ph ^= 1u;
+                            }
+                        }
             }
             const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
             for (uint32_t i = it - n_drain; i < it; ++i) tc::mbar_wait_spin(&full[i % NST], (i / NST) & 1u);
@@ -350,7 +398,9 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(128, BN, false, false);
-            uint32_t it = 0, j = 0;
+            uint32_t j = 0;
+            int s = 0;
+            uint32_t ph = 0;
             bool ok = true;
             if (RES && !tc::mbar_wait_spin(bres_full, 0)) {
                 conv_set_status(STATUS_TIMEOUT);
@@ -367,38 +417,43 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     tc::tc_fence_after();
                 }
                 const uint32_t acc = tmem + buf * BN;
-                for (int u = 0; u < pl.units; ++u, ++it) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
-                    if (!tc::mbar_wait_spin(&full[s], ph)) {
-                        conv_set_status(STATUS_TIMEOUT);
-                        ok = false;
-                        break;
-                    }
-                    tc::tc_fence_after();
-                    const uint32_t sa = tc::smem_u32(smem + s * pl.stage);
-                    for (int v = 0; v < tpu; ++v) {
-                        int tap, cb;
-                        uint32_t abase;
-                        if (ROWBOX) {
-                            const int kh = u / ncb;
-                            cb = u - kh * ncb;
-                            tap = kh * k + v;
-                            abase = sa + (uint32_t)((k - 1 - v) * Mp * 128);
-                        } else {
-                            tap = u / ncb;
-                            cb = u - tap * ncb;
-                            abase = sa;
-                        }
-                        const uint32_t bbase = RES ? tc::smem_u32(bres + (tap * ncb + cb) * BN * 128)
-                                                   : sa + (uint32_t)(pl.a_bytes + v * BN * 128);
+                const DsClass &q = pl.cls[ds_class(pl, t / a.n_col)];
+                const int nkh = ROWBOX ? k : q.nkh, nkw = ROWBOX ? 1 : q.nkw;
+                bool first = true;
+                for (int ih = 0; ih < nkh && ok; ++ih)
+                    for (int iw = 0; iw < nkw && ok; ++iw)
+                        for (int cb = 0; cb < ncb; ++cb) {
+                            if (!tc::mbar_wait_spin(&full[s], ph)) {
+                                conv_set_status(STATUS_TIMEOUT);
+                                ok = false;
+                                break;
+                            }
+                            tc::tc_fence_after();
+                            const uint32_t sa = tc::smem_u32(smem + s * pl.stage);
+                            for (int v = 0; v < tpu; ++v) {
+                                int tap;
+                                uint32_t abase;
+                                if (ROWBOX) {
+                                    tap = ih * k + v;
+                                    abase = sa + (uint32_t)((k - 1 - v) * Mp * 128);
+                                } else {
+                                    tap = (q.kh0 + ih * pl.ts) * k + q.kw0 + iw * pl.ts;
+                                    abase = sa;
+                                }
+                                const uint32_t bbase = RES ? tc::smem_u32(bres + (tap * ncb + cb) * BN * 128)
+                                                           : sa + (uint32_t)(pl.a_bytes + v * BN * 128);
 #pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)
-                            tc::mma_bf16(acc, tc::sdesc_sw128(abase + kk * 32), tc::sdesc_sw128(bbase + kk * 32), idesc,
-                                         (u > 0 || v > 0 || kk > 0) ? 1u : 0u);
-                    }
-                    tc::mma_commit(&empty[s]);
-                }
+                                for (int kk = 0; kk < 4; ++kk)
+                                    tc::mma_bf16(acc, tc::sdesc_sw128(abase + kk * 32), tc::sdesc_sw128(bbase + kk * 32),
+                                                 idesc, (!first || v > 0 || kk > 0) ? 1u : 0u);
+                            }
+                            first = false;
+                            tc::mma_commit(&empty[s]);
+                            if (++s == NST) {
+                                s = 0;
+                                ph ^= 1u;
+                            }
+                        }
                 if (ok) tc::mma_commit(&acc_full[buf]);
             }
         }
@@ -414,7 +469,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
             const int rt = t / a.n_col, ct = t - rt * a.n_col;
             const uint32_t buf = j & 1u;
-            const int p = rt * ppt + pp;
+            const int p = ds_pos(a, pl, ds_class(pl, rt), rt, pp, ppt);
             // the grid step and the two kernel derivatives of the input each
             // lane will own, loaded while the tile's MMAs run
             int wk[NCH];
@@ -424,7 +479,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 wk[h] = -1000;
                 wdR[h] = wdL[h] = 0.f;
                 const int col0 = ct * BN + (group + 2 * h) * 32;
-                if (p < a.P_rows) {
+                if (p >= 0) {
                     const float x = __ldg(a.t_in + (long long)p * a.C_in + col0 + lane);
                     if (isfinite(x)) {
                         const BinW w = bin_weights(a.c, x, true);
@@ -450,7 +505,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
 #pragma unroll
                 for (int u = 0; u < 32; ++u) tb[lane * EPI_LD + u] = v[u];
                 __syncwarp();
-                if (p < a.P_rows && wk[h] > -1000) {
+                if (p >= 0 && wk[h] > -1000) {
                     float g = 0.f;
                     const int k0 = wk[h] - m_base, k1 = wk[h] + 1 - m_base;
                     if (k0 >= 0 && k0 < 32 && wk[h] < a.c.M) g = fmaf(tb[k0 * EPI_LD + lane], wdR[h], g);
@@ -1279,7 +1334,6 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     const int BN = pick_bn(g.C);
     const int ppt = 128 / c.Mp;
     const int ncb = C_out / 64;
-    a.n_row = (a.P_rows + ppt - 1) / ppt;
     a.n_col = g.C / BN;
     a.t_in = t_in;
     a.g_t_in = g_t_in;
@@ -1306,6 +1360,40 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     bool rowbox = row_ok && pl.nst >= 3;
     if (!rowbox) pl = plan(false);
     if (pl.nst < 2) return cudaErrorInvalidConfiguration;
+    // stride classes (one for stride 1); a stride whose s x s classes do not
+    // fit runs every tap in the identity order, off-grid taps reading zeros
+    const bool classes = g.s * g.s <= DS_MAX_CLS;
+    pl.ps = classes ? g.s : 1;
+    pl.ts = classes ? g.s : 1;
+    pl.ncls = 0;
+    a.n_row = 0;
+    for (int py = 0; py < pl.ps; ++py)
+        for (int px = 0; px < pl.ps; ++px) {
+            DsClass q{};
+            q.py = py;
+            q.px = px;
+            q.Hc = g.H > py ? (g.H - py + pl.ps - 1) / pl.ps : 0;
+            q.Wc = g.W > px ? (g.W - px + pl.ps - 1) / pl.ps : 0;
+            q.count = ni * q.Hc * q.Wc;
+            q.kh0 = (py + g.p) % pl.ts;
+            q.kw0 = (px + g.p) % pl.ts;
+            q.nkh = q.kh0 < g.k ? (g.k - q.kh0 + pl.ts - 1) / pl.ts : 0;
+            q.nkw = q.kw0 < g.k ? (g.k - q.kw0 + pl.ts - 1) / pl.ts : 0;
+            if (q.count == 0 || q.nkh * q.nkw == 0) continue;  // no tap reaches it: its gradient stays zero
+            pl.cls[pl.ncls++] = q;
+        }
+    // most taps first, so that the persistent CTAs' last tiles are the light ones
+    for (int i = 1; i < pl.ncls; ++i)
+        for (int j = i; j > 0 && pl.cls[j].nkh * pl.cls[j].nkw > pl.cls[j - 1].nkh * pl.cls[j - 1].nkw; --j) {
+            const DsClass q = pl.cls[j];
+            pl.cls[j] = pl.cls[j - 1];
+            pl.cls[j - 1] = q;
+        }
+    for (int i = 0; i < pl.ncls; ++i) {
+        pl.cls[i].tile0 = a.n_row;
+        a.n_row += (pl.cls[i].count + ppt - 1) / ppt;
+    }
+    if (a.n_row == 0) return cudaSuccess;
     CUtensorMap mA, mB;
     if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, rowbox ? ppt + g.k - 1 : 1) ||
         !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))

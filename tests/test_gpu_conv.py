@@ -169,6 +169,14 @@ BF16_CASES = [
     (128, 6, 256, 2, (1.0, 0.25), 64),    # config 5, layer 14
     (256, 4, 256, 1, (1.0, 0.25), 64),    # config 5, layers 15-19
 ]
+# other filter sizes at stride 2: an odd grid (stride classes of unequal
+# size), 1x1 without padding (positions no tap reaches: zero gradient) and
+# 5x5 with padding 2 (one, two or three tap rows per class)
+BF16_KP_CASES = [c + (3, 1) for c in BF16_CASES] + [
+    (64, 9, 64, 2, (1.0, 0.25), 64, 3, 1),
+    (64, 8, 64, 2, (1.0, 0.25), 64, 1, 0),
+    (64, 9, 128, 2, (INF, INF), 32, 5, 2),
+]
 
 
 def gpu_spike_state(r, B, O, Ho, Wo):
@@ -180,19 +188,19 @@ def gpu_spike_state(r, B, O, Ho, Wo):
     return {"t": t, "q": tr(q).astype(int), "vdot": tr(vd), "fired": np.isfinite(t)}
 
 
-@pytest.mark.parametrize("C,H,O,stride,tau,M", BF16_CASES)
-def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
+@pytest.mark.parametrize("C,H,O,stride,tau,M,k,pad", BF16_KP_CASES)
+def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M, k, pad):
     from paper_2607_14672_gb300 import dstd
     from helpers import (bf16, bf16_ambiguous_ulp, bf16_grad_rel_bound, bf16_potential_bound, check_bf16_times,
                          conv_neurons, grid_of, kernel_max)
     B = 2
-    t, L = conv_case(B, C, H, O, 3, stride, 1, M, tau, seed=7 * C + H + O, wmean=WMEAN64[tau] * 64 / C,
+    t, L = conv_case(B, C, H, O, k, stride, pad, M, tau, seed=7 * C + H + O + k, wmean=WMEAN64[tau] * 64 / C * 9 / k ** 2,
                      gammas=(0.05, 0.01, 1e-3), silent=0.1, t_offset=0.3 * 1.2 / M)
     r = run_conv_fwd(t, L, "bf16")
     T, dt = grid_of(L)
     tv, ti = tau
     s = odstd.binning(t.reshape(B, -1), T, dt, tv, ti).reshape(B, M, C, H, H)
-    what = onet.conv_what(bf16(s), bf16(L["W"]), stride, 1)
+    what = onet.conv_what(bf16(s), bf16(L["W"]), stride, pad)
     _, _, Ho, Wo, _ = what.shape
     flat = odstd.solve(what.reshape(B, O * Ho * Wo, M), T, dt, tv, ti, 1.0)
     ctx = {k: flat[k].reshape(B, O, Ho, Wo) for k in ("t", "q", "vpeak", "vdot", "fired")}
@@ -216,20 +224,20 @@ def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M):
     _, gT = olosses.temporal_penalty(gs["t"], 0.35, 0.8, 0.05, 0.01, nrm)
     g_t_in = torch.empty_like(r["t_in"])
     g_W = torch.empty_like(r["W"])
-    dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g.transpose(0, 2, 3, 1)), stride, 1, r["p"],
+    dstd.conv_bwd(r["t_in"], r["W"], r["t_out"], r["saved"], dev(g.transpose(0, 2, 3, 1)), stride, pad, r["p"],
                   "bf16", g_t_in, g_W, r["ws"])
     torch.cuda.synchronize()
     assert dstd.device_status(clear=True) == 0
     fl = {k: gs[k].reshape(B, -1) for k in ("t", "q", "vdot", "fired")}
     gw = odstd.solve_backward(fl, (g + gT).reshape(B, -1), T, dt, tv, ti, 1.0).reshape(B, O, Ho, Wo, M)
-    gW, gsum = onet.conv_what_adjoint(bf16(gw), bf16(s), bf16(L["W"]), stride, 1)
+    gW, gsum = onet.conv_what_adjoint(bf16(gw), bf16(s), bf16(L["W"]), stride, pad)
     ds = odstd.binning(t.reshape(B, -1), T, dt, tv, ti, derivative=True).reshape(gsum.shape)
     gin = np.sum(gsum * ds, axis=1)
     cnt = (~gs["fired"]).sum((0, 2, 3))
     gW = gW - 1e-3 * nrm * cnt[:, None, None, None]
     # dw^ entries at a bf16 rounding midpoint may round either way (bf16_grad_rel_bound)
     bW, bs = onet.conv_what_adjoint(bf16_ambiguous_ulp(gw, 2.0 ** -16), np.abs(bf16(s)), np.abs(bf16(L["W"])),
-                                    stride, 1)
+                                    stride, pad)
     b_in = np.sum(bs * np.abs(ds), axis=1)
     e_w = rel_l2(host(g_W).transpose(0, 3, 1, 2), gW)
     e_g = rel_l2(host(g_t_in).transpose(0, 3, 1, 2), gin)
