@@ -179,15 +179,20 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
  *          T and Q of conv layers are divided by the spatial size).
  * Tensor-core math modes only (DSTD_MATH_F32 returns DSTD_E_UNSUPPORTED).
  * Padding taps read silent inputs.
- * In DSTD_MATH_BF16 with C_in and C_out multiples of 64 and M <= 128, the
- * layer runs as implicit GEMMs: the grid weights of the input (Eq.
- * DSTD_kernel) are written once, [B, H, W, Mp, C_in] in bf16, and each
- * filter tap reads them through shifted TMA boxes (no im2col copy); dS is
- * the transposed convolution of dw^ with the input-time gradient taken in
- * its epilogue; dW reads the same two arrays. Chunks of whole images keep
- * that scratch near 4 GiB (dstd_conv_set_chunk_images). Other shapes and
- * the three-product mode gather the binned input per tap (im2col) in chunks
- * of whole images near 1 GiB. The workspace query accounts for either. */
+ * In DSTD_MATH_BF16 with C_in and C_out multiples of 64, k <= 7 and M <= 64,
+ * the layer runs as implicit GEMMs: each input spike becomes one 8-byte
+ * record (its grid step and its two nonzero grid weights in bf16, the
+ * compact support of Eq. DSTD_kernel); from those records the binned input
+ * is either written out once per chunk ([images, H, W, Mp, C_in], no im2col
+ * expansion) and read by the forward and dW through TMA boxes shifted per
+ * filter tap, or generated tile by tap in shared memory
+ * (dstd_conv_set_operand_policy); dS is the transposed
+ * convolution of dw^ (TMA boxes shifted per tap, only the taps on the
+ * stride grid) with the input-time gradient taken in its epilogue. Chunks
+ * of whole images keep that scratch (w^ in fp32, dw^ and S in bf16) near 4 GiB
+ * (dstd_conv_set_chunk_images). Other shapes and the three-product mode
+ * gather the binned input per tap (im2col) in chunks of whole images near
+ * 1 GiB. The workspace query accounts for either. */
 size_t dstd_conv_workspace_bytes(int B, int H, int W, int C_in, int C_out, int k, int stride, int pad,
                                  const dstd_params *p, dstd_math math);
 int dstd_conv_fwd(const float *t_in, const float *W, int B, int H, int Wd, int C_in, int C_out, int k, int stride,
@@ -335,6 +340,18 @@ int dstd_set_pair_policy(int policy);
  * after setting it. Returns the previous value (max_images < 0 only reads
  * it). Process-wide; set it between calls, not while other threads launch. */
 int dstd_conv_set_chunk_images(int max_images);
+
+/* Operand of the implicit-GEMM conv forward and dW (bf16 layers above):
+ * 1 generates the binned input tile by tile in shared memory from the
+ * 8-byte records; 2 writes it out once per chunk, S [images, H, W, Mp, C_in]
+ * in bf16 (the two nonzero grid weights of each input at grid steps k and
+ * k + 1, zeros elsewhere), and the contractions read it through TMA boxes
+ * shifted per filter tap; 0 (the default) writes S wherever its writer takes
+ * the channel count (C_in <= 256, or a multiple of 256 up to 1024) and
+ * generates elsewhere. Both compute the same products. It changes the workspace size, so query again after setting
+ * it. Returns the previous value (a policy outside 0..2 only reads it).
+ * Process-wide; set it between calls. */
+int dstd_conv_set_operand_policy(int policy);
 
 /* Kernel timing (tracing). While enabled, the library brackets every kernel
  * it launches with a CUDA event pair on the launching stream and files the

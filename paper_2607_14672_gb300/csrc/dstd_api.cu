@@ -633,9 +633,26 @@ ConvBwdWs conv_bwd_layout(void *base, const ConvPlan &pl, int Cout, int Mp, OpKi
 // scratch.
 constexpr size_t kConvImplBudget = 4ull << 30;  // bytes of per-image operands per chunk
 static int g_conv_chunk_images = 0;             // 0: from the budget; else at most this many images per chunk
+// operand of the implicit-GEMM forward and dW: 0 by layer shape, 1 generated
+// on chip from the records everywhere, 2 the binned input S written out and
+// read through TMA everywhere
+static int g_conv_operand_policy = 0;
+
+// By default both contractions read S wherever its writer takes the
+// channel count: writing S costs one pass at HBM speed per chunk and
+// direction, and the TMA-fed tiles keep the tensor core fed, where the
+// generator warps (one stage per group when the filters stream) do not.
+static bool conv_fwd_tma(const ConvGeom &g, int C_out) {
+    (void)C_out;
+    return conv_bin_S_supported(g.C) && g_conv_operand_policy != 1;
+}
+static bool conv_dw_tma(const ConvGeom &g, int C_out) {
+    (void)C_out;
+    return conv_bin_S_supported(g.C) && g_conv_operand_policy != 1;
+}
 
 struct ConvImplWs {
-    __nv_bfloat16 *Wf = nullptr, *Wt = nullptr, *dwh = nullptr;
+    __nv_bfloat16 *Wf = nullptr, *Wt = nullptr, *dwh = nullptr, *S = nullptr;
     uint2 *rec = nullptr;
     float *rowsum = nullptr, *count = nullptr, *what = nullptr;
     int imgs = 1;
@@ -643,7 +660,8 @@ struct ConvImplWs {
 };
 
 int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
-    const long long per_img = (long long)g.H * g.W * g.C * 8 + (long long)g.Ho * g.Wo * Mp * C_out * 4;
+    long long per_img = (long long)g.H * g.W * g.C * 8 + (long long)g.Ho * g.Wo * Mp * C_out * 4;
+    if (conv_fwd_tma(g, C_out) || conv_dw_tma(g, C_out)) per_img += (long long)g.H * g.W * Mp * g.C * 2;
     long long imgs = (long long)(kConvImplBudget / (size_t)per_img);
     if (g_conv_chunk_images > 0 && imgs > g_conv_chunk_images) imgs = g_conv_chunk_images;
     if (imgs < 1) imgs = 1;
@@ -661,6 +679,8 @@ ConvImplWs conv_impl_layout(void *base, const ConvGeom &g, int C_out, int Mp, bo
     w.Wf = b.take<__nv_bfloat16>((size_t)C_out * K);
     w.Wt = b.take<__nv_bfloat16>((size_t)C_out * K);
     w.rec = b.take<uint2>((size_t)w.imgs * g.H * g.W * g.C);
+    if (fwd ? conv_fwd_tma(g, C_out) : conv_dw_tma(g, C_out))
+        w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * g.C);
     if (fwd)
         w.what = b.take<float>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
     else
@@ -696,10 +716,14 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         {
             Timed tm(KK_BIN, st);
             TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
+            if (ws.S) TRY(cu(launch_bin_S(ws.rec, (long long)ni * g.H * g.W, g.C, Mp, c.M, ws.S, st)));
         }
         {
             Timed tm(KK_GEMM_FWD, st);
-            TRY(cu(launch_conv_fwd_gen(g, ni, C_out, c, ws.rec, ws.Wf, ws.what, st)));
+            if (ws.S)
+                TRY(cu(launch_conv_fwd_tma(g, ni, C_out, c, ws.S, ws.Wf, ws.what, st)));
+            else
+                TRY(cu(launch_conv_fwd_gen(g, ni, C_out, c, ws.rec, ws.Wf, ws.what, st)));
         }
         Timed tm(KK_SCAN, st);
         TRY(cu(launch_scan_solve(ws.what, (long long)Mp * C_out, Mp, 1, (int)P_out, C_out, c, nullptr, ws.rowsum,
@@ -743,9 +767,13 @@ int conv_bwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         {
             Timed tm(KK_BIN_T, st);
             TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
+            if (ws.S) TRY(cu(launch_bin_S(ws.rec, (long long)ni * g.H * g.W, g.C, Mp, c.M, ws.S, st)));
         }
         Timed tm(KK_GEMM_DW, st);
-        TRY(cu(launch_conv_dw_gen(g, ni, C_out, c, ws.rec, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
+        if (ws.S)
+            TRY(cu(launch_conv_dw_tma(g, ni, C_out, c, ws.S, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
+        else
+            TRY(cu(launch_conv_dw_gen(g, ni, C_out, c, ws.rec, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
     }
     return DSTD_OK;
 }
@@ -1563,6 +1591,13 @@ int dstd_conv_set_chunk_images(int max_images) {
     if (max_images < 0) return g_conv_chunk_images;
     const int prev = g_conv_chunk_images;
     g_conv_chunk_images = max_images;
+    return prev;
+}
+
+int dstd_conv_set_operand_policy(int policy) {
+    if (policy < 0 || policy > 2) return g_conv_operand_policy;
+    const int prev = g_conv_operand_policy;
+    g_conv_operand_policy = policy;
     return prev;
 }
 

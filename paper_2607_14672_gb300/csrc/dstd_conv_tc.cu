@@ -169,7 +169,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn, bool 
 
 constexpr int CONV_NEPI = 8;                          // epilogue warps
 constexpr int CONV_THREADS = (2 + CONV_NEPI) * 32;    // + TMA producer warp + MMA warp
-constexpr int CONV_SMEM_BUDGET = 200 * 1024;
 constexpr int EPI_LD = 33;                            // per-warp transpose buffer row stride (floats)
 
 // Geometry of one implicit-GEMM launch over a chunk of ni images.
@@ -228,25 +227,32 @@ __device__ __forceinline__ int ds_class(const DsPlan &pl, int rt) {
     return c;
 }
 
-// input position held by row slot pp of row tile rt (of class c), or -1
-__device__ __forceinline__ int ds_pos(const ConvGemmArgs &a, const DsPlan &pl, int c, int rt, int pp, int ppt) {
+// position held by row slot pp of row tile rt (of class c) in a grid of
+// gh x gw positions per image (dS: the input grid; forward: the output
+// grid), or -1
+__device__ __forceinline__ int ds_pos(const DsPlan &pl, int gh, int gw, int c, int rt, int pp, int ppt) {
     const DsClass &q = pl.cls[c];
     const int j = (rt - q.tile0) * ppt + pp;
     if (j >= q.count) return -1;
     const int per = q.Hc * q.Wc;
     const int b = j / per, r = j - b * per;
     const int yy = r / q.Wc, xx = r - yy * q.Wc;
-    return (b * a.H + q.py + pl.ps * yy) * a.W + q.px + pl.ps * xx;
+    return (b * gh + q.py + pl.ps * yy) * gw + q.px + pl.ps * xx;
 }
 
 constexpr int DS_MAX_STAGES = 8;
 constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
 
 // ---------------------------------------------------------------------------
-// dS with the input-time gradient: rows (input position, m) of 128 per tile
-// (128 / Mp positions), columns BN of the C_in channels; K = k k taps x
-// blocks of 64 output channels of dw^ (the transposed convolution).
-// Persistent: CTA b takes tiles b, b + grid, ...
+// Tap-shifted contraction over a [positions][Mp][channels] bf16 operand read
+// through TMA boxes, in two modes:
+//  FWD  the forward w^ of Eq. DSTD: rows (output position, m), columns BN of
+//       the C_out channels, K = k k taps x blocks of 64 input channels of the
+//       binned input S; the epilogue stores w^ [position][channel][m].
+//  !FWD dS with the input-time gradient: rows (input position, m), columns BN
+//       of the C_in channels; K = k k taps x blocks of 64 output channels of
+//       dw^ (the transposed convolution); the epilogue takes dC/dt_in.
+// 128 / Mp positions per tile. Persistent: CTA b takes tiles b, b + grid, ...
 //   warp 0  TMA producer (one lane): A boxes and the B tiles (or, with RES,
 //           every B tile once)
 //   warp 1  TMEM allocation and MMA issue (one lane)
@@ -254,19 +260,19 @@ constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
 //              chunks (w - 2) / 4, +2, ... of the tile
 // ROWBOX (stride 1, tiles within one image row): one box of 128/Mp + k - 1
 // positions per (kh, channel block) serves all k taps kw of that filter row;
-// tap kw's A tile starts (k - 1 - kw) positions into it.
+// tap kw's A tile starts kw (FWD) or k - 1 - kw (dS) positions into it.
 // Barriers: full/empty per unit; acc_full/acc_empty per accumulator (two).
 // ---------------------------------------------------------------------------
-template <int BN, bool ROWBOX, bool RES>
+template <int BN, bool ROWBOX, bool RES, bool FWD>
 __global__ void __launch_bounds__(CONV_THREADS, 1)
-    k_conv_ds(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a,
-              const __grid_constant__ DsPlan pl) {
+    k_conv_tap_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                    ConvGemmArgs a, const __grid_constant__ DsPlan pl) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int NST = pl.nst;
     uint8_t *bres = smem + NST * pl.stage;
     float *epi = reinterpret_cast<float *>(bres + pl.res_bytes);
-    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + DS_EPI_BYTES);
+    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + (FWD ? 0 : DS_EPI_BYTES));
     uint64_t *empty = full + DS_MAX_STAGES;
     uint64_t *acc_full = empty + DS_MAX_STAGES;  // [2]
     uint64_t *acc_empty = acc_full + 2;          // [2]
@@ -278,7 +284,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
     const int ntiles = a.n_row * a.n_col;
     const int Mp = a.Mp;
     const int ppt = 128 / Mp;  // positions per tile
-    const int ncb = a.C_out >> 6;
+    const int kc = FWD ? a.C_in : a.C_out;  // channels contracted per tap
+    const int ncb = kc >> 6;
     const int k = a.k;
 
     if (threadIdx.x == 0) {
@@ -308,7 +315,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 tc::mbar_expect_tx(bres_full, (uint32_t)(nslices * BN * 128));
                 for (int q = 0; q < nslices; ++q) {
                     const int tap = q / ncb, cb = q - tap * ncb;
-                    tc::tma_load_2d(tc::smem_u32(bres + q * BN * 128), &mapB, bres_full, tap * a.C_out + cb * 64, 0);
+                    tc::tma_load_2d(tc::smem_u32(bres + q * BN * 128), &mapB, bres_full, tap * kc + cb * 64, 0);
                 }
             }
             // one thread issues every copy: the loops below keep its work per
@@ -324,7 +331,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 int b0 = 0, y0 = 0, x0 = 0;
                 int pb[4], pyy[4], pxx[4];  // image and class coordinates of the tile's positions
                 if (ROWBOX) {
-                    pos_decode(rt * ppt, a.H, a.W, b0, y0, x0);
+                    if (FWD) pos_decode(rt * ppt, a.Ho, a.Wo, b0, y0, x0);
+                    else pos_decode(rt * ppt, a.H, a.W, b0, y0, x0);
                 } else {
 #pragma unroll
                     for (int pp = 0; pp < 4; ++pp) {
@@ -337,6 +345,10 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                             const int r = jj - pb[pp] * per;
                             pyy[pp] = r / q.Wc;
                             pxx[pp] = r - pyy[pp] * q.Wc;
+                            if (FWD) {  // input origin of the output position's receptive field
+                                pyy[pp] = pyy[pp] * a.stride - a.pad;
+                                pxx[pp] = pxx[pp] * a.stride - a.pad;
+                            }
                         }
                     }
                 }
@@ -357,19 +369,27 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                             tc::mbar_expect_tx(&full[s], (uint32_t)(pl.a_bytes + pl.b_bytes));
                             const uint32_t st = tc::smem_u32(smem + s * pl.stage);
                             if (ROWBOX) {
-                                // unit (kh, cb): output positions x0 + pad - (k - 1) .. of row y0 + pad - kh
-                                tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 + a.pad - (k - 1), y0 + a.pad - ih, b0);
+                                // unit (kh, cb): FWD input positions x0 - pad .. of row y0 - pad + kh;
+                                // dS output positions x0 + pad - (k - 1) .. of row y0 + pad - kh
+                                if (FWD)
+                                    tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 - a.pad, y0 - a.pad + ih, b0);
+                                else
+                                    tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 + a.pad - (k - 1), y0 + a.pad - ih,
+                                                b0);
                                 if (!RES)
                                     for (int kw = 0; kw < k; ++kw)
                                         tc::tma_load_2d(st + pl.a_bytes + kw * BN * 128, &mapB, &full[s],
-                                                        (ih * k + kw) * a.C_out + cb * 64, ct * BN);
+                                                        (ih * k + kw) * kc + cb * 64, ct * BN);
                             } else {
                                 const int kh = q.kh0 + ih * pl.ts, kw = q.kw0 + iw * pl.ts;
 #pragma unroll
                                 for (int pp = 0; pp < 4; ++pp) {
                                     if (pp >= ppt) break;
                                     int sx, sy;
-                                    if (cls_order) {
+                                    if (FWD) {
+                                        sy = pyy[pp] + kh;
+                                        sx = pxx[pp] + kw;
+                                    } else if (cls_order) {
                                         sy = pyy[pp] + by0 - ih;
                                         sx = pxx[pp] + bx0 - iw;
                                     } else {  // identity order (stride above 2): off-grid taps read zeros
@@ -381,7 +401,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                                     tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, pb[pp]);
                                 }
                                 if (!RES)
-                                    tc::tma_load_2d(st + pl.a_bytes, &mapB, &full[s], (kh * k + kw) * a.C_out + cb * 64,
+                                    tc::tma_load_2d(st + pl.a_bytes, &mapB, &full[s], (kh * k + kw) * kc + cb * 64,
                                                     ct * BN);
                             }
                             if (++s == NST) {
@@ -435,7 +455,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                                 uint32_t abase;
                                 if (ROWBOX) {
                                     tap = ih * k + v;
-                                    abase = sa + (uint32_t)((k - 1 - v) * Mp * 128);
+                                    abase = sa + (uint32_t)((FWD ? v : k - 1 - v) * Mp * 128);
                                 } else {
                                     tap = (q.kh0 + ih * pl.ts) * k + q.kw0 + iw * pl.ts;
                                     abase = sa;
@@ -458,6 +478,36 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             }
         }
         __syncwarp();
+    } else if (FWD) {
+        // w^ [p][o][m]: for each channel o the warp's 32 lanes hold 32
+        // consecutive grid steps, one 128-byte line per store
+        const int quarter = warp & 3, group = (warp - 2) >> 2;
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        const int pp = (quarter * 32) / Mp;
+        const int m = (quarter * 32) % Mp + lane;
+        uint32_t j = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
+            const int rt = t / a.n_col, ct = t - rt * a.n_col;
+            const uint32_t buf = j & 1u;
+            const int p = ds_pos(pl, a.Ho, a.Wo, ds_class(pl, rt), rt, pp, ppt);
+            if (!tc::mbar_wait_sleep(&acc_full[buf], (j >> 1) & 1u)) {
+                conv_set_status(STATUS_TIMEOUT);
+                break;
+            }
+            tc::tc_fence_after();
+            for (int cc = group; cc < BN / 32; cc += 2) {
+                float v[32];
+                tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
+                if (p >= 0) {
+                    float *dst = a.what + ((long long)p * a.C_out + ct * BN + cc * 32) * Mp + m;
+#pragma unroll
+                    for (int u = 0; u < 32; ++u) __stcs(dst + (long long)u * Mp, v[u]);
+                }
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
+        }
     } else {
         const int quarter = warp & 3, group = (warp - 2) >> 2;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
@@ -469,7 +519,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
             const int rt = t / a.n_col, ct = t - rt * a.n_col;
             const uint32_t buf = j & 1u;
-            const int p = ds_pos(a, pl, ds_class(pl, rt), rt, pp, ppt);
+            const int p = ds_pos(pl, a.H, a.W, ds_class(pl, rt), rt, pp, ppt);
             // the grid step and the two kernel derivatives of the input each
             // lane will own, loaded while the tile's MMAs run
             int wk[NCH];
@@ -552,6 +602,76 @@ __global__ void __launch_bounds__(256) k_bin_rec(const float *__restrict__ t, lo
     }
 }
 
+// The binned input written out for the TMA-fed contractions: S [P][Mp][C]
+// bf16, row (p, m) holding grid step m of the C channels, built from the
+// records (the two nonzeros of input (p, c) at m = k and k + 1 < M, zeros
+// elsewhere). A block builds R = 256 / C consecutive positions (one for
+// C >= 256) in shared memory and writes them with one bulk copy; two
+// buffers alternate, and a thread, which owns fixed (position, channel)
+// slots of the buffers, erases the two entries it wrote in a buffer before
+// writing the new ones, so the zeros are written to shared memory once.
+constexpr int BINS_THREADS = 256;
+constexpr int BINS_MAXSPT = 4;  // channels per thread: C <= 1024
+
+__device__ __forceinline__ void bins_put(uint16_t *T, int row0, int C, int c, int kold, uint2 q, int M) {
+    if (kold != REC_SILENT) {
+        if (kold >= 0) T[(row0 + kold) * C + c] = 0;
+        if (kold + 1 < M) T[(row0 + kold + 1) * C + c] = 0;
+    }
+    const int k = (int)q.x;
+    if (k != REC_SILENT) {
+        if (k >= 0) T[(row0 + k) * C + c] = (uint16_t)(q.y & 0xffffu);
+        if (k + 1 < M) T[(row0 + k + 1) * C + c] = (uint16_t)(q.y >> 16);
+    }
+}
+
+__global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const uint2 *__restrict__ rec, int P, int C, int Mp, int M,
+                                                        __nv_bfloat16 *__restrict__ S) {
+    extern __shared__ __align__(128) uint8_t bins_smem[];
+    const int R = C >= BINS_THREADS ? 1 : BINS_THREADS / C;  // positions per group
+    const int tile = R * Mp * C;                            // elements per buffer
+    uint16_t *buf0 = reinterpret_cast<uint16_t *>(bins_smem), *buf1 = buf0 + tile;
+    const int spt = C > BINS_THREADS ? C / BINS_THREADS : (threadIdx.x < R * C ? 1 : 0);
+    const int r = C >= BINS_THREADS ? 0 : threadIdx.x / C;
+    const int c0 = C >= BINS_THREADS ? threadIdx.x : threadIdx.x - r * C;
+    for (int i = threadIdx.x; i < tile / 4; i += blockDim.x) reinterpret_cast<uint4 *>(buf0)[i] = make_uint4(0, 0, 0, 0);
+    int kold0[BINS_MAXSPT], kold1[BINS_MAXSPT];
+#pragma unroll
+    for (int j = 0; j < BINS_MAXSPT; ++j) kold0[j] = kold1[j] = REC_SILENT;
+    const int ngroups = (P + R - 1) / R;
+    int it = 0;
+    for (int gi = blockIdx.x; gi < ngroups; gi += gridDim.x, ++it) {
+        const bool odd = it & 1;
+        uint16_t *T = odd ? buf1 : buf0;
+        // the bulk copy that read this buffer two groups ago is done with it
+        if (threadIdx.x == 0 && it >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+        __syncthreads();
+        const int p = gi * R + r;
+#pragma unroll
+        for (int j = 0; j < BINS_MAXSPT; ++j) {
+            if (j < spt) {
+                const int c = c0 + j * BINS_THREADS;
+                const uint2 q = p < P ? __ldg(rec + (long long)p * C + c) : make_uint2((uint32_t)REC_SILENT, 0u);
+                bins_put(T, r * Mp, C, c, odd ? kold1[j] : kold0[j], q, M);
+                if (odd) kold1[j] = (int)q.x;
+                else kold0[j] = (int)q.x;
+            }
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int np = P - gi * R < R ? P - gi * R : R;
+            const uint32_t bytes = (uint32_t)np * Mp * C * 2;
+            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
+                             S + (long long)gi * R * Mp * C),
+                         "r"(tc::smem_u32(T)), "r"(bytes)
+                         : "memory");
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        }
+    }
+    if (threadIdx.x == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint64_t *bar, int c, int m, int p) {
     asm volatile(
         "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
@@ -600,7 +720,6 @@ __device__ __forceinline__ void gen_put_mn(uint32_t tile, int kr0, int c, int ko
 }
 
 constexpr int GEN_WARPS = 4;                                    // per generator group (one K step)
-constexpr int GEN_THREADS = (2 + CONV_NEPI + GEN_WARPS) * 32;  // 448: dW, one group
 constexpr int FWD_GEN_GROUPS = 4;                               // forward: K steps generated at once
 constexpr int FWD_THREADS = (2 + CONV_NEPI + GEN_WARPS * FWD_GEN_GROUPS) * 32;  // 832
 
@@ -688,21 +807,29 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
                 tc::mbar_wait_spin(bres_full, 0);
             } else {
                 uint32_t it = 0;
+                int s = 0;
+                uint32_t ph = 0;
                 bool ok = true;
                 for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
                     const int ct = t % a.n_col;
+                    int tap = 0, cb = 0;
                     for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
-                        const int s = it % NST;
-                        const uint32_t ph = (it / NST) & 1u;
                         if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
                             conv_set_status(STATUS_TIMEOUT);
                             ok = false;
                             break;
                         }
                         tc::mbar_expect_tx(&full_t[s], (uint32_t)Cfg::B_BYTES);
-                        const int tap = kt / ncb, cb = kt - tap * ncb;
                         tc::tma_load_2d(tc::smem_u32(smem + s * Cfg::STAGE + Cfg::A_BYTES), &mapB, &full_t[s],
                                         tap * a.C_in + cb * 64, ct * BN);
+                        if (++cb == ncb) {
+                            cb = 0;
+                            ++tap;
+                        }
+                        if (++s == NST) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
                     }
                 }
                 const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
@@ -714,7 +841,9 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(128, BN, false, false);
-            uint32_t it = 0, j = 0;
+            uint32_t j = 0;
+            int s = 0;
+            uint32_t ph = 0;
             bool ok = true;
             if (RES && !tc::mbar_wait_spin(bres_full, 0)) {
                 conv_set_status(STATUS_TIMEOUT);
@@ -730,9 +859,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
                     tc::tc_fence_after();
                 }
                 const uint32_t acc = tmem + buf * BN;
-                for (int kt = 0; kt < a.ktiles; ++kt, ++it) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
+                for (int kt = 0; kt < a.ktiles; ++kt) {
                     if ((!RES && !tc::mbar_wait_spin(&full_t[s], ph)) || !tc::mbar_wait_spin(&full_a[s], ph)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
@@ -746,6 +873,10 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
                         tc::mma_bf16(acc, tc::sdesc_sw128(sa + kk * 32), tc::sdesc_sw128(sbb + kk * 32), idesc,
                                      (kt > 0 || kk > 0) ? 1u : 0u);
                     tc::mma_commit(&empty[s]);
+                    if (++s == NST) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
                 if (ok) tc::mma_commit(&acc_full[buf]);
             }
@@ -797,36 +928,68 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
             la_kt -= a.ktiles;
             la_t += gridDim.x;
         }
-        int pc_t = -1, pb[2] = {0, 0}, py[2] = {0, 0}, px[2] = {0, 0};
+        // per slot of tile la_t: the receptive-field origin (ys, xs) and the
+        // record index of its tap (0, 0) channel block 0; the tap (la_kh,
+        // la_kw) and channel block la_cb of step la_kt advance by counting
+        int pc_t = -1, ys[2] = {0, 0}, xs[2] = {0, 0};
+        long long base[2] = {0, 0};
+        bool pv[2] = {false, false};
+        int la_kh = 0, la_kw = 0, la_cb = 0;
+        auto set_tap = [&]() {
+            const int tap = la_kt / ncb;
+            la_cb = la_kt - tap * ncb;
+            la_kh = tap / a.k;
+            la_kw = tap - la_kh * a.k;
+        };
+        set_tap();
         auto load_next = [&](uint2(&dst)[2]) {
             if (la_t < ntiles && la_t != pc_t) {
                 pc_t = la_t;
+                const int p0 = (la_t / a.n_col) * ppt;
 #pragma unroll
                 for (int u = 0; u < 2; ++u) {
-                    const int p = (la_t / a.n_col) * ppt + ((g + u * 128) >> 6);
-                    if (p < a.P_rows) pos_decode(p, a.Ho, a.Wo, pb[u], py[u], px[u]);
-                    else pb[u] = a.ni;
+                    const int slot = g + u * 128, p = p0 + (slot >> 6);
+                    pv[u] = slot < nslots && p < a.P_rows;
+                    if (pv[u]) {
+                        int b, y, x;
+                        pos_decode(p, a.Ho, a.Wo, b, y, x);
+                        ys[u] = y * a.stride - a.pad;
+                        xs[u] = x * a.stride - a.pad;
+                        base[u] = (((long long)b * a.H + ys[u]) * a.W + xs[u]) * a.C_in + (slot & 63);
+                    }
                 }
             }
-            const int tap = la_kt / ncb, cb = la_kt - tap * ncb;
-            const int kh = tap / a.k, kw = tap - kh * a.k;
+            const int off = (la_kh * a.W + la_kw) * a.C_in + la_cb * 64;
 #pragma unroll
             for (int u = 0; u < 2; ++u) {
-                const int slot = g + u * 128;
                 dst[u] = make_uint2((uint32_t)REC_SILENT, 0u);
-                const int sy = py[u] * a.stride + kh - a.pad, sx = px[u] * a.stride + kw - a.pad;
-                if (la_t < ntiles && slot < nslots && pb[u] < a.ni && sx >= 0 && sx < a.W && sy >= 0 && sy < a.H)
-                    dst[u] = __ldg(rec + (((long long)pb[u] * a.H + sy) * a.W + sx) * a.C_in + cb * 64 + (slot & 63));
+                if (la_t < ntiles && pv[u] && (unsigned)(ys[u] + la_kh) < (unsigned)a.H &&
+                    (unsigned)(xs[u] + la_kw) < (unsigned)a.W)
+                    dst[u] = __ldg(rec + base[u] + off);
             }
             la_kt += FWD_GEN_GROUPS;
-            while (la_kt >= a.ktiles && la_t < ntiles) {
-                la_kt -= a.ktiles;
-                la_t += gridDim.x;
+            if (la_kt >= a.ktiles) {
+                while (la_kt >= a.ktiles && la_t < ntiles) {
+                    la_kt -= a.ktiles;
+                    la_t += gridDim.x;
+                }
+                set_tap();
+            } else {
+#pragma unroll
+                for (int i = 0; i < FWD_GEN_GROUPS; ++i)
+                    if (++la_cb == ncb) {
+                        la_cb = 0;
+                        if (++la_kw == a.k) {
+                            la_kw = 0;
+                            ++la_kh;
+                        }
+                    }
             }
         };
 #pragma unroll
         for (int d = 0; d < GEN_AHEAD; ++d) load_next(q[d]);
-        uint32_t it = grp;
+        int s = grp;  // stage of this group's next K step, and its phase
+        uint32_t ph = 0;
         int cur_t = blockIdx.x, cur_kt = grp;
         while (cur_kt >= a.ktiles && cur_t < ntiles) {
             cur_kt -= a.ktiles;
@@ -837,8 +1000,6 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
 #pragma unroll
             for (int d = 0; d < GEN_AHEAD; ++d) {
                 if (cur_t < ntiles && ok) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
                     int w_ok = 1;
                     // generators run ahead of the MMAs: park (suspend hint) rather
                     // than poll, which would take shared-memory cycles from the
@@ -863,7 +1024,11 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
                         __syncwarp();
                         if (lane == 0) tc::mbar_arrive(&full_a[s]);
                         load_next(q[d]);
-                        it += FWD_GEN_GROUPS;
+                        s += FWD_GEN_GROUPS;
+                        if (s >= NST) {
+                            s -= NST;
+                            ph ^= 1u;
+                        }
                         cur_kt += FWD_GEN_GROUPS;
                         while (cur_kt >= a.ktiles && cur_t < ntiles) {
                             cur_kt -= a.ktiles;
@@ -906,23 +1071,6 @@ struct GenDwCfg {
         return nst * stage(G) + prev_bytes(nst, G, kpos) + 1024 + 256;
     }
 };
-
-// record of slot (row block u of the group, position kp, channel c) at K step kt
-__device__ __forceinline__ uint2 dw_record(const ConvGemmArgs &a, const uint2 *__restrict__ rec, int rg, int G, int kt,
-                                           int u, int kp, int c) {
-    const int kpos = 64 / a.Mp;
-    const int ncb = a.C_in >> 6;
-    const int rb = rg * 2 * G + u;
-    const int p = kt * kpos + kp;
-    if (p >= a.P_rows || rb >= a.k * a.k * ncb) return make_uint2((uint32_t)REC_SILENT, 0u);
-    int b, y, x;
-    pos_decode(p, a.Ho, a.Wo, b, y, x);
-    const int tap = rb / ncb, cb = rb - tap * ncb;
-    const int kh = tap / a.k, kw = tap - kh * a.k;
-    const int sx = x * a.stride + kw - a.pad, sy = y * a.stride + kh - a.pad;
-    if (sx < 0 || sx >= a.W || sy < 0 || sy >= a.H) return make_uint2((uint32_t)REC_SILENT, 0u);
-    return __ldg(rec + (((long long)b * a.H + sy) * a.W + sx) * a.C_in + cb * 64 + c);
-}
 
 template <int BN>
 __global__ void __launch_bounds__(DW_THREADS, 1)
@@ -986,13 +1134,13 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
     if (warp == 0) {
         if (lane == 0) {
             uint32_t it = 0;
+            int s = 0;
+            uint32_t ph = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
                 int rg, ct, kt0, nkt;
                 decode(t, rg, ct, kt0, nkt);
                 for (int i = 0; i < nkt; ++i, ++it) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
                     if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
@@ -1002,6 +1150,10 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                     const uint32_t sb = tc::smem_u32(smem + s * STG + a_bytes);
                     for (int gq = 0; gq < BN / 64; ++gq)
                         tma_load_3d(sb + gq * 8192, &mapD, &full_t[s], ct * BN + gq * 64, 0, (kt0 + i) * kpos);
+                    if (++s == NST) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
             }
             const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
@@ -1011,7 +1163,9 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(128, BN, true, true);
-            uint32_t it = 0, j = 0;
+            uint32_t j = 0;
+            int s = 0;
+            uint32_t ph = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
                 int rg, ct, kt0, nkt;
@@ -1023,9 +1177,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                     }
                     tc::tc_fence_after();
                 }
-                for (int i = 0; i < nkt; ++i, ++it) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
+                for (int i = 0; i < nkt; ++i) {
                     if (!tc::mbar_wait_spin(&full_t[s], ph) || !tc::mbar_wait_spin(&full_a[s], ph)) {
                         conv_set_status(STATUS_TIMEOUT);
                         ok = false;
@@ -1041,6 +1193,10 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                                          tc::sdesc_sw128_mn(sbb + kk * 2048, 8192), idesc, (i > 0 || kk > 0) ? 1u : 0u);
                     }
                     tc::mma_commit(&empty[s]);
+                    if (++s == NST) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
                 if (ok) tc::mma_commit(acc_full);
             }
@@ -1085,51 +1241,91 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
         const int gw = warp - (2 + CONV_NEPI);
         const int grp = gw / GEN_WARPS;
         const int g = (gw % GEN_WARPS) * 32 + lane;
-        // advance a (tile, step) position by n K steps of this CTA's sequence
-        auto advance = [&](int &t, int &i, int n) {
-            while (t < ntiles && n > 0) {
-                int rg, ct, kt0, nkt;
-                decode(t, rg, ct, kt0, nkt);
-                const int left = nkt - i;
-                if (n < left) {
-                    i += n;
-                    n = 0;
-                } else {
-                    n -= left;
-                    i = 0;
-                    t += gridDim.x;
+        // K steps of tile t (split-K tiles have kt_per_split but the last)
+        auto tile_nkt = [&](int t) {
+            int rg, ct, kt0, nkt;
+            decode(t, rg, ct, kt0, nkt);
+            return nkt;
+        };
+        // advance a (tile t, step i of its nkt) cursor by n K steps of this CTA's sequence
+        auto advance = [&](int &t, int &i, int &nkt, int n) {
+            i += n;
+            while (t < ntiles && i >= nkt) {
+                i -= nkt;
+                t += gridDim.x;
+                if (t < ntiles) nkt = tile_nkt(t);
+            }
+        };
+        // this thread's slots v: (row block u, position kp, channel c = g & 63),
+        // fixed per tile: packed channel cb 64 + c (bits 0-15), kh (16-19),
+        // kw (20-23), kp (24), u (25-29), valid (31)
+        uint32_t spk[DW_MAX_SPT];
+        int pk_t = -1, la_rg = 0, la_kt0 = 0;
+        auto slot_consts = [&](int t) {
+            pk_t = t;
+            int ct, nkt;
+            decode(t, la_rg, ct, la_kt0, nkt);
+            const int ncb = a.C_in >> 6, nrb = a.k * a.k * ncb;
+#pragma unroll
+            for (int v = 0; v < DW_MAX_SPT; ++v) {
+                const int slot = g + v * 128, qq = slot >> 6;
+                const int u = qq / kpos, kp = qq - u * kpos;
+                const int rb = la_rg * 2 * G + u;
+                spk[v] = 0u;
+                if (slot < slots && rb < nrb) {
+                    const int tap = rb / ncb, cb = rb - tap * ncb;
+                    const int kh = tap / a.k, kw = tap - kh * a.k;
+                    spk[v] = (uint32_t)(cb * 64 + (g & 63)) | ((uint32_t)kh << 16) | ((uint32_t)kw << 20) |
+                             ((uint32_t)kp << 24) | ((uint32_t)u << 25) | 0x80000000u;
                 }
             }
         };
         uint2 q[DW_AHEAD][DW_MAX_SPT];
-        int la_t = blockIdx.x, la_i = 0;  // the K step whose records load next
-        advance(la_t, la_i, grp);
+        int la_t = blockIdx.x, la_i = 0, la_nkt = la_t < ntiles ? tile_nkt(la_t) : 0;  // next K step to load
+        advance(la_t, la_i, la_nkt, grp);
         auto load_next = [&](uint2(&dst)[DW_MAX_SPT]) {
-            int rg = 0, ct, kt0 = 0, nkt = 0;
-            if (la_t < ntiles) decode(la_t, rg, ct, kt0, nkt);
+            int ys[2] = {0, 0}, xs[2] = {0, 0};
+            long long base[2] = {0, 0};
+            bool pv[2] = {false, false};
+            if (la_t < ntiles) {
+                if (la_t != pk_t) slot_consts(la_t);
+                // the step's kpos (<= 2) output positions
 #pragma unroll
-            for (int v = 0; v < DW_MAX_SPT; ++v) {
-                const int slot = g + v * 128;
-                dst[v] = make_uint2((uint32_t)REC_SILENT, 0u);
-                if (la_t < ntiles && slot < slots) {
-                    const int c = slot & 63, qq = slot >> 6;
-                    dst[v] = dw_record(a, rec, rg, G, kt0 + la_i, qq / kpos, qq % kpos, c);
+                for (int kp = 0; kp < 2; ++kp) {
+                    const int p = (la_kt0 + la_i) * kpos + kp;
+                    pv[kp] = kp < kpos && p < a.P_rows;
+                    if (pv[kp]) {
+                        int b, y, x;
+                        pos_decode(p, a.Ho, a.Wo, b, y, x);
+                        ys[kp] = y * a.stride - a.pad;
+                        xs[kp] = x * a.stride - a.pad;
+                        base[kp] = (((long long)b * a.H + ys[kp]) * a.W + xs[kp]) * a.C_in;
+                    }
                 }
             }
-            advance(la_t, la_i, DW_GEN_GROUPS);
+#pragma unroll
+            for (int v = 0; v < DW_MAX_SPT; ++v) {
+                dst[v] = make_uint2((uint32_t)REC_SILENT, 0u);
+                const uint32_t w = spk[v];
+                const int kh = (w >> 16) & 15, kw = (w >> 20) & 15, kp = (w >> 24) & 1;
+                const int ysk = kp ? ys[1] : ys[0], xsk = kp ? xs[1] : xs[0];
+                if ((w >> 31) && (kp ? pv[1] : pv[0]) && (unsigned)(ysk + kh) < (unsigned)a.H &&
+                    (unsigned)(xsk + kw) < (unsigned)a.W)
+                    dst[v] = __ldg(rec + (kp ? base[1] : base[0]) + (kh * a.W + kw) * a.C_in + (w & 0xffffu));
+            }
+            advance(la_t, la_i, la_nkt, DW_GEN_GROUPS);
         };
 #pragma unroll
         for (int d = 0; d < DW_AHEAD; ++d) load_next(q[d]);
-        uint32_t it = grp;
-        int cur_t = blockIdx.x, cur_i = 0;
-        advance(cur_t, cur_i, grp);
+        int s = grp;  // stage of this group's next K step, and its phase
+        uint32_t ph = 0;
+        int cur_t = blockIdx.x, cur_i = 0, cur_nkt = cur_t < ntiles ? tile_nkt(cur_t) : 0;
+        advance(cur_t, cur_i, cur_nkt, grp);
         bool ok = true;
         while (cur_t < ntiles && ok) {
 #pragma unroll
             for (int d = 0; d < DW_AHEAD; ++d) {
                 if (cur_t < ntiles && ok) {
-                    const int s = it % NST;
-                    const uint32_t ph = (it / NST) & 1u;
                     int w_ok = 1;
                     if (lane == 0) w_ok = tc::mbar_wait(&empty[s], ph ^ 1u) ? 1 : 0;
                     w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
@@ -1142,11 +1338,12 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                         for (int v = 0; v < DW_MAX_SPT; ++v) {
                             const int slot = g + v * 128;
                             if (slot < slots) {
-                                const int c = slot & 63, qq = slot >> 6;
-                                const int kp = qq % kpos, u = qq / kpos;
+                                // slot geometry from the index alone (the packed constants
+                                // may already belong to the next tile)
+                                const int qq = slot >> 6, u = kpos == 1 ? qq : qq >> 1, kp = qq - u * kpos;
                                 int16_t *pk = prevk + s * slots + slot;
-                                gen_put_mn(tile0 + (u >> 1) * 16384 + (u & 1) * 8192, kp * Mp, c, (int)*pk, q[d][v],
-                                           a.c.M);
+                                gen_put_mn(tile0 + (u >> 1) * 16384 + (u & 1) * 8192, kp * Mp, g & 63, (int)*pk,
+                                           q[d][v], a.c.M);
                                 *pk = (int16_t)(int)q[d][v].x;
                             }
                         }
@@ -1154,11 +1351,228 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                         __syncwarp();
                         if (lane == 0) tc::mbar_arrive(&full_a[s]);
                         load_next(q[d]);
-                        it += DW_GEN_GROUPS;
-                        advance(cur_t, cur_i, DW_GEN_GROUPS);
+                        s += DW_GEN_GROUPS;
+                        if (s >= NST) {
+                            s -= NST;
+                            ph ^= 1u;
+                        }
+                        advance(cur_t, cur_i, cur_nkt, DW_GEN_GROUPS);
                     }
                 }
             }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tc::tmem_dealloc(tmem, tcols);
+}
+
+// ---------------------------------------------------------------------------
+// dW from the binned input S [P_in][Mp][C_in] read through TMA: the same CTA
+// tiles as k_conv_dw_gen (G row tiles of 128 filter rows (tap, channel) by
+// BN output channels over a range of K = (output position, m), split-K),
+// with the A tiles loaded instead of generated: per K step and row block
+// (tap, 64 channels) one box (64 channels, Mp grid steps) of S per output
+// position of the step, at the input position the tap reads (outside the
+// image: zeros), and BN / 64 boxes of dw^. Warps: 0 TMA (one lane), 1 MMA,
+// 2-9 epilogue (fp32 atomics into g_W, dead-neuron term on the first split).
+// ---------------------------------------------------------------------------
+constexpr int DWT_MAX_STAGES = 8;
+
+template <int BN>
+__global__ void __launch_bounds__(CONV_THREADS, 1)
+    k_conv_dw_tma(const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD, ConvGemmArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const int G = a.groups, NST = a.nst;
+    const int Mp = a.Mp;
+    const int kpos = 64 / Mp;
+    const int a_bytes = G * 128 * 128;
+    const int STG = a_bytes + BN * 128;
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + NST * STG);
+    uint64_t *empty = full + DWT_MAX_STAGES;
+    uint64_t *acc_full = empty + DWT_MAX_STAGES;
+    uint64_t *acc_empty = acc_full + 1;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_grp = a.n_row;
+    const int ntiles = n_grp * a.n_col * a.n_split;
+    const int ncb = a.C_in >> 6;
+    const int nrb = a.k * a.k * ncb;  // row blocks (tap, 64 channels)
+    const int Ktot = a.k * a.k * a.C_in;
+    uint32_t tcols = 32;
+    while ((int)tcols < G * BN) tcols <<= 1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NST; ++s) {
+            tc::mbar_init(&full[s], 1);
+            tc::mbar_init(&empty[s], 1);
+        }
+        tc::mbar_init(acc_full, 1);
+        tc::mbar_init(acc_empty, CONV_NEPI);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) tc::tmem_alloc(tmem_slot, tcols);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    auto decode = [&](int t, int &rg, int &ct, int &kt0, int &nkt) {
+        const int per = n_grp * a.n_col;
+        const int sp = t / per, rem = t - sp * per;
+        rg = rem / a.n_col;
+        ct = rem - rg * a.n_col;
+        kt0 = sp * a.kt_per_split;
+        nkt = a.ktiles - kt0;
+        if (nkt > a.kt_per_split) nkt = a.kt_per_split;
+    };
+
+    if (warp == 0) {
+        if (lane == 0) {
+            const uint32_t tx = (uint32_t)(STG);  // 2G row blocks x kpos boxes of Mp x 128 B, and the dw^ tile
+            uint32_t it = 0;
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                int rg, ct, kt0, nkt;
+                decode(t, rg, ct, kt0, nkt);
+                // the tile's row blocks: (kh, kw, channel block), or none
+                int rkh[2 * DWG_MAX_G], rkw[2 * DWG_MAX_G], rcb[2 * DWG_MAX_G];
+#pragma unroll
+                for (int u = 0; u < 2 * DWG_MAX_G; ++u) {
+                    const int rb = rg * 2 * G + u;
+                    rkh[u] = -1;
+                    rkw[u] = rcb[u] = 0;
+                    if (u < 2 * G && rb < nrb) {
+                        const int tap = rb / ncb;
+                        rcb[u] = rb - tap * ncb;
+                        rkh[u] = tap / a.k;
+                        rkw[u] = tap - rkh[u] * a.k;
+                    }
+                }
+                // first output position of the first K step, stepped by one
+                int p = kt0 * kpos, b, y, x;
+                pos_decode(p, a.Ho, a.Wo, b, y, x);
+                for (int i = 0; i < nkt; ++i, ++it) {
+                    if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
+                        conv_set_status(STATUS_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    tc::mbar_expect_tx(&full[s], tx);
+                    const uint32_t st = tc::smem_u32(smem + s * STG);
+                    for (int kp = 0; kp < kpos; ++kp) {
+                        const bool pv = p < a.P_rows;
+                        const int ys = y * a.stride - a.pad, xs = x * a.stride - a.pad;
+#pragma unroll
+                        for (int u = 0; u < 2 * DWG_MAX_G; ++u) {
+                            if (u < 2 * G) {
+                                // a row block past the filter rows or a position past the
+                                // chunk reads a box outside the tensor (zeros)
+                                const bool on = pv && rkh[u] >= 0;
+                                tma_load_5d(st + (u >> 1) * 16384 + (u & 1) * 8192 + kp * Mp * 128, &mapS, &full[s],
+                                            rcb[u] * 64, 0, on ? xs + rkw[u] : 0, on ? ys + rkh[u] : 0, on ? b : a.ni);
+                            }
+                        }
+                        ++p;
+                        if (++x == a.Wo) {
+                            x = 0;
+                            if (++y == a.Ho) {
+                                y = 0;
+                                ++b;
+                            }
+                        }
+                    }
+                    const uint32_t sb = st + a_bytes;
+                    for (int gq = 0; gq < BN / 64; ++gq)
+                        tma_load_3d(sb + gq * 8192, &mapD, &full[s], ct * BN + gq * 64, 0, (kt0 + i) * kpos);
+                    if (++s == NST) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+            }
+            const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
+            for (uint32_t i = it - n_drain; i < it; ++i) tc::mbar_wait_spin(&full[i % NST], (i / NST) & 1u);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(128, BN, true, true);
+            uint32_t j = 0;
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++j) {
+                int rg, ct, kt0, nkt;
+                decode(t, rg, ct, kt0, nkt);
+                if (j >= 1) {
+                    if (!tc::mbar_wait_spin(acc_empty, (j - 1) & 1u)) {
+                        conv_set_status(STATUS_TIMEOUT);
+                        break;
+                    }
+                    tc::tc_fence_after();
+                }
+                for (int i = 0; i < nkt; ++i) {
+                    if (!tc::mbar_wait_spin(&full[s], ph)) {
+                        conv_set_status(STATUS_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    tc::tc_fence_after();
+                    const uint32_t sa = tc::smem_u32(smem + s * STG);
+                    const uint32_t sbb = sa + a_bytes;
+                    for (int gi = 0; gi < G; ++gi) {
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc::mma_bf16(tmem + gi * BN, tc::sdesc_sw128_mn(sa + gi * 16384 + kk * 2048, 8192),
+                                         tc::sdesc_sw128_mn(sbb + kk * 2048, 8192), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    tc::mma_commit(&empty[s]);
+                    if (++s == NST) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+                if (ok) tc::mma_commit(acc_full);
+            }
+        }
+        __syncwarp();
+    } else {
+        const int quarter = warp & 3, group = (warp - 2) >> 2;
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        const int r = quarter * 32 + lane;
+        uint32_t j = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
+            int rg, ct, kt0, nkt;
+            decode(t, rg, ct, kt0, nkt);
+            if (!tc::mbar_wait_sleep(acc_full, j & 1u)) {
+                conv_set_status(STATUS_TIMEOUT);
+                break;
+            }
+            tc::tc_fence_after();
+            const bool first = kt0 == 0;
+            for (int gi = 0; gi < G; ++gi) {
+                const int kidx = (rg * G + gi) * 128 + r;
+                for (int cc = group; cc < BN / 32; cc += 2) {
+                    float v[32];
+                    tc::tmem_ld32(tmem + lane_base + gi * BN + cc * 32, v);
+                    if (kidx < Ktot) {
+                        const int o0 = ct * BN + cc * 32;
+#pragma unroll
+                        for (int u = 0; u < 32; ++u) {
+                            const float add = (first && a.count) ? a.qcoef * a.count[o0 + u] : 0.f;
+                            atomicAdd(a.g_W + (long long)(o0 + u) * Ktot + kidx, v[u] + add);
+                        }
+                    }
+                }
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(acc_empty);
         }
     }
     tc::tc_fence_before();
@@ -1266,16 +1680,16 @@ static cudaError_t launch_dw_gen_bn(const uint2 *rec, const CUtensorMap &mD, Con
     return cudaGetLastError();
 }
 
-template <int BN, bool ROWBOX, bool RES>
-static cudaError_t launch_ds_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
-                                cudaStream_t st) {
-    const int smem = pl.nst * pl.stage + pl.res_bytes + DS_EPI_BYTES + 1024 + 256;
-    cudaError_t e =
-        cudaFuncSetAttribute(k_conv_ds<BN, ROWBOX, RES>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+template <int BN, bool ROWBOX, bool RES, bool FWD>
+static cudaError_t launch_tap_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
+                                 cudaStream_t st) {
+    const int smem = pl.nst * pl.stage + pl.res_bytes + (FWD ? 0 : DS_EPI_BYTES) + 1024 + 256;
+    cudaError_t e = cudaFuncSetAttribute(k_conv_tap_gemm<BN, ROWBOX, RES, FWD>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ntiles = a.n_row * a.n_col;
     const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_ds<BN, ROWBOX, RES><<<grid, CONV_THREADS, smem, st>>>(mA, mB, a, pl);
+    k_conv_tap_gemm<BN, ROWBOX, RES, FWD><<<grid, CONV_THREADS, smem, st>>>(mA, mB, a, pl);
     return cudaGetLastError();
 }
 
@@ -1298,7 +1712,7 @@ static ConvGemmArgs base_args(const ConvGeom &g, int ni, const LifConst &c) {
 }  // namespace
 
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp) {
-    return g.C % 64 == 0 && C_out % 64 == 0 && (Mp == 32 || Mp == 64 || Mp == 128) && g.k <= 7 &&
+    return g.C % 64 == 0 && C_out % 64 == 0 && (Mp == 32 || Mp == 64) && g.k <= 7 &&
            g.C * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
 }
 
@@ -1324,6 +1738,20 @@ cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, __nv_bf
     return cudaGetLastError();
 }
 
+// shared-memory plan of the tap-shifted contraction (see DsPlan)
+static DsPlan tap_plan(int k, int ppt, int Mp, int BN, bool resident, long long res, bool rowbox, int epi_bytes, int ncb) {
+    DsPlan pl{};
+    pl.taps_per_unit = rowbox ? k : 1;
+    pl.a_bytes = rowbox ? (ppt + k - 1) * Mp * 128 : 128 * 128;
+    pl.b_bytes = resident ? 0 : pl.taps_per_unit * BN * 128;
+    pl.stage = (pl.a_bytes + pl.b_bytes + 1023) & ~1023;
+    pl.res_bytes = resident ? (int)res : 0;
+    pl.units = (rowbox ? k : k * k) * ncb;
+    const int nst = (GEN_SMEM_MAX - pl.res_bytes - epi_bytes - 1280) / pl.stage;
+    pl.nst = nst > DS_MAX_STAGES ? DS_MAX_STAGES : nst;
+    return pl;
+}
+
 // dS of ni images with the input-time gradient: dw^ [ni Ho Wo][Mp][C_out],
 // Wt [C_in][k k C_out], t_in [ni H W][C_in] -> g_t_in (zeroed first)
 cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *dW_hat,
@@ -1343,18 +1771,7 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     // at stride 1 when every tile lies within one image row
     const long long res = (long long)g.k * g.k * ncb * BN * 128;
     const bool resident = a.n_col == 1 && res <= 80 * 1024;
-    auto plan = [&](bool rowbox) {
-        DsPlan pl{};
-        pl.taps_per_unit = rowbox ? g.k : 1;
-        pl.a_bytes = rowbox ? (ppt + g.k - 1) * c.Mp * 128 : 128 * 128;
-        pl.b_bytes = resident ? 0 : pl.taps_per_unit * BN * 128;
-        pl.stage = (pl.a_bytes + pl.b_bytes + 1023) & ~1023;
-        pl.res_bytes = resident ? (int)res : 0;
-        pl.units = (rowbox ? g.k : g.k * g.k) * ncb;
-        int nst = (GEN_SMEM_MAX - pl.res_bytes - DS_EPI_BYTES - 1280) / pl.stage;
-        pl.nst = nst > DS_MAX_STAGES ? DS_MAX_STAGES : nst;
-        return pl;
-    };
+    auto plan = [&](bool rowbox) { return tap_plan(g.k, ppt, c.Mp, BN, resident, res, rowbox, DS_EPI_BYTES, ncb); };
     const bool row_ok = g.s == 1 && g.W % ppt == 0 && ppt + g.k - 1 <= 256;
     DsPlan pl = plan(row_ok);
     bool rowbox = row_ok && pl.nst >= 3;
@@ -1399,15 +1816,147 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
         !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))
         return cudaErrorInvalidValue;
 #define DSTD_DS(BNV)                                                                                   \
-    if (rowbox) return resident ? launch_ds_bn<BNV, true, true>(mA, mB, a, pl, st)                     \
-                                : launch_ds_bn<BNV, true, false>(mA, mB, a, pl, st);                   \
-    return resident ? launch_ds_bn<BNV, false, true>(mA, mB, a, pl, st) : launch_ds_bn<BNV, false, false>(mA, mB, a, pl, st);
+    if (rowbox) return resident ? launch_tap_bn<BNV, true, true, false>(mA, mB, a, pl, st)             \
+                                : launch_tap_bn<BNV, true, false, false>(mA, mB, a, pl, st);           \
+    return resident ? launch_tap_bn<BNV, false, true, false>(mA, mB, a, pl, st)                        \
+                    : launch_tap_bn<BNV, false, false, false>(mA, mB, a, pl, st);
     switch (BN) {
         case 256: { DSTD_DS(256) }
         case 128: { DSTD_DS(128) }
         default: { DSTD_DS(64) }
     }
 #undef DSTD_DS
+}
+
+// forward w^ [ni Ho Wo][C_out][Mp] of ni images from the binned input
+// S [ni H W][Mp][C_in] and the filters Wf [C_out][k k C_in]
+cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
+                                const __nv_bfloat16 *Wf, float *what, cudaStream_t st) {
+    ConvGemmArgs a = base_args(g, ni, c);
+    a.C_out = C_out;
+    a.P_rows = ni * g.Ho * g.Wo;
+    a.what = what;
+    const int BN = pick_bn(C_out);
+    const int ppt = 128 / c.Mp;
+    const int ncb = g.C / 64;
+    a.n_col = C_out / BN;
+    a.n_row = (a.P_rows + ppt - 1) / ppt;
+    if (a.n_row == 0) return cudaSuccess;
+    const long long res = (long long)g.k * g.k * ncb * BN * 128;
+    const bool resident = a.n_col == 1 && res <= 80 * 1024;
+    const bool row_ok = g.s == 1 && g.Wo % ppt == 0 && ppt + g.k - 1 <= 256;
+    DsPlan pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, row_ok, 0, ncb);
+    const bool rowbox = row_ok && pl.nst >= 3;
+    if (!rowbox) pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, false, 0, ncb);
+    if (pl.nst < 2) return cudaErrorInvalidConfiguration;
+    // every tap of every output position, in position order
+    pl.ncls = 1;
+    pl.ps = pl.ts = 1;
+    DsClass &q = pl.cls[0];
+    q.py = q.px = 0;
+    q.Hc = g.Ho;
+    q.Wc = g.Wo;
+    q.count = a.P_rows;
+    q.tile0 = 0;
+    q.kh0 = q.kw0 = 0;
+    q.nkh = q.nkw = g.k;
+    CUtensorMap mA, mB;
+    if (!map_act(&mA, S, ni, g.H, g.W, c.Mp, g.C, rowbox ? ppt + g.k - 1 : 1) ||
+        !map_mat(&mB, Wf, C_out, g.k * g.k * g.C, BN))
+        return cudaErrorInvalidValue;
+#define DSTD_FT(BNV)                                                                                   \
+    if (rowbox) return resident ? launch_tap_bn<BNV, true, true, true>(mA, mB, a, pl, st)              \
+                                : launch_tap_bn<BNV, true, false, true>(mA, mB, a, pl, st);            \
+    return resident ? launch_tap_bn<BNV, false, true, true>(mA, mB, a, pl, st)                         \
+                    : launch_tap_bn<BNV, false, false, true>(mA, mB, a, pl, st);
+    switch (BN) {
+        case 256: { DSTD_FT(256) }
+        case 128: { DSTD_FT(128) }
+        default: { DSTD_FT(64) }
+    }
+#undef DSTD_FT
+}
+
+// dW of ni images from the binned input S [ni H W][Mp][C_in] and dw^
+// [ni Ho Wo][Mp][C_out], added into g_W (zeroed by the caller before the
+// first chunk)
+cudaError_t launch_conv_dw_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
+                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
+                               cudaStream_t st) {
+    ConvGemmArgs a = base_args(g, ni, c);
+    a.C_out = C_out;
+    a.P_rows = ni * g.Ho * g.Wo;
+    if (a.P_rows == 0) return cudaSuccess;
+    const int BN = pick_bn(C_out);
+    const int Ktot = g.k * g.k * g.C;
+    const int row_tiles = (Ktot / 64 + 1) / 2;
+    const int kpos = 64 / c.Mp;
+    const int extra = 1024 + 256;  // alignment and barriers
+    auto stg = [&](int G) { return G * 16384 + BN * 128; };
+    // the most row tiles per CTA (one dw^ tile feeds them all) that TMEM
+    // holds and that leave three stages
+    int gmax = 512 / BN;
+    if (gmax > DWG_MAX_G) gmax = DWG_MAX_G;
+    while (gmax > 1 && 3 * stg(gmax) + extra > GEN_SMEM_MAX) --gmax;
+    const int ngrp = (row_tiles + gmax - 1) / gmax;
+    a.groups = (row_tiles + ngrp - 1) / ngrp;
+    a.n_row = (row_tiles + a.groups - 1) / a.groups;
+    a.n_col = C_out / BN;
+    a.ktiles = (a.P_rows + kpos - 1) / kpos;
+    const int tiles = a.n_row * a.n_col;
+    int splits = (2 * conv_num_sms() + tiles - 1) / tiles;
+    const int max_splits = (a.ktiles + 15) / 16;
+    if (splits > max_splits) splits = max_splits;
+    if (splits < 1) splits = 1;
+    a.kt_per_split = (a.ktiles + splits - 1) / splits;
+    a.n_split = (a.ktiles + a.kt_per_split - 1) / a.kt_per_split;
+    int nst = (GEN_SMEM_MAX - extra) / stg(a.groups);
+    if (nst > DWT_MAX_STAGES) nst = DWT_MAX_STAGES;
+    if (nst < 2) return cudaErrorInvalidConfiguration;
+    a.nst = nst;
+    a.g_W = g_W;
+    a.count = count;
+    a.qcoef = qcoef;
+    CUtensorMap mS, mD;
+    if (!map_act(&mS, S, ni, g.H, g.W, c.Mp, g.C, 1) || !map_act3(&mD, dW_hat, (long long)a.P_rows, c.Mp, C_out))
+        return cudaErrorInvalidValue;
+    const int smem = nst * stg(a.groups) + extra;
+    const int ntiles = tiles * a.n_split;
+    const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
+#define DSTD_DWT(BNV)                                                                                            \
+    {                                                                                                            \
+        cudaError_t e = cudaFuncSetAttribute(k_conv_dw_tma<BNV>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem); \
+        if (e != cudaSuccess) return e;                                                                          \
+        k_conv_dw_tma<BNV><<<grid, CONV_THREADS, smem, st>>>(mS, mD, a);                                         \
+        return cudaGetLastError();                                                                               \
+    }
+    switch (BN) {
+        case 256: DSTD_DWT(256)
+        case 128: DSTD_DWT(128)
+        default: DSTD_DWT(64)
+    }
+#undef DSTD_DWT
+}
+
+bool conv_bin_S_supported(int C) {
+    return C % 64 == 0 && C <= BINS_THREADS * BINS_MAXSPT && (C <= BINS_THREADS || C % BINS_THREADS == 0);
+}
+
+cudaError_t launch_bin_S(const uint2 *rec, long long P, int C, int Mp, int M, __nv_bfloat16 *S, cudaStream_t st) {
+    if (!conv_bin_S_supported(C) || P >= (1ll << 31) || P * Mp * C >= (1ll << 31)) return cudaErrorInvalidValue;
+    if (P == 0) return cudaSuccess;
+    const int R = C >= BINS_THREADS ? 1 : BINS_THREADS / C;
+    const int smem = 2 * R * Mp * C * 2;
+    if (smem > 227 * 1024) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k_bin_S, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const long long ngroups = (P + R - 1) / R;
+    int per_sm = (227 * 1024) / smem;
+    if (per_sm > 8) per_sm = 8;
+    long long blocks = (long long)per_sm * conv_num_sms();
+    if (blocks > ngroups) blocks = ngroups;
+    k_bin_S<<<(unsigned)blocks, BINS_THREADS, smem, st>>>(rec, (int)P, C, Mp, M, S);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_bin_rec(const float *t, long long n, const LifConst &c, uint2 *rec, cudaStream_t st) {

@@ -300,8 +300,8 @@ struct ConvGeom {
     int B, H, W, C, Ho, Wo, k, s, p;
 };
 // Implicit-GEMM conv layer in bf16 (dstd_conv_tc.cu), for C_in and C_out
-// multiples of 64 and Mp in {32, 64, 128}: no im2col operand. ni = images of
-// the chunk; positions NHWC.
+// multiples of 64 and Mp in {32, 64}: no im2col operand. ni = images of the
+// chunk; positions NHWC.
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp);
 // dw^ [P][Mp][C] bf16 from the saved state [P][C]; silent counts per channel
 // added into count (zeroed by the caller)
@@ -323,6 +323,17 @@ cudaError_t launch_bin_rec(const float *t, long long n, const LifConst &c, uint2
 cudaError_t launch_conv_fwd_gen(const ConvGeom &g, int ni, int C_out, const LifConst &c, const uint2 *rec,
                                 const __nv_bfloat16 *Wf, float *what, cudaStream_t st);
 cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifConst &c, const uint2 *rec,
+                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
+                               cudaStream_t st);
+// the binned input written out, S [P][Mp][C] bf16, from the records, and the
+// forward contraction that reads it through tap-shifted TMA boxes (w^ as for
+// launch_conv_fwd_gen)
+bool conv_bin_S_supported(int C);  // channel counts the S writer takes
+cudaError_t launch_bin_S(const uint2 *rec, long long P, int C, int Mp, int M, __nv_bfloat16 *S, cudaStream_t st);
+cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
+                                const __nv_bfloat16 *Wf, float *what, cudaStream_t st);
+// dW from S and dw^ (added into g_W as for launch_conv_dw_gen)
+cudaError_t launch_conv_dw_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
                                const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
                                cudaStream_t st);
 cudaError_t conv_status_read(unsigned int *out, int clear);

@@ -21,7 +21,7 @@ ERRORS = {0: "ok", -1: "invalid argument", -2: "unsupported size or mode", -3: "
 EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning", "dstd_dense_what",
            "dstd_scan_solve", "dstd_dense_fwd", "dstd_dense_fwd_ce", "dstd_dense_bwd", "dstd_ce_loss", "dstd_sum_t_loss",
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
-           "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_conv_set_chunk_images", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
+           "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_conv_set_chunk_images", "dstd_conv_set_operand_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd",
            "dstd_exact_workspace_bytes", "dstd_exact_fwd", "dstd_concat_channels", "dstd_split_channels",
            "dstd_ms_saved_bytes", "dstd_ms_workspace_bytes", "dstd_dense_fwd_ms", "dstd_dense_bwd_ms")
@@ -90,6 +90,7 @@ def load(path=None):
         "dstd_timing_collect": (_I, []),
         "dstd_set_pair_policy": (_I, [_I]),
         "dstd_conv_set_chunk_images": (_I, [_I]),
+        "dstd_conv_set_operand_policy": (_I, [_I]),
         "dstd_exact_workspace_bytes": (_SZ, [_I, _I, _I]),
         "dstd_exact_fwd": (_I, [_P, _P, _I, _I, _I, _PP, _P, _P, _SZ, _P]),
         "dstd_kernel_kind_count": (_I, []),
@@ -408,6 +409,13 @@ def conv_set_chunk_images(max_images):
     the scratch budget). Returns the previous cap; query the workspace size
     again afterwards."""
     return int(load().dstd_conv_set_chunk_images(int(max_images)))
+
+
+def conv_set_operand_policy(policy):
+    """Operand of the implicit-GEMM conv forward and dW: 0 by layer shape,
+    1 generated on chip, 2 the binned input written out and read through
+    TMA. Returns the previous policy; query the workspace size again."""
+    return int(load().dstd_conv_set_operand_policy(int(policy)))
 
 
 def timing_collect():

@@ -188,8 +188,21 @@ def gpu_spike_state(r, B, O, Ho, Wo):
     return {"t": t, "q": tr(q).astype(int), "vdot": tr(vd), "fired": np.isfinite(t)}
 
 
+@pytest.mark.parametrize("policy", [1, 2], ids=["generated", "tma"])
 @pytest.mark.parametrize("C,H,O,stride,tau,M,k,pad", BF16_KP_CASES)
-def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M, k, pad):
+def test_conv_bf16_matches_rounded_oracle(C, H, O, stride, tau, M, k, pad, policy):
+    """Both operand paths of the forward and dW (binned input generated in
+    shared memory from the records, or written out and read through TMA)
+    against the oracle on bf16-rounded operands."""
+    from paper_2607_14672_gb300 import dstd
+    prev = dstd.conv_set_operand_policy(policy)
+    try:
+        _conv_bf16_case(C, H, O, stride, tau, M, k, pad)
+    finally:
+        dstd.conv_set_operand_policy(prev)
+
+
+def _conv_bf16_case(C, H, O, stride, tau, M, k, pad):
     from paper_2607_14672_gb300 import dstd
     from helpers import (bf16, bf16_ambiguous_ulp, bf16_grad_rel_bound, bf16_potential_bound, check_bf16_times,
                          conv_neurons, grid_of, kernel_max)
