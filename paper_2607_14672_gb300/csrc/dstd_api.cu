@@ -660,8 +660,9 @@ struct ConvImplWs {
 };
 
 int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
-    long long per_img = (long long)g.H * g.W * g.C * 8 + (long long)g.Ho * g.Wo * Mp * C_out * 4;
-    if (conv_fwd_tma(g, C_out) || conv_dw_tma(g, C_out)) per_img += (long long)g.H * g.W * Mp * g.C * 2;
+    long long per_img = (long long)g.Ho * g.Wo * Mp * C_out * 4;
+    per_img += (conv_fwd_tma(g, C_out) || conv_dw_tma(g, C_out)) ? (long long)g.H * g.W * Mp * g.C * 2
+                                                                   : (long long)g.H * g.W * g.C * 8;
     long long imgs = (long long)(kConvImplBudget / (size_t)per_img);
     if (g_conv_chunk_images > 0 && imgs > g_conv_chunk_images) imgs = g_conv_chunk_images;
     if (imgs < 1) imgs = 1;
@@ -678,9 +679,10 @@ ConvImplWs conv_impl_layout(void *base, const ConvGeom &g, int C_out, int Mp, bo
     w.count = b.take<float>(C_out);
     w.Wf = b.take<__nv_bfloat16>((size_t)C_out * K);
     w.Wt = b.take<__nv_bfloat16>((size_t)C_out * K);
-    w.rec = b.take<uint2>((size_t)w.imgs * g.H * g.W * g.C);
     if (fwd ? conv_fwd_tma(g, C_out) : conv_dw_tma(g, C_out))
         w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * g.C);
+    else
+        w.rec = b.take<uint2>((size_t)w.imgs * g.H * g.W * g.C);
     if (fwd)
         w.what = b.take<float>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
     else
@@ -715,8 +717,10 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         const long long P_out = (long long)ni * g.Ho * g.Wo;
         {
             Timed tm(KK_BIN, st);
-            TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
-            if (ws.S) TRY(cu(launch_bin_S(ws.rec, (long long)ni * g.H * g.W, g.C, Mp, c.M, ws.S, st)));
+            if (ws.S)
+                TRY(cu(launch_bin_S(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+            else
+                TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
         {
             Timed tm(KK_GEMM_FWD, st);
@@ -766,8 +770,10 @@ int conv_bwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         }
         {
             Timed tm(KK_BIN_T, st);
-            TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
-            if (ws.S) TRY(cu(launch_bin_S(ws.rec, (long long)ni * g.H * g.W, g.C, Mp, c.M, ws.S, st)));
+            if (ws.S)
+                TRY(cu(launch_bin_S(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+            else
+                TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
         Timed tm(KK_GEMM_DW, st);
         if (ws.S)

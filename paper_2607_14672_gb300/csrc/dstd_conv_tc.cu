@@ -65,72 +65,164 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // ---------------------------------------------------------------------------
 // dC/dw^_{p,m,o} = -g K(t - T_m) / v^'(t) for m <= q (0 after the spike's
 // interval and for silent neurons), g = upstream + dT/dt, into [P][Mp][C_out]
-// bf16. A thread takes 8 consecutive neurons of one position (16 bytes per
-// row). K(x), x = t - T_m, falls along m by the factors e^{av dt}, e^{aI dt}
-// from its value at m = 0; the spike's own bin and the one before it (x <
-// 2 dt, where (e^{-av x} - e^{-aI x}) / lam cancels) take the accurate form.
-// Silent neurons are counted per output channel (grid-stride loop, a fixed
-// channel group per thread, one atomic per thread and channel at the end).
+// bf16. A warp writes one position (or one 256-channel segment of it) at a
+// time, a contiguous block of its rows: a thread takes 8 consecutive neurons
+// and every R-th grid step (R = 32 / (channels / 8) rows per warp store, so
+// each store instruction writes up to 512 contiguous bytes). C_out is at
+// most 256 or a multiple of 256. K(x), x = t - T_m, falls along m by the factors
+// e^{av dt}, e^{aI dt}; a thread steps R grid steps at a time. The spike's own
+// bin and the one before it (x < 2 dt, where (e^{-av x} - e^{-aI x}) / lam
+// cancels) take the accurate form. Silent neurons are counted per output
+// channel (the thread of row phase 0 of a channel group adds its counts).
 // ---------------------------------------------------------------------------
+#ifndef DWHAT_NPT
+#define DWHAT_NPT 4
+#endif
+// NPT consecutive bf16 of one row, streamed (evict-first)
+template <int NPT>
+__device__ __forceinline__ void dwhat_store(__nv_bfloat16 *p, const float (&v)[NPT]) {
+    if constexpr (NPT == 8)
+        __stcs(reinterpret_cast<uint4 *>(p), make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                                        pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7])));
+    else
+        __stcs(reinterpret_cast<uint2 *>(p), make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3])));
+}
+
+template <int NPT>
 __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_out, const int *__restrict__ qv,
                                                    const float *__restrict__ sv, const float *__restrict__ vd,
                                                    const float *__restrict__ g_up, long long P, int C, LifConst c,
                                                    __nv_bfloat16 *__restrict__ D, float *count) {
-    const int groups = C >> 3;
-    const int tpb = blockDim.x;
-    const int per_blk = tpb / groups;  // positions per block iteration (blockDim a multiple of groups)
-    const int g = threadIdx.x % groups, pl = threadIdx.x / groups;
-    const int c0 = g * 8;
-    float cnt[8];
+    const int nseg = (C + 32 * NPT - 1) / (32 * NPT);  // segments of a position
+    constexpr int SEGC = 32 * NPT;                    // channels of a segment: one per lane x NPT
+    const int groups = (C < SEGC ? C : SEGC) / NPT;   // NPT-neuron groups of a segment (<= 32)
+    const int R = 32 / groups;                        // rows of a warp store
+    const int lane = threadIdx.x & 31;
+    if (lane >= R * groups) return;                   // idle lanes (C = 192)
+    const int g = lane % groups, r = lane / groups;
+    const int wpb = blockDim.x >> 5;
+    const long long wid = (long long)blockIdx.x * wpb + (threadIdx.x >> 5), nw = (long long)gridDim.x * wpb;
+    float cnt[NPT];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) cnt[u] = 0.f;
-    const float fv = __expf(c.av * c.dt), fI = __expf(c.aI * c.dt);
-    if (pl < per_blk) {
-        for (long long p = (long long)blockIdx.x * per_blk + pl; p < P; p += (long long)gridDim.x * per_blk) {
-            int q[8];
-            float coef[8], ev[8], eI[8], x[8], Kq[8], Kq1[8];
+    for (int u = 0; u < NPT; ++u) cnt[u] = 0.f;
+    const float fv = __expf(c.av * c.dt * R), fI = __expf(c.aI * c.dt * R);
+    int c0 = g * NPT;
+    for (long long item = wid; item < P * nseg; item += nw) {
+        long long p = item;
+        if (nseg > 1) {
+            p = item / nseg;
+            const int seg = (int)(item - p * nseg);
+            // counts of the previous segment's channels
+            if (r == 0) {
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const long long idx = p * C + c0 + u;
-                q[u] = qv[idx];
-                coef[u] = 0.f;
-                x[u] = 0.f;
-                Kq[u] = Kq1[u] = 0.f;
-                if (q[u] < c.M) {
-                    float pv, pg;
-                    penalty_T(c, t_out[idx], pv, pg);
-                    coef[u] = -((g_up ? g_up[idx] : 0.f) + pg) / vd[idx];
-                    const float s0 = sv[idx];
-                    x[u] = s0 + (float)q[u] * c.dt;  // t - T_0
-                    Kq[u] = kernel_K(c, s0);
-                    Kq1[u] = kernel_K(c, s0 + c.dt);
-                } else {
-                    cnt[u] += 1.f;
-                }
-                ev[u] = __expf(-c.av * x[u]);
-                eI[u] = __expf(-c.aI * x[u]);
+                for (int u = 0; u < NPT; ++u)
+                    if (cnt[u] != 0.f) {
+                        if (count) atomicAdd(&count[c0 + u], cnt[u]);
+                        cnt[u] = 0.f;
+                    }
             }
-            uint4 *dst = reinterpret_cast<uint4 *>(D + p * (long long)c.Mp * C + c0);
-            const int step = C >> 3;
-            for (int m = 0; m < c.Mp; ++m) {
-                float v[8];
+            c0 = seg * SEGC + g * NPT;
+        }
+        // every input of the 8 neurons first, without branches
+        int q[NPT];
+        float tt[NPT], gu[NPT], vv[NPT], ss[NPT];
+        const long long idx0 = p * C + c0;
 #pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const float Kf = c.lam_zero ? x[u] * ev[u] : (ev[u] - eI[u]) * c.inv_lam;
-                    const float K = (m == q[u]) ? Kq[u] : ((m == q[u] - 1) ? Kq1[u] : Kf);
-                    v[u] = (m <= q[u] && q[u] < c.M) ? coef[u] * K : 0.f;
-                    ev[u] *= fv;
-                    eI[u] *= fI;
-                    x[u] -= c.dt;
+        for (int u = 0; u < NPT; ++u) {
+            q[u] = __ldg(qv + idx0 + u);
+            tt[u] = __ldg(t_out + idx0 + u);
+            gu[u] = g_up ? __ldg(g_up + idx0 + u) : 0.f;
+            vv[u] = __ldg(vd + idx0 + u);
+            ss[u] = __ldg(sv + idx0 + u);
+        }
+        // per neuron: the recurrence terms at this thread's first row r, the
+        // two accurate rows, and the band [m_lo, m_hi] holding them
+        float a[NPT], b[NPT], K1[NPT], K0[NPT];
+        int m_lo = c.Mp, m_hi = -1;
+#pragma unroll
+        for (int u = 0; u < NPT; ++u) {
+            a[u] = b[u] = K1[u] = K0[u] = 0.f;
+            if (q[u] < c.M) {
+                float pv, pg;
+                penalty_T(c, tt[u], pv, pg);
+                const float coef = -(gu[u] + pg) / vv[u];
+                const float s0 = ss[u];
+                const float x = s0 + (float)(q[u] - r) * c.dt;  // t - T_r
+                K0[u] = coef * kernel_K(c, s0);
+                K1[u] = coef * kernel_K(c, s0 + c.dt);
+                if (c.lam_zero) {
+                    a[u] = coef * __expf(-c.av * x);
+                    b[u] = x;
+                } else {
+                    a[u] = coef * c.inv_lam * __expf(-c.av * x);
+                    b[u] = coef * c.inv_lam * __expf(-c.aI * x);
                 }
-                dst[(long long)m * step] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                                                      pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+                m_lo = min(m_lo, q[u] - 1);
+                m_hi = max(m_hi, q[u]);
+            } else {
+                if (r == 0) cnt[u] += 1.f;
+                q[u] = -1;
             }
         }
-    }
-    if (count) {
+        __nv_bfloat16 *dst = D + p * (long long)c.Mp * C + c0;
+        const int step = C;
+        const float dtR = c.dt * R;
+        int m = r;
+        if (c.lam_zero) {
+            for (; m < m_lo; m += R) {
+                float v[NPT];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
+                for (int u = 0; u < NPT; ++u) {
+                    v[u] = a[u] * b[u];
+                    a[u] *= fv;
+                    b[u] -= dtR;
+                }
+                dwhat_store<NPT>(dst + (long long)m * step, v);
+            }
+            for (; m <= m_hi; m += R) {
+                float v[NPT];
+#pragma unroll
+                for (int u = 0; u < NPT; ++u) {
+                    const float d = a[u] * b[u];
+                    v[u] = m < q[u] - 1 ? d : (m == q[u] - 1 ? K1[u] : (m == q[u] ? K0[u] : 0.f));
+                    a[u] *= fv;
+                    b[u] -= dtR;
+                }
+                dwhat_store<NPT>(dst + (long long)m * step, v);
+            }
+        } else {
+            for (; m < m_lo; m += R) {
+                float v[NPT];
+#pragma unroll
+                for (int u = 0; u < NPT; ++u) {
+                    v[u] = a[u] - b[u];
+                    a[u] *= fv;
+                    b[u] *= fI;
+                }
+                dwhat_store<NPT>(dst + (long long)m * step, v);
+            }
+            for (; m <= m_hi; m += R) {
+                float v[NPT];
+#pragma unroll
+                for (int u = 0; u < NPT; ++u) {
+                    const float d = a[u] - b[u];
+                    v[u] = m < q[u] - 1 ? d : (m == q[u] - 1 ? K1[u] : (m == q[u] ? K0[u] : 0.f));
+                    a[u] *= fv;
+                    b[u] *= fI;
+                }
+                dwhat_store<NPT>(dst + (long long)m * step, v);
+            }
+        }
+        if (m < c.Mp) {
+            float z[NPT];
+#pragma unroll
+            for (int u = 0; u < NPT; ++u) z[u] = 0.f;
+            for (; m < c.Mp; m += R) dwhat_store<NPT>(dst + (long long)m * step, z);
+        }
+    }
+    if (count && r == 0) {
+#pragma unroll
+        for (int u = 0; u < NPT; ++u)
             if (cnt[u] != 0.f) atomicAdd(&count[c0 + u], cnt[u]);
     }
 }
@@ -589,23 +681,26 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
 // ---------------------------------------------------------------------------
 constexpr int REC_SILENT = -128;
 
+// the record of one input spike time x (+inf: silent)
+__device__ __forceinline__ uint2 bin_record(const LifConst &c, float x) {
+    uint2 r = make_uint2((uint32_t)REC_SILENT, 0u);
+    if (isfinite(x)) {
+        const BinW w = bin_weights(c, x, false);
+        if (w.k >= -1 && w.k < c.M) r = make_uint2((uint32_t)w.k, pack_bf16x2(w.wR, w.wL));
+    }
+    return r;
+}
+
 __global__ void __launch_bounds__(256) k_bin_rec(const float *__restrict__ t, long long n, LifConst c,
                                                  uint2 *__restrict__ rec) {
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
-        const float x = __ldg(t + i);
-        uint2 r = make_uint2((uint32_t)REC_SILENT, 0u);
-        if (isfinite(x)) {
-            const BinW w = bin_weights(c, x, false);
-            if (w.k >= -1 && w.k < c.M) r = make_uint2((uint32_t)w.k, pack_bf16x2(w.wR, w.wL));
-        }
-        rec[i] = r;
-    }
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
+        rec[i] = bin_record(c, __ldg(t + i));
 }
 
 // The binned input written out for the TMA-fed contractions: S [P][Mp][C]
-// bf16, row (p, m) holding grid step m of the C channels, built from the
-// records (the two nonzeros of input (p, c) at m = k and k + 1 < M, zeros
-// elsewhere). A block builds R = 256 / C consecutive positions (one for
+// bf16, row (p, m) holding grid step m of the C channels, from the spike
+// times t [P][C] (each input's record, as k_bin_rec forms it: the two
+// nonzeros of input (p, c) at m = k and k + 1 < M, zeros elsewhere). A block builds R = 256 / C consecutive positions (one for
 // C >= 256) in shared memory and writes them with one bulk copy; two
 // buffers alternate, and a thread, which owns fixed (position, channel)
 // slots of the buffers, erases the two entries it wrote in a buffer before
@@ -625,8 +720,9 @@ __device__ __forceinline__ void bins_put(uint16_t *T, int row0, int C, int c, in
     }
 }
 
-__global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const uint2 *__restrict__ rec, int P, int C, int Mp, int M,
+__global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const float *__restrict__ t, int P, int C, LifConst lc,
                                                         __nv_bfloat16 *__restrict__ S) {
+    const int Mp = lc.Mp, M = lc.M;
     extern __shared__ __align__(128) uint8_t bins_smem[];
     const int R = C >= BINS_THREADS ? 1 : BINS_THREADS / C;  // positions per group
     const int tile = R * Mp * C;                            // elements per buffer
@@ -651,7 +747,8 @@ __global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const uint2 *__restrict_
         for (int j = 0; j < BINS_MAXSPT; ++j) {
             if (j < spt) {
                 const int c = c0 + j * BINS_THREADS;
-                const uint2 q = p < P ? __ldg(rec + (long long)p * C + c) : make_uint2((uint32_t)REC_SILENT, 0u);
+                const uint2 q =
+                    p < P ? bin_record(lc, __ldg(t + (long long)p * C + c)) : make_uint2((uint32_t)REC_SILENT, 0u);
                 bins_put(T, r * Mp, C, c, odd ? kold1[j] : kold0[j], q, M);
                 if (odd) kold1[j] = (int)q.x;
                 else kold0[j] = (int)q.x;
@@ -1712,21 +1809,21 @@ static ConvGemmArgs base_args(const ConvGeom &g, int ni, const LifConst &c) {
 }  // namespace
 
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp) {
-    return g.C % 64 == 0 && C_out % 64 == 0 && (Mp == 32 || Mp == 64) && g.k <= 7 &&
-           g.C * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
+    return g.C % 64 == 0 && C_out % 64 == 0 && (C_out <= 256 || C_out % 256 == 0) && (Mp == 32 || Mp == 64) &&
+           g.k <= 7 && g.C * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
 }
 
 cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                              long long P, int C, const LifConst &c, __nv_bfloat16 *D, float *count,
                              cudaStream_t st) {
-    if (C % 8 != 0 || C / 8 > 256) return cudaErrorInvalidValue;
-    const int groups = C / 8;
-    const int per_blk = 256 / groups;
-    long long blocks = (P + per_blk - 1) / per_blk;
+    // a warp covers one position or one segment of 32 NPT channels of it
+    constexpr int NPT = DWHAT_NPT;
+    if (C % 64 != 0 || (C > 32 * NPT && C % (32 * NPT) != 0)) return cudaErrorInvalidValue;
+    long long blocks = (P * ((C + 32 * NPT - 1) / (32 * NPT)) + 7) / 8;  // 8 warps per block
     const long long cap = 8ll * conv_num_sms();
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    k_dwhat_pmc<<<(unsigned)blocks, 256, 0, st>>>(t_out, q, s, vdot, g_up, P, C, c, D, count);
+    k_dwhat_pmc<NPT><<<(unsigned)blocks, 256, 0, st>>>(t_out, q, s, vdot, g_up, P, C, c, D, count);
     return cudaGetLastError();
 }
 
@@ -1942,7 +2039,8 @@ bool conv_bin_S_supported(int C) {
     return C % 64 == 0 && C <= BINS_THREADS * BINS_MAXSPT && (C <= BINS_THREADS || C % BINS_THREADS == 0);
 }
 
-cudaError_t launch_bin_S(const uint2 *rec, long long P, int C, int Mp, int M, __nv_bfloat16 *S, cudaStream_t st) {
+cudaError_t launch_bin_S(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st) {
+    const int Mp = c.Mp;
     if (!conv_bin_S_supported(C) || P >= (1ll << 31) || P * Mp * C >= (1ll << 31)) return cudaErrorInvalidValue;
     if (P == 0) return cudaSuccess;
     const int R = C >= BINS_THREADS ? 1 : BINS_THREADS / C;
@@ -1955,7 +2053,7 @@ cudaError_t launch_bin_S(const uint2 *rec, long long P, int C, int Mp, int M, __
     if (per_sm > 8) per_sm = 8;
     long long blocks = (long long)per_sm * conv_num_sms();
     if (blocks > ngroups) blocks = ngroups;
-    k_bin_S<<<(unsigned)blocks, BINS_THREADS, smem, st>>>(rec, (int)P, C, Mp, M, S);
+    k_bin_S<<<(unsigned)blocks, BINS_THREADS, smem, st>>>(t, (int)P, C, c, S);
     return cudaGetLastError();
 }
 

@@ -325,11 +325,11 @@ cudaError_t launch_conv_fwd_gen(const ConvGeom &g, int ni, int C_out, const LifC
 cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifConst &c, const uint2 *rec,
                                const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
                                cudaStream_t st);
-// the binned input written out, S [P][Mp][C] bf16, from the records, and the
+// the binned input written out, S [P][Mp][C] bf16, from the spike times, and the
 // forward contraction that reads it through tap-shifted TMA boxes (w^ as for
 // launch_conv_fwd_gen)
 bool conv_bin_S_supported(int C);  // channel counts the S writer takes
-cudaError_t launch_bin_S(const uint2 *rec, long long P, int C, int Mp, int M, __nv_bfloat16 *S, cudaStream_t st);
+cudaError_t launch_bin_S(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st);
 cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
                                 const __nv_bfloat16 *Wf, float *what, cudaStream_t st);
 // dW from S and dw^ (added into g_W as for launch_conv_dw_gen)
