@@ -683,7 +683,7 @@ ConvImplWs conv_impl_layout(void *base, const ConvGeom &g, int C_out, int Mp, bo
         w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * g.C);
     else
         w.rec = b.take<uint2>((size_t)w.imgs * g.H * g.W * g.C);
-    if (fwd)
+    if (fwd && !w.S)
         w.what = b.take<float>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
     else
         w.dwh = b.take<__nv_bfloat16>((size_t)w.imgs * g.Ho * g.Wo * Mp * C_out);
@@ -722,12 +722,15 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
             else
                 TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
+        if (ws.S) {  // the scan runs in the contraction's epilogue
+            Timed tm(KK_GEMM_FWD, st);
+            TRY(cu(launch_conv_fwd_tma(g, ni, C_out, c, ws.S, ws.Wf, ws.rowsum, t_out + out_off, sv.q + out_off,
+                                       sv.s + out_off, sv.vdot + out_off, penalty, st)));
+            continue;
+        }
         {
             Timed tm(KK_GEMM_FWD, st);
-            if (ws.S)
-                TRY(cu(launch_conv_fwd_tma(g, ni, C_out, c, ws.S, ws.Wf, ws.what, st)));
-            else
-                TRY(cu(launch_conv_fwd_gen(g, ni, C_out, c, ws.rec, ws.Wf, ws.what, st)));
+            TRY(cu(launch_conv_fwd_gen(g, ni, C_out, c, ws.rec, ws.Wf, ws.what, st)));
         }
         Timed tm(KK_SCAN, st);
         TRY(cu(launch_scan_solve(ws.what, (long long)Mp * C_out, Mp, 1, (int)P_out, C_out, c, nullptr, ws.rowsum,

@@ -281,6 +281,12 @@ struct ConvGemmArgs {
     int nst;             // generated-operand kernels: pipeline stages
     int res_bytes;       // generated-operand forward: resident filter bytes (0: streamed)
     int groups;          // generated-operand dW: row tiles per CTA
+    // forward with the scan in its epilogue: per output neuron [P_out][C_out]
+    float *t_out;
+    int *q_out;
+    float *s_out, *vdot_out;
+    const float *rowsum;  // dead-neuron term per output channel
+    float *penalty;       // [4] sums, or null
     LifConst c;
 };
 
@@ -334,13 +340,19 @@ __device__ __forceinline__ int ds_pos(const DsPlan &pl, int gh, int gw, int c, i
 
 constexpr int DS_MAX_STAGES = 8;
 constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
+// forward epilogue: per (epilogue group, position of the tile) the w^ rows
+// of Mp / 32 chunks of 32 neurons, Mp + 4 floats each (Mp = 64: 2 x 2 x 2 x
+// 32 x 68 floats; Mp = 32: 2 x 4 x 1 x 32 x 36)
+constexpr int FWD_EPI_BYTES = 2 * 2 * 2 * 32 * 68 * 4;
 
 // ---------------------------------------------------------------------------
 // Tap-shifted contraction over a [positions][Mp][channels] bf16 operand read
 // through TMA boxes, in two modes:
 //  FWD  the forward w^ of Eq. DSTD: rows (output position, m), columns BN of
 //       the C_out channels, K = k k taps x blocks of 64 input channels of the
-//       binned input S; the epilogue stores w^ [position][channel][m].
+//       binned input S; the epilogue runs the scan/solve/select of each
+//       neuron on its w^ column (Eq. LIF_Vmem_DSTD, the first threshold
+//       crossing) and writes the spike outputs: w^ never leaves the chip.
 //  !FWD dS with the input-time gradient: rows (input position, m), columns BN
 //       of the C_in channels; K = k k taps x blocks of 64 output channels of
 //       dw^ (the transposed convolution); the epilogue takes dC/dt_in.
@@ -364,7 +376,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
     const int NST = pl.nst;
     uint8_t *bres = smem + NST * pl.stage;
     float *epi = reinterpret_cast<float *>(bres + pl.res_bytes);
-    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + (FWD ? 0 : DS_EPI_BYTES));
+    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + (FWD ? FWD_EPI_BYTES : DS_EPI_BYTES));
     uint64_t *empty = full + DS_MAX_STAGES;
     uint64_t *acc_full = empty + DS_MAX_STAGES;  // [2]
     uint64_t *acc_empty = acc_full + 2;          // [2]
@@ -387,7 +399,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         }
         for (int u = 0; u < 2; ++u) {
             tc::mbar_init(&acc_full[u], 1);
-            tc::mbar_init(&acc_empty[u], CONV_NEPI);
+            // the forward's epilogue groups take alternate tiles (one per accumulator)
+            tc::mbar_init(&acc_empty[u], FWD ? CONV_NEPI / 2 : CONV_NEPI);
         }
         tc::mbar_init(bres_full, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -571,34 +584,89 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         }
         __syncwarp();
     } else if (FWD) {
-        // w^ [p][o][m]: for each channel o the warp's 32 lanes hold 32
-        // consecutive grid steps, one 128-byte line per store
+        // Scan in the epilogue. Epilogue group g takes the tiles of
+        // accumulator g (every other tile). Warp w of the group reads TMEM
+        // lane quarter w % 4 (grid steps mq .. mq + 31 of position pp); per
+        // round the qpp = Mp / 32 warps of a position write qpp chunks of 32
+        // channels as neuron-major rows of their buffers, then, after a
+        // barrier over those warps, each walks one chunk's 32 neurons, one per
+        // lane, as the scan kernel does.
         const int quarter = warp & 3, group = (warp - 2) >> 2;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-        const int pp = (quarter * 32) / Mp;
-        const int m = (quarter * 32) % Mp + lane;
-        uint32_t j = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
+        const int qpp = Mp >> 5;  // lane quarters per position
+        const int pp = quarter / qpp, wip = quarter - pp * qpp, mq = wip * 32;
+        const int LDB = Mp + 4;
+        float *pbuf = epi + (group * ppt + pp) * qpp * 32 * LDB;
+        const int bar_id = 1 + group * ppt + pp;  // named barrier of the position's warps
+        auto sync_pos = [&]() {
+            if (qpp == 1) __syncwarp();
+            else asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "r"(qpp * 32) : "memory");
+        };
+        auto any_pos = [&](bool x) -> bool {
+            if (qpp == 1) return __any_sync(0xffffffffu, x);
+            uint32_t r;
+            asm volatile(
+                "{\n"
+                ".reg .pred pi, po;\n"
+                "setp.ne.u32 pi, %1, 0;\n"
+                "barrier.cta.red.or.pred po, %2, %3, pi;\n"
+                "selp.u32 %0, 1, 0, po;\n"
+                "}\n"
+                : "=r"(r)
+                : "r"((uint32_t)x), "r"(bar_id), "r"(qpp * 32)
+                : "memory");
+            return r != 0;
+        };
+        const int rounds = (BN / 32) / qpp;
+        float pacc[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int j = group, t = blockIdx.x + group * gridDim.x; t < ntiles; j += 2, t += 2 * gridDim.x) {
             const int rt = t / a.n_col, ct = t - rt * a.n_col;
-            const uint32_t buf = j & 1u;
+            const uint32_t buf = (uint32_t)group;
             const int p = ds_pos(pl, a.Ho, a.Wo, ds_class(pl, rt), rt, pp, ppt);
-            if (!tc::mbar_wait_sleep(&acc_full[buf], (j >> 1) & 1u)) {
+            // an expired wait ends the role of every warp of the position
+            // together, so that none is left at their barrier
+            const bool fail = !tc::mbar_wait_sleep(&acc_full[buf], (uint32_t)(j >> 1) & 1u);
+            if (any_pos(fail)) {
                 conv_set_status(STATUS_TIMEOUT);
                 break;
             }
             tc::tc_fence_after();
-            for (int cc = group; cc < BN / 32; cc += 2) {
-                float v[32];
-                tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
-                if (p >= 0) {
-                    float *dst = a.what + ((long long)p * a.C_out + ct * BN + cc * 32) * Mp + m;
+            for (int r = 0; r < rounds; ++r) {
+                for (int k = 0; k < qpp; ++k) {
+                    float v[32];
+                    tc::tmem_ld32(tmem + lane_base + buf * BN + (r * qpp + k) * 32, v);
+                    float *tb = pbuf + k * 32 * LDB;
 #pragma unroll
-                    for (int u = 0; u < 32; ++u) __stcs(dst + (long long)u * Mp, v[u]);
+                    for (int u = 0; u < 32; ++u) tb[u * LDB + mq + lane] = v[u];
                 }
+                if (r == rounds - 1) {  // the tile's last TMEM read of this warp
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
+                }
+                sync_pos();
+                if (p >= 0) {
+                    const float *row = pbuf + (wip * 32 + lane) * LDB;
+                    ScanState st;
+                    scan_reset(st, a.c.M);
+                    float vv = 0.f, I = 0.f;
+                    for (int m0 = 0; m0 < a.c.M; m0 += 32) {
+                        const int mend = (a.c.M - m0) < 32 ? (a.c.M - m0) : 32;
+                        if (scan_walk<32>(a.c, row + m0, m0, mend, vv, I, st)) break;
+                    }
+                    scan_finish(a.c, st);
+                    finish_neuron(a.c, st, p, ct * BN + (r * qpp + wip) * 32 + lane, a.C_out, a.rowsum, a.t_out,
+                                  a.q_out, a.s_out, a.vdot_out, pacc);
+                }
+                sync_pos();
             }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
+        }
+        if (a.penalty) {
+#pragma unroll
+            for (int k2 = 0; k2 < 4; ++k2) {
+                const float sum = warp_sum(pacc[k2]);
+                if (lane == 0 && sum != 0.f) atomicAdd(&a.penalty[k2], sum);
+            }
         }
     } else {
         const int quarter = warp & 3, group = (warp - 2) >> 2;
@@ -1780,7 +1848,7 @@ static cudaError_t launch_dw_gen_bn(const uint2 *rec, const CUtensorMap &mD, Con
 template <int BN, bool ROWBOX, bool RES, bool FWD>
 static cudaError_t launch_tap_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
                                  cudaStream_t st) {
-    const int smem = pl.nst * pl.stage + pl.res_bytes + (FWD ? 0 : DS_EPI_BYTES) + 1024 + 256;
+    const int smem = pl.nst * pl.stage + pl.res_bytes + (FWD ? FWD_EPI_BYTES : DS_EPI_BYTES) + 1024 + 256;
     cudaError_t e = cudaFuncSetAttribute(k_conv_tap_gemm<BN, ROWBOX, RES, FWD>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -1871,7 +1939,7 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     auto plan = [&](bool rowbox) { return tap_plan(g.k, ppt, c.Mp, BN, resident, res, rowbox, DS_EPI_BYTES, ncb); };
     const bool row_ok = g.s == 1 && g.W % ppt == 0 && ppt + g.k - 1 <= 256;
     DsPlan pl = plan(row_ok);
-    bool rowbox = row_ok && pl.nst >= 3;
+    bool rowbox = row_ok && pl.nst >= 2;
     if (!rowbox) pl = plan(false);
     if (pl.nst < 2) return cudaErrorInvalidConfiguration;
     // stride classes (one for stride 1); a stride whose s x s classes do not
@@ -1925,14 +1993,21 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
 #undef DSTD_DS
 }
 
-// forward w^ [ni Ho Wo][C_out][Mp] of ni images from the binned input
-// S [ni H W][Mp][C_in] and the filters Wf [C_out][k k C_in]
+// forward of ni images from the binned input S [ni H W][Mp][C_in] and the
+// filters Wf [C_out][k k C_in], with the scan/solve/select in the epilogue:
+// spike outputs [ni Ho Wo][C_out], penalty sums added into penalty[4]
 cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                                const __nv_bfloat16 *Wf, float *what, cudaStream_t st) {
+                                const __nv_bfloat16 *Wf, const float *rowsum, float *t_out, int *q, float *s,
+                                float *vdot, float *penalty, cudaStream_t st) {
     ConvGemmArgs a = base_args(g, ni, c);
     a.C_out = C_out;
     a.P_rows = ni * g.Ho * g.Wo;
-    a.what = what;
+    a.t_out = t_out;
+    a.q_out = q;
+    a.s_out = s;
+    a.vdot_out = vdot;
+    a.rowsum = rowsum;
+    a.penalty = penalty;
     const int BN = pick_bn(C_out);
     const int ppt = 128 / c.Mp;
     const int ncb = g.C / 64;
@@ -1942,21 +2017,21 @@ cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifC
     const long long res = (long long)g.k * g.k * ncb * BN * 128;
     const bool resident = a.n_col == 1 && res <= 80 * 1024;
     const bool row_ok = g.s == 1 && g.Wo % ppt == 0 && ppt + g.k - 1 <= 256;
-    DsPlan pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, row_ok, 0, ncb);
-    const bool rowbox = row_ok && pl.nst >= 3;
-    if (!rowbox) pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, false, 0, ncb);
+    DsPlan pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, row_ok, FWD_EPI_BYTES, ncb);
+    const bool rowbox = row_ok && pl.nst >= 2;
+    if (!rowbox) pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, false, FWD_EPI_BYTES, ncb);
     if (pl.nst < 2) return cudaErrorInvalidConfiguration;
     // every tap of every output position, in position order
     pl.ncls = 1;
     pl.ps = pl.ts = 1;
-    DsClass &q = pl.cls[0];
-    q.py = q.px = 0;
-    q.Hc = g.Ho;
-    q.Wc = g.Wo;
-    q.count = a.P_rows;
-    q.tile0 = 0;
-    q.kh0 = q.kw0 = 0;
-    q.nkh = q.nkw = g.k;
+    DsClass &cl = pl.cls[0];
+    cl.py = cl.px = 0;
+    cl.Hc = g.Ho;
+    cl.Wc = g.Wo;
+    cl.count = a.P_rows;
+    cl.tile0 = 0;
+    cl.kh0 = cl.kw0 = 0;
+    cl.nkh = cl.nkw = g.k;
     CUtensorMap mA, mB;
     if (!map_act(&mA, S, ni, g.H, g.W, c.Mp, g.C, rowbox ? ppt + g.k - 1 : 1) ||
         !map_mat(&mB, Wf, C_out, g.k * g.k * g.C, BN))

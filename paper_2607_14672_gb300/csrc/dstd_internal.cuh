@@ -250,6 +250,136 @@ __device__ __forceinline__ void penalty_T(const LifConst &c, float t, float &val
 }
 
 // ---------------------------------------------------------------------------
+// The walk over the bins of one neuron from w^ held in shared memory, shared
+// by the scan kernel and the conv forward's fused epilogue, and the per-neuron
+// outputs with the penalty sums.
+// ---------------------------------------------------------------------------
+// Exact test of an interval whose v^ has an interior maximum (dv^/ds > 0 at
+// s = 0, < 0 at s = dt) and whose cheap bound reached v_th: the bracket end
+// for the root, or -1. Before the exact maximum (a log and two exponentials)
+// it tries a tighter bound: on [0, s*] v^ >= v0 and e^{-aI s} <= 1 give
+//   v^(s*) <= v0 + max_s [ -av v0 s + I0 (1 - e^{-aI s}) / aI ],
+// whose maximiser has e^{-aI s} = av v0 / I0. Out of line: it runs rarely.
+static __device__ __noinline__ float interior_test(float av, float aI, float lam, int lam_zero, float rI, float dt,
+                                                   float vth, float v0, float I0, float ve) {
+    if (!(av > 0.0f && aI > 0.0f && I0 > 0.0f)) return -1.0f;
+    float g;
+    const float inv_aI = 1.0f / aI;
+    if (v0 > 0.0f) {
+        const float sm = logf(I0 / (av * v0)) * inv_aI;
+        g = sm < dt ? -av * v0 * sm + (I0 - av * v0) * inv_aI : -av * v0 * dt + I0 * (1.0f - rI) * inv_aI;
+    } else {
+        g = -av * v0 * dt + I0 * (1.0f - rI) * inv_aI;
+    }
+    // margin: rounding of the bound's own terms
+    if (v0 + g + 1e-6f * (fabsf(v0) + fabsf(g)) < vth) return -1.0f;
+    return interval_test(av, aI, lam, lam_zero, rI, dt, vth, v0, I0, ve);
+}
+
+// One interval of the walk, with explicit fma so that the fast pass and the
+// exact pass round alike: the end state and the two flags.
+struct BinStep {
+    float ve, In;
+    bool endp, peak;
+};
+__device__ __forceinline__ BinStep bin_step(const LifConst &c, float v, float I0) {
+    BinStep r;
+    r.ve = fmaf(c.KD, I0, c.rv * v);
+    r.In = c.rI * I0;
+    r.endp = r.ve >= c.vth;
+    r.peak = (fmaf(-c.av, v, I0) > 0.0f) & (fmaf(-c.av, r.ve, r.In) < 0.0f) &
+             (fmaf(fmaxf(I0, 0.0f), c.Kmax, fmaxf(v, 0.0f)) >= c.vth);
+    return r;
+}
+
+// The two passes over SUB bins m0 .. m0+SUB-1 of one neuron, whose w^
+// values sit in row[0 .. SUB) (shared memory, 16-byte aligned, zero past
+// mend), starting from the state (v, I) at T_m0. On a spike, fills st (bin,
+// state at its start, bracket end) and returns true; otherwise leaves (v, I)
+// at the end of the block.
+template <int SUB>
+__device__ __forceinline__ bool scan_walk(const LifConst &c, const float *row, int m0, int mend, float &v, float &I,
+                                          ScanState &st) {
+    static_assert(SUB % 8 == 0 && SUB <= 32, "blocks of 8, 16 or 32 bins");
+    constexpr int NCK = SUB / 8;  // kept states per block
+    float kv[NCK], kI[NCK];
+    uint32_t mask = 0u;
+#pragma unroll
+    for (int g = 0; g < SUB; g += 4) {
+        if ((g & 7) == 0) {
+            kv[g >> 3] = v;
+            kI[g >> 3] = I;
+        }
+        const float4 x = *reinterpret_cast<const float4 *>(row + g);
+        const float xs[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const BinStep r = bin_step(c, v, I + xs[u]);
+            if (r.endp | r.peak) mask |= 1u << (g + u);
+            v = r.ve;
+            I = r.In;
+        }
+    }
+    if (mend < 32) mask &= (1u << mend) - 1u;
+    while (mask) {
+        const int m = __ffs(mask) - 1;
+        mask &= mask - 1u;
+        const int gk = m >> 3;
+        float vw = kv[0], Iw = kI[0];
+#pragma unroll
+        for (int k = 1; k < NCK; ++k) {
+            vw = (gk == k) ? kv[k] : vw;
+            Iw = (gk == k) ? kI[k] : Iw;
+        }
+        for (int k = gk * 8; k < m; ++k) {
+            const BinStep r = bin_step(c, vw, Iw + row[k]);
+            vw = r.ve;
+            Iw = r.In;
+        }
+        const float I0 = Iw + row[m];
+        const BinStep r = bin_step(c, vw, I0);
+        float hi = -1.0f;
+        if (r.endp) hi = c.dt;
+        else if (r.peak) hi = interior_test(c.av, c.aI, c.lam, c.lam_zero, c.rI, c.dt, c.vth, vw, I0, r.ve);
+        if (hi >= 0.0f) {
+            st.q = m0 + m;
+            st.v0 = vw;
+            st.I0 = I0;
+            st.hi = hi;
+            return true;
+        }
+    }
+    return false;
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__device__ __forceinline__ void finish_neuron(const LifConst &c, const ScanState &st, int b, int i, int N,
+                                              const float *rowsum, float *t_out, int *q, float *s, float *vdot,
+                                              float acc[4]) {
+    long long o = (long long)b * N + i;
+    bool fired = st.q < c.M;
+    float t = fired ? c.T0 + (float)st.q * c.dt + st.s : INFINITY;
+    t_out[o] = t;
+    if (q) q[o] = st.q;
+    if (s) s[o] = st.s;
+    if (vdot) vdot[o] = st.vdot;
+    if (fired) {
+        float pv, pg;
+        penalty_T(c, t, pv, pg);
+        acc[0] += pv;
+        acc[3] += 1.0f;
+    } else {
+        if (rowsum) acc[1] += -c.g_q * c.norm * rowsum[i];
+        acc[2] += 1.0f;
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Device status word (bounded waits that expire set it); it lives in the
 // tensor-core translation unit, the only device code that waits.
 // ---------------------------------------------------------------------------
@@ -326,12 +456,14 @@ cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifCo
                                const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
                                cudaStream_t st);
 // the binned input written out, S [P][Mp][C] bf16, from the spike times, and the
-// forward contraction that reads it through tap-shifted TMA boxes (w^ as for
-// launch_conv_fwd_gen)
+// forward contraction that reads it through tap-shifted TMA boxes, with the
+// scan/solve/select of each neuron in its epilogue (outputs as from
+// launch_scan_solve: spike times, q, s, dv^/dt, penalty sums)
 bool conv_bin_S_supported(int C);  // channel counts the S writer takes
 cudaError_t launch_bin_S(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st);
 cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                                const __nv_bfloat16 *Wf, float *what, cudaStream_t st);
+                                const __nv_bfloat16 *Wf, const float *rowsum, float *t_out, int *q, float *s,
+                                float *vdot, float *penalty, cudaStream_t st);
 // dW from S and dw^ (added into g_W as for launch_conv_dw_gen)
 cudaError_t launch_conv_dw_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
                                const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
