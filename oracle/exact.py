@@ -5,7 +5,9 @@ Test infrastructure (see the package header). Float64 throughout.
 Parity status: pinned. Against brute-force RK4 integration of the LIF ODE on
 tiny layers (``lif.ode_first_spike``), against the non-leaky closed form
 Eq. spike_no_leak, and the table closed forms against the bracketed numeric
-solver.
+solver. ``exact_backward`` against central finite differences of
+``exact_forward`` (weights and input times), and its zero pattern (silent
+outputs, inputs after the spike).
 
 Steps (Alg. 1, one layer, one sample):
   1. drop silent inputs and sort the rest, t~_1 <= ... <= t~_K;
@@ -67,6 +69,37 @@ def exact_forward(t_in, W, tau_v, tau_I, v_th, t_end=INF, solver="table", chunk=
             tsel = np.take_along_axis(cand, first[:, None], -1)[:, 0]
             out[b, i0:i0 + chunk] = np.where(anyv, tsel, INF)
     return out
+
+
+def exact_backward(t_in, W, t_out, g_out, tau_v, tau_I):
+    """Gradients through the exact spike times (the implicit function theorem
+    on v_i(t_i) = v_th, Eq. Vmem_analytical at the root of Eq. timing_exact).
+
+    Neuron i fires at t_i with v_i(t_i) = sum_j w_ij K(t_i - t_j) = v_th over
+    its causal inputs (t_j < t_i: the intervals of Alg. 1 up to the one that
+    holds t_i). With the slope at the crossing V'_i = sum_j w_ij K'(t_i - t_j):
+        dt_i/dw_ij = -K(t_i - t_j) / V'_i,    dt_i/dt_j = w_ij K'(t_i - t_j) / V'_i.
+    Silent outputs and inputs at or after t_i contribute nothing.
+
+    t_in [B, N_in], W [N_out, N_in], t_out [B, N_out], g_out = dC/dt_out [B, N_out].
+    Returns (g_W [N_out, N_in], g_t_in [B, N_in]).
+    """
+    t_in = np.atleast_2d(np.asarray(t_in, float))
+    W = np.atleast_2d(np.asarray(W, float))
+    t_out = np.atleast_2d(np.asarray(t_out, float))
+    g_out = np.atleast_2d(np.asarray(g_out, float))
+    fired = np.isfinite(t_out)
+    x = np.where(fired[:, :, None], t_out[:, :, None], 0.0) - np.where(np.isfinite(t_in), t_in, INF)[:, None, :]
+    causal = fired[:, :, None] & np.isfinite(t_in)[:, None, :] & (x > 0)
+    xs = np.where(causal, x, 0.0)
+    Kx = np.where(causal, lif.K(xs, tau_v, tau_I), 0.0)          # [B, N_out, N_in]
+    dK = np.where(causal, lif.K_prime(xs, tau_v, tau_I), 0.0)
+    Vp = np.einsum("bij,ij->bi", dK, W)                            # slope at each spike
+    with np.errstate(divide="ignore", invalid="ignore"):
+        dt_dv = np.where(fired, g_out / Vp, 0.0)                   # dC/dt_i / V'_i
+    g_W = -np.einsum("bi,bij->ij", dt_dv, Kx)
+    g_t_in = np.einsum("bi,ij,bij->bj", dt_dv, W, dK)
+    return g_W, g_t_in
 
 
 def candidate_bytes(B, n_in, n_out, bytes_per_candidate=16):

@@ -90,3 +90,70 @@ def test_window_truncation_and_silence():
 
 def test_candidate_footprint():
     assert exact.candidate_bytes(128, 16384, 16384) == 128 * 16384 * 16384 * 16
+
+
+# ---------------------------------------------------------------------------
+# exact_backward (implicit function theorem at the spike) against central
+# finite differences of exact_forward, whose roots come from the closed forms
+# and the bracketed solver, not from the gradient formula.
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("tau_v,tau_I", [(0.5, 0.25), (INF, INF), (1.0, 1.0), (INF, 0.5), (1.0, 0.5), (0.8, INF)])
+def test_exact_backward_matches_finite_differences(tau_v, tau_I):
+    rng = np.random.default_rng(11)
+    B, N_in, N_out = 2, 6, 5
+    s = np.linspace(1e-3, 5.0, 5001)
+    kmax = lif.K(s, tau_v, tau_I).max()
+    t_in = rng.uniform(0.0, 1.0, (B, N_in))
+    t_in[0, 5] = INF
+    W = rng.normal(3.0 / (N_in * kmax), 0.8 / (N_in * kmax), (N_out, N_in))
+    fwd = lambda ti, w: exact.exact_forward(ti, w, tau_v, tau_I, 1.0)
+    t = fwd(t_in, W)
+    assert np.isfinite(t).sum() >= 6
+    g = rng.normal(0.0, 1.0, t.shape)
+    gW, gT = exact.exact_backward(t_in, W, t, g, tau_v, tau_I)
+    cost = lambda tt: float(np.sum(np.where(np.isfinite(tt), g * np.where(np.isfinite(tt), tt, 0.0), 0.0)))
+    h = 1e-6
+    checked = 0
+    for i in range(N_out):
+        for j in range(N_in):
+            Wp, Wm = W.copy(), W.copy()
+            Wp[i, j] += h
+            Wm[i, j] -= h
+            tp, tm = fwd(t_in, Wp), fwd(t_in, Wm)
+            if not (np.array_equal(np.isfinite(tp), np.isfinite(t)) and np.array_equal(np.isfinite(tm), np.isfinite(t))):
+                continue
+            fd = (cost(tp) - cost(tm)) / (2 * h)
+            assert abs(fd - gW[i, j]) <= 1e-6 * (1.0 + abs(fd)), (i, j, fd, gW[i, j])
+            checked += 1
+    for b in range(B):
+        for j in range(N_in):
+            if not np.isfinite(t_in[b, j]):
+                assert gT[b, j] == 0.0
+                continue
+            tp_in, tm_in = t_in.copy(), t_in.copy()
+            tp_in[b, j] += h
+            tm_in[b, j] -= h
+            tp, tm = fwd(tp_in, W), fwd(tm_in, W)
+            if not (np.array_equal(np.isfinite(tp), np.isfinite(t)) and np.array_equal(np.isfinite(tm), np.isfinite(t))):
+                continue
+            fd = (cost(tp) - cost(tm)) / (2 * h)
+            assert abs(fd - gT[b, j]) <= 1e-6 * (1.0 + abs(fd)), (b, j, fd, gT[b, j])
+            checked += 1
+    assert checked >= 30
+
+
+def test_exact_backward_zero_pattern():
+    """Silent outputs carry no gradient; an input after a neuron's spike has
+    no effect on it (dt_i/dw_ij = 0), and a silent input none at all."""
+    t_in = np.array([[0.1, 0.2, 5.0, INF]])
+    W = np.array([[2.0, 2.0, 3.0, 1.0], [-1.0, -1.0, -1.0, -1.0]])
+    t = exact.exact_forward(t_in, W, INF, INF, 1.0)
+    assert np.isfinite(t[0, 0]) and t[0, 0] < 5.0 and not np.isfinite(t[0, 1])
+    gW, gT = exact.exact_backward(t_in, W, t, np.ones_like(t), INF, INF)
+    assert np.all(gW[1] == 0.0) and gW[0, 2] == 0.0 and gW[0, 3] == 0.0
+    assert gT[0, 2] == 0.0 and gT[0, 3] == 0.0
+    # non-leaky closed form: v = sum_j w_j (t - t_j) = 1 -> t = (1 + sum w t_j) / sum w
+    sw = 4.0
+    assert abs(t[0, 0] - (1.0 + 2.0 * 0.1 + 2.0 * 0.2) / sw) < 1e-12
+    assert abs(gW[0, 0] - (-(t[0, 0] - 0.1) / sw)) < 1e-12
+    assert abs(gT[0, 0] - 2.0 / sw) < 1e-12
