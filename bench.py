@@ -794,6 +794,12 @@ def conv_rooflines(n, per_kind, pk, pk_src, sustained=False):
     return out
 
 
+def exact_candidate_bytes_layer(B, n_in, n_out):
+    """The exact method's candidates of one layer kept for a backward: 16 B
+    per (sample, neuron, input) (Tab. computational_complexity)."""
+    return int(B) * int(n_in) * int(n_out) * 16
+
+
 def exact_candidate_bytes(n):
     """The exact method's retained candidates for a backward (16 B per sample
     x neuron x input, Tab. computational_complexity), over the network."""
@@ -1208,10 +1214,13 @@ def run_multispike(args, local):
 
 
 def run_exact_compare(args, local):
-    """Exact forward (sort + interval sweep, Alg. 1) against the DSTD forward
-    (binning, contraction, scan/solve) of the same layers on one GPU: device
-    time per forward (CUDA events, L2 flushed before each), and how far the
-    two methods' spike times are apart (median over neurons firing in both)."""
+    """Exact method (sort + interval sweep, Alg. 1; backward by the implicit
+    function theorem at each exact spike, K recomputed per pair) against DSTD
+    (binning, contraction, scan/solve; backward through dw^) on the same
+    layers on one GPU: device time per forward and per forward + backward
+    (CUDA events, L2 flushed before each), device bytes each method holds for
+    its backward, and how far the two methods' spike times are apart (median
+    over neurons firing in both)."""
     import numpy as np
     import torch
 
@@ -1244,8 +1253,20 @@ def run_exact_compare(args, local):
         t_e = torch.empty(B, N_out, device=dev)
         saved = torch.empty(dstd.dense_saved_bytes(B, N_out), dtype=torch.uint8, device=dev)
         pen = torch.empty(4, device=dev)
+        g_up = torch.randn(B, N_out, device=dev) * 0.1
+        g_in, g_W = torch.empty(B, N_in, device=dev), torch.empty(N_out, N_in, device=dev)
+
+        def dstd_train():
+            dstd.dense_fwd(t, W, p, "x3", t_d, saved, pen, ws, stream)
+            dstd.dense_bwd(t, W, t_d, saved, g_up, p, "x3", g_in, g_W, ws, stream)
+
+        def exact_train():
+            dstd.exact_fwd(t, W, p, t_e, wse, stream)
+            dstd.exact_bwd(t, W, t_e, g_up, p, g_in, g_W, wse, stream)
+
         runs = {"dstd": lambda: dstd.dense_fwd(t, W, p, "x3", t_d, saved, pen, ws, stream),
-                "exact": lambda: dstd.exact_fwd(t, W, p, t_e, wse, stream)}
+                "exact": lambda: dstd.exact_fwd(t, W, p, t_e, wse, stream),
+                "dstd_train": dstd_train, "exact_train": exact_train}
         ms = {}
         with torch.cuda.stream(stream):
             for k, fn in runs.items():
@@ -1263,13 +1284,19 @@ def run_exact_compare(args, local):
         both = np.isfinite(td) & np.isfinite(te)
         out.append({"layer": name, "B": B, "N_in": N_in, "N_out": N_out, "M": L["M"],
                     "dstd_fwd_ms": ms["dstd"], "exact_fwd_ms": ms["exact"], "exact_over_dstd": ms["exact"] / ms["dstd"],
+                    "dstd_train_ms": ms["dstd_train"], "exact_train_ms": ms["exact_train"],
+                    "exact_over_dstd_train": ms["exact_train"] / ms["dstd_train"],
+                    "dstd_bytes": int(ws.numel() + saved.numel()), "exact_bytes": int(wse.numel()),
+                    "exact_candidate_bytes": exact_candidate_bytes_layer(B, N_in, N_out),
                     "fire_dstd": float(np.isfinite(td).mean()), "fire_exact": float(np.isfinite(te).mean()),
                     "median_abs_dt_fired_both": float(np.median(np.abs(td[both] - te[both]))) if both.any() else None})
     status = dstd.device_status(clear=True)
-    print(json.dumps({"metric": "exact (event-driven) forward time / DSTD forward time, one GB300", "unit": "ratio",
-                      "higher_is_better": True, "cases": out, "reps": reps, "device_status": status,
-                      "note": "forward only (the GPU exact method has no backward); DSTD in the x3 mode; median of "
-                              "the per-rep CUDA-event times, L2 flushed before each"}), flush=True)
+    print(json.dumps({"metric": "exact (event-driven) time / DSTD time, forward and forward + backward, one GB300",
+                      "unit": "ratio", "higher_is_better": True, "cases": out, "reps": reps, "device_status": status,
+                      "note": "DSTD in the x3 mode; median of the per-rep CUDA-event times, L2 flushed before each; "
+                              "the GPU exact backward recomputes K per (sample, neuron, input) pair instead of "
+                              "keeping the candidates, so its device bytes are the workspace only; "
+                              "exact_candidate_bytes is what keeping them takes (16 B each)"}), flush=True)
     return 0 if status == 0 else 1
 
 

@@ -315,7 +315,8 @@ int dstd_adamw_multi(int count, float *const *w, const float *const *g, float *c
  * interval by interval and the first interval that reaches p->v_th holds
  * the spike. Spike times are exact up to fp32 (no grid); a neuron that does
  * not fire before p->t_end gets +inf. Only tau_m, tau_s, v_th and t_end of p
- * are used (t_first, M only for the root's tolerance). No gradient.
+ * are used (t_first, M only for the root's tolerance); dstd_exact_bwd
+ * gives its gradients.
  *  t_in [B, N_in] (+inf = silent), W [N_out, N_in] fp32, t_out [B, N_out] out;
  *  workspace of dstd_exact_workspace_bytes (16-byte aligned).
  * N_in up to 8192 (DSTD_E_UNSUPPORTED beyond). */
@@ -323,6 +324,20 @@ size_t dstd_exact_workspace_bytes(int B, int N_in, int N_out);
 int dstd_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out,
                    const dstd_params *p, float *t_out, void *workspace, size_t ws_bytes,
                    dstd_stream_t stream);
+/* Backward of the exact layer: the implicit function theorem at each exact
+ * spike time (Eq. timing_exact). A neuron i that fires at t_i (from
+ * dstd_exact_fwd) has sum_j w_ij K(t_i - t_j) = v_th over its inputs with
+ * t_j < t_i; with the slope V'_i = sum_j w_ij K'(t_i - t_j) there,
+ *   g_W[i, j]    = -sum_b g_t_out[b, i] K(t_bi - t_bj) / V'_bi,
+ *   g_t_in[b, j] =  sum_i g_t_out[b, i] w_ij K'(t_bi - t_bj) / V'_bi,
+ * over the pairs with t_bj < t_bi; silent neurons and later inputs give 0.
+ * K and K' are recomputed for every pair (nothing per candidate is stored):
+ * O(B N_out N_in) exponentials. No penalty terms: add their dT/dt to
+ * g_t_out. g_t_in may be NULL; g_W and g_t_in are overwritten. Same
+ * workspace as dstd_exact_fwd. */
+int dstd_exact_bwd(const float *t_in, const float *W, const float *t_out, const float *g_t_out,
+                   int B, int N_in, int N_out, const dstd_params *p, float *g_t_in, float *g_W,
+                   void *workspace, size_t ws_bytes, dstd_stream_t stream);
 
 /* How the forward contraction of a wide dense layer is scheduled: on single
  * CTAs (128 x 128 tiles) or on SM pairs (tcgen05 cta_group::2, 256 x 128

@@ -90,12 +90,12 @@ inline int cu(cudaError_t e) { return e == cudaSuccess ? DSTD_OK : DSTD_E_CUDA; 
 enum Kind {
     KK_PREP = 0, KK_BIN, KK_BIN_T, KK_GEMM_FWD, KK_SCAN, KK_DWHAT, KK_GEMM_DS, KK_GT, KK_GEMM_DW, KK_REDUCE,
     KK_LOSS, KK_ADAMW, KK_BIN_PUB, KK_WHAT_PUB, KK_SELFTEST, KK_NARROW_FWD, KK_NARROW_BWD, KK_EXACT_FWD, KK_SKIP,
-    KK_COUNT
+    KK_EXACT_BWD, KK_COUNT
 };
 const char *const kKindNames[KK_COUNT] = {
     "prep_weights", "binning", "binning_T", "gemm_fwd_scan", "scan_solve", "dwhat", "gemm_dS_gradt",
     "gradt_gather", "gemm_dW", "dw_reduce", "loss", "adamw", "binning_public", "what_public", "selftest", "narrow_fwd",
-    "narrow_bwd", "exact_fwd", "skip_channels"};
+    "narrow_bwd", "exact_fwd", "skip_channels", "exact_bwd"};
 
 struct Timing {
     std::mutex mu;
@@ -390,6 +390,7 @@ ExactWs exact_layout(void *base, int B, int N_in, int N_out) {
     w.t_start = bp.take<float>((size_t)B * N_in);
     w.iv = bp.take<float4>((size_t)B * N_in);
     w.count = bp.take<int>((size_t)B);
+    w.coef = bp.take<float>((size_t)B * N_out);
     w.bytes = bp.off;
     return w;
 }
@@ -1306,6 +1307,22 @@ int dstd_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out
     ExactWs ws = exact_layout(workspace, B, N_in, N_out);
     Timed tm(KK_EXACT_FWD, (cudaStream_t)stream);
     return cu(launch_exact_fwd(t_in, W, B, N_in, N_out, c, p->t_end, (float)kmax, ws, t_out, (cudaStream_t)stream));
+}
+
+int dstd_exact_bwd(const float *t_in, const float *W, const float *t_out, const float *g_t_out, int B, int N_in,
+                   int N_out, const dstd_params *p, float *g_t_in, float *g_W, void *workspace, size_t ws_bytes,
+                   dstd_stream_t stream) {
+    if (!t_in || !W || !t_out || !g_t_out || !g_W || !workspace) return DSTD_E_INVALID;
+    TRY(check_sizes(B, N_in, N_out));
+    TRY(check_params(p));
+    if (N_in > kExactMaxIn) return DSTD_E_UNSUPPORTED;
+    if (!aligned16(workspace)) return DSTD_E_INVALID;
+    if (ws_bytes < exact_layout(nullptr, B, N_in, N_out).bytes) return DSTD_E_WORKSPACE;
+    TRY(device_ok());
+    const LifConst c = make_const(*p, padded_M(p->M));
+    ExactWs ws = exact_layout(workspace, B, N_in, N_out);
+    Timed tm(KK_EXACT_BWD, (cudaStream_t)stream);
+    return cu(launch_exact_bwd(t_in, W, t_out, g_t_out, B, N_in, N_out, c, ws, g_t_in, g_W, (cudaStream_t)stream));
 }
 
 // ---------------------------------------------------------------------------

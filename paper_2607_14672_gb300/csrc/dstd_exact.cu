@@ -1,5 +1,6 @@
-// The exact (event-driven) TTFS forward on the GPU: Alg. 1 of the paper, the
-// method DSTD replaces, for an on-device comparison of the two.
+// The exact (event-driven) TTFS layer on the GPU: Alg. 1 of the paper, the
+// method DSTD replaces, forward and backward, for an on-device comparison of
+// the two.
 //
 // Per sample the finite input spike times before the window end are sorted,
 // t~_1 <= ... <= t~_K; on each interval [t~_k, t~_{k+1}) (the last closed at
@@ -145,6 +146,131 @@ cudaError_t launch_exact_fwd(const float *t_in, const float *W, int B, int N_in,
     dim3 grid((N_out + EXACT_WALK_THREADS - 1) / EXACT_WALK_THREADS, B);
     k_exact_walk<<<grid, EXACT_WALK_THREADS, smem_walk, st>>>(ws.Wt, N_in, N_out, c, kmax, ws.perm, ws.t_start,
                                                              ws.iv, ws.count, t_out);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Backward of the exact method: the implicit function theorem at each exact
+// spike time. Neuron i fires at t_i with sum_j w_ij K(t_i - t_j) = v_th over
+// its inputs before t_i; with the slope V'_i = sum_j w_ij K'(t_i - t_j),
+//   dC/dw_ij = -g_i K(t_i - t_j) / V'_i,   dC/dt_j += g_i w_ij K'(t_i - t_j) / V'_i.
+// K(x) = e^{-av x} phi(x) and K'(x) = e^{-aI x} - av K(x) are recomputed for
+// every (sample, neuron, input) pair: nothing per candidate is kept, at the
+// price of O(B N_out N_in) exponentials.
+//   k_exact_slope  one thread per (sample, neuron): V'_i and g_i / V'_i
+//   k_exact_gw     16 x 16 (neuron, input) tiles, samples staged in shared memory
+//   k_exact_gt     one thread per (sample, input), neurons staged in shared memory
+// ---------------------------------------------------------------------------
+constexpr int EXACT_BWD_THREADS = 256, EXACT_BWD_CHUNK = 32;
+
+__device__ __forceinline__ float exact_K(const LifConst &c, float x) { return __expf(-c.av * x) * phi_f(c, x); }
+__device__ __forceinline__ float exact_dK(const LifConst &c, float x) {
+    return __expf(-c.aI * x) - c.av * exact_K(c, x);
+}
+
+__global__ void __launch_bounds__(EXACT_BWD_THREADS) k_exact_slope(const float *__restrict__ t_in,
+                                                                   const float *__restrict__ Wt,
+                                                                   const float *__restrict__ t_out,
+                                                                   const float *__restrict__ g_out, int N_in,
+                                                                   int N_out, LifConst c, float *__restrict__ coef) {
+    extern __shared__ float xs[];  // the sample's input times
+    const int b = blockIdx.y;
+    for (int j = threadIdx.x; j < N_in; j += EXACT_BWD_THREADS) xs[j] = t_in[(long long)b * N_in + j];
+    __syncthreads();
+    const int i = blockIdx.x * EXACT_BWD_THREADS + threadIdx.x;
+    if (i >= N_out) return;
+    const float ti = t_out[(long long)b * N_out + i];
+    float cf = 0.f;
+    if (isfinite(ti)) {
+        float vp = 0.f;
+        for (int j = 0; j < N_in; ++j) {
+            const float x = ti - xs[j];  // +inf inputs give -inf
+            if (x > 0.f) vp = fmaf(Wt[(long long)j * N_out + i], exact_dK(c, x), vp);
+        }
+        cf = g_out[(long long)b * N_out + i] / vp;
+    }
+    coef[(long long)b * N_out + i] = cf;
+}
+
+__global__ void __launch_bounds__(EXACT_BWD_THREADS) k_exact_gw(const float *__restrict__ t_in,
+                                                                const float *__restrict__ t_out,
+                                                                const float *__restrict__ coef, int B, int N_in,
+                                                                int N_out, LifConst c, float *__restrict__ g_W) {
+    __shared__ float so[EXACT_BWD_CHUNK][16], sc[EXACT_BWD_CHUNK][16], si[EXACT_BWD_CHUNK][16];
+    const int tj = threadIdx.x & 15, ti = threadIdx.x >> 4;
+    const int j = blockIdx.x * 16 + tj, i = blockIdx.y * 16 + ti;
+    float acc = 0.f;
+    for (int b0 = 0; b0 < B; b0 += EXACT_BWD_CHUNK) {
+        for (int e = threadIdx.x; e < EXACT_BWD_CHUNK * 16; e += EXACT_BWD_THREADS) {
+            const int bb = e >> 4, u = e & 15, b = b0 + bb;
+            const int ii = blockIdx.y * 16 + u, jj = blockIdx.x * 16 + u;
+            const bool okb = b < B;
+            so[bb][u] = (okb && ii < N_out) ? t_out[(long long)b * N_out + ii] : INFINITY;
+            sc[bb][u] = (okb && ii < N_out) ? coef[(long long)b * N_out + ii] : 0.f;
+            si[bb][u] = (okb && jj < N_in) ? t_in[(long long)b * N_in + jj] : INFINITY;
+        }
+        __syncthreads();
+        const int nb = B - b0 < EXACT_BWD_CHUNK ? B - b0 : EXACT_BWD_CHUNK;
+        for (int bb = 0; bb < nb; ++bb) {
+            const float cf = sc[bb][ti];
+            const float x = so[bb][ti] - si[bb][tj];
+            if (cf != 0.f && x > 0.f) acc = fmaf(cf, exact_K(c, x), acc);
+        }
+        __syncthreads();
+    }
+    if (i < N_out && j < N_in) g_W[(long long)i * N_in + j] = -acc;
+}
+
+__global__ void __launch_bounds__(EXACT_BWD_THREADS) k_exact_gt(const float *__restrict__ t_in,
+                                                                const float *__restrict__ W,
+                                                                const float *__restrict__ t_out,
+                                                                const float *__restrict__ coef, int N_in, int N_out,
+                                                                LifConst c, float *__restrict__ g_t_in) {
+    __shared__ float so[EXACT_BWD_THREADS], sc[EXACT_BWD_THREADS];
+    const int b = blockIdx.y;
+    const int j = blockIdx.x * EXACT_BWD_THREADS + threadIdx.x;
+    const float tj = j < N_in ? t_in[(long long)b * N_in + j] : INFINITY;
+    float acc = 0.f;
+    for (int i0 = 0; i0 < N_out; i0 += EXACT_BWD_THREADS) {
+        const int ii = i0 + threadIdx.x;
+        so[threadIdx.x] = ii < N_out ? t_out[(long long)b * N_out + ii] : INFINITY;
+        sc[threadIdx.x] = ii < N_out ? coef[(long long)b * N_out + ii] : 0.f;
+        __syncthreads();
+        const int ni = N_out - i0 < EXACT_BWD_THREADS ? N_out - i0 : EXACT_BWD_THREADS;
+        if (j < N_in && isfinite(tj)) {
+            for (int u = 0; u < ni; ++u) {
+                const float cf = sc[u];
+                const float x = so[u] - tj;
+                if (cf != 0.f && x > 0.f) acc = fmaf(cf * W[(long long)(i0 + u) * N_in + j], exact_dK(c, x), acc);
+            }
+        }
+        __syncthreads();
+    }
+    if (j < N_in) g_t_in[(long long)b * N_in + j] = acc;
+}
+
+cudaError_t launch_exact_bwd(const float *t_in, const float *W, const float *t_out, const float *g_out, int B,
+                             int N_in, int N_out, const LifConst &c, const ExactWs &ws, float *g_t_in, float *g_W,
+                             cudaStream_t st) {
+    if (N_in < 1 || N_in > kExactMaxIn) return cudaErrorInvalidValue;
+    cudaError_t e = launch_prep_weights(W, N_out, N_in, OpKind::F32, nullptr, nullptr, 0, nullptr, nullptr, 0, ws.Wt,
+                                        N_out, nullptr, st);
+    if (e != cudaSuccess) return e;
+    const size_t smem = (size_t)N_in * sizeof(float);
+    if (smem > 48 * 1024) {
+        e = cudaFuncSetAttribute(k_exact_slope, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    k_exact_slope<<<dim3((N_out + EXACT_BWD_THREADS - 1) / EXACT_BWD_THREADS, B), EXACT_BWD_THREADS, smem, st>>>(
+        t_in, ws.Wt, t_out, g_out, N_in, N_out, c, ws.coef);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_exact_gw<<<dim3((N_in + 15) / 16, (N_out + 15) / 16), EXACT_BWD_THREADS, 0, st>>>(t_in, t_out, ws.coef, B, N_in,
+                                                                                      N_out, c, g_W);
+    e = cudaGetLastError();
+    if (e != cudaSuccess || !g_t_in) return e;
+    k_exact_gt<<<dim3((N_in + EXACT_BWD_THREADS - 1) / EXACT_BWD_THREADS, B), EXACT_BWD_THREADS, 0, st>>>(
+        t_in, W, t_out, ws.coef, N_in, N_out, c, g_t_in);
     return cudaGetLastError();
 }
 

@@ -514,10 +514,16 @@ struct ExactWs {
     float *t_start = nullptr;  // [B][N_in]: its start
     float4 *iv = nullptr;      // [B][N_in]: e^{-av L}, e^{-aI L}, K(L), L
     int *count = nullptr;      // [B]: intervals (finite inputs before the window end)
+    float *coef = nullptr;     // [B][N_out]: dC/dt_i / V'_i (backward)
     size_t bytes = 0;
 };
 cudaError_t launch_exact_fwd(const float *t_in, const float *W, int B, int N_in, int N_out, const LifConst &c,
                              float t_end, float kmax, const ExactWs &ws, float *t_out, cudaStream_t st);
+// the exact method's backward: g_W [N_out][N_in] (overwritten) and, when
+// g_t_in is not null, g_t_in [B][N_in] (overwritten) from g_out [B][N_out]
+cudaError_t launch_exact_bwd(const float *t_in, const float *W, const float *t_out, const float *g_out, int B,
+                             int N_in, int N_out, const LifConst &c, const ExactWs &ws, float *g_t_in, float *g_W,
+                             cudaStream_t st);
 
 // Layers with at most kNarrowMaxOut outputs run forward and backward on CUDA
 // cores in fp32 (sparse over the two grid points of each input spike).

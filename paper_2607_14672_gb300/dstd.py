@@ -23,7 +23,7 @@ EXPORTS = ("dstd_dense_saved_bytes", "dstd_dense_workspace_bytes", "dstd_binning
            "dstd_adamw", "dstd_adamw_multi", "dstd_device_status", "dstd_error_string", "dstd_version", "dstd_timing_enable",
            "dstd_timing_read", "dstd_timing_collect", "dstd_set_pair_policy", "dstd_conv_set_chunk_images", "dstd_conv_set_operand_policy", "dstd_kernel_kind_count", "dstd_kernel_kind_name", "dstd_selftest_wait_timeout",
            "dstd_dense_fwd_noalloc", "dstd_conv_workspace_bytes", "dstd_conv_fwd", "dstd_conv_bwd",
-           "dstd_exact_workspace_bytes", "dstd_exact_fwd", "dstd_concat_channels", "dstd_split_channels",
+           "dstd_exact_workspace_bytes", "dstd_exact_fwd", "dstd_exact_bwd", "dstd_concat_channels", "dstd_split_channels",
            "dstd_ms_saved_bytes", "dstd_ms_workspace_bytes", "dstd_dense_fwd_ms", "dstd_dense_bwd_ms")
 
 
@@ -93,6 +93,7 @@ def load(path=None):
         "dstd_conv_set_operand_policy": (_I, [_I]),
         "dstd_exact_workspace_bytes": (_SZ, [_I, _I, _I]),
         "dstd_exact_fwd": (_I, [_P, _P, _I, _I, _I, _PP, _P, _P, _SZ, _P]),
+        "dstd_exact_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _PP, _P, _P, _P, _SZ, _P]),
         "dstd_kernel_kind_count": (_I, []),
         "dstd_kernel_kind_name": (ctypes.c_char_p, [_I]),
         "dstd_selftest_wait_timeout": (_I, [ctypes.c_uint32, _P]),
@@ -393,6 +394,23 @@ def exact_fwd(t_in, W, p, t_out, workspace, stream=None):
     _f32(t_out, "t_out", (B, N_out))
     _check(load().dstd_exact_fwd(_ptr(t_in), _ptr(W), B, N_in, N_out, ctypes.byref(p), _ptr(t_out), _ptr(workspace),
                                  workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_exact_fwd")
+
+
+def exact_bwd(t_in, W, t_out, g_t_out, p, g_t_in, g_W, workspace, stream=None):
+    """Backward of the exact layer (implicit function theorem at each exact
+    spike time): g_W [N_out, N_in] and g_t_in [B, N_in] (or None), overwritten."""
+    B, N_in = t_in.shape
+    N_out = W.shape[0]
+    _f32(t_in, "t_in")
+    _f32(W, "W", (N_out, N_in))
+    _f32(t_out, "t_out", (B, N_out))
+    _f32(g_t_out, "g_t_out", (B, N_out))
+    _f32(g_W, "g_W", (N_out, N_in))
+    if g_t_in is not None:
+        _f32(g_t_in, "g_t_in", (B, N_in))
+    _check(load().dstd_exact_bwd(_ptr(t_in), _ptr(W), _ptr(t_out), _ptr(g_t_out), B, N_in, N_out, ctypes.byref(p),
+                                 _ptr(g_t_in) if g_t_in is not None else None, _ptr(g_W), _ptr(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)), "dstd_exact_bwd")
 
 
 def set_pair_policy(policy):
