@@ -661,9 +661,14 @@ struct ConvImplWs {
 };
 
 int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
-    long long per_img = (long long)g.Ho * g.Wo * Mp * C_out * 4;
-    per_img += (conv_fwd_tma(g, C_out) || conv_dw_tma(g, C_out)) ? (long long)g.H * g.W * Mp * g.C * 2
-                                                                   : (long long)g.H * g.W * g.C * 8;
+    // per image, the larger of the forward's and the backward's scratch:
+    // S (bf16) or the 8-byte records, and w^ (fp32, generated forward only)
+    // or dw^ (bf16)
+    const long long outs = (long long)g.Ho * g.Wo * Mp * C_out;
+    const long long S = (long long)g.H * g.W * Mp * g.C * 2, rec = (long long)g.H * g.W * g.C * 8;
+    const long long fwd = conv_fwd_tma(g, C_out) ? S : rec + outs * 4;
+    const long long bwd = (conv_dw_tma(g, C_out) ? S : rec) + outs * 2;
+    const long long per_img = fwd > bwd ? fwd : bwd;
     long long imgs = (long long)(kConvImplBudget / (size_t)per_img);
     if (g_conv_chunk_images > 0 && imgs > g_conv_chunk_images) imgs = g_conv_chunk_images;
     if (imgs < 1) imgs = 1;
