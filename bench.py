@@ -65,6 +65,9 @@ def parse():
     ap.add_argument("--profile", action="store_true",
                     help="only warm-up and the timed replays (for an ncu launch list); no clocks, "
                          "per-kernel timing pass, e2e or CPU baseline")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="with --profile and a conv workload: this batch instead of the config's (a small case "
+                         "for single-kernel ncu captures)")
     return ap.parse_args()
 
 
@@ -865,7 +868,7 @@ def run_conv(args, rank, world, local):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    cfg = conv_workload(args.workload)
+    cfg = conv_workload(args.workload, args.batch if args.profile else None)
     B = cfg["batch"]
     n = net.ConvNet(cfg, device=dev, with_adamw=True)
     t0, lab = rank_batch(cfg, rank)
