@@ -643,13 +643,23 @@ static int g_conv_operand_policy = 0;
 // channel count: writing S costs one pass at HBM speed per chunk and
 // direction, and the TMA-fed tiles keep the tensor core fed, where the
 // generator warps (one stage per group when the filters stream) do not.
+// (A layer with fewer than 64 input channels is padded to 64 and always
+// reads S: the generated path takes multiples of 64 only.)
 static bool conv_fwd_tma(const ConvGeom &g, int C_out) {
     (void)C_out;
-    return conv_bin_S_supported(g.C) && g_conv_operand_policy != 1;
+    const int Cp = conv_padded_channels(g.C);
+    return conv_bin_S_supported(Cp) && (g_conv_operand_policy != 1 || Cp != g.C);
 }
 static bool conv_dw_tma(const ConvGeom &g, int C_out) {
     (void)C_out;
-    return conv_bin_S_supported(g.C) && g_conv_operand_policy != 1;
+    const int Cp = conv_padded_channels(g.C);
+    return conv_bin_S_supported(Cp) && (g_conv_operand_policy != 1 || Cp != g.C);
+}
+// the geometry the implicit kernels see: input channels padded to 64
+static ConvGeom conv_padded(const ConvGeom &g) {
+    ConvGeom gp = g;
+    gp.C = conv_padded_channels(g.C);
+    return gp;
 }
 
 struct ConvImplWs {
@@ -665,7 +675,8 @@ int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
     // S (bf16) or the 8-byte records, and w^ (fp32, generated forward only)
     // or dw^ (bf16)
     const long long outs = (long long)g.Ho * g.Wo * Mp * C_out;
-    const long long S = (long long)g.H * g.W * Mp * g.C * 2, rec = (long long)g.H * g.W * g.C * 8;
+    const int Cp = conv_padded_channels(g.C);
+    const long long S = (long long)g.H * g.W * Mp * Cp * 2, rec = (long long)g.H * g.W * g.C * 8;
     const long long fwd = conv_fwd_tma(g, C_out) ? S : rec + outs * 4;
     const long long bwd = (conv_dw_tma(g, C_out) ? S : rec) + outs * 2;
     const long long per_img = fwd > bwd ? fwd : bwd;
@@ -679,14 +690,15 @@ int conv_impl_images(const ConvGeom &g, int C_out, int Mp) {
 ConvImplWs conv_impl_layout(void *base, const ConvGeom &g, int C_out, int Mp, bool fwd) {
     ConvImplWs w;
     Bump b(base);
-    const long long K = (long long)g.k * g.k * g.C;
+    const int Cp = conv_padded_channels(g.C);
+    const long long K = (long long)g.k * g.k * Cp;
     w.imgs = conv_impl_images(g, C_out, Mp);
     w.rowsum = b.take<float>(C_out);
     w.count = b.take<float>(C_out);
     w.Wf = b.take<__nv_bfloat16>((size_t)C_out * K);
     w.Wt = b.take<__nv_bfloat16>((size_t)C_out * K);
     if (fwd ? conv_fwd_tma(g, C_out) : conv_dw_tma(g, C_out))
-        w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * g.C);
+        w.S = b.take<__nv_bfloat16>((size_t)w.imgs * g.H * g.W * Mp * Cp);
     else
         w.rec = b.take<uint2>((size_t)w.imgs * g.H * g.W * g.C);
     if (fwd && !w.S)
@@ -709,12 +721,20 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
     const LifConst c = make_const(*p, Mp);
     const long long npos = (long long)g.B * g.Ho * g.Wo;
     const int K = g.k * g.k * g.C;
+    const ConvGeom gp = conv_padded(g);
     Saved sv = saved_view(saved, npos, C_out);
     if (penalty) TRY(cu(cudaMemsetAsync(penalty, 0, 4 * sizeof(float), st)));
     {
         Timed tm(KK_PREP, st);
-        TRY(cu(launch_prep_weights(W, C_out, K, OpKind::BF16, ws.Wf, nullptr, K, nullptr, nullptr, 0, nullptr, 0,
-                                   ws.rowsum, st)));
+        if (gp.C == g.C) {
+            TRY(cu(launch_prep_weights(W, C_out, K, OpKind::BF16, ws.Wf, nullptr, K, nullptr, nullptr, 0, nullptr, 0,
+                                       ws.rowsum, st)));
+        } else {  // rows (o, tap) of C channels into rows of gp.C (zero padding), row sums per o
+            TRY(cu(launch_prep_weights(W, C_out * g.k * g.k, g.C, OpKind::BF16, ws.Wf, nullptr, gp.C, nullptr,
+                                       nullptr, 0, nullptr, 0, nullptr, st)));
+            TRY(cu(launch_prep_weights(W, C_out, K, OpKind::BF16, nullptr, nullptr, K, nullptr, nullptr, 0, nullptr, 0,
+                                       ws.rowsum, st)));
+        }
     }
     for (int img0 = 0; img0 < g.B; img0 += ws.imgs) {
         const int ni = (g.B - img0) < ws.imgs ? (g.B - img0) : ws.imgs;
@@ -724,13 +744,13 @@ int conv_fwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         {
             Timed tm(KK_BIN, st);
             if (ws.S)
-                TRY(cu(launch_bin_S(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+                TRY(cu(launch_bin_S(t_in + in_off, (long long)ni * g.H * g.W, gp.C, g.C, c, ws.S, st)));
             else
                 TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
         if (ws.S) {  // the scan runs in the contraction's epilogue
             Timed tm(KK_GEMM_FWD, st);
-            TRY(cu(launch_conv_fwd_tma(g, ni, C_out, c, ws.S, ws.Wf, ws.rowsum, t_out + out_off, sv.q + out_off,
+            TRY(cu(launch_conv_fwd_tma(gp, ni, C_out, c, ws.S, ws.Wf, ws.rowsum, t_out + out_off, sv.q + out_off,
                                        sv.s + out_off, sv.vdot + out_off, penalty, st)));
             continue;
         }
@@ -758,9 +778,10 @@ int conv_bwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
     const float qcoef = -p->gamma_q * p->penalty_norm;
     TRY(cu(cudaMemsetAsync(g_W, 0, sizeof(float) * (size_t)C_out * T * g.C, st)));
     TRY(cu(cudaMemsetAsync(ws.count, 0, sizeof(float) * (size_t)C_out, st)));
+    const ConvGeom gp = conv_padded(g);
     if (g_t_in) {
         Timed tm(KK_PREP, st);
-        TRY(cu(launch_filters_t(W, C_out, T, g.C, ws.Wt, st)));
+        TRY(cu(launch_filters_t(W, C_out, T, g.C, gp.C, ws.Wt, st)));
     }
     for (int img0 = 0; img0 < g.B; img0 += ws.imgs) {
         const int ni = (g.B - img0) < ws.imgs ? (g.B - img0) : ws.imgs;
@@ -775,18 +796,19 @@ int conv_bwd_implicit(const float *t_in, const float *W, const ConvGeom &g, int 
         }
         if (g_t_in) {
             Timed tm(KK_GEMM_DS, st);
-            TRY(cu(launch_conv_ds_gemm(g, ni, C_out, c, ws.dwh, ws.Wt, t_in + in_off, g_t_in + in_off, st)));
+            TRY(cu(launch_conv_ds_gemm(gp, ni, C_out, c, ws.dwh, ws.Wt, t_in + in_off, g_t_in + in_off, g.C, st)));
         }
         {
             Timed tm(KK_BIN_T, st);
             if (ws.S)
-                TRY(cu(launch_bin_S(t_in + in_off, (long long)ni * g.H * g.W, g.C, c, ws.S, st)));
+                TRY(cu(launch_bin_S(t_in + in_off, (long long)ni * g.H * g.W, gp.C, g.C, c, ws.S, st)));
             else
                 TRY(cu(launch_bin_rec(t_in + in_off, (long long)ni * g.H * g.W * g.C, c, ws.rec, st)));
         }
         Timed tm(KK_GEMM_DW, st);
         if (ws.S)
-            TRY(cu(launch_conv_dw_tma(g, ni, C_out, c, ws.S, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
+            TRY(cu(launch_conv_dw_tma(gp, ni, C_out, c, ws.S, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, g.C,
+                                      st)));
         else
             TRY(cu(launch_conv_dw_gen(g, ni, C_out, c, ws.rec, ws.dwh, last ? ws.count : nullptr, qcoef, g_W, st)));
     }

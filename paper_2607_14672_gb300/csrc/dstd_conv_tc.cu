@@ -227,15 +227,17 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
     }
 }
 
-// Filters [C_out][T][C_in] fp32 -> Wt [C_in][T][C_out] bf16 (T = k k taps).
-__global__ void k_filters_t(const float *__restrict__ W, int C_out, int T, int C_in, __nv_bfloat16 *__restrict__ Wt) {
-    const long long n = (long long)C_out * T * C_in;
+// Filters [C_out][T][C_in] fp32 -> Wt [C_pad][T][C_out] bf16 (T = k k taps;
+// rows C_in .. C_pad - 1 zero).
+__global__ void k_filters_t(const float *__restrict__ W, int C_out, int T, int C_in, int C_pad,
+                            __nv_bfloat16 *__restrict__ Wt) {
+    const long long n = (long long)C_out * T * C_pad;
     for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
          idx += (long long)gridDim.x * blockDim.x) {
         const int o = (int)(idx % C_out);
         const long long r = idx / C_out;
         const int tap = (int)(r % T), ci = (int)(r / T);
-        Wt[idx] = __float2bfloat16_rn(W[((long long)o * T + tap) * C_in + ci]);
+        Wt[idx] = __float2bfloat16_rn(ci < C_in ? W[((long long)o * T + tap) * C_in + ci] : 0.f);
     }
 }
 
@@ -271,6 +273,7 @@ struct ConvGemmArgs {
     int k, stride, pad;
     int Mp;
     int P_rows;          // row positions (forward: ni Ho Wo; dS: ni H W; dW: K positions ni Ho Wo)
+    int C_t;             // the layer's input channels (C_in is that rounded up to 64 when smaller)
     int n_row, n_col, n_split, kt_per_split, ktiles;
     float *what;         // forward: w^ [P_out][C_out][Mp]
     const float *t_in;   // dS: layer input spike times [P_in][C_in]
@@ -689,8 +692,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 wk[h] = -1000;
                 wdR[h] = wdL[h] = 0.f;
                 const int col0 = ct * BN + (group + 2 * h) * 32;
-                if (p >= 0) {
-                    const float x = __ldg(a.t_in + (long long)p * a.C_in + col0 + lane);
+                if (p >= 0 && col0 + lane < a.C_t) {
+                    const float x = __ldg(a.t_in + (long long)p * a.C_t + col0 + lane);
                     if (isfinite(x)) {
                         const BinW w = bin_weights(a.c, x, true);
                         wk[h] = w.k;
@@ -720,7 +723,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     const int k0 = wk[h] - m_base, k1 = wk[h] + 1 - m_base;
                     if (k0 >= 0 && k0 < 32 && wk[h] < a.c.M) g = fmaf(tb[k0 * EPI_LD + lane], wdR[h], g);
                     if (k1 >= 0 && k1 < 32 && wk[h] + 1 < a.c.M) g = fmaf(tb[k1 * EPI_LD + lane], wdL[h], g);
-                    if (g != 0.f) atomicAdd(a.g_t_in + (long long)p * a.C_in + ct * BN + cc * 32 + lane, g);
+                    if (g != 0.f) atomicAdd(a.g_t_in + (long long)p * a.C_t + ct * BN + cc * 32 + lane, g);
                 }
                 __syncwarp();
             }
@@ -788,8 +791,8 @@ __device__ __forceinline__ void bins_put(uint16_t *T, int row0, int C, int c, in
     }
 }
 
-__global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const float *__restrict__ t, int P, int C, LifConst lc,
-                                                        __nv_bfloat16 *__restrict__ S) {
+__global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const float *__restrict__ t, int P, int C, int Ct,
+                                                        LifConst lc, __nv_bfloat16 *__restrict__ S) {
     const int Mp = lc.Mp, M = lc.M;
     extern __shared__ __align__(128) uint8_t bins_smem[];
     const int R = C >= BINS_THREADS ? 1 : BINS_THREADS / C;  // positions per group
@@ -815,8 +818,9 @@ __global__ void __launch_bounds__(BINS_THREADS) k_bin_S(const float *__restrict_
         for (int j = 0; j < BINS_MAXSPT; ++j) {
             if (j < spt) {
                 const int c = c0 + j * BINS_THREADS;
-                const uint2 q =
-                    p < P ? bin_record(lc, __ldg(t + (long long)p * C + c)) : make_uint2((uint32_t)REC_SILENT, 0u);
+                // channels past the layer's Ct (padding up to C) are silent
+                const uint2 q = p < P && c < Ct ? bin_record(lc, __ldg(t + (long long)p * Ct + c))
+                                                : make_uint2((uint32_t)REC_SILENT, 0u);
                 bins_put(T, r * Mp, C, c, odd ? kold1[j] : kold0[j], q, M);
                 if (odd) kold1[j] = (int)q.x;
                 else kold0[j] = (int)q.x;
@@ -1725,12 +1729,20 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 for (int cc = group; cc < BN / 32; cc += 2) {
                     float v[32];
                     tc::tmem_ld32(tmem + lane_base + gi * BN + cc * 32, v);
-                    if (kidx < Ktot) {
+                    // filter row kidx = (tap, channel) of the padded K; its place in
+                    // g_W [C_out][k k C_t] (rows of padding channels are dropped)
+                    int kreal = kidx, Kreal = Ktot;
+                    if (a.C_t != a.C_in) {
+                        const int tap = kidx / a.C_in, ch = kidx - tap * a.C_in;
+                        kreal = ch < a.C_t ? tap * a.C_t + ch : -1;
+                        Kreal = a.k * a.k * a.C_t;
+                    }
+                    if (kidx < Ktot && kreal >= 0) {
                         const int o0 = ct * BN + cc * 32;
 #pragma unroll
                         for (int u = 0; u < 32; ++u) {
                             const float add = (first && a.count) ? a.qcoef * a.count[o0 + u] : 0.f;
-                            atomicAdd(a.g_W + (long long)(o0 + u) * Ktot + kidx, v[u] + add);
+                            atomicAdd(a.g_W + (long long)(o0 + u) * Kreal + kreal, v[u] + add);
                         }
                     }
                 }
@@ -1864,6 +1876,7 @@ static ConvGemmArgs base_args(const ConvGeom &g, int ni, const LifConst &c) {
     a.H = g.H;
     a.W = g.W;
     a.C_in = g.C;
+    a.C_t = g.C;
     a.Ho = g.Ho;
     a.Wo = g.Wo;
     a.k = g.k;
@@ -1877,9 +1890,12 @@ static ConvGemmArgs base_args(const ConvGeom &g, int ni, const LifConst &c) {
 }  // namespace
 
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp) {
-    return g.C % 64 == 0 && C_out % 64 == 0 && (C_out <= 256 || C_out % 256 == 0) && (Mp == 32 || Mp == 64) &&
-           g.k <= 7 && g.C * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
+    const int Cp = conv_padded_channels(g.C);
+    return Cp % 64 == 0 && C_out % 64 == 0 && (C_out <= 256 || C_out % 256 == 0) && (Mp == 32 || Mp == 64) &&
+           g.k <= 7 && Cp * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
 }
+
+int conv_padded_channels(int C) { return C < 64 ? 64 : C; }
 
 cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                              long long P, int C, const LifConst &c, __nv_bfloat16 *D, float *count,
@@ -1895,11 +1911,12 @@ cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, c
     return cudaGetLastError();
 }
 
-cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, __nv_bfloat16 *Wt, cudaStream_t st) {
-    const long long n = (long long)C_out * T * C_in;
+cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, int C_pad, __nv_bfloat16 *Wt,
+                             cudaStream_t st) {
+    const long long n = (long long)C_out * T * C_pad;
     long long blocks = (n + 255) / 256;
     if (blocks > 4096) blocks = 4096;
-    k_filters_t<<<(unsigned)blocks, 256, 0, st>>>(W, C_out, T, C_in, Wt);
+    k_filters_t<<<(unsigned)blocks, 256, 0, st>>>(W, C_out, T, C_in, C_pad, Wt);
     return cudaGetLastError();
 }
 
@@ -1920,7 +1937,7 @@ static DsPlan tap_plan(int k, int ppt, int Mp, int BN, bool resident, long long 
 // dS of ni images with the input-time gradient: dw^ [ni Ho Wo][Mp][C_out],
 // Wt [C_in][k k C_out], t_in [ni H W][C_in] -> g_t_in (zeroed first)
 cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *dW_hat,
-                                const __nv_bfloat16 *Wt, const float *t_in, float *g_t_in, cudaStream_t st) {
+                                const __nv_bfloat16 *Wt, const float *t_in, float *g_t_in, int C_t, cudaStream_t st) {
     ConvGemmArgs a = base_args(g, ni, c);
     a.C_out = C_out;
     a.P_rows = ni * g.H * g.W;
@@ -1930,7 +1947,8 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     a.n_col = g.C / BN;
     a.t_in = t_in;
     a.g_t_in = g_t_in;
-    cudaError_t e = cudaMemsetAsync(g_t_in, 0, sizeof(float) * (size_t)a.P_rows * g.C, st);
+    a.C_t = C_t;
+    cudaError_t e = cudaMemsetAsync(g_t_in, 0, sizeof(float) * (size_t)a.P_rows * C_t, st);
     if (e != cudaSuccess) return e;
     // resident transposed filters when they are small; one box per filter row
     // at stride 1 when every tile lies within one image row
@@ -2053,9 +2071,10 @@ cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifC
 // [ni Ho Wo][Mp][C_out], added into g_W (zeroed by the caller before the
 // first chunk)
 cudaError_t launch_conv_dw_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
+                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W, int C_t,
                                cudaStream_t st) {
     ConvGemmArgs a = base_args(g, ni, c);
+    a.C_t = C_t;
     a.C_out = C_out;
     a.P_rows = ni * g.Ho * g.Wo;
     if (a.P_rows == 0) return cudaSuccess;
@@ -2114,9 +2133,11 @@ bool conv_bin_S_supported(int C) {
     return C % 64 == 0 && C <= BINS_THREADS * BINS_MAXSPT && (C <= BINS_THREADS || C % BINS_THREADS == 0);
 }
 
-cudaError_t launch_bin_S(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st) {
+cudaError_t launch_bin_S(const float *t, long long P, int C, int Ct, const LifConst &c, __nv_bfloat16 *S,
+                         cudaStream_t st) {
     const int Mp = c.Mp;
-    if (!conv_bin_S_supported(C) || P >= (1ll << 31) || P * Mp * C >= (1ll << 31)) return cudaErrorInvalidValue;
+    if (!conv_bin_S_supported(C) || Ct < 1 || Ct > C || P >= (1ll << 31) || P * Mp * C >= (1ll << 31))
+        return cudaErrorInvalidValue;
     if (P == 0) return cudaSuccess;
     const int R = C >= BINS_THREADS ? 1 : BINS_THREADS / C;
     const int smem = 2 * R * Mp * C * 2;
@@ -2128,7 +2149,7 @@ cudaError_t launch_bin_S(const float *t, long long P, int C, const LifConst &c, 
     if (per_sm > 8) per_sm = 8;
     long long blocks = (long long)per_sm * conv_num_sms();
     if (blocks > ngroups) blocks = ngroups;
-    k_bin_S<<<(unsigned)blocks, BINS_THREADS, smem, st>>>(t, (int)P, C, c, S);
+    k_bin_S<<<(unsigned)blocks, BINS_THREADS, smem, st>>>(t, (int)P, C, Ct, c, S);
     return cudaGetLastError();
 }
 

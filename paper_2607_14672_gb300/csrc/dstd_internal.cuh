@@ -433,17 +433,22 @@ struct ConvGeom {
 // multiples of 64 and Mp in {32, 64}: no im2col operand. ni = images of the
 // chunk; positions NHWC.
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp);
+// input channels of the implicit path: C_in below 64 is padded to 64 (silent
+// inputs, zero filter rows)
+int conv_padded_channels(int C);
 // dw^ [P][Mp][C] bf16 from the saved state [P][C]; silent counts per channel
 // added into count (zeroed by the caller)
 cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, const float *vdot, const float *g_up,
                              long long P, int C, const LifConst &c, __nv_bfloat16 *D, float *count, cudaStream_t st);
-// filters [C_out][T][C_in] fp32 -> [C_in][T][C_out] bf16
-cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, __nv_bfloat16 *Wt, cudaStream_t st);
+// filters [C_out][T][C_in] fp32 -> [C_pad][T][C_out] bf16 (padding rows zero)
+cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, int C_pad, __nv_bfloat16 *Wt,
+                             cudaStream_t st);
 // dS of ni images (the transposed convolution of dw^ [ni Ho Wo][Mp][C_out]
 // with Wt [C_in][k k C_out]) with the input-time gradient in the epilogue:
 // g_t_in [ni H W][C_in] (zeroed first) from t_in [ni H W][C_in]
+// (g.C may be the padded channel count; t_in and g_t_in have C_t channels)
 cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *dW_hat,
-                                const __nv_bfloat16 *Wt, const float *t_in, float *g_t_in, cudaStream_t st);
+                                const __nv_bfloat16 *Wt, const float *t_in, float *g_t_in, int C_t, cudaStream_t st);
 // the binned operand generated on chip: one 8-byte record per input
 // (grid step, bf16 pair of its two weights), then the forward (w^ [ni Ho
 // Wo][C_out][Mp] fp32) and dW (added into g_W [C_out][k k C_in], zeroed by
@@ -460,13 +465,16 @@ cudaError_t launch_conv_dw_gen(const ConvGeom &g, int ni, int C_out, const LifCo
 // scan/solve/select of each neuron in its epilogue (outputs as from
 // launch_scan_solve: spike times, q, s, dv^/dt, penalty sums)
 bool conv_bin_S_supported(int C);  // channel counts the S writer takes
-cudaError_t launch_bin_S(const float *t, long long P, int C, const LifConst &c, __nv_bfloat16 *S, cudaStream_t st);
+// t has Ct <= C channels; channels Ct .. C - 1 of S are silent
+cudaError_t launch_bin_S(const float *t, long long P, int C, int Ct, const LifConst &c, __nv_bfloat16 *S,
+                         cudaStream_t st);
 cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
                                 const __nv_bfloat16 *Wf, const float *rowsum, float *t_out, int *q, float *s,
                                 float *vdot, float *penalty, cudaStream_t st);
 // dW from S and dw^ (added into g_W as for launch_conv_dw_gen)
+// (g.C may be the padded channel count; g_W is [C_out][k k C_t])
 cudaError_t launch_conv_dw_tma(const ConvGeom &g, int ni, int C_out, const LifConst &c, const __nv_bfloat16 *S,
-                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W,
+                               const __nv_bfloat16 *dW_hat, const float *count, float qcoef, float *g_W, int C_t,
                                cudaStream_t st);
 cudaError_t conv_status_read(unsigned int *out, int clear);
 // im2col binning of positions [pos0, pos0 + npos): the grid weights of the
