@@ -35,6 +35,7 @@ struct LifConst {
     int M, Mp;             // steps, padded bin axis of the internal layouts
     float vdot_floor;      // lower bound on dv^/dt at a spike (1e-6 v_th / dt)
     float Kmax;            // max of K(s) over s in [0, dt] (with a 1e-6 relative margin)
+    float Kmax4;           // the same over [0, 4 dt]
     float t_head, t_tail, g_head, g_tail, g_q, norm;
 };
 
@@ -312,12 +313,26 @@ __device__ __forceinline__ bool scan_walk(const LifConst &c, const float *row, i
         }
         const float4 x = *reinterpret_cast<const float4 *>(row + g);
         const float xs[4] = {x.x, x.y, x.z, x.w};
+        // over these four bins the potential is at most max(v, 0) + Kmax4
+        // (max(I, 0) + the positive inputs), Kmax4 the largest K(s) over four
+        // steps (K >= 0, and the current only decays between inputs); well
+        // below v_th no bin can hold the spike and the flags are not formed
+        const float ipos = fmaxf(I, 0.0f) + fmaxf(x.x, 0.0f) + fmaxf(x.y, 0.0f) + fmaxf(x.z, 0.0f) + fmaxf(x.w, 0.0f);
+        if (fmaf(ipos, c.Kmax4, fmaxf(v, 0.0f)) < c.vth * 0.99999f) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const BinStep r = bin_step(c, v, I + xs[u]);
-            if (r.endp | r.peak) mask |= 1u << (g + u);
-            v = r.ve;
-            I = r.In;
+            for (int u = 0; u < 4; ++u) {
+                const float I0 = I + xs[u];
+                v = fmaf(c.KD, I0, c.rv * v);
+                I = c.rI * I0;
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const BinStep r = bin_step(c, v, I + xs[u]);
+                if (r.endp | r.peak) mask |= 1u << (g + u);
+                v = r.ve;
+                I = r.In;
+            }
         }
     }
     if (mend < 32) mask &= (1u << mend) - 1u;

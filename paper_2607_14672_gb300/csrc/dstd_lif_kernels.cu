@@ -41,11 +41,14 @@ LifConst make_const(const dstd_params &p, int Mp) {
     {
         // K(s) = e^{-av s} phi(s) rises to a single maximum (or keeps rising
         // when av = 0 or aI = 0); take it at min(dt, peak time)
-        double tp = dt;
+        double tp = INFINITY;  // keeps rising: the end of the window
         if (av > 0.0 && aI > 0.0) tp = (lam == 0.0) ? 1.0 / av : log(aI / av) / lam;
         const double s_ = tp < dt ? tp : dt;
         const double phis = lam == 0.0 ? s_ : -expm1(-lam * s_) / lam;
         c.Kmax = (float)(exp(-av * s_) * phis * (1.0 + 1e-6));
+        const double s4 = tp < 4.0 * dt ? tp : 4.0 * dt;
+        const double phi4 = lam == 0.0 ? s4 : -expm1(-lam * s4) / lam;
+        c.Kmax4 = (float)(exp(-av * s4) * phi4 * (1.0 + 1e-6));
     }
     c.t_head = p.t_head;
     c.t_tail = p.t_tail;
@@ -531,46 +534,69 @@ cudaError_t launch_fwd_operands_f16(const float *t, int B, int N, const LifConst
     return cudaGetLastError();
 }
 
-// row j, columns (b, m): a warp takes 32 consecutive samples of one input j,
-// zero-fills their 32 x Mp bins (consecutive 16-byte chunks, one per lane per
-// round), then each lane stores the two weights of its own sample; with bw
-// != null it also writes (k, ds/dt at T_k, ds/dt at T_{k+1}) of its sample
-// to bw[b*N + j] (k = -100 for a silent input) for the input-time gradient.
+// row j, columns (b, m), for a tile of 32 inputs x 32 samples per block (4
+// warps): first the tile's spike times are read along j (coalesced), binned,
+// and with bw != null the per-input records (k, ds/dt at T_k, at T_{k+1}; k =
+// -100 for a silent input) written along j to bw[b*N + j]; the bin and the
+// two weights (hi and lo halves packed in pairs) go to shared memory. Then
+// each warp writes 8 of the tile's rows: the 32 samples' Mp bins of row j are
+// consecutive, and lane g of a round builds 16-byte chunk g of them from the
+// bin and weights of its sample (at most two nonzero halves), so a store
+// instruction covers 512 contiguous bytes.
 template <int OP>
-__global__ void k_binning_cols8(const float *__restrict__ t, int B, int N, LifConst c, uint16_t *hi, uint16_t *lo,
-                                int ld, float4 *bw) {
+__global__ void __launch_bounds__(128) k_binning_cols8(const float *__restrict__ t, int B, int N, LifConst c,
+                                                       uint16_t *hi, uint16_t *lo, int ld, float4 *bw) {
+    __shared__ int sk[32][33];
+    __shared__ uint32_t swh[32][33], swl[32][33];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int b0 = (blockIdx.x * (blockDim.x >> 5) + warp) * 32;
-    if (b0 >= B) return;
-    const int ns = (B - b0) < 32 ? (B - b0) : 32;
-    const int nch = ns * c.Mp / 8;  // 16-byte chunks of the warp's samples
-    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-    const int b = b0 + lane;
-    for (int j = blockIdx.y; j < N; j += gridDim.y) {
-        const long long rowbase = (long long)j * ld + (long long)b0 * c.Mp;
-        for (int g = lane; g < nch; g += 32) {
-            *reinterpret_cast<uint4 *>(hi + rowbase + 8 * g) = z;
-            if (OP != 2) *reinterpret_cast<uint4 *>(lo + rowbase + 8 * g) = z;
-        }
-        // the zeros of a lane's sample were stored by other lanes: order them
-        // before its weights
-        __syncwarp();
-        if (b >= B) continue;
+    const int j0 = blockIdx.x * 32, b0 = blockIdx.y * 32;
+    const int j = j0 + lane;
+    for (int bb = warp; bb < 32; bb += 4) {
+        const int b = b0 + bb;
         BinW w{-100, 0.f, 0.f, 0.f, 0.f};
-        const float x = t[(long long)b * N + j];
-        if (isfinite(x)) w = bin_weights(c, x, bw != nullptr);
-        if (bw) bw[(long long)b * N + j] = make_float4(__int_as_float(w.k), w.dR, w.dL, 0.f);
-        const long long o = rowbase + (long long)lane * c.Mp;
-        uint16_t h, l;
-        if (w.k >= 0 && w.k < c.M) {
-            split16<OP>(w.wR, h, l);
-            hi[o + w.k] = h;
-            if (OP != 2) lo[o + w.k] = l;
+        if (b < B && j < N) {
+            const float x = __ldg(t + (long long)b * N + j);
+            if (isfinite(x)) w = bin_weights(c, x, bw != nullptr);
+            if (bw) bw[(long long)b * N + j] = make_float4(__int_as_float(w.k), w.dR, w.dL, 0.f);
         }
-        if (w.k + 1 >= 0 && w.k + 1 < c.M) {
-            split16<OP>(w.wL, h, l);
-            hi[o + w.k + 1] = h;
-            if (OP != 2) lo[o + w.k + 1] = l;
+        uint16_t hR = 0, lR = 0, hL = 0, lL = 0;
+        if (w.k >= 0 && w.k < c.M) split16<OP>(w.wR, hR, lR);
+        if (w.k + 1 >= 0 && w.k + 1 < c.M) split16<OP>(w.wL, hL, lL);
+        sk[lane][bb] = w.k;
+        swh[lane][bb] = (uint32_t)hR | ((uint32_t)hL << 16);
+        swl[lane][bb] = (uint32_t)lR | ((uint32_t)lL << 16);
+    }
+    __syncthreads();
+    const int ns = (B - b0) < 32 ? (B - b0) : 32;
+    const int cps = c.Mp >> 3;  // 16-byte chunks per sample
+    const int nch = ns * cps;
+    for (int jj = warp; jj < 32; jj += 4) {
+        const int jr = j0 + jj;
+        if (jr >= N) break;
+        const long long rowbase = (long long)jr * ld + (long long)b0 * c.Mp;
+        for (int g = lane; g < nch; g += 32) {
+            const int bb = g / cps, q = g - bb * cps;
+            const int k = sk[jj][bb];
+            // the sample's weight at T_k sits at half e1 of the chunk, at T_{k+1} at e1 + 1
+            const int e1 = k - 8 * q;
+            const uint32_t ph = swh[jj][bb], pl = swl[jj][bb];
+            uint32_t h[4] = {0u, 0u, 0u, 0u}, l[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                // halves 2i and 2i + 1 of the chunk
+                if (e1 == 2 * i) {
+                    h[i] = ph;
+                    l[i] = pl;
+                } else if (e1 == 2 * i - 1) {
+                    h[i] = ph >> 16;
+                    l[i] = pl >> 16;
+                } else if (e1 == 2 * i + 1) {
+                    h[i] = ph << 16;
+                    l[i] = pl << 16;
+                }
+            }
+            *reinterpret_cast<uint4 *>(hi + rowbase + 8 * g) = make_uint4(h[0], h[1], h[2], h[3]);
+            if (OP != 2) *reinterpret_cast<uint4 *>(lo + rowbase + 8 * g) = make_uint4(l[0], l[1], l[2], l[3]);
         }
     }
 }
@@ -596,12 +622,14 @@ cudaError_t launch_binning(const float *t, int B, int N, const LifConst &c, OpKi
         else if (op == OpKind::F16X3) k_binning_rows<3><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
         else k_binning_rows<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld);
     } else {
-        dim3 grid(blocks_for(B, 128), N < 65535 ? N : 65535);
         if (sparse && op != OpKind::F16X3) {
-            if (op == OpKind::BF16X3) k_binning_cols8<1><<<grid, 128, 0, st>>>(t, B, N, c, h16, l16, ld, bw);
-            else k_binning_cols8<2><<<grid, 128, 0, st>>>(t, B, N, c, h16, l16, ld, bw);
+            if ((N + 31) / 32 > 0x7fffffff || (B + 31) / 32 > 65535) return cudaErrorInvalidValue;
+            dim3 g8((unsigned)((N + 31) / 32), (unsigned)((B + 31) / 32));
+            if (op == OpKind::BF16X3) k_binning_cols8<1><<<g8, 128, 0, st>>>(t, B, N, c, h16, l16, ld, bw);
+            else k_binning_cols8<2><<<g8, 128, 0, st>>>(t, B, N, c, h16, l16, ld, bw);
             return cudaGetLastError();
         }
+        dim3 grid(blocks_for(B, 128), N < 65535 ? N : 65535);
         if (op == OpKind::F32) k_binning_cols<0><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
         else if (op == OpKind::BF16X3) k_binning_cols<1><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
         else k_binning_cols<2><<<grid, 128, 0, st>>>(t, B, N, c, hi, lo, ld, bw);
@@ -1410,14 +1438,18 @@ __global__ void k_dwhat(const float *__restrict__ t_out, const int *__restrict__
     }
 }
 
-// The same values in the (i, (b, m)) layout only, written row-contiguously:
-// a warp per neuron i and a block per 8 neurons x spb (<= 32) samples. Lane
-// k first takes the scalars of sample b0 + k (coefficient, s, q and the two
-// kernel values next to the spike); then lane f of the warp's (sample,
-// 16-byte chunk) sequence fetches its sample's scalars from the owning lane
-// and writes chunk f, so every store instruction covers up to 512 contiguous
-// bytes of row i (the samples of a row are adjacent: column b Mp + m).
-// Silent neurons are counted per warp and added with one atomic.
+// The same values in the (i, (b, m)) layout only, written row-contiguously,
+// a block per 32 neurons x spb (<= 32) samples. First the block reads the
+// per-(sample, neuron) inputs along the neurons (coalesced) and keeps each
+// neuron's bin q, the coefficient -g/v^' folded into the two exponential
+// terms of K at T_0, and the two accurate kernel values next to the spike
+// in shared memory. Then each warp writes the rows of 4 neurons: lane f of a
+// row's (sample, 16-byte chunk) sequence writes chunk f, so every store
+// instruction covers up to 512 contiguous bytes (column b Mp + m). A chunk
+// wholly before the spike's last two bins is the bare geometric recurrence
+// in m (factors e^{av dt}, e^{aI dt}), a chunk after the spike is zero, and
+// only the chunk holding bins q - 1, q selects per bin. Silent neurons are
+// counted per block column and added with one atomic each.
 template <int OP>
 __global__ void __launch_bounds__(256) k_dwhat_rows(const float *__restrict__ t_out, const int *__restrict__ qv,
                                                     const float *__restrict__ sv, const float *__restrict__ vd,
@@ -1425,71 +1457,100 @@ __global__ void __launch_bounds__(256) k_dwhat_rows(const float *__restrict__ t_
                                                     void *a_hi, void *a_lo, int lda, float *count, int spb) {
     constexpr int EB = OP == 0 ? 4 : 2;
     constexpr int BPC = 16 / EB;
-    const int lane = threadIdx.x & 31;
-    const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
-    if (i >= N) return;
-    const int b0 = blockIdx.y * spb;
+    __shared__ int sq[32][33];
+    __shared__ float sa[32][33], sb[32][33], sk0[32][33], sk1[32][33];
+    __shared__ int scount[32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int i0 = blockIdx.x * 32, b0 = blockIdx.y * spb;
     const int nb = (B - b0) < spb ? (B - b0) : spb;
+    if (threadIdx.x < 32) scount[threadIdx.x] = 0;
+    __syncthreads();
+    {
+        const int i = i0 + lane;
+        int silent = 0;
+        for (int bl = warp; bl < nb; bl += 8) {
+            int q = c.M;
+            float A = 0.f, Bt = 0.f, K0 = 0.f, K1 = 0.f;
+            if (i < N) {
+                const long long idx = (long long)(b0 + bl) * N + i;
+                q = __ldg(qv + idx);
+                const float to = __ldg(t_out + idx), gu = g_up ? __ldg(g_up + idx) : 0.f, vdi = __ldg(vd + idx),
+                            s0 = __ldg(sv + idx);
+                if (q < c.M) {
+                    float pv, pg;
+                    penalty_T(c, to, pv, pg);
+                    const float coef = -(gu + pg) / vdi;
+                    const float x = s0 + (float)q * c.dt;  // t - T_0
+                    K0 = coef * kernel_K(c, s0);
+                    K1 = coef * kernel_K(c, s0 + c.dt);
+                    if (c.lam_zero) {
+                        A = coef * __expf(-c.av * x);
+                        Bt = x;
+                    } else {
+                        A = coef * c.inv_lam * __expf(-c.av * x);
+                        Bt = coef * c.inv_lam * __expf(-c.aI * x);
+                    }
+                } else {
+                    ++silent;
+                }
+            }
+            sq[lane][bl] = q;
+            sa[lane][bl] = A;
+            sb[lane][bl] = Bt;
+            sk0[lane][bl] = K0;
+            sk1[lane][bl] = K1;
+        }
+        if (silent) atomicAdd(&scount[lane], silent);
+    }
+    __syncthreads();
+    if (count && threadIdx.x < 32 && i0 + threadIdx.x < N && scount[threadIdx.x])
+        atomicAdd(&count[i0 + threadIdx.x], (float)scount[threadIdx.x]);
     const int cps = c.Mp / BPC;
     const int total = nb * cps;
-    int pq = c.M;
-    float pcoef = 0.f, ps0 = 0.f, pKq = 0.f, pKq1 = 0.f;
-    if (lane < nb) {
-        const long long idx = (long long)(b0 + lane) * N + i;
-        pq = qv[idx];
-        const float to = t_out[idx], gu = g_up ? g_up[idx] : 0.f, vdi = vd[idx], s0 = sv[idx];
-        if (pq < c.M) {
-            float pv, pg;
-            penalty_T(c, to, pv, pg);
-            pcoef = -(gu + pg) / vdi;
-            ps0 = s0;
-            pKq = kernel_K(c, s0);
-            pKq1 = kernel_K(c, s0 + c.dt);
-        }
-    }
-    if (count) {
-        const int silent = __popc(__ballot_sync(0xffffffffu, lane < nb && pq >= c.M));
-        if (lane == 0 && silent) atomicAdd(&count[i], (float)silent);
-    }
     const float fv = __expf(c.av * c.dt), fI = __expf(c.aI * c.dt);
-    for (int f0 = 0; f0 < total; f0 += 32) {
-        const int f = f0 + lane;
-        const bool valid = f < total;
-        const int bl = f / cps, ch = f - bl * cps;
-        const int src = valid ? bl : 0;
-        const int q = __shfl_sync(0xffffffffu, pq, src);
-        const float coef = __shfl_sync(0xffffffffu, pcoef, src);
-        const float s0 = __shfl_sync(0xffffffffu, ps0, src);
-        const float Kq = __shfl_sync(0xffffffffu, pKq, src);
-        const float Kq1 = __shfl_sync(0xffffffffu, pKq1, src);
-        if (!valid) continue;
-        const int m0 = ch * BPC;
-        float v[BPC];
+    for (int il = warp; il < 32; il += 8) {
+        const int i = i0 + il;
+        if (i >= N) break;
+        for (int f = lane; f < total; f += 32) {
+            const int bl = f / cps, ch = f - bl * cps;
+            const int q = sq[il][bl];
+            const int m0 = ch * BPC;
+            float v[BPC];
 #pragma unroll
-        for (int u = 0; u < BPC; ++u) v[u] = 0.f;
-        if (q < c.M && m0 <= q) {
-            float x = s0 + (float)(q - m0) * c.dt;
-            float ev = __expf(-c.av * x), eI = __expf(-c.aI * x);
+            for (int u = 0; u < BPC; ++u) v[u] = 0.f;
+            if (q < c.M && m0 <= q) {
+                // the terms at T_m0: e^{av m0 dt}, e^{aI m0 dt} times those at T_0
+                const float gv = __expf(c.av * c.dt * (float)m0), gI = __expf(c.aI * c.dt * (float)m0);
+                float A = sa[il][bl] * gv, Bt = c.lam_zero ? sb[il][bl] - (float)m0 * c.dt : sb[il][bl] * gI;
+                if (m0 + BPC - 1 < q - 1) {
 #pragma unroll
-            for (int u = 0; u < BPC; ++u) {
-                const int m = m0 + u;
-                const float Kf = c.lam_zero ? x * ev : (ev - eI) * c.inv_lam;
-                const float K = (m == q) ? Kq : ((m == q - 1) ? Kq1 : Kf);
-                v[u] = (m <= q) ? coef * K : 0.f;
-                ev *= fv;
-                eI *= fI;
-                x -= c.dt;
+                    for (int u = 0; u < BPC; ++u) {
+                        v[u] = c.lam_zero ? A * Bt : A - Bt;
+                        A *= fv;
+                        Bt = c.lam_zero ? Bt - c.dt : Bt * fI;
+                    }
+                } else {
+                    const float K0 = sk0[il][bl], K1 = sk1[il][bl];
+#pragma unroll
+                    for (int u = 0; u < BPC; ++u) {
+                        const int m = m0 + u;
+                        const float d = c.lam_zero ? A * Bt : A - Bt;
+                        v[u] = m < q - 1 ? d : (m == q - 1 ? K1 : (m == q ? K0 : 0.f));
+                        A *= fv;
+                        Bt = c.lam_zero ? Bt - c.dt : Bt * fI;
+                    }
+                }
             }
-        }
-        const long long o = (long long)i * lda + (long long)(b0 + bl) * c.Mp + m0;
-        if (OP == 0) {
-            *reinterpret_cast<float4 *>((float *)a_hi + o) = make_float4(v[0], v[1], v[2], v[3]);
-        } else {
-            __align__(16) __nv_bfloat16 hh[BPC], ll[BPC];
+            const long long o = (long long)i * lda + (long long)(b0 + bl) * c.Mp + m0;
+            if (OP == 0) {
+                *reinterpret_cast<float4 *>((float *)a_hi + o) = make_float4(v[0], v[1], v[2], v[3]);
+            } else {
+                __align__(16) __nv_bfloat16 hh[BPC], ll[BPC];
 #pragma unroll
-            for (int u = 0; u < BPC; ++u) split_bf16(v[u], hh[u], ll[u]);
-            *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + o) = *reinterpret_cast<uint4 *>(hh);
-            if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + o) = *reinterpret_cast<uint4 *>(ll);
+                for (int u = 0; u < BPC; ++u) split_bf16(v[u], hh[u], ll[u]);
+                *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_hi + o) = *reinterpret_cast<uint4 *>(hh);
+                if (OP == 1) *reinterpret_cast<uint4 *>((__nv_bfloat16 *)a_lo + o) = *reinterpret_cast<uint4 *>(ll);
+            }
         }
     }
 }
@@ -1506,7 +1567,7 @@ cudaError_t launch_dwhat(const float *t_out, const int *q, const float *s, const
     const int spb = cps >= 32 ? 2 : (64 / cps > 32 ? 32 : 64 / cps);
     const long long gy = ((long long)B + spb - 1) / spb;
     if (!b_hi && gy <= 65535) {
-        dim3 grid((unsigned)((N + 7) / 8), (unsigned)gy);
+        dim3 grid((unsigned)((N + 31) / 32), (unsigned)gy);
         if (op == OpKind::F32)
             k_dwhat_rows<0><<<grid, 256, 0, st>>>(t_out, q, s, vdot, g_up, B, N, c, a_hi, a_lo, lda, silent_count, spb);
         else if (op == OpKind::BF16X3)
