@@ -402,8 +402,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         }
         for (int u = 0; u < 2; ++u) {
             tc::mbar_init(&acc_full[u], 1);
-            // the forward's epilogue groups take alternate tiles (one per accumulator)
-            tc::mbar_init(&acc_empty[u], FWD ? CONV_NEPI / 2 : CONV_NEPI);
+            // the epilogue groups take alternate tiles (one per accumulator)
+            tc::mbar_init(&acc_empty[u], CONV_NEPI / 2);
         }
         tc::mbar_init(bres_full, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -570,10 +570,11 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                                 }
                                 const uint32_t bbase = RES ? tc::smem_u32(bres + (tap * ncb + cb) * BN * 128)
                                                            : sa + (uint32_t)(pl.a_bytes + v * BN * 128);
+                                // descriptors built once; each 16-deep slice is 32 bytes on (+2)
+                                const uint64_t ad = tc::sdesc_sw128(abase), bd = tc::sdesc_sw128(bbase);
+                                tc::mma_bf16(acc, ad, bd, idesc, (!first || v > 0) ? 1u : 0u);
 #pragma unroll
-                                for (int kk = 0; kk < 4; ++kk)
-                                    tc::mma_bf16(acc, tc::sdesc_sw128(abase + kk * 32), tc::sdesc_sw128(bbase + kk * 32),
-                                                 idesc, (!first || v > 0 || kk > 0) ? 1u : 0u);
+                                for (int kk = 1; kk < 4; ++kk) tc::mma_bf16(acc, ad + 2 * kk, bd + 2 * kk, idesc, 1u);
                             }
                             first = false;
                             tc::mma_commit(&empty[s]);
@@ -672,16 +673,17 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             }
         }
     } else {
+        // dS: epilogue group g takes the tiles of accumulator g (every other
+        // tile), all BN columns of them; warp w reads TMEM lane quarter w % 4
         const int quarter = warp & 3, group = (warp - 2) >> 2;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
         float *tb = epi + (warp - 2) * 32 * EPI_LD;
         const int pp = (quarter * 32) / Mp;      // position of this warp's rows (Mp >= 32)
         const int m_base = (quarter * 32) % Mp;  // first grid step of this warp's rows
-        constexpr int NCH = BN / 64;             // 32-column chunks of this warp
-        uint32_t j = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++j) {
+        constexpr int NCH = BN / 32;             // 32-column chunks of the tile
+        for (int j = group, t = blockIdx.x + group * gridDim.x; t < ntiles; j += 2, t += 2 * gridDim.x) {
             const int rt = t / a.n_col, ct = t - rt * a.n_col;
-            const uint32_t buf = j & 1u;
+            const uint32_t buf = (uint32_t)group;
             const int p = ds_pos(pl, a.H, a.W, ds_class(pl, rt), rt, pp, ppt);
             // the grid step and the two kernel derivatives of the input each
             // lane will own, loaded while the tile's MMAs run
@@ -691,7 +693,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
             for (int h = 0; h < NCH; ++h) {
                 wk[h] = -1000;
                 wdR[h] = wdL[h] = 0.f;
-                const int col0 = ct * BN + (group + 2 * h) * 32;
+                const int col0 = ct * BN + h * 32;
                 if (p >= 0 && col0 + lane < a.C_t) {
                     const float x = __ldg(a.t_in + (long long)p * a.C_t + col0 + lane);
                     if (isfinite(x)) {
@@ -702,16 +704,20 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     }
                 }
             }
-            if (!tc::mbar_wait_sleep(&acc_full[buf], (j >> 1) & 1u)) {
+            if (!tc::mbar_wait_sleep(&acc_full[buf], (uint32_t)(j >> 1) & 1u)) {
                 conv_set_status(STATUS_TIMEOUT);
                 break;
             }
             tc::tc_fence_after();
 #pragma unroll
             for (int h = 0; h < NCH; ++h) {
-                const int cc = group + 2 * h;
                 float v[32];
-                tc::tmem_ld32(tmem + lane_base + buf * BN + cc * 32, v);
+                tc::tmem_ld32(tmem + lane_base + buf * BN + h * 32, v);
+                if (h == NCH - 1) {  // the tile's last TMEM read of this warp
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
+                }
                 // lane m of the warp holds grid step m_base + m of 32 channels;
                 // transpose through shared memory so that lane u owns channel
                 // col0 + u and reads its two grid steps
@@ -723,13 +729,10 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     const int k0 = wk[h] - m_base, k1 = wk[h] + 1 - m_base;
                     if (k0 >= 0 && k0 < 32 && wk[h] < a.c.M) g = fmaf(tb[k0 * EPI_LD + lane], wdR[h], g);
                     if (k1 >= 0 && k1 < 32 && wk[h] + 1 < a.c.M) g = fmaf(tb[k1 * EPI_LD + lane], wdL[h], g);
-                    if (g != 0.f) atomicAdd(a.g_t_in + (long long)p * a.C_t + ct * BN + cc * 32 + lane, g);
+                    if (g != 0.f) atomicAdd(a.g_t_in + (long long)p * a.C_t + ct * BN + h * 32 + lane, g);
                 }
                 __syncwarp();
             }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
         }
     }
     tc::tc_fence_before();
@@ -1037,10 +1040,10 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
                     tc::tc_fence_after();
                     const uint32_t sa = tc::smem_u32(smem + s * Cfg::STAGE);
                     const uint32_t sbb = RES ? tc::smem_u32(bres + kt * BN * 128) : sa + Cfg::A_BYTES;
+                    const uint64_t sad = tc::sdesc_sw128(sa), sbd = tc::sdesc_sw128(sbb);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        tc::mma_bf16(acc, tc::sdesc_sw128(sa + kk * 32), tc::sdesc_sw128(sbb + kk * 32), idesc,
-                                     (kt > 0 || kk > 0) ? 1u : 0u);
+                        tc::mma_bf16(acc, sad + 2 * kk, sbd + 2 * kk, idesc, (kt > 0 || kk > 0) ? 1u : 0u);
                     tc::mma_commit(&empty[s]);
                     if (++s == NST) {
                         s = 0;
@@ -1355,11 +1358,14 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                     tc::tc_fence_after();
                     const uint32_t sa = tc::smem_u32(smem + s * STG);
                     const uint32_t sbb = sa + a_bytes;
+                    // descriptors built once: a row tile is 16 KB on (+1024), a
+                    // 16-deep slice 2 KB (+128)
+                    const uint64_t ad0 = tc::sdesc_sw128_mn(sa, 8192), bd0 = tc::sdesc_sw128_mn(sbb, 8192);
                     for (int gi = 0; gi < G; ++gi) {
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
-                            tc::mma_bf16(tmem + gi * BN, tc::sdesc_sw128_mn(sa + gi * 16384 + kk * 2048, 8192),
-                                         tc::sdesc_sw128_mn(sbb + kk * 2048, 8192), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                            tc::mma_bf16(tmem + gi * BN, ad0 + (uint64_t)(gi * 1024 + kk * 128), bd0 + (uint64_t)(kk * 128),
+                                         idesc, (i > 0 || kk > 0) ? 1u : 0u);
                     }
                     tc::mma_commit(&empty[s]);
                     if (++s == NST) {
@@ -1694,11 +1700,14 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     tc::tc_fence_after();
                     const uint32_t sa = tc::smem_u32(smem + s * STG);
                     const uint32_t sbb = sa + a_bytes;
+                    // descriptors built once: a row tile is 16 KB on (+1024), a
+                    // 16-deep slice 2 KB (+128)
+                    const uint64_t ad0 = tc::sdesc_sw128_mn(sa, 8192), bd0 = tc::sdesc_sw128_mn(sbb, 8192);
                     for (int gi = 0; gi < G; ++gi) {
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
-                            tc::mma_bf16(tmem + gi * BN, tc::sdesc_sw128_mn(sa + gi * 16384 + kk * 2048, 8192),
-                                         tc::sdesc_sw128_mn(sbb + kk * 2048, 8192), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                            tc::mma_bf16(tmem + gi * BN, ad0 + (uint64_t)(gi * 1024 + kk * 128), bd0 + (uint64_t)(kk * 128),
+                                         idesc, (i > 0 || kk > 0) ? 1u : 0u);
                     }
                     tc::mma_commit(&empty[s]);
                     if (++s == NST) {
