@@ -180,7 +180,7 @@ int dstd_dense_bwd(const float *t_in, const float *W, const float *t_out, const 
  * Tensor-core math modes only (DSTD_MATH_F32 returns DSTD_E_UNSUPPORTED).
  * Padding taps read silent inputs.
  * In DSTD_MATH_BF16 with C_in below 64 (padded to 64 with silent inputs) or a
- * multiple of 64, C_out a multiple of 64 (at most 256 or a multiple of 256),
+ * multiple of 64, C_out a multiple of 64 (at most 128 or a multiple of 128),
  * k <= 7 and M <= 64,
  * the layer runs as implicit GEMMs: each input spike becomes one 8-byte
  * record (its grid step and its two nonzero grid weights in bf16, the

@@ -65,12 +65,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // ---------------------------------------------------------------------------
 // dC/dw^_{p,m,o} = -g K(t - T_m) / v^'(t) for m <= q (0 after the spike's
 // interval and for silent neurons), g = upstream + dT/dt, into [P][Mp][C_out]
-// bf16. A warp writes one position (or one 256-channel segment of it) at a
-// time, a contiguous block of its rows: a thread takes 8 consecutive neurons
-// and every R-th grid step (R = 32 / (channels / 8) rows per warp store, so
-// each store instruction writes up to 512 contiguous bytes). C_out is at
-// most 256 or a multiple of 256. K(x), x = t - T_m, falls along m by the factors
-// e^{av dt}, e^{aI dt}; a thread steps R grid steps at a time. The spike's own
+// bf16. A warp writes one position (or one 128-channel segment of it) at a
+// time, a contiguous block of its rows: a thread takes 4 consecutive neurons
+// and every R-th grid step (R = 32 / (channels / 4)). C_out is at most 128 or
+// a multiple of 128. With C_out = 64 the block is built in the warp's shared
+// buffer and written with one bulk copy; otherwise every store instruction
+// writes whole lines (streaming stores).
+// K(x), x = t - T_m, falls along m by the factors e^{av dt}, e^{aI dt}; a
+// thread steps R grid steps at a time. The spike's own
 // bin and the one before it (x < 2 dt, where (e^{-av x} - e^{-aI x}) / lam
 // cancels) take the accurate form. Silent neurons are counted per output
 // channel (the thread of row phase 0 of a channel group adds its counts).
@@ -79,16 +81,22 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 #define DWHAT_NPT 4
 #endif
 // NPT consecutive bf16 of one row, streamed (evict-first)
-template <int NPT>
+// (SHARED: p is in shared memory, a plain store; else a streaming global store)
+template <int NPT, bool SHARED>
 __device__ __forceinline__ void dwhat_store(__nv_bfloat16 *p, const float (&v)[NPT]) {
-    if constexpr (NPT == 8)
-        __stcs(reinterpret_cast<uint4 *>(p), make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                                                        pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7])));
-    else
-        __stcs(reinterpret_cast<uint2 *>(p), make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3])));
+    if constexpr (NPT == 8) {
+        const uint4 x = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                                   pack_bf16x2(v[6], v[7]));
+        if constexpr (SHARED) *reinterpret_cast<uint4 *>(p) = x;
+        else __stcs(reinterpret_cast<uint4 *>(p), x);
+    } else {
+        const uint2 x = make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]));
+        if constexpr (SHARED) *reinterpret_cast<uint2 *>(p) = x;
+        else __stcs(reinterpret_cast<uint2 *>(p), x);
+    }
 }
 
-template <int NPT>
+template <int NPT, bool BULK>
 __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_out, const int *__restrict__ qv,
                                                    const float *__restrict__ sv, const float *__restrict__ vd,
                                                    const float *__restrict__ g_up, long long P, int C, LifConst c,
@@ -101,6 +109,11 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
     if (lane >= R * groups) return;                   // idle lanes (C = 192)
     const int g = lane % groups, r = lane / groups;
     const int wpb = blockDim.x >> 5;
+    // BULK (C <= 32 NPT, one segment): a position's Mp x C block is built in
+    // this warp's shared buffer and written with one bulk copy
+    extern __shared__ __align__(128) uint8_t dw_smem[];
+    __nv_bfloat16 *wbuf = reinterpret_cast<__nv_bfloat16 *>(dw_smem) + (threadIdx.x >> 5) * c.Mp * C;
+    bool pending = false;
     const long long wid = (long long)blockIdx.x * wpb + (threadIdx.x >> 5), nw = (long long)gridDim.x * wpb;
     float cnt[NPT];
 #pragma unroll
@@ -164,7 +177,11 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
                 q[u] = -1;
             }
         }
-        __nv_bfloat16 *dst = D + p * (long long)c.Mp * C + c0;
+        if (BULK && pending) {  // the previous position's copy has read the buffer
+            if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+            __syncwarp();
+        }
+        __nv_bfloat16 *dst = (BULK ? wbuf : D + p * (long long)c.Mp * C) + c0;
         const int step = C;
         const float dtR = c.dt * R;
         int m = r;
@@ -177,7 +194,7 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
                     a[u] *= fv;
                     b[u] -= dtR;
                 }
-                dwhat_store<NPT>(dst + (long long)m * step, v);
+                dwhat_store<NPT, BULK>(dst + (long long)m * step, v);
             }
             for (; m <= m_hi; m += R) {
                 float v[NPT];
@@ -188,7 +205,7 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
                     a[u] *= fv;
                     b[u] -= dtR;
                 }
-                dwhat_store<NPT>(dst + (long long)m * step, v);
+                dwhat_store<NPT, BULK>(dst + (long long)m * step, v);
             }
         } else {
             for (; m < m_lo; m += R) {
@@ -199,7 +216,7 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
                     a[u] *= fv;
                     b[u] *= fI;
                 }
-                dwhat_store<NPT>(dst + (long long)m * step, v);
+                dwhat_store<NPT, BULK>(dst + (long long)m * step, v);
             }
             for (; m <= m_hi; m += R) {
                 float v[NPT];
@@ -210,16 +227,29 @@ __global__ void __launch_bounds__(256) k_dwhat_pmc(const float *__restrict__ t_o
                     a[u] *= fv;
                     b[u] *= fI;
                 }
-                dwhat_store<NPT>(dst + (long long)m * step, v);
+                dwhat_store<NPT, BULK>(dst + (long long)m * step, v);
             }
         }
         if (m < c.Mp) {
             float z[NPT];
 #pragma unroll
             for (int u = 0; u < NPT; ++u) z[u] = 0.f;
-            for (; m < c.Mp; m += R) dwhat_store<NPT>(dst + (long long)m * step, z);
+            for (; m < c.Mp; m += R) dwhat_store<NPT, BULK>(dst + (long long)m * step, z);
+        }
+        if (BULK) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) {
+                asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
+                                 D + p * (long long)c.Mp * C),
+                             "r"(tc::smem_u32(wbuf)), "r"((uint32_t)(c.Mp * C * 2))
+                             : "memory");
+                asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            }
+            pending = true;
         }
     }
+    if (BULK && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     if (count && r == 0) {
 #pragma unroll
         for (int u = 0; u < NPT; ++u)
@@ -1900,7 +1930,7 @@ static ConvGemmArgs base_args(const ConvGeom &g, int ni, const LifConst &c) {
 
 bool conv_implicit_supported(const ConvGeom &g, int C_out, int Mp) {
     const int Cp = conv_padded_channels(g.C);
-    return Cp % 64 == 0 && C_out % 64 == 0 && (C_out <= 256 || C_out % 256 == 0) && (Mp == 32 || Mp == 64) &&
+    return Cp % 64 == 0 && C_out % 64 == 0 && (C_out <= 128 || C_out % 128 == 0) && (Mp == 32 || Mp == 64) &&
            g.k <= 7 && Cp * g.k * g.k <= 65535 && C_out * g.k * g.k <= 65535;
 }
 
@@ -1913,10 +1943,21 @@ cudaError_t launch_dwhat_pmc(const float *t_out, const int *q, const float *s, c
     constexpr int NPT = DWHAT_NPT;
     if (C % 64 != 0 || (C > 32 * NPT && C % (32 * NPT) != 0)) return cudaErrorInvalidValue;
     long long blocks = (P * ((C + 32 * NPT - 1) / (32 * NPT)) + 7) / 8;  // 8 warps per block
-    const long long cap = 8ll * conv_num_sms();
+    // 64-channel positions: each warp builds the position's block in shared
+    // memory (8 KB; at 128 channels the 16 KB buffers leave one block per SM,
+    // and direct stores are faster)
+    const bool bulk = C <= 64;
+    const int smem = bulk ? 8 * c.Mp * C * 2 : 0;
+    const long long cap = (long long)(bulk ? (227 * 1024) / smem : 8) * conv_num_sms();
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    k_dwhat_pmc<NPT><<<(unsigned)blocks, 256, 0, st>>>(t_out, q, s, vdot, g_up, P, C, c, D, count);
+    if (bulk) {
+        cudaError_t e = cudaFuncSetAttribute(k_dwhat_pmc<NPT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        k_dwhat_pmc<NPT, true><<<(unsigned)blocks, 256, smem, st>>>(t_out, q, s, vdot, g_up, P, C, c, D, count);
+    } else {
+        k_dwhat_pmc<NPT, false><<<(unsigned)blocks, 256, 0, st>>>(t_out, q, s, vdot, g_up, P, C, c, D, count);
+    }
     return cudaGetLastError();
 }
 
