@@ -348,6 +348,7 @@ struct DsClass {
 };
 struct DsPlan {
     int a_bytes, b_bytes, stage, res_bytes, nst, units, taps_per_unit;
+    int epi_bytes;     // the epilogue's shared memory
     int ncls, ps, ts;  // classes, position step within a class, tap step
     DsClass cls[DS_MAX_CLS];
 };
@@ -374,9 +375,13 @@ __device__ __forceinline__ int ds_pos(const DsPlan &pl, int gh, int gw, int c, i
 constexpr int DS_MAX_STAGES = 8;
 constexpr int DS_EPI_BYTES = CONV_NEPI * 32 * EPI_LD * 4;
 // forward epilogue: per (epilogue group, position of the tile) the w^ rows
-// of Mp / 32 chunks of 32 neurons, Mp + 4 floats each (Mp = 64: 2 x 2 x 2 x
-// 32 x 68 floats; Mp = 32: 2 x 4 x 1 x 32 x 36)
-constexpr int FWD_EPI_BYTES = 2 * 2 * 2 * 32 * 68 * 4;
+// of Mp / 32 chunks of 32 neurons, Mp + pad floats each (Mp = 64: 2 x 2 x 2
+// x 32 x (64 + pad) floats; Mp = 32: 2 x 4 x 1 x 32 x (32 + pad)). Rows are
+// read as float4 with pad 4; the 128-channel forward on row boxes reads them
+// one float at a time with pad 1 (still free of bank conflicts), which
+// leaves room for two row-box stages
+__host__ __device__ constexpr int fwd_epi_pad(bool tight) { return tight ? 1 : 4; }
+__host__ __device__ constexpr int fwd_epi_bytes(bool tight) { return 2 * 2 * 2 * 32 * (64 + fwd_epi_pad(tight)) * 4; }
 
 // ---------------------------------------------------------------------------
 // Tap-shifted contraction over a [positions][Mp][channels] bf16 operand read
@@ -409,7 +414,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
     const int NST = pl.nst;
     uint8_t *bres = smem + NST * pl.stage;
     float *epi = reinterpret_cast<float *>(bres + pl.res_bytes);
-    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + (FWD ? FWD_EPI_BYTES : DS_EPI_BYTES));
+    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + pl.epi_bytes);
     uint64_t *empty = full + DS_MAX_STAGES;
     uint64_t *acc_full = empty + DS_MAX_STAGES;  // [2]
     uint64_t *acc_empty = acc_full + 2;          // [2]
@@ -629,7 +634,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
         const int qpp = Mp >> 5;  // lane quarters per position
         const int pp = quarter / qpp, wip = quarter - pp * qpp, mq = wip * 32;
-        const int LDB = Mp + 4;
+        constexpr bool TIGHT = FWD && BN == 128 && ROWBOX;
+        const int LDB = Mp + fwd_epi_pad(TIGHT);
         float *pbuf = epi + (group * ppt + pp) * qpp * 32 * LDB;
         const int bar_id = 1 + group * ppt + pp;  // named barrier of the position's warps
         auto sync_pos = [&]() {
@@ -686,7 +692,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                     float vv = 0.f, I = 0.f;
                     for (int m0 = 0; m0 < a.c.M; m0 += 32) {
                         const int mend = (a.c.M - m0) < 32 ? (a.c.M - m0) : 32;
-                        if (scan_walk<32>(a.c, row + m0, m0, mend, vv, I, st)) break;
+                        if (scan_walk<32, !TIGHT>(a.c, row + m0, m0, mend, vv, I, st)) break;
                     }
                     scan_finish(a.c, st);
                     finish_neuron(a.c, st, p, ct * BN + (r * qpp + wip) * 32 + lane, a.C_out, a.rowsum, a.t_out,
@@ -1899,7 +1905,7 @@ static cudaError_t launch_dw_gen_bn(const uint2 *rec, const CUtensorMap &mD, Con
 template <int BN, bool ROWBOX, bool RES, bool FWD>
 static cudaError_t launch_tap_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
                                  cudaStream_t st) {
-    const int smem = pl.nst * pl.stage + pl.res_bytes + (FWD ? FWD_EPI_BYTES : DS_EPI_BYTES) + 1024 + 256;
+    const int smem = pl.nst * pl.stage + pl.res_bytes + pl.epi_bytes + 1024 + 256;
     cudaError_t e = cudaFuncSetAttribute(k_conv_tap_gemm<BN, ROWBOX, RES, FWD>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -1971,7 +1977,8 @@ cudaError_t launch_filters_t(const float *W, int C_out, int T, int C_in, int C_p
 }
 
 // shared-memory plan of the tap-shifted contraction (see DsPlan)
-static DsPlan tap_plan(int k, int ppt, int Mp, int BN, bool resident, long long res, bool rowbox, int epi_bytes, int ncb) {
+static DsPlan tap_plan(int k, int ppt, int Mp, int BN, bool resident, long long res, bool rowbox, int epi_bytes, int ncb,
+                       int smem_max = GEN_SMEM_MAX) {
     DsPlan pl{};
     pl.taps_per_unit = rowbox ? k : 1;
     pl.a_bytes = rowbox ? (ppt + k - 1) * Mp * 128 : 128 * 128;
@@ -1979,7 +1986,8 @@ static DsPlan tap_plan(int k, int ppt, int Mp, int BN, bool resident, long long 
     pl.stage = (pl.a_bytes + pl.b_bytes + 1023) & ~1023;
     pl.res_bytes = resident ? (int)res : 0;
     pl.units = (rowbox ? k : k * k) * ncb;
-    const int nst = (GEN_SMEM_MAX - pl.res_bytes - epi_bytes - 1280) / pl.stage;
+    pl.epi_bytes = epi_bytes;
+    const int nst = (smem_max - pl.res_bytes - epi_bytes - 1280) / pl.stage;
     pl.nst = nst > DS_MAX_STAGES ? DS_MAX_STAGES : nst;
     return pl;
 }
@@ -2085,9 +2093,16 @@ cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifC
     const long long res = (long long)g.k * g.k * ncb * BN * 128;
     const bool resident = a.n_col == 1 && res <= 80 * 1024;
     const bool row_ok = g.s == 1 && g.Wo % ppt == 0 && ppt + g.k - 1 <= 256;
-    DsPlan pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, row_ok, FWD_EPI_BYTES, ncb);
+    DsPlan pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, row_ok, fwd_epi_bytes(false), ncb);
+    if (row_ok && pl.nst < 2 && BN == 128) {
+        // the tight epilogue rows and the device's whole opt-in shared memory
+        int dev = 0, optin = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) == cudaSuccess)
+            pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, true, fwd_epi_bytes(true), ncb, optin);
+    }
     const bool rowbox = row_ok && pl.nst >= 2;
-    if (!rowbox) pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, false, FWD_EPI_BYTES, ncb);
+    if (!rowbox) pl = tap_plan(g.k, ppt, c.Mp, BN, resident, res, false, fwd_epi_bytes(false), ncb);
     if (pl.nst < 2) return cudaErrorInvalidConfiguration;
     // every tap of every output position, in position order
     pl.ncls = 1;

@@ -294,31 +294,43 @@ __device__ __forceinline__ BinStep bin_step(const LifConst &c, float v, float I0
 }
 
 // The two passes over SUB bins m0 .. m0+SUB-1 of one neuron, whose w^
-// values sit in row[0 .. SUB) (shared memory, 16-byte aligned, zero past
-// mend), starting from the state (v, I) at T_m0. On a spike, fills st (bin,
-// state at its start, bracket end) and returns true; otherwise leaves (v, I)
-// at the end of the block.
-template <int SUB>
+// values sit in row[0 .. SUB) (shared memory, zero past mend; 16-byte
+// aligned when VEC, read as float4), starting from the state (v, I) at T_m0.
+// On a spike, fills st (bin, state at its start, bracket end) and returns
+// true; otherwise leaves (v, I) at the end of the block.
+template <int SUB, bool VEC = true>
 __device__ __forceinline__ bool scan_walk(const LifConst &c, const float *row, int m0, int mend, float &v, float &I,
                                           ScanState &st) {
     static_assert(SUB % 8 == 0 && SUB <= 32, "blocks of 8, 16 or 32 bins");
     constexpr int NCK = SUB / 8;  // kept states per block
     float kv[NCK], kI[NCK];
     uint32_t mask = 0u;
+    const unsigned lanes = __activemask();
 #pragma unroll
     for (int g = 0; g < SUB; g += 4) {
         if ((g & 7) == 0) {
             kv[g >> 3] = v;
             kI[g >> 3] = I;
         }
-        const float4 x = *reinterpret_cast<const float4 *>(row + g);
-        const float xs[4] = {x.x, x.y, x.z, x.w};
+        float xs[4];
+        if (VEC) {
+            const float4 x = *reinterpret_cast<const float4 *>(row + g);
+            xs[0] = x.x; xs[1] = x.y; xs[2] = x.z; xs[3] = x.w;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) xs[u] = row[g + u];
+        }
         // over these four bins the potential is at most max(v, 0) + Kmax4
         // (max(I, 0) + the positive inputs), Kmax4 the largest K(s) over four
         // steps (K >= 0, and the current only decays between inputs); well
-        // below v_th no bin can hold the spike and the flags are not formed
-        const float ipos = fmaxf(I, 0.0f) + fmaxf(x.x, 0.0f) + fmaxf(x.y, 0.0f) + fmaxf(x.z, 0.0f) + fmaxf(x.w, 0.0f);
-        if (fmaf(ipos, c.Kmax4, fmaxf(v, 0.0f)) < c.vth * 0.99999f) {
+        // below v_th no bin can hold the spike and its flags are not needed
+        const float ipos = fmaxf(I, 0.0f) + fmaxf(xs[0], 0.0f) + fmaxf(xs[1], 0.0f) + fmaxf(xs[2], 0.0f) +
+                           fmaxf(xs[3], 0.0f);
+        const bool quiet = fmaf(ipos, c.Kmax4, fmaxf(v, 0.0f)) < c.vth * 0.99999f;
+        // one path per group for the whole warp: the flagged pass (its flags
+        // kept only where the bound is not met) unless every lane is quiet;
+        // both passes round alike, so the state does not depend on the path
+        if (__all_sync(lanes, quiet)) {
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const float I0 = I + xs[u];
@@ -329,7 +341,7 @@ __device__ __forceinline__ bool scan_walk(const LifConst &c, const float *row, i
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const BinStep r = bin_step(c, v, I + xs[u]);
-                if (r.endp | r.peak) mask |= 1u << (g + u);
+                if (!quiet && (r.endp | r.peak)) mask |= 1u << (g + u);
                 v = r.ve;
                 I = r.In;
             }
