@@ -349,6 +349,7 @@ struct DsClass {
 struct DsPlan {
     int a_bytes, b_bytes, stage, res_bytes, nst, units, taps_per_unit;
     int epi_bytes;     // the epilogue's shared memory
+    int run_ok;        // the map of ppt-position boxes is valid
     int ncls, ps, ts;  // classes, position step within a class, tap step
     DsClass cls[DS_MAX_CLS];
 };
@@ -408,7 +409,7 @@ __host__ __device__ constexpr int fwd_epi_bytes(bool tight) { return 2 * 2 * 2 *
 template <int BN, bool ROWBOX, bool RES, bool FWD>
 __global__ void __launch_bounds__(CONV_THREADS, 1)
     k_conv_tap_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-                    ConvGemmArgs a, const __grid_constant__ DsPlan pl) {
+                    const __grid_constant__ CUtensorMap mapR, ConvGemmArgs a, const __grid_constant__ DsPlan pl) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const int NST = pl.nst;
@@ -498,6 +499,13 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                 // class coordinates: tap (kh0 + ih ts, kw0 + iw ts) reads output
                 // position (yy + by0 - ih, xx + bx0 - iw)
                 const bool cls_order = pl.ps == a.stride;
+                // the tile's positions read one run of consecutive positions of
+                // a row for every tap (stride 1 forward; dS in stride classes):
+                // one box of ppt positions (mapR) instead of ppt boxes
+                bool run = !ROWBOX && pl.run_ok && ppt > 1 && (FWD ? a.stride == 1 : cls_order);
+#pragma unroll
+                for (int pp = 1; pp < 4; ++pp)
+                    if (pp < ppt) run = run && pb[pp] == pb[0] && pyy[pp] == pyy[0] && pxx[pp] == pxx[0] + pp;
                 const int by0 = cls_order ? (q.py + a.pad - q.kh0) / pl.ts : 0;
                 const int bx0 = cls_order ? (q.px + a.pad - q.kw0) / pl.ts : 0;
                 const int nkh = ROWBOX ? k : q.nkh, nkw = ROWBOX ? 1 : q.nkw;
@@ -527,7 +535,7 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                                 const int kh = q.kh0 + ih * pl.ts, kw = q.kw0 + iw * pl.ts;
 #pragma unroll
                                 for (int pp = 0; pp < 4; ++pp) {
-                                    if (pp >= ppt) break;
+                                    if (pp >= (run ? 1 : ppt)) break;
                                     int sx, sy;
                                     if (FWD) {
                                         sy = pyy[pp] + kh;
@@ -541,7 +549,8 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
                                         sy = on ? ny / a.stride : -1;
                                         sx = on ? nx / a.stride : 0;
                                     }
-                                    tma_load_5d(st + pp * Mp * 128, &mapA, &full[s], cb * 64, 0, sx, sy, pb[pp]);
+                                    tma_load_5d(st + pp * Mp * 128, run ? &mapR : &mapA, &full[s], cb * 64, 0, sx, sy,
+                                                pb[pp]);
                                 }
                                 if (!RES)
                                     tc::tma_load_2d(st + pl.a_bytes, &mapB, &full[s], (kh * k + kw) * kc + cb * 64,
@@ -1903,15 +1912,15 @@ static cudaError_t launch_dw_gen_bn(const uint2 *rec, const CUtensorMap &mD, Con
 }
 
 template <int BN, bool ROWBOX, bool RES, bool FWD>
-static cudaError_t launch_tap_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
-                                 cudaStream_t st) {
+static cudaError_t launch_tap_bn(const CUtensorMap &mA, const CUtensorMap &mB, const CUtensorMap &mR, ConvGemmArgs a,
+                                 DsPlan pl, cudaStream_t st) {
     const int smem = pl.nst * pl.stage + pl.res_bytes + pl.epi_bytes + 1024 + 256;
     cudaError_t e = cudaFuncSetAttribute(k_conv_tap_gemm<BN, ROWBOX, RES, FWD>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ntiles = a.n_row * a.n_col;
     const int grid = ntiles < conv_num_sms() ? ntiles : conv_num_sms();
-    k_conv_tap_gemm<BN, ROWBOX, RES, FWD><<<grid, CONV_THREADS, smem, st>>>(mA, mB, a, pl);
+    k_conv_tap_gemm<BN, ROWBOX, RES, FWD><<<grid, CONV_THREADS, smem, st>>>(mA, mB, mR, a, pl);
     return cudaGetLastError();
 }
 
@@ -2052,15 +2061,17 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
         a.n_row += (pl.cls[i].count + ppt - 1) / ppt;
     }
     if (a.n_row == 0) return cudaSuccess;
-    CUtensorMap mA, mB;
+    CUtensorMap mA, mB, mR;
     if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, rowbox ? ppt + g.k - 1 : 1) ||
         !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))
         return cudaErrorInvalidValue;
+    pl.run_ok = map_act(&mR, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, ppt) ? 1 : 0;
+    if (!pl.run_ok) mR = mA;
 #define DSTD_DS(BNV)                                                                                   \
-    if (rowbox) return resident ? launch_tap_bn<BNV, true, true, false>(mA, mB, a, pl, st)             \
-                                : launch_tap_bn<BNV, true, false, false>(mA, mB, a, pl, st);           \
-    return resident ? launch_tap_bn<BNV, false, true, false>(mA, mB, a, pl, st)                        \
-                    : launch_tap_bn<BNV, false, false, false>(mA, mB, a, pl, st);
+    if (rowbox) return resident ? launch_tap_bn<BNV, true, true, false>(mA, mB, mR, a, pl, st)         \
+                                : launch_tap_bn<BNV, true, false, false>(mA, mB, mR, a, pl, st);       \
+    return resident ? launch_tap_bn<BNV, false, true, false>(mA, mB, mR, a, pl, st)                    \
+                    : launch_tap_bn<BNV, false, false, false>(mA, mB, mR, a, pl, st);
     switch (BN) {
         case 256: { DSTD_DS(256) }
         case 128: { DSTD_DS(128) }
@@ -2115,15 +2126,17 @@ cudaError_t launch_conv_fwd_tma(const ConvGeom &g, int ni, int C_out, const LifC
     cl.tile0 = 0;
     cl.kh0 = cl.kw0 = 0;
     cl.nkh = cl.nkw = g.k;
-    CUtensorMap mA, mB;
+    CUtensorMap mA, mB, mR;
     if (!map_act(&mA, S, ni, g.H, g.W, c.Mp, g.C, rowbox ? ppt + g.k - 1 : 1) ||
         !map_mat(&mB, Wf, C_out, g.k * g.k * g.C, BN))
         return cudaErrorInvalidValue;
+    pl.run_ok = map_act(&mR, S, ni, g.H, g.W, c.Mp, g.C, ppt) ? 1 : 0;
+    if (!pl.run_ok) mR = mA;
 #define DSTD_FT(BNV)                                                                                   \
-    if (rowbox) return resident ? launch_tap_bn<BNV, true, true, true>(mA, mB, a, pl, st)              \
-                                : launch_tap_bn<BNV, true, false, true>(mA, mB, a, pl, st);            \
-    return resident ? launch_tap_bn<BNV, false, true, true>(mA, mB, a, pl, st)                         \
-                    : launch_tap_bn<BNV, false, false, true>(mA, mB, a, pl, st);
+    if (rowbox) return resident ? launch_tap_bn<BNV, true, true, true>(mA, mB, mR, a, pl, st)          \
+                                : launch_tap_bn<BNV, true, false, true>(mA, mB, mR, a, pl, st);        \
+    return resident ? launch_tap_bn<BNV, false, true, true>(mA, mB, mR, a, pl, st)                     \
+                    : launch_tap_bn<BNV, false, false, true>(mA, mB, mR, a, pl, st);
     switch (BN) {
         case 256: { DSTD_FT(256) }
         case 128: { DSTD_FT(128) }
