@@ -786,6 +786,231 @@ __global__ void __launch_bounds__(CONV_THREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
+// dS of two row tiles at once (stride 1, image rows a multiple of 2 ppt
+// positions wide). The pair's 2 ppt input positions are consecutive in one
+// row, so one box of 2 ppt + k - 1 positions of dw^ per (filter row,
+// channel block) serves both tiles and all k taps of the row, and every
+// filter slice feeds two MMAs back to back (one per tile, each into its own
+// accumulator): consecutive MMAs on the same B operand issue faster than
+// MMAs that each fetch new operands. TMEM: two pair slots x two tiles x BN
+// columns. Epilogue group g takes tile g of every pair (the same work per
+// warp as the single-tile kernel's epilogue); acc_empty counts all eight
+// epilogue warps. Warps and barriers otherwise as in k_conv_tap_gemm.
+// ---------------------------------------------------------------------------
+template <int BN, bool RES>
+__global__ void __launch_bounds__(CONV_THREADS, 1)
+    k_conv_ds_pair(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, ConvGemmArgs a,
+                   const __grid_constant__ DsPlan pl) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const int NST = pl.nst;
+    uint8_t *bres = smem + NST * pl.stage;
+    float *epi = reinterpret_cast<float *>(bres + pl.res_bytes);
+    uint64_t *full = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(epi) + pl.epi_bytes);
+    uint64_t *empty = full + DS_MAX_STAGES;
+    uint64_t *acc_full = empty + DS_MAX_STAGES;  // [2] pair slots
+    uint64_t *acc_empty = acc_full + 2;          // [2]
+    uint64_t *bres_full = acc_empty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bres_full + 1);
+    constexpr uint32_t TMEM_COLS = 4 * BN;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int npairs = (a.n_row >> 1) * a.n_col;
+    const int Mp = a.Mp;
+    const int ppt = 128 / Mp;  // positions per tile
+    const int kc = a.C_out;    // channels contracted per tap
+    const int ncb = kc >> 6;
+    const int k = a.k;
+    const uint32_t tile_bytes = (uint32_t)(ppt * Mp * 128);  // the second tile's rows in the box
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NST; ++s) {
+            tc::mbar_init(&full[s], 1);
+            tc::mbar_init(&empty[s], 1);
+        }
+        for (int u = 0; u < 2; ++u) {
+            tc::mbar_init(&acc_full[u], 1);
+            tc::mbar_init(&acc_empty[u], CONV_NEPI);  // both groups read every pair slot
+        }
+        tc::mbar_init(bres_full, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            if (RES) {
+                const int nslices = k * k * ncb;
+                tc::mbar_expect_tx(bres_full, (uint32_t)(nslices * BN * 128));
+                for (int q = 0; q < nslices; ++q) {
+                    const int tap = q / ncb, cb = q - tap * ncb;
+                    tc::tma_load_2d(tc::smem_u32(bres + q * BN * 128), &mapB, bres_full, tap * kc + cb * 64, 0);
+                }
+            }
+            uint32_t it = 0;
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int pr = blockIdx.x; pr < npairs && ok; pr += gridDim.x) {
+                const int rp = pr / a.n_col, ct = pr - rp * a.n_col;
+                int b0, y0, x0;
+                pos_decode(rp * 2 * ppt, a.H, a.W, b0, y0, x0);
+                for (int ih = 0; ih < k && ok; ++ih)
+                    for (int cb = 0; cb < ncb; ++cb, ++it) {
+                        if (!tc::mbar_wait_spin(&empty[s], ph ^ 1u)) {
+                            conv_set_status(STATUS_TIMEOUT);
+                            ok = false;
+                            break;
+                        }
+                        tc::mbar_expect_tx(&full[s], (uint32_t)(pl.a_bytes + pl.b_bytes));
+                        const uint32_t st = tc::smem_u32(smem + s * pl.stage);
+                        // output positions x0 + pad - (k - 1) .. of row y0 + pad - kh
+                        tma_load_5d(st, &mapA, &full[s], cb * 64, 0, x0 + a.pad - (k - 1), y0 + a.pad - ih, b0);
+                        if (!RES)
+                            for (int kw = 0; kw < k; ++kw)
+                                tc::tma_load_2d(st + pl.a_bytes + kw * BN * 128, &mapB, &full[s],
+                                                (ih * k + kw) * kc + cb * 64, ct * BN);
+                        if (++s == NST) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
+                    }
+            }
+            const uint32_t n_drain = it < (uint32_t)NST ? it : (uint32_t)NST;
+            for (uint32_t i = it - n_drain; i < it; ++i) tc::mbar_wait_spin(&full[i % NST], (i / NST) & 1u);
+            if (RES) tc::mbar_wait_spin(bres_full, 0);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(128, BN, false, false);
+            uint32_t j = 0;
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            if (RES && !tc::mbar_wait_spin(bres_full, 0)) {
+                conv_set_status(STATUS_TIMEOUT);
+                ok = false;
+            }
+            for (int pr = blockIdx.x; pr < npairs && ok; pr += gridDim.x, ++j) {
+                const uint32_t slot = j & 1u;
+                if (j >= 2) {
+                    if (!tc::mbar_wait_spin(&acc_empty[slot], ((j >> 1) + 1u) & 1u)) {
+                        conv_set_status(STATUS_TIMEOUT);
+                        break;
+                    }
+                    tc::tc_fence_after();
+                }
+                const uint32_t acc0 = tmem + slot * 2 * BN, acc1 = acc0 + BN;
+                bool first = true;
+                for (int ih = 0; ih < k && ok; ++ih)
+                    for (int cb = 0; cb < ncb; ++cb) {
+                        if (!tc::mbar_wait_spin(&full[s], ph)) {
+                            conv_set_status(STATUS_TIMEOUT);
+                            ok = false;
+                            break;
+                        }
+                        tc::tc_fence_after();
+                        const uint32_t sa = tc::smem_u32(smem + s * pl.stage);
+                        for (int v = 0; v < k; ++v) {
+                            const int tap = ih * k + v;
+                            const uint32_t abase = sa + (uint32_t)((k - 1 - v) * Mp * 128);
+                            const uint32_t bbase = RES ? tc::smem_u32(bres + (tap * ncb + cb) * BN * 128)
+                                                       : sa + (uint32_t)(pl.a_bytes + v * BN * 128);
+                            const uint64_t ad0 = tc::sdesc_sw128(abase), ad1 = tc::sdesc_sw128(abase + tile_bytes);
+                            const uint64_t bd = tc::sdesc_sw128(bbase);
+                            const uint32_t acc_in = (!first || v > 0) ? 1u : 0u;
+                            tc::mma_bf16(acc0, ad0, bd, idesc, acc_in);
+                            tc::mma_bf16(acc1, ad1, bd, idesc, acc_in);
+#pragma unroll
+                            for (int kk = 1; kk < 4; ++kk) {
+                                tc::mma_bf16(acc0, ad0 + 2 * kk, bd + 2 * kk, idesc, 1u);
+                                tc::mma_bf16(acc1, ad1 + 2 * kk, bd + 2 * kk, idesc, 1u);
+                            }
+                        }
+                        first = false;
+                        tc::mma_commit(&empty[s]);
+                        if (++s == NST) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
+                    }
+                if (ok) tc::mma_commit(&acc_full[slot]);
+            }
+        }
+        __syncwarp();
+    } else {
+        // group g reads tile g of every pair, all BN columns; warp w reads
+        // TMEM lane quarter w % 4
+        const int quarter = warp & 3, group = (warp - 2) >> 2;
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        float *tb = epi + (warp - 2) * 32 * EPI_LD;
+        const int pp = (quarter * 32) / Mp;      // position of this warp's rows (Mp >= 32)
+        const int m_base = (quarter * 32) % Mp;  // first grid step of this warp's rows
+        constexpr int NCH = BN / 32;
+        uint32_t j = 0;
+        for (int pr = blockIdx.x; pr < npairs; pr += gridDim.x, ++j) {
+            const int rp = pr / a.n_col, ct = pr - rp * a.n_col;
+            const int rt = rp * 2 + group;
+            const uint32_t slot = j & 1u;
+            const int p = ds_pos(pl, a.H, a.W, 0, rt, pp, ppt);
+            int wk[NCH];
+            float wdR[NCH], wdL[NCH];
+#pragma unroll
+            for (int h = 0; h < NCH; ++h) {
+                wk[h] = -1000;
+                wdR[h] = wdL[h] = 0.f;
+                const int col0 = ct * BN + h * 32;
+                if (p >= 0 && col0 + lane < a.C_t) {
+                    const float x = __ldg(a.t_in + (long long)p * a.C_t + col0 + lane);
+                    if (isfinite(x)) {
+                        const BinW w = bin_weights(a.c, x, true);
+                        wk[h] = w.k;
+                        wdR[h] = w.dR;
+                        wdL[h] = w.dL;
+                    }
+                }
+            }
+            if (!tc::mbar_wait_sleep(&acc_full[slot], (j >> 1) & 1u)) {
+                conv_set_status(STATUS_TIMEOUT);
+                break;
+            }
+            tc::tc_fence_after();
+            const uint32_t acc = tmem + (slot * 2 + (uint32_t)group) * BN;
+#pragma unroll
+            for (int h = 0; h < NCH; ++h) {
+                float v[32];
+                tc::tmem_ld32(acc + lane_base + h * 32, v);
+                if (h == NCH - 1) {  // the pair slot's last TMEM read of this warp
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(&acc_empty[slot]);
+                }
+#pragma unroll
+                for (int u = 0; u < 32; ++u) tb[lane * EPI_LD + u] = v[u];
+                __syncwarp();
+                if (p >= 0 && wk[h] > -1000) {
+                    float g = 0.f;
+                    const int k0 = wk[h] - m_base, k1 = wk[h] + 1 - m_base;
+                    if (k0 >= 0 && k0 < 32 && wk[h] < a.c.M) g = fmaf(tb[k0 * EPI_LD + lane], wdR[h], g);
+                    if (k1 >= 0 && k1 < 32 && wk[h] + 1 < a.c.M) g = fmaf(tb[k1 * EPI_LD + lane], wdL[h], g);
+                    if (g != 0.f) atomicAdd(a.g_t_in + (long long)p * a.C_t + ct * BN + h * 32 + lane, g);
+                }
+                __syncwarp();
+            }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tc::tmem_dealloc(tmem, TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------
 // Binned operand generated on chip (the compact support of K_DSTD: each
 // input spike has two nonzero grid weights among Mp). The binning writes
 // one 8-byte record per input, rec[p][c] = (grid step k, bf16 pair (w at
@@ -1924,6 +2149,19 @@ static cudaError_t launch_tap_bn(const CUtensorMap &mA, const CUtensorMap &mB, c
     return cudaGetLastError();
 }
 
+template <int BN, bool RES>
+static cudaError_t launch_ds_pair_bn(const CUtensorMap &mA, const CUtensorMap &mB, ConvGemmArgs a, DsPlan pl,
+                                     cudaStream_t st) {
+    const int smem = pl.nst * pl.stage + pl.res_bytes + pl.epi_bytes + 1024 + 256;
+    cudaError_t e =
+        cudaFuncSetAttribute(k_conv_ds_pair<BN, RES>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const int npairs = (a.n_row / 2) * a.n_col;
+    const int grid = npairs < conv_num_sms() ? npairs : conv_num_sms();
+    k_conv_ds_pair<BN, RES><<<grid, CONV_THREADS, smem, st>>>(mA, mB, a, pl);
+    return cudaGetLastError();
+}
+
 static ConvGemmArgs base_args(const ConvGeom &g, int ni, const LifConst &c) {
     ConvGemmArgs a{};
     a.ni = ni;
@@ -2062,9 +2300,22 @@ cudaError_t launch_conv_ds_gemm(const ConvGeom &g, int ni, int C_out, const LifC
     }
     if (a.n_row == 0) return cudaSuccess;
     CUtensorMap mA, mB, mR;
-    if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, rowbox ? ppt + g.k - 1 : 1) ||
-        !map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN))
-        return cudaErrorInvalidValue;
+    if (!map_mat(&mB, Wt, g.C, g.k * g.k * C_out, BN)) return cudaErrorInvalidValue;
+    // two row tiles at once when image rows hold whole pairs (one class,
+    // an even number of row tiles), for 64-wide column tiles
+    if (rowbox && g.W % (2 * ppt) == 0 && 2 * ppt + g.k - 1 <= 256 && BN == 64 && pl.ncls == 1 &&
+        a.n_row % 2 == 0) {
+        DsPlan pq = pl;
+        pq.a_bytes = (2 * ppt + g.k - 1) * c.Mp * 128;
+        pq.b_bytes = resident ? 0 : g.k * BN * 128;
+        pq.stage = (pq.a_bytes + pq.b_bytes + 1023) & ~1023;
+        const int nst = (GEN_SMEM_MAX - pq.res_bytes - pq.epi_bytes - 1280) / pq.stage;
+        pq.nst = nst > DS_MAX_STAGES ? DS_MAX_STAGES : nst;
+        if (pq.nst >= 2 && map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, 2 * ppt + g.k - 1))
+            return resident ? launch_ds_pair_bn<64, true>(mA, mB, a, pq, st)
+                            : launch_ds_pair_bn<64, false>(mA, mB, a, pq, st);
+    }
+    if (!map_act(&mA, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, rowbox ? ppt + g.k - 1 : 1)) return cudaErrorInvalidValue;
     pl.run_ok = map_act(&mR, dW_hat, ni, g.Ho, g.Wo, c.Mp, C_out, ppt) ? 1 : 0;
     if (!pl.run_ok) mR = mA;
 #define DSTD_DS(BNV)                                                                                   \
