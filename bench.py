@@ -448,16 +448,11 @@ class ClockSampler:
 # DRAM bytes read + written per launch, averaged over the kind's launches in
 # one step, from `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum`
 # on `python bench.py --steps 5 --warmup 3 --profile` (the per-launch table
-# in profiles/launches_cfg2_step.md); to be set to None when the kernel
-# changes after that capture.
+# in profiles/launches_cfg2_step.md); kinds whose kernels changed after that
+# capture (the contractions, the scan, dw^ and the transposed binning) have
+# no entry, so their traffic is reported as null.
 TRAFFIC_PER_LAUNCH = {
-    ("gemm_dW", "x3"): 54.8e6,
-    ("gemm_fwd_scan", "x3"): 28.6e6,
-    ("gemm_dS_gradt", "x3"): 32.2e6,
-    ("scan_solve", "x3"): 26.3e6,
-    ("dwhat", "x3"): 3.9e6,
     ("binning", "x3"): 3.37e6,          # k_fwd_operands_f16: binning + the hi/lo split of W
-    ("binning_T", "x3"): 0.82e6,
     ("prep_weights", "x3"): 2.57e6,     # the backward's W^T split
     ("loss", "x3"): 0.04e6,
     ("adamw", "x3"): 20.4e6,
